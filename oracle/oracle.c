@@ -1,0 +1,402 @@
+/*
+ * oracle.c -- plain, slow, fp64 CPU oracle of the FastEagle cascaded drafter.
+ *
+ * TEST INFRASTRUCTURE. Only the tests, __graft_entry__.smoke() and the CPU-baseline
+ * leg of bench.py may load or run this library. It shares no code, header, table or
+ * helper with the CUDA path (paper_2509_20416_gb300/), and it never reads a value the
+ * CUDA path produced: it is the yardstick the CUDA path is measured against.
+ *
+ * What it computes (FastEagle, arXiv 2509.20416):
+ *   - Sec. 2.1 and Eq. 1: fused feature g = FC(concat(l, m, h)) from the target's
+ *     three hidden-state levels, then x0 = FC(concat(g, e)) with e the embedding of
+ *     the next token; both FCs are bias-free linear maps.
+ *   - Eq. 2: the cascade h_i = L_i(h_{i-1}), i = 1..N (h_0 = x0), each L_i a
+ *     lightweight pre-norm decoder layer with its own parameters. Sec. 2.1 builds on
+ *     EAGLE-3's single decoder layer; its internals are read as the standard LLaMA
+ *     block: RMSNorm, QKV, rotate-half RoPE, (grouped-query) attention over the
+ *     layer's own prefix K/V cache plus the drafted row's own key/value, O-proj and
+ *     residual, RMSNorm, SwiGLU MLP and residual.
+ *   - Sec. 2.1: every h_i goes through the target's frozen LM head (after the
+ *     target's final RMSNorm) to give the distribution q_{t+i}.
+ *   - Sec. 2.2: top-k per depth and the Backbone Expansion tree with its
+ *     tree-attention (ancestor-or-self) mask.
+ * Every stored bf16/fp32 input is widened exactly to double; nothing is rounded in
+ * between. Loops are the definitions written out: no blocking, no fusion, no
+ * reordering of a sum. OpenMP only splits independent output rows across threads,
+ * so results do not depend on the thread count.
+ *
+ * Parity pins: every function here is pinned by the `-m "not gpu"` tests (closed
+ * forms, brute force, library special cases, invariants, a hand-worked tree). The
+ * OR_MUTANT switch plants one known mistake per build so that a test can show the
+ * pins catch it; the default build (OR_MUTANT == 0) has none.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifndef OR_MUTANT
+#define OR_MUTANT 0
+#endif
+#define MUT(n) (OR_MUTANT == (n))
+
+typedef struct {
+    int32_t d, n_heads, n_kv_heads, head_dim, ffn, vocab, n_layers;
+    int32_t dtype;             /* storage type of every input tensor: 0 float32, 1 bfloat16 */
+    double rope_theta, rms_eps;
+    int32_t rope_layer_offset; /* reading of the query position: 0 -> every layer at P (default),
+                                  1 -> layer i at P + i - 1 */
+    int32_t final_norm;        /* 1 -> RMSNorm(gamma_out) before the LM head (default), 0 -> none */
+} or_config;
+
+/* ---- storage ------------------------------------------------------------------ */
+
+static double ld(const void *p, int32_t dtype, int64_t i)
+{
+    if (dtype == 0)
+        return (double)((const float *)p)[i];
+    uint32_t u = (uint32_t)((const uint16_t *)p)[i] << 16; /* bf16 -> f32 is exact */
+    float f;
+    memcpy(&f, &u, 4);
+    return (double)f;
+}
+
+void or_widen(const void *src, int32_t dtype, int64_t n, double *dst)
+{
+    for (int64_t i = 0; i < n; ++i)
+        dst[i] = ld(src, dtype, i);
+}
+
+/* ---- primitives ---------------------------------------------------------------- */
+
+/* y = W x with W row-major [M, K]: y_m = sum_k W[m, k] x_k. */
+void or_matvec(const void *W, int32_t dtype, int64_t M, int64_t K, const double *x, double *y)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t m = 0; m < M; ++m) {
+        double s = 0.0;
+        for (int64_t k = 0; k < K; ++k) {
+            int64_t idx = MUT(1) ? k * M + m : m * K + k;
+            s += ld(W, dtype, idx) * x[k];
+        }
+        y[m] = s;
+    }
+}
+
+/* RMSNorm: y_j = gamma_j * x_j / sqrt(mean(x^2) + eps). */
+void or_rmsnorm(const double *x, const void *gamma, int32_t dtype, int64_t n, double eps, double *y)
+{
+    double ss = 0.0;
+    for (int64_t j = 0; j < n; ++j)
+        ss += x[j] * x[j];
+    double ms = MUT(6) ? ss : ss / (double)n;
+    double r = 1.0 / sqrt(MUT(24) ? ms : ms + eps);
+    for (int64_t j = 0; j < n; ++j)
+        y[j] = ld(gamma, dtype, j) * x[j] * r;
+}
+
+/* Rotary position embedding, rotate-half pairing (j, j + hd/2), j < hd/2, rotating
+ * the pair by the angle pos * theta^(-2j/hd). Applied in place to one head. */
+void or_rope(double *v, int32_t hd, double pos, double theta)
+{
+    const int32_t half = hd / 2;
+    if (MUT(3)) { /* planted mistake: interleaved pairs (2j, 2j+1) */
+        for (int32_t j = 0; j < half; ++j) {
+            double ang = pos * pow(theta, -2.0 * (double)j / (double)hd);
+            double c = cos(ang), s = sin(ang);
+            double a = v[2 * j], b = v[2 * j + 1];
+            v[2 * j] = a * c - b * s;
+            v[2 * j + 1] = b * c + a * s;
+        }
+        return;
+    }
+    for (int32_t j = 0; j < half; ++j) {
+        double ang = pos * pow(theta, -2.0 * (double)j / (double)hd);
+        double c = cos(ang), s = sin(ang);
+        double a = v[j], b = v[j + half];
+        if (MUT(2)) {
+            v[j] = a * c + b * s;
+            v[j + half] = b * c - a * s;
+        } else {
+            v[j] = a * c - b * s;
+            v[j + half] = b * c + a * s;
+        }
+    }
+}
+
+/* Decode attention of one drafted row of one sequence.
+ *   q      [H][hd]     queries (RoPE already applied)
+ *   kc, vc [Hkv][cap][hd] this layer's cache for this sequence (storage dtype); rows
+ *          0..P-1 are the prefix (keys already rotated)
+ *   k_new, v_new [Hkv][hd] the row's own key (rotated) and value, key index P
+ *   out    [H][hd]
+ * Query head h reads KV head g(h) = floor(h * Hkv / H); scores are scaled by
+ * 1/sqrt(hd); the softmax subtracts the row maximum. */
+void or_attention(const double *q, int32_t H, int32_t Hkv, int32_t hd, const void *kc,
+                  const void *vc, int32_t dtype, int64_t cap, int32_t P, const double *k_new,
+                  const double *v_new, double *out)
+{
+    const double scale = MUT(4) ? 1.0 : 1.0 / sqrt((double)hd);
+    const int32_t P_read = MUT(22) ? (P > 0 ? P - 1 : 0) : P;
+#pragma omp parallel for schedule(static)
+    for (int32_t h = 0; h < H; ++h) {
+        const int32_t g = MUT(5) ? h % Hkv : (int32_t)(((int64_t)h * Hkv) / H);
+        const double *qh = q + (int64_t)h * hd;
+        const int32_t nk = MUT(11) ? P_read : P_read + 1;
+        double *s = (double *)malloc(sizeof(double) * (size_t)(nk > 0 ? nk : 1));
+        double mx = -INFINITY;
+        for (int32_t t = 0; t < nk; ++t) {
+            double dot = 0.0;
+            if (t < P_read) {
+                int64_t base = ((int64_t)g * cap + t) * hd;
+                for (int32_t j = 0; j < hd; ++j)
+                    dot += qh[j] * ld(kc, dtype, base + j);
+            } else {
+                for (int32_t j = 0; j < hd; ++j)
+                    dot += qh[j] * k_new[(int64_t)g * hd + j];
+            }
+            s[t] = dot * scale;
+            if (s[t] > mx)
+                mx = s[t];
+        }
+        double den = 0.0;
+        for (int32_t t = 0; t < nk; ++t) {
+            s[t] = exp(s[t] - mx);
+            den += s[t];
+        }
+        for (int32_t j = 0; j < hd; ++j) {
+            double acc = 0.0;
+            for (int32_t t = 0; t < nk; ++t) {
+                double vv = (t < P_read) ? ld(vc, dtype, ((int64_t)g * cap + t) * hd + j)
+                                         : v_new[(int64_t)g * hd + j];
+                acc += s[t] * vv;
+            }
+            out[(int64_t)h * hd + j] = acc / den;
+        }
+        free(s);
+    }
+}
+
+/* SiLU(a) = a / (1 + e^-a); the SwiGLU product silu(gate) * up. */
+void or_silu_mul(const double *gate, const double *up, int64_t n, double *y)
+{
+    for (int64_t j = 0; j < n; ++j) {
+        double a = MUT(9) ? up[j] : gate[j];
+        double b = MUT(9) ? gate[j] : up[j];
+        double sig = 1.0 / (1.0 + exp(-a));
+        y[j] = (MUT(23) ? sig : a * sig) * b;
+    }
+}
+
+/* One cascade layer L_i (Eq. 2) for one sequence, x updated in place.
+ * lw: attn_norm, w_qkv [(H+2Hkv)hd, d], w_o [d, H hd], mlp_norm, w_gate [F,d],
+ * w_up [F,d], w_down [d,F]. The drafted row sits at sequence position `pos`; it
+ * attends to its P prefix rows in (kc, vc) plus its own key/value. */
+void or_layer(const or_config *c, const void *const *lw, double pos, const void *kc,
+              const void *vc, int64_t cap, int32_t P, double *x)
+{
+    const int32_t d = c->d, H = c->n_heads, Hkv = c->n_kv_heads, hd = c->head_dim, F = c->ffn;
+    const int64_t nq = (int64_t)H * hd, nkv = (int64_t)Hkv * hd;
+    double *u = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qkv = (double *)malloc(sizeof(double) * (size_t)(nq + 2 * nkv));
+    double *o = (double *)malloc(sizeof(double) * (size_t)nq);
+    double *t = (double *)malloc(sizeof(double) * (size_t)d);
+    double *gt = (double *)malloc(sizeof(double) * (size_t)F);
+    double *up = (double *)malloc(sizeof(double) * (size_t)F);
+    double *a = (double *)malloc(sizeof(double) * (size_t)F);
+
+    /* attention block */
+    or_rmsnorm(x, lw[0], c->dtype, d, c->rms_eps, u);
+    or_matvec(lw[1], c->dtype, nq + 2 * nkv, d, u, qkv);
+    double *q = qkv, *k = qkv + nq, *v = qkv + nq + nkv;
+    if (MUT(26)) { double *tmp = k; k = v; v = tmp; }
+    for (int32_t h = 0; h < H; ++h)
+        or_rope(q + (int64_t)h * hd, hd, pos, c->rope_theta);
+    for (int32_t g = 0; g < Hkv; ++g) {
+        or_rope(k + (int64_t)g * hd, hd, pos, c->rope_theta);
+        if (MUT(27))
+            or_rope(v + (int64_t)g * hd, hd, pos, c->rope_theta);
+    }
+    or_attention(q, H, Hkv, hd, kc, vc, c->dtype, cap, P, k, v, o);
+    or_matvec(lw[2], c->dtype, d, nq, o, t);
+    for (int32_t j = 0; j < d; ++j)
+        x[j] = MUT(7) ? t[j] : x[j] + t[j];
+
+    /* MLP block */
+    or_rmsnorm(x, lw[3], c->dtype, d, c->rms_eps, u);
+    or_matvec(lw[4], c->dtype, F, d, u, gt);
+    or_matvec(lw[5], c->dtype, F, d, u, up);
+    or_silu_mul(gt, up, F, a);
+    or_matvec(lw[6], c->dtype, d, F, a, t);
+    for (int32_t j = 0; j < d; ++j)
+        x[j] = MUT(8) ? t[j] : x[j] + t[j];
+
+    free(u); free(qkv); free(o); free(t); free(gt); free(up); free(a);
+}
+
+/* Sec. 2.1: logits of one hidden state through the (optional) final RMSNorm and the
+ * frozen LM head W_lm [V, d]. */
+void or_lm_head(const or_config *c, const void *lm_head, const void *final_norm,
+                const double *h, double *logits)
+{
+    double *z = (double *)malloc(sizeof(double) * (size_t)c->d);
+    if (c->final_norm && !MUT(17))
+        or_rmsnorm(h, final_norm, c->dtype, c->d, c->rms_eps, z);
+    else
+        memcpy(z, h, sizeof(double) * (size_t)c->d);
+    or_matvec(lm_head, c->dtype, c->vocab, c->d, z, logits);
+    free(z);
+}
+
+/* Softmax of logits / T with its log-normaliser: lse = max + log sum exp(l/T - max),
+ * p_v = exp(l_v/T - lse). T <= 0 (greedy decoding) uses T = 1: the distribution the
+ * drafter proposes from. */
+void or_softmax(const double *logits, int64_t V, double T, double *p, double *lse)
+{
+    const double tt = (T > 0.0 && !MUT(20)) ? T : 1.0;
+    double mx = -INFINITY;
+    for (int64_t v = 0; v < V; ++v)
+        if (logits[v] / tt > mx)
+            mx = logits[v] / tt;
+    double s = 0.0;
+    for (int64_t v = 0; v < V; ++v)
+        s += exp(logits[v] / tt - mx);
+    double l = MUT(21) ? log(s) : mx + log(s);
+    if (lse)
+        *lse = l;
+    if (p)
+        for (int64_t v = 0; v < V; ++v)
+            p[v] = exp(logits[v] / tt - l);
+}
+
+/* The k most probable tokens, best first: the first k entries of a stable sort by
+ * (descending logit, ascending id). Selection by repeated scan. */
+void or_topk(const double *logits, int64_t V, int32_t k, int32_t *ids)
+{
+    unsigned char *taken = (unsigned char *)calloc((size_t)V, 1);
+    for (int32_t r = 0; r < k; ++r) {
+        int64_t best = -1;
+        for (int64_t v = 0; v < V; ++v) {
+            if (taken[v])
+                continue;
+            if (best < 0 || logits[v] > logits[best] ||
+                (MUT(12) && logits[v] == logits[best]))
+                best = v;
+        }
+        ids[r] = (int32_t)best;
+        taken[best] = 1;
+    }
+    free(taken);
+}
+
+/* Sec. 2.2, Backbone Expansion, in level-major order with T = 1 + N k nodes.
+ *   node 0: the root, token `root` (the last verified token whose embedding fed the
+ *           cascade), parent -1, depth 0;
+ *   level i = 1..N: nodes 1 + (i-1)k + r, r = 0..k-1, hold topk[i-1][r] in rank
+ *           order at depth i; their parent is the root for i = 1 and the previous
+ *           level's rank-0 (backbone) node 1 + (i-2)k otherwise;
+ *   mask[a][c] = 1 iff c is a or an ancestor of a. */
+void or_tree(int32_t N, int32_t k, int32_t root, const int32_t *topk, int32_t *tok,
+             int32_t *parent, int32_t *depth, uint8_t *mask)
+{
+    const int32_t T = 1 + N * k;
+    tok[0] = root;
+    parent[0] = -1;
+    depth[0] = 0;
+    for (int32_t i = 1; i <= N; ++i) {
+        for (int32_t r = 0; r < k; ++r) {
+            int32_t n = 1 + (i - 1) * k + r;
+            tok[n] = topk[(int64_t)(i - 1) * k + r];
+            depth[n] = MUT(28) ? i - 1 : i;
+            if (i == 1)
+                parent[n] = 0;
+            else
+                parent[n] = MUT(13) ? 1 + (i - 2) * k + (k - 1) : 1 + (i - 2) * k;
+        }
+    }
+    memset(mask, 0, (size_t)T * (size_t)T);
+    for (int32_t a = 0; a < T; ++a) {
+        if (!MUT(16))
+            mask[(int64_t)a * T + a] = 1;
+        for (int32_t c = parent[a]; c >= 0; c = parent[c])
+            mask[(int64_t)a * T + c] = 1;
+    }
+}
+
+/* The whole draft of one sequence (Eq. 1, Eq. 2, Sec. 2.1 LM head, Sec. 2.2 top-k).
+ *   w     : 5 + 7N pointers: w_fuse [d,3d], w_in [d,2d], embed [V,d], lm_head [V,d],
+ *           final_norm [d], then per layer attn_norm, w_qkv, w_o, mlp_norm, w_gate,
+ *           w_up, w_down
+ *   feat  : [3d] = concat(l, m, h) of the last verified position
+ *   tok   : the next token t+1 whose embedding joins the fused feature
+ *   P     : prefix length (the drafted row's sequence position under the default reading)
+ *   kc, vc: N pointers, each this sequence's [Hkv][cap][hd] cache of layer i
+ * Outputs: hidden [N][d]; logits [N][V] (may be NULL); lse [N]; topk_id [N][k];
+ * topk_logit [N][k]; topk_prob [N][k]. */
+int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat, int32_t tok,
+                     int32_t P, const void *const *kc, const void *const *vc, int64_t cap,
+                     int32_t top_k, double temperature, double *hidden, double *logits,
+                     double *lse, int32_t *topk_id, double *topk_logit, double *topk_prob)
+{
+    const int32_t d = c->d, V = c->vocab, N = c->n_layers;
+    if (tok < 0 || tok >= V || P < 0 || P + 1 > cap || top_k < 1 || top_k > V)
+        return -1;
+    double *f = (double *)malloc(sizeof(double) * (size_t)(3 * d));
+    double *ge = (double *)malloc(sizeof(double) * (size_t)(2 * d));
+    double *x0 = (double *)malloc(sizeof(double) * (size_t)d);
+    double *x = (double *)malloc(sizeof(double) * (size_t)d);
+    double *lg = (double *)malloc(sizeof(double) * (size_t)V);
+    double *pr = (double *)malloc(sizeof(double) * (size_t)V);
+
+    /* g = FC(concat(l, m, h)) */
+    or_widen(feat, c->dtype, 3 * d, f);
+    if (MUT(18))
+        for (int32_t j = 2 * d; j < 3 * d; ++j)
+            f[j] = 0.0;
+    double *g = MUT(14) ? ge + d : ge;
+    double *e = MUT(14) ? ge : ge + d;
+    or_matvec(w[0], c->dtype, d, 3 * d, f, g);
+    /* e = Embed[tok] */
+    const int64_t row = MUT(15) ? (tok + 1) % V : tok;
+    for (int32_t j = 0; j < d; ++j)
+        e[j] = ld(w[2], c->dtype, row * d + j);
+    /* x0 = FC(concat(g, e))   (Eq. 1) */
+    or_matvec(w[1], c->dtype, d, 2 * d, ge, x0);
+    memcpy(x, x0, sizeof(double) * (size_t)d);
+
+    /* h_i = L_i(h_{i-1})      (Eq. 2) */
+    for (int32_t i = 0; i < N; ++i) {
+        if (MUT(10))
+            memcpy(x, x0, sizeof(double) * (size_t)d);
+        double pos = (double)P + (c->rope_layer_offset ? (double)i : 0.0) + (MUT(19) ? 1.0 : 0.0);
+        or_layer(c, w + 5 + 7 * i, pos, kc[i], vc[i], cap, P, x);
+        memcpy(hidden + (int64_t)i * d, x, sizeof(double) * (size_t)d);
+    }
+
+    /* q_{t+i} through the frozen LM head; top-k per depth (Sec. 2.1, Sec. 2.2) */
+    for (int32_t i = 0; i < N; ++i) {
+        or_lm_head(c, w[3], w[4], hidden + (int64_t)i * d, lg);
+        or_softmax(lg, V, temperature, pr, lse + i);
+        or_topk(lg, V, top_k, topk_id + (int64_t)i * top_k);
+        for (int32_t r = 0; r < top_k; ++r) {
+            int32_t id = topk_id[(int64_t)i * top_k + r];
+            topk_logit[(int64_t)i * top_k + r] = lg[id];
+            topk_prob[(int64_t)i * top_k + r] = pr[id];
+        }
+        if (logits)
+            memcpy(logits + (int64_t)i * V, lg, sizeof(double) * (size_t)V);
+    }
+    free(f); free(ge); free(x0); free(x); free(lg); free(pr);
+    return 0;
+}
+
+/* Threads the OpenMP runtime will use (reported beside CPU timings). */
+int32_t or_max_threads(void)
+{
+#ifdef _OPENMP
+    extern int omp_get_max_threads(void);
+    return (int32_t)omp_get_max_threads();
+#else
+    return 1;
+#endif
+}

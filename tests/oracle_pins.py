@@ -1,0 +1,366 @@
+"""Pins of the fp64 oracle: checks against what the paper and mathematics fix.
+
+Each ``pin_*`` takes an ``oracle.Oracle`` and raises AssertionError when the oracle
+disagrees with a closed form, a brute-force sum, a library special case, an invariant
+or the hand-worked tree fixtures under tests/golden/. ``test_oracle_pins.py`` runs them
+on the real oracle; ``test_oracle_mutants.py`` runs them on builds with one planted
+mistake each and requires every mutant to fail at least one pin.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import torch
+
+import fe_synth
+from fe_synth import workloads as wl
+
+import torch_ref
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _bf16_bits(x: np.ndarray) -> np.ndarray:
+    """float32 -> bfloat16 bit patterns (uint16), round to nearest even."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return u.astype(np.uint16)
+
+
+def _bf16_value(b: np.ndarray) -> np.ndarray:
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+# ---- linear algebra -------------------------------------------------------------------
+
+def pin_matvec_bruteforce(orc):
+    """y = W x on a non-square matrix against an exact rational sum (both storage types)."""
+    rng = np.random.default_rng(11)
+    W = rng.standard_normal((5, 7)).astype(np.float32)
+    x = rng.standard_normal(7)
+    exact = [sum(Fraction(float(W[m, k])) * Fraction(float(x[k])) for k in range(7))
+             for m in range(5)]
+    y = orc.matvec(W, x)
+    for m in range(5):
+        assert abs(y[m] - float(exact[m])) <= 1e-13 * (1 + abs(float(exact[m]))), (m, y[m])
+    Wb = _bf16_bits(W)
+    Wv = _bf16_value(Wb)
+    exact = [sum(Fraction(float(Wv[m, k])) * Fraction(float(x[k])) for k in range(7))
+             for m in range(5)]
+    y = orc.matvec(Wb, x)
+    for m in range(5):
+        assert abs(y[m] - float(exact[m])) <= 1e-13 * (1 + abs(float(exact[m])))
+
+
+def pin_rmsnorm(orc):
+    n = 12
+    # constant vector: mean(x^2) = c^2, so y = gamma c / sqrt(c^2 + eps); eps matters at c=1e-3
+    c, eps = 1e-3, 1e-5
+    gamma = np.linspace(0.5, 2.0, n).astype(np.float32)
+    y = orc.rmsnorm(np.full(n, c), gamma, eps)
+    want = gamma.astype(np.float64) * c / math.sqrt(c * c + eps)
+    assert np.allclose(y, want, rtol=1e-13, atol=0)
+    # unit gain, eps = 0: the output has root-mean-square exactly 1 and is scale invariant
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal(n) * 7.0
+    y = orc.rmsnorm(x, np.ones(n, np.float32), 0.0)
+    assert abs(math.sqrt(np.mean(y * y)) - 1.0) < 1e-14
+    y2 = orc.rmsnorm(x * 1e3, np.ones(n, np.float32), 0.0)
+    assert np.allclose(y, y2, rtol=1e-13)
+
+
+# ---- RoPE -----------------------------------------------------------------------------
+
+def pin_rope(orc):
+    hd, theta = 8, 10000.0
+    half = hd // 2
+    rng = np.random.default_rng(5)
+    v = rng.standard_normal(hd)
+    assert np.allclose(orc.rope(v, 0.0, theta), v, rtol=0, atol=0)  # position 0: identity
+    for m in (1.0, 3.0, 17.0):
+        for j in range(half):
+            w = m * theta ** (-2.0 * j / hd)
+            e = np.zeros(hd)
+            e[j] = 1.0
+            r = orc.rope(e, m, theta)
+            want = np.zeros(hd)
+            want[j], want[j + half] = math.cos(w), math.sin(w)
+            assert np.allclose(r, want, atol=1e-15), (m, j, r)
+            e = np.zeros(hd)
+            e[j + half] = 1.0
+            r = orc.rope(e, m, theta)
+            want = np.zeros(hd)
+            want[j], want[j + half] = -math.sin(w), math.cos(w)
+            assert np.allclose(r, want, atol=1e-15), (m, j, r)
+    # norm preservation and dependence on the relative position only
+    q, k = rng.standard_normal(hd), rng.standard_normal(hd)
+    assert abs(np.linalg.norm(orc.rope(q, 9.0, theta)) - np.linalg.norm(q)) < 1e-13
+    a = orc.rope(q, 5.0, theta) @ orc.rope(k, 2.0, theta)
+    b = orc.rope(q, 105.0, theta) @ orc.rope(k, 102.0, theta)
+    assert abs(a - b) < 1e-12
+    # the complex-rotation form
+    want = torch_ref.rope_complex(torch.tensor(q), 7.0, theta).numpy()
+    assert np.allclose(orc.rope(q, 7.0, theta), want, atol=1e-14)
+
+
+# ---- attention ------------------------------------------------------------------------
+
+def _kv(rng, Hkv, cap, hd):
+    return (rng.standard_normal((Hkv, cap, hd)).astype(np.float32),
+            rng.standard_normal((Hkv, cap, hd)).astype(np.float32))
+
+
+def pin_attention(orc):
+    rng = np.random.default_rng(7)
+    H, Hkv, hd, cap = 4, 2, 8, 10
+    kc, vc = _kv(rng, Hkv, cap, hd)
+    q = rng.standard_normal((H, hd))
+    kn, vn = rng.standard_normal((Hkv, hd)), rng.standard_normal((Hkv, hd))
+    # P = 0: the only key is the row's own; output = own value of the head's group
+    o = orc.attention(q, kc, vc, 0, kn, vn)
+    for h in range(H):
+        assert np.allclose(o[h], vn[h * Hkv // H], atol=1e-15)
+    # all keys equal: uniform weights, output = mean of the P + 1 values
+    P = 6
+    kc_eq = np.repeat(kn.astype(np.float32)[:, None, :], cap, axis=1)
+    kn_eq = kc_eq[:, 0, :].astype(np.float64)
+    o = orc.attention(q, kc_eq, vc, P, kn_eq, vn)
+    for h in range(H):
+        g = h * Hkv // H
+        mean = (vc[g, :P].astype(np.float64).sum(0) + vn[g]) / (P + 1)
+        assert np.allclose(o[h], mean, atol=1e-13)
+    # two keys, closed form of the scaled softmax
+    q1 = np.zeros((1, 4)); q1[0, 0] = 1.0
+    kc1 = np.zeros((1, 2, 4), np.float32); kc1[0, 0, 0] = 2.0
+    vc1 = np.zeros((1, 2, 4), np.float32); vc1[0, 0, 1] = 1.0
+    kn1 = np.zeros((1, 4)); kn1[0, 0] = -1.0
+    vn1 = np.zeros((1, 4)); vn1[0, 2] = 1.0
+    o = orc.attention(q1, kc1, vc1, 1, kn1, vn1)
+    s0, s1 = 2.0 / 2.0, -1.0 / 2.0  # q.k / sqrt(4)
+    w0 = math.exp(s0) / (math.exp(s0) + math.exp(s1))
+    assert np.allclose(o[0], [0.0, w0, 1.0 - w0, 0.0], atol=1e-15)
+    # grouped-query attention equals MHA over replicated KV heads
+    rep = H // Hkv
+    kc_r = np.repeat(kc, rep, axis=0)
+    vc_r = np.repeat(vc, rep, axis=0)
+    o_gqa = orc.attention(q, kc, vc, P, kn, vn)
+    o_mha = orc.attention(q, kc_r, vc_r, P, np.repeat(kn, rep, 0), np.repeat(vn, rep, 0))
+    assert np.allclose(o_gqa, o_mha, atol=1e-14)
+    # library special case: torch scaled_dot_product_attention in fp64
+    keys = torch.cat([torch.tensor(kc_r[:, :P], dtype=torch.float64),
+                      torch.tensor(np.repeat(kn, rep, 0))[:, None]], 1)
+    vals = torch.cat([torch.tensor(vc_r[:, :P], dtype=torch.float64),
+                      torch.tensor(np.repeat(vn, rep, 0))[:, None]], 1)
+    ref = torch.nn.functional.scaled_dot_product_attention(torch.tensor(q)[:, None], keys, vals)
+    assert np.allclose(o_gqa, ref[:, 0].numpy(), atol=1e-13)
+
+
+def pin_silu_mul(orc):
+    g = np.array([0.0, 1.0, -2.0, 30.0])
+    u = np.array([5.0, 2.0, 3.0, 0.5])
+    y = orc.silu_mul(g, u)
+    want = [0.0, 2.0 / (1.0 + math.exp(-1.0)), -6.0 / (1.0 + math.exp(2.0)),
+            15.0 / (1.0 + math.exp(-30.0))]
+    assert np.allclose(y, want, rtol=1e-15, atol=0)
+
+
+# ---- softmax, top-k, tree ---------------------------------------------------------------
+
+def pin_softmax(orc):
+    p, lse = orc.softmax(np.log([1.0, 2.0, 3.0]))
+    assert np.allclose(p, [1 / 6, 2 / 6, 3 / 6], rtol=1e-14) and abs(lse - math.log(6)) < 1e-14
+    p, lse = orc.softmax(np.log([1.0, 2.0, 3.0]), T=2.0)  # p ~ sqrt of the weights
+    s = 1 + math.sqrt(2) + math.sqrt(3)
+    assert np.allclose(p, [1 / s, math.sqrt(2) / s, math.sqrt(3) / s], rtol=1e-14)
+    assert abs(lse - math.log(s)) < 1e-14
+    p0, _ = orc.softmax(np.log([1.0, 2.0, 3.0]), T=0.0)  # greedy: the T = 1 distribution
+    assert np.allclose(p0, [1 / 6, 2 / 6, 3 / 6], rtol=1e-14)
+    rng = np.random.default_rng(9)
+    lg = rng.standard_normal(5000) * 4 + 600.0  # large offset: needs the max shift
+    p, lse = orc.softmax(lg)
+    assert abs(p.sum() - 1.0) < 1e-12
+    m = lg.max()
+    assert abs(lse - (m + math.log(math.fsum(math.exp(v - m) for v in lg)))) < 1e-10
+
+
+def pin_topk(orc):
+    rng = np.random.default_rng(2)
+    lg = np.round(rng.standard_normal(300) * 3, 1)  # many exact ties
+    for k in (1, 5, 17, 300):
+        want = np.argsort(-lg, kind="stable")[:k]
+        assert np.array_equal(orc.topk(lg, k), want), k
+
+
+def _check_tree_invariants(N, k, root, topk, tok, par, dep, mask):
+    T = 1 + N * k
+    assert tok.shape == (T,) and mask.shape == (T, T)
+    assert tok[0] == root and par[0] == -1 and dep[0] == 0
+    assert dep.max() == N and (dep <= N).all()
+    for n in range(1, T):
+        assert 0 <= par[n] < n and dep[n] == dep[par[n]] + 1
+    # level i holds q_{t+i}'s candidates in rank order
+    for i in range(1, N + 1):
+        assert list(tok[1 + (i - 1) * k: 1 + i * k]) == list(topk[i - 1])
+    # exactly one backbone chain of length N made of rank-0 nodes; side branches are leaves
+    backbone = [0] + [1 + (i - 1) * k for i in range(1, N + 1)]
+    for a, b in zip(backbone, backbone[1:]):
+        assert par[b] == a
+    has_child = set(int(p) for p in par[1:])
+    assert has_child == set(backbone[:-1])
+    for i in range(1, N + 1):  # at most k - 1 side branches per level
+        assert sum(1 for n in range(T) if dep[n] == i and n not in backbone) == k - 1
+    # mask: ancestor-or-self, lower-triangular, popcount = depth + 1
+    assert (np.triu(mask, 1) == 0).all() and (np.diag(mask) == 1).all()
+    for a in range(T):
+        anc = {a}
+        c = par[a]
+        while c >= 0:
+            anc.add(int(c))
+            c = par[c]
+        assert set(np.nonzero(mask[a])[0].tolist()) == anc
+        assert mask[a].sum() == dep[a] + 1
+    if k == 1:
+        assert list(par) == list(range(-1, T - 1))
+
+
+def pin_tree(orc):
+    for name in ("tree_backbone_n3_k3.json", "tree_chain_n4_k1.json"):
+        with open(os.path.join(GOLDEN, name)) as f:
+            G = json.load(f)
+        tok, par, dep, mask = orc.tree(G["N"], G["k"], G["root"], np.array(G["topk"]))
+        assert tok.tolist() == G["tok"], name
+        assert par.tolist() == G["parent"], name
+        assert dep.tolist() == G["depth"], name
+        assert ["".join(str(int(b)) for b in row) for row in mask] == G["mask"], name
+    rng = np.random.default_rng(4)
+    for N, k in ((1, 1), (1, 5), (5, 1), (4, 3), (8, 10)):
+        topk = rng.integers(0, 1000, size=(N, k)).astype(np.int32)
+        out = orc.tree(N, k, 77, topk)
+        _check_tree_invariants(N, k, 77, topk, *out)
+
+
+# ---- the whole cascade -------------------------------------------------------------------
+
+def mini_cfg(**kw):
+    base = dict(d=16, n_heads=4, n_kv_heads=2, head_dim=4, ffn=24, vocab=40, n_layers=3,
+                dtype="f32", B=2, prefix=3, top_k=5, rope_theta=100.0, seed=21, page_size=0,
+                max_seq=8)
+    base.update(kw)
+    return wl.make_config(base)
+
+
+def _mini_problem(cfg):
+    W = wl.make_weights(cfg)
+    # non-trivial gains so a norm with a wrong gain index would show
+    for L in W["layers"]:
+        for key in ("attn_norm", "mlp_norm"):
+            t = torch.empty(cfg["d"], dtype=wl.torch_dtype(cfg))
+            fe_synth.fill_normal(t, cfg["seed"], 900 + len(key), 0.3)
+            L[key] = (t.float() + 1.0).to(t.dtype)
+    t = torch.empty(cfg["d"], dtype=wl.torch_dtype(cfg))
+    fe_synth.fill_normal(t, cfg["seed"], 950, 0.3)
+    W["final_norm"] = (t.float() + 1.0).to(t.dtype)
+    # larger weights than 0.02 so every block moves the hidden state visibly
+    scale = 0.4
+    for key in ("w_fuse", "w_in", "embed", "lm_head"):
+        W[key] = (W[key].float() * (scale / 0.02)).to(W[key].dtype)
+    for L in W["layers"]:
+        for key in ("w_qkv", "w_o", "w_gate", "w_up", "w_down"):
+            L[key] = (L[key].float() * (scale / 0.02)).to(L[key].dtype)
+    I = wl.make_inputs(cfg)
+    ks, vs = wl.make_caches(cfg)
+    return W, I, ks, vs
+
+
+def _draft_both(orc, cfg, W, I, ks, vs, b, **kw):
+    P = int(I["prefix_len"][b])
+    kcs = [k[b].contiguous() for k in ks]
+    vcs = [v[b].contiguous() for v in vs]
+    o = orc.draft_seq(cfg, W, I["feat"][b].contiguous(), int(I["next_tok"][b]), P, kcs, vcs,
+                      cfg["max_seq"], cfg["top_k"], cfg["temperature"], **kw)
+    r = torch_ref.draft(cfg, W, I["feat"][b], int(I["next_tok"][b]), P, kcs, vcs, cfg["top_k"],
+                        cfg["temperature"], kw.get("rope_layer_offset", 0))
+    return o, r
+
+
+def _agree(o, r, tol=1e-10):
+    for key in ("hidden", "logits", "lse"):
+        a, b = o[key], r[key].numpy()
+        assert np.allclose(a, b, rtol=tol, atol=tol * max(1.0, np.abs(b).max())), key
+    # probabilities of the chosen candidates, and the candidates themselves
+    p = r["prob"].numpy()
+    for i in range(o["topk_id"].shape[0]):
+        assert np.array_equal(o["topk_id"][i], r["topk_id"][i].numpy())
+        assert np.allclose(o["topk_prob"][i], p[i][o["topk_id"][i]], rtol=tol, atol=1e-15)
+        assert np.allclose(o["topk_logit"][i], o["logits"][i][o["topk_id"][i]], rtol=0, atol=0)
+
+
+def pin_draft_n1(orc):
+    """N = 1: the drafter is a single EAGLE-style decoder layer plus the LM head."""
+    for dtype in ("f32", "bf16"):
+        cfg = mini_cfg(n_layers=1, dtype=dtype)
+        W, I, ks, vs = _mini_problem(cfg)
+        for b in range(cfg["B"]):
+            o, r = _draft_both(orc, cfg, W, I, ks, vs, b)
+            _agree(o, r)
+
+
+def pin_cascade(orc):
+    """N = 3 with grouped-query heads: h_i = L_i(h_{i-1}) (Eq. 2), T = 1 and T = 0.7."""
+    for T in (0.0, 0.7):
+        cfg = mini_cfg(temperature=T)
+        W, I, ks, vs = _mini_problem(cfg)
+        o, r = _draft_both(orc, cfg, W, I, ks, vs, 1)
+        _agree(o, r)
+    cfg = mini_cfg(n_layers=2, rope_layer_offset=1)
+    W, I, ks, vs = _mini_problem(cfg)
+    o, r = _draft_both(orc, cfg, W, I, ks, vs, 0, rope_layer_offset=1)
+    _agree(o, r)
+
+
+def pin_truncation(orc):
+    """Layers 1..j of an N-layer cascade equal a j-layer cascade with the same first j layers."""
+    cfg = mini_cfg(n_layers=4, B=1)
+    W, I, ks, vs = _mini_problem(cfg)
+    o4 = orc.draft_seq(cfg, W, I["feat"][0].contiguous(), int(I["next_tok"][0]), 3,
+                       [k[0].contiguous() for k in ks], [v[0].contiguous() for v in vs],
+                       cfg["max_seq"], cfg["top_k"])
+    cfg2 = dict(cfg, n_layers=2)
+    W2 = dict(W, layers=W["layers"][:2])
+    o2 = orc.draft_seq(cfg2, W2, I["feat"][0].contiguous(), int(I["next_tok"][0]), 3,
+                       [k[0].contiguous() for k in ks[:2]], [v[0].contiguous() for v in vs[:2]],
+                       cfg["max_seq"], cfg["top_k"])
+    for key in ("hidden", "logits", "lse", "topk_id"):
+        assert np.array_equal(o4[key][:2], o2[key]), key
+
+
+def pin_zero_blocks(orc):
+    """W_o = W_down = 0: every layer passes x0 through, so all N distributions coincide."""
+    cfg = mini_cfg(n_layers=3, B=1)
+    W, I, ks, vs = _mini_problem(cfg)
+    for L in W["layers"]:
+        L["w_o"] = torch.zeros_like(L["w_o"])
+        L["w_down"] = torch.zeros_like(L["w_down"])
+    o = orc.draft_seq(cfg, W, I["feat"][0].contiguous(), int(I["next_tok"][0]), 3,
+                      [k[0].contiguous() for k in ks], [v[0].contiguous() for v in vs],
+                      cfg["max_seq"], cfg["top_k"])
+    f = I["feat"][0].double()
+    x0 = W["w_in"].double() @ torch.cat([W["w_fuse"].double() @ f,
+                                         W["embed"].double()[int(I["next_tok"][0])]])
+    for i in range(3):
+        assert np.allclose(o["hidden"][i], x0.numpy(), rtol=1e-13, atol=1e-13)
+        assert np.array_equal(o["topk_id"][i], o["topk_id"][0])
+        assert np.array_equal(o["logits"][i], o["logits"][0])
+    tok, par, dep, mask = orc.tree(3, cfg["top_k"], 1, o["topk_id"])
+    k = cfg["top_k"]
+    for i in range(1, 3):
+        assert list(tok[1 + i * k: 1 + (i + 1) * k]) == list(tok[1:1 + k])
+
+
+ALL_PINS = [pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
+            pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
+            pin_zero_blocks]
