@@ -1,0 +1,299 @@
+#!/usr/bin/env python3
+"""Benchmark: drafts/s of the single-pass cascaded drafter on one GB300 per rank.
+
+One step = fe_draft_forward + fe_build_tree over one batch of the workload (the whole
+hot path: fused-feature input FCs, N cascade layers, LM head with fused softmax/top-k,
+Backbone Expansion tree). Default workload: the Vicuna-13B-shaped drafter (d=5120,
+40 heads x 128, F=13824, V=32000, N=5, B=1, P=512, k=8, bf16 weights/caches), with
+seeded synthetic inputs. The 3.8 GB of weights read per step exceed the 129 MB L2, so
+no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Multi-GPU (torchrun): replicas only. Every rank drafts its own batch with its own copy
+of the drafter; there is no collective on the data path (a barrier brackets the timed
+region and the slowest rank's time is reported), so the scaling is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+HBM_FALLBACK_GBS = 6800.0  # used only when MEASURED_PEAKS.json is absent
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="vic13b")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    return HBM_FALLBACK_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def make_problem(name: str):
+    from fe_synth import workloads as wl
+    cfg = wl.make_config(name)
+    W = wl.make_weights(cfg)
+    I = wl.make_inputs(cfg)
+    ks, vs = wl.make_caches(cfg)
+    return cfg, W, I, ks, vs
+
+
+def time_oracle(cfg, W, I, ks, vs, budget_s: float, max_runs: int | None = None):
+    """The fp64 oracle as it stands, on the host cores, over a bounded sample of drafts
+    (sequence b = run % B). Returns (drafts/s, runs, threads, seconds)."""
+    import oracle
+    orc = oracle.load()
+    B = cfg["B"]
+    runs, t0 = 0, time.perf_counter()
+    while True:
+        b = runs % B
+        orc.draft_seq(cfg, W, I["feat"][b].contiguous(), int(I["next_tok"][b]), int(I["prefix_len"][b]),
+                      [k[b].contiguous() for k in ks], [v[b].contiguous() for v in vs], cfg["max_seq"],
+                      cfg["top_k"], cfg["temperature"], want_logits=False)
+        runs += 1
+        el = time.perf_counter() - t0
+        if (max_runs and runs >= max_runs) or (not max_runs and el >= budget_s and runs >= 2):
+            break
+    return runs / el, runs, orc.max_threads(), el
+
+
+def workload_config(cfg, wl) -> dict:
+    return {"workload": cfg.get("name", ""), "shape": wl.describe(cfg), "B": cfg["B"], "N": cfg["n_layers"],
+            "top_k": cfg["top_k"], "d": cfg["d"], "vocab": cfg["vocab"], "accum": "f32",
+            "l2": "inputs larger than L2 (every step streams all weights, >129 MB)" if cfg["dtype"] == "bf16"
+            else "L2-resident (no flush)"}
+
+
+def run_reference(args, ws, rank):
+    """The oracle, timed on this machine's host cores (the reference arm of this benchmark)."""
+    if rank != 0:
+        return
+    from fe_synth import workloads as wl
+    cfg, W, I, ks, vs = make_problem(args.workload)
+    cfg["name"] = args.workload
+    # warm-up runs, then a bounded number of timed steps (one draft of sequence step % B each)
+    time_oracle(cfg, W, I, ks, vs, 0, max_runs=max(1, min(args.warmup, 2)))
+    one, _, thr, _ = time_oracle(cfg, W, I, ks, vs, 0, max_runs=1)
+    steps = max(1, min(args.steps, int(120.0 * one)))  # keep the arm within ~2 minutes
+    rate, runs, thr, el = time_oracle(cfg, W, I, ks, vs, 0, max_runs=steps)
+    value = rate  # drafts/s (one sequence's N-token draft per step)
+    line = {"metric": "drafts/s", "value": value, "unit": "drafts/s", "n_gpus": ws, "steps": runs,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * el / runs, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
+            "config": workload_config(cfg, wl), "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": "drafts/s", "cores": thr, "kind": "oracle",
+                             "sample": f"{runs} single-sequence drafts of the workload"},
+            "e2e": {"value": value, "unit": "drafts/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    import torch
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import paper_2509_20416_gb300 as fe
+    from fe_synth import workloads as wl
+
+    cfg, W, I, ks, vs = make_problem(args.workload)
+    cfg["name"] = args.workload
+    B, N, k = cfg["B"], cfg["n_layers"], cfg["top_k"]
+    h = fe.fe_draft_init(dict(cfg, max_batch=B), W)
+    if cfg["page_size"]:
+        table, n_pages = wl.page_plan(cfg, I["prefix_len"])
+        kd = [wl.paginate(cfg, t, table, n_pages).cuda() for t in ks]
+        vd = [wl.paginate(cfg, t, table, n_pages).cuda() for t in vs]
+        table = table.cuda()
+    else:
+        kd, vd, table, n_pages = [t.cuda() for t in ks], [t.cuda() for t in vs], None, 0
+    feat, tok, plen = I["feat"].cuda(), I["next_tok"].cuda(), I["prefix_len"].cuda()
+    out = fe.alloc_outputs(h, B, k)
+    tree = fe.alloc_tree(h, B, k)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        fe.fe_draft_forward(h, feat, tok, plen, kd, vd, k, cfg["temperature"], page_table=table,
+                            n_pages=n_pages, out=out, stream=stream)
+        fe.fe_build_tree(h, tok, out["topk_id"], k, out=tree, stream=stream)
+
+    def barrier():
+        if ws > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    st = fe.fe_last_device_status(h)
+    if st != fe.FE_OK:
+        raise SystemExit(f"device status after warm-up: {fe.fe_status_str(st)}")
+
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1)
+    if ws > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = ws * B / (ms_step / 1e3)
+    st = fe.fe_last_device_status(h)
+    if st != fe.FE_OK:
+        raise SystemExit(f"device status after the timed region: {fe.fe_status_str(st)}")
+
+    # ---- end to end through the public API with host buffers ------------------------------
+    pin = {n: t.pin_memory() for n, t in (("feat", I["feat"]), ("tok", I["next_tok"]),
+                                          ("plen", I["prefix_len"]))}
+    host_out = {n: torch.empty_like(t, device="cpu").pin_memory() for n, t in out.items()}
+    host_tree = {n: torch.empty_like(t, device="cpu").pin_memory() for n, t in tree.items()}
+    h2d = sum(t.numel() * t.element_size() for t in pin.values())
+    d2h = sum(t.numel() * t.element_size() for t in list(out.values()) + list(tree.values()))
+
+    def e2e_step():
+        feat.copy_(pin["feat"], non_blocking=True)
+        tok.copy_(pin["tok"], non_blocking=True)
+        plen.copy_(pin["plen"], non_blocking=True)
+        step()
+        for n, t in out.items():
+            host_out[n].copy_(t, non_blocking=True)
+        for n, t in tree.items():
+            host_tree[n].copy_(t, non_blocking=True)
+        stream.synchronize()
+
+    for _ in range(3):
+        e2e_step()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+    if ws > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    # ---- roofline of the draft step ------------------------------------------------------
+    peak, peak_kind = peaks()
+    alg_bytes = wl.algorithmic_bytes(cfg, I["prefix_len"].tolist())
+    achieved = alg_bytes / (ms_step / 1e3) / 1e9
+    launches = fe.fe_launch_count(h, B, True)
+
+    line = {"metric": "drafts/s", "value": value, "unit": "drafts/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "us_per_draft": ms_step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
+            "data": "synthetic (seeded generator)", "config": workload_config(cfg, wl),
+            "roofline": {"bound": "hbm", "kernel": "draft step (fe_draft_forward + fe_build_tree)",
+                         "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "peak_kind": peak_kind, "algorithmic_bytes": alg_bytes, "traffic": None},
+            "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches * args.steps, "launches_per_step": launches,
+            "clocks": clocks}
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        rate, runs, thr, el = time_oracle(cfg, W, I, ks, vs, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": rate, "unit": "drafts/s", "cores": thr, "kind": "oracle",
+                                "sample": f"{runs} single-sequence drafts of the workload ({el:.1f} s)"}
+    h.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -70,6 +70,9 @@ def make_config(name_or_dict, **overrides) -> dict:
     w.setdefault("temperature", 0.0)
     p = w["prefix"]
     pmax = p[1] if isinstance(p, (tuple, list)) else p
+    if w.get("prefix_list") is not None:  # explicit per-sequence prefix lengths
+        assert len(w["prefix_list"]) == w["B"]
+        pmax = max(w["prefix_list"])
     # capacity: the prefix plus the drafted row, rounded up to a whole 16-row block
     w.setdefault("max_seq", ((pmax + 1 + 15) // 16) * 16)
     w.setdefault("top_k_max", max(16, w["top_k"]))
@@ -119,7 +122,9 @@ def make_inputs(cfg: dict) -> dict:
     fill_uniform_int(tok, s, TID_TOK, 0, V - 1)
     p = cfg["prefix"]
     plen = torch.empty(B, dtype=torch.int32)
-    if isinstance(p, (tuple, list)):
+    if cfg.get("prefix_list") is not None:
+        plen = torch.tensor(cfg["prefix_list"], dtype=torch.int32)
+    elif isinstance(p, (tuple, list)):
         fill_uniform_int(plen, s, TID_PREFIX, p[0], p[1])
     else:
         plen.fill_(p)

@@ -1,0 +1,186 @@
+/*
+ * fe_draft.h -- C ABI of the GB300 (sm_103a) FastEagle cascaded drafter.
+ *
+ * FastEagle (arXiv 2509.20416) drafts N tokens in one forward pass: the target's
+ * multi-level features of the last verified position are fused by an FC layer,
+ * joined with the next token's embedding and a second FC (Sec. 2.1, Eq. 1), and
+ * pushed through N serially connected decoder layers h_i = L_i(h_{i-1}) (Eq. 2).
+ * Every h_i goes through the target's frozen LM head to give the distribution
+ * q_{t+i} (Sec. 2.1). The k most probable tokens per depth are then arranged into
+ * the Backbone Expansion draft tree (Sec. 2.2) that the target verifies with tree
+ * attention (Sec. 2.4).
+ *
+ * Conventions for every call:
+ *  - Weight matrices are row-major [out, in] (y = W x). Storage type is the
+ *    config's dtype (float32 or bfloat16) for weights, features and K/V caches;
+ *    activations are float32 inside the library and all float outputs are float32.
+ *  - "device" pointers are CUDA device (or managed) memory on the handle's device;
+ *    "host" pointers are ordinary host memory. Memory passed to a call stays owned
+ *    by the caller.
+ *  - Calls that take a stream enqueue work on it and return before it runs.
+ *    Argument errors are detected on the host and returned synchronously, with
+ *    nothing enqueued. Errors found while the kernels run (an out-of-range token,
+ *    a prefix longer than the cache, a bad page id, a timed-out device wait) are
+ *    recorded in a device status word and reported by fe_last_device_status();
+ *    the offending work item is skipped, and no kernel traps.
+ *  - No global state: several handles may coexist. One handle must not be used
+ *    from two streams concurrently (its scratch buffers are shared by its calls).
+ *  - No exceptions cross the ABI.
+ */
+#ifndef FE_DRAFT_H
+#define FE_DRAFT_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FE_API __attribute__((visibility("default")))
+#else
+#define FE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FE_OK = 0,
+    FE_ERR_INVALID_ARG = -1, /* a null pointer, a bad shape or an out-of-range scalar */
+    FE_ERR_UNSUPPORTED = -2, /* a legal shape this build does not implement */
+    FE_ERR_CUDA = -3,        /* a CUDA runtime call failed */
+    FE_ERR_OOM = -4,         /* device allocation failed */
+    FE_ERR_CAPACITY = -5,    /* a prefix does not fit its cache (P_b + 1 > max_seq) */
+    FE_ERR_TIMEOUT = -6,     /* a bounded device-side wait ran out */
+    FE_ERR_DEVICE = -7       /* a device-side range check failed (token, page id) */
+} fe_status;
+
+typedef enum { FE_F32 = 0, FE_BF16 = 1 } fe_dtype;
+
+/* Shape of one drafter. Sec. 2.1 fixes the structure (N layers, shared frozen LM
+ * head); the layer internals follow the LLaMA-style block EAGLE-3 uses. */
+typedef struct {
+    int32_t d;          /* hidden size of the drafter and the target */
+    int32_t n_heads;    /* query heads H */
+    int32_t n_kv_heads; /* key/value heads Hkv (H % Hkv == 0; Hkv == H is plain MHA) */
+    int32_t head_dim;   /* hd: 64 or 128 */
+    int32_t ffn;        /* SwiGLU intermediate size F */
+    int32_t vocab;      /* V, rows of the embedding table and of the LM head */
+    int32_t n_layers;   /* N, cascade depth (Eq. 2), 1..16 */
+    int32_t top_k_max;  /* largest top_k any call will ask for, 1..32 */
+    int32_t max_batch;  /* largest B any call will pass */
+    int32_t max_seq;    /* cache rows per sequence: a call needs prefix_len[b] + 1 <= max_seq */
+    int32_t page_size;  /* 0: contiguous caches; > 0: rows per page of paged caches */
+    float rope_theta;   /* RoPE base */
+    float rms_eps;      /* RMSNorm epsilon */
+    fe_dtype dtype;     /* storage type of weights, features and caches */
+} fe_config;
+
+/* One cascade layer L_i (Eq. 2): RMSNorm gains [d]; w_qkv [(H + 2 Hkv) hd, d] with the
+ * q rows first, then k, then v; w_o [d, H hd]; w_gate, w_up [F, d]; w_down [d, F]. */
+typedef struct {
+    const void *attn_norm, *w_qkv, *w_o, *mlp_norm, *w_gate, *w_up, *w_down;
+} fe_layer_weights;
+
+/* w_fuse [d, 3d] fuses concat(l, m, h) into g (Sec. 2.1); w_in [d, 2d] maps concat(g, e)
+ * to the cascade input (Eq. 1); embed [V, d]; lm_head [V, d] and final_norm [d] are the
+ * target's frozen LM head and its final RMSNorm; layers points to n_layers entries. */
+typedef struct {
+    const void *w_fuse, *w_in, *embed, *lm_head, *final_norm;
+    const fe_layer_weights *layers;
+} fe_weights;
+
+/* Arguments of one draft (Sec. 2.4, "Non-Autoregressive Drafting").
+ *
+ *  feat       device [B, 3d] dtype   concat(l, m, h) of each sequence's last verified position
+ *  next_tok   device [B] int32       the token t+1 whose embedding joins the fused feature
+ *  prefix_len device [B] int32       P_b, rows already in each layer's cache; the drafted row
+ *                                    takes sequence position P_b and cache slot P_b
+ *  k_cache,   host arrays of n_layers device pointers, layer i's K and V cache:
+ *  v_cache      page_size == 0: [max_batch, Hkv, max_seq, hd] dtype, row p of sequence b
+ *                 and KV head g at ((b * Hkv + g) * max_seq + p) * hd
+ *               page_size  > 0: a page pool [n_pages, Hkv, page_size, hd] dtype; row p of
+ *                 sequence b lives in page page_table[b * max_pages + p / page_size],
+ *                 slot p % page_size, with max_pages = ceil(max_seq / page_size)
+ *               Cached keys are stored after RoPE. The call writes each layer's new key
+ *               (rotated) and value into slot P_b and reads rows 0..P_b-1; it does not
+ *               advance prefix_len (committing accepted rows is the caller's step).
+ *  page_table device [B, max_pages] int32 (paged only; entries past the last used page
+ *             are ignored), n_pages the pool size (paged only)
+ *  top_k      candidates per depth, 1..top_k_max
+ *  temperature  T > 0 scales the reported probabilities and lse as softmax(logit / T);
+ *             T <= 0 (greedy) reports the T = 1 distribution. Candidates are always the
+ *             k largest logits, ties broken by the smaller token id.
+ * Outputs (device, float32 unless stated):
+ *  topk_id [B, N, top_k] int32, topk_logit [B, N, top_k], topk_prob [B, N, top_k], lse [B, N]
+ *  dbg_logits [B, N, V] or NULL: full logits, for parity checks only (costs V floats a row)
+ *  dbg_hidden [N, B, d] or NULL: the cascade's hidden states h_i
+ */
+typedef struct {
+    int32_t B, top_k;
+    float temperature;
+    const void *feat;
+    const int32_t *next_tok;
+    const int32_t *prefix_len;
+    void *const *k_cache;
+    void *const *v_cache;
+    const int32_t *page_table;
+    int32_t n_pages;
+    int32_t *topk_id;
+    float *topk_logit, *topk_prob, *lse;
+    float *dbg_logits, *dbg_hidden;
+} fe_forward_args;
+
+/* The draft tree of B sequences, device buffers with T = 1 + N * top_k nodes each:
+ * tok [B, T] int32, parent [B, T] int32 (-1 for the root), depth [B, T] int32,
+ * mask [B, T, T] uint8 (mask[b][a][c] = 1 iff node c is node a or one of its ancestors). */
+typedef struct {
+    int32_t *tok, *parent, *depth;
+    uint8_t *mask;
+} fe_tree;
+
+typedef struct fe_handle fe_handle;
+
+/* Create a drafter on the current CUDA device. Copies (and repacks) every weight into
+ * memory the handle owns, so the caller may free its weights once the call returns.
+ * Weight pointers may be host or device memory (any memory cudaMemcpyDefault reads).
+ * Precomputes the RoPE table in double precision. `stream` orders the copies; the
+ * call synchronises it before returning. Errors: FE_ERR_INVALID_ARG (null pointer,
+ * inconsistent shape), FE_ERR_UNSUPPORTED, FE_ERR_OOM, FE_ERR_CUDA. *out is set only
+ * on FE_OK. */
+FE_API fe_status fe_draft_init(const fe_config *cfg, const fe_weights *w, void *stream, fe_handle **out);
+
+/* One single-pass draft (Eq. 1, Eq. 2, Sec. 2.1): the cascade, the LM head for all
+ * N hidden states at once, softmax statistics and top-k per depth. No full-vocab
+ * logits reach memory unless dbg_logits is given. */
+FE_API fe_status fe_draft_forward(fe_handle *h, const fe_forward_args *args, void *stream);
+
+/* Backbone Expansion (Sec. 2.2) from fe_draft_forward's topk_id [B, N, top_k]: node 0 is
+ * the root (next_tok[b]); level i = 1..N holds that depth's candidates in rank order at
+ * nodes 1 + (i-1) top_k + r; level 1 hangs under the root and level i >= 2 under the
+ * previous level's rank-0 node, the backbone. A token id outside [0, V) sets
+ * FE_ERR_DEVICE in the status word. */
+FE_API fe_status fe_build_tree(fe_handle *h, int32_t B, int32_t top_k, const int32_t *next_tok,
+                        const int32_t *topk_id, fe_tree *out, void *stream);
+
+/* Synchronise `stream`, return and clear the handle's device status word
+ * (FE_OK, FE_ERR_CAPACITY, FE_ERR_DEVICE or FE_ERR_TIMEOUT). */
+FE_API fe_status fe_last_device_status(fe_handle *h, void *stream);
+
+/* Release everything the handle owns (synchronises the device first). NULL is a no-op. */
+FE_API void fe_free(fe_handle *h);
+
+/* A static, human-readable name of a status code. */
+FE_API const char *fe_status_str(fe_status s);
+
+/* Number of kernels fe_draft_forward (plus fe_build_tree when with_tree != 0) launches for
+ * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
+FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);
+
+/* Failure-detection self-test: launches one CTA whose bounded wait on a barrier that
+ * nothing completes gives up after `timeout_ns` nanoseconds (1e3..1e9) and records
+ * FE_ERR_TIMEOUT in the handle's status word. The GPU stays usable. */
+FE_API fe_status fe_selftest_timeout(fe_handle *h, int64_t timeout_ns, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FE_DRAFT_H */

@@ -1,0 +1,209 @@
+"""GB300 (sm_103a) FastEagle cascaded drafter: Python binding of libfe_draft.so.
+
+The functions here carry the C ABI's names (include/fe_draft.h) and only marshal
+arguments: torch tensors become device pointers, dicts become the ABI's structs, and
+PyTorch provides device memory and the current CUDA stream. Every step of a draft runs
+in the library's CUDA kernels; there is no CPU or PyTorch fallback. If the compiled
+library is missing, importing this package raises (build it with
+``python -c "import __graft_entry__ as g; g.build()"``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfe_draft.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: the CUDA extension has not been built "
+                      "(run __graft_entry__.build())")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+FE_OK, FE_ERR_INVALID_ARG, FE_ERR_UNSUPPORTED, FE_ERR_CUDA = 0, -1, -2, -3
+FE_ERR_OOM, FE_ERR_CAPACITY, FE_ERR_TIMEOUT, FE_ERR_DEVICE = -4, -5, -6, -7
+FE_F32, FE_BF16 = 0, 1
+
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+
+
+class fe_config(ctypes.Structure):
+    _fields_ = [("d", _i32), ("n_heads", _i32), ("n_kv_heads", _i32), ("head_dim", _i32),
+                ("ffn", _i32), ("vocab", _i32), ("n_layers", _i32), ("top_k_max", _i32),
+                ("max_batch", _i32), ("max_seq", _i32), ("page_size", _i32),
+                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int)]
+
+
+class fe_layer_weights(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate", "w_up", "w_down")]
+
+
+class fe_weights(ctypes.Structure):
+    _fields_ = [("w_fuse", _vp), ("w_in", _vp), ("embed", _vp), ("lm_head", _vp), ("final_norm", _vp),
+                ("layers", ctypes.POINTER(fe_layer_weights))]
+
+
+class fe_forward_args(ctypes.Structure):
+    _fields_ = [("B", _i32), ("top_k", _i32), ("temperature", ctypes.c_float),
+                ("feat", _vp), ("next_tok", _vp), ("prefix_len", _vp),
+                ("k_cache", ctypes.POINTER(_vp)), ("v_cache", ctypes.POINTER(_vp)),
+                ("page_table", _vp), ("n_pages", _i32),
+                ("topk_id", _vp), ("topk_logit", _vp), ("topk_prob", _vp), ("lse", _vp),
+                ("dbg_logits", _vp), ("dbg_hidden", _vp)]
+
+
+class fe_tree(ctypes.Structure):
+    _fields_ = [("tok", _vp), ("parent", _vp), ("depth", _vp), ("mask", _vp)]
+
+
+_lib.fe_draft_init.argtypes = [ctypes.POINTER(fe_config), ctypes.POINTER(fe_weights), _vp, ctypes.POINTER(_vp)]
+_lib.fe_draft_init.restype = ctypes.c_int
+_lib.fe_draft_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp]
+_lib.fe_draft_forward.restype = ctypes.c_int
+_lib.fe_build_tree.argtypes = [_vp, _i32, _i32, _vp, _vp, ctypes.POINTER(fe_tree), _vp]
+_lib.fe_build_tree.restype = ctypes.c_int
+_lib.fe_last_device_status.argtypes = [_vp, _vp]
+_lib.fe_last_device_status.restype = ctypes.c_int
+_lib.fe_free.argtypes = [_vp]
+_lib.fe_free.restype = None
+_lib.fe_status_str.argtypes = [ctypes.c_int]
+_lib.fe_status_str.restype = ctypes.c_char_p
+_lib.fe_launch_count.argtypes = [_vp, _i32, _i32]
+_lib.fe_launch_count.restype = _i32
+_lib.fe_selftest_timeout.argtypes = [_vp, ctypes.c_int64, _vp]
+_lib.fe_selftest_timeout.restype = ctypes.c_int
+
+
+class FeError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {fe_status_str(code)} ({code})")
+        self.code = code
+
+
+def fe_status_str(code: int) -> str:
+    return _lib.fe_status_str(code).decode()
+
+
+def _check(code: int, where: str) -> None:
+    if code != FE_OK:
+        raise FeError(code, where)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _p(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    assert t.is_contiguous(), "buffers passed to the drafter must be contiguous"
+    return t.data_ptr()
+
+
+def make_config(cfg: dict) -> fe_config:
+    return fe_config(cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"], cfg["ffn"], cfg["vocab"],
+                     cfg["n_layers"], cfg["top_k_max"], cfg.get("max_batch", cfg.get("B", 1)), cfg["max_seq"],
+                     cfg.get("page_size", 0), float(cfg["rope_theta"]), float(cfg["rms_eps"]),
+                     FE_F32 if cfg["dtype"] == "f32" else FE_BF16)
+
+
+class Handle:
+    """An initialised drafter (owns a fe_handle*)."""
+
+    def __init__(self, ptr: int, cfg: dict):
+        self.ptr = ptr
+        self.cfg = dict(cfg)
+
+    def __del__(self):
+        self.close()
+
+    def close(self):
+        if getattr(self, "ptr", None):
+            _lib.fe_free(self.ptr)
+            self.ptr = None
+
+
+def fe_draft_init(cfg: dict, weights: dict, stream=None) -> Handle:
+    """weights: dict of tensors (host or device) in the canonical layout:
+    w_fuse, w_in, embed, lm_head, final_norm, and layers: list of dicts with attn_norm,
+    w_qkv, w_o, mlp_norm, w_gate, w_up, w_down."""
+    L = weights["layers"]
+    arr = (fe_layer_weights * len(L))()
+    for i, l in enumerate(L):
+        arr[i] = fe_layer_weights(_p(l["attn_norm"]), _p(l["w_qkv"]), _p(l["w_o"]), _p(l["mlp_norm"]),
+                                  _p(l["w_gate"]), _p(l["w_up"]), _p(l["w_down"]))
+    w = fe_weights(_p(weights["w_fuse"]), _p(weights["w_in"]), _p(weights["embed"]), _p(weights["lm_head"]),
+                   _p(weights["final_norm"]), arr)
+    c = make_config(cfg)
+    out = _vp()
+    _check(_lib.fe_draft_init(ctypes.byref(c), ctypes.byref(w), _stream(stream), ctypes.byref(out)),
+           "fe_draft_init")
+    return Handle(out.value, cfg)
+
+
+def alloc_outputs(h: Handle, B: int, top_k: int, device="cuda") -> dict:
+    N = h.cfg["n_layers"]
+    return dict(topk_id=torch.empty((B, N, top_k), dtype=torch.int32, device=device),
+                topk_logit=torch.empty((B, N, top_k), dtype=torch.float32, device=device),
+                topk_prob=torch.empty((B, N, top_k), dtype=torch.float32, device=device),
+                lse=torch.empty((B, N), dtype=torch.float32, device=device))
+
+
+def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
+                     temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
+                     dbg_logits=None, dbg_hidden=None, stream=None) -> dict:
+    """One draft. feat [B, 3d], next_tok [B] i32, prefix_len [B] i32 (device tensors);
+    k_cache / v_cache: lists of per-layer device tensors (see include/fe_draft.h)."""
+    B = int(next_tok.shape[0])
+    if out is None:
+        out = alloc_outputs(h, B, top_k, feat.device)
+    N = h.cfg["n_layers"]
+    kc = (_vp * N)(*[_p(t) for t in k_cache])
+    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
+                        _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
+                        _p(out["topk_prob"]), _p(out["lse"]), _p(dbg_logits), _p(dbg_hidden))
+    _check(_lib.fe_draft_forward(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_forward")
+    return out
+
+
+def alloc_tree(h: Handle, B: int, top_k: int, device="cuda") -> dict:
+    T = 1 + h.cfg["n_layers"] * top_k
+    return dict(tok=torch.empty((B, T), dtype=torch.int32, device=device),
+                parent=torch.empty((B, T), dtype=torch.int32, device=device),
+                depth=torch.empty((B, T), dtype=torch.int32, device=device),
+                mask=torch.empty((B, T, T), dtype=torch.uint8, device=device))
+
+
+def fe_build_tree(h: Handle, next_tok, topk_id, top_k: int, out: dict | None = None, stream=None) -> dict:
+    B = int(next_tok.shape[0])
+    if out is None:
+        out = alloc_tree(h, B, top_k, next_tok.device)
+    t = fe_tree(_p(out["tok"]), _p(out["parent"]), _p(out["depth"]), _p(out["mask"]))
+    _check(_lib.fe_build_tree(h.ptr, B, top_k, _p(next_tok), _p(topk_id), ctypes.byref(t), _stream(stream)),
+           "fe_build_tree")
+    return out
+
+
+def fe_last_device_status(h: Handle, stream=None) -> int:
+    return int(_lib.fe_last_device_status(h.ptr, _stream(stream)))
+
+
+def fe_free(h: Handle) -> None:
+    h.close()
+
+
+def fe_launch_count(h: Handle, B: int, with_tree: bool = True) -> int:
+    return int(_lib.fe_launch_count(h.ptr, B, 1 if with_tree else 0))
+
+
+def fe_selftest_timeout(h: Handle, timeout_ns: int, stream=None) -> int:
+    return int(_lib.fe_selftest_timeout(h.ptr, int(timeout_ns), _stream(stream)))

@@ -1,0 +1,126 @@
+// Internal launch interface of the drafter's kernels (host side). Not part of the ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fe_draft.h"
+
+namespace fe {
+
+// status-word bits (combined with atomicOr; the host maps them back to fe_status)
+enum : int {
+    ST_CAPACITY = 1,  // prefix_len[b] + 1 > max_seq or negative
+    ST_DEVICE = 2,    // a token id or page id out of range
+    ST_TIMEOUT = 4,   // a bounded wait ran out
+};
+
+// how a weight-streaming phase stages its activations X[b][k]
+enum Prologue : int {
+    PRO_F32 = 0,         // x is float32 [B, ldx]
+    PRO_STORAGE = 1,     // x is in the storage type [B, ldx]
+    PRO_RMSNORM = 2,     // x float32; X = gamma * x / sqrt(mean(x^2) + eps)
+    PRO_CONCAT_EMB = 3,  // X = concat(x[b][0:d_split] (float32), embed[tok[b]] (storage))
+};
+
+// ---- weight-streaming linear phase: Y = epilogue(W . prologue(X)) ---------------------
+enum Epilogue : int {
+    EPI_STORE = 0,   // y[b, m] = acc
+    EPI_RESID = 1,   // y[b, m] += acc; y2[b, m] = the new y (if y2)
+    EPI_SWIGLU = 2,  // rows (2j, 2j+1) are (gate_j, up_j): y[b, j] = silu(gate) * up
+};
+
+struct LinearArgs {
+    const void* W;  // [M, K] storage type, 16-byte aligned, K % 8 == 0
+    int M, K;
+    int B;  // activation rows
+    // prologue
+    int pro;
+    const void* x;
+    int ldx;
+    const void* gamma;
+    float eps;
+    const void* embed;
+    const int* tok;
+    int d_split;
+    int vocab;
+    // epilogue
+    int epi;
+    float* y;
+    int ldy;
+    float* y2;
+    int ldy2;
+    int* status;
+};
+
+struct DeviceInfo {
+    int num_sms;
+    int max_smem_optin;
+};
+
+cudaError_t linear_prepare(const DeviceInfo& dev);
+cudaError_t launch_linear(fe_dtype dt, const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st);
+// number of kernels launch_linear() issues for these shapes (always 1)
+inline int linear_launches() { return 1; }
+
+// ---- LM head + fused softmax statistics + per-slab top-k ------------------------------
+struct LmHeadArgs {
+    const void* W;  // lm_head [V, d]
+    const void* gamma;  // final_norm [d]
+    int V, d;
+    int R;  // rows of hidden states (N * B), row r = i * B + b
+    int B, N;
+    const float* hid;  // [R, d] float32
+    float eps;
+    float inv_temp;
+    int top_k;
+    int n_slabs;  // filled by lmhead_plan()
+    int* part_id;      // [R, n_slabs, top_k]
+    float* part_val;   // [R, n_slabs, top_k]
+    float* part_ms;    // [R, n_slabs, 2] (max, sum of exp) of logit * inv_temp
+    float* dbg_logits; // [B, N, V] or null
+    int* status;
+};
+cudaError_t lmhead_prepare(const DeviceInfo& dev);
+int lmhead_slabs(int V, const DeviceInfo& dev);
+int lmhead_launches(int R, int d, const DeviceInfo& dev);
+cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st);
+
+struct MergeArgs {
+    int R, B, N, n_slabs, top_k;
+    float inv_temp;
+    const int* part_id;
+    const float* part_val;
+    const float* part_ms;
+    int* topk_id;       // [B, N, k]
+    float* topk_logit;  // [B, N, k]
+    float* topk_prob;   // [B, N, k]
+    float* lse;         // [B, N]
+};
+cudaError_t launch_topk_merge(const MergeArgs& a, cudaStream_t st);
+
+// ---- decode attention ----------------------------------------------------------------
+struct AttnArgs {
+    const float* qkv;  // [B, (H + 2 Hkv) hd] float32, before RoPE
+    void* kc;          // layer cache (storage type)
+    void* vc;
+    const int* prefix_len;  // [B]
+    const int* page_table;  // [B, max_pages] or null
+    int max_pages, n_pages, page_size, max_seq;
+    const float* rope_cs;   // [max_seq, hd/2, 2] (cos, sin)
+    int B, H, Hkv, hd;
+    int split, n_split;     // keys per work item, work items per (sequence, KV head)
+    float* part;            // [B, H, n_split, hd + 2]
+    float* out;             // [B, H * hd]
+    int* status;
+};
+int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
+cudaError_t launch_attention(fe_dtype dt, const AttnArgs& a, cudaStream_t st);   // 2 kernels
+inline int attention_launches() { return 2; }
+
+// ---- draft tree + failure-detection probe ------------------------------------------------
+cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,
+                        int* depth, uint8_t* mask, int* status, cudaStream_t st);
+cudaError_t launch_timeout_probe(int64_t timeout_ns, int* status, cudaStream_t st);
+
+}  // namespace fe

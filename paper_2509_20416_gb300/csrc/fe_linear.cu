@@ -1,0 +1,138 @@
+// Linear phases of the cascade (Eq. 1 FCs; QKV, O-proj, gate/up and down projections
+// of each layer L_i, Eq. 2) as weight-streaming CTAs (fe_stream.cuh) with a fused
+// prologue (RMSNorm / concat with the token embedding) and epilogue (store, residual
+// add, SwiGLU).
+#include "fe_kernels.h"
+#include "fe_stream.cuh"
+
+namespace fe {
+
+struct LinearEpi {
+    const LinearArgs* a;
+    int b0, nb;
+    template <int BT>
+    __device__ __forceinline__ void run(int g, const float* red) const {
+        const int t = threadIdx.x;
+        if (a->epi == EPI_SWIGLU) {
+            if (t < 2 * BT) {
+                const int pr = t / BT, b = t % BT;
+                const int m = g * kGroupRows + 2 * pr;
+                if (b < nb && m + 1 < a->M) {
+                    const float gate = group_sum<BT>(red, 2 * pr, b);
+                    const float up = group_sum<BT>(red, 2 * pr + 1, b);
+                    a->y[(size_t)(b0 + b) * a->ldy + (m >> 1)] = silu(gate) * up;
+                }
+            }
+        } else if (t < kGroupRows * BT) {
+            const int r = t / BT, b = t % BT;
+            const int m = g * kGroupRows + r;
+            if (b < nb && m < a->M) {
+                const float v = group_sum<BT>(red, r, b);
+                float* yp = a->y + (size_t)(b0 + b) * a->ldy + m;
+                if (a->epi == EPI_RESID) {
+                    const float nv = *yp + v;
+                    *yp = nv;
+                    if (a->y2) a->y2[(size_t)(b0 + b) * a->ldy2 + m] = nv;
+                } else {
+                    *yp = v;
+                }
+            }
+        }
+    }
+};
+
+template <int BT>
+struct EpiAdapter {
+    const LinearEpi& e;
+    __device__ __forceinline__ void operator()(int g, const float* red) const { e.template run<BT>(g, red); }
+};
+
+template <typename WT, int BT>
+__global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int ns) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int Kpad = (a.K + 3) & ~3;
+    const int b0 = blockIdx.y * BT;
+    const int nb = min(BT, a.B - b0);
+    StreamSmem s = carve_stream_smem(smem, ns, min(BT, a.B), Kpad, BT);
+    stream_init_barriers(s, ns);
+
+    const int GM = (a.M + kGroupRows - 1) / kGroupRows;
+    const int g0 = (int)(((int64_t)blockIdx.x * GM) / gridDim.x);
+    const int g1 = (int)(((int64_t)(blockIdx.x + 1) * GM) / gridDim.x);
+
+    if (threadIdx.x >= kConsumers) {
+        if (threadIdx.x == kConsumers)
+            stream_produce<WT>((const unsigned char*)a.W, a.M, a.K, g0, g1, s, ns, a.status);
+        return;
+    }
+    ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
+    stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red);
+    named_sync(1, kConsumers);
+    LinearEpi e{&a, b0, nb};
+    EpiAdapter<BT> ep{e};
+    stream_consume<WT, BT>(a.K, g0, g1, s, ns, Kpad, nb, a.status, ep);
+}
+
+// ---- host side ----------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kXBudget = 128 * 1024;  // activations held in shared memory per CTA
+
+template <typename WT, int BT>
+cudaError_t set_attr(const DeviceInfo& dev) {
+    return cudaFuncSetAttribute(linear_kernel<WT, BT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                dev.max_smem_optin);
+}
+
+int pick_bt(int B, int K) {
+    const size_t row = (size_t)((K + 3) & ~3) * sizeof(float);
+    int bt = 8;
+    while (bt > 1 && ((size_t)(bt < B ? bt : B) * row > kXBudget || bt / 2 >= B)) bt >>= 1;
+    return bt;
+}
+
+template <typename WT, int BT>
+cudaError_t launch_bt(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {
+    const int Kpad = (a.K + 3) & ~3;
+    const int xrows = BT < a.B ? BT : a.B;
+    const size_t fixed = stream_smem_bytes(0, xrows, Kpad, BT);
+    int ns = (int)(((size_t)dev.max_smem_optin - fixed) / (kStageBytes + 16));
+    ns = ns > kMaxStages ? kMaxStages : ns;
+    if (ns < 2) return cudaErrorInvalidValue;
+    const size_t smem = stream_smem_bytes(ns, xrows, Kpad, BT);
+    const int GM = (a.M + kGroupRows - 1) / kGroupRows;
+    dim3 grid(GM < dev.num_sms ? GM : dev.num_sms, (a.B + BT - 1) / BT);
+    linear_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, ns);
+    return cudaGetLastError();
+}
+
+template <typename WT>
+cudaError_t launch_t(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {
+    switch (pick_bt(a.B, a.K)) {
+        case 1: return launch_bt<WT, 1>(a, dev, st);
+        case 2: return launch_bt<WT, 2>(a, dev, st);
+        case 4: return launch_bt<WT, 4>(a, dev, st);
+        default: return launch_bt<WT, 8>(a, dev, st);
+    }
+}
+
+}  // namespace
+
+cudaError_t linear_prepare(const DeviceInfo& dev) {
+    cudaError_t e;
+    if ((e = set_attr<float, 1>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<float, 2>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<float, 4>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<float, 8>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<bf16_t, 1>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<bf16_t, 2>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<bf16_t, 4>(dev)) != cudaSuccess) return e;
+    return set_attr<bf16_t, 8>(dev);
+}
+
+cudaError_t launch_linear(fe_dtype dt, const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {
+    if (a.M <= 0 || a.B <= 0) return cudaSuccess;
+    return dt == FE_F32 ? launch_t<float>(a, dev, st) : launch_t<bf16_t>(a, dev, st);
+}
+
+}  // namespace fe

@@ -1,0 +1,448 @@
+// C ABI of the drafter (include/fe_draft.h): handle, weight packing, RoPE table, scratch
+// buffers, the launch sequence of one draft, and its CUDA-graph replay.
+//
+// One draft (Eq. 1, Eq. 2, Sec. 2.1) is this stream-ordered sequence:
+//   g  = W_fuse concat(l, m, h)                 linear, prologue: storage -> float
+//   x  = W_in concat(g, Embed[next_tok])        linear, prologue: concat with the embedding
+//   for each layer L_i:
+//     qkv = W_qkv RMSNorm(x; gamma_1)            linear, prologue: RMSNorm
+//     o   = attention(RoPE(q), cache_i + own row) split-KV attention + combine (writes slot P_b)
+//     x  += W_o o                                linear, epilogue: residual add
+//     a   = silu(W_gate u) * (W_up u), u = RMSNorm(x; gamma_2)   linear over the interleaved
+//                                                [gate; up] rows, epilogue: SwiGLU
+//     x  += W_down a;  h_i = x                   linear, epilogue: residual add + copy to h_i
+//   logits of all N*B rows h_i through RMSNorm(gamma_out) and the LM head, fused with the
+//   softmax statistics and a per-slab top-k; then a merge per row.
+// The sequence is captured once per distinct argument set into a CUDA graph on an
+// internal stream and replayed on the caller's stream.
+#include <math.h>
+#include <string.h>
+
+#include <cstdlib>
+#include <new>
+#include <vector>
+
+#include "fe_kernels.h"
+
+using namespace fe;
+
+namespace {
+
+struct LayerPacked {
+    const void *attn_norm, *w_qkv, *w_o, *mlp_norm, *w_gu, *w_down;
+};
+
+struct GraphKey {
+    fe_forward_args args;
+    std::vector<void*> kc, vc;
+    bool operator==(const GraphKey& o) const {
+        const fe_forward_args &x = args, &y = o.args;
+        return x.B == y.B && x.top_k == y.top_k && x.temperature == y.temperature && x.feat == y.feat &&
+               x.next_tok == y.next_tok && x.prefix_len == y.prefix_len && x.page_table == y.page_table &&
+               x.n_pages == y.n_pages && x.topk_id == y.topk_id && x.topk_logit == y.topk_logit &&
+               x.topk_prob == y.topk_prob && x.lse == y.lse && x.dbg_logits == y.dbg_logits &&
+               x.dbg_hidden == y.dbg_hidden && kc == o.kc && vc == o.vc;
+    }
+};
+
+}  // namespace
+
+struct fe_handle {
+    fe_config cfg;
+    int device = 0;
+    DeviceInfo dev{};
+    size_t es = 2;
+    void* wbuf = nullptr;
+    const void *w_fuse = nullptr, *w_in = nullptr, *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
+    std::vector<LayerPacked> layers;
+    float* rope_cs = nullptr;
+    void* sbuf = nullptr;
+    float *g = nullptr, *x = nullptr, *qkv = nullptr, *o = nullptr, *act = nullptr, *hid = nullptr;
+    float* attn_part = nullptr;
+    int* lm_part_id = nullptr;
+    float *lm_part_val = nullptr, *lm_part_ms = nullptr;
+    int* status = nullptr;
+    int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
+    cudaStream_t cap = nullptr;
+    cudaGraphExec_t gexec = nullptr;
+    GraphKey gkey;
+    bool use_graph = true;
+};
+
+namespace {
+
+inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+fe_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return FE_OK;
+    if (e == cudaErrorMemoryAllocation) return FE_ERR_OOM;
+    return FE_ERR_CUDA;
+}
+
+#define FE_TRY(call)                                  \
+    do {                                              \
+        cudaError_t _e = (call);                      \
+        if (_e != cudaSuccess) return from_cuda(_e);  \
+    } while (0)
+
+bool valid_config(const fe_config* c) {
+    if (!c) return false;
+    if (c->d <= 0 || c->n_heads <= 0 || c->n_kv_heads <= 0 || c->ffn <= 0 || c->vocab <= 0) return false;
+    if (c->n_heads % c->n_kv_heads) return false;
+    if (c->n_layers < 1 || c->n_layers > 16) return false;
+    if (c->top_k_max < 1 || c->top_k_max > 32 || c->top_k_max > c->vocab) return false;
+    if (c->max_batch < 1 || c->max_seq < 1 || c->page_size < 0) return false;
+    if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f)) return false;
+    if (c->dtype != FE_F32 && c->dtype != FE_BF16) return false;
+    if (c->head_dim <= 0 || c->head_dim % 2) return false;
+    return true;
+}
+
+// legal shapes this build's kernels cover
+bool supported_config(const fe_config* c) {
+    const int G = c->n_heads / c->n_kv_heads;
+    if (c->head_dim != 64 && c->head_dim != 128) return false;
+    if (G != 1 && G != 2 && G != 4 && G != 8) return false;
+    // every matrix row must be a whole number of 16-byte vectors
+    if (c->d % 8 || c->ffn % 8 || (c->n_heads * c->head_dim) % 8) return false;
+    return true;
+}
+
+struct Sizes {
+    size_t w_fuse, w_in, embed, lm_head, norm, qkv, wo, gu, down;
+};
+
+Sizes weight_sizes(const fe_config& c, size_t es) {
+    const size_t d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    Sizes s;
+    s.w_fuse = d * 3 * d * es;
+    s.w_in = d * 2 * d * es;
+    s.embed = V * d * es;
+    s.lm_head = V * d * es;
+    s.norm = d * es;
+    s.qkv = (H + 2 * Hkv) * hd * d * es;
+    s.wo = d * H * hd * es;
+    s.gu = 2 * F * d * es;
+    s.down = d * F * es;
+    return s;
+}
+
+fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t st) {
+    const fe_config& c = h->cfg;
+    const int B = a->B, d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    const int N = c.n_layers, nqkv = (H + 2 * Hkv) * hd;
+    const fe_dtype dt = c.dtype;
+
+    LinearArgs la{};
+    la.status = h->status;
+    la.eps = c.rms_eps;
+    la.B = B;
+    // g = W_fuse concat(l, m, h)
+    la.W = h->w_fuse; la.M = d; la.K = 3 * d;
+    la.pro = PRO_STORAGE; la.x = a->feat; la.ldx = 3 * d;
+    la.epi = EPI_STORE; la.y = h->g; la.ldy = d; la.y2 = nullptr;
+    FE_TRY(launch_linear(dt, la, h->dev, st));
+    // x0 = W_in concat(g, e)
+    la.W = h->w_in; la.M = d; la.K = 2 * d;
+    la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
+    la.d_split = d; la.vocab = V;
+    la.epi = EPI_STORE; la.y = h->x; la.ldy = d;
+    FE_TRY(launch_linear(dt, la, h->dev, st));
+
+    AttnArgs aa{};
+    aa.qkv = h->qkv; aa.prefix_len = a->prefix_len; aa.page_table = a->page_table;
+    aa.page_size = c.page_size; aa.max_seq = c.max_seq; aa.n_pages = a->n_pages;
+    aa.max_pages = c.page_size > 0 ? (c.max_seq + c.page_size - 1) / c.page_size : 0;
+    aa.rope_cs = h->rope_cs; aa.B = B; aa.H = H; aa.Hkv = Hkv; aa.hd = hd;
+    aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
+    aa.part = h->attn_part; aa.out = h->o; aa.status = h->status;
+
+    for (int i = 0; i < N; ++i) {
+        const LayerPacked& L = h->layers[i];
+        // qkv = W_qkv RMSNorm(x)
+        la.W = L.w_qkv; la.M = nqkv; la.K = d;
+        la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.attn_norm;
+        la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
+        FE_TRY(launch_linear(dt, la, h->dev, st));
+        // attention over the layer's cache (+ own row), appends slot P_b
+        aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
+        FE_TRY(launch_attention(dt, aa, st));
+        // x += W_o o
+        la.W = L.w_o; la.M = d; la.K = H * hd;
+        la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
+        la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr;
+        FE_TRY(launch_linear(dt, la, h->dev, st));
+        // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
+        la.W = L.w_gu; la.M = 2 * F; la.K = d;
+        la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm;
+        la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
+        FE_TRY(launch_linear(dt, la, h->dev, st));
+        // x += W_down a; h_i = x
+        la.W = L.w_down; la.M = d; la.K = F;
+        la.pro = PRO_F32; la.x = h->act; la.ldx = F;
+        la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = h->hid + (size_t)i * B * d; la.ldy2 = d;
+        FE_TRY(launch_linear(dt, la, h->dev, st));
+    }
+
+    const float inv_temp = a->temperature > 0.f ? 1.0f / a->temperature : 1.0f;
+    LmHeadArgs lm{};
+    lm.W = h->lm_head; lm.gamma = h->final_norm; lm.V = V; lm.d = d; lm.R = N * B; lm.B = B; lm.N = N;
+    lm.hid = h->hid; lm.eps = c.rms_eps; lm.inv_temp = inv_temp; lm.top_k = a->top_k; lm.n_slabs = h->lm_slabs;
+    lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
+    lm.dbg_logits = a->dbg_logits; lm.status = h->status;
+    FE_TRY(launch_lmhead(dt, lm, h->dev, st));
+    MergeArgs mg{};
+    mg.R = N * B; mg.B = B; mg.N = N; mg.n_slabs = h->lm_slabs; mg.top_k = a->top_k; mg.inv_temp = inv_temp;
+    mg.part_id = h->lm_part_id; mg.part_val = h->lm_part_val; mg.part_ms = h->lm_part_ms;
+    mg.topk_id = a->topk_id; mg.topk_logit = a->topk_logit; mg.topk_prob = a->topk_prob; mg.lse = a->lse;
+    FE_TRY(launch_topk_merge(mg, st));
+    if (a->dbg_hidden)
+        FE_TRY(cudaMemcpyAsync(a->dbg_hidden, h->hid, (size_t)N * B * d * sizeof(float), cudaMemcpyDeviceToDevice,
+                               st));
+    return FE_OK;
+}
+
+void release(fe_handle* h) {
+    if (!h) return;
+    if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    if (h->cap) cudaStreamDestroy(h->cap);
+    if (h->wbuf) cudaFree(h->wbuf);
+    if (h->sbuf) cudaFree(h->sbuf);
+    delete h;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* fe_status_str(fe_status s) {
+    switch (s) {
+        case FE_OK: return "ok";
+        case FE_ERR_INVALID_ARG: return "invalid argument";
+        case FE_ERR_UNSUPPORTED: return "unsupported shape";
+        case FE_ERR_CUDA: return "CUDA error";
+        case FE_ERR_OOM: return "out of device memory";
+        case FE_ERR_CAPACITY: return "prefix does not fit the cache";
+        case FE_ERR_TIMEOUT: return "device wait timed out";
+        case FE_ERR_DEVICE: return "device-side range check failed";
+    }
+    return "unknown status";
+}
+
+fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream, fe_handle** out) {
+    if (!out) return FE_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!valid_config(cfg) || !w) return FE_ERR_INVALID_ARG;
+    if (!w->w_fuse || !w->w_in || !w->embed || !w->lm_head || !w->final_norm || !w->layers) return FE_ERR_INVALID_ARG;
+    for (int i = 0; i < cfg->n_layers; ++i) {
+        const fe_layer_weights& L = w->layers[i];
+        if (!L.attn_norm || !L.w_qkv || !L.w_o || !L.mlp_norm || !L.w_gate || !L.w_up || !L.w_down)
+            return FE_ERR_INVALID_ARG;
+    }
+    if (!supported_config(cfg)) return FE_ERR_UNSUPPORTED;
+
+    fe_handle* h = new (std::nothrow) fe_handle();
+    if (!h) return FE_ERR_OOM;
+    h->cfg = *cfg;
+    const char* g = getenv("FE_DRAFT_GRAPH");
+    h->use_graph = !(g && g[0] == '0');
+    cudaStream_t st = (cudaStream_t)stream;
+    fe_status rc = FE_OK;
+    do {
+        const fe_config& c = h->cfg;
+        h->es = c.dtype == FE_F32 ? 4 : 2;
+        if ((rc = from_cuda(cudaGetDevice(&h->device))) != FE_OK) break;
+        if ((rc = from_cuda(cudaDeviceGetAttribute(&h->dev.num_sms, cudaDevAttrMultiProcessorCount, h->device))) != FE_OK)
+            break;
+        if ((rc = from_cuda(cudaDeviceGetAttribute(&h->dev.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin,
+                                                   h->device))) != FE_OK)
+            break;
+        if ((rc = from_cuda(linear_prepare(h->dev))) != FE_OK) break;
+        if ((rc = from_cuda(lmhead_prepare(h->dev))) != FE_OK) break;
+
+        // ---- packed weights: one allocation, every matrix 256-byte aligned ----
+        const Sizes sz = weight_sizes(c, h->es);
+        size_t total = align256(sz.w_fuse) + align256(sz.w_in) + align256(sz.embed) + align256(sz.lm_head) +
+                       align256(sz.norm);
+        total += (size_t)c.n_layers *
+                 (2 * align256(sz.norm) + align256(sz.qkv) + align256(sz.wo) + align256(sz.gu) + align256(sz.down));
+        if ((rc = from_cuda(cudaMalloc(&h->wbuf, total))) != FE_OK) break;
+        char* p = (char*)h->wbuf;
+        auto put = [&](const void* src, size_t bytes) -> const void* {
+            void* dst = p;
+            p += align256(bytes);
+            if (cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, st) != cudaSuccess) rc = FE_ERR_CUDA;
+            return dst;
+        };
+        h->w_fuse = put(w->w_fuse, sz.w_fuse);
+        h->w_in = put(w->w_in, sz.w_in);
+        h->embed = put(w->embed, sz.embed);
+        h->lm_head = put(w->lm_head, sz.lm_head);
+        h->final_norm = put(w->final_norm, sz.norm);
+        h->layers.resize(c.n_layers);
+        for (int i = 0; i < c.n_layers && rc == FE_OK; ++i) {
+            const fe_layer_weights& L = w->layers[i];
+            LayerPacked& P = h->layers[i];
+            P.attn_norm = put(L.attn_norm, sz.norm);
+            P.mlp_norm = put(L.mlp_norm, sz.norm);
+            P.w_qkv = put(L.w_qkv, sz.qkv);
+            P.w_o = put(L.w_o, sz.wo);
+            // [gate; up] interleaved by row: row 2j = gate_j, row 2j+1 = up_j
+            void* gu = p;
+            p += align256(sz.gu);
+            const size_t rowb = (size_t)c.d * h->es;
+            if (cudaMemcpy2DAsync(gu, 2 * rowb, L.w_gate, rowb, rowb, c.ffn, cudaMemcpyDefault, st) != cudaSuccess ||
+                cudaMemcpy2DAsync((char*)gu + rowb, 2 * rowb, L.w_up, rowb, rowb, c.ffn, cudaMemcpyDefault, st) !=
+                    cudaSuccess)
+                rc = FE_ERR_CUDA;
+            P.w_gu = gu;
+            P.w_down = put(L.w_down, sz.down);
+        }
+        if (rc != FE_OK) break;
+
+        // ---- RoPE table (cos, sin) per position and pair, computed in double ----
+        const int half = c.head_dim / 2;
+        std::vector<float> cs((size_t)c.max_seq * half * 2);
+        for (int pos = 0; pos < c.max_seq; ++pos)
+            for (int i = 0; i < half; ++i) {
+                const double ang = (double)pos * pow((double)c.rope_theta, -2.0 * i / (double)c.head_dim);
+                cs[((size_t)pos * half + i) * 2] = (float)cos(ang);
+                cs[((size_t)pos * half + i) * 2 + 1] = (float)sin(ang);
+            }
+
+        // ---- scratch ----
+        const size_t B = c.max_batch, d = c.d, F = c.ffn, H = c.n_heads, hd = c.head_dim;
+        const size_t nqkv = (size_t)(c.n_heads + 2 * c.n_kv_heads) * hd;
+        h->attn_split_rows = attn_split(c.max_batch, c.n_kv_heads, c.max_seq, h->dev);
+        h->attn_nsplit = (c.max_seq + h->attn_split_rows - 1) / h->attn_split_rows;
+        h->lm_slabs = lmhead_slabs(c.vocab, h->dev);
+        const size_t R = (size_t)c.n_layers * B;
+        const size_t k = c.top_k_max;
+        size_t off[12], n = 0, tot = 0;
+        const size_t bytes[12] = {
+            cs.size() * sizeof(float),                             // rope
+            B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
+            B * F * 4, R * d * 4,                                  // act, hid
+            B * H * h->attn_nsplit * (hd + 2) * 4,                 // attention partials
+            R * h->lm_slabs * k * 4, R * h->lm_slabs * k * 4,      // LM-head partial ids, values
+            R * h->lm_slabs * 2 * 4,                               // LM-head partial (max, sum)
+            256};                                                  // status
+        for (n = 0; n < 12; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+        if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
+        char* s = (char*)h->sbuf;
+        h->rope_cs = (float*)(s + off[0]);
+        h->g = (float*)(s + off[1]);
+        h->x = (float*)(s + off[2]);
+        h->qkv = (float*)(s + off[3]);
+        h->o = (float*)(s + off[4]);
+        h->act = (float*)(s + off[5]);
+        h->hid = (float*)(s + off[6]);
+        h->attn_part = (float*)(s + off[7]);
+        h->lm_part_id = (int*)(s + off[8]);
+        h->lm_part_val = (float*)(s + off[9]);
+        h->lm_part_ms = (float*)(s + off[10]);
+        h->status = (int*)(s + off[11]);
+        if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
+            break;
+        if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, 256, st))) != FE_OK) break;
+        if ((rc = from_cuda(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking))) != FE_OK) break;
+        if ((rc = from_cuda(cudaStreamSynchronize(st))) != FE_OK) break;
+    } while (0);
+    if (rc != FE_OK) {
+        cudaStreamSynchronize(st);
+        release(h);
+        return rc;
+    }
+    *out = h;
+    return FE_OK;
+}
+
+fe_status fe_draft_forward(fe_handle* h, const fe_forward_args* a, void* stream) {
+    if (!h || !a) return FE_ERR_INVALID_ARG;
+    const fe_config& c = h->cfg;
+    if (a->B < 1 || a->B > c.max_batch) return FE_ERR_INVALID_ARG;
+    if (a->top_k < 1 || a->top_k > c.top_k_max) return FE_ERR_INVALID_ARG;
+    if (!a->feat || !a->next_tok || !a->prefix_len || !a->k_cache || !a->v_cache) return FE_ERR_INVALID_ARG;
+    if (!a->topk_id || !a->topk_logit || !a->topk_prob || !a->lse) return FE_ERR_INVALID_ARG;
+    for (int i = 0; i < c.n_layers; ++i)
+        if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
+    if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
+    if (!(a->temperature == a->temperature)) return FE_ERR_INVALID_ARG;  // NaN
+    cudaStream_t st = (cudaStream_t)stream;
+    try {
+        if (!h->use_graph) return enqueue_forward(h, a, st);
+        GraphKey key;
+        key.args = *a;
+        key.args.k_cache = nullptr;
+        key.args.v_cache = nullptr;
+        key.kc.assign(a->k_cache, a->k_cache + c.n_layers);
+        key.vc.assign(a->v_cache, a->v_cache + c.n_layers);
+        if (!h->gexec || !(key == h->gkey)) {
+            cudaGraph_t graph = nullptr;
+            FE_TRY(cudaStreamBeginCapture(h->cap, cudaStreamCaptureModeThreadLocal));
+            fe_status rc = enqueue_forward(h, a, h->cap);
+            cudaError_t e = cudaStreamEndCapture(h->cap, &graph);
+            if (rc != FE_OK) {
+                if (graph) cudaGraphDestroy(graph);
+                return rc;
+            }
+            FE_TRY(e);
+            cudaGraphExec_t ex = nullptr;
+            e = cudaGraphInstantiate(&ex, graph, 0);
+            cudaGraphDestroy(graph);
+            FE_TRY(e);
+            if (h->gexec) cudaGraphExecDestroy(h->gexec);
+            h->gexec = ex;
+            h->gkey = key;
+        }
+        FE_TRY(cudaGraphLaunch(h->gexec, st));
+        return FE_OK;
+    } catch (...) {
+        return FE_ERR_OOM;
+    }
+}
+
+fe_status fe_build_tree(fe_handle* h, int32_t B, int32_t top_k, const int32_t* next_tok, const int32_t* topk_id,
+                        fe_tree* out, void* stream) {
+    if (!h || !out || !next_tok || !topk_id) return FE_ERR_INVALID_ARG;
+    if (!out->tok || !out->parent || !out->depth || !out->mask) return FE_ERR_INVALID_ARG;
+    if (B < 1 || B > h->cfg.max_batch || top_k < 1 || top_k > h->cfg.top_k_max) return FE_ERR_INVALID_ARG;
+    FE_TRY(launch_tree(B, h->cfg.n_layers, top_k, h->cfg.vocab, next_tok, topk_id, out->tok, out->parent, out->depth,
+                       out->mask, h->status, (cudaStream_t)stream));
+    return FE_OK;
+}
+
+fe_status fe_last_device_status(fe_handle* h, void* stream) {
+    if (!h) return FE_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    int v = 0;
+    FE_TRY(cudaStreamSynchronize(st));
+    FE_TRY(cudaMemcpy(&v, h->status, sizeof(int), cudaMemcpyDeviceToHost));
+    FE_TRY(cudaMemset(h->status, 0, sizeof(int)));
+    if (v & ST_TIMEOUT) return FE_ERR_TIMEOUT;
+    if (v & ST_CAPACITY) return FE_ERR_CAPACITY;
+    if (v & ST_DEVICE) return FE_ERR_DEVICE;
+    return FE_OK;
+}
+
+void fe_free(fe_handle* h) {
+    if (!h) return;
+    cudaDeviceSynchronize();
+    release(h);
+}
+
+int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
+    if (!h || B < 1) return -1;
+    const int N = h->cfg.n_layers;
+    int n = 2 * linear_launches() + N * (4 * linear_launches() + attention_launches()) +
+            lmhead_launches(N * B, h->cfg.d, h->dev);
+    return n + (with_tree ? 1 : 0);
+}
+
+fe_status fe_selftest_timeout(fe_handle* h, int64_t timeout_ns, void* stream) {
+    if (!h || timeout_ns < 1000 || timeout_ns > 1000000000LL) return FE_ERR_INVALID_ARG;
+    FE_TRY(launch_timeout_probe(timeout_ns, h->status, (cudaStream_t)stream));
+    return FE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,62 @@
+"""The C-ABI library without a GPU: it loads, exports every entry point include/*.h
+declares, and rejects bad arguments on the host before touching CUDA."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = []
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = open(h).read()
+        names += re.findall(r"FE_API\s+[\w\s\*]+?\b(\w+)\s*\(", src)
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__
+    __graft_entry__.build_lib_only()
+    import paper_2509_20416_gb300 as fe
+    return fe
+
+
+def test_header_declares_the_boundary():
+    names = set(_declared())
+    for n in ("fe_draft_init", "fe_draft_forward", "fe_build_tree", "fe_free", "fe_status_str",
+              "fe_last_device_status"):
+        assert n in names, n
+
+
+def test_every_declared_symbol_is_exported(lib):
+    so = ctypes.CDLL(lib.LIB_PATH)
+    for n in _declared():
+        assert hasattr(so, n), f"{n} declared in include/ but not exported"
+
+
+def test_status_strings(lib):
+    assert lib.fe_status_str(lib.FE_OK) == "ok"
+    assert lib.fe_status_str(lib.FE_ERR_CAPACITY) == "prefix does not fit the cache"
+    assert lib.fe_status_str(12345) == "unknown status"
+
+
+def test_host_side_validation_needs_no_gpu(lib):
+    so = lib._lib
+    out = ctypes.c_void_p()
+    # null config / weights / out pointer: rejected before any CUDA call
+    assert so.fe_draft_init(None, None, None, ctypes.byref(out)) == lib.FE_ERR_INVALID_ARG
+    c = lib.make_config(dict(d=256, n_heads=4, n_kv_heads=3, head_dim=64, ffn=688, vocab=4096, n_layers=3,
+                             top_k_max=8, max_seq=80, rope_theta=1e4, rms_eps=1e-5, dtype="f32"))
+    w = lib.fe_weights()
+    assert so.fe_draft_init(ctypes.byref(c), ctypes.byref(w), None, ctypes.byref(out)) == lib.FE_ERR_INVALID_ARG
+    assert out.value is None
+    assert so.fe_draft_forward(None, None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_build_tree(None, 1, 1, None, None, None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_last_device_status(None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_launch_count(None, 1, 1) == -1
+    so.fe_free(None)  # no-op

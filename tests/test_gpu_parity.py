@@ -1,0 +1,133 @@
+"""CUDA path (through the C ABI) against the fp64 oracle on identical seeded inputs.
+
+Small cases span several row groups, vocabulary slabs and attention splits with ragged
+tails (V % 4 != 0, prefixes that end mid-page, P = 0); the five named workloads run at
+full size, with the oracle computing every compared sequence one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+from fe_synth import workloads as wl
+import harness as H
+import torch_ref
+
+pytestmark = pytest.mark.gpu
+
+
+def _problem(cfg):
+    W = wl.make_weights(cfg)
+    I = wl.make_inputs(cfg)
+    ks, vs = wl.make_caches(cfg)
+    return W, I, ks, vs
+
+
+def _new_row_ref(cfg, W, I, o, b, i):
+    """Expected key (after RoPE) and value the call appends to layer i's slot P_b."""
+    d, Hh, Hkv, hd = cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
+    if i == 0:
+        f = I["feat"][b].double()
+        g = W["w_fuse"].double() @ f
+        e = W["embed"].double()[int(I["next_tok"][b])]
+        x = W["w_in"].double() @ torch.cat([g, e])
+    else:
+        x = torch.tensor(o["hidden"][i - 1])
+    L = W["layers"][i]
+    u = torch.nn.functional.rms_norm(x, (d,), weight=L["attn_norm"].double(), eps=cfg["rms_eps"])
+    qkv = L["w_qkv"].double() @ u
+    k = qkv[Hh * hd:(Hh + Hkv) * hd].view(Hkv, hd)
+    v = qkv[(Hh + Hkv) * hd:].view(Hkv, hd)
+    k = torch_ref.rope_complex(k, int(I["prefix_len"][b]), cfg["rope_theta"])
+    return k, v
+
+
+def _check_cache_rows(cfg, W, I, ks, vs, g, o, b):
+    P = int(I["prefix_len"][b])
+    ps = cfg["page_size"]
+    for i in range(cfg["n_layers"]):
+        kref, vref = _new_row_ref(cfg, W, I, o, b, i)
+        for cache, logical, ref in ((g["k_cache"][i], ks[i], kref), (g["v_cache"][i], vs[i], vref)):
+            if ps:
+                tab = g["page_table"]
+                new = cache[int(tab[b, P // ps]), :, P % ps, :].double()
+                old = (torch.stack([cache[int(tab[b, p // ps]), :, p % ps, :] for p in range(P)], 1)
+                       if P else None)
+            else:
+                new = cache[b, :, P, :].double()
+                old = cache[b, :, :P, :]
+            if P:
+                assert torch.equal(old, logical[b, :, :P, :]), f"layer {i}: prefix rows were modified"
+            # the new row is stored in the cache's type: one rounding of the fp32 value
+            rel = 2.0 ** -8 if cfg["dtype"] == "bf16" else 1e-5
+            assert torch.allclose(new, ref, rtol=rel, atol=1e-4 * max(1.0, ref.abs().max().item())), i
+
+
+SMALL = {
+    "tiny_f32": dict(name="tiny"),
+    "gqa4_bf16_ragged": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376, vocab=5003,
+                                       n_layers=4, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
+                                       seed=3, page_size=0), prefix_list=[37, 0, 150]),
+    "gqa4_bf16_paged": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376, vocab=5003,
+                                      n_layers=3, dtype="bf16", B=4, prefix=0, top_k=8, rope_theta=5e5,
+                                      seed=4, page_size=16), prefix_list=[15, 16, 1, 200]),
+    "mha128_f32_temp": dict(name=dict(d=256, n_heads=2, n_kv_heads=2, head_dim=128, ffn=520, vocab=777,
+                                      n_layers=2, dtype="f32", B=2, prefix=0, top_k=3, rope_theta=1e4,
+                                      seed=5, page_size=0), prefix_list=[5, 63], temperature=0.7),
+    "gqa8_bf16_k32": dict(name=dict(d=512, n_heads=8, n_kv_heads=1, head_dim=64, ffn=512, vocab=4100,
+                                    n_layers=2, dtype="bf16", B=2, prefix=0, top_k=32, rope_theta=1e4,
+                                    seed=6, page_size=0), prefix_list=[300, 1]),
+    "chain_k1_b5": dict(name=dict(d=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=688, vocab=4096,
+                                  n_layers=5, dtype="bf16", B=5, prefix=0, top_k=1, rope_theta=1e4,
+                                  seed=8, page_size=0), prefix_list=[0, 1, 2, 33, 64]),
+}
+
+
+@pytest.mark.parametrize("case", list(SMALL))
+def test_parity_small(orc, case):
+    spec = dict(SMALL[case])
+    name = spec.pop("name")
+    cfg = wl.make_config(name, **spec)
+    W, I, ks, vs = _problem(cfg)
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert g["status"] == 0, g["status"]
+    for b in range(cfg["B"]):
+        o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
+        H.compare(orc, cfg, g, o, b)
+        _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
+
+
+def test_repeat_and_graph_replay_bit_identical():
+    """Two calls with identical arguments (the second replays the captured CUDA graph)
+    and a call without dbg buffers all give the same bits."""
+    import paper_2509_20416_gb300 as fe
+    cfg = wl.make_config(SMALL["gqa4_bf16_ragged"]["name"], prefix_list=[37, 0, 150])
+    W, I, ks, vs = _problem(cfg)
+    h = fe.fe_draft_init(dict(cfg, max_batch=cfg["B"]), W)
+    a = H.run_gpu(cfg, W, I, ks, vs, handle=h)
+    b = H.run_gpu(cfg, W, I, ks, vs, handle=h)
+    c = H.run_gpu(cfg, W, I, ks, vs, handle=h, dbg=False)
+    for key in ("topk_id", "topk_logit", "topk_prob", "lse", "tree_mask"):
+        assert np.array_equal(a[key], b[key]) and np.array_equal(a[key], c[key]), key
+    assert np.array_equal(a["logits"], b["logits"])
+    h.close()
+
+
+FULL = ["vic13b", "l31_8b", "l33_70b", "b32_l31"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_parity_full_size(orc, name):
+    """The named workloads at full size, in the launch configuration the benchmark times."""
+    cfg = wl.make_config(name)
+    W, I, ks, vs = _problem(cfg)
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert g["status"] == 0, g["status"]
+    B = cfg["B"]
+    plen = I["prefix_len"].tolist()
+    seqs = sorted({0, B - 1, int(np.argmin(plen)), int(np.argmax(plen))})
+    stats = []
+    for b in seqs:
+        o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
+        stats.append(H.compare(orc, cfg, g, o, b))
+        _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
+    print(name, stats)
