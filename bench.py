@@ -40,6 +40,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
+                    help="override a workload field (e.g. n_layers=1) for profiling runs")
     return ap.parse_args()
 
 
@@ -104,9 +106,13 @@ def dist_env():
     return ws, rank, local
 
 
-def make_problem(name: str):
+def make_problem(name: str, overrides=()):
     from fe_synth import workloads as wl
-    cfg = wl.make_config(name)
+    kw = {}
+    for o in overrides:
+        k, v = o.split("=", 1)
+        kw[k] = type(wl.WORKLOADS[name][k])(v) if k in wl.WORKLOADS[name] else float(v)
+    cfg = wl.make_config(name, **kw)
     W = wl.make_weights(cfg)
     I = wl.make_inputs(cfg)
     ks, vs = wl.make_caches(cfg)
@@ -133,7 +139,7 @@ def time_oracle(cfg, W, I, ks, vs, budget_s: float, max_runs: int | None = None)
 
 
 def workload_config(cfg, wl) -> dict:
-    return {"workload": cfg.get("name", ""), "shape": wl.describe(cfg), "B": cfg["B"], "N": cfg["n_layers"],
+    return {"workload": cfg.get("name", "") + "".join(f" {o}" for o in cfg.get("overrides", [])), "shape": wl.describe(cfg), "B": cfg["B"], "N": cfg["n_layers"],
             "top_k": cfg["top_k"], "d": cfg["d"], "vocab": cfg["vocab"], "accum": "f32",
             "l2": "inputs larger than L2 (every step streams all weights, >129 MB)" if cfg["dtype"] == "bf16"
             else "L2-resident (no flush)"}
@@ -144,8 +150,9 @@ def run_reference(args, ws, rank):
     if rank != 0:
         return
     from fe_synth import workloads as wl
-    cfg, W, I, ks, vs = make_problem(args.workload)
+    cfg, W, I, ks, vs = make_problem(args.workload, args.set)
     cfg["name"] = args.workload
+    cfg["overrides"] = list(args.set)
     # warm-up runs, then a bounded number of timed steps (one draft of sequence step % B each)
     time_oracle(cfg, W, I, ks, vs, 0, max_runs=max(1, min(args.warmup, 2)))
     one, _, thr, _ = time_oracle(cfg, W, I, ks, vs, 0, max_runs=1)
@@ -176,8 +183,9 @@ def main():
     import paper_2509_20416_gb300 as fe
     from fe_synth import workloads as wl
 
-    cfg, W, I, ks, vs = make_problem(args.workload)
+    cfg, W, I, ks, vs = make_problem(args.workload, args.set)
     cfg["name"] = args.workload
+    cfg["overrides"] = list(args.set)
     B, N, k = cfg["B"], cfg["n_layers"], cfg["top_k"]
     h = fe.fe_draft_init(dict(cfg, max_batch=B), W)
     if cfg["page_size"]:

@@ -30,8 +30,12 @@ enum Epilogue : int {
     EPI_SWIGLU = 2,  // rows (2j, 2j+1) are (gate_j, up_j): y[b, j] = silu(gate) * up
 };
 
+// tile-packed weight layout (fe_pack.cu / fe_stream.cuh)
+size_t packed_bytes(int M, int K, int es);
+cudaError_t launch_pack_tiles(const void* src, void* dst, int M, int K, int es, cudaStream_t st);
+
 struct LinearArgs {
-    const void* W;  // [M, K] storage type, 16-byte aligned, K % 8 == 0
+    const void* W;  // tile-packed [ceil(M/4)*4, K] storage type, 16-byte aligned, K % 8 == 0
     int M, K;
     int B;  // activation rows
     // prologue
@@ -65,7 +69,7 @@ inline int linear_launches() { return 1; }
 
 // ---- LM head + fused softmax statistics + per-slab top-k ------------------------------
 struct LmHeadArgs {
-    const void* W;  // lm_head [V, d]
+    const void* W;  // lm_head, tile-packed [ceil(V/4)*4, d]
     const void* gamma;  // final_norm [d]
     int V, d;
     int R;  // rows of hidden states (N * B), row r = i * B + b
@@ -78,26 +82,18 @@ struct LmHeadArgs {
     int* part_id;      // [R, n_slabs, top_k]
     float* part_val;   // [R, n_slabs, top_k]
     float* part_ms;    // [R, n_slabs, 2] (max, sum of exp) of logit * inv_temp
+    int* counters;     // [ceil(R / 8)] slab-completion counters, zero between calls
     float* dbg_logits; // [B, N, V] or null
+    int* topk_id;       // [B, N, k]
+    float* topk_logit;  // [B, N, k]
+    float* topk_prob;   // [B, N, k]
+    float* lse;         // [B, N]
     int* status;
 };
 cudaError_t lmhead_prepare(const DeviceInfo& dev);
 int lmhead_slabs(int V, const DeviceInfo& dev);
 int lmhead_launches(int R, int d, const DeviceInfo& dev);
 cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st);
-
-struct MergeArgs {
-    int R, B, N, n_slabs, top_k;
-    float inv_temp;
-    const int* part_id;
-    const float* part_val;
-    const float* part_ms;
-    int* topk_id;       // [B, N, k]
-    float* topk_logit;  // [B, N, k]
-    float* topk_prob;   // [B, N, k]
-    float* lse;         // [B, N]
-};
-cudaError_t launch_topk_merge(const MergeArgs& a, cudaStream_t st);
 
 // ---- decode attention ----------------------------------------------------------------
 struct AttnArgs {
@@ -111,12 +107,13 @@ struct AttnArgs {
     int B, H, Hkv, hd;
     int split, n_split;     // keys per work item, work items per (sequence, KV head)
     float* part;            // [B, H, n_split, hd + 2]
+    int* counters;          // [B, Hkv] split-completion counters, zero between calls
     float* out;             // [B, H * hd]
     int* status;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
-cudaError_t launch_attention(fe_dtype dt, const AttnArgs& a, cudaStream_t st);   // 2 kernels
-inline int attention_launches() { return 2; }
+cudaError_t launch_attention(fe_dtype dt, const AttnArgs& a, cudaStream_t st);
+inline int attention_launches() { return 1; }
 
 // ---- draft tree + failure-detection probe ------------------------------------------------
 cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,

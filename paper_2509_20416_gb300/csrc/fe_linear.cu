@@ -62,7 +62,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearA
 
     if (threadIdx.x >= kConsumers) {
         if (threadIdx.x == kConsumers)
-            stream_produce<WT>((const unsigned char*)a.W, a.M, a.K, g0, g1, s, ns, a.status);
+            stream_produce<WT>((const unsigned char*)a.W, a.K, g0, g1, s, ns, a.status);
         return;
     }
     ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};

@@ -1,15 +1,22 @@
 // The frozen LM head applied to every cascade output h_i (Sec. 2.1), fused with the
-// softmax statistics and the top-k selection of Sec. 2.2, so the [N*B, V] logits never
-// reach global memory.
+// softmax statistics and the top-k selection of Sec. 2.2, in one kernel: the [N*B, V]
+// logits never reach global memory (unless the caller asks for them for a parity check).
 //
-// Kernel 1 (lmhead_kernel): one weight-streaming CTA per vocabulary slab (a contiguous
-// range of LM-head rows). The hidden rows z_r = RMSNorm(h_r; gamma_out) of all N*B rows
-// are staged once in shared memory, so the LM head is read from HBM once for all N
-// depths. Per row r the CTA keeps a running top-k (by logit, ties to the smaller id)
-// and the running (max, sum of exp) of logit / T, and writes them as the slab's partial.
-// Kernel 2 (topk_merge_kernel): one CTA per row merges the slabs' partials: k rounds of
-// a block arg-max over n_slabs * k candidates, lse = M + log sum_j s_j e^(m_j - M), and
-// prob = exp(logit / T - lse).
+// Grid: (n_slabs, ceil(R / BT)). Each CTA streams one vocabulary slab (a contiguous range
+// of LM-head row groups) through the weight-streaming core (fe_stream.cuh) against the
+// RMSNorm'd hidden rows z_r = RMSNorm(h_r; gamma_out) of its tile of BT rows, staged once
+// in shared memory, so the LM head is read from HBM once for all N depths.
+//  - Per row group, warp 0 holds the 4 x BT new logits (one per lane), stores them in a
+//    shared-memory slab buffer, and tests them against each row's current k-th best
+//    (ties to the smaller id); the few that pass are inserted into the row's sorted
+//    top-k list one lane at a time.
+//  - At the end of the slab, warp b computes row b's (max, sum of exp) of logit / T over
+//    the buffered logits and writes the slab's partial (top-k list and statistics).
+//  - The last CTA to finish a row tile (an atomic counter per tile) merges all slabs'
+//    partials: lse = M + log sum_j s_j e^(m_j - M); the global top-k is taken from the
+//    candidates not below tau = max over slabs of the slab's k-th value (a slab holds k
+//    candidates >= tau, so nothing below tau can be among the k best); probabilities are
+//    exp(logit / T - lse).
 #include <float.h>
 
 #include "fe_kernels.h"
@@ -18,165 +25,132 @@
 namespace fe {
 
 constexpr int kMaxTopK = 32;
+constexpr int kLmTile = 8;           // rows of z per tile (BT <= 8)
+constexpr int kMergeCap = 256;       // survivors per row kept in shared memory for the merge
 
 __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
     return va > vb || (va == vb && ia < ib);
 }
 
 struct TopkState {
-    int id[8][kMaxTopK];
-    float val[8][kMaxTopK];
-    int cnt[8];
-    float m[8], s[8];
+    int id[kLmTile][kMaxTopK];
+    float val[kLmTile][kMaxTopK];
+    int cnt[kLmTile];
+    int last;
 };
 
 template <int BT>
 struct LmEpi {
     const LmHeadArgs* a;
     TopkState* st;
-    int b0, nb;
+    float* slab;  // [BT][slab_cap]
+    int slab_cap, b0, nb, g0;
     __device__ __forceinline__ void operator()(int g, const float* red) const {
         const int t = threadIdx.x;
-        if (t >= nb) return;
-        const int zr = b0 + t;
-        const int k = a->top_k;
-        int* ids = st->id[t];
-        float* vals = st->val[t];
-        int cnt = st->cnt[t];
-        float m = st->m[t], s = st->s[t];
-        for (int r = 0; r < kGroupRows; ++r) {
-            const int v = g * kGroupRows + r;
-            if (v >= a->V) break;
-            const float lg = group_sum<BT>(red, r, t);
+        if (t >= 32) return;  // warp 0 only: lane t holds candidate (row r = t / BT, z-row b = t % BT)
+        const int r = t / BT, b = t % BT;
+        const int v = g * kGroupRows + r;
+        const bool valid = t < kGroupRows * BT && b < nb && v < a->V;
+        float lg = -INFINITY;
+        if (valid) {
+            lg = group_sum<BT>(red, r, b);
+            slab[b * slab_cap + (g - g0) * kGroupRows + r] = lg;
             if (a->dbg_logits) {
-                const int i = zr / a->B, b = zr % a->B;
-                a->dbg_logits[((size_t)b * a->N + i) * a->V + v] = lg;
+                const int zr = b0 + b;
+                const int i = zr / a->B, sb = zr % a->B;
+                a->dbg_logits[((size_t)sb * a->N + i) * a->V + v] = lg;
             }
-            const float lt = lg * a->inv_temp;
-            if (lt > m) {
-                s = s * expf(m - lt) + 1.0f;
-                m = lt;
-            } else {
-                s += expf(lt - m);
-            }
-            int pos;
-            if (cnt < k) {
-                pos = cnt++;
-            } else if (better(lg, v, vals[k - 1], ids[k - 1])) {
-                pos = k - 1;
-            } else {
-                continue;
-            }
-            while (pos > 0 && better(lg, v, vals[pos - 1], ids[pos - 1])) {
-                vals[pos] = vals[pos - 1];
-                ids[pos] = ids[pos - 1];
-                --pos;
-            }
-            vals[pos] = lg;
-            ids[pos] = v;
         }
-        st->cnt[t] = cnt;
-        st->m[t] = m;
-        st->s[t] = s;
+        const int k = a->top_k;
+        bool pass = false;
+        if (valid) {
+            const int c = st->cnt[b];
+            pass = c < k || better(lg, v, st->val[b][k - 1], st->id[b][k - 1]);
+        }
+        unsigned mask = __ballot_sync(0xffffffffu, pass);
+        while (mask) {
+            const int j = __ffs(mask) - 1;
+            mask &= mask - 1;
+            if (t == j) {  // insert (lg, v) into row b's sorted list
+                int c = st->cnt[b];
+                int pos;
+                if (c < k) {
+                    pos = c;
+                    st->cnt[b] = c + 1;
+                } else if (better(lg, v, st->val[b][k - 1], st->id[b][k - 1])) {
+                    pos = k - 1;
+                } else {
+                    pos = -1;
+                }
+                if (pos >= 0) {
+                    while (pos > 0 && better(lg, v, st->val[b][pos - 1], st->id[b][pos - 1])) {
+                        st->val[b][pos] = st->val[b][pos - 1];
+                        st->id[b][pos] = st->id[b][pos - 1];
+                        --pos;
+                    }
+                    st->val[b][pos] = lg;
+                    st->id[b][pos] = v;
+                }
+            }
+            __syncwarp();
+        }
     }
 };
 
-template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int ns) {
-    extern __shared__ __align__(128) unsigned char smem[];
-    __shared__ TopkState st;
-    const int K = a.d;
-    const int Kpad = (K + 3) & ~3;
-    const int b0 = blockIdx.y * BT;
-    const int nb = min(BT, a.R - b0);
-    StreamSmem s = carve_stream_smem(smem, ns, min(BT, a.R), Kpad, BT);
-    if (threadIdx.x < 8) {
-        st.cnt[threadIdx.x] = 0;
-        st.m[threadIdx.x] = -INFINITY;
-        st.s[threadIdx.x] = 0.f;
-    }
-    stream_init_barriers(s, ns);
-
-    const int GM = (a.V + kGroupRows - 1) / kGroupRows;
-    const int slab = blockIdx.x;
-    const int g0 = (int)(((int64_t)slab * GM) / gridDim.x);
-    const int g1 = (int)(((int64_t)(slab + 1) * GM) / gridDim.x);
-
-    if (threadIdx.x >= kConsumers) {
-        if (threadIdx.x == kConsumers) stream_produce<WT>((const unsigned char*)a.W, a.V, K, g0, g1, s, ns, a.status);
-        return;
-    }
-    ProParams pp{PRO_RMSNORM, a.hid, a.d, a.gamma, a.eps, nullptr, nullptr, 0, 0};
-    stage_activations<WT>(pp, K, s.X, Kpad, b0, nb, a.status, s.red);
-    named_sync(1, kConsumers);
-    LmEpi<BT> ep{&a, &st, b0, nb};
-    stream_consume<WT, BT>(K, g0, g1, s, ns, Kpad, nb, a.status, ep);
-
-    // partials of this slab (entries past cnt are padding that loses every comparison)
-    const int t = threadIdx.x;
-    if (t < nb) {
-        const int zr = b0 + t;
-        const size_t base = ((size_t)zr * a.n_slabs + slab);
-        for (int j = 0; j < a.top_k; ++j) {
-            const bool ok = j < st.cnt[t];
-            a.part_id[base * a.top_k + j] = ok ? st.id[t][j] : INT_MAX;
-            a.part_val[base * a.top_k + j] = ok ? st.val[t][j] : -INFINITY;
-        }
-        a.part_ms[base * 2 + 0] = st.m[t];
-        a.part_ms[base * 2 + 1] = st.s[t];
-    }
-}
-
-__global__ void __launch_bounds__(256) topk_merge_kernel(const MergeArgs a) {
-    extern __shared__ __align__(16) unsigned char smem[];
-    const int zr = blockIdx.x;
-    const int n = a.n_slabs * a.top_k;
-    float* vals = (float*)smem;
-    int* ids = (int*)(vals + n);
-    __shared__ float rv[8];
-    __shared__ int ri[8], rp[8];
-    __shared__ float s_lse;
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    for (int j = t; j < n; j += 256) {
-        vals[j] = a.part_val[(size_t)zr * n + j];
-        ids[j] = a.part_id[(size_t)zr * n + j];
-    }
-    // lse of logit / T from the slabs' (max, sum) pairs
+// Merge of all slabs' partials for one row zr, by one warp.
+__device__ void merge_row(const LmHeadArgs& a, int zr, float* sv, int* si, int* scount, unsigned* taken) {
+    const int lane = threadIdx.x & 31;
+    const int k = a.top_k, ns = a.n_slabs;
+    const float* pv = a.part_val + (size_t)zr * ns * k;
+    const int* pi = a.part_id + (size_t)zr * ns * k;
+    const float* pm = a.part_ms + (size_t)zr * ns * 2;
+    // log-sum-exp of logit / T over the whole vocabulary
     float M = -INFINITY;
-    for (int j = t; j < a.n_slabs; j += 256) M = fmaxf(M, a.part_ms[((size_t)zr * a.n_slabs + j) * 2]);
+    for (int j = lane; j < ns; j += 32) M = fmaxf(M, __ldcg(pm + 2 * j));
     M = warp_max(M);
-    if (lane == 0) rv[warp] = M;
-    __syncthreads();
-    M = rv[0];
-    for (int w = 1; w < 8; ++w) M = fmaxf(M, rv[w]);
-    __syncthreads();
     float S = 0.f;
-    for (int j = t; j < a.n_slabs; j += 256) {
-        const float mj = a.part_ms[((size_t)zr * a.n_slabs + j) * 2];
-        const float sj = a.part_ms[((size_t)zr * a.n_slabs + j) * 2 + 1];
-        if (sj > 0.f) S += sj * expf(mj - M);
+    for (int j = lane; j < ns; j += 32) {
+        const float sj = __ldcg(pm + 2 * j + 1);
+        if (sj > 0.f) S += sj * expf(__ldcg(pm + 2 * j) - M);
     }
     S = warp_sum(S);
-    if (lane == 0) rv[warp] = S;
-    __syncthreads();
-    if (t == 0) {
-        float tot = 0.f;
-        for (int w = 0; w < 8; ++w) tot += rv[w];
-        s_lse = M + logf(tot);
+    const float lse = M + logf(S);
+    // tau: the largest k-th value over slabs
+    float tau = -INFINITY;
+    for (int j = lane; j < ns; j += 32) tau = fmaxf(tau, __ldcg(pv + (size_t)j * k + k - 1));
+    tau = warp_max(tau);
+    if (lane == 0) *scount = 0;
+    __syncwarp();
+    bool overflow = false;
+    for (int j = lane; j < ns; j += 32) {
+        for (int r = 0; r < k; ++r) {
+            const float v = __ldcg(pv + (size_t)j * k + r);
+            if (v < tau) break;  // slab lists are sorted, descending
+            const int pos = atomicAdd(scount, 1);
+            if (pos < kMergeCap) {
+                sv[pos] = v;
+                si[pos] = __ldcg(pi + (size_t)j * k + r);
+            } else {
+                overflow = true;
+            }
+        }
     }
-    __syncthreads();
-    const float lse = s_lse;
+    overflow = __any_sync(0xffffffffu, overflow);
+    __syncwarp();
+    const int n = overflow ? ns * k : min(*scount, kMergeCap);
+    // k rounds of a warp arg-max (desc value, asc id); taken entries flagged in a bitmap
+    for (int w = lane; w < (n + 31) / 32; w += 32) taken[w] = 0u;
+    __syncwarp();
     const int i = zr / a.B, b = zr % a.B;
-    const size_t ob = ((size_t)b * a.N + i) * a.top_k;
-    for (int r = 0; r < a.top_k; ++r) {
+    const size_t ob = ((size_t)b * a.N + i) * k;
+    for (int r = 0; r < k; ++r) {
         float bv = -INFINITY;
         int bi = INT_MAX, bp = -1;
-        for (int j = t; j < n; j += 256) {
-            if (bp < 0 || better(vals[j], ids[j], bv, bi)) {
-                bv = vals[j];
-                bi = ids[j];
-                bp = j;
-            }
+        for (int j = lane; j < n; j += 32) {
+            if (taken[j >> 5] & (1u << (j & 31))) continue;
+            const float v = overflow ? __ldcg(pv + j) : sv[j];
+            const int id = overflow ? __ldcg(pi + j) : si[j];
+            if (bp < 0 || better(v, id, bv, bi)) { bv = v; bi = id; bp = j; }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -185,21 +159,88 @@ __global__ void __launch_bounds__(256) topk_merge_kernel(const MergeArgs a) {
             const int op = __shfl_xor_sync(0xffffffffu, bp, o);
             if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
         }
-        if (lane == 0) { rv[warp] = bv; ri[warp] = bi; rp[warp] = bp; }
-        __syncthreads();
-        if (t == 0) {
-            for (int w = 1; w < 8; ++w)
-                if (rp[w] >= 0 && (rp[0] < 0 || better(rv[w], ri[w], rv[0], ri[0]))) {
-                    rv[0] = rv[w]; ri[0] = ri[w]; rp[0] = rp[w];
-                }
-            a.topk_id[ob + r] = ri[0];
-            a.topk_logit[ob + r] = rv[0];
-            a.topk_prob[ob + r] = expf(rv[0] * a.inv_temp - lse);
-            if (rp[0] >= 0) { vals[rp[0]] = -INFINITY; ids[rp[0]] = INT_MAX; }
+        if (lane == 0) {
+            a.topk_id[ob + r] = bi;
+            a.topk_logit[ob + r] = bv;
+            a.topk_prob[ob + r] = expf(bv * a.inv_temp - lse);
+            if (bp >= 0) taken[bp >> 5] |= 1u << (bp & 31);
         }
-        __syncthreads();
+        __syncwarp();
     }
-    if (t == 0) a.lse[(size_t)b * a.N + i] = lse;
+    if (lane == 0) a.lse[(size_t)b * a.N + i] = lse;
+}
+
+template <typename WT, int BT>
+__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int ns, int slab_cap) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ TopkState st;
+    const int K = a.d;
+    const int Kpad = (K + 3) & ~3;
+    const int tile = blockIdx.y;
+    const int b0 = tile * BT;
+    const int nb = min(BT, a.R - b0);
+    const int xrows = min(BT, a.R);
+    StreamSmem s = carve_stream_smem(smem, ns, xrows, Kpad, BT);
+    float* slab = (float*)(smem + stream_smem_bytes(ns, xrows, Kpad, BT));
+    if (threadIdx.x < kLmTile) st.cnt[threadIdx.x] = 0;
+    stream_init_barriers(s, ns);
+
+    const int GM = (a.V + kGroupRows - 1) / kGroupRows;
+    const int sl = blockIdx.x;
+    const int g0 = (int)(((int64_t)sl * GM) / gridDim.x);
+    const int g1 = (int)(((int64_t)(sl + 1) * GM) / gridDim.x);
+
+    if (threadIdx.x >= kConsumers) {
+        if (threadIdx.x == kConsumers) stream_produce<WT>((const unsigned char*)a.W, K, g0, g1, s, ns, a.status);
+        return;
+    }
+    ProParams pp{PRO_RMSNORM, a.hid, a.d, a.gamma, a.eps, nullptr, nullptr, 0, 0};
+    stage_activations<WT>(pp, K, s.X, Kpad, b0, nb, a.status, s.red);
+    named_sync(1, kConsumers);
+    LmEpi<BT> ep{&a, &st, slab, slab_cap, b0, nb, g0};
+    stream_consume<WT, BT>(K, g0, g1, s, ns, Kpad, nb, a.status, ep);
+    named_sync(1, kConsumers);
+
+    // this slab's partial for each row of the tile (warp b <-> row b)
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int nrows = min((g1 - g0) * kGroupRows, a.V - g0 * kGroupRows);
+    if (warp < nb) {
+        const int zr = b0 + warp;
+        const float* sb = slab + warp * slab_cap;
+        float m = -INFINITY;
+        for (int j = lane; j < nrows; j += 32) m = fmaxf(m, sb[j] * a.inv_temp);
+        m = warp_max(m);
+        float sum = 0.f;
+        for (int j = lane; j < nrows; j += 32) sum += expf(sb[j] * a.inv_temp - m);
+        sum = warp_sum(sum);
+        const size_t base = (size_t)zr * a.n_slabs + sl;
+        for (int j = lane; j < a.top_k; j += 32) {
+            const bool ok = j < st.cnt[warp];
+            a.part_id[base * a.top_k + j] = ok ? st.id[warp][j] : INT_MAX;
+            a.part_val[base * a.top_k + j] = ok ? st.val[warp][j] : -INFINITY;
+        }
+        if (lane == 0) {
+            a.part_ms[base * 2 + 0] = m;
+            a.part_ms[base * 2 + 1] = sum;
+        }
+    }
+    // the last slab CTA of this tile merges the tile's rows
+    __threadfence();
+    named_sync(1, kConsumers);
+    if (t == 0) st.last = atomicAdd(&a.counters[tile], 1) == (int)gridDim.x - 1;
+    named_sync(1, kConsumers);
+    if (!st.last) return;
+    __threadfence();
+    // shared memory of the finished stream is reused: per warp kMergeCap values, ids, a
+    // counter and a taken-bitmap sized for the overflow fallback
+    const int bitmap_words = (a.n_slabs * a.top_k + 31) / 32;
+    unsigned char* base = smem + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
+    float* sv = (float*)base;
+    int* si = (int*)(sv + kMergeCap);
+    int* scount = si + kMergeCap;
+    unsigned* taken = (unsigned*)(scount + 4);
+    if (warp < nb) merge_row(a, b0 + warp, sv, si, scount, taken);
+    if (t == 0) a.counters[tile] = 0;
 }
 
 // ---- host side ----------------------------------------------------------------------------
@@ -224,13 +265,21 @@ template <typename WT, int BT>
 cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st) {
     const int Kpad = (a.d + 3) & ~3;
     const int xrows = BT < a.R ? BT : a.R;
+    const int GM = (a.V + kGroupRows - 1) / kGroupRows;
+    const int slab_cap = ((GM + a.n_slabs - 1) / a.n_slabs) * kGroupRows;
     const size_t budget = (size_t)dev.max_smem_optin - kStaticReserve;
-    const size_t fixed = stream_smem_bytes(0, xrows, Kpad, BT);
+    const size_t extra = (size_t)xrows * slab_cap * sizeof(float);
+    const size_t merge = (size_t)kLmTile * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
+    const size_t fixed = stream_smem_bytes(0, xrows, Kpad, BT) + extra;
+    if (fixed >= budget) return cudaErrorInvalidValue;
     int ns = (int)((budget - fixed) / (kStageBytes + 16));
     ns = ns > kMaxStages ? kMaxStages : ns;
     if (ns < 2) return cudaErrorInvalidValue;
+    size_t smem = stream_smem_bytes(ns, xrows, Kpad, BT) + extra;
+    if (smem < merge) smem = merge;
+    if (smem > budget) return cudaErrorInvalidValue;
     dim3 grid(a.n_slabs, (a.R + BT - 1) / BT);
-    lmhead_kernel<WT, BT><<<grid, kStreamThreads, stream_smem_bytes(ns, xrows, Kpad, BT), st>>>(a, ns);
+    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, ns, slab_cap);
     return cudaGetLastError();
 }
 
@@ -262,16 +311,11 @@ int lmhead_slabs(int V, const DeviceInfo& dev) {
     return GM < dev.num_sms ? GM : dev.num_sms;
 }
 
-int lmhead_launches(int, int, const DeviceInfo&) { return 2; }
+int lmhead_launches(int, int, const DeviceInfo&) { return 1; }
 
 cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st) {
+    if (a.top_k < 1 || a.top_k > kMaxTopK) return cudaErrorInvalidValue;
     return dt == FE_F32 ? launch_t<float>(a, dev, st) : launch_t<bf16_t>(a, dev, st);
-}
-
-cudaError_t launch_topk_merge(const MergeArgs& a, cudaStream_t st) {
-    const size_t smem = (size_t)a.n_slabs * a.top_k * (sizeof(float) + sizeof(int));
-    topk_merge_kernel<<<a.R, 256, smem, st>>>(a);
-    return cudaGetLastError();
 }
 
 }  // namespace fe

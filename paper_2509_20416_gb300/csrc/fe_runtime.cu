@@ -18,6 +18,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <cstdlib>
 #include <new>
 #include <vector>
@@ -62,6 +63,8 @@ struct fe_handle {
     int* lm_part_id = nullptr;
     float *lm_part_val = nullptr, *lm_part_ms = nullptr;
     int* status = nullptr;
+    int* attn_counters = nullptr;
+    int* lm_counters = nullptr;
     int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
     cudaStream_t cap = nullptr;
     cudaGraphExec_t gexec = nullptr;
@@ -112,18 +115,21 @@ struct Sizes {
     size_t w_fuse, w_in, embed, lm_head, norm, qkv, wo, gu, down;
 };
 
+// bytes of each matrix in the tile-packed layout (rows padded to a multiple of 4); the
+// embedding and the norm gains stay in their canonical layout
 Sizes weight_sizes(const fe_config& c, size_t es) {
-    const size_t d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    const int d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    const int e = (int)es;
     Sizes s;
-    s.w_fuse = d * 3 * d * es;
-    s.w_in = d * 2 * d * es;
-    s.embed = V * d * es;
-    s.lm_head = V * d * es;
-    s.norm = d * es;
-    s.qkv = (H + 2 * Hkv) * hd * d * es;
-    s.wo = d * H * hd * es;
-    s.gu = 2 * F * d * es;
-    s.down = d * F * es;
+    s.w_fuse = packed_bytes(d, 3 * d, e);
+    s.w_in = packed_bytes(d, 2 * d, e);
+    s.embed = (size_t)V * d * es;
+    s.lm_head = packed_bytes(V, d, e);
+    s.norm = (size_t)d * es;
+    s.qkv = packed_bytes((H + 2 * Hkv) * hd, d, e);
+    s.wo = packed_bytes(d, H * hd, e);
+    s.gu = packed_bytes(2 * F, d, e);
+    s.down = packed_bytes(d, F, e);
     return s;
 }
 
@@ -155,7 +161,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     aa.max_pages = c.page_size > 0 ? (c.max_seq + c.page_size - 1) / c.page_size : 0;
     aa.rope_cs = h->rope_cs; aa.B = B; aa.H = H; aa.Hkv = Hkv; aa.hd = hd;
     aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
-    aa.part = h->attn_part; aa.out = h->o; aa.status = h->status;
+    aa.part = h->attn_part; aa.counters = h->attn_counters; aa.out = h->o; aa.status = h->status;
 
     for (int i = 0; i < N; ++i) {
         const LayerPacked& L = h->layers[i];
@@ -189,13 +195,9 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.W = h->lm_head; lm.gamma = h->final_norm; lm.V = V; lm.d = d; lm.R = N * B; lm.B = B; lm.N = N;
     lm.hid = h->hid; lm.eps = c.rms_eps; lm.inv_temp = inv_temp; lm.top_k = a->top_k; lm.n_slabs = h->lm_slabs;
     lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
-    lm.dbg_logits = a->dbg_logits; lm.status = h->status;
+    lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
+    lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
     FE_TRY(launch_lmhead(dt, lm, h->dev, st));
-    MergeArgs mg{};
-    mg.R = N * B; mg.B = B; mg.N = N; mg.n_slabs = h->lm_slabs; mg.top_k = a->top_k; mg.inv_temp = inv_temp;
-    mg.part_id = h->lm_part_id; mg.part_val = h->lm_part_val; mg.part_ms = h->lm_part_ms;
-    mg.topk_id = a->topk_id; mg.topk_logit = a->topk_logit; mg.topk_prob = a->topk_prob; mg.lse = a->lse;
-    FE_TRY(launch_topk_merge(mg, st));
     if (a->dbg_hidden)
         FE_TRY(cudaMemcpyAsync(a->dbg_hidden, h->hid, (size_t)N * B * d * sizeof(float), cudaMemcpyDeviceToDevice,
                                st));
@@ -268,16 +270,32 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                  (2 * align256(sz.norm) + align256(sz.qkv) + align256(sz.wo) + align256(sz.gu) + align256(sz.down));
         if ((rc = from_cuda(cudaMalloc(&h->wbuf, total))) != FE_OK) break;
         char* p = (char*)h->wbuf;
+        const int es = (int)h->es;
+        // staging buffer for one canonical [M, K] matrix before it is tile-packed
+        const size_t stage_bytes = std::max({(size_t)c.vocab * c.d, (size_t)c.d * 3 * c.d,
+                                             (size_t)2 * c.ffn * c.d,
+                                             (size_t)(c.n_heads + 2 * c.n_kv_heads) * c.head_dim * c.d}) * h->es;
+        void* staging = nullptr;
+        if ((rc = from_cuda(cudaMalloc(&staging, stage_bytes))) != FE_OK) break;
         auto put = [&](const void* src, size_t bytes) -> const void* {
             void* dst = p;
             p += align256(bytes);
             if (cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, st) != cudaSuccess) rc = FE_ERR_CUDA;
             return dst;
         };
-        h->w_fuse = put(w->w_fuse, sz.w_fuse);
-        h->w_in = put(w->w_in, sz.w_in);
+        auto put_packed = [&](const void* src, int M, int K) -> const void* {
+            void* dst = p;
+            p += align256(packed_bytes(M, K, es));
+            if (cudaMemcpyAsync(staging, src, (size_t)M * K * es, cudaMemcpyDefault, st) != cudaSuccess ||
+                launch_pack_tiles(staging, dst, M, K, es, st) != cudaSuccess)
+                rc = FE_ERR_CUDA;
+            return dst;
+        };
+        const int dm = c.d, nq = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim, hq = c.n_heads * c.head_dim;
+        h->w_fuse = put_packed(w->w_fuse, dm, 3 * dm);
+        h->w_in = put_packed(w->w_in, dm, 2 * dm);
         h->embed = put(w->embed, sz.embed);
-        h->lm_head = put(w->lm_head, sz.lm_head);
+        h->lm_head = put_packed(w->lm_head, c.vocab, dm);
         h->final_norm = put(w->final_norm, sz.norm);
         h->layers.resize(c.n_layers);
         for (int i = 0; i < c.n_layers && rc == FE_OK; ++i) {
@@ -285,19 +303,23 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             LayerPacked& P = h->layers[i];
             P.attn_norm = put(L.attn_norm, sz.norm);
             P.mlp_norm = put(L.mlp_norm, sz.norm);
-            P.w_qkv = put(L.w_qkv, sz.qkv);
-            P.w_o = put(L.w_o, sz.wo);
-            // [gate; up] interleaved by row: row 2j = gate_j, row 2j+1 = up_j
+            P.w_qkv = put_packed(L.w_qkv, nq, dm);
+            P.w_o = put_packed(L.w_o, dm, hq);
+            // [gate; up] interleaved by row (row 2j = gate_j, row 2j+1 = up_j), then packed
             void* gu = p;
             p += align256(sz.gu);
-            const size_t rowb = (size_t)c.d * h->es;
-            if (cudaMemcpy2DAsync(gu, 2 * rowb, L.w_gate, rowb, rowb, c.ffn, cudaMemcpyDefault, st) != cudaSuccess ||
-                cudaMemcpy2DAsync((char*)gu + rowb, 2 * rowb, L.w_up, rowb, rowb, c.ffn, cudaMemcpyDefault, st) !=
-                    cudaSuccess)
+            const size_t rowb = (size_t)dm * h->es;
+            if (cudaMemcpy2DAsync(staging, 2 * rowb, L.w_gate, rowb, rowb, c.ffn, cudaMemcpyDefault, st) !=
+                    cudaSuccess ||
+                cudaMemcpy2DAsync((char*)staging + rowb, 2 * rowb, L.w_up, rowb, rowb, c.ffn, cudaMemcpyDefault,
+                                  st) != cudaSuccess ||
+                launch_pack_tiles(staging, gu, 2 * c.ffn, dm, es, st) != cudaSuccess)
                 rc = FE_ERR_CUDA;
             P.w_gu = gu;
-            P.w_down = put(L.w_down, sz.down);
+            P.w_down = put_packed(L.w_down, dm, c.ffn);
         }
+        cudaStreamSynchronize(st);
+        cudaFree(staging);
         if (rc != FE_OK) break;
 
         // ---- RoPE table (cos, sin) per position and pair, computed in double ----
@@ -318,16 +340,18 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lm_slabs = lmhead_slabs(c.vocab, h->dev);
         const size_t R = (size_t)c.n_layers * B;
         const size_t k = c.top_k_max;
-        size_t off[12], n = 0, tot = 0;
-        const size_t bytes[12] = {
+        size_t off[14], n = 0, tot = 0;
+        const size_t bytes[14] = {
             cs.size() * sizeof(float),                             // rope
             B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
             B * F * 4, R * d * 4,                                  // act, hid
             B * H * h->attn_nsplit * (hd + 2) * 4,                 // attention partials
             R * h->lm_slabs * k * 4, R * h->lm_slabs * k * 4,      // LM-head partial ids, values
             R * h->lm_slabs * 2 * 4,                               // LM-head partial (max, sum)
-            256};                                                  // status
-        for (n = 0; n < 12; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            256,                                                   // status
+            B * c.n_kv_heads * 4,                                  // attention split counters
+            R * 4};                                                // LM-head slab counters
+        for (n = 0; n < 14; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -342,9 +366,12 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lm_part_val = (float*)(s + off[9]);
         h->lm_part_ms = (float*)(s + off[10]);
         h->status = (int*)(s + off[11]);
+        h->attn_counters = (int*)(s + off[12]);
+        h->lm_counters = (int*)(s + off[13]);
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
-        if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, 256, st))) != FE_OK) break;
+        // status word and completion counters start (and stay, between calls) at zero
+        if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, off[13] + bytes[13] - off[11], st))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamSynchronize(st))) != FE_OK) break;
     } while (0);

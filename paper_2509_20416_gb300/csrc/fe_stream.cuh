@@ -5,16 +5,20 @@
 // matrix once and does 2 flops per weight: the phases are bound by HBM bandwidth, not
 // by arithmetic. So the CTA is built around keeping HBM busy:
 //
-//   - warp 8 (one elected thread) is the producer: it walks the CTA's contiguous range
-//     of 4-row groups of W and issues bulk TMA copies (cp.async.bulk, global -> shared)
-//     of up to 16 KB per stage into a ring of n_stages stages, each stage completing on
-//     its own mbarrier; it runs as far ahead as the ring allows;
-//   - warps 0..7 are consumers: stage t holds 4 rows x KS columns; thread t handles rows
-//     {2h, 2h+1} (h = t / 128) at 16-byte column vectors t % 128, t % 128 + 128, ... and
-//     multiplies them by the activations X, which sit in shared memory as float32 for
-//     the whole phase. Each X vector is reused for two weight rows. Partial sums are
-//     reduced across the 128 threads of a half once per row group (warp shuffles, then
-//     4 warps through shared memory) and handed to the phase's epilogue.
+//   - Weights are tile-packed at init (fe_pack.cu): each matrix is cut into groups of 4
+//     rows, and each group into K-slices of kKS columns; the 4 x width block of one
+//     (group, slice) is stored contiguously, so one stage of the stream is ONE
+//     contiguous bulk copy of up to 16 KB. (Row-major stages made of 4 row pieces at the
+//     row stride measured at ~3.7 TB/s on GB300; contiguous 4-16 KB copies at ~6.4 TB/s.)
+//   - Warp 8 (one elected thread) is the producer: it walks the CTA's contiguous range of
+//     row groups and issues cp.async.bulk (TMA) copies into a ring of n_stages stages,
+//     each completing on its own mbarrier, running as far ahead as the ring allows.
+//   - Warps 0..7 are consumers: thread t handles 16-byte column vectors t, t+256, ... of
+//     all 4 rows of a stage and multiplies them by the activations X (float32 in shared
+//     memory for the whole phase, staged once with a fused prologue), so each X vector is
+//     reused for 4 weight rows. Per row group the 4 x BT partial sums are reduced across
+//     each warp with a transposing shuffle reduction, then across the 8 warps through
+//     shared memory, and handed to the phase's epilogue.
 //
 // Accumulation is float32 FMA on CUDA cores: at 1..8 activation rows the tensor pipe
 // would idle, and this keeps fp32 weights (the small parity workload) on exact fp32
@@ -30,40 +34,47 @@ constexpr int kConsumers = kConsumerWarps * 32;  // 256 threads
 constexpr int kStreamThreads = kConsumers + 32;  // + the producer warp
 constexpr int kGroupRows = 4;                    // weight rows per group
 constexpr int kStageBytes = 16384;               // 4 rows x 4 KB
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 13;
 
 template <typename WT>
 struct StreamGeom {
     static constexpr int kES = Storage<WT>::kBytes;
-    static constexpr int kVec = Vec16<WT>::kN;                       // elements per 16 B
-    static constexpr int kKS = kStageBytes / (kGroupRows * kES);     // columns per stage
+    static constexpr int kVec = Vec16<WT>::kN;                    // elements per 16 B
+    static constexpr int kKS = kStageBytes / (kGroupRows * kES);  // columns per full slice
 };
+
+// Element offset of tile (group g, slice s) in a tile-packed [ceil(M/4)*4, K] matrix.
+template <typename WT>
+__host__ __device__ __forceinline__ int64_t tile_offset(int g, int s, int K) {
+    return (int64_t)g * kGroupRows * K + (int64_t)s * kGroupRows * StreamGeom<WT>::kKS;
+}
 
 struct StreamSmem {
     unsigned char* ring;  // n_stages x kStageBytes (128-byte aligned)
-    float* X;             // [nb][Kpad] activations
-    float* red;           // [2][kConsumerWarps][2][BT] partial sums (double-buffered)
+    float* X;             // [xrows][Kpad] activations
+    float* red;           // [2][kConsumerWarps][4 * BT] per-warp partial sums (double-buffered)
     uint64_t* full;       // [n_stages]
     uint64_t* empty;      // [n_stages]
     int* abort;           // set when any wait of this CTA gave up
 };
 
-// Bytes of dynamic shared memory a streaming CTA needs (before epilogue extras).
-__host__ __device__ inline size_t stream_smem_bytes(int n_stages, int nb, int Kpad, int BT) {
+// Bytes of dynamic shared memory a streaming CTA needs (before any epilogue extras).
+__host__ __device__ inline size_t stream_smem_bytes(int n_stages, int xrows, int Kpad, int BT) {
     size_t b = (size_t)n_stages * kStageBytes;
-    b += (size_t)nb * Kpad * sizeof(float);
-    b += (size_t)2 * kConsumerWarps * 2 * BT * sizeof(float);
+    b += (size_t)xrows * Kpad * sizeof(float);
+    b += (size_t)2 * kConsumerWarps * kGroupRows * BT * sizeof(float);
     b = (b + 15) & ~(size_t)15;
     b += (size_t)2 * n_stages * sizeof(uint64_t) + 16;
     return b;
 }
 
-__device__ inline StreamSmem carve_stream_smem(unsigned char* smem, int n_stages, int nb, int Kpad, int BT) {
+__device__ inline StreamSmem carve_stream_smem(unsigned char* smem, int n_stages, int xrows, int Kpad, int BT) {
     StreamSmem s;
     s.ring = smem;
     s.X = (float*)(smem + (size_t)n_stages * kStageBytes);
-    s.red = s.X + (size_t)nb * Kpad;
-    size_t off = (size_t)n_stages * kStageBytes + ((size_t)nb * Kpad + 2 * kConsumerWarps * 2 * BT) * sizeof(float);
+    s.red = s.X + (size_t)xrows * Kpad;
+    size_t off = (size_t)n_stages * kStageBytes +
+                 ((size_t)xrows * Kpad + 2 * kConsumerWarps * kGroupRows * BT) * sizeof(float);
     off = (off + 15) & ~(size_t)15;
     s.full = (uint64_t*)(smem + off);
     s.empty = s.full + n_stages;
@@ -99,10 +110,9 @@ __device__ inline void stream_init_barriers(StreamSmem& s, int n_stages) {
     __syncthreads();
 }
 
-// Producer: one thread streams the row groups [g0, g1) of W [M, K] through the ring.
+// Producer: one thread streams the row groups [g0, g1) of the tile-packed W through the ring.
 template <typename WT>
-__device__ void stream_produce(const unsigned char* W, int M, int K, int g0, int g1, StreamSmem& s, int ns,
-                               int* status) {
+__device__ void stream_produce(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int ns, int* status) {
     using G = StreamGeom<WT>;
     const int nks = (K + G::kKS - 1) / G::kKS;
     const int total = (g1 - g0) * nks;
@@ -111,47 +121,66 @@ __device__ void stream_produce(const unsigned char* W, int M, int K, int g0, int
         const int slot = it % ns;
         const uint32_t u = (uint32_t)(it / ns);
         if (!mbar_wait_abortable(&s.empty[slot], (u & 1u) ^ 1u, status, s.abort)) break;
-        const int g = g0 + it / nks;
-        const int kc = (it % nks) * G::kKS;
-        const int width = min(G::kKS, K - kc);
-        const uint32_t rowbytes = (uint32_t)width * G::kES;
-        const int rows = min(kGroupRows, M - g * kGroupRows);
-        mbar_arrive_expect_tx(&s.full[slot], (uint32_t)rows * rowbytes);
-        unsigned char* dst = s.ring + (size_t)slot * kStageBytes;
-        for (int r = 0; r < rows; ++r)
-            bulk_g2s(dst + (size_t)r * G::kKS * G::kES,
-                     W + ((int64_t)(g * kGroupRows + r) * K + kc) * G::kES, rowbytes, &s.full[slot]);
+        const int g = g0 + it / nks, ks = it % nks;
+        const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
+        mbar_arrive_expect_tx(&s.full[slot], bytes);
+        bulk_g2s(s.ring + (size_t)slot * kStageBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &s.full[slot]);
     }
     // Do not leave the CTA with copies in flight: wait for the last issued stages to land.
     for (int j = max(0, it - ns); j < it; ++j) mbar_wait(&s.full[j % ns], (uint32_t)(j / ns) & 1u, status);
 }
 
-// Sum of row r (0..3) of the group, batch column b, from one red buffer.
+// Transposing warp reduction of V = 4 * BT values per lane: afterwards lane l holds, in
+// v[0], the warp-wide sum of value index (l >> (5 - log2 V)). V - 1 + 5 - log2(V)
+// shuffles instead of 5 V.
+template <int V>
+struct WarpMultiSum {
+    template <int N, int O>
+    __device__ __forceinline__ static void step(float* v, int lane) {
+        if constexpr (N > 1) {
+            constexpr int H = N / 2;
+            const bool upper = (lane & O) != 0;
+#pragma unroll
+            for (int i = 0; i < H; ++i) {
+                const float send = upper ? v[i] : v[i + H];
+                const float keep = upper ? v[i + H] : v[i];
+                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, O);
+            }
+            step<H, O / 2>(v, lane);
+        } else {
+#pragma unroll
+            for (int o = O; o >= 1; o >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+        }
+    }
+    __device__ __forceinline__ static void run(float* v, int lane) { step<V, 16>(v, lane); }
+    static constexpr int kLog = V >= 32 ? 5 : V >= 16 ? 4 : V >= 8 ? 3 : V >= 4 ? 2 : V >= 2 ? 1 : 0;
+    // which lanes hold a result, and for which value index
+    __device__ __forceinline__ static bool owner(int lane) { return (lane & ((32 >> kLog) - 1)) == 0; }
+    __device__ __forceinline__ static int index(int lane) { return lane >> (5 - kLog); }
+};
+
+// Sum over the 8 consumer warps of partial (row r, batch column b) from one red buffer.
 template <int BT>
 __device__ __forceinline__ float group_sum(const float* red, int r, int b) {
-    const int h = r >> 1, j = r & 1;
     float v = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) v += red[((h * 4 + w) * 2 + j) * BT + b];
+    for (int w = 0; w < kConsumerWarps; ++w) v += red[w * kGroupRows * BT + r * BT + b];
     return v;
 }
 
-// One stage: 4 weight rows x `width` columns starting at column kc.
+// One stage: 4 weight rows x `width` columns (rows at stride `width`) starting at column kc.
 template <typename WT, int BT>
 __device__ __forceinline__ void stage_compute(const unsigned char* st, const float* X, int Kpad, int kc, int width,
-                                              int nb, int t, float (&acc0)[BT], float (&acc1)[BT]) {
+                                              int nb, int t, float (&acc)[kGroupRows][BT]) {
     using G = StreamGeom<WT>;
     constexpr int V = G::kVec;
-    const int half = t >> 7, cv = t & 127;
-    const unsigned char* r0 = st + (size_t)(2 * half) * G::kKS * G::kES;
-    const unsigned char* r1 = r0 + (size_t)G::kKS * G::kES;
+    const size_t rs = (size_t)width * G::kES;
     const int nv = width / V;
-    for (int v = cv; v < nv; v += 128) {
-        const uint4 a = *reinterpret_cast<const uint4*>(r0 + (size_t)v * 16);
-        const uint4 c = *reinterpret_cast<const uint4*>(r1 + (size_t)v * 16);
-        float fa[V], fc[V];
-        Vec16<WT>::widen(a, fa);
-        Vec16<WT>::widen(c, fc);
+    for (int v = t; v < nv; v += kConsumers) {
+        float f[kGroupRows][V];
+#pragma unroll
+        for (int r = 0; r < kGroupRows; ++r)
+            Vec16<WT>::widen(*reinterpret_cast<const uint4*>(st + r * rs + (size_t)v * 16), f[r]);
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
             if (b < nb) {
@@ -163,56 +192,49 @@ __device__ __forceinline__ void stage_compute(const unsigned char* st, const flo
                     xv[4 * q] = x4.x; xv[4 * q + 1] = x4.y; xv[4 * q + 2] = x4.z; xv[4 * q + 3] = x4.w;
                 }
 #pragma unroll
-                for (int j = 0; j < V; ++j) {
-                    acc0[b] = fmaf(fa[j], xv[j], acc0[b]);
-                    acc1[b] = fmaf(fc[j], xv[j], acc1[b]);
-                }
+                for (int r = 0; r < kGroupRows; ++r)
+#pragma unroll
+                    for (int j = 0; j < V; ++j) acc[r][b] = fmaf(f[r][j], xv[j], acc[r][b]);
             }
         }
     }
 }
 
-// Consumers: compute every row group of [g0, g1); after each group call
-// epi(g, red_buffer) on all 256 consumer threads (the epilogue reads group_sum()).
+// Consumers: compute every row group of [g0, g1); after each group call epi(g, red) on
+// all 256 consumer threads (the epilogue reads group_sum<BT>(red, r, b)).
 template <typename WT, int BT, typename Epi>
 __device__ void stream_consume(int K, int g0, int g1, StreamSmem& s, int ns, int Kpad, int nb, int* status, Epi& epi) {
     using G = StreamGeom<WT>;
+    using R = WarpMultiSum<kGroupRows * BT>;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int nks = (K + G::kKS - 1) / G::kKS;
     int it = 0;
     for (int g = g0; g < g1; ++g) {
-        float acc0[BT], acc1[BT];
+        float acc[kGroupRows][BT];
 #pragma unroll
-        for (int b = 0; b < BT; ++b) { acc0[b] = 0.f; acc1[b] = 0.f; }
+        for (int r = 0; r < kGroupRows; ++r)
+#pragma unroll
+            for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
         for (int ks = 0; ks < nks; ++ks, ++it) {
             const int slot = it % ns;
             const uint32_t u = (uint32_t)(it / ns);
-            const bool ok = mbar_wait_abortable(&s.full[slot], u & 1u, status, s.abort);
-            if (ok) {
+            if (mbar_wait_abortable(&s.full[slot], u & 1u, status, s.abort)) {
                 const int kc = ks * G::kKS;
-                stage_compute<WT, BT>(s.ring + (size_t)slot * kStageBytes, s.X, Kpad, kc, min(G::kKS, K - kc), nb, t,
-                                      acc0, acc1);
+                stage_compute<WT, BT>(s.ring + (size_t)slot * kStageBytes, s.X, Kpad, kc, min(G::kKS, K - kc), nb,
+                                      t, acc);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.empty[slot]);
         }
-        float* red = s.red + (size_t)((g - g0) & 1) * kConsumerWarps * 2 * BT;
-#pragma unroll
-        for (int b = 0; b < BT; ++b) {
-            const float v0 = warp_sum(acc0[b]);
-            const float v1 = warp_sum(acc1[b]);
-            if (lane == 0) {
-                red[(warp * 2 + 0) * BT + b] = v0;
-                red[(warp * 2 + 1) * BT + b] = v1;
-            }
-        }
+        float* red = s.red + (size_t)((g - g0) & 1) * kConsumerWarps * kGroupRows * BT;
+        R::run(&acc[0][0], lane);
+        if (R::owner(lane)) red[warp * kGroupRows * BT + R::index(lane)] = acc[0][0];
         named_sync(1, kConsumers);
         epi(g, red);
     }
 }
 
 // Stage activations X[b][k] (b < nb, k < K) into shared memory (see Prologue).
-
 struct ProParams {
     int pro;
     const void* x;
