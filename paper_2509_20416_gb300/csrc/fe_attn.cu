@@ -198,7 +198,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
         }
         __syncwarp();
     }
-    if (bad_page && lane == 0) atomicOr(a.status, ST_DEVICE);
+    if (bad_page) atomicOr(a.status, ST_DEVICE);  // any lane may have owned the bad key
 
     // ---- merge the warps into this split's partial per head
 #pragma unroll
