@@ -2,40 +2,34 @@
 // sequence, over that layer's own prefix K/V cache (the per-layer cache the paper's
 // vLLM study refers to, Sec. 3.2) plus the row's own key and value.
 //
-// One kernel, split-KV: work item (split s, KV head g, sequence b) covers keys
+// One kernel, split-KV. Work item (split s, KV head g, sequence b) covers keys
 // [s*split, min((s+1)*split, P_b + 1)) for the G = H / Hkv query heads sharing KV head g,
-// so each K/V row is read once for all of its query heads. Four warps take 32-key chunks:
-//   - scores: lane j owns key j of the chunk and streams its row with independent 16-byte
-//     loads (no per-key dependency chain), dotting it with the G rotated, pre-scaled
-//     queries read from shared memory (broadcast);
-//   - online softmax per head across chunks (warp max / warp sum);
-//   - P.V: lane j owns hd/32 dimensions; V rows are read coalesced, one per key.
+// so each K/V row is read once for all of its query heads.
+//   - Each of the 4 warps runs its own pipeline over 32-key chunks of the item: lane 0
+//     issues bulk TMA copies (cp.async.bulk) of the chunk's K and V rows into the warp's
+//     shared-memory slots — one copy per contiguous run of rows (the whole chunk when the
+//     cache is contiguous, one per page when it is paged) — completing on the slot's
+//     mbarrier; with two slots the next chunk streams in while the warp computes.
+//   - Scores: lane l holds dimensions l*hd/32 .. of every query head in registers, reads
+//     the same dimensions of each key row from shared memory (conflict-free), and the
+//     32 / G keys x G heads partial dots of a batch are summed across lanes with one
+//     transposing shuffle reduction (31 shuffles for 32 scores).
+//   - Online softmax per head across chunks; P.V from shared memory, lane l owning the
+//     same hd/32 dimensions of the output.
 // The warps' states merge into one partial (max, sum, accumulator) per head. The last
 // split to finish for a (sequence, KV head) — an atomic counter — merges the splits with
 // the usual max-shifted weights and writes o. The item holding key P_b also rotates the
-// new key and writes the row's key and value into cache slot P_b.
+// new key and writes the row's key and value into cache slot P_b (keys are cached after
+// RoPE); the own row is used from shared memory, unrounded.
 #include "fe_kernels.h"
 #include "fe_common.cuh"
+#include "fe_stream.cuh"
 
 namespace fe {
 
-// address of cache row `pos` of sequence b, KV head g (null if the page id is invalid)
-template <typename CT>
-__device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int g, int pos, int hd) {
-    if (a.page_table) {
-        const int pg = a.page_table[(size_t)b * a.max_pages + pos / a.page_size];
-        if (pg < 0 || pg >= a.n_pages) return nullptr;
-        return base + (((size_t)pg * a.Hkv + g) * a.page_size + pos % a.page_size) * hd;
-    }
-    return base + (((size_t)b * a.Hkv + g) * a.max_seq + pos) * hd;
-}
-
-template <typename CT>
-__device__ __forceinline__ void widen16(const uint4& v, float* f);
-template <>
-__device__ __forceinline__ void widen16<bf16_t>(const uint4& v, float* f) { Vec16<bf16_t>::widen(v, f); }
-template <>
-__device__ __forceinline__ void widen16<float>(const uint4& v, float* f) { Vec16<float>::widen(v, f); }
+constexpr int kAttnWarps = 4;
+constexpr int kChunkKeys = 32;
+constexpr int kAttnMaxSlots = 2;
 
 template <typename CT, int DPL>
 __device__ __forceinline__ void load_dims(const CT* p, float* out) {
@@ -49,31 +43,54 @@ __device__ __forceinline__ void load_dims<bf16_t, 4>(const bf16_t* p, float* out
     out[2] = __uint_as_float(v.y << 16); out[3] = __uint_as_float(v.y & 0xFFFF0000u);
 }
 template <>
+__device__ __forceinline__ void load_dims<bf16_t, 2>(const bf16_t* p, float* out) {
+    const uint32_t v = *reinterpret_cast<const uint32_t*>(p);
+    out[0] = __uint_as_float(v << 16); out[1] = __uint_as_float(v & 0xFFFF0000u);
+}
+template <>
 __device__ __forceinline__ void load_dims<float, 4>(const float* p, float* out) {
     const float4 v = *reinterpret_cast<const float4*>(p);
     out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
 }
+template <>
+__device__ __forceinline__ void load_dims<float, 2>(const float* p, float* out) {
+    const float2 v = *reinterpret_cast<const float2*>(p);
+    out[0] = v.x; out[1] = v.y;
+}
 
-constexpr int kAttnWarps = 4;
+// address of cache row `pos` of sequence b, KV head g (null if the page id is invalid)
+template <typename CT>
+__device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int g, int pos, int hd) {
+    if (a.page_table) {
+        const int pg = a.page_table[(size_t)b * a.max_pages + pos / a.page_size];
+        if (pg < 0 || pg >= a.n_pages) return nullptr;
+        return base + (((size_t)pg * a.Hkv + g) * a.page_size + pos % a.page_size) * hd;
+    }
+    return base + (((size_t)b * a.Hkv + g) * a.max_seq + pos) * hd;
+}
 
 template <typename CT, int HD, int G>
-__global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a, int S) {
     constexpr int HALF = HD / 2;
-    constexpr int DPL = HD / 32;               // dims per lane in P.V
-    constexpr int VE = 16 / sizeof(CT);        // elements per 16-byte vector
-    constexpr int NV = HD / VE;                // vectors per key row
+    constexpr int DPL = HD / 32;                  // dims per lane
+    constexpr int KB = 32 / G;                    // keys per score batch (KB * G = 32 scores)
+    constexpr int NB = kChunkKeys / KB;           // batches per chunk
+    constexpr uint32_t ROWB = HD * sizeof(CT);    // bytes per cache row
+    constexpr uint32_t CHB = kChunkKeys * ROWB;   // bytes per chunk of K (or V)
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ __align__(16) float qs[G][HD];
+    __shared__ __align__(16) float kn[HD];
+    __shared__ __align__(16) float vn[HD];
+    __shared__ float pw[kAttnWarps][kChunkKeys * G];
+    __shared__ float wm[kAttnWarps][G], wl[kAttnWarps][G];
+    __shared__ float wacc[kAttnWarps][G][HD];
+    __shared__ __align__(8) uint64_t bars[kAttnWarps][kAttnMaxSlots];
+    __shared__ int s_last, s_abort;
+
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int P = a.prefix_len[b];
     const int ldq = (a.H + 2 * a.Hkv) * HD;
-
-    __shared__ __align__(16) float qs[G][HD];
-    __shared__ __align__(16) float kn[HD];
-    __shared__ __align__(16) float vn[HD];
-    __shared__ float pw[kAttnWarps][G][32];
-    __shared__ float wm[kAttnWarps][G], wl[kAttnWarps][G];
-    __shared__ float wacc[kAttnWarps][G][HD];
-    __shared__ int s_last;
 
     float* out = a.out + (size_t)b * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
@@ -88,6 +105,60 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
     if (t0 > P) return;  // beyond this sequence's keys: not an active split
     const int t1 = min(t0 + a.split, P + 1);
     const int n_act = min(a.n_split, P / a.split + 1);
+    const int nchunks = (t1 - t0 + kChunkKeys - 1) / kChunkKeys;
+
+    unsigned char* kbuf = dsm + (size_t)warp * S * 2 * CHB;  // [S][K chunk, V chunk]
+    uint64_t* bar = bars[warp];
+    if (lane == 0) {
+        for (int i = 0; i < S; ++i) mbar_init(&bar[i], 1);
+        mbar_fence_init();
+    }
+    if (t == 0) s_abort = 0;
+
+    // Chunk j of this warp covers keys [c0, c0 + 32), c0 = t0 + (warp + 4 j) * 32; its rows
+    // below P come from the cache. Returns the mask of rows whose page id was invalid.
+    auto issue = [&](int j, int slot) -> uint32_t {
+        const int c0 = t0 + (warp + kAttnWarps * j) * kChunkKeys;
+        const int rows = max(0, min(kChunkKeys, min(t1, P) - c0));
+        unsigned char* kd = kbuf + (size_t)slot * 2 * CHB;
+        unsigned char* vd = kd + CHB;
+        uint32_t bad = 0, bytes = 0;
+        if (a.page_table) {
+            for (int p = c0; p < c0 + rows;) {
+                const int n = min(a.page_size - p % a.page_size, c0 + rows - p);
+                const CT* kr = cache_row<CT>((CT*)a.kc, a, b, g, p, HD);
+                const CT* vr = cache_row<CT>((CT*)a.vc, a, b, g, p, HD);
+                if (kr && vr) bytes += 2u * n * ROWB;
+                else bad |= (n >= 32 ? 0xffffffffu : ((1u << n) - 1u)) << (p - c0);
+                p += n;
+            }
+        } else {
+            bytes = 2u * rows * ROWB;
+        }
+        mbar_arrive_expect_tx(&bar[slot], bytes);
+        if (a.page_table) {
+            for (int p = c0; p < c0 + rows;) {
+                const int n = min(a.page_size - p % a.page_size, c0 + rows - p);
+                const CT* kr = cache_row<CT>((CT*)a.kc, a, b, g, p, HD);
+                const CT* vr = cache_row<CT>((CT*)a.vc, a, b, g, p, HD);
+                if (kr && vr) {
+                    bulk_g2s(kd + (size_t)(p - c0) * ROWB, kr, n * ROWB, &bar[slot]);
+                    bulk_g2s(vd + (size_t)(p - c0) * ROWB, vr, n * ROWB, &bar[slot]);
+                }
+                p += n;
+            }
+        } else if (rows > 0) {
+            bulk_g2s(kd, cache_row<CT>((CT*)a.kc, a, b, g, c0, HD), rows * ROWB, &bar[slot]);
+            bulk_g2s(vd, cache_row<CT>((CT*)a.vc, a, b, g, c0, HD), rows * ROWB, &bar[slot]);
+        }
+        return bad;
+    };
+    const int my_chunks = warp < nchunks ? (nchunks - warp + kAttnWarps - 1) / kAttnWarps : 0;
+    uint32_t badmask[kAttnMaxSlots] = {0u, 0u};  // per slot, meaningful on lane 0
+    int issued = 0;
+    __syncthreads();  // barriers initialised
+    if (lane == 0)
+        for (int j = 0; j < S && j < my_chunks; ++j, ++issued) badmask[j] = issue(j, j);
 
     // queries of the group, rotated at position P and pre-scaled by 1/sqrt(hd)
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
@@ -122,6 +193,11 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
     }
     __syncthreads();
 
+    float qv[G][DPL];
+#pragma unroll
+    for (int j = 0; j < G; ++j)
+#pragma unroll
+        for (int e = 0; e < DPL; ++e) qv[j][e] = qs[j][lane * DPL + e];
     float m[G], l[G], acc[G][DPL];
 #pragma unroll
     for (int j = 0; j < G; ++j) {
@@ -130,96 +206,127 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
 #pragma unroll
         for (int e = 0; e < DPL; ++e) acc[j][e] = 0.f;
     }
-    bool bad_page = false;
-    for (int base = t0 + warp * 32; base < t1; base += kAttnWarps * 32) {
-        // ---- scores: lane owns key base + lane
-        const int key = base + lane;
-        bool kval = key < t1;
-        float sc[G];
+    using R = WarpMultiSum<32>;
+    const int head = lane % G;
+    for (int j = 0; j < my_chunks; ++j) {
+        const int slot = j % S;
+        const int c0 = t0 + (warp + kAttnWarps * j) * kChunkKeys;
+        const int nk = min(kChunkKeys, t1 - c0);
+        const uint32_t bad = __shfl_sync(0xffffffffu, badmask[slot], 0);
+        if (bad && lane == 0) atomicOr(a.status, ST_DEVICE);
+        mbar_wait_abortable(&bar[slot], (uint32_t)(j / S) & 1u, a.status, &s_abort);
+        const CT* kc = (const CT*)(kbuf + (size_t)slot * 2 * CHB);
+        const CT* vc = (const CT*)(kbuf + (size_t)slot * 2 * CHB + CHB);
+        // ---- scores: batch bt holds keys bt*KB .. bt*KB + KB - 1 for all G heads; after the
+        // reduction lane l holds (key bt*KB + l / G, head l % G)
+        float sc[NB];
 #pragma unroll
-        for (int j = 0; j < G; ++j) sc[j] = 0.f;
-        if (kval) {
-            const CT* kr = nullptr;
-            if (key < P) {
-                kr = cache_row<CT>((CT*)a.kc, a, b, g, key, HD);
-                if (!kr) { kval = false; bad_page = true; }
-            }
-            if (kval) {
-#pragma unroll 4
-                for (int v = 0; v < NV; ++v) {
-                    float kk[VE];
-                    if (kr) {
-                        widen16<CT>(*reinterpret_cast<const uint4*>(kr + v * VE), kk);
-                    } else {
+        for (int bt = 0; bt < NB; ++bt) {
+            float part[32];
 #pragma unroll
-                        for (int e = 0; e < VE; ++e) kk[e] = kn[v * VE + e];
-                    }
+            for (int kk = 0; kk < KB; ++kk) {
+                const int key = bt * KB + kk;
+                float kv[DPL];
+                if (key < nk && c0 + key < P) {
+                    load_dims<CT, DPL>(kc + (size_t)key * HD + lane * DPL, kv);
+                } else {
 #pragma unroll
-                    for (int j = 0; j < G; ++j)
+                    for (int e = 0; e < DPL; ++e) kv[e] = key < nk ? kn[lane * DPL + e] : 0.f;
+                }
 #pragma unroll
-                        for (int e = 0; e < VE; ++e) sc[j] = fmaf(qs[j][v * VE + e], kk[e], sc[j]);
+                for (int hh = 0; hh < G; ++hh) {
+                    float d = 0.f;
+#pragma unroll
+                    for (int e = 0; e < DPL; ++e) d = fmaf(qv[hh][e], kv[e], d);
+                    part[kk * G + hh] = d;
                 }
             }
+            R::run(part, lane);
+            const int key = bt * KB + lane / G;
+            const bool ok = key < nk && !((bad >> key) & 1u);
+            sc[bt] = ok ? part[0] : -INFINITY;
         }
-        // ---- online softmax per head over this chunk
+        // ---- online softmax per head (lanes with lane % G == h hold head h's scores)
+        float cm = -INFINITY;
 #pragma unroll
-        for (int j = 0; j < G; ++j) {
-            const float sj = kval ? sc[j] : -INFINITY;
-            const float mn = fmaxf(m[j], warp_max(sj));
-            const float c = m[j] == -INFINITY ? 0.f : expf(m[j] - mn);
-            const float p = kval ? expf(sj - mn) : 0.f;
-            l[j] = l[j] * c + warp_sum(p);
+        for (int bt = 0; bt < NB; ++bt) cm = fmaxf(cm, sc[bt]);
 #pragma unroll
-            for (int e = 0; e < DPL; ++e) acc[j][e] *= c;
-            m[j] = mn;
-            pw[warp][j][lane] = p;
+        for (int o = 16; o >= G; o >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, o));
+        float mnew[G], corr[G];
+        float mine = 0.f;
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            const float cmh = __shfl_sync(0xffffffffu, cm, hh);
+            mnew[hh] = fmaxf(m[hh], cmh);
+            corr[hh] = m[hh] == -INFINITY ? 0.f : expf(m[hh] - mnew[hh]);
+            if (head == hh) mine = mnew[hh];
+        }
+        float csum = 0.f;
+#pragma unroll
+        for (int bt = 0; bt < NB; ++bt) {
+            const float p = sc[bt] == -INFINITY ? 0.f : expf(sc[bt] - mine);
+            csum += p;
+            pw[warp][(bt * KB + lane / G) * G + head] = p;
+        }
+#pragma unroll
+        for (int o = 16; o >= G; o >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, o);
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            l[hh] = l[hh] * corr[hh] + __shfl_sync(0xffffffffu, csum, hh);
+#pragma unroll
+            for (int e = 0; e < DPL; ++e) acc[hh][e] *= corr[hh];
+            m[hh] = mnew[hh];
         }
         __syncwarp();
-        // ---- P.V: lane owns dims lane*DPL .. lane*DPL + DPL - 1
-        const int nk = min(32, t1 - base);
-#pragma unroll 4
-        for (int kk = 0; kk < nk; ++kk) {
-            const int pos = base + kk;
+        // ---- P.V for the chunk
+        for (int key = 0; key < nk; ++key) {
+            if ((bad >> key) & 1u) continue;
             float vv[DPL];
-            if (pos < P) {
-                const CT* vr = cache_row<CT>((CT*)a.vc, a, b, g, pos, HD);
-                if (!vr) continue;
-                load_dims<CT, DPL>(vr + lane * DPL, vv);
+            if (c0 + key < P) {
+                load_dims<CT, DPL>(vc + (size_t)key * HD + lane * DPL, vv);
             } else {
 #pragma unroll
                 for (int e = 0; e < DPL; ++e) vv[e] = vn[lane * DPL + e];
             }
 #pragma unroll
-            for (int j = 0; j < G; ++j) {
-                const float p = pw[warp][j][kk];
+            for (int hh = 0; hh < G; ++hh) {
+                const float p = pw[warp][key * G + hh];
 #pragma unroll
-                for (int e = 0; e < DPL; ++e) acc[j][e] = fmaf(p, vv[e], acc[j][e]);
+                for (int e = 0; e < DPL; ++e) acc[hh][e] = fmaf(p, vv[e], acc[hh][e]);
             }
         }
         __syncwarp();
+        // refill the slot with this warp's chunk j + S
+        if (lane == 0 && j + S < my_chunks && !*(volatile int*)&s_abort) {
+            badmask[slot] = issue(j + S, slot);
+            ++issued;
+        }
+        __syncwarp();
     }
-    if (bad_page) atomicOr(a.status, ST_DEVICE);  // any lane may have owned the bad key
+    // never leave with copies in flight (only possible after an aborted wait)
+    if (lane == 0 && *(volatile int*)&s_abort)
+        for (int j = max(0, issued - S); j < issued; ++j) mbar_wait(&bar[j % S], (uint32_t)(j / S) & 1u, a.status, 100000000LL);
 
     // ---- merge the warps into this split's partial per head
 #pragma unroll
-    for (int j = 0; j < G; ++j) {
+    for (int hh = 0; hh < G; ++hh) {
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) wacc[warp][j][lane * DPL + e] = acc[j][e];
-        if (lane == 0) { wm[warp][j] = m[j]; wl[warp][j] = l[j]; }
+        for (int e = 0; e < DPL; ++e) wacc[warp][hh][lane * DPL + e] = acc[hh][e];
+        if (lane == 0) { wm[warp][hh] = m[hh]; wl[warp][hh] = l[hh]; }
     }
     __syncthreads();
     for (int idx = t; idx < G * HD; idx += blockDim.x) {
-        const int j = idx / HD, dd = idx % HD;
-        float M = wm[0][j];
-        for (int w = 1; w < kAttnWarps; ++w) M = fmaxf(M, wm[w][j]);
+        const int hh = idx / HD, dd = idx % HD;
+        float M = wm[0][hh];
+        for (int w = 1; w < kAttnWarps; ++w) M = fmaxf(M, wm[w][hh]);
         float v = 0.f, L = 0.f;
         for (int w = 0; w < kAttnWarps; ++w) {
-            if (wm[w][j] == -INFINITY) continue;
-            const float f = expf(wm[w][j] - M);
-            v = fmaf(f, wacc[w][j][dd], v);
-            L = fmaf(f, wl[w][j], L);
+            if (wm[w][hh] == -INFINITY) continue;
+            const float f = expf(wm[w][hh] - M);
+            v = fmaf(f, wacc[w][hh][dd], v);
+            L = fmaf(f, wl[w][hh], L);
         }
-        float* pp = a.part + (((size_t)b * a.H + g * G + j) * a.n_split + s) * (HD + 2);
+        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * (HD + 2);
         pp[dd] = v;
         if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
     }
@@ -231,8 +338,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
     if (!s_last) return;
     __threadfence();
     for (int idx = t; idx < G * HD; idx += blockDim.x) {
-        const int j = idx / HD, dd = idx % HD;
-        const float* pb = a.part + (((size_t)b * a.H + g * G + j) * a.n_split) * (HD + 2);
+        const int hh = idx / HD, dd = idx % HD;
+        const float* pb = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split) * (HD + 2);
         float M = -INFINITY;
         for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
         float v = 0.f, L = 0.f;
@@ -244,26 +351,38 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a)
             v = fmaf(f, __ldcg(p + dd), v);
             L = fmaf(f, __ldcg(p + HD + 1), L);
         }
-        out[(size_t)j * HD + dd] = L > 0.f ? v / L : 0.f;
+        out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
     }
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
-// Keys per work item: aim at ~4 small CTAs per SM over all (sequence, KV head) pairs, in
-// whole 32-key chunks, at least 64 keys.
+// Keys per work item: aim at ~4 CTAs per SM over all (sequence, KV head) pairs, in whole
+// chunks of 32 keys, at least 64 keys.
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev) {
     const int items = B * Hkv;
     int per = (4 * dev.num_sms + items - 1) / items;  // splits per (sequence, KV head)
     if (per < 1) per = 1;
     int split = (max_seq + per - 1) / per;
-    split = ((split + 31) / 32) * 32;
-    return split < 64 ? 64 : split;
+    split = ((split + kChunkKeys - 1) / kChunkKeys) * kChunkKeys;
+    return split < 2 * kChunkKeys ? 2 * kChunkKeys : split;
+}
+
+// Pipeline slots per warp: one when no warp has more than one chunk, else two.
+static int attn_slots(int split) { return split > kAttnWarps * kChunkKeys ? 2 : 1; }
+
+static size_t attn_smem(int hd, int es, int S) { return (size_t)kAttnWarps * S * 2 * kChunkKeys * hd * es; }
+
+template <typename CT, int HD, int G>
+static cudaError_t prepare_g() {
+    return cudaFuncSetAttribute(attn_kernel<CT, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)attn_smem(HD, sizeof(CT), kAttnMaxSlots));
 }
 
 template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
+    const int S = attn_slots(a.split);
     dim3 grid(a.n_split, a.Hkv, a.B);
-    attn_kernel<CT, HD, G><<<grid, kAttnWarps * 32, 0, st>>>(a);
+    attn_kernel<CT, HD, G><<<grid, kAttnWarps * 32, attn_smem(HD, sizeof(CT), S), st>>>(a, S);
     return cudaGetLastError();
 }
 
@@ -276,6 +395,23 @@ static cudaError_t launch_hd(const AttnArgs& a, cudaStream_t st) {
         case 8: return launch_g<CT, HD, 8>(a, st);
         default: return cudaErrorInvalidValue;
     }
+}
+
+template <typename CT, int HD>
+static cudaError_t prepare_hd() {
+    cudaError_t e;
+    if ((e = prepare_g<CT, HD, 1>()) != cudaSuccess) return e;
+    if ((e = prepare_g<CT, HD, 2>()) != cudaSuccess) return e;
+    if ((e = prepare_g<CT, HD, 4>()) != cudaSuccess) return e;
+    return prepare_g<CT, HD, 8>();
+}
+
+cudaError_t attention_prepare() {
+    cudaError_t e;
+    if ((e = prepare_hd<float, 64>()) != cudaSuccess) return e;
+    if ((e = prepare_hd<float, 128>()) != cudaSuccess) return e;
+    if ((e = prepare_hd<bf16_t, 64>()) != cudaSuccess) return e;
+    return prepare_hd<bf16_t, 128>();
 }
 
 cudaError_t launch_attention(fe_dtype dt, const AttnArgs& a, cudaStream_t st) {

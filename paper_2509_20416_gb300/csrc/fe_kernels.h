@@ -112,6 +112,7 @@ struct AttnArgs {
     int* status;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
+cudaError_t attention_prepare();
 cudaError_t launch_attention(fe_dtype dt, const AttnArgs& a, cudaStream_t st);
 inline int attention_launches() { return 1; }
 

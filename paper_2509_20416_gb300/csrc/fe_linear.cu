@@ -7,27 +7,29 @@
 
 namespace fe {
 
+template <int BT>
 struct LinearEpi {
     const LinearArgs* a;
     int b0, nb;
-    template <int BT>
-    __device__ __forceinline__ void run(int g, const float* red) const {
-        const int t = threadIdx.x;
-        if (a->epi == EPI_SWIGLU) {
-            if (t < 2 * BT) {
-                const int pr = t / BT, b = t % BT;
-                const int m = g * kGroupRows + 2 * pr;
+    __device__ __forceinline__ void chunk(int cg0, int cg1, const float* red) const {
+        const int ng = cg1 - cg0;
+        if (a->epi == EPI_SWIGLU) {  // rows (2j, 2j+1) of the packed [gate; up] matrix
+            for (int q = threadIdx.x; q < ng * 2 * BT; q += kStreamThreads) {
+                const int gl = q / (2 * BT), pr = (q / BT) % 2, b = q % BT;
+                const int m = (cg0 + gl) * kGroupRows + 2 * pr;
                 if (b < nb && m + 1 < a->M) {
-                    const float gate = group_sum<BT>(red, 2 * pr, b);
-                    const float up = group_sum<BT>(red, 2 * pr + 1, b);
+                    const float gate = chunk_value<BT>(red, gl, 2 * pr, b);
+                    const float up = chunk_value<BT>(red, gl, 2 * pr + 1, b);
                     a->y[(size_t)(b0 + b) * a->ldy + (m >> 1)] = silu(gate) * up;
                 }
             }
-        } else if (t < kGroupRows * BT) {
-            const int r = t / BT, b = t % BT;
-            const int m = g * kGroupRows + r;
+            return;
+        }
+        for (int q = threadIdx.x; q < ng * kGroupRows * BT; q += kStreamThreads) {
+            const int gl = q / (kGroupRows * BT), r = (q / BT) % kGroupRows, b = q % BT;
+            const int m = (cg0 + gl) * kGroupRows + r;
             if (b < nb && m < a->M) {
-                const float v = group_sum<BT>(red, r, b);
+                const float v = chunk_value<BT>(red, gl, r, b);
                 float* yp = a->y + (size_t)(b0 + b) * a->ldy + m;
                 if (a->epi == EPI_RESID) {
                     const float nv = *yp + v;
@@ -41,42 +43,28 @@ struct LinearEpi {
     }
 };
 
-template <int BT>
-struct EpiAdapter {
-    const LinearEpi& e;
-    __device__ __forceinline__ void operator()(int g, const float* red) const { e.template run<BT>(g, red); }
-};
-
 template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int ns) {
+__global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int D) {
     extern __shared__ __align__(128) unsigned char smem[];
     const int Kpad = (a.K + 3) & ~3;
     const int b0 = blockIdx.y * BT;
     const int nb = min(BT, a.B - b0);
-    StreamSmem s = carve_stream_smem(smem, ns, min(BT, a.B), Kpad, BT);
-    stream_init_barriers(s, ns);
-
+    StreamSmem s = carve_stream_smem(smem, D, min(BT, a.B), Kpad, BT);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     const int g0 = (int)(((int64_t)blockIdx.x * GM) / gridDim.x);
     const int g1 = (int)(((int64_t)(blockIdx.x + 1) * GM) / gridDim.x);
-
-    if (threadIdx.x >= kConsumers) {
-        if (threadIdx.x == kConsumers)
-            stream_produce<WT>((const unsigned char*)a.W, a.K, g0, g1, s, ns, a.status);
-        return;
-    }
     ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
     stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red);
-    named_sync(1, kConsumers);
-    LinearEpi e{&a, b0, nb};
-    EpiAdapter<BT> ep{e};
-    stream_consume<WT, BT>(a.K, g0, g1, s, ns, Kpad, nb, a.status, ep);
+    __syncthreads();
+    LinearEpi<BT> e{&a, b0, nb};
+    stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e);
 }
 
 // ---- host side ----------------------------------------------------------------------------
 namespace {
 
 constexpr size_t kXBudget = 128 * 1024;  // activations held in shared memory per CTA
+constexpr int kPreferredSlots = 2;       // per-warp pipeline depth (2 x 8 KB measured best)
 
 template <typename WT, int BT>
 cudaError_t set_attr(const DeviceInfo& dev) {
@@ -95,14 +83,13 @@ template <typename WT, int BT>
 cudaError_t launch_bt(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {
     const int Kpad = (a.K + 3) & ~3;
     const int xrows = BT < a.B ? BT : a.B;
-    const size_t fixed = stream_smem_bytes(0, xrows, Kpad, BT);
-    int ns = (int)(((size_t)dev.max_smem_optin - fixed) / (kStageBytes + 16));
-    ns = ns > kMaxStages ? kMaxStages : ns;
-    if (ns < 2) return cudaErrorInvalidValue;
-    const size_t smem = stream_smem_bytes(ns, xrows, Kpad, BT);
+    int D = stream_slots((size_t)dev.max_smem_optin, stream_smem_bytes(0, xrows, Kpad, BT));
+    D = D > kPreferredSlots ? kPreferredSlots : D;
+    if (D < 1) return cudaErrorInvalidValue;
+    const size_t smem = stream_smem_bytes(D, xrows, Kpad, BT);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     dim3 grid(GM < dev.num_sms ? GM : dev.num_sms, (a.B + BT - 1) / BT);
-    linear_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, ns);
+    linear_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D);
     return cudaGetLastError();
 }
 

@@ -6,10 +6,10 @@
 // of LM-head row groups) through the weight-streaming core (fe_stream.cuh) against the
 // RMSNorm'd hidden rows z_r = RMSNorm(h_r; gamma_out) of its tile of BT rows, staged once
 // in shared memory, so the LM head is read from HBM once for all N depths.
-//  - Per row group, warp 0 holds the 4 x BT new logits (one per lane), stores them in a
-//    shared-memory slab buffer, and tests them against each row's current k-th best
-//    (ties to the smaller id); the few that pass are inserted into the row's sorted
-//    top-k list one lane at a time.
+//  - Per chunk of row groups, the CTA writes the chunk's logits into a shared-memory slab
+//    buffer; warp b then tests row b's new logits against the row's current k-th best
+//    (ties to the smaller id) and inserts the few that pass into the row's sorted top-k
+//    list one lane at a time.
 //  - At the end of the slab, warp b computes row b's (max, sum of exp) of logit / T over
 //    the buffered logits and writes the slab's partial (top-k list and statistics).
 //  - The last CTA to finish a row tile (an atomic counter per tile) merges all slabs'
@@ -39,60 +39,69 @@ struct TopkState {
     int last;
 };
 
+__device__ __forceinline__ void topk_insert(TopkState* st, int b, int k, float lg, int v) {
+    const int c = st->cnt[b];
+    int pos;
+    if (c < k) {
+        pos = c;
+        st->cnt[b] = c + 1;
+    } else if (better(lg, v, st->val[b][k - 1], st->id[b][k - 1])) {
+        pos = k - 1;
+    } else {
+        return;
+    }
+    while (pos > 0 && better(lg, v, st->val[b][pos - 1], st->id[b][pos - 1])) {
+        st->val[b][pos] = st->val[b][pos - 1];
+        st->id[b][pos] = st->id[b][pos - 1];
+        --pos;
+    }
+    st->val[b][pos] = lg;
+    st->id[b][pos] = v;
+}
+
 template <int BT>
 struct LmEpi {
     const LmHeadArgs* a;
     TopkState* st;
-    float* slab;  // [BT][slab_cap]
+    float* slab;  // [BT][slab_cap] logits of this CTA's slab
     int slab_cap, b0, nb, g0;
-    __device__ __forceinline__ void operator()(int g, const float* red) const {
-        const int t = threadIdx.x;
-        if (t >= 32) return;  // warp 0 only: lane t holds candidate (row r = t / BT, z-row b = t % BT)
-        const int r = t / BT, b = t % BT;
-        const int v = g * kGroupRows + r;
-        const bool valid = t < kGroupRows * BT && b < nb && v < a->V;
-        float lg = -INFINITY;
-        if (valid) {
-            lg = group_sum<BT>(red, r, b);
-            slab[b * slab_cap + (g - g0) * kGroupRows + r] = lg;
-            if (a->dbg_logits) {
-                const int zr = b0 + b;
-                const int i = zr / a->B, sb = zr % a->B;
-                a->dbg_logits[((size_t)sb * a->N + i) * a->V + v] = lg;
-            }
-        }
-        const int k = a->top_k;
-        bool pass = false;
-        if (valid) {
-            const int c = st->cnt[b];
-            pass = c < k || better(lg, v, st->val[b][k - 1], st->id[b][k - 1]);
-        }
-        unsigned mask = __ballot_sync(0xffffffffu, pass);
-        while (mask) {
-            const int j = __ffs(mask) - 1;
-            mask &= mask - 1;
-            if (t == j) {  // insert (lg, v) into row b's sorted list
-                int c = st->cnt[b];
-                int pos;
-                if (c < k) {
-                    pos = c;
-                    st->cnt[b] = c + 1;
-                } else if (better(lg, v, st->val[b][k - 1], st->id[b][k - 1])) {
-                    pos = k - 1;
-                } else {
-                    pos = -1;
-                }
-                if (pos >= 0) {
-                    while (pos > 0 && better(lg, v, st->val[b][pos - 1], st->id[b][pos - 1])) {
-                        st->val[b][pos] = st->val[b][pos - 1];
-                        st->id[b][pos] = st->id[b][pos - 1];
-                        --pos;
-                    }
-                    st->val[b][pos] = lg;
-                    st->id[b][pos] = v;
+    __device__ void chunk(int cg0, int cg1, const float* red) const {
+        const int ng = cg1 - cg0;
+        // 1. the chunk's logits, into the slab buffer (and the optional full-logit dump)
+        for (int q = threadIdx.x; q < ng * kGroupRows * BT; q += kStreamThreads) {
+            const int gl = q / (kGroupRows * BT), r = (q / BT) % kGroupRows, b = q % BT;
+            const int v = (cg0 + gl) * kGroupRows + r;
+            if (b < nb && v < a->V) {
+                const float lg = chunk_value<BT>(red, gl, r, b);
+                slab[b * slab_cap + (cg0 - g0 + gl) * kGroupRows + r] = lg;
+                if (a->dbg_logits) {
+                    const int zr = b0 + b;
+                    const int i = zr / a->B, sb = zr % a->B;
+                    a->dbg_logits[((size_t)sb * a->N + i) * a->V + v] = lg;
                 }
             }
-            __syncwarp();
+        }
+        __syncthreads();
+        // 2. warp b updates row b's top-k with the chunk's candidates, in vocabulary order
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        if (warp < nb) {
+            const int k = a->top_k;
+            const int n = min(ng * kGroupRows, a->V - cg0 * kGroupRows);
+            const float* sb = slab + warp * slab_cap + (cg0 - g0) * kGroupRows;
+            for (int base = 0; base < n; base += 32) {
+                const int idx = base + lane;
+                const bool valid = idx < n;
+                const float lg = valid ? sb[idx] : -INFINITY;
+                const int v = cg0 * kGroupRows + idx;
+                const bool pass = valid && (st->cnt[warp] < k || better(lg, v, st->val[warp][k - 1], st->id[warp][k - 1]));
+                unsigned mask = __ballot_sync(0xffffffffu, pass);
+                while (mask) {
+                    const int j = __ffs(mask) - 1;
+                    mask &= mask - 1;
+                    if (lane == j) topk_insert(st, warp, k, lg, v);
+                    __syncwarp();
+                }
+            }
         }
     }
 };
@@ -171,7 +180,7 @@ __device__ void merge_row(const LmHeadArgs& a, int zr, float* sv, int* si, int* 
 }
 
 template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int ns, int slab_cap) {
+__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D, int slab_cap) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ TopkState st;
     const int K = a.d;
@@ -180,26 +189,21 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     const int b0 = tile * BT;
     const int nb = min(BT, a.R - b0);
     const int xrows = min(BT, a.R);
-    StreamSmem s = carve_stream_smem(smem, ns, xrows, Kpad, BT);
-    float* slab = (float*)(smem + stream_smem_bytes(ns, xrows, Kpad, BT));
+    StreamSmem s = carve_stream_smem(smem, D, xrows, Kpad, BT);
+    float* slab = (float*)(smem + stream_smem_bytes(D, xrows, Kpad, BT));
     if (threadIdx.x < kLmTile) st.cnt[threadIdx.x] = 0;
-    stream_init_barriers(s, ns);
 
     const int GM = (a.V + kGroupRows - 1) / kGroupRows;
     const int sl = blockIdx.x;
     const int g0 = (int)(((int64_t)sl * GM) / gridDim.x);
     const int g1 = (int)(((int64_t)(sl + 1) * GM) / gridDim.x);
 
-    if (threadIdx.x >= kConsumers) {
-        if (threadIdx.x == kConsumers) stream_produce<WT>((const unsigned char*)a.W, K, g0, g1, s, ns, a.status);
-        return;
-    }
     ProParams pp{PRO_RMSNORM, a.hid, a.d, a.gamma, a.eps, nullptr, nullptr, 0, 0};
     stage_activations<WT>(pp, K, s.X, Kpad, b0, nb, a.status, s.red);
-    named_sync(1, kConsumers);
+    __syncthreads();
     LmEpi<BT> ep{&a, &st, slab, slab_cap, b0, nb, g0};
-    stream_consume<WT, BT>(K, g0, g1, s, ns, Kpad, nb, a.status, ep);
-    named_sync(1, kConsumers);
+    stream_run<WT, BT>((const unsigned char*)a.W, K, g0, g1, s, D, Kpad, nb, a.status, ep);
+    __syncthreads();
 
     // this slab's partial for each row of the tile (warp b <-> row b)
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
@@ -226,16 +230,16 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     }
     // the last slab CTA of this tile merges the tile's rows
     __threadfence();
-    named_sync(1, kConsumers);
+    __syncthreads();
     if (t == 0) st.last = atomicAdd(&a.counters[tile], 1) == (int)gridDim.x - 1;
-    named_sync(1, kConsumers);
+    __syncthreads();
     if (!st.last) return;
     __threadfence();
     // shared memory of the finished stream is reused: per warp kMergeCap values, ids, a
     // counter and a taken-bitmap sized for the overflow fallback
     const int bitmap_words = (a.n_slabs * a.top_k + 31) / 32;
-    unsigned char* base = smem + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
-    float* sv = (float*)base;
+    unsigned char* mbase = smem + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
+    float* sv = (float*)mbase;
     int* si = (int*)(sv + kMergeCap);
     int* scount = si + kMergeCap;
     unsigned* taken = (unsigned*)(scount + 4);
@@ -246,6 +250,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
 // ---- host side ----------------------------------------------------------------------------
 namespace {
 constexpr size_t kXBudget = 128 * 1024;
+constexpr int kPreferredSlots = 2;
 constexpr size_t kStaticReserve = sizeof(TopkState) + 256;
 
 int pick_bt(int R, int K) {
@@ -270,16 +275,14 @@ cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t s
     const size_t budget = (size_t)dev.max_smem_optin - kStaticReserve;
     const size_t extra = (size_t)xrows * slab_cap * sizeof(float);
     const size_t merge = (size_t)kLmTile * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
-    const size_t fixed = stream_smem_bytes(0, xrows, Kpad, BT) + extra;
-    if (fixed >= budget) return cudaErrorInvalidValue;
-    int ns = (int)((budget - fixed) / (kStageBytes + 16));
-    ns = ns > kMaxStages ? kMaxStages : ns;
-    if (ns < 2) return cudaErrorInvalidValue;
-    size_t smem = stream_smem_bytes(ns, xrows, Kpad, BT) + extra;
+    int D = stream_slots(budget, stream_smem_bytes(0, xrows, Kpad, BT) + extra);
+    D = D > kPreferredSlots ? kPreferredSlots : D;
+    if (D < 1) return cudaErrorInvalidValue;
+    size_t smem = stream_smem_bytes(D, xrows, Kpad, BT) + extra;
     if (smem < merge) smem = merge;
     if (smem > budget) return cudaErrorInvalidValue;
     dim3 grid(a.n_slabs, (a.R + BT - 1) / BT);
-    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, ns, slab_cap);
+    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D, slab_cap);
     return cudaGetLastError();
 }
 

@@ -30,7 +30,7 @@ size_t packed_bytes(int M, int K, int es) {
 
 cudaError_t launch_pack_tiles(const void* src, void* dst, int M, int K, int es, cudaStream_t st) {
     const int Kv = K * es / 16;
-    const int KSv = kStageBytes / (kGroupRows * 16);  // 16-byte vectors per row of a full slice
+    const int KSv = kTileBytes / (kGroupRows * 16);  // 16-byte vectors per row of a full slice
     const int64_t total = (int64_t)packed_bytes(M, K, es) / 16;
     const int blocks = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
     pack_tiles_kernel<<<blocks, 256, 0, st>>>((const uint4*)src, (uint4*)dst, M, Kv, KSv, total);

@@ -261,6 +261,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             break;
         if ((rc = from_cuda(linear_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(lmhead_prepare(h->dev))) != FE_OK) break;
+        if ((rc = from_cuda(attention_prepare())) != FE_OK) break;
 
         // ---- packed weights: one allocation, every matrix 256-byte aligned ----
         const Sizes sz = weight_sizes(c, h->es);
