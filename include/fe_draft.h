@@ -171,6 +171,11 @@ FE_API void fe_free(fe_handle *h);
 /* A static, human-readable name of a status code. */
 FE_API const char *fe_status_str(fe_status s);
 
+/* The calling thread's description of the last failing CUDA call inside the library
+ * (which call, where, and CUDA's error string); "" if none. Valid until the thread's next
+ * failing call. */
+FE_API const char *fe_last_error_detail(void);
+
 /* Number of kernels fe_draft_forward (plus fe_build_tree when with_tree != 0) launches for
  * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
 FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);

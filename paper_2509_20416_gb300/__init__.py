@@ -76,12 +76,19 @@ _lib.fe_launch_count.argtypes = [_vp, _i32, _i32]
 _lib.fe_launch_count.restype = _i32
 _lib.fe_selftest_timeout.argtypes = [_vp, ctypes.c_int64, _vp]
 _lib.fe_selftest_timeout.restype = ctypes.c_int
+_lib.fe_last_error_detail.argtypes = []
+_lib.fe_last_error_detail.restype = ctypes.c_char_p
 
 
 class FeError(RuntimeError):
     def __init__(self, code: int, where: str):
-        super().__init__(f"{where}: {fe_status_str(code)} ({code})")
+        detail = fe_last_error_detail() if code in (FE_ERR_CUDA, FE_ERR_OOM) else ""
+        super().__init__(f"{where}: {fe_status_str(code)} ({code})" + (f" [{detail}]" if detail else ""))
         self.code = code
+
+
+def fe_last_error_detail() -> str:
+    return _lib.fe_last_error_detail().decode()
 
 
 def fe_status_str(code: int) -> str:

@@ -367,20 +367,24 @@ int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev) {
     return split < 2 * kChunkKeys ? 2 * kChunkKeys : split;
 }
 
-// Pipeline slots per warp: one when no warp has more than one chunk, else two.
-static int attn_slots(int split) { return split > kAttnWarps * kChunkKeys ? 2 : 1; }
+// Pipeline slots per warp: two when a warp has more than one chunk and a chunk of K (or
+// V) is at most 8 KB (bf16, hd 128), else one; at most 128 KB of dynamic shared memory.
+static int max_slots(int hd, int es) { return kChunkKeys * hd * es <= 8192 ? kAttnMaxSlots : 1; }
+static int attn_slots(int split, int hd, int es) {
+    return split > kAttnWarps * kChunkKeys ? max_slots(hd, es) : 1;
+}
 
 static size_t attn_smem(int hd, int es, int S) { return (size_t)kAttnWarps * S * 2 * kChunkKeys * hd * es; }
 
 template <typename CT, int HD, int G>
 static cudaError_t prepare_g() {
     return cudaFuncSetAttribute(attn_kernel<CT, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)attn_smem(HD, sizeof(CT), kAttnMaxSlots));
+                                (int)attn_smem(HD, sizeof(CT), max_slots(HD, sizeof(CT))));
 }
 
 template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
-    const int S = attn_slots(a.split);
+    const int S = attn_slots(a.split, HD, sizeof(CT));
     dim3 grid(a.n_split, a.Hkv, a.B);
     attn_kernel<CT, HD, G><<<grid, kAttnWarps * 32, attn_smem(HD, sizeof(CT), S), st>>>(a, S);
     return cudaGetLastError();

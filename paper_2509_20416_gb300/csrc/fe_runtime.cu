@@ -16,6 +16,7 @@
 // The sequence is captured once per distinct argument set into a CUDA graph on an
 // internal stream and replayed on the caller's stream.
 #include <math.h>
+#include <stdio.h>
 #include <string.h>
 
 #include <algorithm>
@@ -76,16 +77,20 @@ namespace {
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-fe_status from_cuda(cudaError_t e) {
-    if (e == cudaSuccess) return FE_OK;
+thread_local char g_detail[256] = "";
+
+fe_status fail(cudaError_t e, const char* what, int line) {
+    snprintf(g_detail, sizeof(g_detail), "%s (fe_runtime.cu:%d): %s", what, line, cudaGetErrorString(e));
     if (e == cudaErrorMemoryAllocation) return FE_ERR_OOM;
     return FE_ERR_CUDA;
 }
 
-#define FE_TRY(call)                                  \
-    do {                                              \
-        cudaError_t _e = (call);                      \
-        if (_e != cudaSuccess) return from_cuda(_e);  \
+#define from_cuda(call) (((_fe_e = (call)) == cudaSuccess) ? FE_OK : fail(_fe_e, #call, __LINE__))
+
+#define FE_TRY(call)                                       \
+    do {                                                   \
+        cudaError_t _e = (call);                           \
+        if (_e != cudaSuccess) return fail(_e, #call, __LINE__); \
     } while (0)
 
 bool valid_config(const fe_config* c) {
@@ -245,6 +250,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
 
     fe_handle* h = new (std::nothrow) fe_handle();
     if (!h) return FE_ERR_OOM;
+    cudaError_t _fe_e = cudaSuccess;
     h->cfg = *cfg;
     const char* g = getenv("FE_DRAFT_GRAPH");
     h->use_graph = !(g && g[0] == '0');
@@ -281,15 +287,16 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         auto put = [&](const void* src, size_t bytes) -> const void* {
             void* dst = p;
             p += align256(bytes);
-            if (cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, st) != cudaSuccess) rc = FE_ERR_CUDA;
+            if ((_fe_e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, st)) != cudaSuccess)
+                rc = fail(_fe_e, "copy of a weight", __LINE__);
             return dst;
         };
         auto put_packed = [&](const void* src, int M, int K) -> const void* {
             void* dst = p;
             p += align256(packed_bytes(M, K, es));
-            if (cudaMemcpyAsync(staging, src, (size_t)M * K * es, cudaMemcpyDefault, st) != cudaSuccess ||
-                launch_pack_tiles(staging, dst, M, K, es, st) != cudaSuccess)
-                rc = FE_ERR_CUDA;
+            if ((_fe_e = cudaMemcpyAsync(staging, src, (size_t)M * K * es, cudaMemcpyDefault, st)) != cudaSuccess ||
+                (_fe_e = launch_pack_tiles(staging, dst, M, K, es, st)) != cudaSuccess)
+                rc = fail(_fe_e, "copy or packing of a weight matrix", __LINE__);
             return dst;
         };
         const int dm = c.d, nq = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim, hq = c.n_heads * c.head_dim;
@@ -315,7 +322,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                 cudaMemcpy2DAsync((char*)staging + rowb, 2 * rowb, L.w_up, rowb, rowb, c.ffn, cudaMemcpyDefault,
                                   st) != cudaSuccess ||
                 launch_pack_tiles(staging, gu, 2 * c.ffn, dm, es, st) != cudaSuccess)
-                rc = FE_ERR_CUDA;
+                rc = fail(cudaGetLastError(), "interleave or packing of gate/up", __LINE__);
             P.w_gu = gu;
             P.w_down = put_packed(L.w_down, dm, c.ffn);
         }
@@ -458,6 +465,8 @@ void fe_free(fe_handle* h) {
     cudaDeviceSynchronize();
     release(h);
 }
+
+const char* fe_last_error_detail(void) { return g_detail; }
 
 int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     if (!h || B < 1) return -1;
