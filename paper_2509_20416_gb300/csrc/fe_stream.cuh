@@ -225,7 +225,9 @@ __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, Strea
 #pragma unroll
                 for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
         }
-        while (g >= chunk_end && chunk_end - kChunk < g1) {  // every warp passes every chunk boundary once
+        // every warp passes every chunk boundary once: when its next group lies beyond the
+        // chunk, or (for the last, possibly partial, chunks) when its items are exhausted
+        while ((g >= chunk_end || i >= total) && chunk_end - kChunk < g1) {
             __syncthreads();
             epi.chunk(chunk_end - kChunk, min(chunk_end, g1), s.red);
             __syncthreads();
