@@ -6,12 +6,12 @@
 // of LM-head row groups) through the weight-streaming core (fe_stream.cuh) against the
 // RMSNorm'd hidden rows z_r = RMSNorm(h_r; gamma_out) of its tile of BT rows, staged once
 // in shared memory, so the LM head is read from HBM once for all N depths.
-//  - Per chunk of row groups, the CTA writes the chunk's logits into a shared-memory slab
-//    buffer; warp b then tests row b's new logits against the row's current k-th best
-//    (ties to the smaller id) and inserts the few that pass into the row's sorted top-k
-//    list one lane at a time.
-//  - At the end of the slab, warp b computes row b's (max, sum of exp) of logit / T over
-//    the buffered logits and writes the slab's partial (top-k list and statistics).
+//  - Per chunk of row groups, the CTA writes the chunk's logits into a small shared-memory
+//    buffer; warp b then folds row b's new logits into per-lane running (max, sum of exp)
+//    of logit / T, tests them against the row's current k-th best (ties to the smaller
+//    id) and inserts the few that pass into the row's sorted top-k list, one lane at a time.
+//  - At the end of the slab, warp b reduces row b's per-lane statistics and writes the
+//    slab's partial (top-k list and statistics).
 //  - The last CTA to finish a row tile (an atomic counter per tile) merges all slabs'
 //    partials: lse = M + log sum_j s_j e^(m_j - M); the global top-k is taken from the
 //    candidates not below tau = max over slabs of the slab's k-th value (a slab holds k
@@ -63,17 +63,19 @@ template <int BT>
 struct LmEpi {
     const LmHeadArgs* a;
     TopkState* st;
-    float* slab;  // [BT][slab_cap] logits of this CTA's slab
-    int slab_cap, b0, nb, g0;
-    __device__ void chunk(int cg0, int cg1, const float* red) const {
+    float* cbuf;  // [BT][chunk_groups(BT) * 4] logits of the current chunk
+    int b0, nb;
+    float m = -INFINITY, sum = 0.f;  // this lane's running statistics of its warp's row
+    __device__ void chunk(int cg0, int cg1, const float* red) {
+        constexpr int CW = chunk_groups(BT) * kGroupRows;
         const int ng = cg1 - cg0;
-        // 1. the chunk's logits, into the slab buffer (and the optional full-logit dump)
+        // 1. the chunk's logits, into the chunk buffer (and the optional full-logit dump)
         for (int q = threadIdx.x; q < ng * kGroupRows * BT; q += kStreamThreads) {
             const int gl = q / (kGroupRows * BT), r = (q / BT) % kGroupRows, b = q % BT;
             const int v = (cg0 + gl) * kGroupRows + r;
             if (b < nb && v < a->V) {
                 const float lg = chunk_value<BT>(red, gl, r, b);
-                slab[b * slab_cap + (cg0 - g0 + gl) * kGroupRows + r] = lg;
+                cbuf[b * CW + gl * kGroupRows + r] = lg;
                 if (a->dbg_logits) {
                     const int zr = b0 + b;
                     const int i = zr / a->B, sb = zr % a->B;
@@ -82,18 +84,28 @@ struct LmEpi {
             }
         }
         __syncthreads();
-        // 2. warp b updates row b's top-k with the chunk's candidates, in vocabulary order
+        // 2. warp b folds row b's candidates into its statistics and top-k, in vocabulary order
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
         if (warp < nb) {
             const int k = a->top_k;
             const int n = min(ng * kGroupRows, a->V - cg0 * kGroupRows);
-            const float* sb = slab + warp * slab_cap + (cg0 - g0) * kGroupRows;
+            const float* sb = cbuf + warp * CW;
             for (int base = 0; base < n; base += 32) {
                 const int idx = base + lane;
                 const bool valid = idx < n;
                 const float lg = valid ? sb[idx] : -INFINITY;
+                if (valid) {
+                    const float lt = lg * a->inv_temp;
+                    if (lt > m) {
+                        sum = sum * expf(m - lt) + 1.0f;
+                        m = lt;
+                    } else {
+                        sum += expf(lt - m);
+                    }
+                }
                 const int v = cg0 * kGroupRows + idx;
-                const bool pass = valid && (st->cnt[warp] < k || better(lg, v, st->val[warp][k - 1], st->id[warp][k - 1]));
+                const bool pass =
+                    valid && (st->cnt[warp] < k || better(lg, v, st->val[warp][k - 1], st->id[warp][k - 1]));
                 unsigned mask = __ballot_sync(0xffffffffu, pass);
                 while (mask) {
                     const int j = __ffs(mask) - 1;
@@ -180,7 +192,7 @@ __device__ void merge_row(const LmHeadArgs& a, int zr, float* sv, int* si, int* 
 }
 
 template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D, int slab_cap) {
+__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ TopkState st;
     const int K = a.d;
@@ -190,7 +202,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     const int nb = min(BT, a.R - b0);
     const int xrows = min(BT, a.R);
     StreamSmem s = carve_stream_smem(smem, D, xrows, Kpad, BT);
-    float* slab = (float*)(smem + stream_smem_bytes(D, xrows, Kpad, BT));
+    __shared__ float cbuf[kLmTile * 32 * kGroupRows / 4 * 4];  // >= BT * chunk_groups(BT) * 4
+    static_assert(BT * chunk_groups(BT) * kGroupRows <= kLmTile * 32 * kGroupRows / 4 * 4, "chunk buffer");
     if (threadIdx.x < kLmTile) st.cnt[threadIdx.x] = 0;
 
     const int GM = (a.V + kGroupRows - 1) / kGroupRows;
@@ -201,21 +214,16 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     ProParams pp{PRO_RMSNORM, a.hid, a.d, a.gamma, a.eps, nullptr, nullptr, 0, 0};
     stage_activations<WT>(pp, K, s.X, Kpad, b0, nb, a.status, s.red);
     __syncthreads();
-    LmEpi<BT> ep{&a, &st, slab, slab_cap, b0, nb, g0};
+    LmEpi<BT> ep{&a, &st, cbuf, b0, nb};
     stream_run<WT, BT>((const unsigned char*)a.W, K, g0, g1, s, D, Kpad, nb, a.status, ep);
     __syncthreads();
 
     // this slab's partial for each row of the tile (warp b <-> row b)
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int nrows = min((g1 - g0) * kGroupRows, a.V - g0 * kGroupRows);
     if (warp < nb) {
         const int zr = b0 + warp;
-        const float* sb = slab + warp * slab_cap;
-        float m = -INFINITY;
-        for (int j = lane; j < nrows; j += 32) m = fmaxf(m, sb[j] * a.inv_temp);
-        m = warp_max(m);
-        float sum = 0.f;
-        for (int j = lane; j < nrows; j += 32) sum += expf(sb[j] * a.inv_temp - m);
+        const float m = warp_max(ep.m);
+        float sum = ep.m == -INFINITY ? 0.f : ep.sum * expf(ep.m - m);
         sum = warp_sum(sum);
         const size_t base = (size_t)zr * a.n_slabs + sl;
         for (int j = lane; j < a.top_k; j += 32) {
@@ -251,7 +259,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
 namespace {
 constexpr size_t kXBudget = 128 * 1024;
 constexpr int kPreferredSlots = 2;
-constexpr size_t kStaticReserve = sizeof(TopkState) + 256;
+constexpr size_t kStaticReserve = sizeof(TopkState) + kLmTile * 32 * kGroupRows * sizeof(float) + 256;
 
 int pick_bt(int R, int K) {
     const size_t row = (size_t)((K + 3) & ~3) * sizeof(float);
@@ -270,19 +278,16 @@ template <typename WT, int BT>
 cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st) {
     const int Kpad = (a.d + 3) & ~3;
     const int xrows = BT < a.R ? BT : a.R;
-    const int GM = (a.V + kGroupRows - 1) / kGroupRows;
-    const int slab_cap = ((GM + a.n_slabs - 1) / a.n_slabs) * kGroupRows;
     const size_t budget = (size_t)dev.max_smem_optin - kStaticReserve;
-    const size_t extra = (size_t)xrows * slab_cap * sizeof(float);
     const size_t merge = (size_t)kLmTile * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
-    int D = stream_slots(budget, stream_smem_bytes(0, xrows, Kpad, BT) + extra);
+    int D = stream_slots(budget, stream_smem_bytes(0, xrows, Kpad, BT));
     D = D > kPreferredSlots ? kPreferredSlots : D;
     if (D < 1) return cudaErrorInvalidValue;
-    size_t smem = stream_smem_bytes(D, xrows, Kpad, BT) + extra;
+    size_t smem = stream_smem_bytes(D, xrows, Kpad, BT);
     if (smem < merge) smem = merge;
     if (smem > budget) return cudaErrorInvalidValue;
     dim3 grid(a.n_slabs, (a.R + BT - 1) / BT);
-    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D, slab_cap);
+    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D);
     return cudaGetLastError();
 }
 

@@ -39,7 +39,11 @@ constexpr int kWarps = 8;
 constexpr int kStreamThreads = kWarps * 32;  // 256
 constexpr int kGroupRows = 4;                // weight rows per group
 constexpr int kTileBytes = 8192;             // 4 rows x 2 KB
-constexpr int kChunk = 32;                   // row groups per epilogue round
+constexpr int kChunk = 32;                   // row groups per epilogue round (BT <= 2)
+
+// Row groups per epilogue round for BT activation rows: the per-warp partial sums of a
+// chunk take kWarps * 4 * BT floats per group, so larger BT gets shorter chunks.
+__host__ __device__ constexpr int chunk_groups(int BT) { return BT >= 8 ? 8 : BT >= 4 ? 16 : kChunk; }
 constexpr int kMaxSlots = 3;                 // pipeline depth per warp
 
 template <typename WT>
@@ -58,7 +62,7 @@ __host__ __device__ __forceinline__ int64_t tile_offset(int g, int s, int K) {
 struct StreamSmem {
     unsigned char* ring;  // [kWarps][D][kTileBytes] (128-byte aligned)
     float* X;             // [xrows][Kpad] activations
-    float* red;           // [kChunk][kWarps][4 * BT] per-warp partial sums of the current chunk
+    float* red;           // [chunk_groups(BT)][kWarps][4 * BT] per-warp partial sums of the current chunk
     uint64_t* full;       // [kWarps][D]
     int* abort;           // set when any wait of this CTA gave up
 };
@@ -67,7 +71,7 @@ struct StreamSmem {
 __host__ __device__ inline size_t stream_smem_bytes(int D, int xrows, int Kpad, int BT) {
     size_t b = (size_t)kWarps * D * kTileBytes;
     b += (size_t)xrows * Kpad * sizeof(float);
-    b += (size_t)kChunk * kWarps * kGroupRows * BT * sizeof(float);
+    b += (size_t)chunk_groups(BT) * kWarps * kGroupRows * BT * sizeof(float);
     b = (b + 15) & ~(size_t)15;
     b += (size_t)kWarps * D * sizeof(uint64_t) + 16;
     return b;
@@ -79,7 +83,7 @@ __device__ inline StreamSmem carve_stream_smem(unsigned char* smem, int D, int x
     s.X = (float*)(smem + (size_t)kWarps * D * kTileBytes);
     s.red = s.X + (size_t)xrows * Kpad;
     size_t off = (size_t)kWarps * D * kTileBytes +
-                 ((size_t)xrows * Kpad + (size_t)kChunk * kWarps * kGroupRows * BT) * sizeof(float);
+                 ((size_t)xrows * Kpad + (size_t)chunk_groups(BT) * kWarps * kGroupRows * BT) * sizeof(float);
     off = (off + 15) & ~(size_t)15;
     s.full = (uint64_t*)(smem + off);
     s.abort = (int*)(s.full + kWarps * D);
@@ -183,13 +187,14 @@ __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, Strea
     using G = StreamGeom<WT>;
     using R = WarpMultiSum<kGroupRows * BT>;
     constexpr int RV = kGroupRows * BT;
+    constexpr int CH = chunk_groups(BT);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nks = (K + G::kKS - 1) / G::kKS;
     const int total = (g1 - g0) * nks;
     uint64_t* full = s.full + warp * D;
     unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
 
-    for (int i = threadIdx.x; i < kChunk * kWarps * RV; i += kStreamThreads) s.red[i] = 0.f;
+    for (int i = threadIdx.x; i < CH * kWarps * RV; i += kStreamThreads) s.red[i] = 0.f;
     if (lane == 0) {
         for (int d = 0; d < D; ++d) mbar_init(&full[d], 1);
         if (warp == 0) *s.abort = 0;
@@ -213,13 +218,13 @@ __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, Strea
 #pragma unroll
         for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
     int cur_g = -1;
-    int chunk_end = g0 + kChunk;
+    int chunk_end = g0 + CH;
     for (int j = 0;; ++j) {
         const int i = warp + kWarps * j;
         const int g = i < total ? g0 + i / nks : g1;
         if (g != cur_g && cur_g >= 0) {  // leaving a group: fold this warp's partials into the chunk buffer
             R::run(&acc[0][0], lane);
-            if (R::owner(lane)) s.red[((size_t)(cur_g - chunk_end + kChunk) * kWarps + warp) * RV + R::index(lane)] += acc[0][0];
+            if (R::owner(lane)) s.red[((size_t)(cur_g - chunk_end + CH) * kWarps + warp) * RV + R::index(lane)] += acc[0][0];
 #pragma unroll
             for (int r = 0; r < kGroupRows; ++r)
 #pragma unroll
@@ -227,13 +232,13 @@ __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, Strea
         }
         // every warp passes every chunk boundary once: when its next group lies beyond the
         // chunk, or (for the last, possibly partial, chunks) when its items are exhausted
-        while ((g >= chunk_end || i >= total) && chunk_end - kChunk < g1) {
+        while ((g >= chunk_end || i >= total) && chunk_end - CH < g1) {
             __syncthreads();
-            epi.chunk(chunk_end - kChunk, min(chunk_end, g1), s.red);
+            epi.chunk(chunk_end - CH, min(chunk_end, g1), s.red);
             __syncthreads();
-            for (int q = threadIdx.x; q < kChunk * kWarps * RV; q += kStreamThreads) s.red[q] = 0.f;
+            for (int q = threadIdx.x; q < CH * kWarps * RV; q += kStreamThreads) s.red[q] = 0.f;
             __syncthreads();
-            chunk_end += kChunk;
+            chunk_end += CH;
         }
         if (i >= total) break;
         cur_g = g;
