@@ -95,6 +95,15 @@ int lmhead_slabs(int V, const DeviceInfo& dev);
 int lmhead_launches(int R, int d, const DeviceInfo& dev);
 cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st);
 
+// tensor-core LM head (bf16 storage, N*B <= 16 rows, d % 64 == 0): W in the swizzled MMA
+// layout (launch_pack_mma), zb scratch of lmhead_mma_zb_bytes(); n_slabs = CTAs
+bool lmhead_mma_ok(const LmHeadArgs& a);
+size_t lmhead_mma_zb_bytes(int R, int d);
+size_t mma_packed_bytes(int M, int K);
+cudaError_t launch_pack_mma(const void* src, void* dst, int M, int K, cudaStream_t st);
+cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);
+cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st);
+
 // ---- decode attention ----------------------------------------------------------------
 struct AttnArgs {
     const float* qkv;  // [B, (H + 2 Hkv) hd] float32, before RoPE

@@ -21,6 +21,7 @@
 
 #include "fe_kernels.h"
 #include "fe_stream.cuh"
+#include "fe_tc.cuh"
 
 namespace fe {
 
@@ -255,6 +256,272 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     if (t == 0) a.counters[tile] = 0;
 }
 
+// ---- tensor-core LM head (bf16 storage, up to kMmaMaxRows hidden rows) --------------------
+//
+// z_r = RMSNorm(h_r; gamma_out) is split into z_hi = bf16(z) and z_lo = bf16(z - z_hi)
+// (zprep_kernel), so W_lm z = W_lm z_hi + W_lm z_lo keeps ~16 more bits than one bf16
+// rounding of z; both halves are the B operand [2 R_pad rows x d] of one M=128 x N=2 R_pad
+// tcgen05.mma per 16 columns, accumulating in float32 in TMEM. Warp roles: warp 4 streams
+// 16 KB weight blocks (and the matching B blocks) with bulk TMA copies into a ring of
+// stages; warp 5 (one thread) issues the MMAs and commits each stage back to its producer;
+// warps 0..3 read the double-buffered accumulator from TMEM (TMEM lane = vocabulary row)
+// and keep per-warp softmax statistics and top-k lists, merged per slab at the end.
+constexpr int kMmaMaxRows = 16;
+constexpr int kMmaThreads = 6 * 32;
+constexpr int kMmaMaxStages = 12;
+
+// zb [d/64][N rows x 128 B] in the 128B-swizzled layout: rows [0, R_pad) hold z_hi, rows
+// [R_pad, 2 R_pad) hold z_lo; rows of padding (r >= R) are zero. One CTA per row r < R_pad.
+template <typename WT>
+__global__ void __launch_bounds__(256) zprep_kernel(const float* __restrict__ hid, const WT* __restrict__ gamma, int R,
+                                                    int R_pad, int d, float eps, uint16_t* __restrict__ zb) {
+    const int r = blockIdx.x, t = threadIdx.x;
+    const int N = 2 * R_pad;
+    __shared__ float red[8];
+    float rs = 0.f;
+    if (r < R) {
+        float ss = 0.f;
+        for (int k = t; k < d; k += 256) {
+            const float v = hid[(size_t)r * d + k];
+            ss = fmaf(v, v, ss);
+        }
+        ss = warp_sum(ss);
+        if ((t & 31) == 0) red[t >> 5] = ss;
+        __syncthreads();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        rs = 1.0f / sqrtf(tot / (float)d + eps);
+    }
+    for (int k = t; k < d; k += 256) {
+        uint16_t hi = 0, lo = 0;
+        if (r < R) {
+            const float z = hid[(size_t)r * d + k] * rs * Storage<WT>::load(gamma, k);
+            hi = f32_to_bf16(z);
+            lo = f32_to_bf16(z - bf16_to_f32(hi));
+        }
+        const int kb = k / 64, c = (k % 64) / 8, e = k % 8;
+        unsigned char* blk = (unsigned char*)zb + (size_t)kb * N * 128;
+        *(uint16_t*)(blk + sw128_offset(r, c) + e * 2) = hi;
+        *(uint16_t*)(blk + sw128_offset(R_pad + r, c) + e * 2) = lo;
+    }
+}
+
+struct MmaState {
+    float m[4][kMmaMaxRows], s[4][kMmaMaxRows];
+    int cnt[4][kMmaMaxRows];
+    int id[4][kMmaMaxRows][kMaxTopK];
+    float val[4][kMmaMaxRows][kMaxTopK];
+    uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2];
+    uint32_t tmem_base;
+    int last, abort;
+};
+
+__device__ __forceinline__ void warp_list_insert(MmaState& st, int w, int r, int k, float lg, int v) {
+    const int c = st.cnt[w][r];
+    int pos;
+    if (c < k) {
+        pos = c;
+        st.cnt[w][r] = c + 1;
+    } else if (better(lg, v, st.val[w][r][k - 1], st.id[w][r][k - 1])) {
+        pos = k - 1;
+    } else {
+        return;
+    }
+    while (pos > 0 && better(lg, v, st.val[w][r][pos - 1], st.id[w][r][pos - 1])) {
+        st.val[w][r][pos] = st.val[w][r][pos - 1];
+        st.id[w][r][pos] = st.id[w][r][pos - 1];
+        --pos;
+    }
+    st.val[w][r][pos] = lg;
+    st.id[w][r][pos] = v;
+}
+
+__global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
+                                                                    int S, int stage_bytes, uint32_t tmem_cols) {
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ MmaState st;
+    // 1024-byte aligned ring (the 128B swizzle pattern is a function of address bits 4..9)
+    unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int N = 2 * R_pad, R = a.R, k = a.top_k;
+    const int nkb = a.d / 64;
+    const int ntiles = (a.V + 127) / 128;
+    const int t0 = (int)(((int64_t)blockIdx.x * ntiles) / gridDim.x);
+    const int t1 = (int)(((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x);
+
+    if (t == 0) {
+        for (int i = 0; i < S; ++i) {
+            mbar_init(&st.full[i], 1);
+            mbar_init(&st.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&st.tfull[i], 1);
+            mbar_init(&st.tempty[i], 4);
+        }
+        st.abort = 0;
+        mbar_fence_init();
+    }
+    for (int i = t; i < 4 * kMmaMaxRows; i += blockDim.x) {
+        st.m[i / kMmaMaxRows][i % kMmaMaxRows] = -INFINITY;
+        st.s[i / kMmaMaxRows][i % kMmaMaxRows] = 0.f;
+        st.cnt[i / kMmaMaxRows][i % kMmaMaxRows] = 0;
+    }
+    if (warp == 0) tc_alloc(&st.tmem_base, tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = st.tmem_base;
+
+    if (warp == 4) {  // ---- TMA producer
+        if (lane == 0) {
+            int it = 0;
+            for (int tile = t0; tile < t1; ++tile)
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int slot = it % S;
+                    const uint32_t u = (uint32_t)(it / S);
+                    if (!mbar_wait_abortable(&st.empty[slot], (u & 1u) ^ 1u, a.status, &st.abort)) goto producer_done;
+                    unsigned char* dst = ring + (size_t)slot * stage_bytes;
+                    mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
+                    bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384, 16384, &st.full[slot]);
+                    bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
+                             &st.full[slot]);
+                }
+        producer_done:;
+        }
+    } else if (warp == 5) {  // ---- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, N);
+            int it = 0;
+            for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
+                const int buf = j & 1;
+                if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * N);
+                bool ok = true;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int slot = it % S;
+                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(ring + (size_t)slot * stage_bytes);
+                    const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + 16384);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)  // K = 16 per MMA: +32 bytes inside the swizzled rows
+                        tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
+                    tc_commit(&st.empty[slot]);
+                }
+                if (!ok) break;
+                tc_commit(&st.tfull[buf]);
+            }
+        }
+    } else {  // ---- epilogue warps 0..3: TMEM lanes 32 w .. 32 w + 31 = vocabulary rows of the tile
+        for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
+            const int buf = j & 1;
+            if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
+            tc_fence_after();
+            float acc[2 * kMmaMaxRows];
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * N);
+            for (int c = 0; c < N; c += 16) tc_ld16(taddr + c, acc + c);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&st.tempty[buf]);
+            const int v = tile * 128 + warp * 32 + lane;
+            const bool valid = v < a.V;
+            for (int r = 0; r < R; ++r) {
+                const float lg = acc[r] + acc[R_pad + r];
+                if (valid && a.dbg_logits) {
+                    const int i = r / a.B, sb = r % a.B;
+                    a.dbg_logits[((size_t)sb * a.N + i) * a.V + v] = lg;
+                }
+                const float lt = valid ? lg * a.inv_temp : -INFINITY;
+                const float M = warp_max(lt);
+                const float e = valid ? expf(lt - M) : 0.f;
+                const float Ssum = warp_sum(e);
+                if (lane == 0 && M != -INFINITY) {
+                    const float m0 = st.m[warp][r];
+                    const float mn = fmaxf(m0, M);
+                    st.s[warp][r] = (m0 == -INFINITY ? 0.f : st.s[warp][r] * expf(m0 - mn)) + Ssum * expf(M - mn);
+                    st.m[warp][r] = mn;
+                }
+                const bool pass = valid && (st.cnt[warp][r] < k ||
+                                            better(lg, v, st.val[warp][r][k - 1], st.id[warp][r][k - 1]));
+                unsigned mask = __ballot_sync(0xffffffffu, pass);
+                while (mask) {
+                    const int jj = __ffs(mask) - 1;
+                    mask &= mask - 1;
+                    if (lane == jj) warp_list_insert(st, warp, r, k, lg, v);
+                    __syncwarp();
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tc_dealloc(tmem, tmem_cols);
+
+    // ---- this slab's partial per row: merge the 4 warps' statistics and lists (warp w: rows w, w+4, ..)
+    if (warp < 4) {
+        for (int r = warp; r < R; r += 4) {
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) M = fmaxf(M, st.m[w][r]);
+            float Ssum = 0.f;
+#pragma unroll
+            for (int w = 0; w < 4; ++w)
+                if (st.m[w][r] != -INFINITY) Ssum += st.s[w][r] * expf(st.m[w][r] - M);
+            const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
+            // lane l holds candidate (w = l / 8, j = l % 8 + 8 q) for q = 0..k/8
+            for (int j = 0; j < k; ++j) {
+                float bv = -INFINITY;
+                int bi = INT_MAX, bp = -1;
+                for (int q = lane; q < 4 * k; q += 32) {
+                    const int w = q / k, jj = q % k;
+                    if (jj >= st.cnt[w][r]) continue;
+                    const float cv = st.val[w][r][jj];
+                    const int ci = st.id[w][r][jj];
+                    if (bp < 0 || better(cv, ci, bv, bi)) { bv = cv; bi = ci; bp = q; }
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                    const int op = __shfl_xor_sync(0xffffffffu, bp, o);
+                    if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
+                }
+                if (lane == 0) {
+                    a.part_id[base * k + j] = bp >= 0 ? bi : INT_MAX;
+                    a.part_val[base * k + j] = bp >= 0 ? bv : -INFINITY;
+                    if (bp >= 0) st.val[bp / k][r][bp % k] = -INFINITY, st.id[bp / k][r][bp % k] = INT_MAX;
+                }
+                __syncwarp();
+            }
+            if (lane == 0) {
+                a.part_ms[base * 2 + 0] = M;
+                a.part_ms[base * 2 + 1] = Ssum;
+            }
+        }
+    }
+    // ---- the last CTA merges every row
+    __threadfence();
+    __syncthreads();
+    if (t == 0) st.last = atomicAdd(&a.counters[0], 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!st.last) return;
+    __threadfence();
+    const int bitmap_words = (a.n_slabs * k + 31) / 32;
+    unsigned char* mb = ring + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
+    float* sv = (float*)mb;
+    int* si = (int*)(sv + kMergeCap);
+    int* scount = si + kMergeCap;
+    unsigned* taken = (unsigned*)(scount + 4);
+    for (int r = warp; r < R; r += kMmaThreads / 32) merge_row(a, r, sv, si, scount, taken);
+    if (t == 0) a.counters[0] = 0;
+}
+
 // ---- host side ----------------------------------------------------------------------------
 namespace {
 constexpr size_t kXBudget = 128 * 1024;
@@ -324,6 +591,41 @@ int lmhead_launches(int, int, const DeviceInfo&) { return 1; }
 cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t st) {
     if (a.top_k < 1 || a.top_k > kMaxTopK) return cudaErrorInvalidValue;
     return dt == FE_F32 ? launch_t<float>(a, dev, st) : launch_t<bf16_t>(a, dev, st);
+}
+
+
+bool lmhead_mma_ok(const LmHeadArgs& a) {
+    return a.R <= kMmaMaxRows && a.d % 64 == 0 && a.top_k <= kMaxTopK;
+}
+
+size_t lmhead_mma_zb_bytes(int R, int d) {
+    const int R_pad = (R + 7) / 8 * 8;
+    return (size_t)2 * R_pad * d * 2;
+}
+
+cudaError_t lmhead_mma_prepare(const DeviceInfo& dev) {
+    return cudaFuncSetAttribute(lmhead_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                dev.max_smem_optin - (int)sizeof(MmaState) - 256);
+}
+
+cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st) {
+    const int R_pad = (a.R + 7) / 8 * 8;
+    const int N = 2 * R_pad;
+    zprep_kernel<bf16_t><<<R_pad, 256, 0, st>>>(a.hid, (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
+    const size_t budget = (size_t)dev.max_smem_optin - sizeof(MmaState) - 256;
+    int S = (int)((budget - 1024) / stage_bytes);
+    S = S > kMmaMaxStages ? kMmaMaxStages : S;
+    if (S < 2) return cudaErrorInvalidValue;
+    const size_t merge = 1024 + (size_t)(kMmaThreads / 32) * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
+    size_t smem = 1024 + (size_t)S * stage_bytes;
+    if (smem < merge) smem = merge;
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(2 * N)) cols <<= 1;
+    lmhead_mma_kernel<<<a.n_slabs, kMmaThreads, smem, st>>>(a, zb, R_pad, S, stage_bytes, cols);
+    return cudaGetLastError();
 }
 
 }  // namespace fe

@@ -66,6 +66,8 @@ struct fe_handle {
     int* status = nullptr;
     int* attn_counters = nullptr;
     int* lm_counters = nullptr;
+    bool lm_mma = false;      // LM head packed for (and run on) the tensor cores
+    uint16_t* lm_zb = nullptr;  // tensor-core LM head: bf16 hi/lo operand of the hidden rows
     int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
     cudaStream_t cap = nullptr;
     cudaGraphExec_t gexec = nullptr;
@@ -202,7 +204,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
-    FE_TRY(launch_lmhead(dt, lm, h->dev, st));
+    if (h->lm_mma) {
+        lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
+        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st));
+    } else {
+        FE_TRY(launch_lmhead(dt, lm, h->dev, st));
+    }
     if (a->dbg_hidden)
         FE_TRY(cudaMemcpyAsync(a->dbg_hidden, h->hid, (size_t)N * B * d * sizeof(float), cudaMemcpyDeviceToDevice,
                                st));
@@ -268,11 +275,12 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         if ((rc = from_cuda(linear_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(lmhead_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(attention_prepare())) != FE_OK) break;
+        if ((rc = from_cuda(lmhead_mma_prepare(h->dev))) != FE_OK) break;
 
         // ---- packed weights: one allocation, every matrix 256-byte aligned ----
         const Sizes sz = weight_sizes(c, h->es);
-        size_t total = align256(sz.w_fuse) + align256(sz.w_in) + align256(sz.embed) + align256(sz.lm_head) +
-                       align256(sz.norm);
+        size_t total = align256(sz.w_fuse) + align256(sz.w_in) + align256(sz.embed) +
+                       std::max(align256(sz.lm_head), align256(mma_packed_bytes(c.vocab, c.d))) + align256(sz.norm);
         total += (size_t)c.n_layers *
                  (2 * align256(sz.norm) + align256(sz.qkv) + align256(sz.wo) + align256(sz.gu) + align256(sz.down));
         if ((rc = from_cuda(cudaMalloc(&h->wbuf, total))) != FE_OK) break;
@@ -303,7 +311,21 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->w_fuse = put_packed(w->w_fuse, dm, 3 * dm);
         h->w_in = put_packed(w->w_in, dm, 2 * dm);
         h->embed = put(w->embed, sz.embed);
-        h->lm_head = put_packed(w->lm_head, c.vocab, dm);
+        // the LM head runs on the tensor cores when every call fits that path (bf16, at most 16
+        // hidden rows, d a multiple of 64); it is then packed in the swizzled MMA layout
+        h->lm_mma = c.dtype == FE_BF16 && (int64_t)c.n_layers * c.max_batch <= 16 && c.d % 64 == 0 &&
+                    !(getenv("FE_DRAFT_LMHEAD_CUDA_CORES") && getenv("FE_DRAFT_LMHEAD_CUDA_CORES")[0] == '1');
+        if (h->lm_mma) {
+            void* dst = p;
+            p += align256(mma_packed_bytes(c.vocab, dm));
+            if ((_fe_e = cudaMemcpyAsync(staging, w->lm_head, (size_t)c.vocab * dm * es, cudaMemcpyDefault, st)) !=
+                    cudaSuccess ||
+                (_fe_e = launch_pack_mma(staging, dst, c.vocab, dm, st)) != cudaSuccess)
+                rc = fail(_fe_e, "copy or packing of the LM head", __LINE__);
+            h->lm_head = dst;
+        } else {
+            h->lm_head = put_packed(w->lm_head, c.vocab, dm);
+        }
         h->final_norm = put(w->final_norm, sz.norm);
         h->layers.resize(c.n_layers);
         for (int i = 0; i < c.n_layers && rc == FE_OK; ++i) {
@@ -348,8 +370,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lm_slabs = lmhead_slabs(c.vocab, h->dev);
         const size_t R = (size_t)c.n_layers * B;
         const size_t k = c.top_k_max;
-        size_t off[14], n = 0, tot = 0;
-        const size_t bytes[14] = {
+        size_t off[15], n = 0, tot = 0;
+        const size_t bytes[15] = {
             cs.size() * sizeof(float),                             // rope
             B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
             B * F * 4, R * d * 4,                                  // act, hid
@@ -358,8 +380,9 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             R * h->lm_slabs * 2 * 4,                               // LM-head partial (max, sum)
             256,                                                   // status
             B * c.n_kv_heads * 4,                                  // attention split counters
-            R * 4};                                                // LM-head slab counters
-        for (n = 0; n < 14; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            R * 4,                                                 // LM-head slab counters
+            h->lm_mma ? lmhead_mma_zb_bytes((int)R, c.d) : 0};     // tensor-core LM-head operand
+        for (n = 0; n < 15; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -376,6 +399,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->status = (int*)(s + off[11]);
         h->attn_counters = (int*)(s + off[12]);
         h->lm_counters = (int*)(s + off[13]);
+        h->lm_zb = h->lm_mma ? (uint16_t*)(s + off[14]) : nullptr;
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
@@ -472,7 +496,7 @@ int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     if (!h || B < 1) return -1;
     const int N = h->cfg.n_layers;
     int n = 2 * linear_launches() + N * (4 * linear_launches() + attention_launches()) +
-            lmhead_launches(N * B, h->cfg.d, h->dev);
+            (h->lm_mma ? 2 : lmhead_launches(N * B, h->cfg.d, h->dev));
     return n + (with_tree ? 1 : 0);
 }
 
