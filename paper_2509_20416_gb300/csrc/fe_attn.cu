@@ -95,6 +95,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     float* out = a.out + (size_t)b * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
+        griddep_launch_dependents();
+        griddep_wait();
         if (s == 0) {
             if (g == 0 && t == 0) atomicOr(a.status, ST_CAPACITY);
             for (int i = t; i < G * HD; i += blockDim.x) out[i] = 0.f;
@@ -102,7 +104,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
         return;
     }
     const int t0 = s * a.split;
-    if (t0 > P) return;  // beyond this sequence's keys: not an active split
+    if (t0 > P) {  // beyond this sequence's keys: not an active split
+        griddep_launch_dependents();
+        return;
+    }
     const int t1 = min(t0 + a.split, P + 1);
     const int n_act = min(a.n_split, P / a.split + 1);
     const int nchunks = (t1 - t0 + kChunkKeys - 1) / kChunkKeys;
@@ -157,8 +162,12 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     uint32_t badmask[kAttnMaxSlots] = {0u, 0u};  // per slot, meaningful on lane 0
     int issued = 0;
     __syncthreads();  // barriers initialised
+    // cached prefix rows (< P) are not written by the earlier kernels of this draft: copy
+    // them before waiting for the QKV projection
     if (lane == 0)
         for (int j = 0; j < S && j < my_chunks; ++j, ++issued) badmask[j] = issue(j, j);
+    griddep_launch_dependents();
+    griddep_wait();
 
     // queries of the group, rotated at position P and pre-scaled by 1/sqrt(hd)
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
@@ -386,8 +395,7 @@ template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
     const int S = attn_slots(a.split, HD, sizeof(CT));
     dim3 grid(a.n_split, a.Hkv, a.B);
-    attn_kernel<CT, HD, G><<<grid, kAttnWarps * 32, attn_smem(HD, sizeof(CT), S), st>>>(a, S);
-    return cudaGetLastError();
+    return launch_k(attn_kernel<CT, HD, G>, grid, dim3(kAttnWarps * 32), attn_smem(HD, sizeof(CT), S), st, a.pdl, a, S);
 }
 
 template <typename CT, int HD>

@@ -4,9 +4,30 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "fe_draft.h"
 
 namespace fe {
+
+// Launch `kern` on `st`; with pdl the launch may overlap the previous kernel of the stream
+// (programmatic stream serialization; the kernel calls griddepcontrol.wait before it
+// touches anything an earlier kernel wrote).
+template <typename... P, typename... A>
+inline cudaError_t launch_k(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool pdl,
+                            A&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<A>(args)...);
+}
 
 // status-word bits (combined with atomicOr; the host maps them back to fe_status)
 enum : int {
@@ -55,6 +76,7 @@ struct LinearArgs {
     float* y2;
     int ldy2;
     int* status;
+    bool pdl;  // launch overlapping the previous kernel (programmatic dependent launch)
 };
 
 struct DeviceInfo {
@@ -89,6 +111,7 @@ struct LmHeadArgs {
     float* topk_prob;   // [B, N, k]
     float* lse;         // [B, N]
     int* status;
+    bool pdl;
 };
 cudaError_t lmhead_prepare(const DeviceInfo& dev);
 int lmhead_slabs(int V, const DeviceInfo& dev);
@@ -119,6 +142,7 @@ struct AttnArgs {
     int* counters;          // [B, Hkv] split-completion counters, zero between calls
     float* out;             // [B, H * hd]
     int* status;
+    bool pdl;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();

@@ -53,11 +53,15 @@ __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearA
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     const int g0 = (int)(((int64_t)blockIdx.x * GM) / gridDim.x);
     const int g1 = (int)(((int64_t)(blockIdx.x + 1) * GM) / gridDim.x);
+    // weights do not depend on the previous kernel: start streaming them first
+    const int issued = stream_begin<WT>((const unsigned char*)a.W, a.K, g0, g1, s, D);
+    griddep_launch_dependents();
+    griddep_wait();
     ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
     stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red);
     __syncthreads();
     LinearEpi<BT> e{&a, b0, nb};
-    stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e);
+    stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e, issued);
 }
 
 // ---- host side ----------------------------------------------------------------------------
@@ -89,8 +93,7 @@ cudaError_t launch_bt(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t s
     const size_t smem = stream_smem_bytes(D, xrows, Kpad, BT);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     dim3 grid(GM < dev.num_sms ? GM : dev.num_sms, (a.B + BT - 1) / BT);
-    linear_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D);
-    return cudaGetLastError();
+    return launch_k(linear_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D);
 }
 
 template <typename WT>

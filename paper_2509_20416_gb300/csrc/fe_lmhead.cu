@@ -212,11 +212,14 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     const int g0 = (int)(((int64_t)sl * GM) / gridDim.x);
     const int g1 = (int)(((int64_t)(sl + 1) * GM) / gridDim.x);
 
+    const int issued = stream_begin<WT>((const unsigned char*)a.W, K, g0, g1, s, D);
+    griddep_launch_dependents();
+    griddep_wait();
     ProParams pp{PRO_RMSNORM, a.hid, a.d, a.gamma, a.eps, nullptr, nullptr, 0, 0};
     stage_activations<WT>(pp, K, s.X, Kpad, b0, nb, a.status, s.red);
     __syncthreads();
     LmEpi<BT> ep{&a, &st, cbuf, b0, nb};
-    stream_run<WT, BT>((const unsigned char*)a.W, K, g0, g1, s, D, Kpad, nb, a.status, ep);
+    stream_run<WT, BT>((const unsigned char*)a.W, K, g0, g1, s, D, Kpad, nb, a.status, ep, issued);
     __syncthreads();
 
     // this slab's partial for each row of the tile (warp b <-> row b)
@@ -278,6 +281,8 @@ __global__ void __launch_bounds__(256) zprep_kernel(const float* __restrict__ hi
     const int r = blockIdx.x, t = threadIdx.x;
     const int N = 2 * R_pad;
     __shared__ float red[8];
+    griddep_launch_dependents();
+    griddep_wait();
     float rs = 0.f;
     if (r < R) {
         float ss = 0.f;
@@ -373,21 +378,33 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     tc_fence_after();
     const uint32_t tmem = st.tmem_base;
 
+    griddep_launch_dependents();
     if (warp == 4) {  // ---- TMA producer
         if (lane == 0) {
-            int it = 0;
-            for (int tile = t0; tile < t1; ++tile)
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
-                    const int slot = it % S;
-                    const uint32_t u = (uint32_t)(it / S);
-                    if (!mbar_wait_abortable(&st.empty[slot], (u & 1u) ^ 1u, a.status, &st.abort)) goto producer_done;
-                    unsigned char* dst = ring + (size_t)slot * stage_bytes;
-                    mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
-                    bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384, 16384, &st.full[slot]);
-                    bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
-                             &st.full[slot]);
-                }
-        producer_done:;
+            // the first stages' weight blocks do not depend on the previous kernel (zprep)
+            const int total = (t1 - t0) * nkb;
+            const int pre = min(S, total);
+            for (int it = 0; it < pre; ++it) {
+                mbar_arrive_expect_tx(&st.full[it], 16384u + (uint32_t)N * 128u);
+                const int tile = t0 + it / nkb, kb = it % nkb;
+                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384,
+                         16384, &st.full[it]);
+            }
+            griddep_wait();
+            for (int it = 0; it < pre; ++it)
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * N * 128,
+                         (uint32_t)N * 128, &st.full[it]);
+            for (int it = pre; it < total; ++it) {
+                const int slot = it % S;
+                const uint32_t u = (uint32_t)(it / S);
+                if (!mbar_wait_abortable(&st.empty[slot], (u & 1u) ^ 1u, a.status, &st.abort)) break;
+                const int tile = t0 + it / nkb, kb = it % nkb;
+                unsigned char* dst = ring + (size_t)slot * stage_bytes;
+                mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
+                bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384, 16384, &st.full[slot]);
+                bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
+                         &st.full[slot]);
+            }
         }
     } else if (warp == 5) {  // ---- MMA issuer
         if (lane == 0) {
@@ -420,7 +437,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     } else {  // ---- epilogue warps 0..3: TMEM lanes 32 w .. 32 w + 31 = vocabulary rows of the tile
         for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
             const int buf = j & 1;
-            if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
+            if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort, 20000)) break;
             tc_fence_after();
             float acc[2 * kMmaMaxRows];
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * N);
@@ -506,6 +523,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
         }
     }
     // ---- the last CTA merges every row
+    griddep_wait();  // (already satisfied: the producer waited; makes the order explicit for all threads)
     __threadfence();
     __syncthreads();
     if (t == 0) st.last = atomicAdd(&a.counters[0], 1) == (int)gridDim.x - 1;
@@ -554,8 +572,7 @@ cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t s
     if (smem < merge) smem = merge;
     if (smem > budget) return cudaErrorInvalidValue;
     dim3 grid(a.n_slabs, (a.R + BT - 1) / BT);
-    lmhead_kernel<WT, BT><<<grid, kStreamThreads, smem, st>>>(a, D);
-    return cudaGetLastError();
+    return launch_k(lmhead_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D);
 }
 
 template <typename WT>
@@ -611,8 +628,8 @@ cudaError_t lmhead_mma_prepare(const DeviceInfo& dev) {
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st) {
     const int R_pad = (a.R + 7) / 8 * 8;
     const int N = 2 * R_pad;
-    zprep_kernel<bf16_t><<<R_pad, 256, 0, st>>>(a.hid, (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb);
     if (e != cudaSuccess) return e;
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(MmaState) - 256;
@@ -624,8 +641,8 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     if (smem < merge) smem = merge;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
-    lmhead_mma_kernel<<<a.n_slabs, kMmaThreads, smem, st>>>(a, zb, R_pad, S, stage_bytes, cols);
-    return cudaGetLastError();
+    return launch_k(lmhead_mma_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb,
+                    R_pad, S, stage_bytes, cols);
 }
 
 }  // namespace fe

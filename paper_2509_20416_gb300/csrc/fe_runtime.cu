@@ -73,6 +73,7 @@ struct fe_handle {
     cudaGraphExec_t gexec = nullptr;
     GraphKey gkey;
     bool use_graph = true;
+    bool use_pdl = true;
 };
 
 namespace {
@@ -150,11 +151,15 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.status = h->status;
     la.eps = c.rms_eps;
     la.B = B;
-    // g = W_fuse concat(l, m, h)
+    // g = W_fuse concat(l, m, h). The first kernel of a draft waits for everything before it
+    // on the stream (it is launched without programmatic dependence); later kernels may
+    // overlap their predecessor's tail (see griddep_wait()).
+    la.pdl = false;
     la.W = h->w_fuse; la.M = d; la.K = 3 * d;
     la.pro = PRO_STORAGE; la.x = a->feat; la.ldx = 3 * d;
     la.epi = EPI_STORE; la.y = h->g; la.ldy = d; la.y2 = nullptr;
     FE_TRY(launch_linear(dt, la, h->dev, st));
+    la.pdl = h->use_pdl;
     // x0 = W_in concat(g, e)
     la.W = h->w_in; la.M = d; la.K = 2 * d;
     la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
@@ -169,6 +174,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     aa.rope_cs = h->rope_cs; aa.B = B; aa.H = H; aa.Hkv = Hkv; aa.hd = hd;
     aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
     aa.part = h->attn_part; aa.counters = h->attn_counters; aa.out = h->o; aa.status = h->status;
+    aa.pdl = h->use_pdl;
 
     for (int i = 0; i < N; ++i) {
         const LayerPacked& L = h->layers[i];
@@ -204,6 +210,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
+    lm.pdl = h->use_pdl;
     if (h->lm_mma) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st));
@@ -261,6 +268,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
     h->cfg = *cfg;
     const char* g = getenv("FE_DRAFT_GRAPH");
     h->use_graph = !(g && g[0] == '0');
+    const char* pd = getenv("FE_DRAFT_PDL");
+    h->use_pdl = !(pd && pd[0] == '0');
     cudaStream_t st = (cudaStream_t)stream;
     fe_status rc = FE_OK;
     do {

@@ -91,12 +91,14 @@ __device__ inline StreamSmem carve_stream_smem(unsigned char* smem, int D, int x
 }
 
 // Wait on a phase of `bar`; gives up when the CTA's abort flag is raised or after the
-// wall-clock budget (then raises the flag and records ST_TIMEOUT).
-__device__ __forceinline__ bool mbar_wait_abortable(uint64_t* bar, uint32_t parity, int* status, int* abort) {
+// wall-clock budget (then raises the flag and records ST_TIMEOUT). With sleep_ns > 0 the
+// thread sleeps (up to sleep_ns per try) instead of spinning.
+__device__ __forceinline__ bool mbar_wait_abortable(uint64_t* bar, uint32_t parity, int* status, int* abort,
+                                                    uint32_t sleep_ns = 0) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (sleep_ns ? mbar_try_wait_sleep(bar, parity, sleep_ns) : mbar_try_wait(bar, parity)) return true;
         if (*(volatile int*)abort) return false;
         if ((int64_t)(globaltimer_ns() - t0) > kWaitBudgetNs) {
             atomicOr(status, ST_TIMEOUT);
@@ -181,9 +183,43 @@ __device__ __forceinline__ void tile_compute(const unsigned char* st, const floa
 // Must be called by all 256 threads after X is staged. Calls epi.chunk(cg0, cg1, red)
 // on all threads once per chunk of up to kChunk groups; the epilogue reads values with
 // chunk_value<BT>(red, g - cg0, r, b).
+// Issue copy i (the warp's item i of the CTA's tile range) into the warp's slot.
+template <typename WT>
+__device__ __forceinline__ void stream_issue(const unsigned char* Wt, int K, int g0, int nks, int i, int slot,
+                                             uint64_t* full, unsigned char* ring) {
+    using G = StreamGeom<WT>;
+    const int g = g0 + i / nks, ks = i % nks;
+    const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
+    mbar_arrive_expect_tx(&full[slot], bytes);
+    bulk_g2s(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot]);
+}
+
+// First half of a stream: initialise the per-warp barriers and issue every warp's first D
+// copies. Touches only the (read-only) weights, so it may run before griddep_wait().
+// Must be called by all 256 threads; returns the number of copies this warp issued.
+template <typename WT>
+__device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D) {
+    using G = StreamGeom<WT>;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nks = (K + G::kKS - 1) / G::kKS;
+    const int total = (g1 - g0) * nks;
+    uint64_t* full = s.full + warp * D;
+    unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
+    int issued = 0;
+    if (lane == 0) {
+        for (int d = 0; d < D; ++d) mbar_init(&full[d], 1);
+        if (warp == 0) *s.abort = 0;
+        mbar_fence_init();
+        for (int j = 0; j < D && warp + kWarps * j < total; ++j, ++issued)
+            stream_issue<WT>(Wt, K, g0, nks, warp + kWarps * j, j, full, ring);
+    }
+    return issued;
+}
+
+// Second half: the main loop. `issued` is stream_begin's return value.
 template <typename WT, int BT, typename Epi>
 __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D, int Kpad, int nb,
-                           int* status, Epi& epi) {
+                           int* status, Epi& epi, int issued) {
     using G = StreamGeom<WT>;
     using R = WarpMultiSum<kGroupRows * BT>;
     constexpr int RV = kGroupRows * BT;
@@ -195,22 +231,8 @@ __device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, Strea
     unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
 
     for (int i = threadIdx.x; i < CH * kWarps * RV; i += kStreamThreads) s.red[i] = 0.f;
-    if (lane == 0) {
-        for (int d = 0; d < D; ++d) mbar_init(&full[d], 1);
-        if (warp == 0) *s.abort = 0;
-        mbar_fence_init();
-    }
     __syncthreads();
-
-    auto issue = [&](int i, int slot) {
-        const int g = g0 + i / nks, ks = i % nks;
-        const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
-        mbar_arrive_expect_tx(&full[slot], bytes);
-        bulk_g2s(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot]);
-    };
-    int issued = 0;  // items of this warp issued so far (lane 0's count)
-    if (lane == 0)
-        for (int j = 0; j < D && warp + kWarps * j < total; ++j, ++issued) issue(warp + kWarps * j, j);
+    auto issue = [&](int i, int slot) { stream_issue<WT>(Wt, K, g0, nks, i, slot, full, ring); };
 
     float acc[kGroupRows][BT];
 #pragma unroll
