@@ -119,81 +119,130 @@ struct LmEpi {
     }
 };
 
-// Merge of all slabs' partials for one row zr, by one warp.
-__device__ void merge_row(const LmHeadArgs& a, int zr, float* sv, int* si, int* scount, unsigned* taken) {
-    const int lane = threadIdx.x & 31;
-    const int k = a.top_k, ns = a.n_slabs;
-    const float* pv = a.part_val + (size_t)zr * ns * k;
-    const int* pi = a.part_id + (size_t)zr * ns * k;
-    const float* pm = a.part_ms + (size_t)zr * ns * 2;
-    // log-sum-exp of logit / T over the whole vocabulary
-    float M = -INFINITY;
-    for (int j = lane; j < ns; j += 32) M = fmaxf(M, __ldcg(pm + 2 * j));
-    M = warp_max(M);
-    float S = 0.f;
-    for (int j = lane; j < ns; j += 32) {
-        const float sj = __ldcg(pm + 2 * j + 1);
-        if (sj > 0.f) S += sj * expf(__ldcg(pm + 2 * j) - M);
-    }
-    S = warp_sum(S);
-    const float lse = M + logf(S);
-    // tau: the largest k-th value over slabs
-    float tau = -INFINITY;
-    for (int j = lane; j < ns; j += 32) tau = fmaxf(tau, __ldcg(pv + (size_t)j * k + k - 1));
-    tau = warp_max(tau);
-    if (lane == 0) *scount = 0;
-    __syncwarp();
-    bool overflow = false;
-    for (int j = lane; j < ns; j += 32) {
-        for (int r = 0; r < k; ++r) {
-            const float v = __ldcg(pv + (size_t)j * k + r);
-            if (v < tau) break;  // slab lists are sorted, descending
-            const int pos = atomicAdd(scount, 1);
-            if (pos < kMergeCap) {
-                sv[pos] = v;
-                si[pos] = __ldcg(pi + (size_t)j * k + r);
-            } else {
-                overflow = true;
+// Merge of all slabs' partials for rows [r0, r1), by every thread of the calling CTA.
+// The rows' partials are first copied into shared memory (`buf`, the finished stream's
+// ring) in one coalesced pass, in batches of rows that fit; then warp w merges row
+// r0 + w, r0 + w + nwarps, ... of the batch from shared memory:
+//   lse = M + log sum_j s_j e^(m_j - M) over the slabs' (max, sum of exp) pairs;
+//   tau = the largest k-th value over slabs (a slab holds k candidates >= tau, so
+//   nothing below tau can be among the k best); the candidates >= tau (all of them if
+//   there are more than kMergeCap) go through k rounds of a warp arg-max (descending
+//   value, ascending id); probabilities are exp(logit / T - lse).
+__device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* buf, size_t buf_bytes) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5, nw = blockDim.x >> 5;
+    const int ns = a.n_slabs, k = a.top_k;
+    const size_t per_row = (size_t)ns * (2 * k + 2) * 4;
+    const size_t per_warp = (size_t)kMergeCap * 8 + 16;
+    if (buf_bytes <= nw * per_warp + per_row) return;  // never happens: the host sizes the buffer
+    const int batch = (int)((buf_bytes - nw * per_warp) / per_row);
+    float* cand_v = (float*)(buf + nw * per_warp);  // [batch][ns * k]
+    for (int rb = r0; rb < r1; rb += batch) {
+        const int nr = min(batch, r1 - rb);
+        float* bv_ = cand_v;
+        int* bi_ = (int*)(cand_v + (size_t)nr * ns * k);
+        float* bm_ = (float*)(bi_ + (size_t)nr * ns * k);
+        // 8 independent loads in flight per thread (a load-then-store loop would wait a full
+        // L2 round trip per element)
+        const size_t nc = (size_t)nr * ns * k, nm = (size_t)nr * ns * 2;
+        for (size_t q0 = t; q0 < nc; q0 += 8 * (size_t)blockDim.x) {
+            float v[8];
+            int id[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const size_t q = q0 + u * (size_t)blockDim.x;
+                v[u] = q < nc ? __ldcg(a.part_val + (size_t)rb * ns * k + q) : 0.f;
+                id[u] = q < nc ? __ldcg(a.part_id + (size_t)rb * ns * k + q) : 0;
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const size_t q = q0 + u * (size_t)blockDim.x;
+                if (q < nc) { bv_[q] = v[u]; bi_[q] = id[u]; }
             }
         }
-    }
-    overflow = __any_sync(0xffffffffu, overflow);
-    __syncwarp();
-    const int n = overflow ? ns * k : min(*scount, kMergeCap);
-    // k rounds of a warp arg-max (desc value, asc id); taken entries flagged in a bitmap
-    for (int w = lane; w < (n + 31) / 32; w += 32) taken[w] = 0u;
-    __syncwarp();
-    const int i = zr / a.B, b = zr % a.B;
-    const size_t ob = ((size_t)b * a.N + i) * k;
-    for (int r = 0; r < k; ++r) {
-        float bv = -INFINITY;
-        int bi = INT_MAX, bp = -1;
-        for (int j = lane; j < n; j += 32) {
-            if (taken[j >> 5] & (1u << (j & 31))) continue;
-            const float v = overflow ? __ldcg(pv + j) : sv[j];
-            const int id = overflow ? __ldcg(pi + j) : si[j];
-            if (bp < 0 || better(v, id, bv, bi)) { bv = v; bi = id; bp = j; }
-        }
+        for (size_t q0 = t; q0 < nm; q0 += 8 * (size_t)blockDim.x) {
+            float v[8];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            const int op = __shfl_xor_sync(0xffffffffu, bp, o);
-            if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
+            for (int u = 0; u < 8; ++u) {
+                const size_t q = q0 + u * (size_t)blockDim.x;
+                v[u] = q < nm ? __ldcg(a.part_ms + (size_t)rb * ns * 2 + q) : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const size_t q = q0 + u * (size_t)blockDim.x;
+                if (q < nm) bm_[q] = v[u];
+            }
         }
-        if (lane == 0) {
-            a.topk_id[ob + r] = bi;
-            a.topk_logit[ob + r] = bv;
-            a.topk_prob[ob + r] = expf(bv * a.inv_temp - lse);
-            if (bp >= 0) taken[bp >> 5] |= 1u << (bp & 31);
+        __syncthreads();
+        for (int rr = warp; rr < nr; rr += nw) {
+            const int zr = rb + rr;
+            float* pv = bv_ + (size_t)rr * ns * k;
+            int* pi = bi_ + (size_t)rr * ns * k;
+            const float* pm = bm_ + (size_t)rr * ns * 2;
+            float* sv = (float*)(buf + warp * per_warp);
+            int* si = (int*)(sv + kMergeCap);
+            int* scount = si + kMergeCap;
+            float M = -INFINITY;
+            for (int j = lane; j < ns; j += 32) M = fmaxf(M, pm[2 * j]);
+            M = warp_max(M);
+            float S = 0.f;
+            for (int j = lane; j < ns; j += 32)
+                if (pm[2 * j + 1] > 0.f) S += pm[2 * j + 1] * expf(pm[2 * j] - M);
+            S = warp_sum(S);
+            const float lse = M + logf(S);
+            float tau = -INFINITY;
+            for (int j = lane; j < ns; j += 32) tau = fmaxf(tau, pv[(size_t)j * k + k - 1]);
+            tau = warp_max(tau);
+            if (lane == 0) *scount = 0;
+            __syncwarp();
+            bool overflow = false;
+            for (int q = lane; q < ns * k; q += 32) {
+                if (pv[q] < tau) continue;
+                const int pos = atomicAdd(scount, 1);
+                if (pos < kMergeCap) { sv[pos] = pv[q]; si[pos] = pi[q]; }
+                else overflow = true;
+            }
+            overflow = __any_sync(0xffffffffu, overflow);
+            __syncwarp();
+            // candidates: the survivors, or every staged candidate if there were too many
+            float* cv = overflow ? pv : sv;
+            int* ci = overflow ? pi : si;
+            const int n = overflow ? ns * k : min(*scount, kMergeCap);
+            const int i = zr / a.B, b = zr % a.B;
+            const size_t ob = ((size_t)b * a.N + i) * k;
+            for (int r = 0; r < k; ++r) {
+                float bv = -INFINITY;
+                int bi = INT_MAX, bp = -1;
+                for (int j = lane; j < n; j += 32) {
+                    if (bp < 0 || better(cv[j], ci[j], bv, bi)) { bv = cv[j]; bi = ci[j]; bp = j; }
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                    const int op = __shfl_xor_sync(0xffffffffu, bp, o);
+                    if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
+                }
+                if (lane == 0) {
+                    a.topk_id[ob + r] = bi;
+                    a.topk_logit[ob + r] = bv;
+                    a.topk_prob[ob + r] = expf(bv * a.inv_temp - lse);
+                    if (bp >= 0) { cv[bp] = -INFINITY; ci[bp] = INT_MAX; }  // taken
+                }
+                __syncwarp();
+            }
+            if (lane == 0) a.lse[(size_t)b * a.N + i] = lse;
         }
-        __syncwarp();
+        __syncthreads();
     }
-    if (lane == 0) a.lse[(size_t)b * a.N + i] = lse;
+}
+
+// shared memory merge_rows needs for at least one row at a time
+__host__ __device__ inline size_t merge_smem_bytes(int nwarps, int n_slabs, int top_k) {
+    return (size_t)nwarps * (kMergeCap * 8 + 16) + (size_t)n_slabs * (2 * top_k + 2) * 4 + 64;
 }
 
 template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D) {
+__global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D, size_t smem_bytes) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ TopkState st;
     const int K = a.d;
@@ -247,15 +296,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
     __syncthreads();
     if (!st.last) return;
     __threadfence();
-    // shared memory of the finished stream is reused: per warp kMergeCap values, ids, a
-    // counter and a taken-bitmap sized for the overflow fallback
-    const int bitmap_words = (a.n_slabs * a.top_k + 31) / 32;
-    unsigned char* mbase = smem + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
-    float* sv = (float*)mbase;
-    int* si = (int*)(sv + kMergeCap);
-    int* scount = si + kMergeCap;
-    unsigned* taken = (unsigned*)(scount + 4);
-    if (warp < nb) merge_row(a, b0 + warp, sv, si, scount, taken);
+    // the finished stream's shared memory holds the merge
+    merge_rows(a, b0, b0 + nb, smem, smem_bytes);
     if (t == 0) a.counters[tile] = 0;
 }
 
@@ -268,7 +310,9 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
 // 16 KB weight blocks (and the matching B blocks) with bulk TMA copies into a ring of
 // stages; warp 5 (one thread) issues the MMAs and commits each stage back to its producer;
 // warps 0..3 read the double-buffered accumulator from TMEM (TMEM lane = vocabulary row)
-// and keep per-warp softmax statistics and top-k lists, merged per slab at the end.
+// into a shared-memory buffer holding the slab's logits. After the slab, each of the 6
+// warps takes rows: softmax statistics over the buffer, and the row's top-k by k rounds of
+// a warp arg-max (each lane caches its best; only the round's winner rescans).
 constexpr int kMmaMaxRows = 16;
 constexpr int kMmaThreads = 6 * 32;
 constexpr int kMmaMaxStages = 12;
@@ -313,41 +357,20 @@ __global__ void __launch_bounds__(256) zprep_kernel(const float* __restrict__ hi
 }
 
 struct MmaState {
-    float m[4][kMmaMaxRows], s[4][kMmaMaxRows];
-    int cnt[4][kMmaMaxRows];
-    int id[4][kMmaMaxRows][kMaxTopK];
-    float val[4][kMmaMaxRows][kMaxTopK];
     uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2];
     uint32_t tmem_base;
     int last, abort;
 };
 
-__device__ __forceinline__ void warp_list_insert(MmaState& st, int w, int r, int k, float lg, int v) {
-    const int c = st.cnt[w][r];
-    int pos;
-    if (c < k) {
-        pos = c;
-        st.cnt[w][r] = c + 1;
-    } else if (better(lg, v, st.val[w][r][k - 1], st.id[w][r][k - 1])) {
-        pos = k - 1;
-    } else {
-        return;
-    }
-    while (pos > 0 && better(lg, v, st.val[w][r][pos - 1], st.id[w][r][pos - 1])) {
-        st.val[w][r][pos] = st.val[w][r][pos - 1];
-        st.id[w][r][pos] = st.id[w][r][pos - 1];
-        --pos;
-    }
-    st.val[w][r][pos] = lg;
-    st.id[w][r][pos] = v;
-}
-
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
-                                                                    int S, int stage_bytes, uint32_t tmem_cols) {
+                                                                    int S, int stage_bytes, uint32_t tmem_cols,
+                                                                    int slab_cap) {
     extern __shared__ unsigned char dsm_raw[];
     __shared__ MmaState st;
-    // 1024-byte aligned ring (the 128B swizzle pattern is a function of address bits 4..9)
+    // 1024-byte aligned ring (the 128B swizzle pattern is a function of address bits 4..9),
+    // then the slab's logits [R][slab_cap]
     unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    float* slab = (float*)(ring + (size_t)S * stage_bytes);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int N = 2 * R_pad, R = a.R, k = a.top_k;
     const int nkb = a.d / 64;
@@ -366,11 +389,6 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
         }
         st.abort = 0;
         mbar_fence_init();
-    }
-    for (int i = t; i < 4 * kMmaMaxRows; i += blockDim.x) {
-        st.m[i / kMmaMaxRows][i % kMmaMaxRows] = -INFINITY;
-        st.s[i / kMmaMaxRows][i % kMmaMaxRows] = 0.f;
-        st.cnt[i / kMmaMaxRows][i % kMmaMaxRows] = 0;
     }
     if (warp == 0) tc_alloc(&st.tmem_base, tmem_cols);
     tc_fence_before();
@@ -445,32 +463,14 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&st.tempty[buf]);
+            const int row = j * 128 + warp * 32 + lane;  // row of the slab
             const int v = tile * 128 + warp * 32 + lane;
-            const bool valid = v < a.V;
             for (int r = 0; r < R; ++r) {
                 const float lg = acc[r] + acc[R_pad + r];
-                if (valid && a.dbg_logits) {
+                slab[(size_t)r * slab_cap + row] = v < a.V ? lg : -INFINITY;
+                if (v < a.V && a.dbg_logits) {
                     const int i = r / a.B, sb = r % a.B;
                     a.dbg_logits[((size_t)sb * a.N + i) * a.V + v] = lg;
-                }
-                const float lt = valid ? lg * a.inv_temp : -INFINITY;
-                const float M = warp_max(lt);
-                const float e = valid ? expf(lt - M) : 0.f;
-                const float Ssum = warp_sum(e);
-                if (lane == 0 && M != -INFINITY) {
-                    const float m0 = st.m[warp][r];
-                    const float mn = fmaxf(m0, M);
-                    st.s[warp][r] = (m0 == -INFINITY ? 0.f : st.s[warp][r] * expf(m0 - mn)) + Ssum * expf(M - mn);
-                    st.m[warp][r] = mn;
-                }
-                const bool pass = valid && (st.cnt[warp][r] < k ||
-                                            better(lg, v, st.val[warp][r][k - 1], st.id[warp][r][k - 1]));
-                unsigned mask = __ballot_sync(0xffffffffu, pass);
-                while (mask) {
-                    const int jj = __ffs(mask) - 1;
-                    mask &= mask - 1;
-                    if (lane == jj) warp_list_insert(st, warp, r, k, lg, v);
-                    __syncwarp();
                 }
             }
         }
@@ -480,39 +480,45 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     tc_fence_after();
     if (warp == 0) tc_dealloc(tmem, tmem_cols);
 
-    // ---- this slab's partial per row: merge the 4 warps' statistics and lists (warp w: rows w, w+4, ..)
-    if (warp < 4) {
-        for (int r = warp; r < R; r += 4) {
+    // ---- this slab's partial per row (warp w: rows w, w + 6, ..): statistics and top-k
+    {
+        const int n = (t1 - t0) * 128;
+        const int first = t0 * 128;
+        for (int r = warp; r < R; r += kMmaThreads / 32) {
+            float* sb = slab + (size_t)r * slab_cap;
             float M = -INFINITY;
-#pragma unroll
-            for (int w = 0; w < 4; ++w) M = fmaxf(M, st.m[w][r]);
+            for (int j = lane; j < n; j += 32) M = fmaxf(M, sb[j] * a.inv_temp);
+            M = warp_max(M);
             float Ssum = 0.f;
-#pragma unroll
-            for (int w = 0; w < 4; ++w)
-                if (st.m[w][r] != -INFINITY) Ssum += st.s[w][r] * expf(st.m[w][r] - M);
+            for (int j = lane; j < n; j += 32)
+                if (sb[j] != -INFINITY) Ssum += expf(sb[j] * a.inv_temp - M);
+            Ssum = warp_sum(Ssum);
+            // each lane's best among its strided entries; ascending j keeps the smaller id on ties
+            float lv = -INFINITY;
+            int lp = -1;
+            for (int j = lane; j < n; j += 32)
+                if (lp < 0 || sb[j] > lv) { lv = sb[j]; lp = j; }
             const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
-            // lane l holds candidate (w = l / 8, j = l % 8 + 8 q) for q = 0..k/8
-            for (int j = 0; j < k; ++j) {
-                float bv = -INFINITY;
-                int bi = INT_MAX, bp = -1;
-                for (int q = lane; q < 4 * k; q += 32) {
-                    const int w = q / k, jj = q % k;
-                    if (jj >= st.cnt[w][r]) continue;
-                    const float cv = st.val[w][r][jj];
-                    const int ci = st.id[w][r][jj];
-                    if (bp < 0 || better(cv, ci, bv, bi)) { bv = cv; bi = ci; bp = q; }
-                }
+            for (int jj = 0; jj < k; ++jj) {
+                float bv = lv;
+                int bp = lp;
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) {
                     const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
                     const int op = __shfl_xor_sync(0xffffffffu, bp, o);
-                    if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
+                    if (op >= 0 && (bp < 0 || better(ov, op, bv, bp))) { bv = ov; bp = op; }
                 }
+                const bool ok = bp >= 0 && bv != -INFINITY;
                 if (lane == 0) {
-                    a.part_id[base * k + j] = bp >= 0 ? bi : INT_MAX;
-                    a.part_val[base * k + j] = bp >= 0 ? bv : -INFINITY;
-                    if (bp >= 0) st.val[bp / k][r][bp % k] = -INFINITY, st.id[bp / k][r][bp % k] = INT_MAX;
+                    a.part_id[base * k + jj] = ok ? first + bp : INT_MAX;
+                    a.part_val[base * k + jj] = ok ? bv : -INFINITY;
+                }
+                if (ok && (bp & 31) == lane) {  // the winner's lane removes it and rescans its entries
+                    sb[bp] = -INFINITY;
+                    lv = -INFINITY;
+                    lp = -1;
+                    for (int j = lane; j < n; j += 32)
+                        if (lp < 0 || sb[j] > lv) { lv = sb[j]; lp = j; }
                 }
                 __syncwarp();
             }
@@ -530,13 +536,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     __syncthreads();
     if (!st.last) return;
     __threadfence();
-    const int bitmap_words = (a.n_slabs * k + 31) / 32;
-    unsigned char* mb = ring + (size_t)warp * (kMergeCap * 8 + 16 + bitmap_words * 4);
-    float* sv = (float*)mb;
-    int* si = (int*)(sv + kMergeCap);
-    int* scount = si + kMergeCap;
-    unsigned* taken = (unsigned*)(scount + 4);
-    for (int r = warp; r < R; r += kMmaThreads / 32) merge_row(a, r, sv, si, scount, taken);
+    merge_rows(a, 0, R, ring, (size_t)S * stage_bytes);
     if (t == 0) a.counters[0] = 0;
 }
 
@@ -564,7 +564,7 @@ cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t s
     const int Kpad = (a.d + 3) & ~3;
     const int xrows = BT < a.R ? BT : a.R;
     const size_t budget = (size_t)dev.max_smem_optin - kStaticReserve;
-    const size_t merge = (size_t)kLmTile * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
+    const size_t merge = merge_smem_bytes(kStreamThreads / 32, a.n_slabs, a.top_k);
     int D = stream_slots(budget, stream_smem_bytes(0, xrows, Kpad, BT));
     D = D > kPreferredSlots ? kPreferredSlots : D;
     if (D < 1) return cudaErrorInvalidValue;
@@ -572,7 +572,7 @@ cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t s
     if (smem < merge) smem = merge;
     if (smem > budget) return cudaErrorInvalidValue;
     dim3 grid(a.n_slabs, (a.R + BT - 1) / BT);
-    return launch_k(lmhead_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D);
+    return launch_k(lmhead_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D, smem);
 }
 
 template <typename WT>
@@ -633,16 +633,19 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     if (e != cudaSuccess) return e;
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(MmaState) - 256;
-    int S = (int)((budget - 1024) / stage_bytes);
+    const int ntiles = (a.V + 127) / 128;
+    const int slab_cap = (ntiles + a.n_slabs - 1) / a.n_slabs * 128;  // rows of the largest slab
+    const size_t slab_bytes = (size_t)a.R * slab_cap * sizeof(float);
+    if (budget < 1024 + slab_bytes + 2 * (size_t)stage_bytes) return cudaErrorInvalidValue;
+    int S = (int)((budget - 1024 - slab_bytes) / stage_bytes);
     S = S > kMmaMaxStages ? kMmaMaxStages : S;
     if (S < 2) return cudaErrorInvalidValue;
-    const size_t merge = 1024 + (size_t)(kMmaThreads / 32) * (kMergeCap * 8 + 16 + ((a.n_slabs * a.top_k + 31) / 32) * 4);
-    size_t smem = 1024 + (size_t)S * stage_bytes;
-    if (smem < merge) smem = merge;
+    if ((size_t)S * stage_bytes < merge_smem_bytes(kMmaThreads / 32, a.n_slabs, a.top_k)) return cudaErrorInvalidValue;
+    const size_t smem = 1024 + (size_t)S * stage_bytes + slab_bytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
     return launch_k(lmhead_mma_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb,
-                    R_pad, S, stage_bytes, cols);
+                    R_pad, S, stage_bytes, cols, slab_cap);
 }
 
 }  // namespace fe
