@@ -180,6 +180,27 @@ FE_API const char *fe_last_error_detail(void);
  * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
 FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);
 
+/* The LM head with its fused softmax statistics and top-k (the tail of fe_draft_forward)
+ * over caller-provided hidden states, for callers that cannot allocate device memory at
+ * the point they need it (a frozen memory pool or arena, a path that must not call
+ * cudaMalloc, a serving loop whose memory was fixed at start-up). The paper has no
+ * counterpart; this is a packaging of the same kernels.
+ *   hidden     device [n_layers, B, d] float32: the cascade's hidden states (the layout of
+ *              fe_forward_args.dbg_hidden)
+ *   outputs    device topk_id [B, N, top_k] int32, topk_logit / topk_prob [B, N, top_k],
+ *              lse [B, N] float32, as fe_draft_forward; temperature as there
+ * It allocates nothing: it reads the LM head and final norm the handle already holds and
+ * keeps its working memory in one fixed ~2.1 MB device array that the library reserves on
+ * every device it is loaded on, for the life of the process. Limits: n_layers * B <= 16,
+ * d <= 16384, top_k <= 32; larger requests return FE_ERR_INVALID_ARG (reason in
+ * fe_last_error_detail()). All calls share that array and leave their data in it: calls
+ * that can overlap on the GPU (several streams or host threads) race and must be
+ * serialised by the caller. The first call on a device looks the array up with
+ * cudaGetSymbolAddress; make that first call before any stream capture. */
+FE_API fe_status fe_lm_head_topk_noalloc(fe_handle *h, const float *hidden, int32_t B, int32_t top_k,
+                                         float temperature, int32_t *topk_id, float *topk_logit,
+                                         float *topk_prob, float *lse, void *stream);
+
 /* Failure-detection self-test: launches one CTA whose bounded wait on a barrier that
  * nothing completes gives up after `timeout_ns` nanoseconds (1e3..1e9) and records
  * FE_ERR_TIMEOUT in the handle's status word. The GPU stays usable. */

@@ -76,6 +76,8 @@ _lib.fe_launch_count.argtypes = [_vp, _i32, _i32]
 _lib.fe_launch_count.restype = _i32
 _lib.fe_selftest_timeout.argtypes = [_vp, ctypes.c_int64, _vp]
 _lib.fe_selftest_timeout.restype = ctypes.c_int
+_lib.fe_lm_head_topk_noalloc.argtypes = [_vp, _vp, _i32, _i32, ctypes.c_float, _vp, _vp, _vp, _vp, _vp]
+_lib.fe_lm_head_topk_noalloc.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
 _lib.fe_last_error_detail.restype = ctypes.c_char_p
 
@@ -214,3 +216,16 @@ def fe_launch_count(h: Handle, B: int, with_tree: bool = True) -> int:
 
 def fe_selftest_timeout(h: Handle, timeout_ns: int, stream=None) -> int:
     return int(_lib.fe_selftest_timeout(h.ptr, int(timeout_ns), _stream(stream)))
+
+
+def fe_lm_head_topk_noalloc(h: Handle, hidden, B: int, top_k: int, temperature: float = 0.0,
+                            out: dict | None = None, stream=None) -> dict:
+    """LM head + softmax statistics + top-k over hidden [N, B, d] (float32, device) without
+    allocating device memory inside the library (see include/fe_draft.h). Output buffers
+    are allocated here by PyTorch unless given in ``out``."""
+    if out is None:
+        out = alloc_outputs(h, B, top_k, hidden.device)
+    _check(_lib.fe_lm_head_topk_noalloc(h.ptr, _p(hidden), int(B), int(top_k), float(temperature),
+                                        _p(out["topk_id"]), _p(out["topk_logit"]), _p(out["topk_prob"]),
+                                        _p(out["lse"]), _stream(stream)), "fe_lm_head_topk_noalloc")
+    return out

@@ -127,6 +127,22 @@ cudaError_t launch_pack_mma(const void* src, void* dst, int M, int K, cudaStream
 cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st);
 
+// Read-only view of what a handle holds for its LM head (for entry points outside
+// fe_runtime.cu). Returns false for a null handle.
+struct LmHeadView {
+    const void* lm_head;     // packed for the tensor cores (mma) or tile-packed
+    const void* final_norm;  // [d]
+    bool mma;
+    fe_dtype dtype;
+    int d, V, N, max_batch, top_k_max, n_slabs;
+    float eps;
+    int* status;
+    DeviceInfo dev;
+};
+bool handle_lmhead_view(const fe_handle* h, LmHeadView* v);
+// record a message for fe_last_error_detail() (calling thread)
+void set_error_detail(const char* msg);
+
 // ---- decode attention ----------------------------------------------------------------
 struct AttnArgs {
     const float* qkv;  // [B, (H + 2 Hkv) hd] float32, before RoPE

@@ -234,6 +234,26 @@ void release(fe_handle* h) {
 
 }  // namespace
 
+void fe::set_error_detail(const char* msg) { snprintf(g_detail, sizeof(g_detail), "%s", msg); }
+
+bool fe::handle_lmhead_view(const fe_handle* h, LmHeadView* v) {
+    if (!h || !v) return false;
+    v->lm_head = h->lm_head;
+    v->final_norm = h->final_norm;
+    v->mma = h->lm_mma;
+    v->dtype = h->cfg.dtype;
+    v->d = h->cfg.d;
+    v->V = h->cfg.vocab;
+    v->N = h->cfg.n_layers;
+    v->max_batch = h->cfg.max_batch;
+    v->top_k_max = h->cfg.top_k_max;
+    v->n_slabs = h->lm_mma ? std::min(h->dev.num_sms, (h->cfg.vocab + 127) / 128) : h->lm_slabs;
+    v->eps = h->cfg.rms_eps;
+    v->status = h->status;
+    v->dev = h->dev;
+    return true;
+}
+
 extern "C" {
 
 const char* fe_status_str(fe_status s) {
