@@ -38,11 +38,29 @@ def parse():
     ap.add_argument("--workload", default="vic13b")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--profile-steps", type=int, default=50,
+                    help="drafts timed launch by launch (CUDA events) for the per-kernel roofline")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
                     help="override a workload field (e.g. n_layers=1) for profiling runs")
     return ap.parse_args()
+
+
+# DRAM traffic of the dominant kernel family from an ncu capture (dram__bytes_read.sum +
+# dram__bytes_write.sum over the linear launches of one draft of this workload), with the
+# SHA-256 of the kernel sources it was taken on: a changed kernel reports traffic null.
+TRAFFIC = {}
+KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
+
+
+def kernel_source_hash() -> str:
+    import hashlib
+    hsh = hashlib.sha256()
+    for n in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2509_20416_gb300", "csrc", n), "rb") as f:
+            hsh.update(f.read())
+    return hsh.hexdigest()[:16]
 
 
 def peaks():
@@ -274,19 +292,55 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
 
-    # ---- roofline of the draft step ------------------------------------------------------
+    # ---- per-kernel device times: every launch bracketed by CUDA events on its stream -----
+    per = {}
+    n_prof = 0
+    for _ in range(max(1, args.profile_steps)):
+        for kind, us in fe.fe_profile_forward(h, feat, tok, plen, kd, vd, k, cfg["temperature"], page_table=table,
+                                              n_pages=n_pages, out=out, stream=stream):
+            c = per.setdefault(kind, [0, 0.0])
+            c[0] += 1
+            c[1] += us
+        n_prof += 1
+    st = fe.fe_last_device_status(h)
+    if st != fe.FE_OK:
+        raise SystemExit(f"device status after the profiled drafts: {fe.fe_status_str(st)}")
+    prof_total = sum(v[1] for v in per.values())
+    kernels = {kind: {"launches_per_draft": v[0] / n_prof, "us_per_draft": v[1] / n_prof,
+                      "us_per_launch": v[1] / v[0], "share": v[1] / prof_total} for kind, v in per.items()}
+
+    # ---- roofline of the dominant kernel (and of the whole step, for context) ----------------
     peak, peak_kind = peaks()
-    alg_bytes = wl.algorithmic_bytes(cfg, I["prefix_len"].tolist())
-    achieved = alg_bytes / (ms_step / 1e3) / 1e9
+    plist = I["prefix_len"].tolist()
+    alg_bytes = wl.algorithmic_bytes(cfg, plist)
+    kbytes = wl.kernel_bytes(cfg, plist)
+    for kind, v in kernels.items():
+        if kind in kbytes:
+            v["algorithmic_bytes_per_draft"] = kbytes[kind]
+            v["achieved_gbs"] = kbytes[kind] / (v["us_per_draft"] * 1e-6) / 1e9
+    top = max(kernels, key=lambda x: kernels[x]["us_per_draft"])
+    kt = kernels[top]
+    bytes_per_launch = kbytes.get(top, 0) / kt["launches_per_draft"]
+    achieved = bytes_per_launch / (kt["us_per_launch"] * 1e-6) / 1e9
+    traffic = None
+    tr = TRAFFIC.get(f"{args.workload}{''.join(' ' + o for o in args.set)}")
+    if tr and top == "linear" and tr["src"] == kernel_source_hash():
+        traffic = tr["bytes_per_draft"] / kt["launches_per_draft"]
+    step_achieved = alg_bytes / (ms_step / 1e3) / 1e9
     launches = fe.fe_launch_count(h, B, True)
 
     line = {"metric": "drafts/s", "value": value, "unit": "drafts/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "us_per_draft": ms_step * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
             "data": "synthetic (seeded generator)", "config": workload_config(cfg, wl),
-            "roofline": {"bound": "hbm", "kernel": "draft step (fe_draft_forward + fe_build_tree)",
-                         "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                         "peak_kind": peak_kind, "algorithmic_bytes": alg_bytes, "traffic": None},
+            "roofline": {"bound": "hbm", "kernel": top, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "peak_kind": peak_kind, "traffic": traffic,
+                         "algorithmic_bytes_per_launch": bytes_per_launch,
+                         "us_per_launch": kt["us_per_launch"], "launches_per_draft": kt["launches_per_draft"],
+                         "timing": f"CUDA events around every launch, {n_prof} drafts launched eagerly",
+                         "step": {"achieved": step_achieved, "frac": step_achieved / peak,
+                                  "algorithmic_bytes": alg_bytes}},
+            "kernels": kernels,
             "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": launches * args.steps, "launches_per_step": launches,

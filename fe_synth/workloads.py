@@ -194,6 +194,21 @@ def algorithmic_bytes(cfg: dict, prefix_len) -> int:
     return int((w + kv + emb + feat) * es)
 
 
+def kernel_bytes(cfg: dict, prefix_len) -> dict:
+    """algorithmic_bytes split by kernel family (the parts sum to it): 'linear' = the
+    weight-streaming phases (W_fuse, W_in and every layer's W_qkv, W_o, W_gate/up, W_down
+    with the layer's two norm gains, plus the features and gathered embedding rows they
+    read), 'attention' = every layer's K/V traffic, 'lm_head' = the LM head and final norm."""
+    d, H, Hkv, hd, F, V, N = (cfg[k] for k in ("d", "n_heads", "n_kv_heads", "head_dim", "ffn",
+                                               "vocab", "n_layers"))
+    es = 4 if cfg["dtype"] == "f32" else 2
+    B = len(prefix_len)
+    lin = d * 3 * d + d * 2 * d + N * ((H + 2 * Hkv) * hd * d + d * H * hd + 2 * F * d + d * F + 2 * d)
+    lin += B * d + B * 3 * d
+    kv = N * sum(int(p) + 1 for p in prefix_len) * 2 * Hkv * hd
+    return {"linear": int(lin * es), "attention": int(kv * es), "lm_head": int((V * d + d) * es)}
+
+
 def algorithmic_flops(cfg: dict, prefix_len) -> int:
     d, H, Hkv, hd, F, V, N = (cfg[k] for k in ("d", "n_heads", "n_kv_heads", "head_dim", "ffn",
                                                "vocab", "n_layers"))

@@ -180,13 +180,33 @@ FE_API const char *fe_last_error_detail(void);
  * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
 FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);
 
+/* Kernel families of one draft, as fe_profile_forward reports them. */
+typedef enum {
+    FE_KERNEL_LINEAR = 0,    /* weight-streaming linear phase (W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down) */
+    FE_KERNEL_ATTENTION = 1, /* RoPE + K/V append + decode attention of one layer */
+    FE_KERNEL_LM_PREP = 2,   /* tensor-core LM head: RMSNorm of the hidden rows into its bf16 operand */
+    FE_KERNEL_LM_HEAD = 3,   /* LM head + softmax statistics + top-k (and its merge) */
+    FE_KERNEL_COPY = 4       /* the dbg_hidden copy */
+} fe_kernel_kind;
+
+/* Measurement aid: runs one draft exactly as fe_draft_forward computes it, but launched
+ * eagerly (no CUDA graph, no overlap of a kernel with its predecessor) with a CUDA event
+ * recorded on `stream` before the first launch and after every launch. It then waits for
+ * the stream and writes, for launch j < *n_launches, its family kinds[j] (fe_kernel_kind)
+ * and its device time usec[j] in microseconds (event to event). Arguments and outputs are
+ * those of fe_draft_forward; kinds and usec are HOST arrays of `cap` entries, and
+ * cap >= fe_launch_count(h, B, 0) + 1 is enough. Returns FE_ERR_INVALID_ARG for bad
+ * arguments or too small a cap. Not for use inside stream capture. */
+FE_API fe_status fe_profile_forward(fe_handle *h, const fe_forward_args *args, void *stream, int32_t cap,
+                                    int32_t *kinds, float *usec, int32_t *n_launches);
+
 /* The LM head with its fused softmax statistics and top-k (the tail of fe_draft_forward)
  * over caller-provided hidden states, for callers that cannot allocate device memory at
  * the point they need it (a frozen memory pool or arena, a path that must not call
  * cudaMalloc, a serving loop whose memory was fixed at start-up). The paper has no
  * counterpart; this is a packaging of the same kernels.
- *   hidden     device [n_layers, B, d] float32: the cascade's hidden states (the layout of
- *              fe_forward_args.dbg_hidden)
+ *   hidden     device [n_layers, B, d] float32, 16-byte aligned: the cascade's hidden
+ *              states (the layout of fe_forward_args.dbg_hidden)
  *   outputs    device topk_id [B, N, top_k] int32, topk_logit / topk_prob [B, N, top_k],
  *              lse [B, N] float32, as fe_draft_forward; temperature as there
  * It allocates nothing: it reads the LM head and final norm the handle already holds and

@@ -78,6 +78,8 @@ _lib.fe_selftest_timeout.argtypes = [_vp, ctypes.c_int64, _vp]
 _lib.fe_selftest_timeout.restype = ctypes.c_int
 _lib.fe_lm_head_topk_noalloc.argtypes = [_vp, _vp, _i32, _i32, ctypes.c_float, _vp, _vp, _vp, _vp, _vp]
 _lib.fe_lm_head_topk_noalloc.restype = ctypes.c_int
+_lib.fe_profile_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _i32, _vp, _vp, ctypes.POINTER(_i32)]
+_lib.fe_profile_forward.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
 _lib.fe_last_error_detail.restype = ctypes.c_char_p
 
@@ -182,6 +184,32 @@ def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, to
                         _p(out["topk_prob"]), _p(out["lse"]), _p(dbg_logits), _p(dbg_hidden))
     _check(_lib.fe_draft_forward(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_forward")
     return out
+
+
+FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "copy"}
+
+
+def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
+                       temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
+                       dbg_hidden=None, stream=None) -> list[tuple[str, float]]:
+    """One draft launched eagerly with a CUDA event after every launch (include/fe_draft.h).
+    Returns [(kernel family, device microseconds)] in launch order."""
+    B = int(next_tok.shape[0])
+    if out is None:
+        out = alloc_outputs(h, B, top_k, feat.device)
+    N = h.cfg["n_layers"]
+    kc = (_vp * N)(*[_p(t) for t in k_cache])
+    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
+                        _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
+                        _p(out["topk_prob"]), _p(out["lse"]), None, _p(dbg_hidden))
+    cap = fe_launch_count(h, B, False) + 1
+    kinds = (_i32 * cap)()
+    usec = (ctypes.c_float * cap)()
+    n = _i32(0)
+    _check(_lib.fe_profile_forward(h.ptr, ctypes.byref(a), _stream(stream), cap, ctypes.cast(kinds, _vp),
+                                   ctypes.cast(usec, _vp), ctypes.byref(n)), "fe_profile_forward")
+    return [(FE_KERNEL_NAMES.get(kinds[j], str(kinds[j])), float(usec[j])) for j in range(n.value)]
 
 
 def alloc_tree(h: Handle, B: int, top_k: int, device="cuda") -> dict:

@@ -125,7 +125,9 @@ size_t lmhead_mma_zb_bytes(int R, int d);
 size_t mma_packed_bytes(int M, int K);
 cudaError_t launch_pack_mma(const void* src, void* dst, int M, int K, cudaStream_t st);
 cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);
-cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st);
+// after_prep (optional): an event recorded on st between the two kernels it launches
+cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
+                              cudaEvent_t after_prep = nullptr);
 
 // Read-only view of what a handle holds for its LM head (for entry points outside
 // fe_runtime.cu). Returns false for a null handle.

@@ -318,41 +318,74 @@ constexpr int kMmaThreads = 6 * 32;
 constexpr int kMmaMaxStages = 12;
 
 // zb [d/64][N rows x 128 B] in the 128B-swizzled layout: rows [0, R_pad) hold z_hi, rows
-// [R_pad, 2 R_pad) hold z_lo; rows of padding (r >= R) are zero. One CTA per row r < R_pad.
+// [R_pad, 2 R_pad) hold z_lo; rows of padding (r >= R) are zero. One CTA per row r < R_pad;
+// thread t owns the 16-byte chunks (8 values) t, t + 256, ... of the row, kept in
+// registers between the sum of squares and the split (d <= kZprepMaxChunks * 8 * 256).
+constexpr int kZprepMaxChunks = 8;
+
 template <typename WT>
-__global__ void __launch_bounds__(256) zprep_kernel(const float* __restrict__ hid, const WT* __restrict__ gamma, int R,
-                                                    int R_pad, int d, float eps, uint16_t* __restrict__ zb) {
+// hid is written by the previous kernel, which may still be running when this one starts
+// (programmatic launch): it is read only after griddep_wait(), through L2 (ld.global.cg),
+// and is deliberately not a __restrict__ pointer, whose loads the compiler may treat as
+// invariant and move above the wait.
+__global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* __restrict__ gamma, int R,
+                                                    int R_pad, int d, float eps, uint16_t* zb) {
+    static_assert(sizeof(WT) == 2, "the tensor-core LM head takes bf16 weights");
     const int r = blockIdx.x, t = threadIdx.x;
     const int N = 2 * R_pad;
+    const int nc = d / 8;  // 16-byte chunks of a bf16 row
     __shared__ float red[8];
+    // the gains do not depend on the previous kernel
+    uint4 gv[kZprepMaxChunks];
+#pragma unroll
+    for (int j = 0; j < kZprepMaxChunks; ++j) {
+        const int c = t + 256 * j;
+        gv[j] = c < nc ? reinterpret_cast<const uint4*>(gamma)[c] : make_uint4(0u, 0u, 0u, 0u);
+    }
     griddep_launch_dependents();
     griddep_wait();
-    float rs = 0.f;
-    if (r < R) {
-        float ss = 0.f;
-        for (int k = t; k < d; k += 256) {
-            const float v = hid[(size_t)r * d + k];
-            ss = fmaf(v, v, ss);
-        }
-        ss = warp_sum(ss);
-        if ((t & 31) == 0) red[t >> 5] = ss;
-        __syncthreads();
-        float tot = 0.f;
+    float x[kZprepMaxChunks][8];
+    float ss = 0.f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) tot += red[w];
-        rs = 1.0f / sqrtf(tot / (float)d + eps);
-    }
-    for (int k = t; k < d; k += 256) {
-        uint16_t hi = 0, lo = 0;
-        if (r < R) {
-            const float z = hid[(size_t)r * d + k] * rs * Storage<WT>::load(gamma, k);
-            hi = f32_to_bf16(z);
-            lo = f32_to_bf16(z - bf16_to_f32(hi));
+    for (int j = 0; j < kZprepMaxChunks; ++j) {
+        const int c = t + 256 * j;
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
+        if (r < R && c < nc) {
+            const float4* hp = reinterpret_cast<const float4*>(hid + (size_t)r * d) + 2 * c;
+            a = __ldcg(hp);
+            b = __ldcg(hp + 1);
         }
-        const int kb = k / 64, c = (k % 64) / 8, e = k % 8;
+        x[j][0] = a.x; x[j][1] = a.y; x[j][2] = a.z; x[j][3] = a.w;
+        x[j][4] = b.x; x[j][5] = b.y; x[j][6] = b.z; x[j][7] = b.w;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ss = fmaf(x[j][e], x[j][e], ss);
+    }
+    ss = warp_sum(ss);
+    if ((t & 31) == 0) red[t >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    const float rs = r < R ? 1.0f / sqrtf(tot / (float)d + eps) : 0.f;
+#pragma unroll
+    for (int j = 0; j < kZprepMaxChunks; ++j) {
+        const int c = t + 256 * j;
+        if (c >= nc) continue;
+        float g[8];
+        Vec16<WT>::widen(gv[j], g);
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+            const float z0 = x[j][e] * rs * g[e], z1 = x[j][e + 1] * rs * g[e + 1];
+            const uint16_t h0 = f32_to_bf16(z0), h1 = f32_to_bf16(z1);
+            const uint16_t l0 = f32_to_bf16(z0 - bf16_to_f32(h0)), l1 = f32_to_bf16(z1 - bf16_to_f32(h1));
+            hi[e / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            lo[e / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+        }
+        const int kb = c / 8, cc = c % 8;  // 64-column block, 16-byte chunk within it
         unsigned char* blk = (unsigned char*)zb + (size_t)kb * N * 128;
-        *(uint16_t*)(blk + sw128_offset(r, c) + e * 2) = hi;
-        *(uint16_t*)(blk + sw128_offset(R_pad + r, c) + e * 2) = lo;
+        *reinterpret_cast<uint4*>(blk + sw128_offset(r, cc)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(blk + sw128_offset(R_pad + r, cc)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
     }
 }
 
@@ -612,7 +645,7 @@ cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& de
 
 
 bool lmhead_mma_ok(const LmHeadArgs& a) {
-    return a.R <= kMmaMaxRows && a.d % 64 == 0 && a.top_k <= kMaxTopK;
+    return a.R <= kMmaMaxRows && a.d % 64 == 0 && a.d <= kZprepMaxChunks * 8 * 256 && a.top_k <= kMaxTopK;
 }
 
 size_t lmhead_mma_zb_bytes(int R, int d) {
@@ -625,12 +658,15 @@ cudaError_t lmhead_mma_prepare(const DeviceInfo& dev) {
                                 dev.max_smem_optin - (int)sizeof(MmaState) - 256);
 }
 
-cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st) {
+cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
+                              cudaEvent_t after_prep) {
+    if (!lmhead_mma_ok(a) || (reinterpret_cast<uintptr_t>(a.hid) & 15)) return cudaErrorInvalidValue;
     const int R_pad = (a.R + 7) / 8 * 8;
     const int N = 2 * R_pad;
     cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
                              (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb);
     if (e != cudaSuccess) return e;
+    if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(MmaState) - 256;
     const int ntiles = (a.V + 127) / 128;

@@ -56,6 +56,7 @@ extern "C" FE_API fe_status fe_lm_head_topk_noalloc(fe_handle* h, const float* h
     LmHeadView v;
     if (!handle_lmhead_view(h, &v) || !hidden || !topk_id || !topk_logit || !topk_prob || !lse)
         return FE_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(hidden) & 15) return FE_ERR_INVALID_ARG;  // read as 16-byte vectors
     if (B < 1 || B > v.max_batch || top_k < 1 || top_k > v.top_k_max || top_k > kMaxTopK)
         return FE_ERR_INVALID_ARG;
     if (!(temperature == temperature)) return FE_ERR_INVALID_ARG;

@@ -74,6 +74,7 @@ struct fe_handle {
     GraphKey gkey;
     bool use_graph = true;
     bool use_pdl = true;
+    std::vector<cudaEvent_t> prof_ev;  // fe_profile_forward's events (created on first use)
 };
 
 namespace {
@@ -123,6 +124,21 @@ struct Sizes {
     size_t w_fuse, w_in, embed, lm_head, norm, qkv, wo, gu, down;
 };
 
+// fe_profile_forward's recorder: ev[0] is recorded before the first launch and ev[j + 1]
+// after launch j, whose family is kinds[j]
+struct Prof {
+    cudaEvent_t* ev;
+    int32_t* kinds;
+    int cap, n;
+};
+
+inline cudaError_t mark(Prof* pf, int kind, cudaStream_t st) {
+    if (!pf) return cudaSuccess;
+    if (pf->n >= pf->cap) return cudaErrorInvalidValue;
+    pf->kinds[pf->n] = kind;
+    return cudaEventRecord(pf->ev[++pf->n], st);
+}
+
 // bytes of each matrix in the tile-packed layout (rows padded to a multiple of 4); the
 // embedding and the norm gains stay in their canonical layout
 Sizes weight_sizes(const fe_config& c, size_t es) {
@@ -141,11 +157,13 @@ Sizes weight_sizes(const fe_config& c, size_t es) {
     return s;
 }
 
-fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t st) {
+fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t st, Prof* pf = nullptr) {
     const fe_config& c = h->cfg;
     const int B = a->B, d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
     const int N = c.n_layers, nqkv = (H + 2 * Hkv) * hd;
     const fe_dtype dt = c.dtype;
+    const bool pdl = h->use_pdl && !pf;  // profiled launches do not overlap
+    if (pf) FE_TRY(cudaEventRecord(pf->ev[0], st));
 
     LinearArgs la{};
     la.status = h->status;
@@ -159,13 +177,15 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.pro = PRO_STORAGE; la.x = a->feat; la.ldx = 3 * d;
     la.epi = EPI_STORE; la.y = h->g; la.ldy = d; la.y2 = nullptr;
     FE_TRY(launch_linear(dt, la, h->dev, st));
-    la.pdl = h->use_pdl;
+    FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+    la.pdl = pdl;
     // x0 = W_in concat(g, e)
     la.W = h->w_in; la.M = d; la.K = 2 * d;
     la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
     la.d_split = d; la.vocab = V;
     la.epi = EPI_STORE; la.y = h->x; la.ldy = d;
     FE_TRY(launch_linear(dt, la, h->dev, st));
+    FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
 
     AttnArgs aa{};
     aa.qkv = h->qkv; aa.prefix_len = a->prefix_len; aa.page_table = a->page_table;
@@ -174,7 +194,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     aa.rope_cs = h->rope_cs; aa.B = B; aa.H = H; aa.Hkv = Hkv; aa.hd = hd;
     aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
     aa.part = h->attn_part; aa.counters = h->attn_counters; aa.out = h->o; aa.status = h->status;
-    aa.pdl = h->use_pdl;
+    aa.pdl = pdl;
 
     for (int i = 0; i < N; ++i) {
         const LayerPacked& L = h->layers[i];
@@ -183,24 +203,29 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.attn_norm;
         la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
         FE_TRY(launch_linear(dt, la, h->dev, st));
+        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
         FE_TRY(launch_attention(dt, aa, st));
+        FE_TRY(mark(pf, FE_KERNEL_ATTENTION, st));
         // x += W_o o
         la.W = L.w_o; la.M = d; la.K = H * hd;
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr;
         FE_TRY(launch_linear(dt, la, h->dev, st));
+        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm;
         la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
         FE_TRY(launch_linear(dt, la, h->dev, st));
+        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
         // x += W_down a; h_i = x
         la.W = L.w_down; la.M = d; la.K = F;
         la.pro = PRO_F32; la.x = h->act; la.ldx = F;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = h->hid + (size_t)i * B * d; la.ldy2 = d;
         FE_TRY(launch_linear(dt, la, h->dev, st));
+        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
     }
 
     const float inv_temp = a->temperature > 0.f ? 1.0f / a->temperature : 1.0f;
@@ -210,21 +235,45 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
-    lm.pdl = h->use_pdl;
+    lm.pdl = pdl;
     if (h->lm_mma) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
-        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st));
+        if (pf) {
+            if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
+            pf->kinds[pf->n] = FE_KERNEL_LM_PREP;
+            ++pf->n;
+        }
+        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n] : nullptr));
+        FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     } else {
         FE_TRY(launch_lmhead(dt, lm, h->dev, st));
+        FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     }
-    if (a->dbg_hidden)
+    if (a->dbg_hidden) {
         FE_TRY(cudaMemcpyAsync(a->dbg_hidden, h->hid, (size_t)N * B * d * sizeof(float), cudaMemcpyDeviceToDevice,
                                st));
+        FE_TRY(mark(pf, FE_KERNEL_COPY, st));
+    }
     return FE_OK;
+}
+
+bool forward_args_ok(const fe_handle* h, const fe_forward_args* a) {
+    if (!h || !a) return false;
+    const fe_config& c = h->cfg;
+    if (a->B < 1 || a->B > c.max_batch) return false;
+    if (a->top_k < 1 || a->top_k > c.top_k_max) return false;
+    if (!a->feat || !a->next_tok || !a->prefix_len || !a->k_cache || !a->v_cache) return false;
+    if (!a->topk_id || !a->topk_logit || !a->topk_prob || !a->lse) return false;
+    for (int i = 0; i < c.n_layers; ++i)
+        if (!a->k_cache[i] || !a->v_cache[i]) return false;
+    if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return false;
+    if (!(a->temperature == a->temperature)) return false;  // NaN
+    return true;
 }
 
 void release(fe_handle* h) {
     if (!h) return;
+    for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
     if (h->cap) cudaStreamDestroy(h->cap);
     if (h->wbuf) cudaFree(h->wbuf);
@@ -342,7 +391,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->embed = put(w->embed, sz.embed);
         // the LM head runs on the tensor cores when every call fits that path (bf16, at most 16
         // hidden rows, d a multiple of 64); it is then packed in the swizzled MMA layout
-        h->lm_mma = c.dtype == FE_BF16 && (int64_t)c.n_layers * c.max_batch <= 16 && c.d % 64 == 0 &&
+        h->lm_mma = c.dtype == FE_BF16 && (int64_t)c.n_layers * c.max_batch <= 16 && c.d % 64 == 0 && c.d <= 16384 &&
                     !(getenv("FE_DRAFT_LMHEAD_CUDA_CORES") && getenv("FE_DRAFT_LMHEAD_CUDA_CORES")[0] == '1');
         if (h->lm_mma) {
             void* dst = p;
@@ -446,16 +495,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
 }
 
 fe_status fe_draft_forward(fe_handle* h, const fe_forward_args* a, void* stream) {
-    if (!h || !a) return FE_ERR_INVALID_ARG;
+    if (!forward_args_ok(h, a)) return FE_ERR_INVALID_ARG;
     const fe_config& c = h->cfg;
-    if (a->B < 1 || a->B > c.max_batch) return FE_ERR_INVALID_ARG;
-    if (a->top_k < 1 || a->top_k > c.top_k_max) return FE_ERR_INVALID_ARG;
-    if (!a->feat || !a->next_tok || !a->prefix_len || !a->k_cache || !a->v_cache) return FE_ERR_INVALID_ARG;
-    if (!a->topk_id || !a->topk_logit || !a->topk_prob || !a->lse) return FE_ERR_INVALID_ARG;
-    for (int i = 0; i < c.n_layers; ++i)
-        if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
-    if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
-    if (!(a->temperature == a->temperature)) return FE_ERR_INVALID_ARG;  // NaN
     cudaStream_t st = (cudaStream_t)stream;
     try {
         if (!h->use_graph) return enqueue_forward(h, a, st);
@@ -484,6 +525,36 @@ fe_status fe_draft_forward(fe_handle* h, const fe_forward_args* a, void* stream)
             h->gkey = key;
         }
         FE_TRY(cudaGraphLaunch(h->gexec, st));
+        return FE_OK;
+    } catch (...) {
+        return FE_ERR_OOM;
+    }
+}
+
+fe_status fe_profile_forward(fe_handle* h, const fe_forward_args* a, void* stream, int32_t cap, int32_t* kinds,
+                             float* usec, int32_t* n_launches) {
+    if (!forward_args_ok(h, a) || !kinds || !usec || !n_launches || cap < 1 || cap > 4096) return FE_ERR_INVALID_ARG;
+    if (cap < fe_launch_count(h, a->B, 0) + (a->dbg_hidden ? 1 : 0)) return FE_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    try {
+        while ((int)h->prof_ev.size() < cap + 1) {
+            cudaEvent_t e = nullptr;
+            FE_TRY(cudaEventCreate(&e));
+            h->prof_ev.push_back(e);
+        }
+        Prof pf{h->prof_ev.data(), kinds, cap, 0};
+        const fe_status rc = enqueue_forward(h, a, st, &pf);
+        if (rc != FE_OK) {
+            cudaStreamSynchronize(st);
+            return rc;
+        }
+        FE_TRY(cudaEventSynchronize(pf.ev[pf.n]));
+        for (int j = 0; j < pf.n; ++j) {
+            float ms = 0.f;
+            FE_TRY(cudaEventElapsedTime(&ms, pf.ev[j], pf.ev[j + 1]));
+            usec[j] = 1000.f * ms;
+        }
+        *n_launches = pf.n;
         return FE_OK;
     } catch (...) {
         return FE_ERR_OOM;

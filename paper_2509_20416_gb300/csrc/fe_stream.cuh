@@ -295,39 +295,114 @@ struct ProParams {
     int vocab;
 };
 
+// Copy n values of src (storage type T, global) widened to float into dst (shared); returns
+// this thread's sum of squares when SQ. Uses 16-byte loads with up to 8 in flight per
+// thread when both ends are 16-byte aligned and n is a whole number of vectors: the
+// activations are read after griddep_wait(), and a latency-bound prologue would leave the
+// weight stream idle once the first copies have landed. src may have been written by the
+// previous kernel: it is read through L2 (ld.global.cg) and is not a __restrict__ pointer,
+// so no load can be treated as invariant and moved above griddep_wait().
+template <typename T, bool SQ>
+__device__ __forceinline__ float stage_span(const T* src, float* dst, int n) {
+    constexpr int V = Vec16<T>::kN;
+    constexpr int U = 8;
+    float ss = 0.f;
+    const bool vec = ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0 && n % V == 0;
+    if (vec) {
+        const uint4* s4 = reinterpret_cast<const uint4*>(src);
+        const int nv = n / V;
+        for (int base = threadIdx.x; base < nv; base += kStreamThreads * U) {
+            uint4 r[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * kStreamThreads;
+                r[u] = i < nv ? __ldcg(s4 + i) : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * kStreamThreads;
+                if (i < nv) {
+                    float f[V];
+                    Vec16<T>::widen(r[u], f);
+                    if (SQ) {
+#pragma unroll
+                        for (int j = 0; j < V; ++j) ss = fmaf(f[j], f[j], ss);
+                    }
+                    float4* d4 = reinterpret_cast<float4*>(dst + (size_t)i * V);
+#pragma unroll
+                    for (int q = 0; q < V / 4; ++q) d4[q] = make_float4(f[4 * q], f[4 * q + 1], f[4 * q + 2], f[4 * q + 3]);
+                }
+            }
+        }
+    } else {
+        for (int k = threadIdx.x; k < n; k += kStreamThreads) {
+            const float v = Storage<T>::load(src, k);
+            dst[k] = v;
+            if (SQ) ss = fmaf(v, v, ss);
+        }
+    }
+    return ss;
+}
+
+// dst[k] = dst[k] * rs * gamma[k] for k < n (dst shared, gamma global storage type), with
+// the gains read as 16-byte vectors, 8 in flight per thread, when aligned.
+template <typename T>
+__device__ __forceinline__ void scale_span(const T* __restrict__ gamma, float* dst, int n, float rs) {
+    constexpr int V = Vec16<T>::kN;
+    constexpr int U = 8;
+    const bool vec = ((reinterpret_cast<uintptr_t>(gamma) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0 && n % V == 0;
+    if (vec) {
+        const uint4* g4 = reinterpret_cast<const uint4*>(gamma);
+        const int nv = n / V;
+        for (int base = threadIdx.x; base < nv; base += kStreamThreads * U) {
+            uint4 r[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * kStreamThreads;
+                r[u] = i < nv ? g4[i] : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int i = base + u * kStreamThreads;
+                if (i < nv) {
+                    float f[V];
+                    Vec16<T>::widen(r[u], f);
+                    float* d = dst + (size_t)i * V;
+#pragma unroll
+                    for (int j = 0; j < V; ++j) d[j] = d[j] * rs * f[j];
+                }
+            }
+        }
+    } else {
+        for (int k = threadIdx.x; k < n; k += kStreamThreads) dst[k] = dst[k] * rs * Storage<T>::load(gamma, k);
+    }
+}
+
 template <typename WT>
 __device__ void stage_activations(const ProParams& p, int K, float* X, int Kpad, int b0, int nb, int* status,
                                   float* scratch /* >= kWarps floats */) {
-    using S = Storage<WT>;
     const int t = threadIdx.x;
     for (int b = 0; b < nb; ++b) {
         const int row = b0 + b;
         float* Xb = X + (size_t)b * Kpad;
         if (p.pro == PRO_F32) {
-            const float* xr = (const float*)p.x + (size_t)row * p.ldx;
-            for (int k = t; k < K; k += kStreamThreads) Xb[k] = xr[k];
+            stage_span<float, false>((const float*)p.x + (size_t)row * p.ldx, Xb, K);
         } else if (p.pro == PRO_STORAGE) {
-            const WT* xr = (const WT*)p.x + (size_t)row * p.ldx;
-            for (int k = t; k < K; k += kStreamThreads) Xb[k] = S::load(xr, k);
+            stage_span<WT, false>((const WT*)p.x + (size_t)row * p.ldx, Xb, K);
         } else if (p.pro == PRO_CONCAT_EMB) {
-            const float* xr = (const float*)p.x + (size_t)row * p.ldx;
             int tok = p.tok[row];
             if (tok < 0 || tok >= p.vocab) {
                 if (t == 0) atomicOr(status, ST_DEVICE);
                 tok = -1;
             }
             const int de = K - p.d_split;
-            const WT* er = (const WT*)p.embed + (size_t)(tok < 0 ? 0 : tok) * de;
-            for (int k = t; k < K; k += kStreamThreads)
-                Xb[k] = k < p.d_split ? xr[k] : (tok < 0 ? 0.f : S::load(er, k - p.d_split));
+            stage_span<float, false>((const float*)p.x + (size_t)row * p.ldx, Xb, p.d_split);
+            if (tok >= 0)
+                stage_span<WT, false>((const WT*)p.embed + (size_t)tok * de, Xb + p.d_split, de);
+            else
+                for (int k = t; k < de; k += kStreamThreads) Xb[p.d_split + k] = 0.f;
         } else {  // PRO_RMSNORM
-            const float* xr = (const float*)p.x + (size_t)row * p.ldx;
-            float ss = 0.f;
-            for (int k = t; k < K; k += kStreamThreads) {
-                const float v = xr[k];
-                Xb[k] = v;
-                ss = fmaf(v, v, ss);
-            }
+            float ss = stage_span<float, true>((const float*)p.x + (size_t)row * p.ldx, Xb, K);
             ss = warp_sum(ss);
             if ((t & 31) == 0) scratch[t >> 5] = ss;
             __syncthreads();
@@ -335,8 +410,7 @@ __device__ void stage_activations(const ProParams& p, int K, float* X, int Kpad,
 #pragma unroll
             for (int w = 0; w < kWarps; ++w) tot += scratch[w];
             const float rs = 1.0f / sqrtf(tot / (float)K + p.eps);
-            const WT* gm = (const WT*)p.gamma;
-            for (int k = t; k < K; k += kStreamThreads) Xb[k] = Xb[k] * rs * S::load(gm, k);
+            scale_span<WT>((const WT*)p.gamma, Xb, K, rs);
             __syncthreads();  // scratch reuse by the next row
         }
     }

@@ -60,3 +60,9 @@ def test_host_side_validation_needs_no_gpu(lib):
     assert so.fe_last_device_status(None, None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_launch_count(None, 1, 1) == -1
     so.fe_free(None)  # no-op
+
+
+def test_profile_entry_point_validates_on_host(lib):
+    so = lib._lib
+    n = ctypes.c_int32(0)
+    assert so.fe_profile_forward(None, None, None, 8, None, None, ctypes.byref(n)) == lib.FE_ERR_INVALID_ARG

@@ -1,0 +1,38 @@
+"""fe_profile_forward: the launch-by-launch timing that bench.py's per-kernel roofline
+uses. It must run the same kernels as fe_draft_forward (same outputs, bit for bit) and
+report one entry per launch in launch order."""
+import pytest
+import torch
+
+from fe_synth import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("spec", [dict(name="tiny"),
+                                  dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376,
+                                                 vocab=5003, n_layers=3, dtype="bf16", B=2, prefix=40, top_k=8,
+                                                 rope_theta=1e4, seed=41, page_size=0))])
+def test_profile_forward_matches_forward(spec):
+    import paper_2509_20416_gb300 as fe
+    cfg = wl.make_config(spec["name"])
+    W, I = wl.make_weights(cfg), wl.make_inputs(cfg)
+    ks, vs = wl.make_caches(cfg)
+    h = fe.fe_draft_init(dict(cfg, max_batch=cfg["B"]), W)
+    args = (I["feat"].cuda(), I["next_tok"].cuda(), I["prefix_len"].cuda(), [t.cuda() for t in ks],
+            [t.cuda() for t in vs], cfg["top_k"], cfg["temperature"])
+    ref = fe.fe_draft_forward(h, *args)
+    out = fe.alloc_outputs(h, cfg["B"], cfg["top_k"])
+    prof = fe.fe_profile_forward(h, *args, out=out)
+    torch.cuda.synchronize()
+    assert fe.fe_last_device_status(h) == fe.FE_OK
+    for key in ref:
+        assert torch.equal(ref[key], out[key]), key
+    N = cfg["n_layers"]
+    kinds = [k for k, _ in prof]
+    assert len(prof) == fe.fe_launch_count(h, cfg["B"], False)
+    assert kinds[:2] == ["linear", "linear"]
+    assert kinds[2:2 + 5 * N] == ["linear", "attention", "linear", "linear", "linear"] * N
+    assert kinds[-1] == "lm_head"
+    assert all(us > 0 for _, us in prof)
+    h.close()
