@@ -346,34 +346,101 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    for (int idx = t; idx < G * HD; idx += blockDim.x) {
-        const int hh = idx / HD, dd = idx % HD;
-        const float* pb = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split) * (HD + 2);
-        float M = -INFINITY;
-        for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
-        float v = 0.f, L = 0.f;
-        for (int q = 0; q < n_act; ++q) {
-            const float* p = pb + (size_t)q * (HD + 2);
-            const float mq = __ldcg(p + HD);
-            if (mq == -INFINITY) continue;
-            const float f = expf(mq - M);
-            v = fmaf(f, __ldcg(p + dd), v);
-            L = fmaf(f, __ldcg(p + HD + 1), L);
+    // Each split's (max, sum) per head goes to shared memory (the K/V slots are free now) in
+    // one round trip; each head's weights exp(M_q - M) are formed there; each output then
+    // sums its splits with eight loads in flight (a load-then-accumulate loop would wait a
+    // full L2 round trip per split).
+    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * (HD + 2);
+    float* wq = reinterpret_cast<float*>(dsm);  // [n_act][G] weights, then [n_act][G] sums
+    float* lq = wq + n_act * G;
+    __shared__ float hl[G];
+    if ((size_t)2 * n_act * G * sizeof(float) <= (size_t)kAttnWarps * S * 2 * CHB) {
+        for (int idx = t; idx < n_act * G; idx += blockDim.x) {
+            const int q = idx / G, hh = idx % G;
+            const float* p = pb0 + ((size_t)hh * a.n_split + q) * (HD + 2) + HD;
+            wq[idx] = __ldcg(p);
+            lq[idx] = __ldcg(p + 1);
         }
-        out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
+        __syncthreads();
+        for (int hh = warp; hh < G; hh += kAttnWarps) {
+            float M = -INFINITY;
+            for (int q = lane; q < n_act; q += 32) M = fmaxf(M, wq[q * G + hh]);
+            M = warp_max(M);
+            float L = 0.f;
+            for (int q = lane; q < n_act; q += 32) {
+                const float mq = wq[q * G + hh];
+                const float f = mq == -INFINITY ? 0.f : expf(mq - M);
+                wq[q * G + hh] = f;
+                L = fmaf(f, lq[q * G + hh], L);
+            }
+            L = warp_sum(L);
+            if (lane == 0) hl[hh] = L;
+        }
+        __syncthreads();
+        // thread t owns outputs t, t + 128, ... (NO of them) and loads QB splits of each at once
+        constexpr int NO = (G * HD + kAttnWarps * 32 - 1) / (kAttnWarps * 32);
+        constexpr int QB = NO >= 32 ? 1 : 32 / NO;
+        float v[NO];
+#pragma unroll
+        for (int o = 0; o < NO; ++o) v[o] = 0.f;
+        for (int q0 = 0; q0 < n_act; q0 += QB) {
+            float x[NO][QB];
+#pragma unroll
+            for (int o = 0; o < NO; ++o) {
+                const int idx = t + o * kAttnWarps * 32, hh = idx / HD, dd = idx % HD;
+                const float* p = pb0 + (size_t)hh * a.n_split * (HD + 2) + dd;
+#pragma unroll
+                for (int u = 0; u < QB; ++u)
+                    x[o][u] = idx < G * HD && q0 + u < n_act ? __ldcg(p + (size_t)(q0 + u) * (HD + 2)) : 0.f;
+            }
+#pragma unroll
+            for (int o = 0; o < NO; ++o) {
+                const int idx = t + o * kAttnWarps * 32, hh = (idx / HD) % G;
+#pragma unroll
+                for (int u = 0; u < QB; ++u)
+                    if (q0 + u < n_act) v[o] = fmaf(wq[(q0 + u) * G + hh], x[o][u], v[o]);
+            }
+        }
+#pragma unroll
+        for (int o = 0; o < NO; ++o) {
+            const int idx = t + o * kAttnWarps * 32;
+            if (idx < G * HD) {
+                const int hh = idx / HD, dd = idx % HD;
+                out[(size_t)hh * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
+            }
+        }
+    } else {  // more splits than the slots hold: the same sums, one split at a time
+        for (int idx = t; idx < G * HD; idx += blockDim.x) {
+            const int hh = idx / HD, dd = idx % HD;
+            const float* pb = pb0 + (size_t)hh * a.n_split * (HD + 2);
+            float M = -INFINITY;
+            for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
+            float v = 0.f, L = 0.f;
+            for (int q = 0; q < n_act; ++q) {
+                const float* p = pb + (size_t)q * (HD + 2);
+                const float mq = __ldcg(p + HD);
+                if (mq == -INFINITY) continue;
+                const float f = expf(mq - M);
+                v = fmaf(f, __ldcg(p + dd), v);
+                L = fmaf(f, __ldcg(p + HD + 1), L);
+            }
+            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
+        }
     }
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
 // Keys per work item: aim at ~4 CTAs per SM over all (sequence, KV head) pairs, in whole
-// chunks of 32 keys, at least 64 keys.
+// multiples of one chunk per warp (128 keys), so that every warp of a CTA has work and the
+// last split's combine has few partials to read.
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev) {
+    constexpr int unit = kAttnWarps * kChunkKeys;
     const int items = B * Hkv;
     int per = (4 * dev.num_sms + items - 1) / items;  // splits per (sequence, KV head)
     if (per < 1) per = 1;
     int split = (max_seq + per - 1) / per;
-    split = ((split + kChunkKeys - 1) / kChunkKeys) * kChunkKeys;
-    return split < 2 * kChunkKeys ? 2 * kChunkKeys : split;
+    split = ((split + unit - 1) / unit) * unit;
+    return split < unit ? unit : split;
 }
 
 // Pipeline slots per warp: two when a warp has more than one chunk and a chunk of K (or

@@ -33,6 +33,155 @@ __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
     return va > vb || (va == vb && ia < ib);
 }
 
+// ---- exact top-k of a candidate list, by one warp ------------------------------------------
+// A lone warp scanning shared memory pays a full load latency per dependent step, so the
+// selection keeps the dependent steps few: one pass for each lane's best (value, id); the
+// k-th largest of the 32 lane bests as a threshold T (k candidates are >= T, so the k best
+// are too); one pass compacting the candidates >= T (ballot, no atomics); then k rounds of
+// a warp arg-max over survivors held in registers. Order: larger value first, then smaller id.
+constexpr int kSelPerLane = kMergeCap / 32;
+
+__device__ __forceinline__ void warp_argmax(float& v, int& id) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, id, o);
+        if (better(ov, oi, v, id)) { v = ov; id = oi; }
+    }
+}
+
+// The k-th largest (1 <= k <= 32) of the warp's 32 values: a descending bitonic sort
+// across the lanes, then lane k - 1's value.
+__device__ __forceinline__ float warp_kth_largest(float x, int k) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const float y = __shfl_xor_sync(0xffffffffu, x, stride);
+            const bool desc = (lane & size) == 0, low = (lane & stride) == 0;
+            x = (low == desc) ? fmaxf(x, y) : fminf(x, y);
+        }
+    }
+    return __shfl_sync(0xffffffffu, x, k - 1);
+}
+
+// Top-k of n candidates vals[j] with ids ids[j] (or id_base + j when ids is null), in
+// shared memory; sv / si: this warp's scratch of kMergeCap entries. Calls out(q, value, id)
+// on lane 0 for q < k; past the finite candidates the value is -inf and the id INT_MAX.
+// With STATS, also returns (max, sum of exp(x - max)) of x = value * inv_temp over the
+// finite candidates (all lanes). vals may be overwritten.
+template <bool STATS, typename Out>
+__device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_base, int n, int k, float inv_temp,
+                                            float* sv, int* si, Out&& out) {
+    const int lane = threadIdx.x & 31;
+    constexpr int U = 4;
+    float lv = -INFINITY, m = -INFINITY, sum = 0.f;
+    int li = INT_MAX;
+    for (int j0 = 0; j0 < n; j0 += 32 * U) {
+        float v[U];
+        int id[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int j = j0 + 32 * u + lane;
+            v[u] = j < n ? vals[j] : -INFINITY;
+            id[u] = j < n ? (ids ? ids[j] : id_base + j) : INT_MAX;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (better(v[u], id[u], lv, li)) { lv = v[u]; li = id[u]; }
+            if (STATS && v[u] != -INFINITY) {
+                const float x = v[u] * inv_temp;
+                if (x > m) { sum = sum * expf(m - x) + 1.f; m = x; }
+                else sum += expf(x - m);
+            }
+        }
+    }
+    if (STATS) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float om = __shfl_xor_sync(0xffffffffu, m, o), os = __shfl_xor_sync(0xffffffffu, sum, o);
+            const float nm = fmaxf(m, om);
+            sum = (m == -INFINITY ? 0.f : sum * expf(m - nm)) + (om == -INFINITY ? 0.f : os * expf(om - nm));
+            m = nm;
+        }
+    }
+    const float T = warp_kth_largest(lv, k);
+    int cnt = 0;
+    for (int j0 = 0; j0 < n; j0 += 32 * U) {
+        float v[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int j = j0 + 32 * u + lane;
+            v[u] = j < n ? vals[j] : -INFINITY;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int j = j0 + 32 * u + lane;
+            const bool p = j < n && v[u] >= T;
+            const unsigned bal = __ballot_sync(0xffffffffu, p);
+            const int pos = cnt + __popc(bal & ((1u << lane) - 1u));
+            if (p && pos < kMergeCap) { sv[pos] = v[u]; si[pos] = ids ? ids[j] : id_base + j; }
+            cnt += __popc(bal);
+        }
+    }
+    __syncwarp();
+    if (cnt <= kMergeCap) {
+        float rv[kSelPerLane];
+        int ri[kSelPerLane];
+        float bv = -INFINITY;
+        int bi = INT_MAX;
+#pragma unroll
+        for (int q = 0; q < kSelPerLane; ++q) {
+            const int j = lane + 32 * q;
+            rv[q] = j < cnt ? sv[j] : -INFINITY;
+            ri[q] = j < cnt ? si[j] : INT_MAX;
+            if (better(rv[q], ri[q], bv, bi)) { bv = rv[q]; bi = ri[q]; }
+        }
+        for (int r = 0; r < k; ++r) {
+            float wv = bv;
+            int wi = bi;
+            warp_argmax(wv, wi);
+            if (lane == 0) out(r, wv, wv == -INFINITY ? INT_MAX : wi);
+            if (wi == bi && wv == bv) {  // this lane held the winner: drop it, find its next best
+                bv = -INFINITY;
+                bi = INT_MAX;
+#pragma unroll
+                for (int q = 0; q < kSelPerLane; ++q) {
+                    if (ri[q] == wi && rv[q] == wv) { rv[q] = -INFINITY; ri[q] = INT_MAX; }
+                    if (better(rv[q], ri[q], bv, bi)) { bv = rv[q]; bi = ri[q]; }
+                }
+            }
+        }
+    } else {  // too many ties at T to hold: rounds over all candidates, marking the taken ones
+        float bv = -INFINITY;
+        int bi = INT_MAX, bp = -1;
+        auto rescan = [&]() {
+            bv = -INFINITY;
+            bi = INT_MAX;
+            bp = -1;
+            for (int j = lane; j < n; j += 32) {
+                const float v = vals[j];
+                const int id = ids ? ids[j] : id_base + j;
+                if (bp < 0 || better(v, id, bv, bi)) { bv = v; bi = id; bp = j; }
+            }
+        };
+        rescan();
+        for (int r = 0; r < k; ++r) {
+            float wv = bv;
+            int wi = bi;
+            warp_argmax(wv, wi);
+            if (lane == 0) out(r, wv, wv == -INFINITY ? INT_MAX : wi);
+            if (bp >= 0 && wi == bi && wv == bv) {
+                vals[bp] = -INFINITY;
+                rescan();
+            }
+            __syncwarp();
+        }
+    }
+    return make_float2(m, sum);
+}
+
 struct TopkState {
     int id[kLmTile][kMaxTopK];
     float val[kLmTile][kMaxTopK];
@@ -180,7 +329,6 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
             const float* pm = bm_ + (size_t)rr * ns * 2;
             float* sv = (float*)(buf + warp * per_warp);
             int* si = (int*)(sv + kMergeCap);
-            int* scount = si + kMergeCap;
             float M = -INFINITY;
             for (int j = lane; j < ns; j += 32) M = fmaxf(M, pm[2 * j]);
             M = warp_max(M);
@@ -189,47 +337,13 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
                 if (pm[2 * j + 1] > 0.f) S += pm[2 * j + 1] * expf(pm[2 * j] - M);
             S = warp_sum(S);
             const float lse = M + logf(S);
-            float tau = -INFINITY;
-            for (int j = lane; j < ns; j += 32) tau = fmaxf(tau, pv[(size_t)j * k + k - 1]);
-            tau = warp_max(tau);
-            if (lane == 0) *scount = 0;
-            __syncwarp();
-            bool overflow = false;
-            for (int q = lane; q < ns * k; q += 32) {
-                if (pv[q] < tau) continue;
-                const int pos = atomicAdd(scount, 1);
-                if (pos < kMergeCap) { sv[pos] = pv[q]; si[pos] = pi[q]; }
-                else overflow = true;
-            }
-            overflow = __any_sync(0xffffffffu, overflow);
-            __syncwarp();
-            // candidates: the survivors, or every staged candidate if there were too many
-            float* cv = overflow ? pv : sv;
-            int* ci = overflow ? pi : si;
-            const int n = overflow ? ns * k : min(*scount, kMergeCap);
             const int i = zr / a.B, b = zr % a.B;
             const size_t ob = ((size_t)b * a.N + i) * k;
-            for (int r = 0; r < k; ++r) {
-                float bv = -INFINITY;
-                int bi = INT_MAX, bp = -1;
-                for (int j = lane; j < n; j += 32) {
-                    if (bp < 0 || better(cv[j], ci[j], bv, bi)) { bv = cv[j]; bi = ci[j]; bp = j; }
-                }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                    const int op = __shfl_xor_sync(0xffffffffu, bp, o);
-                    if (op >= 0 && (bp < 0 || better(ov, oi, bv, bi))) { bv = ov; bi = oi; bp = op; }
-                }
-                if (lane == 0) {
-                    a.topk_id[ob + r] = bi;
-                    a.topk_logit[ob + r] = bv;
-                    a.topk_prob[ob + r] = expf(bv * a.inv_temp - lse);
-                    if (bp >= 0) { cv[bp] = -INFINITY; ci[bp] = INT_MAX; }  // taken
-                }
-                __syncwarp();
-            }
+            warp_topk<false>(pv, pi, 0, ns * k, k, a.inv_temp, sv, si, [&](int q, float v, int id) {
+                a.topk_id[ob + q] = id;
+                a.topk_logit[ob + q] = v;
+                a.topk_prob[ob + q] = v == -INFINITY ? 0.f : expf(v * a.inv_temp - lse);
+            });
             if (lane == 0) a.lse[(size_t)b * a.N + i] = lse;
         }
         __syncthreads();
@@ -513,51 +627,23 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     tc_fence_after();
     if (warp == 0) tc_dealloc(tmem, tmem_cols);
 
-    // ---- this slab's partial per row (warp w: rows w, w + 6, ..): statistics and top-k
+    // ---- this slab's partial per row (warp w: rows w, w + 6, ..): statistics and top-k;
+    // the ring is free now and holds each warp's selection scratch
     {
         const int n = (t1 - t0) * 128;
         const int first = t0 * 128;
+        float* sv = (float*)(ring + (size_t)warp * kMergeCap * 8);
+        int* si = (int*)(sv + kMergeCap);
         for (int r = warp; r < R; r += kMmaThreads / 32) {
-            float* sb = slab + (size_t)r * slab_cap;
-            float M = -INFINITY;
-            for (int j = lane; j < n; j += 32) M = fmaxf(M, sb[j] * a.inv_temp);
-            M = warp_max(M);
-            float Ssum = 0.f;
-            for (int j = lane; j < n; j += 32)
-                if (sb[j] != -INFINITY) Ssum += expf(sb[j] * a.inv_temp - M);
-            Ssum = warp_sum(Ssum);
-            // each lane's best among its strided entries; ascending j keeps the smaller id on ties
-            float lv = -INFINITY;
-            int lp = -1;
-            for (int j = lane; j < n; j += 32)
-                if (lp < 0 || sb[j] > lv) { lv = sb[j]; lp = j; }
             const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
-            for (int jj = 0; jj < k; ++jj) {
-                float bv = lv;
-                int bp = lp;
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                    const int op = __shfl_xor_sync(0xffffffffu, bp, o);
-                    if (op >= 0 && (bp < 0 || better(ov, op, bv, bp))) { bv = ov; bp = op; }
-                }
-                const bool ok = bp >= 0 && bv != -INFINITY;
-                if (lane == 0) {
-                    a.part_id[base * k + jj] = ok ? first + bp : INT_MAX;
-                    a.part_val[base * k + jj] = ok ? bv : -INFINITY;
-                }
-                if (ok && (bp & 31) == lane) {  // the winner's lane removes it and rescans its entries
-                    sb[bp] = -INFINITY;
-                    lv = -INFINITY;
-                    lp = -1;
-                    for (int j = lane; j < n; j += 32)
-                        if (lp < 0 || sb[j] > lv) { lv = sb[j]; lp = j; }
-                }
-                __syncwarp();
-            }
+            const float2 ms = warp_topk<true>(slab + (size_t)r * slab_cap, nullptr, first, n, k, a.inv_temp, sv, si,
+                                              [&](int q, float v, int id) {
+                                                  a.part_id[base * k + q] = id;
+                                                  a.part_val[base * k + q] = v;
+                                              });
             if (lane == 0) {
-                a.part_ms[base * 2 + 0] = M;
-                a.part_ms[base * 2 + 1] = Ssum;
+                a.part_ms[base * 2 + 0] = ms.x;
+                a.part_ms[base * 2 + 1] = ms.y;
             }
         }
     }
