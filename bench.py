@@ -50,7 +50,14 @@ def parse():
 # DRAM traffic of the dominant kernel family from an ncu capture (dram__bytes_read.sum +
 # dram__bytes_write.sum over the linear launches of one draft of this workload), with the
 # SHA-256 of the kernel sources it was taken on: a changed kernel reports traffic null.
-TRAFFIC = {}
+TRAFFIC = {
+    # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum
+    #     -k regex:linear_kernel -s 18 -c 6 on `bench.py --set n_layers=1` (one draft's six
+    # linear launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down); the five-layer draft
+    # repeats the four per-layer launches five times with the same shapes.
+    "vic13b": {"bytes_per_draft": 160491008 + 105316864 + 5 * (157492480 + 52532480 + 283694080 + 141830656),
+               "src": "42b9bf7bf13086c0"},
+}
 KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
 
 

@@ -186,7 +186,8 @@ typedef enum {
     FE_KERNEL_ATTENTION = 1, /* RoPE + K/V append + decode attention of one layer */
     FE_KERNEL_LM_PREP = 2,   /* tensor-core LM head: RMSNorm of the hidden rows into its bf16 operand */
     FE_KERNEL_LM_HEAD = 3,   /* LM head + softmax statistics + top-k (and its merge) */
-    FE_KERNEL_COPY = 4       /* the dbg_hidden copy */
+    FE_KERNEL_COPY = 4,      /* the dbg_hidden copy */
+    FE_KERNEL_LINEAR_PREP = 5 /* tensor-core linear phase: prologue into its bf16 operand */
 } fe_kernel_kind;
 
 /* Measurement aid: runs one draft exactly as fe_draft_forward computes it, but launched

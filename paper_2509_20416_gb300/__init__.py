@@ -186,7 +186,7 @@ def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, to
     return out
 
 
-FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "copy"}
+FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "copy", 5: "linear_prep"}
 
 
 def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,

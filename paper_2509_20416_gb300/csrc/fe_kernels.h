@@ -89,6 +89,21 @@ cudaError_t launch_linear(fe_dtype dt, const LinearArgs& a, const DeviceInfo& de
 // number of kernels launch_linear() issues for these shapes (always 1)
 inline int linear_launches() { return 1; }
 
+// ---- tensor-core linear phase (bf16 weights, batches of 1..kLinMmaMaxBatch) -------------
+// W packed by launch_pack_mma (interleaved gate/up rows for EPI_SWIGLU); xb scratch of
+// linear_mma_xb_bytes(K_max, max_batch); part of linear_mma_part_bytes(); counters:
+// 4 * ceil(M_max / 128) ints, zero between calls. Two kernels: operand prep + product.
+constexpr int kLinMmaMaxBatch = 32;
+int linear_mma_bpad(int B);
+bool linear_mma_ok(int M, int K, int B);
+size_t linear_mma_xb_bytes(int K, int B);
+size_t linear_mma_part_bytes(int B, const DeviceInfo& dev);
+int linear_mma_grid(int M, int K, const DeviceInfo& dev);
+cudaError_t linear_mma_prepare(const DeviceInfo& dev);
+// after_prep (optional): an event recorded on st between the two kernels it launches
+cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, int* counters, const DeviceInfo& dev,
+                              cudaStream_t st, cudaEvent_t after_prep = nullptr);
+
 // ---- LM head + fused softmax statistics + per-slab top-k ------------------------------
 struct LmHeadArgs {
     const void* W;  // lm_head, tile-packed [ceil(V/4)*4, d]
@@ -128,6 +143,16 @@ cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);
 // after_prep (optional): an event recorded on st between the two kernels it launches
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
                               cudaEvent_t after_prep = nullptr);
+
+// wide tensor-core LM head (bf16, 16 < R <= 256 rows, top_k <= 16, d % 64 == 0): the same
+// packed W, z rounded to bf16 (zb of lmhead_wide_zb_bytes()), n_slabs = lmhead_wide_slabs()
+// CTAs; three kernels (operand prep, product + per-slab top-k, per-row merge)
+bool lmhead_wide_ok(const LmHeadArgs& a);
+size_t lmhead_wide_zb_bytes(int R, int d);
+int lmhead_wide_slabs(int V, const DeviceInfo& dev);
+cudaError_t lmhead_wide_prepare(const DeviceInfo& dev);
+cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
+                               cudaEvent_t after_prep = nullptr, cudaEvent_t after_main = nullptr);
 
 // Read-only view of what a handle holds for its LM head (for entry points outside
 // fe_runtime.cu). Returns false for a null handle.

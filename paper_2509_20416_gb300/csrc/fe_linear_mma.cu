@@ -1,0 +1,384 @@
+// Linear phases of the cascade on the tensor cores (tcgen05 + TMEM), for batches of
+// sequences: Y[b, m] = epilogue(sum_k W[m, k] X[b, k]) for b < B (Eq. 1 FCs; QKV, O-proj,
+// gate/up and down projections of every layer L_i, Eq. 2).
+//
+// At batch 1 a linear phase is a matrix-vector product and the CUDA-core streaming kernel
+// (fe_linear.cu) is the right tool. With many sequences it re-reads the weights once per
+// batch tile; here every weight is read once for the whole batch and the products run on
+// the tensor cores:
+//   - xprep_kernel applies the phase's prologue (RMSNorm, concat with the token embedding,
+//     storage or float32 input) and writes the activations as a bf16 B operand split into
+//     hi and lo parts (x = hi + lo to ~16 significant bits, so the products keep float32
+//     accuracy): rows [0, B_pad) hold hi, [B_pad, 2 B_pad) hold lo, in the 128-byte-
+//     swizzled K-major layout of fe_tc.cuh, one 2 B_pad x 64 block per 64 columns.
+//   - linear_mma_kernel: the weights are packed at init in 128 x 64 swizzled blocks
+//     (fe_pack.cu), so one TMA bulk copy lands one A operand. The (tile of 128 output rows,
+//     64-column block) units are split evenly over the CTAs in tile-major order (stream-K),
+//     so every SM streams the same number of bytes whatever the matrix shape. Warp 4 issues
+//     the copies (weights block + activation block per stage, a ring of S stages), warp 5
+//     issues tcgen05.mma (M = 128, N = 2 B_pad, K = 16; float32 accumulators in TMEM, two
+//     buffers), warps 0-3 read TMEM (thread = output row) and add hi + lo.
+//   - A tile whose units all fall in one CTA is finished there. A tile split between CTAs
+//     leaves one float32 partial per CTA in global scratch; the last CTA to finish its
+//     share of the tile (an atomic counter) sums the partials in CTA order (so results do
+//     not depend on timing) and applies the epilogue: store, residual add (+ copy into the
+//     hidden-state buffer), or SwiGLU over the interleaved gate/up rows (the partner row
+//     sits in the neighbouring lane).
+#include "fe_kernels.h"
+#include "fe_stream.cuh"
+#include "fe_tc.cuh"
+
+namespace fe {
+
+namespace {
+
+constexpr int kLmThreads = 192;  // 4 epilogue warps, 1 producer warp, 1 MMA warp
+constexpr int kLinMaxStages = 8;
+
+struct LinMmaState {
+    uint64_t full[kLinMaxStages], empty[kLinMaxStages], tfull[2], tempty[2];
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ void split_bf16(float z, uint16_t& hi, uint16_t& lo) {
+    hi = f32_to_bf16(z);
+    lo = f32_to_bf16(z - bf16_to_f32(hi));
+}
+
+}  // namespace
+
+// ---- activation operand ------------------------------------------------------------------
+// One CTA per operand row b < B_pad (rows b >= B are zero). Reads what the previous kernel
+// wrote only after griddep_wait(), through L2, and never through a __restrict__ pointer.
+__global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
+    const int b = blockIdx.x, t = threadIdx.x;
+    const int N = 2 * B_pad, K = a.K, nc = K / 8;
+    __shared__ float red[8];
+    griddep_launch_dependents();
+    griddep_wait();
+    const bool live = b < a.B;
+    int tok = 0;
+    if (live && a.pro == PRO_CONCAT_EMB) {
+        tok = a.tok[b];
+        if (tok < 0 || tok >= a.vocab) {
+            if (t == 0) atomicOr(a.status, ST_DEVICE);
+            tok = -1;
+        }
+    }
+    const float* xf = (const float*)a.x + (size_t)b * a.ldx;
+    float rs = 1.f;
+    if (live && a.pro == PRO_RMSNORM) {
+        float ss = 0.f;
+#pragma unroll 4
+        for (int c = t; c < nc; c += 256) {
+            const float4 p = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c);
+            const float4 q = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c + 1);
+            ss += p.x * p.x + p.y * p.y + p.z * p.z + p.w * p.w + q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+        }
+        ss = warp_sum(ss);
+        if ((t & 31) == 0) red[t >> 5] = ss;
+        __syncthreads();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        rs = 1.0f / sqrtf(tot / (float)K + a.eps);
+    }
+#pragma unroll 4
+    for (int c = t; c < nc; c += 256) {
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = 0.f;
+        if (live) {
+            const int k0 = 8 * c;
+            if (a.pro == PRO_STORAGE) {
+                Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.x + (size_t)b * a.ldx + k0), v);
+            } else if (a.pro == PRO_CONCAT_EMB && k0 >= a.d_split) {
+                if (tok >= 0)
+                    Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.embed +
+                                                                         (size_t)tok * (K - a.d_split) + (k0 - a.d_split)),
+                                         v);
+            } else {  // float32 input (PRO_F32, PRO_RMSNORM, or the float part of PRO_CONCAT_EMB)
+                const float4 p = __ldcg(reinterpret_cast<const float4*>(xf + k0));
+                const float4 q = __ldcg(reinterpret_cast<const float4*>(xf + k0) + 1);
+                v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
+                if (a.pro == PRO_RMSNORM) {
+                    float g[8];
+                    Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + k0), g);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = v[e] * rs * g[e];
+                }
+            }
+        }
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+            uint16_t h0, l0, h1, l1;
+            split_bf16(v[e], h0, l0);
+            split_bf16(v[e + 1], h1, l1);
+            hi[e / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            lo[e / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+        }
+        unsigned char* blk = (unsigned char*)xb + (size_t)(c / 8) * N * 128;
+        *reinterpret_cast<uint4*>(blk + sw128_offset(b, c % 8)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(blk + sw128_offset(B_pad + b, c % 8)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    }
+}
+
+// ---- the product ---------------------------------------------------------------------------
+// first unit of CTA c when U units are split over G CTAs
+__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
+
+// the CTA whose range holds unit u
+__device__ __forceinline__ int unit_owner(int64_t u, int64_t U, int G) {
+    int c = (int)((u * G) / U);
+    while (c + 1 < G && unit_begin(c + 1, U, G) <= u) ++c;
+    while (c > 0 && unit_begin(c, U, G) > u) --c;
+    return c;
+}
+
+// Epilogue for output row m of all B sequences; v[b] is the finished dot product.
+// SwiGLU pairs rows (2j, 2j + 1) held by neighbouring lanes of one warp.
+template <int BP>
+__device__ __forceinline__ void lin_epilogue(const LinearArgs& a, int m, const float (&v)[BP]) {
+    const int lane = threadIdx.x & 31;
+    if (a.epi == EPI_SWIGLU) {
+#pragma unroll
+        for (int b = 0; b < BP; ++b) {
+            const float up = __shfl_xor_sync(0xffffffffu, v[b], 1);
+            if (b < a.B && !(lane & 1) && m + 1 < a.M) a.y[(size_t)b * a.ldy + (m >> 1)] = silu(v[b]) * up;
+        }
+        return;
+    }
+    if (m >= a.M) return;
+#pragma unroll
+    for (int b = 0; b < BP; ++b) {
+        if (b >= a.B) break;
+        float* yp = a.y + (size_t)b * a.ldy + m;
+        if (a.epi == EPI_RESID) {
+            const float nv = *yp + v[b];
+            *yp = nv;
+            if (a.y2) a.y2[(size_t)b * a.ldy2 + m] = nv;
+        } else {
+            *yp = v[b];
+        }
+    }
+}
+
+template <int BP>  // B_pad: 8, 16, 24 or 32
+__global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearArgs a, const uint16_t* xb, int S,
+                                                                   int stage_bytes, uint32_t tmem_cols, float* part,
+                                                                   int* counters) {
+    constexpr int N = 2 * BP;
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ LinMmaState st;
+    unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int G = gridDim.x, cta = blockIdx.x;
+    const int nkb = a.K / 64;
+    const int ntiles = (a.M + 127) / 128;
+    const int64_t U = (int64_t)ntiles * nkb;
+    const int64_t u0 = unit_begin(cta, U, G), u1 = unit_begin(cta + 1, U, G);
+    const int tile0 = (int)(u0 / nkb), tile1 = (int)((u1 - 1) / nkb);  // tiles this CTA touches
+
+    if (t == 0) {
+        for (int i = 0; i < S; ++i) {
+            mbar_init(&st.full[i], 1);
+            mbar_init(&st.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&st.tfull[i], 1);
+            mbar_init(&st.tempty[i], 4);
+        }
+        st.abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0) tc_alloc(&st.tmem_base, tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = st.tmem_base;
+    griddep_launch_dependents();
+
+    if (warp == 4) {  // ---- TMA producer
+        if (lane == 0) {
+            const int total = (int)(u1 - u0);
+            const int pre = min(S, total);
+            const uint32_t xbytes = (uint32_t)N * 128u;
+            // the weights do not depend on earlier kernels: the first stages go out at once
+            for (int it = 0; it < pre; ++it) {
+                mbar_arrive_expect_tx(&st.full[it], 16384u + xbytes);
+                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384,
+                         &st.full[it]);
+            }
+            griddep_wait();
+            for (int it = 0; it < pre; ++it)
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384,
+                         (const unsigned char*)xb + (size_t)((u0 + it) % nkb) * xbytes, xbytes, &st.full[it]);
+            for (int it = pre; it < total; ++it) {
+                const int slot = it % S;
+                if (!mbar_wait_abortable(&st.empty[slot], ((uint32_t)(it / S) & 1u) ^ 1u, a.status, &st.abort)) break;
+                unsigned char* dst = ring + (size_t)slot * stage_bytes;
+                mbar_arrive_expect_tx(&st.full[slot], 16384u + xbytes);
+                bulk_g2s(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot]);
+                bulk_g2s(dst + 16384, (const unsigned char*)xb + (size_t)((u0 + it) % nkb) * xbytes, xbytes,
+                         &st.full[slot]);
+            }
+        }
+    } else if (warp == 5) {  // ---- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, N);
+            int64_t u = u0;
+            int it = 0;
+            for (int tile = tile0, j = 0; tile <= tile1; ++tile, ++j) {
+                const int buf = j & 1;
+                const int64_t ue = min(u1, (int64_t)(tile + 1) * nkb);
+                if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * N);
+                bool ok = true;
+                for (bool first = true; u < ue; ++u, ++it, first = false) {
+                    const int slot = it % S;
+                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(ring + (size_t)slot * stage_bytes);
+                    const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + 16384);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (!first || kk) ? 1u : 0u);
+                    tc_commit(&st.empty[slot]);
+                }
+                if (!ok) break;
+                tc_commit(&st.tfull[buf]);
+            }
+        }
+    } else {  // ---- epilogue warps 0..3: TMEM lane 32 w + l = output row of the tile
+        griddep_wait();  // the epilogue reads and writes activations of earlier kernels
+        const int r = warp * 32 + lane;
+        for (int tile = tile0, j = 0; tile <= tile1; ++tile, ++j) {
+            const int buf = j & 1;
+            if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
+            tc_fence_after();
+            float acc[N];
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * N);
+#pragma unroll
+            for (int c = 0; c < N; c += 16) tc_ld16(taddr + c, acc + c);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&st.tempty[buf]);
+            float v[BP];
+#pragma unroll
+            for (int b = 0; b < BP; ++b) v[b] = acc[b] + acc[BP + b];
+            const int m = tile * 128 + r;
+            const int c_first = unit_owner((int64_t)tile * nkb, U, G);
+            const int c_last = unit_owner((int64_t)(tile + 1) * nkb - 1, U, G);
+            if (c_first == c_last) {  // the whole tile was ours
+                lin_epilogue<BP>(a, m, v);
+                continue;
+            }
+            // leave this CTA's share: slot 0 for its first tile, 1 for its last. Rows are
+            // independent, so each warp finishes its own 32 rows (its own counter): no wait
+            // on another warp.
+            const int slot = tile == tile0 ? 0 : 1;
+            float* pp = part + ((size_t)(cta * 2 + slot) * BP) * 128 + r;
+#pragma unroll
+            for (int b = 0; b < BP; ++b) pp[(size_t)b * 128] = v[b];
+            __threadfence();
+            __syncwarp();
+            int last = 0;
+            if (lane == 0) last = atomicAdd(&counters[tile * 4 + warp], 1) == c_last - c_first;
+            last = __shfl_sync(0xffffffffu, last, 0);
+            if (!last) continue;
+            __threadfence();
+            float s[BP];
+#pragma unroll
+            for (int b = 0; b < BP; ++b) s[b] = 0.f;
+            for (int c = c_first; c <= c_last; ++c) {
+                const int cs = (int)(unit_begin(c, U, G) / nkb) == tile ? 0 : 1;
+                const float* q = part + ((size_t)(c * 2 + cs) * BP) * 128 + r;
+                float x[BP];
+#pragma unroll
+                for (int b = 0; b < BP; ++b) x[b] = __ldcg(q + (size_t)b * 128);
+#pragma unroll
+                for (int b = 0; b < BP; ++b) s[b] += x[b];
+            }
+            lin_epilogue<BP>(a, m, s);
+            if (lane == 0) counters[tile * 4 + warp] = 0;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tc_dealloc(tmem, tmem_cols);
+}
+
+// ---- host side -----------------------------------------------------------------------------
+namespace {
+
+template <int BP>
+cudaError_t set_attr(const DeviceInfo& dev) {
+    return cudaFuncSetAttribute(linear_mma_kernel<BP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                dev.max_smem_optin - (int)sizeof(LinMmaState) - 256);
+}
+
+template <int BP>
+cudaError_t launch_bp(const LinearArgs& a, const uint16_t* xb, float* part, int* counters, const DeviceInfo& dev,
+                      cudaStream_t st, int grid) {
+    constexpr int N = 2 * BP;
+    const int stage_bytes = 16384 + N * 128;
+    const size_t budget = (size_t)dev.max_smem_optin - sizeof(LinMmaState) - 256 - 1024;
+    int S = (int)(budget / stage_bytes);
+    S = S > kLinMaxStages ? kLinMaxStages : S;
+    if (S < 2) return cudaErrorInvalidValue;
+    const size_t smem = 1024 + (size_t)S * stage_bytes;
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(2 * N)) cols <<= 1;
+    return launch_k(linear_mma_kernel<BP>, dim3(grid), dim3(kLmThreads), smem, st, a.pdl, a, xb, S, stage_bytes, cols,
+                    part, counters);
+}
+
+}  // namespace
+
+int linear_mma_bpad(int B) { return (B + 7) / 8 * 8; }
+
+bool linear_mma_ok(int M, int K, int B) { return M > 0 && K % 64 == 0 && B >= 1 && B <= kLinMmaMaxBatch; }
+
+size_t linear_mma_xb_bytes(int K, int B) { return (size_t)2 * linear_mma_bpad(B) * K * 2; }
+
+int linear_mma_grid(int M, int K, const DeviceInfo& dev) {
+    const int64_t U = (int64_t)((M + 127) / 128) * (K / 64);
+    return (int)(U < dev.num_sms ? U : dev.num_sms);
+}
+
+size_t linear_mma_part_bytes(int B, const DeviceInfo& dev) {
+    return (size_t)dev.num_sms * 2 * linear_mma_bpad(B) * 128 * sizeof(float);
+}
+
+cudaError_t linear_mma_prepare(const DeviceInfo& dev) {
+    cudaError_t e;
+    if ((e = set_attr<8>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<16>(dev)) != cudaSuccess) return e;
+    if ((e = set_attr<24>(dev)) != cudaSuccess) return e;
+    return set_attr<32>(dev);
+}
+
+cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, int* counters, const DeviceInfo& dev,
+                              cudaStream_t st, cudaEvent_t after_prep) {
+    if (!linear_mma_ok(a.M, a.K, a.B)) return cudaErrorInvalidValue;
+    const int BP = linear_mma_bpad(a.B);
+    cudaError_t e = launch_k(xprep_kernel, dim3(BP), dim3(256), 0, st, a.pdl, a, BP, xb);
+    if (e != cudaSuccess) return e;
+    if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
+    const int grid = linear_mma_grid(a.M, a.K, dev);
+    switch (BP) {
+        case 8: return launch_bp<8>(a, xb, part, counters, dev, st, grid);
+        case 16: return launch_bp<16>(a, xb, part, counters, dev, st, grid);
+        case 24: return launch_bp<24>(a, xb, part, counters, dev, st, grid);
+        default: return launch_bp<32>(a, xb, part, counters, dev, st, grid);
+    }
+}
+
+}  // namespace fe

@@ -432,7 +432,8 @@ constexpr int kMmaThreads = 6 * 32;
 constexpr int kMmaMaxStages = 12;
 
 // zb [d/64][N rows x 128 B] in the 128B-swizzled layout: rows [0, R_pad) hold z_hi, rows
-// [R_pad, 2 R_pad) hold z_lo; rows of padding (r >= R) are zero. One CTA per row r < R_pad;
+// [R_pad, 2 R_pad) hold z_lo (N = 2 R_pad), or, without lo, z rounded to bf16 alone
+// (N = R_pad); rows of padding (r >= R) are zero. One CTA per row r < R_pad;
 // thread t owns the 16-byte chunks (8 values) t, t + 256, ... of the row, kept in
 // registers between the sum of squares and the split (d <= kZprepMaxChunks * 8 * 256).
 constexpr int kZprepMaxChunks = 8;
@@ -443,10 +444,10 @@ template <typename WT>
 // and is deliberately not a __restrict__ pointer, whose loads the compiler may treat as
 // invariant and move above the wait.
 __global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* __restrict__ gamma, int R,
-                                                    int R_pad, int d, float eps, uint16_t* zb) {
+                                                    int R_pad, int d, float eps, uint16_t* zb, int with_lo) {
     static_assert(sizeof(WT) == 2, "the tensor-core LM head takes bf16 weights");
     const int r = blockIdx.x, t = threadIdx.x;
-    const int N = 2 * R_pad;
+    const int N = with_lo ? 2 * R_pad : R_pad;
     const int nc = d / 8;  // 16-byte chunks of a bf16 row
     __shared__ float red[8];
     // the gains do not depend on the previous kernel
@@ -499,7 +500,8 @@ __global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* 
         const int kb = c / 8, cc = c % 8;  // 64-column block, 16-byte chunk within it
         unsigned char* blk = (unsigned char*)zb + (size_t)kb * N * 128;
         *reinterpret_cast<uint4*>(blk + sw128_offset(r, cc)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(blk + sw128_offset(R_pad + r, cc)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        if (with_lo)
+            *reinterpret_cast<uint4*>(blk + sw128_offset(R_pad + r, cc)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
     }
 }
 
@@ -750,7 +752,7 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     const int R_pad = (a.R + 7) / 8 * 8;
     const int N = 2 * R_pad;
     cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
-                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb);
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 1);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
@@ -768,6 +770,316 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
     return launch_k(lmhead_mma_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb,
                     R_pad, S, stage_bytes, cols, slab_cap);
+}
+
+
+// ==== wide tensor-core LM head: up to 256 hidden rows (batched serving) =====================
+// At B sequences x N depths the LM head sees R = N * B rows (192 at B = 32, N = 6). The
+// 16-row kernel above keeps every slab logit in shared memory and splits z into bf16
+// hi + lo; neither holds at this R. Here:
+//   - z is rounded once to bf16 (N = R_pad MMA columns, R_pad <= 256); every product is
+//     accumulated in float32. The logit error this leaves is of the order of
+//     |W_v| |z| 2^-9 / sqrt(3), a few 1e-3 at d = 4096 with weights ~ N(0, 0.02^2).
+//   - TMEM holds two R_pad-column accumulators, so the epilogue of tile j overlaps the
+//     MMAs of tile j + 1.
+//   - The epilogue transposes each tile through shared memory, 64 rows at a time, so that
+//     a thread owns one hidden row r and half of the tile's 128 vocabulary entries: its
+//     softmax statistics are exact online (max, sum of exp) and its running top-k is a
+//     sorted list in registers (an entry enters only if it beats the current k-th best,
+//     ties to the smaller id), with no cross-thread reduction per tile. At the end of the
+//     slab the two halves of each row merge and write the slab's partial.
+//   - lmhead_merge_kernel (one CTA per row) then merges the slabs as merge_rows does.
+constexpr int kWideKMax = 16;     // top_k limit of this kernel (a sorted list in registers)
+constexpr int kWideRowsMax = 256;
+constexpr int kWideGroup = 64;    // rows staged per transpose round
+constexpr int kWideTileStride = kWideGroup + 1;  // floats per staged vocabulary entry (no bank conflicts)
+
+struct WideState {
+    uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2], ebar[2];
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ void wide_insert(float (&tv)[kWideKMax], int (&ti)[kWideKMax], int k, float x, int id) {
+#pragma unroll
+    for (int q = 0; q < kWideKMax; ++q) {
+        if (q < k && better(x, id, tv[q], ti[q])) {
+            const float sv = tv[q];
+            const int si = ti[q];
+            tv[q] = x;
+            ti[q] = id;
+            x = sv;
+            id = si;
+        }
+    }
+}
+
+__device__ __forceinline__ void wide_kth(const float (&tv)[kWideKMax], const int (&ti)[kWideKMax], int k, float& v,
+                                         int& id) {
+#pragma unroll
+    for (int q = 0; q < kWideKMax; ++q)
+        if (q == k - 1) { v = tv[q]; id = ti[q]; }
+}
+
+__device__ __forceinline__ void online_add(float& m, float& s, float x) {
+    if (x > m) { s = s * expf(m - x) + 1.f; m = x; }
+    else s += expf(x - m);
+}
+
+__global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
+                                                                     int S, int stage_bytes, uint32_t tmem_cols) {
+    extern __shared__ unsigned char dsm_raw[];
+    __shared__ WideState st;
+    unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    float* tbuf = (float*)(ring + (size_t)S * stage_bytes);  // [128 vocab][kWideTileStride]
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int R = a.R, k = a.top_k;
+    const int nkb = a.d / 64;
+    const int ntiles = (a.V + 127) / 128;
+    const int t0 = (int)(((int64_t)blockIdx.x * ntiles) / gridDim.x);
+    const int t1 = (int)(((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x);
+    const int ngroups = (R_pad + kWideGroup - 1) / kWideGroup;
+    const uint32_t zbytes = (uint32_t)R_pad * 128u;
+
+    if (t == 0) {
+        for (int i = 0; i < S; ++i) {
+            mbar_init(&st.full[i], 1);
+            mbar_init(&st.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&st.tfull[i], 1);
+            mbar_init(&st.tempty[i], 4);
+            mbar_init(&st.ebar[i], 4);
+        }
+        st.abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0) tc_alloc(&st.tmem_base, tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = st.tmem_base;
+    griddep_launch_dependents();
+
+    if (warp == 4) {  // ---- TMA producer
+        if (lane == 0) {
+            const int total = (t1 - t0) * nkb;
+            const int pre = min(S, total);
+            for (int it = 0; it < pre; ++it) {
+                mbar_arrive_expect_tx(&st.full[it], 16384u + zbytes);
+                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + ((size_t)t0 * nkb + it) * 16384,
+                         16384, &st.full[it]);
+            }
+            griddep_wait();
+            for (int it = 0; it < pre; ++it)
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * zbytes,
+                         zbytes, &st.full[it]);
+            for (int it = pre; it < total; ++it) {
+                const int slot = it % S;
+                if (!mbar_wait_abortable(&st.empty[slot], ((uint32_t)(it / S) & 1u) ^ 1u, a.status, &st.abort)) break;
+                unsigned char* dst = ring + (size_t)slot * stage_bytes;
+                mbar_arrive_expect_tx(&st.full[slot], 16384u + zbytes);
+                bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)t0 * nkb + it) * 16384, 16384, &st.full[slot]);
+                bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * zbytes, zbytes, &st.full[slot]);
+            }
+        }
+    } else if (warp == 5) {  // ---- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, R_pad);
+            int it = 0;
+            for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
+                const int buf = j & 1;
+                if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * R_pad);
+                bool ok = true;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int slot = it % S;
+                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(ring + (size_t)slot * stage_bytes);
+                    const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + 16384);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
+                    tc_commit(&st.empty[slot]);
+                }
+                if (!ok) break;
+                tc_commit(&st.tfull[buf]);
+            }
+        }
+    } else {  // ---- epilogue warps 0..3
+        griddep_wait();
+        const int rg = t & (kWideGroup - 1), half = t / kWideGroup;  // row within a group, vocabulary half
+        float tv[4][kWideKMax], thv[4], m[4], s[4];
+        int ti[4][kWideKMax], thi[4];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+#pragma unroll
+            for (int q = 0; q < kWideKMax; ++q) { tv[g][q] = -INFINITY; ti[g][q] = INT_MAX; }
+            thv[g] = -INFINITY;
+            thi[g] = INT_MAX;
+            m[g] = -INFINITY;
+            s[g] = 0.f;
+        }
+        uint32_t eb = 0;  // epilogue barriers passed (two mbarriers used alternately)
+        auto epi_sync = [&]() -> bool {
+            __syncwarp();
+            uint64_t* bar = &st.ebar[eb & 1];
+            if (lane == 0) mbar_arrive(bar);
+            const bool ok = mbar_wait_abortable(bar, (eb >> 1) & 1u, a.status, &st.abort);
+            ++eb;
+            return ok;
+        };
+        bool ok = true;
+        for (int tile = t0, j = 0; tile < t1 && ok; ++tile, ++j) {
+            const int buf = j & 1;
+            if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
+            tc_fence_after();
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * R_pad);
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+                if (g >= ngroups || !ok) break;
+                // stage: vocabulary entry 32 w + lane, rows [64 g, 64 g + 64) of the tile
+                float* trow = tbuf + (size_t)(warp * 32 + lane) * kWideTileStride;
+#pragma unroll
+                for (int c0 = 0; c0 < kWideGroup; c0 += 16) {
+                    if (g * kWideGroup + c0 < R_pad) {
+                        float v16[16];
+                        tc_ld16(taddr + (uint32_t)(g * kWideGroup + c0), v16);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) trow[c0 + i] = v16[i];
+                    }
+                }
+                if (g == ngroups - 1) {  // the accumulator is fully read: hand it back to the MMA warp
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&st.tempty[buf]);
+                }
+                if (!(ok = epi_sync())) break;
+                // consume: this thread's row r, vocabulary entries [64 half, 64 half + 64)
+                const int r = g * kWideGroup + rg;
+                if (r < R) {
+                    const int rb = r % a.B, ri = r / a.B;
+                    for (int v = half * 64; v < half * 64 + 64; ++v) {
+                        const int id = tile * 128 + v;
+                        if (id >= a.V) break;
+                        const float x = tbuf[(size_t)v * kWideTileStride + rg];
+                        online_add(m[g], s[g], x * a.inv_temp);
+                        if (better(x, id, thv[g], thi[g])) {
+                            wide_insert(tv[g], ti[g], k, x, id);
+                            wide_kth(tv[g], ti[g], k, thv[g], thi[g]);
+                        }
+                        if (a.dbg_logits) a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id] = x;
+                    }
+                }
+                if (!(ok = epi_sync())) break;
+            }
+        }
+        // ---- the slab's partial per row: the upper half hands its list to the lower half
+        float* xs = tbuf;  // [64][2 * kWideKMax + 2]
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            if (g >= ngroups || !ok) break;
+            float* mine = xs + (size_t)rg * (2 * kWideKMax + 2);
+            if (half == 1) {
+#pragma unroll
+                for (int q = 0; q < kWideKMax; ++q) {
+                    mine[q] = tv[g][q];
+                    mine[kWideKMax + q] = __int_as_float(ti[g][q]);
+                }
+                mine[2 * kWideKMax] = m[g];
+                mine[2 * kWideKMax + 1] = s[g];
+            }
+            if (!(ok = epi_sync())) break;
+            const int r = g * kWideGroup + rg;
+            if (half == 0 && r < R) {
+#pragma unroll
+                for (int q = 0; q < kWideKMax; ++q) {
+                    const float ov = mine[q];
+                    const int oi = __float_as_int(mine[kWideKMax + q]);
+                    if (q < k && better(ov, oi, thv[g], thi[g])) {
+                        wide_insert(tv[g], ti[g], k, ov, oi);
+                        wide_kth(tv[g], ti[g], k, thv[g], thi[g]);
+                    }
+                }
+                const float om = mine[2 * kWideKMax], os = mine[2 * kWideKMax + 1];
+                const float nm = fmaxf(m[g], om);
+                const float ns = (m[g] == -INFINITY ? 0.f : s[g] * expf(m[g] - nm)) +
+                                 (om == -INFINITY ? 0.f : os * expf(om - nm));
+                const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
+#pragma unroll
+                for (int q = 0; q < kWideKMax; ++q) {
+                    if (q < k) {
+                        a.part_id[base * k + q] = tv[g][q] == -INFINITY ? INT_MAX : ti[g][q];
+                        a.part_val[base * k + q] = tv[g][q];
+                    }
+                }
+                a.part_ms[base * 2 + 0] = nm;
+                a.part_ms[base * 2 + 1] = ns;
+            }
+            if (!(ok = epi_sync())) break;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tc_dealloc(tmem, tmem_cols);
+}
+
+// One CTA per row: merges every slab's partial of that row (merge_rows).
+__global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, size_t smem_bytes) {
+    extern __shared__ __align__(16) unsigned char msm[];
+    griddep_launch_dependents();
+    griddep_wait();
+    merge_rows(a, blockIdx.x, blockIdx.x + 1, msm, smem_bytes);
+}
+
+bool lmhead_wide_ok(const LmHeadArgs& a) {
+    return a.R > 0 && a.R <= kWideRowsMax && a.d % 64 == 0 && a.d <= kZprepMaxChunks * 8 * 256 &&
+           a.top_k >= 1 && a.top_k <= kWideKMax;
+}
+
+size_t lmhead_wide_zb_bytes(int R, int d) { return (size_t)((R + 15) / 16 * 16) * d * 2; }
+
+int lmhead_wide_slabs(int V, const DeviceInfo& dev) {
+    const int ntiles = (V + 127) / 128;
+    return ntiles < dev.num_sms ? ntiles : dev.num_sms;
+}
+
+cudaError_t lmhead_wide_prepare(const DeviceInfo& dev) {
+    cudaError_t e = cudaFuncSetAttribute(lmhead_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         dev.max_smem_optin - (int)sizeof(WideState) - 256);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+}
+
+cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
+                               cudaEvent_t after_prep, cudaEvent_t after_main) {
+    if (!lmhead_wide_ok(a) || (reinterpret_cast<uintptr_t>(a.hid) & 15)) return cudaErrorInvalidValue;
+    const int R_pad = (a.R + 15) / 16 * 16;
+    cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 0);
+    if (e != cudaSuccess) return e;
+    if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
+    const int stage_bytes = 16384 + R_pad * 128;
+    const size_t tbytes = (size_t)128 * kWideTileStride * sizeof(float);
+    const size_t budget = (size_t)dev.max_smem_optin - sizeof(WideState) - 256;
+    if (budget < 1024 + tbytes + 2 * (size_t)stage_bytes) return cudaErrorInvalidValue;
+    int S = (int)((budget - 1024 - tbytes) / stage_bytes);
+    S = S > kMmaMaxStages ? kMmaMaxStages : S;
+    const size_t smem = 1024 + (size_t)S * stage_bytes + tbytes;
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(2 * R_pad)) cols <<= 1;
+    e = launch_k(lmhead_wide_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad,
+                 S, stage_bytes, cols);
+    if (e != cudaSuccess) return e;
+    if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;
+    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k);
+    if (msmem > 64 * 1024) return cudaErrorInvalidValue;
+    return launch_k(lmhead_merge_kernel, dim3(a.R), dim3(128), msmem, st, a.pdl, a, msmem);
 }
 
 }  // namespace fe

@@ -67,6 +67,10 @@ struct fe_handle {
     int* attn_counters = nullptr;
     int* lm_counters = nullptr;
     bool lm_mma = false;      // LM head packed for (and run on) the tensor cores
+    bool lin_mma = false;     // linear phases packed for (and run on) the tensor cores
+    uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
+    float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
+    int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
     uint16_t* lm_zb = nullptr;  // tensor-core LM head: bf16 hi/lo operand of the hidden rows
     int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
     cudaStream_t cap = nullptr;
@@ -141,19 +145,20 @@ inline cudaError_t mark(Prof* pf, int kind, cudaStream_t st) {
 
 // bytes of each matrix in the tile-packed layout (rows padded to a multiple of 4); the
 // embedding and the norm gains stay in their canonical layout
-Sizes weight_sizes(const fe_config& c, size_t es) {
+Sizes weight_sizes(const fe_config& c, size_t es, bool mma) {
     const int d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
     const int e = (int)es;
+    auto pk = [&](int M, int K) { return mma ? mma_packed_bytes(M, K) : packed_bytes(M, K, e); };
     Sizes s;
-    s.w_fuse = packed_bytes(d, 3 * d, e);
-    s.w_in = packed_bytes(d, 2 * d, e);
+    s.w_fuse = pk(d, 3 * d);
+    s.w_in = pk(d, 2 * d);
     s.embed = (size_t)V * d * es;
     s.lm_head = packed_bytes(V, d, e);
     s.norm = (size_t)d * es;
-    s.qkv = packed_bytes((H + 2 * Hkv) * hd, d, e);
-    s.wo = packed_bytes(d, H * hd, e);
-    s.gu = packed_bytes(2 * F, d, e);
-    s.down = packed_bytes(d, F, e);
+    s.qkv = pk((H + 2 * Hkv) * hd, d);
+    s.wo = pk(d, H * hd);
+    s.gu = pk(2 * F, d);
+    s.down = pk(d, F);
     return s;
 }
 
@@ -164,6 +169,27 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     const fe_dtype dt = c.dtype;
     const bool pdl = h->use_pdl && !pf;  // profiled launches do not overlap
     if (pf) FE_TRY(cudaEventRecord(pf->ev[0], st));
+    // one linear phase: the CUDA-core streaming kernel, or operand prep + tensor-core product
+    auto linear = [&](const LinearArgs& L) -> fe_status {
+        cudaError_t e;
+        if (h->lin_mma) {
+            if (pf) {
+                if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
+                pf->kinds[pf->n++] = FE_KERNEL_LINEAR_PREP;
+            }
+            e = launch_linear_mma(L, h->lin_xb, h->lin_part, h->lin_counters, h->dev, st, pf ? pf->ev[pf->n] : nullptr);
+        } else {
+            e = launch_linear(dt, L, h->dev, st);
+        }
+        if (e != cudaSuccess) return fail(e, "linear phase launch", __LINE__);
+        if ((e = mark(pf, FE_KERNEL_LINEAR, st)) != cudaSuccess) return fail(e, "profiling event", __LINE__);
+        return FE_OK;
+    };
+    fe_status lrc;
+#define FE_LINEAR(L)                                \
+    do {                                            \
+        if ((lrc = linear(L)) != FE_OK) return lrc; \
+    } while (0)
 
     LinearArgs la{};
     la.status = h->status;
@@ -176,16 +202,14 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.W = h->w_fuse; la.M = d; la.K = 3 * d;
     la.pro = PRO_STORAGE; la.x = a->feat; la.ldx = 3 * d;
     la.epi = EPI_STORE; la.y = h->g; la.ldy = d; la.y2 = nullptr;
-    FE_TRY(launch_linear(dt, la, h->dev, st));
-    FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+    FE_LINEAR(la);
     la.pdl = pdl;
     // x0 = W_in concat(g, e)
     la.W = h->w_in; la.M = d; la.K = 2 * d;
     la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
     la.d_split = d; la.vocab = V;
     la.epi = EPI_STORE; la.y = h->x; la.ldy = d;
-    FE_TRY(launch_linear(dt, la, h->dev, st));
-    FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+    FE_LINEAR(la);
 
     AttnArgs aa{};
     aa.qkv = h->qkv; aa.prefix_len = a->prefix_len; aa.page_table = a->page_table;
@@ -202,8 +226,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         la.W = L.w_qkv; la.M = nqkv; la.K = d;
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.attn_norm;
         la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
-        FE_TRY(launch_linear(dt, la, h->dev, st));
-        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+        FE_LINEAR(la);
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
         FE_TRY(launch_attention(dt, aa, st));
@@ -212,20 +235,17 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         la.W = L.w_o; la.M = d; la.K = H * hd;
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr;
-        FE_TRY(launch_linear(dt, la, h->dev, st));
-        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+        FE_LINEAR(la);
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm;
         la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
-        FE_TRY(launch_linear(dt, la, h->dev, st));
-        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+        FE_LINEAR(la);
         // x += W_down a; h_i = x
         la.W = L.w_down; la.M = d; la.K = F;
         la.pro = PRO_F32; la.x = h->act; la.ldx = F;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = h->hid + (size_t)i * B * d; la.ldy2 = d;
-        FE_TRY(launch_linear(dt, la, h->dev, st));
-        FE_TRY(mark(pf, FE_KERNEL_LINEAR, st));
+        FE_LINEAR(la);
     }
 
     const float inv_temp = a->temperature > 0.f ? 1.0f / a->temperature : 1.0f;
@@ -236,7 +256,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
     lm.pdl = pdl;
-    if (h->lm_mma) {
+    if (h->lm_mma && N * B <= 16) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         if (pf) {
             if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
@@ -244,6 +264,17 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
             ++pf->n;
         }
         FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n] : nullptr));
+        FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
+    } else if (h->lm_mma) {
+        lm.n_slabs = lmhead_wide_slabs(V, h->dev);
+        if (pf) {
+            if (pf->n + 3 > pf->cap) return FE_ERR_INVALID_ARG;
+            pf->kinds[pf->n] = FE_KERNEL_LM_PREP;
+            pf->kinds[pf->n + 1] = FE_KERNEL_LM_HEAD;
+            pf->n += 2;
+        }
+        FE_TRY(launch_lmhead_wide(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n - 1] : nullptr,
+                                  pf ? pf->ev[pf->n] : nullptr));
         FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     } else {
         FE_TRY(launch_lmhead(dt, lm, h->dev, st));
@@ -255,6 +286,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         FE_TRY(mark(pf, FE_KERNEL_COPY, st));
     }
     return FE_OK;
+#undef FE_LINEAR
 }
 
 bool forward_args_ok(const fe_handle* h, const fe_forward_args* a) {
@@ -268,6 +300,7 @@ bool forward_args_ok(const fe_handle* h, const fe_forward_args* a) {
         if (!a->k_cache[i] || !a->v_cache[i]) return false;
     if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return false;
     if (!(a->temperature == a->temperature)) return false;  // NaN
+    if (h->lin_mma && (reinterpret_cast<uintptr_t>(a->feat) & 15)) return false;  // read as 16-byte vectors
     return true;
 }
 
@@ -354,9 +387,21 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         if ((rc = from_cuda(lmhead_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(attention_prepare())) != FE_OK) break;
         if ((rc = from_cuda(lmhead_mma_prepare(h->dev))) != FE_OK) break;
+        if ((rc = from_cuda(linear_mma_prepare(h->dev))) != FE_OK) break;
+        if ((rc = from_cuda(lmhead_wide_prepare(h->dev))) != FE_OK) break;
+        // the linear phases run on the tensor cores for batched handles (bf16, every K a
+        // multiple of 64, at most kLinMmaMaxBatch sequences); FE_DRAFT_LINEAR_MMA=1 / 0
+        // forces the choice where the shapes allow it
+        {
+            const fe_config& c = h->cfg;
+            const bool shapes = c.dtype == FE_BF16 && c.max_batch <= kLinMmaMaxBatch && c.d % 64 == 0 &&
+                                c.ffn % 64 == 0 && (c.n_heads * c.head_dim) % 64 == 0;
+            const char* lm = getenv("FE_DRAFT_LINEAR_MMA");
+            h->lin_mma = shapes && (lm ? lm[0] == '1' : c.max_batch > 8);
+        }
 
         // ---- packed weights: one allocation, every matrix 256-byte aligned ----
-        const Sizes sz = weight_sizes(c, h->es);
+        const Sizes sz = weight_sizes(c, h->es, h->lin_mma);
         size_t total = align256(sz.w_fuse) + align256(sz.w_in) + align256(sz.embed) +
                        std::max(align256(sz.lm_head), align256(mma_packed_bytes(c.vocab, c.d))) + align256(sz.norm);
         total += (size_t)c.n_layers *
@@ -377,11 +422,18 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                 rc = fail(_fe_e, "copy of a weight", __LINE__);
             return dst;
         };
+        // a layer matrix in the layout of the linear path in use; the LM head is packed below
+        auto pack = [&](const void* staged, void* dst, int M, int K) -> cudaError_t {
+            return h->lin_mma ? launch_pack_mma(staged, dst, M, K, st) : launch_pack_tiles(staged, dst, M, K, es, st);
+        };
+        auto packed_size = [&](int M, int K) {
+            return h->lin_mma ? mma_packed_bytes(M, K) : packed_bytes(M, K, es);
+        };
         auto put_packed = [&](const void* src, int M, int K) -> const void* {
             void* dst = p;
-            p += align256(packed_bytes(M, K, es));
+            p += align256(packed_size(M, K));
             if ((_fe_e = cudaMemcpyAsync(staging, src, (size_t)M * K * es, cudaMemcpyDefault, st)) != cudaSuccess ||
-                (_fe_e = launch_pack_tiles(staging, dst, M, K, es, st)) != cudaSuccess)
+                (_fe_e = pack(staging, dst, M, K)) != cudaSuccess)
                 rc = fail(_fe_e, "copy or packing of a weight matrix", __LINE__);
             return dst;
         };
@@ -389,10 +441,15 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->w_fuse = put_packed(w->w_fuse, dm, 3 * dm);
         h->w_in = put_packed(w->w_in, dm, 2 * dm);
         h->embed = put(w->embed, sz.embed);
-        // the LM head runs on the tensor cores when every call fits that path (bf16, at most 16
-        // hidden rows, d a multiple of 64); it is then packed in the swizzled MMA layout
-        h->lm_mma = c.dtype == FE_BF16 && (int64_t)c.n_layers * c.max_batch <= 16 && c.d % 64 == 0 && c.d <= 16384 &&
-                    !(getenv("FE_DRAFT_LMHEAD_CUDA_CORES") && getenv("FE_DRAFT_LMHEAD_CUDA_CORES")[0] == '1');
+        // the LM head runs on the tensor cores when every call fits one of their two kernels
+        // (bf16, d a multiple of 64, at most 16 hidden rows; or at most 256 rows with
+        // top_k_max <= 16); it is then packed in the swizzled MMA layout
+        {
+            const int64_t rmax = (int64_t)c.n_layers * c.max_batch;
+            h->lm_mma = c.dtype == FE_BF16 && c.d % 64 == 0 && c.d <= 16384 &&
+                        (rmax <= 16 || (rmax <= 256 && c.top_k_max <= 16)) &&
+                        !(getenv("FE_DRAFT_LMHEAD_CUDA_CORES") && getenv("FE_DRAFT_LMHEAD_CUDA_CORES")[0] == '1');
+        }
         if (h->lm_mma) {
             void* dst = p;
             p += align256(mma_packed_bytes(c.vocab, dm));
@@ -402,7 +459,13 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                 rc = fail(_fe_e, "copy or packing of the LM head", __LINE__);
             h->lm_head = dst;
         } else {
-            h->lm_head = put_packed(w->lm_head, c.vocab, dm);
+            void* dst = p;
+            p += align256(packed_bytes(c.vocab, dm, es));
+            if ((_fe_e = cudaMemcpyAsync(staging, w->lm_head, (size_t)c.vocab * dm * es, cudaMemcpyDefault, st)) !=
+                    cudaSuccess ||
+                (_fe_e = launch_pack_tiles(staging, dst, c.vocab, dm, es, st)) != cudaSuccess)
+                rc = fail(_fe_e, "copy or packing of the LM head", __LINE__);
+            h->lm_head = dst;
         }
         h->final_norm = put(w->final_norm, sz.norm);
         h->layers.resize(c.n_layers);
@@ -421,7 +484,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                     cudaSuccess ||
                 cudaMemcpy2DAsync((char*)staging + rowb, 2 * rowb, L.w_up, rowb, rowb, c.ffn, cudaMemcpyDefault,
                                   st) != cudaSuccess ||
-                launch_pack_tiles(staging, gu, 2 * c.ffn, dm, es, st) != cudaSuccess)
+                pack(staging, gu, 2 * c.ffn, dm) != cudaSuccess)
                 rc = fail(cudaGetLastError(), "interleave or packing of gate/up", __LINE__);
             P.w_gu = gu;
             P.w_down = put_packed(L.w_down, dm, c.ffn);
@@ -448,8 +511,10 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lm_slabs = lmhead_slabs(c.vocab, h->dev);
         const size_t R = (size_t)c.n_layers * B;
         const size_t k = c.top_k_max;
-        size_t off[15], n = 0, tot = 0;
-        const size_t bytes[15] = {
+        const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
+        const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
+        size_t off[18], n = 0, tot = 0;
+        const size_t bytes[18] = {
             cs.size() * sizeof(float),                             // rope
             B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
             B * F * 4, R * d * 4,                                  // act, hid
@@ -459,8 +524,12 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             256,                                                   // status
             B * c.n_kv_heads * 4,                                  // attention split counters
             R * 4,                                                 // LM-head slab counters
-            h->lm_mma ? lmhead_mma_zb_bytes((int)R, c.d) : 0};     // tensor-core LM-head operand
-        for (n = 0; n < 15; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            h->lm_mma ? std::max(lmhead_mma_zb_bytes((int)std::min<size_t>(R, 16), c.d),
+                                 lmhead_wide_zb_bytes((int)R, c.d)) : 0,  // tensor-core LM-head operand
+            h->lin_mma ? linear_mma_xb_bytes((int)kmax, c.max_batch) : 0,  // tensor-core linear operand
+            h->lin_mma ? linear_mma_part_bytes(c.max_batch, h->dev) : 0,   // its split-tile partials
+            h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0};      // its completion counters
+        for (n = 0; n < 18; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -478,10 +547,14 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->attn_counters = (int*)(s + off[12]);
         h->lm_counters = (int*)(s + off[13]);
         h->lm_zb = h->lm_mma ? (uint16_t*)(s + off[14]) : nullptr;
+        h->lin_xb = h->lin_mma ? (uint16_t*)(s + off[15]) : nullptr;
+        h->lin_part = h->lin_mma ? (float*)(s + off[16]) : nullptr;
+        h->lin_counters = h->lin_mma ? (int*)(s + off[17]) : nullptr;
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
         if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, off[13] + bytes[13] - off[11], st))) != FE_OK) break;
+        if (h->lin_mma && (rc = from_cuda(cudaMemsetAsync(h->lin_counters, 0, bytes[17], st))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamSynchronize(st))) != FE_OK) break;
     } while (0);
@@ -595,8 +668,9 @@ const char* fe_last_error_detail(void) { return g_detail; }
 int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     if (!h || B < 1) return -1;
     const int N = h->cfg.n_layers;
-    int n = 2 * linear_launches() + N * (4 * linear_launches() + attention_launches()) +
-            (h->lm_mma ? 2 : lmhead_launches(N * B, h->cfg.d, h->dev));
+    const int lin = h->lin_mma ? 2 : linear_launches();
+    int n = 2 * lin + N * (4 * lin + attention_launches()) +
+            (h->lm_mma ? (N * B <= 16 ? 2 : 3) : lmhead_launches(N * B, h->cfg.d, h->dev));
     return n + (with_tree ? 1 : 0);
 }
 

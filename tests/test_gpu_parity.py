@@ -79,6 +79,20 @@ SMALL = {
     "chain_k1_b5": dict(name=dict(d=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=688, vocab=4096,
                                   n_layers=5, dtype="bf16", B=5, prefix=0, top_k=1, rope_theta=1e4,
                                   seed=8, page_size=0), prefix_list=[0, 1, 2, 33, 64]),
+    # batched handles (max_batch > 8): the linear phases run on the tensor cores; several
+    # tiles per matrix, tiles split between CTAs, ragged and paged prefixes
+    "tc_linear_b12_ragged": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1408, vocab=5003,
+                                           n_layers=3, dtype="bf16", B=12, prefix=0, top_k=8, rope_theta=1e4,
+                                           seed=9, page_size=0),
+                                 prefix_list=[37, 0, 150, 1, 64, 5, 300, 2, 128, 129, 7, 90]),
+    "tc_linear_b9_paged": dict(name=dict(d=1024, n_heads=8, n_kv_heads=8, head_dim=128, ffn=2816, vocab=3001,
+                                         n_layers=2, dtype="bf16", B=9, prefix=0, top_k=4, rope_theta=5e5,
+                                         seed=10, page_size=16), prefix_list=[15, 16, 1, 200, 0, 31, 33, 64, 100]),
+    # N * B = 160 rows: the wide tensor-core LM head with three 64-row transpose groups
+    "wide_lmhead_r160": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=3001,
+                                       n_layers=5, dtype="bf16", B=32, prefix=0, top_k=8, rope_theta=1e4,
+                                       seed=12, page_size=0),
+                             prefix_list=[(53 * b + 7) % 97 for b in range(32)]),
 }
 
 
@@ -91,6 +105,24 @@ def test_parity_small(orc, case):
     g = H.run_gpu(cfg, W, I, ks, vs)
     assert g["status"] == 0, g["status"]
     for b in range(cfg["B"]):
+        o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
+        H.compare(orc, cfg, g, o, b)
+        _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
+
+
+@pytest.mark.parametrize("B", [1, 2, 32])
+def test_parity_tensor_core_linear_forced(orc, monkeypatch, B):
+    """The tensor-core linear path chosen explicitly, at one and two sequences (operand rows
+    padded to 8) and at its maximum batch of 32."""
+    monkeypatch.setenv("FE_DRAFT_LINEAR_MMA", "1")
+    plist = [(37 * b + 11) % 160 for b in range(B)]
+    cfg = wl.make_config(dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1408, vocab=4000, n_layers=2,
+                              dtype="bf16", B=B, prefix=0, top_k=8, rope_theta=1e4, seed=11 + B, page_size=0),
+                         prefix_list=plist)
+    W, I, ks, vs = _problem(cfg)
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert g["status"] == 0, g["status"]
+    for b in sorted({0, B - 1, B // 2}):
         o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
         H.compare(orc, cfg, g, o, b)
         _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
