@@ -30,6 +30,7 @@ namespace fe {
 constexpr int kAttnWarps = 4;
 constexpr int kChunkKeys = 32;
 constexpr int kAttnMaxSlots = 2;
+constexpr int kAttnPageSmem = 32 * 1024;  // dynamic shared memory reserved for an item's page ids
 
 template <typename CT, int DPL>
 __device__ __forceinline__ void load_dims(const CT* p, float* out) {
@@ -83,7 +84,6 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     __shared__ __align__(16) float vn[HD];
     __shared__ float pw[kAttnWarps][kChunkKeys * G];
     __shared__ float wm[kAttnWarps][G], wl[kAttnWarps][G];
-    __shared__ float wacc[kAttnWarps][G][HD];
     __shared__ __align__(8) uint64_t bars[kAttnWarps][kAttnMaxSlots];
     __shared__ int s_last, s_abort;
 
@@ -119,6 +119,24 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
         mbar_fence_init();
     }
     if (t == 0) s_abort = 0;
+    // Paged caches: this item's page ids, read once into shared memory (after the K/V slots;
+    // -1 marks an invalid id), so that issuing a chunk needs no round trip to the table.
+    int* spg = reinterpret_cast<int*>(dsm + (size_t)kAttnWarps * S * 2 * CHB);
+    const int pg0 = a.page_table ? t0 / a.page_size : 0;
+    if (a.page_table) {
+        const int last_row = min(t1, P) - 1;  // cached rows are < P
+        const int npg = last_row >= t0 ? last_row / a.page_size - pg0 + 1 : 0;
+        for (int i = t; i < npg; i += blockDim.x) {
+            const int pg = a.page_table[(size_t)b * a.max_pages + pg0 + i];
+            spg[i] = (pg < 0 || pg >= a.n_pages) ? -1 : pg;
+        }
+    }
+    // address of cached row `pos` (< P) of this item from the staged page ids (null if invalid)
+    auto prow = [&](CT* base, int pos) -> CT* {
+        const int pg = spg[pos / a.page_size - pg0];
+        if (pg < 0) return nullptr;
+        return base + (((size_t)pg * a.Hkv + g) * a.page_size + pos % a.page_size) * HD;
+    };
 
     // Chunk j of this warp covers keys [c0, c0 + 32), c0 = t0 + (warp + 4 j) * 32; its rows
     // below P come from the cache. Returns the mask of rows whose page id was invalid.
@@ -131,9 +149,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
         if (a.page_table) {
             for (int p = c0; p < c0 + rows;) {
                 const int n = min(a.page_size - p % a.page_size, c0 + rows - p);
-                const CT* kr = cache_row<CT>((CT*)a.kc, a, b, g, p, HD);
-                const CT* vr = cache_row<CT>((CT*)a.vc, a, b, g, p, HD);
-                if (kr && vr) bytes += 2u * n * ROWB;
+                if (spg[p / a.page_size - pg0] >= 0) bytes += 2u * n * ROWB;
                 else bad |= (n >= 32 ? 0xffffffffu : ((1u << n) - 1u)) << (p - c0);
                 p += n;
             }
@@ -144,8 +160,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
         if (a.page_table) {
             for (int p = c0; p < c0 + rows;) {
                 const int n = min(a.page_size - p % a.page_size, c0 + rows - p);
-                const CT* kr = cache_row<CT>((CT*)a.kc, a, b, g, p, HD);
-                const CT* vr = cache_row<CT>((CT*)a.vc, a, b, g, p, HD);
+                const CT* kr = prow((CT*)a.kc, p);
+                const CT* vr = prow((CT*)a.vc, p);
                 if (kr && vr) {
                     bulk_g2s(kd + (size_t)(p - c0) * ROWB, kr, n * ROWB, &bar[slot]);
                     bulk_g2s(vd + (size_t)(p - c0) * ROWB, vr, n * ROWB, &bar[slot]);
@@ -316,7 +332,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     if (lane == 0 && *(volatile int*)&s_abort)
         for (int j = max(0, issued - S); j < issued; ++j) mbar_wait(&bar[j % S], (uint32_t)(j / S) & 1u, a.status, 100000000LL);
 
-    // ---- merge the warps into this split's partial per head
+    // ---- merge the warps into this split's partial per head (the K/V slots are free now
+    // and hold the warps' accumulators)
+    float (*wacc)[G][HD] = reinterpret_cast<float (*)[G][HD]>(dsm);
+    __syncthreads();
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
 #pragma unroll
@@ -445,24 +464,32 @@ int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev) {
 
 // Pipeline slots per warp: two when a warp has more than one chunk and a chunk of K (or
 // V) is at most 8 KB (bf16, hd 128), else one; at most 128 KB of dynamic shared memory.
-static int max_slots(int hd, int es) { return kChunkKeys * hd * es <= 8192 ? kAttnMaxSlots : 1; }
-static int attn_slots(int split, int hd, int es) {
-    return split > kAttnWarps * kChunkKeys ? max_slots(hd, es) : 1;
-}
+// One slot per warp: a CTA then needs ~70 KB (bf16, hd 128) and three fit on an SM. The
+// per-chunk work is a chain of shared-memory loads and shuffles, latency-bound in one warp,
+// so more warps per SM (other CTAs) hide it better than a second slot per warp does.
+static int max_slots(int, int) { return 1; }
+static int attn_slots(int, int, int) { return 1; }
 
 static size_t attn_smem(int hd, int es, int S) { return (size_t)kAttnWarps * S * 2 * kChunkKeys * hd * es; }
+// page ids one work item covers (paged caches)
+static size_t attn_page_ints(const AttnArgs& a) {
+    return a.page_table ? (size_t)(a.split + a.page_size - 1) / a.page_size + 1 : 0;
+}
 
 template <typename CT, int HD, int G>
 static cudaError_t prepare_g() {
     return cudaFuncSetAttribute(attn_kernel<CT, HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)attn_smem(HD, sizeof(CT), max_slots(HD, sizeof(CT))));
+                                (int)attn_smem(HD, sizeof(CT), max_slots(HD, sizeof(CT))) + kAttnPageSmem);
 }
 
 template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
     const int S = attn_slots(a.split, HD, sizeof(CT));
+    const size_t pg = attn_page_ints(a) * sizeof(int);
+    if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
     dim3 grid(a.n_split, a.Hkv, a.B);
-    return launch_k(attn_kernel<CT, HD, G>, grid, dim3(kAttnWarps * 32), attn_smem(HD, sizeof(CT), S), st, a.pdl, a, S);
+    return launch_k(attn_kernel<CT, HD, G>, grid, dim3(kAttnWarps * 32), attn_smem(HD, sizeof(CT), S) + pg, st, a.pdl,
+                    a, S);
 }
 
 template <typename CT, int HD>

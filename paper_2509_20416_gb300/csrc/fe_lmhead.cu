@@ -800,24 +800,25 @@ struct WideState {
     int abort;
 };
 
-__device__ __forceinline__ void wide_insert(float (&tv)[kWideKMax], int (&ti)[kWideKMax], int k, float x, int id) {
+// insertion into the sorted list as a branch-free compare-exchange down the list
+template <int KM>
+__device__ __forceinline__ void wide_insert(float (&tv)[KM], int (&ti)[KM], int k, float x, int id) {
 #pragma unroll
-    for (int q = 0; q < kWideKMax; ++q) {
-        if (q < k && better(x, id, tv[q], ti[q])) {
-            const float sv = tv[q];
-            const int si = ti[q];
-            tv[q] = x;
-            ti[q] = id;
-            x = sv;
-            id = si;
-        }
+    for (int q = 0; q < KM; ++q) {
+        const bool sw = q < k && better(x, id, tv[q], ti[q]);
+        const float ov = tv[q];
+        const int oi = ti[q];
+        tv[q] = sw ? x : ov;
+        ti[q] = sw ? id : oi;
+        x = sw ? ov : x;
+        id = sw ? oi : id;
     }
 }
 
-__device__ __forceinline__ void wide_kth(const float (&tv)[kWideKMax], const int (&ti)[kWideKMax], int k, float& v,
-                                         int& id) {
+template <int KM>
+__device__ __forceinline__ void wide_kth(const float (&tv)[KM], const int (&ti)[KM], int k, float& v, int& id) {
 #pragma unroll
-    for (int q = 0; q < kWideKMax; ++q)
+    for (int q = 0; q < KM; ++q)
         if (q == k - 1) { v = tv[q]; id = ti[q]; }
 }
 
@@ -826,6 +827,37 @@ __device__ __forceinline__ void online_add(float& m, float& s, float x) {
     else s += expf(x - m);
 }
 
+// A running (softmax statistics, top-k) state of one hidden row over part of the vocabulary;
+// KM >= k entries of the sorted list are kept.
+template <int KM>
+struct WideRow {
+    float v[KM];
+    int i[KM];
+    float thv, m, s;  // the current k-th value, max and sum of exp of logit / T
+    int thi;
+    __device__ __forceinline__ void init() {
+#pragma unroll
+        for (int q = 0; q < KM; ++q) { v[q] = -INFINITY; i[q] = INT_MAX; }
+        thv = -INFINITY;
+        thi = INT_MAX;
+        m = -INFINITY;
+        s = 0.f;
+    }
+    // a candidate for the top-k list only
+    __device__ __forceinline__ void offer(int k, float x, int id) {
+        if (better(x, id, thv, thi)) {
+            wide_insert(v, i, k, x, id);
+            wide_kth(v, i, k, thv, thi);
+        }
+    }
+    // a logit: statistics and top-k
+    __device__ __forceinline__ void add(int k, float x, int id, float inv_temp) {
+        online_add(m, s, x * inv_temp);
+        offer(k, x, id);
+    }
+};
+
+template <int KM>
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
                                                                      int S, int stage_bytes, uint32_t tmem_cols) {
     extern __shared__ unsigned char dsm_raw[];
@@ -913,25 +945,19 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
     } else {  // ---- epilogue warps 0..3
         griddep_wait();
         const int rg = t & (kWideGroup - 1), half = t / kWideGroup;  // row within a group, vocabulary half
-        float tv[4][kWideKMax], thv[4], m[4], s[4];
-        int ti[4][kWideKMax], thi[4];
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-#pragma unroll
-            for (int q = 0; q < kWideKMax; ++q) { tv[g][q] = -INFINITY; ti[g][q] = INT_MAX; }
-            thv[g] = -INFINITY;
-            thi[g] = INT_MAX;
-            m[g] = -INFINITY;
-            s[g] = 0.f;
-        }
+        WideRow<KM> w0, w1, w2, w3;  // one state per 64-row group
+        w0.init();
+        w1.init();
+        w2.init();
+        w3.init();
         uint32_t eb = 0;  // epilogue barriers passed (two mbarriers used alternately)
         auto epi_sync = [&]() -> bool {
             __syncwarp();
             uint64_t* bar = &st.ebar[eb & 1];
             if (lane == 0) mbar_arrive(bar);
-            const bool ok = mbar_wait_abortable(bar, (eb >> 1) & 1u, a.status, &st.abort);
+            const bool r = mbar_wait_abortable(bar, (eb >> 1) & 1u, a.status, &st.abort);
             ++eb;
-            return ok;
+            return r;
         };
         bool ok = true;
         for (int tile = t0, j = 0; tile < t1 && ok; ++tile, ++j) {
@@ -939,9 +965,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
             if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
             tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * R_pad);
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                if (g >= ngroups || !ok) break;
+            auto group = [&](WideRow<KM>& w, int g) {
+                if (g >= ngroups || !ok) return;
                 // stage: vocabulary entry 32 w + lane, rows [64 g, 64 g + 64) of the tile
                 float* trow = tbuf + (size_t)(warp * 32 + lane) * kWideTileStride;
 #pragma unroll
@@ -958,7 +983,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&st.tempty[buf]);
                 }
-                if (!(ok = epi_sync())) break;
+                if (!(ok = epi_sync())) return;
                 // consume: this thread's row r, vocabulary entries [64 half, 64 half + 64)
                 const int r = g * kWideGroup + rg;
                 if (r < R) {
@@ -967,61 +992,57 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
                         const int id = tile * 128 + v;
                         if (id >= a.V) break;
                         const float x = tbuf[(size_t)v * kWideTileStride + rg];
-                        online_add(m[g], s[g], x * a.inv_temp);
-                        if (better(x, id, thv[g], thi[g])) {
-                            wide_insert(tv[g], ti[g], k, x, id);
-                            wide_kth(tv[g], ti[g], k, thv[g], thi[g]);
-                        }
+                        w.add(k, x, id, a.inv_temp);
                         if (a.dbg_logits) a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id] = x;
                     }
                 }
-                if (!(ok = epi_sync())) break;
-            }
+                ok = epi_sync();
+            };
+            group(w0, 0);
+            group(w1, 1);
+            group(w2, 2);
+            group(w3, 3);
         }
         // ---- the slab's partial per row: the upper half hands its list to the lower half
-        float* xs = tbuf;  // [64][2 * kWideKMax + 2]
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-            if (g >= ngroups || !ok) break;
-            float* mine = xs + (size_t)rg * (2 * kWideKMax + 2);
+        auto finish = [&](WideRow<KM>& w, int g) {
+            if (g >= ngroups || !ok) return;
+            float* mine = tbuf + (size_t)rg * (2 * KM + 2);
             if (half == 1) {
 #pragma unroll
-                for (int q = 0; q < kWideKMax; ++q) {
-                    mine[q] = tv[g][q];
-                    mine[kWideKMax + q] = __int_as_float(ti[g][q]);
+                for (int q = 0; q < KM; ++q) {
+                    mine[q] = w.v[q];
+                    mine[KM + q] = __int_as_float(w.i[q]);
                 }
-                mine[2 * kWideKMax] = m[g];
-                mine[2 * kWideKMax + 1] = s[g];
+                mine[2 * KM] = w.m;
+                mine[2 * KM + 1] = w.s;
             }
-            if (!(ok = epi_sync())) break;
+            if (!(ok = epi_sync())) return;
             const int r = g * kWideGroup + rg;
             if (half == 0 && r < R) {
 #pragma unroll
-                for (int q = 0; q < kWideKMax; ++q) {
-                    const float ov = mine[q];
-                    const int oi = __float_as_int(mine[kWideKMax + q]);
-                    if (q < k && better(ov, oi, thv[g], thi[g])) {
-                        wide_insert(tv[g], ti[g], k, ov, oi);
-                        wide_kth(tv[g], ti[g], k, thv[g], thi[g]);
-                    }
-                }
-                const float om = mine[2 * kWideKMax], os = mine[2 * kWideKMax + 1];
-                const float nm = fmaxf(m[g], om);
-                const float ns = (m[g] == -INFINITY ? 0.f : s[g] * expf(m[g] - nm)) +
-                                 (om == -INFINITY ? 0.f : os * expf(om - nm));
+                for (int q = 0; q < KM; ++q)
+                    if (q < k) w.offer(k, mine[q], __float_as_int(mine[KM + q]));
+                const float om = mine[2 * KM], os = mine[2 * KM + 1];
+                const float nm = fmaxf(w.m, om);
+                const float ns =
+                    (w.m == -INFINITY ? 0.f : w.s * expf(w.m - nm)) + (om == -INFINITY ? 0.f : os * expf(om - nm));
                 const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
 #pragma unroll
-                for (int q = 0; q < kWideKMax; ++q) {
+                for (int q = 0; q < KM; ++q) {
                     if (q < k) {
-                        a.part_id[base * k + q] = tv[g][q] == -INFINITY ? INT_MAX : ti[g][q];
-                        a.part_val[base * k + q] = tv[g][q];
+                        a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];
+                        a.part_val[base * k + q] = w.v[q];
                     }
                 }
                 a.part_ms[base * 2 + 0] = nm;
                 a.part_ms[base * 2 + 1] = ns;
             }
-            if (!(ok = epi_sync())) break;
-        }
+            ok = epi_sync();
+        };
+        finish(w0, 0);
+        finish(w1, 1);
+        finish(w2, 2);
+        finish(w3, 3);
     }
     tc_fence_before();
     __syncthreads();
@@ -1050,8 +1071,11 @@ int lmhead_wide_slabs(int V, const DeviceInfo& dev) {
 }
 
 cudaError_t lmhead_wide_prepare(const DeviceInfo& dev) {
-    cudaError_t e = cudaFuncSetAttribute(lmhead_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(lmhead_wide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          dev.max_smem_optin - (int)sizeof(WideState) - 256);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(lmhead_wide_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             dev.max_smem_optin - (int)sizeof(WideState) - 256);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
 }
@@ -1073,8 +1097,10 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
     const size_t smem = 1024 + (size_t)S * stage_bytes + tbytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * R_pad)) cols <<= 1;
-    e = launch_k(lmhead_wide_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad,
-                 S, stage_bytes, cols);
+    e = a.top_k <= 8 ? launch_k(lmhead_wide_kernel<8>, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a,
+                                (const uint16_t*)zb, R_pad, S, stage_bytes, cols)
+                     : launch_k(lmhead_wide_kernel<16>, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a,
+                                (const uint16_t*)zb, R_pad, S, stage_bytes, cols);
     if (e != cudaSuccess) return e;
     if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;
     const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k);
