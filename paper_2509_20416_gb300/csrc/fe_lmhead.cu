@@ -782,16 +782,17 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
 //     |W_v| |z| 2^-9 / sqrt(3), a few 1e-3 at d = 4096 with weights ~ N(0, 0.02^2).
 //   - TMEM holds two R_pad-column accumulators, so the epilogue of tile j overlaps the
 //     MMAs of tile j + 1.
-//   - The epilogue transposes each tile through shared memory, 64 rows at a time, so that
-//     a thread owns one hidden row r and half of the tile's 128 vocabulary entries: its
-//     softmax statistics are exact online (max, sum of exp) and its running top-k is a
-//     sorted list in registers (an entry enters only if it beats the current k-th best,
-//     ties to the smaller id), with no cross-thread reduction per tile. At the end of the
-//     slab the two halves of each row merge and write the slab's partial.
+//   - The epilogue transposes each tile through shared memory, 128 rows at a time, so that
+//     a thread owns one hidden row r (two for R > 128) and reads the tile's 128 logits of
+//     that row: its softmax statistics are exact (the tile's max, then its sum of exp, then
+//     one rescale of the running pair) and its running top-k is a sorted list in registers
+//     (an entry enters only if it beats the current k-th best, ties to the smaller id),
+//     with no cross-thread reduction per tile. At the end of the slab it writes the row's
+//     partial.
 //   - lmhead_merge_kernel (one CTA per row) then merges the slabs as merge_rows does.
 constexpr int kWideKMax = 16;     // top_k limit of this kernel (a sorted list in registers)
 constexpr int kWideRowsMax = 256;
-constexpr int kWideGroup = 64;    // rows staged per transpose round
+constexpr int kWideGroup = 128;   // rows staged per transpose round (one per epilogue thread)
 constexpr int kWideTileStride = kWideGroup + 1;  // floats per staged vocabulary entry (no bank conflicts)
 
 struct WideState {
@@ -815,47 +816,102 @@ __device__ __forceinline__ void wide_insert(float (&tv)[KM], int (&ti)[KM], int 
     }
 }
 
-template <int KM>
-__device__ __forceinline__ void wide_kth(const float (&tv)[KM], const int (&ti)[KM], int k, float& v, int& id) {
-#pragma unroll
-    for (int q = 0; q < KM; ++q)
-        if (q == k - 1) { v = tv[q]; id = ti[q]; }
-}
-
-__device__ __forceinline__ void online_add(float& m, float& s, float x) {
-    if (x > m) { s = s * expf(m - x) + 1.f; m = x; }
-    else s += expf(x - m);
-}
-
-// A running (softmax statistics, top-k) state of one hidden row over part of the vocabulary;
-// KM >= k entries of the sorted list are kept.
+// A running (softmax statistics, top-k) state of one hidden row: the first k of the KM
+// entries form the sorted list (larger value first, ties to the smaller id; the rest stay
+// -inf); (m, s) are the max and sum of exp of logit / T so far.
 template <int KM>
 struct WideRow {
     float v[KM];
     int i[KM];
-    float thv, m, s;  // the current k-th value, max and sum of exp of logit / T
-    int thi;
+    float m, s;
     __device__ __forceinline__ void init() {
 #pragma unroll
         for (int q = 0; q < KM; ++q) { v[q] = -INFINITY; i[q] = INT_MAX; }
-        thv = -INFINITY;
-        thi = INT_MAX;
         m = -INFINITY;
         s = 0.f;
     }
-    // a candidate for the top-k list only
-    __device__ __forceinline__ void offer(int k, float x, int id) {
-        if (better(x, id, thv, thi)) {
-            wide_insert(v, i, k, x, id);
-            wide_kth(v, i, k, thv, thi);
-        }
-    }
-    // a logit: statistics and top-k
-    __device__ __forceinline__ void add(int k, float x, int id, float inv_temp) {
-        online_add(m, s, x * inv_temp);
-        offer(k, x, id);
-    }
 };
+
+// One 128-row group g of a tile for row state w (inside lmhead_wide_kernel's epilogue).
+// Expanded textually for each group: written as a lambda or function taking the state by
+// reference, the compiler keeps a state in local memory, and each step of the loop below
+// then waits on a round trip to L2.
+//   stage:   warp w copies TMEM lanes 32 w .. 32 w + 31 (vocabulary entries) x the group's
+//            128 columns (hidden rows) into tbuf[entry][row];
+//   consume: thread t reads row r = 128 g + t across the tile's entries: the max (eight
+//            independent loads at a time) and a 128-bit mask of the entries that reach the
+//            list's last value; only those (a few per tile) run through the branch-free
+//            insertion network, whose serial compare-exchange chain is too slow to run on
+//            every entry; then the sum of exp against that max and one rescale of the
+//            running (max, sum).
+#define FE_WIDE_GROUP(w, g)                                                                        \
+    do {                                                                                           \
+        if ((g) >= ngroups || !ok) break;                                                          \
+        float* trow = tbuf + (size_t)(warp * 32 + lane) * kWideTileStride;                         \
+        for (int c0 = 0; c0 < kWideGroup && (g) * kWideGroup + c0 < R_pad; c0 += 16) {             \
+            float v16[16];                                                                         \
+            tc_ld16(taddr + (uint32_t)((g) * kWideGroup + c0), v16);                               \
+            _Pragma("unroll") for (int i = 0; i < 16; ++i) trow[c0 + i] = v16[i];                  \
+        }                                                                                          \
+        if ((g) == ngroups - 1) { /* the accumulator is read: hand it back to the MMA warp */      \
+            tc_fence_before();                                                                     \
+            __syncwarp();                                                                          \
+            if (lane == 0) mbar_arrive(&st.tempty[buf]);                                           \
+        }                                                                                          \
+        if (!(ok = epi_sync())) break;                                                             \
+        const int r = (g) * kWideGroup + t;                                                        \
+        if (r < R) {                                                                               \
+            const int id0 = tile * 128;                                                            \
+            const int nv = min(128, a.V - id0);                                                    \
+            const float* col = tbuf + t;                                                           \
+            const float th = w.v[KM - 1];                                                          \
+            float M = -INFINITY;                                                                   \
+            uint32_t cm0 = 0u, cm1 = 0u, cm2 = 0u, cm3 = 0u; /* entries >= th, one bit each */     \
+            _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                     \
+                uint32_t bits = 0u;                                                                \
+                for (int b0 = 0; b0 < 32; b0 += 8) {                                               \
+                    float x[8];                                                                    \
+                    _Pragma("unroll") for (int u = 0; u < 8; ++u) {                                \
+                        const int e = wd * 32 + b0 + u;                                            \
+                        x[u] = e < nv ? col[(size_t)e * kWideTileStride] : -INFINITY;              \
+                    }                                                                              \
+                    _Pragma("unroll") for (int u = 0; u < 8; ++u) {                                \
+                        M = fmaxf(M, x[u]);                                                        \
+                        bits |= (x[u] >= th ? 1u : 0u) << (b0 + u);                                \
+                    }                                                                              \
+                }                                                                                  \
+                if (wd == 0) cm0 = bits;                                                           \
+                else if (wd == 1) cm1 = bits;                                                      \
+                else if (wd == 2) cm2 = bits;                                                      \
+                else cm3 = bits;                                                                   \
+            }                                                                                      \
+            _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                     \
+                uint32_t bits = wd == 0 ? cm0 : wd == 1 ? cm1 : wd == 2 ? cm2 : cm3;               \
+                while (bits) {                                                                     \
+                    const int e = wd * 32 + __ffs(bits) - 1;                                       \
+                    bits &= bits - 1u;                                                             \
+                    wide_insert(w.v, w.i, k, col[(size_t)e * kWideTileStride], id0 + e);           \
+                }                                                                                  \
+            }                                                                                      \
+            if (nv > 0) {                                                                          \
+                const float Mt = M * a.inv_temp;                                                   \
+                float S = 0.f;                                                                     \
+                for (int u0 = 0; u0 < nv; u0 += 8) {                                               \
+                    _Pragma("unroll") for (int u = 0; u < 8; ++u)                                  \
+                        if (u0 + u < nv) S += expf(col[(size_t)(u0 + u) * kWideTileStride] * a.inv_temp - Mt); \
+                }                                                                                  \
+                const float nm = fmaxf(w.m, Mt);                                                   \
+                w.s = (w.m == -INFINITY ? 0.f : w.s * expf(w.m - nm)) + S * expf(Mt - nm);         \
+                w.m = nm;                                                                          \
+            }                                                                                      \
+            if (a.dbg_logits) {                                                                    \
+                const int rb = r % a.B, ri = r / a.B;                                              \
+                for (int u = 0; u < nv; ++u)                                                       \
+                    a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id0 + u] = col[(size_t)u * kWideTileStride]; \
+            }                                                                                      \
+        }                                                                                          \
+        ok = epi_sync();                                                                           \
+    } while (0)
 
 template <int KM>
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
@@ -942,14 +998,11 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
                 tc_commit(&st.tfull[buf]);
             }
         }
-    } else {  // ---- epilogue warps 0..3
+    } else {  // ---- epilogue warps 0..3: thread t owns rows t and 128 + t
         griddep_wait();
-        const int rg = t & (kWideGroup - 1), half = t / kWideGroup;  // row within a group, vocabulary half
-        WideRow<KM> w0, w1, w2, w3;  // one state per 64-row group
+        WideRow<KM> w0, w1;
         w0.init();
         w1.init();
-        w2.init();
-        w3.init();
         uint32_t eb = 0;  // epilogue barriers passed (two mbarriers used alternately)
         auto epi_sync = [&]() -> bool {
             __syncwarp();
@@ -965,90 +1018,35 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
             if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
             tc_fence_after();
             const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * R_pad);
-            auto group = [&](WideRow<KM>& w, int g) {
-                if (g >= ngroups || !ok) return;
-                // stage: vocabulary entry 32 w + lane, rows [64 g, 64 g + 64) of the tile
-                float* trow = tbuf + (size_t)(warp * 32 + lane) * kWideTileStride;
-#pragma unroll
-                for (int c0 = 0; c0 < kWideGroup; c0 += 16) {
-                    if (g * kWideGroup + c0 < R_pad) {
-                        float v16[16];
-                        tc_ld16(taddr + (uint32_t)(g * kWideGroup + c0), v16);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) trow[c0 + i] = v16[i];
-                    }
-                }
-                if (g == ngroups - 1) {  // the accumulator is fully read: hand it back to the MMA warp
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&st.tempty[buf]);
-                }
-                if (!(ok = epi_sync())) return;
-                // consume: this thread's row r, vocabulary entries [64 half, 64 half + 64)
-                const int r = g * kWideGroup + rg;
-                if (r < R) {
-                    const int rb = r % a.B, ri = r / a.B;
-                    for (int v = half * 64; v < half * 64 + 64; ++v) {
-                        const int id = tile * 128 + v;
-                        if (id >= a.V) break;
-                        const float x = tbuf[(size_t)v * kWideTileStride + rg];
-                        w.add(k, x, id, a.inv_temp);
-                        if (a.dbg_logits) a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id] = x;
-                    }
-                }
-                ok = epi_sync();
-            };
-            group(w0, 0);
-            group(w1, 1);
-            group(w2, 2);
-            group(w3, 3);
+            FE_WIDE_GROUP(w0, 0);
+            FE_WIDE_GROUP(w1, 1);
         }
-        // ---- the slab's partial per row: the upper half hands its list to the lower half
-        auto finish = [&](WideRow<KM>& w, int g) {
-            if (g >= ngroups || !ok) return;
-            float* mine = tbuf + (size_t)rg * (2 * KM + 2);
-            if (half == 1) {
-#pragma unroll
-                for (int q = 0; q < KM; ++q) {
-                    mine[q] = w.v[q];
-                    mine[KM + q] = __int_as_float(w.i[q]);
-                }
-                mine[2 * KM] = w.m;
-                mine[2 * KM + 1] = w.s;
-            }
-            if (!(ok = epi_sync())) return;
-            const int r = g * kWideGroup + rg;
-            if (half == 0 && r < R) {
-#pragma unroll
-                for (int q = 0; q < KM; ++q)
-                    if (q < k) w.offer(k, mine[q], __float_as_int(mine[KM + q]));
-                const float om = mine[2 * KM], os = mine[2 * KM + 1];
-                const float nm = fmaxf(w.m, om);
-                const float ns =
-                    (w.m == -INFINITY ? 0.f : w.s * expf(w.m - nm)) + (om == -INFINITY ? 0.f : os * expf(om - nm));
-                const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
-#pragma unroll
-                for (int q = 0; q < KM; ++q) {
-                    if (q < k) {
-                        a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];
-                        a.part_val[base * k + q] = w.v[q];
-                    }
-                }
-                a.part_ms[base * 2 + 0] = nm;
-                a.part_ms[base * 2 + 1] = ns;
-            }
-            ok = epi_sync();
-        };
-        finish(w0, 0);
-        finish(w1, 1);
-        finish(w2, 2);
-        finish(w3, 3);
+        // ---- the slab's partial of each owned row
+#define FE_WIDE_FINISH(w, g)                                                                           \
+    do {                                                                                               \
+        const int r = (g) * kWideGroup + t;                                                            \
+        if ((g) >= ngroups || !ok || r >= R) break;                                                    \
+        const size_t base = (size_t)r * a.n_slabs + blockIdx.x;                                        \
+        _Pragma("unroll") for (int q = 0; q < KM; ++q) {                                               \
+            if (q < k) {                                                                               \
+                a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];                      \
+                a.part_val[base * k + q] = w.v[q];                                                     \
+            }                                                                                          \
+        }                                                                                              \
+        a.part_ms[base * 2 + 0] = w.m;                                                                 \
+        a.part_ms[base * 2 + 1] = w.s;                                                                 \
+    } while (0)
+        FE_WIDE_FINISH(w0, 0);
+        FE_WIDE_FINISH(w1, 1);
+#undef FE_WIDE_FINISH
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tc_dealloc(tmem, tmem_cols);
 }
+
+#undef FE_WIDE_GROUP
 
 // One CTA per row: merges every slab's partial of that row (merge_rows).
 __global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, size_t smem_bytes) {
