@@ -49,8 +49,12 @@ __device__ __forceinline__ void split_bf16(float z, uint16_t& hi, uint16_t& lo) 
 }  // namespace
 
 // ---- activation operand ------------------------------------------------------------------
-// One CTA per operand row b < B_pad (rows b >= B are zero). Reads what the previous kernel
-// wrote only after griddep_wait(), through L2, and never through a __restrict__ pointer.
+// Grid (B_pad, ceil(K / 2048)): CTA (b, y) writes row b's 16-byte chunks [256 y, 256 y + 256)
+// (rows b >= B are zero); with RMSNorm every CTA of the row reads the whole row for its sum
+// of squares (an L2 read of 4 d bytes). Reads what the previous kernel wrote only after
+// griddep_wait(), through L2, and never through a __restrict__ pointer.
+constexpr int kXprepChunks = 256;  // 16-byte chunks per CTA (one per thread)
+
 __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
     const int b = blockIdx.x, t = threadIdx.x;
     const int N = 2 * B_pad, K = a.K, nc = K / 8;
@@ -84,8 +88,9 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
         for (int w = 0; w < 8; ++w) tot += red[w];
         rs = 1.0f / sqrtf(tot / (float)K + a.eps);
     }
-#pragma unroll 4
-    for (int c = t; c < nc; c += 256) {
+    {
+        const int c = blockIdx.y * kXprepChunks + t;
+        if (c >= nc) return;
         float v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = 0.f;
@@ -369,7 +374,8 @@ cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, in
                               cudaStream_t st, cudaEvent_t after_prep) {
     if (!linear_mma_ok(a.M, a.K, a.B)) return cudaErrorInvalidValue;
     const int BP = linear_mma_bpad(a.B);
-    cudaError_t e = launch_k(xprep_kernel, dim3(BP), dim3(256), 0, st, a.pdl, a, BP, xb);
+    const int ny = (a.K / 8 + kXprepChunks - 1) / kXprepChunks;
+    cudaError_t e = launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int grid = linear_mma_grid(a.M, a.K, dev);
