@@ -75,6 +75,11 @@ __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }
 
+// retire an mbarrier (no pending arrivals or copies) before its memory is initialised again
+__device__ __forceinline__ void mbar_inval(uint64_t* bar) {
+    asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 __device__ __forceinline__ void mbar_fence_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
@@ -151,6 +156,51 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 // global -> L2 prefetch of `bytes` (16-byte aligned address, multiple of 16); no completion
 __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
+// ---- grid-wide barrier of a persistent kernel ----------------------------------------------
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Grid-wide barrier of a persistent kernel, split in two so that work that does not
+// depend on the other CTAs (issuing weight copies) can go between arrive and wait. Every
+// CTA arrives once on *count (zero at launch) per barrier; the k-th barrier (k = 1, 2, ...)
+// completes when *count reaches k * gridDim.x. All CTAs must be resident at once (grid <=
+// SMs, one CTA per SM). Writes made before grid_arrive are visible to L2-coherent reads
+// (ld.global.cg, TMA) after grid_wait. The arriving / polling thread is lane 1 of warp 0,
+// which issues no asynchronous copies, so its fence does not wait for any. Both are called
+// by every thread of the CTA.
+constexpr int kGridBarrierThread = 1;
+
+__device__ __forceinline__ void grid_arrive(uint32_t* count) {
+    __syncthreads();
+    if (threadIdx.x == kGridBarrierThread) {
+        __threadfence();
+        atomicAdd(count, 1u);
+    }
+}
+
+// Bounded: after kWaitBudgetNs it records ST_TIMEOUT, raises *abort and returns false.
+__device__ __forceinline__ bool grid_wait(uint32_t* count, uint32_t k, int* status, int* abort) {
+    if (threadIdx.x == kGridBarrierThread) {
+        const uint32_t target = k * gridDim.x;
+        if (ld_acquire_gpu(count) < target) {
+            const uint64_t t0 = globaltimer_ns();
+            while (ld_acquire_gpu(count) < target) {
+                if ((int64_t)(globaltimer_ns() - t0) > kWaitBudgetNs) {
+                    atomicOr(status, ST_TIMEOUT);
+                    *(volatile int*)abort = 1;
+                    break;
+                }
+            }
+        }
+        __threadfence();
+    }
+    __syncthreads();
+    return !*(volatile int*)abort;
 }
 
 // ---- named barriers (a subset of the CTA's warps) ---------------------------------------

@@ -89,6 +89,18 @@ cudaError_t launch_linear(fe_dtype dt, const LinearArgs& a, const DeviceInfo& de
 // number of kernels launch_linear() issues for these shapes (always 1)
 inline int linear_launches() { return 1; }
 
+// A persistent stack of consecutive linear phases at B = 1 (one launch; grid-wide barriers
+// between phases on *barrier, which must be zero at launch). ph[0].pdl decides the launch's
+// programmatic dependence; the others' pdl is ignored.
+constexpr int kMaxStackPhases = 4;
+struct StackArgs {
+    LinearArgs ph[kMaxStackPhases];
+    int nph;
+    uint32_t* barrier;
+};
+int stack_slots(int k_max, const DeviceInfo& dev);
+cudaError_t launch_stack(fe_dtype dt, const StackArgs& sa, const DeviceInfo& dev, cudaStream_t st);
+
 // ---- tensor-core linear phase (bf16 weights, batches of 1..kLinMmaMaxBatch) -------------
 // W packed by launch_pack_mma (interleaved gate/up rows for EPI_SWIGLU); xb scratch of
 // linear_mma_xb_bytes(K_max, max_batch); part of linear_mma_part_bytes(); counters:

@@ -32,7 +32,7 @@ struct LinearEpi {
                 const float v = chunk_value<BT>(red, gl, r, b);
                 float* yp = a->y + (size_t)(b0 + b) * a->ldy + m;
                 if (a->epi == EPI_RESID) {
-                    const float nv = *yp + v;
+                    const float nv = __ldcg(yp) + v;  // (L2: another CTA may have written it in a persistent kernel)
                     *yp = nv;
                     if (a->y2) a->y2[(size_t)(b0 + b) * a->ldy2 + m] = nv;
                 } else {
@@ -62,6 +62,52 @@ __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearA
     __syncthreads();
     LinearEpi<BT> e{&a, b0, nb};
     stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e, issued);
+}
+
+// ---- persistent stack of linear phases --------------------------------------------------------
+// Runs sa.nph consecutive linear phases (e.g. W_o, W_gate/up, W_down and the next layer's
+// W_qkv) in one launch of one CTA per SM: between phases every CTA issues its first copies
+// of the next phase's weights (they do not depend on the phase in flight) and then meets the
+// others at a grid-wide barrier, after which the next phase's activations — written by all
+// CTAs — are complete. This removes the per-launch pipeline fill and tail of separate
+// launches. Each phase computes exactly what linear_kernel computes for it (same row
+// partition, same order of operations).
+template <typename WT, int BT>
+__global__ void __launch_bounds__(kStreamThreads, 1) stack_kernel(const StackArgs sa, int D, int Kpad_max) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    StreamSmem s = carve_stream_smem(smem, D, 1, Kpad_max, BT);
+    int issued = 0;
+    for (int p = 0; p < sa.nph; ++p) {
+        const LinearArgs& a = sa.ph[p];
+        const int Kpad = (a.K + 3) & ~3;
+        const int GM = (a.M + kGroupRows - 1) / kGroupRows;
+        const int g0 = (int)(((int64_t)blockIdx.x * GM) / gridDim.x);
+        const int g1 = (int)(((int64_t)(blockIdx.x + 1) * GM) / gridDim.x);
+        if (p == 0) {
+            issued = stream_begin<WT>((const unsigned char*)a.W, a.K, g0, g1, s, D);
+            griddep_launch_dependents();
+            griddep_wait();
+        }
+        ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
+        stage_activations<WT>(pp, a.K, s.X, Kpad, 0, a.B, a.status, s.red);
+        __syncthreads();
+        LinearEpi<BT> e{&a, 0, a.B};
+        stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, a.B, a.status, e, issued);
+        if (p + 1 == sa.nph || *(volatile int*)s.abort) break;
+        const LinearArgs& nx = sa.ph[p + 1];
+        const int GMn = (nx.M + kGroupRows - 1) / kGroupRows;
+        const int h0 = (int)(((int64_t)blockIdx.x * GMn) / gridDim.x);
+        const int h1 = (int)(((int64_t)(blockIdx.x + 1) * GMn) / gridDim.x);
+        grid_arrive(sa.barrier);  // (its __syncthreads: every warp is done with the ring and its barriers)
+        issued = stream_begin<WT>((const unsigned char*)nx.W, nx.K, h0, h1, s, D, true);
+        if (!grid_wait(sa.barrier, (uint32_t)(p + 1), a.status, s.abort)) {
+            // never leave with copies in flight: wait (bounded) for this warp's first copies
+            const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+            if (lane == 0)
+                for (int j = 0; j < issued; ++j) mbar_wait(&s.full[warp * D + j], 0u, a.status, 100000000LL);
+            break;
+        }
+    }
 }
 
 // ---- host side ----------------------------------------------------------------------------
@@ -108,8 +154,15 @@ cudaError_t launch_t(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st
 
 }  // namespace
 
+template <typename WT, int BT>
+cudaError_t set_stack_attr(const DeviceInfo& dev) {
+    return cudaFuncSetAttribute(stack_kernel<WT, BT>, cudaFuncAttributeMaxDynamicSharedMemorySize, dev.max_smem_optin);
+}
+
 cudaError_t linear_prepare(const DeviceInfo& dev) {
     cudaError_t e;
+    if ((e = set_stack_attr<float, 1>(dev)) != cudaSuccess) return e;
+    if ((e = set_stack_attr<bf16_t, 1>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<float, 1>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<float, 2>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<float, 4>(dev)) != cudaSuccess) return e;
@@ -118,6 +171,31 @@ cudaError_t linear_prepare(const DeviceInfo& dev) {
     if ((e = set_attr<bf16_t, 2>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<bf16_t, 4>(dev)) != cudaSuccess) return e;
     return set_attr<bf16_t, 8>(dev);
+}
+
+// pipeline slots per warp for a stack whose largest K is k_max (B = 1); 0 if it does not fit
+int stack_slots(int k_max, const DeviceInfo& dev) {
+    const int Kpad = (k_max + 3) & ~3;
+    int D = stream_slots((size_t)dev.max_smem_optin, stream_smem_bytes(0, 1, Kpad, 1));
+    return D > kPreferredSlots ? kPreferredSlots : D;
+}
+
+cudaError_t launch_stack(fe_dtype dt, const StackArgs& sa, const DeviceInfo& dev, cudaStream_t st) {
+    if (sa.nph < 1 || sa.nph > kMaxStackPhases || !sa.barrier) return cudaErrorInvalidValue;
+    int kmax = 0;
+    for (int p = 0; p < sa.nph; ++p) {
+        if (sa.ph[p].B != 1 || sa.ph[p].M <= 0) return cudaErrorInvalidValue;
+        kmax = sa.ph[p].K > kmax ? sa.ph[p].K : kmax;
+    }
+    const int D = stack_slots(kmax, dev);
+    if (D < 1) return cudaErrorInvalidValue;
+    const int Kpad = (kmax + 3) & ~3;
+    const size_t smem = stream_smem_bytes(D, 1, Kpad, 1);
+    // one CTA per SM, all resident at once (the grid barrier needs them all)
+    const int grid = dev.num_sms;
+    return dt == FE_F32 ? launch_k(stack_kernel<float, 1>, dim3(grid), dim3(kStreamThreads), smem, st, sa.ph[0].pdl, sa, D, Kpad)
+                        : launch_k(stack_kernel<bf16_t, 1>, dim3(grid), dim3(kStreamThreads), smem, st, sa.ph[0].pdl, sa, D,
+                                   Kpad);
 }
 
 cudaError_t launch_linear(fe_dtype dt, const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {

@@ -71,6 +71,8 @@ struct fe_handle {
     uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
     float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
     int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
+    bool use_stack = false;      // B = 1 drafts run their linear phases as persistent stacks
+    uint32_t* stack_bar = nullptr;  // grid-barrier counters, one per stack of a draft
     uint16_t* lm_zb = nullptr;  // tensor-core LM head: bf16 hi/lo operand of the hidden rows
     int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
     cudaStream_t cap = nullptr;
@@ -168,10 +170,38 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     const int N = c.n_layers, nqkv = (H + 2 * Hkv) * hd;
     const fe_dtype dt = c.dtype;
     const bool pdl = h->use_pdl && !pf;  // profiled launches do not overlap
+    const bool stacked = h->use_stack && B == 1;
+    if (stacked) {
+        // the stacks' barrier counters start at zero in every draft
+        FE_TRY(cudaMemsetAsync(h->stack_bar, 0, (size_t)(N + 1) * sizeof(uint32_t), st));
+    }
     if (pf) FE_TRY(cudaEventRecord(pf->ev[0], st));
     // one linear phase: the CUDA-core streaming kernel, or operand prep + tensor-core product
+    // persistent stacks: linear phases are queued and launched together at the next
+    // attention (or at the LM head)
+    StackArgs sq{};
+    sq.nph = 0;
+    int nstack = 0;
+    auto flush_stack = [&]() -> fe_status {
+        if (sq.nph == 0) return FE_OK;
+        sq.barrier = h->stack_bar + nstack;
+        cudaError_t e = launch_stack(dt, sq, h->dev, st);
+        if (e != cudaSuccess) return fail(e, "linear stack launch", __LINE__);
+        if ((e = mark(pf, FE_KERNEL_LINEAR, st)) != cudaSuccess) return fail(e, "profiling event", __LINE__);
+        sq.nph = 0;
+        ++nstack;
+        return FE_OK;
+    };
     auto linear = [&](const LinearArgs& L) -> fe_status {
         cudaError_t e;
+        if (stacked) {
+            if (sq.nph == kMaxStackPhases) {
+                const fe_status r = flush_stack();
+                if (r != FE_OK) return r;
+            }
+            sq.ph[sq.nph++] = L;
+            return FE_OK;
+        }
         if (h->lin_mma) {
             if (pf) {
                 if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
@@ -190,6 +220,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     do {                                            \
         if ((lrc = linear(L)) != FE_OK) return lrc; \
     } while (0)
+
 
     LinearArgs la{};
     la.status = h->status;
@@ -229,6 +260,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         FE_LINEAR(la);
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
+        if ((lrc = flush_stack()) != FE_OK) return lrc;
         FE_TRY(launch_attention(dt, aa, st));
         FE_TRY(mark(pf, FE_KERNEL_ATTENTION, st));
         // x += W_o o
@@ -248,6 +280,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         FE_LINEAR(la);
     }
 
+    if ((lrc = flush_stack()) != FE_OK) return lrc;
     const float inv_temp = a->temperature > 0.f ? 1.0f / a->temperature : 1.0f;
     LmHeadArgs lm{};
     lm.W = h->lm_head; lm.gamma = h->final_norm; lm.V = V; lm.d = d; lm.R = N * B; lm.B = B; lm.N = N;
@@ -398,6 +431,14 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                                 c.ffn % 64 == 0 && (c.n_heads * c.head_dim) % 64 == 0;
             const char* lm = getenv("FE_DRAFT_LINEAR_MMA");
             h->lin_mma = shapes && (lm ? lm[0] == '1' : c.max_batch > 8);
+            // FE_DRAFT_STACK=1: B = 1 drafts on the CUDA-core path run their linear phases as
+            // persistent stacks (when one pipeline slot per warp fits next to the largest
+            // activation row). Off by default: measured on GB300, the separate launches with
+            // programmatic dependent launch inside the CUDA graph are faster (720 vs 762 us
+            // per Vicuna-13B-shaped draft); the stacks win only without programmatic launch.
+            const int kmax = std::max({3 * c.d, c.ffn, c.n_heads * c.head_dim});
+            const char* sk = getenv("FE_DRAFT_STACK");
+            h->use_stack = !h->lin_mma && sk && sk[0] == '1' && stack_slots(kmax, h->dev) >= 1;
         }
 
         // ---- packed weights: one allocation, every matrix 256-byte aligned ----
@@ -513,8 +554,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         const size_t k = c.top_k_max;
         const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
         const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
-        size_t off[18], n = 0, tot = 0;
-        const size_t bytes[18] = {
+        size_t off[19], n = 0, tot = 0;
+        const size_t bytes[19] = {
             cs.size() * sizeof(float),                             // rope
             B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
             B * F * 4, R * d * 4,                                  // act, hid
@@ -528,8 +569,9 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                                  lmhead_wide_zb_bytes((int)R, c.d)) : 0,  // tensor-core LM-head operand
             h->lin_mma ? linear_mma_xb_bytes((int)kmax, c.max_batch) : 0,  // tensor-core linear operand
             h->lin_mma ? linear_mma_part_bytes(c.max_batch, h->dev) : 0,   // its split-tile partials
-            h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0};      // its completion counters
-        for (n = 0; n < 18; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0,      // its completion counters
+            h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0};  // stack barrier counters
+        for (n = 0; n < 19; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -550,6 +592,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lin_xb = h->lin_mma ? (uint16_t*)(s + off[15]) : nullptr;
         h->lin_part = h->lin_mma ? (float*)(s + off[16]) : nullptr;
         h->lin_counters = h->lin_mma ? (int*)(s + off[17]) : nullptr;
+        h->stack_bar = h->use_stack ? (uint32_t*)(s + off[18]) : nullptr;
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
@@ -669,7 +712,9 @@ int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     if (!h || B < 1) return -1;
     const int N = h->cfg.n_layers;
     const int lin = h->lin_mma ? 2 : linear_launches();
-    int n = 2 * lin + N * (4 * lin + attention_launches()) +
+    // stacked: N + 1 stack launches hold all linear phases
+    const int lin_total = (h->use_stack && B == 1) ? N + 1 : 2 * lin + N * 4 * lin;
+    int n = lin_total + N * attention_launches() +
             (h->lm_mma ? (N * B <= 16 ? 2 : 3) : lmhead_launches(N * B, h->cfg.d, h->dev));
     return n + (with_tree ? 1 : 0);
 }

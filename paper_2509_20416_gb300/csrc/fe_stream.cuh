@@ -197,8 +197,11 @@ __device__ __forceinline__ void stream_issue(const unsigned char* Wt, int K, int
 // First half of a stream: initialise the per-warp barriers and issue every warp's first D
 // copies. Touches only the (read-only) weights, so it may run before griddep_wait().
 // Must be called by all 256 threads; returns the number of copies this warp issued.
+// `again`: a later stream of the same CTA (persistent kernel): the barriers are retired
+// first (the previous stream consumed every copy) and the abort flag is kept.
 template <typename WT>
-__device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D) {
+__device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D,
+                            bool again = false) {
     using G = StreamGeom<WT>;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nks = (K + G::kKS - 1) / G::kKS;
@@ -207,8 +210,11 @@ __device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, Stre
     unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
     int issued = 0;
     if (lane == 0) {
-        for (int d = 0; d < D; ++d) mbar_init(&full[d], 1);
-        if (warp == 0) *s.abort = 0;
+        for (int d = 0; d < D; ++d) {
+            if (again) mbar_inval(&full[d]);
+            mbar_init(&full[d], 1);
+        }
+        if (warp == 0 && !again) *s.abort = 0;
         mbar_fence_init();
         for (int j = 0; j < D && warp + kWarps * j < total; ++j, ++issued)
             stream_issue<WT>(Wt, K, g0, nks, warp + kWarps * j, j, full, ring);

@@ -31,8 +31,13 @@ def test_profile_forward_matches_forward(spec):
     N = cfg["n_layers"]
     kinds = [k for k, _ in prof]
     assert len(prof) == fe.fe_launch_count(h, cfg["B"], False)
-    assert kinds[:2] == ["linear", "linear"]
-    assert kinds[2:2 + 5 * N] == ["linear", "attention", "linear", "linear", "linear"] * N
-    assert kinds[-1] == "lm_head"
+    # linear phases run as separate launches (2 + 4 per layer) or, at B = 1 with
+    # FE_DRAFT_STACK=1, as N + 1 persistent stacks
+    att = [j for j, kd in enumerate(kinds) if kd == "attention"]
+    assert len(att) == N
+    n_lin = kinds.count("linear")
+    assert n_lin in (2 + 4 * N, N + 1)
+    assert all(kinds[j - 1] == "linear" for j in att)
+    assert kinds[0] == "linear" and kinds[-1] == "lm_head"
     assert all(us > 0 for _, us in prof)
     h.close()
