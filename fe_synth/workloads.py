@@ -68,6 +68,7 @@ def make_config(name_or_dict, **overrides) -> dict:
     w.update(overrides)
     w.setdefault("rms_eps", RMS_EPS)
     w.setdefault("temperature", 0.0)
+    w.setdefault("parallel_layers", 0)  # 1: the parallel (non-cascaded) ablation, Sec. 3.2
     p = w["prefix"]
     pmax = p[1] if isinstance(p, (tuple, list)) else p
     if w.get("prefix_list") is not None:  # explicit per-sequence prefix lengths

@@ -72,6 +72,9 @@ typedef struct {
     float rope_theta;   /* RoPE base */
     float rms_eps;      /* RMSNorm epsilon */
     fe_dtype dtype;     /* storage type of weights, features and caches */
+    int32_t parallel_layers; /* 0: the cascade, L_i consumes h_{i-1} (Eq. 2); 1: every L_i
+                                consumes x0 — the "w/o cascaded structure" ablation of
+                                Sec. 3.2 (Table 2), parallel instead of serial layers */
 } fe_config;
 
 /* One cascade layer L_i (Eq. 2): RMSNorm gains [d]; w_qkv [(H + 2 Hkv) hd, d] with the

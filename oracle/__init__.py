@@ -53,7 +53,8 @@ class Config(ctypes.Structure):
                 ("ffn", ctypes.c_int32), ("vocab", ctypes.c_int32),
                 ("n_layers", ctypes.c_int32), ("dtype", ctypes.c_int32),
                 ("rope_theta", ctypes.c_double), ("rms_eps", ctypes.c_double),
-                ("rope_layer_offset", ctypes.c_int32), ("final_norm", ctypes.c_int32)]
+                ("rope_layer_offset", ctypes.c_int32), ("final_norm", ctypes.c_int32),
+                ("parallel_layers", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -186,7 +187,7 @@ class Oracle:
     def draft_seq(self, cfg: dict, weights: dict, feat_b, tok: int, P: int, kcs, vcs, cap: int,
                   top_k: int, temperature: float = 0.0, want_logits: bool = True,
                   rope_layer_offset: int = 0, final_norm: int = 1):
-        """One sequence's draft. ``weights`` holds host tensors in the canonical layout
+        """One sequence's draft (cfg["parallel_layers"] = 1: every layer consumes x0). ``weights`` holds host tensors in the canonical layout
         (see fe_synth.workloads); ``kcs``/``vcs`` are N host buffers of this sequence's
         [Hkv, cap, hd] cache. Returns a dict of float64 / int32 numpy arrays."""
         c = config_struct(cfg, rope_layer_offset, final_norm)
@@ -228,7 +229,8 @@ class Oracle:
 def config_struct(cfg: dict, rope_layer_offset: int = 0, final_norm: int = 1) -> Config:
     return Config(cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"], cfg["ffn"],
                   cfg["vocab"], cfg["n_layers"], 0 if cfg["dtype"] == "f32" else 1,
-                  float(cfg["rope_theta"]), float(cfg["rms_eps"]), rope_layer_offset, final_norm)
+                  float(cfg["rope_theta"]), float(cfg["rms_eps"]), rope_layer_offset, final_norm,
+                  int(cfg.get("parallel_layers", 0)))
 
 
 def load(mutant: int = 0, outdir: str | None = None) -> Oracle:

@@ -47,6 +47,9 @@ typedef struct {
     int32_t rope_layer_offset; /* reading of the query position: 0 -> every layer at P (default),
                                   1 -> layer i at P + i - 1 */
     int32_t final_norm;        /* 1 -> RMSNorm(gamma_out) before the LM head (default), 0 -> none */
+    int32_t parallel_layers;   /* 0 -> the cascade, L_i consumes h_{i-1} (Eq. 2, default);
+                                  1 -> every L_i consumes x0: the "w/o cascaded structure"
+                                  ablation of Sec. 3.2 (Table 2), parallel instead of serial */
 } or_config;
 
 /* ---- storage ------------------------------------------------------------------ */
@@ -364,9 +367,9 @@ int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat,
     or_matvec(w[1], c->dtype, d, 2 * d, ge, x0);
     memcpy(x, x0, sizeof(double) * (size_t)d);
 
-    /* h_i = L_i(h_{i-1})      (Eq. 2) */
+    /* h_i = L_i(h_{i-1})      (Eq. 2), or h_i = L_i(x0) for the parallel ablation */
     for (int32_t i = 0; i < N; ++i) {
-        if (MUT(10))
+        if (c->parallel_layers || MUT(10))
             memcpy(x, x0, sizeof(double) * (size_t)d);
         double pos = (double)P + (c->rope_layer_offset ? (double)i : 0.0) + (MUT(19) ? 1.0 : 0.0);
         or_layer(c, w + 5 + 7 * i, pos, kc[i], vc[i], cap, P, x);

@@ -35,7 +35,8 @@ class fe_config(ctypes.Structure):
     _fields_ = [("d", _i32), ("n_heads", _i32), ("n_kv_heads", _i32), ("head_dim", _i32),
                 ("ffn", _i32), ("vocab", _i32), ("n_layers", _i32), ("top_k_max", _i32),
                 ("max_batch", _i32), ("max_seq", _i32), ("page_size", _i32),
-                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int)]
+                ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int),
+                ("parallel_layers", _i32)]
 
 
 class fe_layer_weights(ctypes.Structure):
@@ -123,7 +124,7 @@ def make_config(cfg: dict) -> fe_config:
     return fe_config(cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"], cfg["ffn"], cfg["vocab"],
                      cfg["n_layers"], cfg["top_k_max"], cfg.get("max_batch", cfg.get("B", 1)), cfg["max_seq"],
                      cfg.get("page_size", 0), float(cfg["rope_theta"]), float(cfg["rms_eps"]),
-                     FE_F32 if cfg["dtype"] == "f32" else FE_BF16)
+                     FE_F32 if cfg["dtype"] == "f32" else FE_BF16, int(cfg.get("parallel_layers", 0)))
 
 
 class Handle:

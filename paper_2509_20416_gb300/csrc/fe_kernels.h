@@ -75,6 +75,7 @@ struct LinearArgs {
     int ldy;
     float* y2;
     int ldy2;
+    const float* ybase;  // EPI_RESID: y = ybase + acc (same layout as y) when set, else y += acc
     int* status;
     bool pdl;  // launch overlapping the previous kernel (programmatic dependent launch)
 };

@@ -32,7 +32,8 @@ struct LinearEpi {
                 const float v = chunk_value<BT>(red, gl, r, b);
                 float* yp = a->y + (size_t)(b0 + b) * a->ldy + m;
                 if (a->epi == EPI_RESID) {
-                    const float nv = __ldcg(yp) + v;  // (L2: another CTA may have written it in a persistent kernel)
+                    // (read through L2: another CTA may have written it in a persistent kernel)
+                    const float nv = __ldcg(a->ybase ? a->ybase + (size_t)(b0 + b) * a->ldy + m : yp) + v;
                     *yp = nv;
                     if (a->y2) a->y2[(size_t)(b0 + b) * a->ldy2 + m] = nv;
                 } else {

@@ -161,7 +161,7 @@ __device__ __forceinline__ void lin_epilogue(const LinearArgs& a, int m, const f
         if (b >= a.B) break;
         float* yp = a.y + (size_t)b * a.ldy + m;
         if (a.epi == EPI_RESID) {
-            const float nv = *yp + v[b];
+            const float nv = __ldcg(a.ybase ? a.ybase + (size_t)b * a.ldy + m : yp) + v[b];
             *yp = nv;
             if (a.y2) a.y2[(size_t)b * a.ldy2 + m] = nv;
         } else {

@@ -60,6 +60,7 @@ struct fe_handle {
     float* rope_cs = nullptr;
     void* sbuf = nullptr;
     float *g = nullptr, *x = nullptr, *qkv = nullptr, *o = nullptr, *act = nullptr, *hid = nullptr;
+    float* x0 = nullptr;  // the cascade input x0 (Eq. 1), kept for layer 1 and the parallel ablation
     float* attn_part = nullptr;
     int* lm_part_id = nullptr;
     float *lm_part_val = nullptr, *lm_part_ms = nullptr;
@@ -113,6 +114,7 @@ bool valid_config(const fe_config* c) {
     if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f)) return false;
     if (c->dtype != FE_F32 && c->dtype != FE_BF16) return false;
     if (c->head_dim <= 0 || c->head_dim % 2) return false;
+    if (c->parallel_layers != 0 && c->parallel_layers != 1) return false;
     return true;
 }
 
@@ -239,7 +241,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.W = h->w_in; la.M = d; la.K = 2 * d;
     la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
     la.d_split = d; la.vocab = V;
-    la.epi = EPI_STORE; la.y = h->x; la.ldy = d;
+    la.epi = EPI_STORE; la.y = h->x0; la.ldy = d;
     FE_LINEAR(la);
 
     AttnArgs aa{};
@@ -255,7 +257,9 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         const LayerPacked& L = h->layers[i];
         // qkv = W_qkv RMSNorm(x)
         la.W = L.w_qkv; la.M = nqkv; la.K = d;
-        la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.attn_norm;
+        // L_1 (and every L_i of the parallel ablation) reads x0; the cascade's L_i reads h_{i-1}
+        const bool from_x0 = i == 0 || c.parallel_layers;
+        la.pro = PRO_RMSNORM; la.x = from_x0 ? h->x0 : h->x; la.ldx = d; la.gamma = L.attn_norm;
         la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
         FE_LINEAR(la);
         // attention over the layer's cache (+ own row), appends slot P_b
@@ -266,11 +270,11 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         // x += W_o o
         la.W = L.w_o; la.M = d; la.K = H * hd;
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
-        la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr;
+        la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr; la.ybase = from_x0 ? h->x0 : nullptr;
         FE_LINEAR(la);
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
-        la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm;
+        la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm; la.ybase = nullptr;
         la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
         FE_LINEAR(la);
         // x += W_down a; h_i = x
@@ -554,8 +558,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         const size_t k = c.top_k_max;
         const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
         const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
-        size_t off[19], n = 0, tot = 0;
-        const size_t bytes[19] = {
+        size_t off[20], n = 0, tot = 0;
+        const size_t bytes[20] = {
             cs.size() * sizeof(float),                             // rope
             B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
             B * F * 4, R * d * 4,                                  // act, hid
@@ -570,8 +574,9 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             h->lin_mma ? linear_mma_xb_bytes((int)kmax, c.max_batch) : 0,  // tensor-core linear operand
             h->lin_mma ? linear_mma_part_bytes(c.max_batch, h->dev) : 0,   // its split-tile partials
             h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0,      // its completion counters
-            h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0};  // stack barrier counters
-        for (n = 0; n < 19; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0,  // stack barrier counters
+            B * d * 4};                                                       // x0
+        for (n = 0; n < 20; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -593,6 +598,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lin_part = h->lin_mma ? (float*)(s + off[16]) : nullptr;
         h->lin_counters = h->lin_mma ? (int*)(s + off[17]) : nullptr;
         h->stack_bar = h->use_stack ? (uint32_t*)(s + off[18]) : nullptr;
+        h->x0 = (float*)(s + off[19]);
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero

@@ -338,6 +338,26 @@ def pin_truncation(orc):
         assert np.array_equal(o4[key][:2], o2[key]), key
 
 
+def pin_parallel_layers(orc):
+    """The parallel ablation (Sec. 3.2, Table 2: every L_i consumes x0): layer i's output
+    equals a one-layer cascade built from L_i alone (same features, token, position and
+    layer-i cache), and differs from the cascade's h_i beyond the first layer."""
+    cfg = mini_cfg(n_layers=3, B=1)
+    W, I, ks, vs = _mini_problem(cfg)
+    feat, tok = I["feat"][0].contiguous(), int(I["next_tok"][0])
+    kb = [k[0].contiguous() for k in ks]
+    vb = [v[0].contiguous() for v in vs]
+    par = orc.draft_seq(dict(cfg, parallel_layers=1), W, feat, tok, 3, kb, vb, cfg["max_seq"], cfg["top_k"])
+    cas = orc.draft_seq(cfg, W, feat, tok, 3, kb, vb, cfg["max_seq"], cfg["top_k"])
+    for i in range(cfg["n_layers"]):
+        one = orc.draft_seq(dict(cfg, n_layers=1), dict(W, layers=[W["layers"][i]]), feat, tok, 3, [kb[i]],
+                            [vb[i]], cfg["max_seq"], cfg["top_k"])
+        for key in ("hidden", "logits", "lse", "topk_id"):
+            assert np.array_equal(par[key][i], one[key][0]), (i, key)
+    assert np.array_equal(par["hidden"][0], cas["hidden"][0])
+    assert np.abs(par["hidden"][1:] - cas["hidden"][1:]).max() > 1e-3
+
+
 def pin_zero_blocks(orc):
     """W_o = W_down = 0: every layer passes x0 through, so all N distributions coincide."""
     cfg = mini_cfg(n_layers=3, B=1)
@@ -361,6 +381,6 @@ def pin_zero_blocks(orc):
         assert list(tok[1 + i * k: 1 + (i + 1) * k]) == list(tok[1:1 + k])
 
 
-ALL_PINS = [pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
+ALL_PINS = [pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
             pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]

@@ -25,7 +25,7 @@ def _problem(cfg):
 def _new_row_ref(cfg, W, I, o, b, i):
     """Expected key (after RoPE) and value the call appends to layer i's slot P_b."""
     d, Hh, Hkv, hd = cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
-    if i == 0:
+    if i == 0 or cfg.get("parallel_layers", 0):  # the layer's input is x0
         f = I["feat"][b].double()
         g = W["w_fuse"].double() @ f
         e = W["embed"].double()[int(I["next_tok"][b])]
@@ -88,6 +88,14 @@ SMALL = {
     "tc_linear_b9_paged": dict(name=dict(d=1024, n_heads=8, n_kv_heads=8, head_dim=128, ffn=2816, vocab=3001,
                                          n_layers=2, dtype="bf16", B=9, prefix=0, top_k=4, rope_theta=5e5,
                                          seed=10, page_size=16), prefix_list=[15, 16, 1, 200, 0, 31, 33, 64, 100]),
+    # the "w/o cascaded structure" ablation (Sec. 3.2, Table 2): every layer consumes x0
+    "parallel_gqa4_bf16": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376, vocab=5003,
+                                         n_layers=4, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
+                                         seed=13, page_size=0, parallel_layers=1), prefix_list=[37, 0, 150]),
+    "parallel_tc_b12": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1408, vocab=5003,
+                                      n_layers=3, dtype="bf16", B=12, prefix=0, top_k=8, rope_theta=1e4,
+                                      seed=14, page_size=0, parallel_layers=1),
+                            prefix_list=[37, 0, 150, 1, 64, 5, 300, 2, 128, 129, 7, 90]),
     # N * B = 160 rows: the wide tensor-core LM head with three 64-row transpose groups
     "wide_lmhead_r160": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=3001,
                                        n_layers=5, dtype="bf16", B=32, prefix=0, top_k=8, rope_theta=1e4,
