@@ -316,6 +316,21 @@ def main():
     kernels = {kind: {"launches_per_draft": v[0] / n_prof, "us_per_draft": v[1] / n_prof,
                       "us_per_launch": v[1] / v[0], "share": v[1] / prof_total} for kind, v in per.items()}
 
+    # ---- verification side (not part of the draft step): positions + greedy acceptance walk --
+    T = 1 + N * k
+    g = torch.Generator().manual_seed(1)
+    target_next = torch.randint(0, cfg["vocab"], (B, T), generator=g, dtype=torch.int32).cuda()
+    vout = fe.fe_verify_greedy(h, plen, tree, target_next, k, stream=stream)
+    for _ in range(3):
+        fe.fe_verify_greedy(h, plen, tree, target_next, k, out=vout, stream=stream)
+    v0, v1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    v0.record(stream)
+    for _ in range(100):
+        fe.fe_verify_greedy(h, plen, tree, target_next, k, out=vout, stream=stream)
+    v1.record(stream)
+    v1.synchronize()
+    verify_us = 1000.0 * v0.elapsed_time(v1) / 100
+
     # ---- roofline of the dominant kernel (and of the whole step, for context) ----------------
     peak, peak_kind = peaks()
     plist = I["prefix_len"].tolist()
@@ -348,6 +363,8 @@ def main():
                          "step": {"achieved": step_achieved, "frac": step_achieved / peak,
                                   "algorithmic_bytes": alg_bytes}},
             "kernels": kernels,
+            "verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
+                              "note": "fe_verify_greedy after the step (positions + greedy acceptance walk)"},
             "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": launches * args.steps, "launches_per_step": launches,

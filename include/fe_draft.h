@@ -183,6 +183,25 @@ FE_API const char *fe_last_error_detail(void);
  * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
 FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);
 
+/* Verification side of a cycle (Sec. 2.4, "Parallel Verification"), after the target model
+ * has scored the draft tree under tree attention. For each sequence b of a tree built by
+ * fe_build_tree (top_k candidates per level, T = 1 + N top_k nodes):
+ *   pos_ids [B, T] = prefix_len[b] + depth: the nodes' sequence positions for the target's
+ *            tree-attention pass (the root, the token fed to the drafter, sits right after
+ *            the P_b-token prefix);
+ *   the greedy acceptance walk: from the root, the child (first in node order) whose token
+ *   equals target_next[b, current] — the target's greedy token after the current node —
+ *   is accepted and becomes current, until no child matches:
+ *   n_accept [B] accepted draft tokens (0..N), path [B, N] their node ids (-1 after),
+ *   bonus [B] = target_next at the last accepted node (or the root): the target's own
+ *   next token, which a cycle emits in addition.
+ * All pointers are device pointers (tree: tok, parent and depth are read; mask is not);
+ * target_next [B, T] int32. Asynchronous on `stream`; FE_ERR_INVALID_ARG for bad arguments.
+ * Stochastic (T > 0) speculative sampling over the tree is not covered. */
+FE_API fe_status fe_verify_greedy(fe_handle *h, int32_t B, int32_t top_k, const int32_t *prefix_len,
+                                  const fe_tree *tree, const int32_t *target_next, int32_t *pos_ids,
+                                  int32_t *path, int32_t *n_accept, int32_t *bonus, void *stream);
+
 /* Kernel families of one draft, as fe_profile_forward reports them. */
 typedef enum {
     FE_KERNEL_LINEAR = 0,    /* weight-streaming linear phase (W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down) */

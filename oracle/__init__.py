@@ -27,7 +27,7 @@ _lock = threading.Lock()
 _cache: dict = {}
 
 # Number of planted-mistake variants compiled by build(mutant=n) (n = 1..N_MUTANTS).
-N_MUTANTS = 28
+N_MUTANTS = 30
 _UNUSED_MUTANTS = {25}  # ids with no planted mistake
 
 
@@ -99,6 +99,9 @@ class Oracle:
         L.or_lm_head.argtypes = [ctypes.POINTER(Config), _P, _P, _D, _D]
         L.or_softmax.argtypes = [_D, ctypes.c_int64, ctypes.c_double, _D, _D]
         L.or_topk.argtypes = [_D, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]
+        _I = ctypes.POINTER(ctypes.c_int32)
+        L.or_accept_greedy.argtypes = [ctypes.c_int32, _I, _I, _I, _I, ctypes.c_int32, ctypes.c_int32, _I, _I, _I]
+        L.or_accept_greedy.restype = ctypes.c_int32
         L.or_tree.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                               ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
                               ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
@@ -179,6 +182,22 @@ class Oracle:
                        par.ctypes.data_as(i32), dep.ctypes.data_as(i32),
                        mask.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
         return tok, par, dep, mask
+
+    def accept_greedy(self, tok, parent, depth, target_next, P: int, max_path: int):
+        """Tree positions and the greedy acceptance walk of one sequence (Sec. 2.4).
+        Returns (pos [T], path [max_path] with -1 after the accepted nodes, n, bonus)."""
+        i32 = ctypes.POINTER(ctypes.c_int32)
+        tok, parent, depth, target_next = (np.ascontiguousarray(a, dtype=np.int32) for a in
+                                           (tok, parent, depth, target_next))
+        T = tok.shape[0]
+        pos = np.zeros(T, np.int32)
+        path = np.zeros(max_path, np.int32)
+        bonus = ctypes.c_int32(0)
+        n = self.L.or_accept_greedy(T, tok.ctypes.data_as(i32), parent.ctypes.data_as(i32),
+                                    depth.ctypes.data_as(i32), target_next.ctypes.data_as(i32), int(P),
+                                    int(max_path), pos.ctypes.data_as(i32), path.ctypes.data_as(i32),
+                                    ctypes.byref(bonus))
+        return pos, path, int(n), int(bonus.value)
 
     def max_threads(self) -> int:
         return int(self.L.or_max_threads())

@@ -326,6 +326,38 @@ void or_tree(int32_t N, int32_t k, int32_t root, const int32_t *topk, int32_t *t
     }
 }
 
+/* Verification side of one cycle (Sec. 2.4, "Parallel Verification"), for one sequence's
+ * draft tree of T nodes (or_tree's tok, parent, depth):
+ *   pos[a] = P + depth[a]: the sequence position of node a under tree attention (the root,
+ *            the token fed to the drafter, sits right after the P-token prefix);
+ *   the greedy acceptance walk: starting at the root, the child of the current node whose
+ *   token equals target_next[current] (the target model's greedy token after that node) is
+ *   accepted and becomes current, until no child matches. path[0..n) are the accepted node
+ *   ids (-1 after), *bonus = target_next[last accepted node, or the root]; returns n. Children
+ *   are searched in node order, so with repeated tokens among siblings the first one wins. */
+int32_t or_accept_greedy(int32_t T, const int32_t *tok, const int32_t *parent, const int32_t *depth,
+                         const int32_t *target_next, int32_t P, int32_t max_path, int32_t *pos,
+                         int32_t *path, int32_t *bonus)
+{
+    for (int32_t a = 0; a < T; ++a)
+        pos[a] = P + depth[a] + (MUT(29) ? 1 : 0);
+    int32_t cur = 0, n = 0;
+    while (n < max_path) {
+        int32_t next = -1;
+        for (int32_t c = 1; c < T && next < 0; ++c)
+            if (parent[c] == cur && tok[c] == target_next[MUT(30) ? c : cur])
+                next = c;
+        if (next < 0)
+            break;
+        path[n++] = next;
+        cur = next;
+    }
+    for (int32_t i = n; i < max_path; ++i)
+        path[i] = -1;
+    *bonus = target_next[cur];
+    return n;
+}
+
 /* The whole draft of one sequence (Eq. 1, Eq. 2, Sec. 2.1 LM head, Sec. 2.2 top-k).
  *   w     : 5 + 7N pointers: w_fuse [d,3d], w_in [d,2d], embed [V,d], lm_head [V,d],
  *           final_norm [d], then per layer attn_norm, w_qkv, w_o, mlp_norm, w_gate,

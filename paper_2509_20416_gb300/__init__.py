@@ -81,6 +81,8 @@ _lib.fe_lm_head_topk_noalloc.argtypes = [_vp, _vp, _i32, _i32, ctypes.c_float, _
 _lib.fe_lm_head_topk_noalloc.restype = ctypes.c_int
 _lib.fe_profile_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _i32, _vp, _vp, ctypes.POINTER(_i32)]
 _lib.fe_profile_forward.restype = ctypes.c_int
+_lib.fe_verify_greedy.argtypes = [_vp, _i32, _i32, _vp, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp]
+_lib.fe_verify_greedy.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
 _lib.fe_last_error_detail.restype = ctypes.c_char_p
 
@@ -228,6 +230,26 @@ def fe_build_tree(h: Handle, next_tok, topk_id, top_k: int, out: dict | None = N
     t = fe_tree(_p(out["tok"]), _p(out["parent"]), _p(out["depth"]), _p(out["mask"]))
     _check(_lib.fe_build_tree(h.ptr, B, top_k, _p(next_tok), _p(topk_id), ctypes.byref(t), _stream(stream)),
            "fe_build_tree")
+    return out
+
+
+def fe_verify_greedy(h: Handle, prefix_len, tree: dict, target_next, top_k: int, out: dict | None = None,
+                     stream=None) -> dict:
+    """Tree positions and the greedy acceptance walk (include/fe_draft.h). tree: the dict
+    fe_build_tree returns; target_next [B, T] int32 (device)."""
+    B = int(prefix_len.shape[0])
+    N = h.cfg["n_layers"]
+    T = 1 + N * top_k
+    dev = prefix_len.device
+    if out is None:
+        out = dict(pos_ids=torch.empty((B, T), dtype=torch.int32, device=dev),
+                   path=torch.empty((B, N), dtype=torch.int32, device=dev),
+                   n_accept=torch.empty(B, dtype=torch.int32, device=dev),
+                   bonus=torch.empty(B, dtype=torch.int32, device=dev))
+    t = fe_tree(_p(tree["tok"]), _p(tree["parent"]), _p(tree["depth"]), _p(tree["mask"]))
+    _check(_lib.fe_verify_greedy(h.ptr, B, int(top_k), _p(prefix_len), ctypes.byref(t), _p(target_next),
+                                 _p(out["pos_ids"]), _p(out["path"]), _p(out["n_accept"]), _p(out["bonus"]),
+                                 _stream(stream)), "fe_verify_greedy")
     return out
 
 

@@ -693,6 +693,18 @@ fe_status fe_build_tree(fe_handle* h, int32_t B, int32_t top_k, const int32_t* n
     return FE_OK;
 }
 
+fe_status fe_verify_greedy(fe_handle* h, int32_t B, int32_t top_k, const int32_t* prefix_len, const fe_tree* tree,
+                           const int32_t* target_next, int32_t* pos_ids, int32_t* path, int32_t* n_accept,
+                           int32_t* bonus, void* stream) {
+    if (!h || !tree || !prefix_len || !target_next || !pos_ids || !path || !n_accept || !bonus) return FE_ERR_INVALID_ARG;
+    if (!tree->tok || !tree->parent || !tree->depth) return FE_ERR_INVALID_ARG;
+    if (B < 1 || B > h->cfg.max_batch || top_k < 1 || top_k > h->cfg.top_k_max) return FE_ERR_INVALID_ARG;
+    const int N = h->cfg.n_layers, T = 1 + N * top_k;
+    FE_TRY(launch_verify(B, T, N, prefix_len, tree->tok, tree->parent, tree->depth, target_next, pos_ids, path,
+                         n_accept, bonus, (cudaStream_t)stream));
+    return FE_OK;
+}
+
 fe_status fe_last_device_status(fe_handle* h, void* stream) {
     if (!h) return FE_ERR_INVALID_ARG;
     cudaStream_t st = (cudaStream_t)stream;

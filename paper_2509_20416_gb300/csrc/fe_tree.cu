@@ -52,6 +52,54 @@ cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const i
     return cudaGetLastError();
 }
 
+// ---- verification side (Sec. 2.4, "Parallel Verification") --------------------------------
+// One warp per sequence: the tree positions pos[a] = P_b + depth[a], then the greedy
+// acceptance walk — from the root, the child (first in node order) whose token equals the
+// target's greedy token after the current node is accepted and becomes current, until no
+// child matches; the children of a node are found with one ballot per 32 nodes. Every
+// index the walk follows comes from the node range, so malformed parents or tokens can
+// only end the walk early.
+__global__ void verify_kernel(int T, int max_path, const int* prefix_len, const int* tok, const int* parent,
+                              const int* depth, const int* target_next, int* pos, int* path, int* n_accept,
+                              int* bonus) {
+    const int b = blockIdx.x, lane = threadIdx.x;
+    const int* tk = tok + (size_t)b * T;
+    const int* pr = parent + (size_t)b * T;
+    const int* tn = target_next + (size_t)b * T;
+    const int P = prefix_len[b];
+    for (int a = lane; a < T; a += 32) pos[(size_t)b * T + a] = P + depth[(size_t)b * T + a];
+    int cur = 0, n = 0;
+    while (n < max_path) {
+        const int want = tn[cur];
+        int next = -1;
+        for (int c0 = 1; c0 < T; c0 += 32) {
+            const int c = c0 + lane;
+            const unsigned m = __ballot_sync(0xffffffffu, c < T && pr[c] == cur && tk[c] == want);
+            if (m) {
+                next = c0 + __ffs(m) - 1;
+                break;
+            }
+        }
+        if (next < 0) break;
+        if (lane == 0) path[(size_t)b * max_path + n] = next;
+        ++n;
+        cur = next;
+    }
+    for (int i = n + lane; i < max_path; i += 32) path[(size_t)b * max_path + i] = -1;
+    if (lane == 0) {
+        n_accept[b] = n;
+        bonus[b] = tn[cur];
+    }
+}
+
+cudaError_t launch_verify(int B, int T, int max_path, const int* prefix_len, const int* tok, const int* parent,
+                          const int* depth, const int* target_next, int* pos, int* path, int* n_accept, int* bonus,
+                          cudaStream_t st) {
+    verify_kernel<<<B, 32, 0, st>>>(T, max_path, prefix_len, tok, parent, depth, target_next, pos, path, n_accept,
+                                    bonus);
+    return cudaGetLastError();
+}
+
 // One thread waits on an mbarrier that nothing will complete; the bounded wait gives up
 // after timeout_ns and records ST_TIMEOUT. Exercises the failure path of every ring and
 // grid wait without hanging the GPU.

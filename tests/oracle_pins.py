@@ -358,6 +358,44 @@ def pin_parallel_layers(orc):
     assert np.abs(par["hidden"][1:] - cas["hidden"][1:]).max() > 1e-3
 
 
+def pin_accept_greedy(orc):
+    """Tree positions and the greedy acceptance walk (Sec. 2.4): hand-worked cases on a
+    Backbone Expansion tree, and brute force over every root-to-node path of random trees
+    (the walk must end at the deepest node whose whole path matches the target)."""
+    g = json.load(open(os.path.join(GOLDEN, "accept_greedy_n3_k3.json")))
+    for case in g["cases"]:
+        pos, path, n, bonus = orc.accept_greedy(g["tok"], g["parent"], g["depth"], case["target_next"], g["P"],
+                                                g["N"])
+        assert pos.tolist() == g["pos"], case["why"]
+        assert (n, path.tolist(), bonus) == (case["n"], case["path"], case["bonus"]), case["why"]
+    rng = np.random.default_rng(5)
+    for trial in range(200):
+        N, k, V = int(rng.integers(1, 6)), int(rng.integers(1, 5)), 12
+        topk = np.stack([rng.permutation(V)[:k] for _ in range(N)]).astype(np.int32)
+        tok, par, dep, _ = orc.tree(N, k, int(rng.integers(0, V)), topk)
+        T = len(tok)
+        tn = rng.integers(0, V, T).astype(np.int32)
+        for a in range(1, T):  # plant matches so that walks of every length occur
+            if rng.random() < 0.6:
+                tn[par[a]] = tok[a]
+        pos, path, n, bonus = orc.accept_greedy(tok, par, dep, tn, 7, N)
+        assert np.array_equal(pos, 7 + dep)
+
+        def ok(a):  # every edge on a's root path carries the target's token
+            while par[a] >= 0:
+                if tok[a] != tn[par[a]]:
+                    return False
+                a = par[a]
+            return True
+        best = max((a for a in range(T) if ok(a)), key=lambda a: (dep[a], -a))
+        assert n == dep[best] and bonus == tn[best]
+        chain, a = [], best
+        while par[a] >= 0:
+            chain.append(a)
+            a = par[a]
+        assert path[:n].tolist() == chain[::-1] and (path[n:] == -1).all()
+
+
 def pin_zero_blocks(orc):
     """W_o = W_down = 0: every layer passes x0 through, so all N distributions coincide."""
     cfg = mini_cfg(n_layers=3, B=1)
@@ -381,6 +419,6 @@ def pin_zero_blocks(orc):
         assert list(tok[1 + i * k: 1 + (i + 1) * k]) == list(tok[1:1 + k])
 
 
-ALL_PINS = [pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
+ALL_PINS = [pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
             pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]
