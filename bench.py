@@ -331,6 +331,25 @@ def main():
     v1.synchronize()
     verify_us = 1000.0 * v0.elapsed_time(v1) / 100
 
+    # ---- training-objective forward (not part of the draft step): fe_draft_loss = the draft with
+    # its full-vocabulary logits and hidden states written out, then the loss kernels ----------
+    V, d = cfg["vocab"], cfg["d"]
+    teacher = torch.softmax(torch.randn((B, N, V), generator=g), dim=-1).cuda()
+    target_feat = torch.randn((N, B, d), generator=g).cuda()
+    for _ in range(3):
+        fe.fe_draft_loss(h, feat, tok, plen, kd, vd, teacher, target_feat, k, page_table=table, n_pages=n_pages,
+                         stream=stream)
+    v0.record(stream)
+    for _ in range(20):
+        fe.fe_draft_loss(h, feat, tok, plen, kd, vd, teacher, target_feat, k, page_table=table, n_pages=n_pages,
+                         stream=stream)
+    v1.record(stream)
+    v1.synchronize()
+    loss_us = 1000.0 * v0.elapsed_time(v1) / 20
+    st = fe.fe_last_device_status(h)
+    if st != fe.FE_OK:
+        raise SystemExit(f"device status after the loss forward: {fe.fe_status_str(st)}")
+
     # ---- roofline of the dominant kernel (and of the whole step, for context) ----------------
     peak, peak_kind = peaks()
     plist = I["prefix_len"].tolist()
@@ -365,6 +384,9 @@ def main():
             "kernels": kernels,
             "verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
                               "note": "fe_verify_greedy after the step (positions + greedy acceptance walk)"},
+            "draft_loss": {"us_per_call": loss_us,
+                           "note": "fe_draft_loss: the draft with logits [B,N,V] and hidden states written out, "
+                                   "then CE + Smooth L1 (Sec. 2.3); outside the timed step"},
             "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": launches * args.steps, "launches_per_step": launches,

@@ -183,6 +183,21 @@ FE_API const char *fe_last_error_detail(void);
  * a batch of B, so a caller can count launches. Returns -1 for a bad handle. */
 FE_API int32_t fe_launch_count(const fe_handle *h, int32_t B, int32_t with_tree);
 
+/* Forward of the multi-level training objective (Sec. 2.3, Eq. 3-6) for one draft: runs
+ * fe_draft_forward (args->dbg_logits [B, N, V] and args->dbg_hidden [N, B, d] are required:
+ * the loss reads the full-vocabulary logits and hidden states from them), then, for each
+ * sequence b and depth i = 1..N:
+ *   ce [B, N]        = -sum_k p_k log q_k with q = softmax(logits) at temperature 1 (Eq. 4),
+ *                      p = teacher_p [B, N, V] (the target's teacher distribution, float32)
+ *   feat_loss [B, N] = sum_j SmoothL1(h_ij - f_ij), f = target_feat [N, B, d] float32 (Eq. 5-6)
+ *   total [B]        = sum_i decay^(N - i) (alpha ce + beta feat_loss) (Eq. 3; the paper uses
+ *                      decay 0.9, alpha 0.1, beta 1).
+ * Device pointers, asynchronous on `stream`. Errors as fe_draft_forward, plus
+ * FE_ERR_INVALID_ARG for a missing buffer or a NaN coefficient. Forward only (no gradients). */
+FE_API fe_status fe_draft_loss(fe_handle *h, const fe_forward_args *args, const float *teacher_p,
+                               const float *target_feat, float alpha, float beta, float decay, float *ce,
+                               float *feat_loss, float *total, void *stream);
+
 /* Verification side of a cycle (Sec. 2.4, "Parallel Verification"), after the target model
  * has scored the draft tree under tree attention. For each sequence b of a tree built by
  * fe_build_tree (top_k candidates per level, T = 1 + N top_k nodes):

@@ -27,7 +27,7 @@ _lock = threading.Lock()
 _cache: dict = {}
 
 # Number of planted-mistake variants compiled by build(mutant=n) (n = 1..N_MUTANTS).
-N_MUTANTS = 30
+N_MUTANTS = 33
 _UNUSED_MUTANTS = {25}  # ids with no planted mistake
 
 
@@ -99,6 +99,11 @@ class Oracle:
         L.or_lm_head.argtypes = [ctypes.POINTER(Config), _P, _P, _D, _D]
         L.or_softmax.argtypes = [_D, ctypes.c_int64, ctypes.c_double, _D, _D]
         L.or_topk.argtypes = [_D, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]
+        L.or_smooth_l1.argtypes = [ctypes.c_double]
+        L.or_smooth_l1.restype = ctypes.c_double
+        L.or_loss.argtypes = [ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, _D, _D, _D, _D, ctypes.c_double,
+                              ctypes.c_double, ctypes.c_double, _D, _D]
+        L.or_loss.restype = ctypes.c_double
         _I = ctypes.POINTER(ctypes.c_int32)
         L.or_accept_greedy.argtypes = [ctypes.c_int32, _I, _I, _I, _I, ctypes.c_int32, ctypes.c_int32, _I, _I, _I]
         L.or_accept_greedy.restype = ctypes.c_int32
@@ -198,6 +203,22 @@ class Oracle:
                                     int(max_path), pos.ctypes.data_as(i32), path.ctypes.data_as(i32),
                                     ctypes.byref(bonus))
         return pos, path, int(n), int(bonus.value)
+
+    def smooth_l1(self, x: float) -> float:
+        return float(self.L.or_smooth_l1(float(x)))
+
+    def loss(self, logits, teacher, hidden, feat, alpha: float = 0.1, beta: float = 1.0, decay: float = 0.9):
+        """Training objective of Sec. 2.3 for one sequence: logits, teacher [N, V]; hidden,
+        feat [N, d]. Returns (total, ce [N], feat_loss [N])."""
+        logits, teacher, hidden, feat = (np.ascontiguousarray(a, dtype=np.float64) for a in
+                                         (logits, teacher, hidden, feat))
+        N, V = logits.shape
+        d = hidden.shape[1]
+        ce = np.zeros(N)
+        fl = np.zeros(N)
+        tot = self.L.or_loss(N, V, d, _dp(logits), _dp(teacher), _dp(hidden), _dp(feat), float(alpha), float(beta),
+                             float(decay), _dp(ce), _dp(fl))
+        return float(tot), ce, fl
 
     def max_threads(self) -> int:
         return int(self.L.or_max_threads())

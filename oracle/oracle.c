@@ -326,6 +326,46 @@ void or_tree(int32_t N, int32_t k, int32_t root, const int32_t *topk, int32_t *t
     }
 }
 
+/* Smooth L1 of Eq. 6: 0.5 x^2 for |x| < 1, |x| - 0.5 otherwise. */
+double or_smooth_l1(double x)
+{
+    const double a = fabs(x);
+    return a < 1.0 ? (MUT(32) ? x * x : 0.5 * x * x) : a - 0.5;
+}
+
+/* The multi-level training objective of Sec. 2.3 (Eq. 3-6), forward only, for one sequence:
+ *   logits [N][V]: the drafter's logits of depth i, q_i = softmax(logits_i) (temperature 1);
+ *   teacher [N][V]: the target model's teacher distribution p_{t+i};
+ *   hidden, feat [N][d]: the drafter's h_i and the target features f_i.
+ * ce[i] = -sum_k p_k log q_k (Eq. 4); fl[i] = sum_j SmoothL1(h_ij - f_ij) (Eq. 5);
+ * returns L_total = sum_i w_i (alpha ce[i] + beta fl[i]) with w_i = decay^(N - i) for the
+ * 1-based depth i (Eq. 3; the paper uses decay 0.9, alpha 0.1, beta 1). */
+double or_loss(int32_t N, int64_t V, int64_t d, const double *logits, const double *teacher,
+               const double *hidden, const double *feat, double alpha, double beta, double decay,
+               double *ce, double *fl)
+{
+    double *q = (double *)malloc(sizeof(double) * (size_t)V);
+    double total = 0.0;
+    for (int32_t i = 0; i < N; ++i) {
+        double lse;
+        or_softmax(logits + (int64_t)i * V, V, 1.0, q, &lse);
+        double c = 0.0;
+        for (int64_t k = 0; k < V; ++k) {
+            const double pk = teacher[(int64_t)i * V + k];
+            c -= MUT(33) ? q[k] * log(pk) : pk * log(q[k]);
+        }
+        double f = 0.0;
+        for (int64_t j = 0; j < d; ++j)
+            f += or_smooth_l1(hidden[(int64_t)i * d + j] - feat[(int64_t)i * d + j]);
+        ce[i] = c;
+        fl[i] = f;
+        const double w = pow(decay, (double)(MUT(31) ? i : N - 1 - i));
+        total += w * (alpha * c + beta * f);
+    }
+    free(q);
+    return total;
+}
+
 /* Verification side of one cycle (Sec. 2.4, "Parallel Verification"), for one sequence's
  * draft tree of T nodes (or_tree's tok, parent, depth):
  *   pos[a] = P + depth[a]: the sequence position of node a under tree attention (the root,

@@ -81,6 +81,9 @@ _lib.fe_lm_head_topk_noalloc.argtypes = [_vp, _vp, _i32, _i32, ctypes.c_float, _
 _lib.fe_lm_head_topk_noalloc.restype = ctypes.c_int
 _lib.fe_profile_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _i32, _vp, _vp, ctypes.POINTER(_i32)]
 _lib.fe_profile_forward.restype = ctypes.c_int
+_lib.fe_draft_loss.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, ctypes.c_float, ctypes.c_float,
+                               ctypes.c_float, _vp, _vp, _vp, _vp]
+_lib.fe_draft_loss.restype = ctypes.c_int
 _lib.fe_verify_greedy.argtypes = [_vp, _i32, _i32, _vp, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp]
 _lib.fe_verify_greedy.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
@@ -213,6 +216,30 @@ def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
     _check(_lib.fe_profile_forward(h.ptr, ctypes.byref(a), _stream(stream), cap, ctypes.cast(kinds, _vp),
                                    ctypes.cast(usec, _vp), ctypes.byref(n)), "fe_profile_forward")
     return [(FE_KERNEL_NAMES.get(kinds[j], str(kinds[j])), float(usec[j])) for j in range(n.value)]
+
+
+def fe_draft_loss(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, teacher_p, target_feat, top_k: int,
+                  alpha: float = 0.1, beta: float = 1.0, decay: float = 0.9, page_table=None, n_pages: int = 0,
+                  stream=None) -> dict:
+    """Forward of the training objective (include/fe_draft.h): teacher_p [B, N, V], target_feat
+    [N, B, d] (float32, device). Returns the draft's outputs plus logits, hidden, ce, feat_loss
+    and total."""
+    B = int(next_tok.shape[0])
+    N, d, V = h.cfg["n_layers"], h.cfg["d"], h.cfg["vocab"]
+    dev = feat.device
+    out = alloc_outputs(h, B, top_k, dev)
+    out.update(logits=torch.empty((B, N, V), device=dev), hidden=torch.empty((N, B, d), device=dev),
+               ce=torch.empty((B, N), device=dev), feat_loss=torch.empty((B, N), device=dev),
+               total=torch.empty(B, device=dev))
+    kc = (_vp * N)(*[_p(t) for t in k_cache])
+    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, 1.0, _p(feat), _p(next_tok), _p(prefix_len), kc, vc, _p(page_table),
+                        int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]), _p(out["topk_prob"]),
+                        _p(out["lse"]), _p(out["logits"]), _p(out["hidden"]))
+    _check(_lib.fe_draft_loss(h.ptr, ctypes.byref(a), _p(teacher_p), _p(target_feat), float(alpha), float(beta),
+                              float(decay), _p(out["ce"]), _p(out["feat_loss"]), _p(out["total"]), _stream(stream)),
+           "fe_draft_loss")
+    return out
 
 
 def alloc_tree(h: Handle, B: int, top_k: int, device="cuda") -> dict:

@@ -209,6 +209,10 @@ inline int attention_launches() { return 1; }
 cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,
                         int* depth, uint8_t* mask, int* status, cudaStream_t st);
 cudaError_t launch_timeout_probe(int64_t timeout_ns, int* status, cudaStream_t st);
+// training-objective forward (fe_loss.cu): ce, fl [B, N]; total [B]
+cudaError_t launch_loss(int N, int B, int V, int d, const float* logits, const float* teacher, const float* hidden,
+                        const float* feat, float alpha, float beta, float decay, float* ce, float* fl, float* total,
+                        cudaStream_t st);
 cudaError_t launch_verify(int B, int T, int max_path, const int* prefix_len, const int* tok, const int* parent,
                           const int* depth, const int* target_next, int* pos, int* path, int* n_accept, int* bonus,
                           cudaStream_t st);

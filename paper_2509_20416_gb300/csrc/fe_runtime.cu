@@ -693,6 +693,20 @@ fe_status fe_build_tree(fe_handle* h, int32_t B, int32_t top_k, const int32_t* n
     return FE_OK;
 }
 
+fe_status fe_draft_loss(fe_handle* h, const fe_forward_args* a, const float* teacher_p, const float* target_feat,
+                        float alpha, float beta, float decay, float* ce, float* feat_loss, float* total, void* stream) {
+    if (!forward_args_ok(h, a) || !a->dbg_logits || !a->dbg_hidden || !teacher_p || !target_feat || !ce ||
+        !feat_loss || !total)
+        return FE_ERR_INVALID_ARG;
+    if (!(alpha == alpha) || !(beta == beta) || !(decay == decay)) return FE_ERR_INVALID_ARG;
+    const fe_status rc = fe_draft_forward(h, a, stream);
+    if (rc != FE_OK) return rc;
+    const fe_config& c = h->cfg;
+    FE_TRY(launch_loss(c.n_layers, a->B, c.vocab, c.d, a->dbg_logits, teacher_p, a->dbg_hidden, target_feat, alpha,
+                       beta, decay, ce, feat_loss, total, (cudaStream_t)stream));
+    return FE_OK;
+}
+
 fe_status fe_verify_greedy(fe_handle* h, int32_t B, int32_t top_k, const int32_t* prefix_len, const fe_tree* tree,
                            const int32_t* target_next, int32_t* pos_ids, int32_t* path, int32_t* n_accept,
                            int32_t* bonus, void* stream) {

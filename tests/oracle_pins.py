@@ -396,6 +396,47 @@ def pin_accept_greedy(orc):
         assert path[:n].tolist() == chain[::-1] and (path[n:] == -1).all()
 
 
+def pin_loss(orc):
+    """The training objective of Sec. 2.3 (Eq. 3-6): Smooth L1 closed forms, a two-layer,
+    three-token example worked by hand, and the reductions of the cross-entropy to a library
+    log-sum-exp (one-hot teacher) and to the entropy (teacher = drafter)."""
+    # Eq. 6
+    for x, want in ((0.0, 0.0), (0.5, 0.125), (-0.5, 0.125), (2.0, 1.5), (-3.0, 2.5), (1.0, 0.5), (-1.0, 0.5)):
+        assert abs(orc.smooth_l1(x) - want) < 1e-15, x
+    assert abs(orc.smooth_l1(1 - 1e-9) - orc.smooth_l1(1 + 1e-9)) < 1e-8  # continuous at |x| = 1
+    # worked by hand: layer 1 uniform q over 3 tokens, one-hot p -> log 3; h - f = (0.5, 2) ->
+    # 0.125 + 1.5. Layer 2 logits (0, ln 3, 0) -> q = (1/5, 3/5, 1/5), p = (0, 1/2, 1/2) ->
+    # -(ln(3/5) + ln(1/5)) / 2 = ln(25/3) / 2; h - f = (-3, 0.75) -> 2.5 + 0.28125.
+    # w = (0.9, 1) for N = 2 (w_i = 0.9^(N - i)), alpha 0.1, beta 1.
+    logits = np.array([[0.0, 0.0, 0.0], [0.0, math.log(3.0), 0.0]])
+    teacher = np.array([[1.0, 0.0, 0.0], [0.0, 0.5, 0.5]])
+    hidden = np.array([[0.5, 2.0], [-3.0, 1.0]])
+    feat = np.array([[0.0, 0.0], [0.0, 0.25]])
+    ce_want = [math.log(3.0), 0.5 * math.log(25.0 / 3.0)]
+    fl_want = [1.625, 2.78125]
+    tot_want = 0.9 * (0.1 * ce_want[0] + fl_want[0]) + 1.0 * (0.1 * ce_want[1] + fl_want[1])
+    tot, ce, fl = orc.loss(logits, teacher, hidden, feat)
+    assert np.allclose(ce, ce_want, rtol=1e-14, atol=1e-14) and np.allclose(fl, fl_want, rtol=0, atol=1e-15)
+    assert abs(tot - tot_want) < 1e-13
+    # reductions to library routines, random data
+    rng = np.random.default_rng(3)
+    N, V, d = 4, 50, 16
+    lg = rng.normal(0, 2, (N, V))
+    lse = np.log(np.exp(lg - lg.max(1, keepdims=True)).sum(1)) + lg.max(1)
+    y = rng.integers(0, V, N)
+    onehot = np.zeros((N, V))
+    onehot[np.arange(N), y] = 1.0
+    z = np.zeros((N, d))
+    tot, ce, fl = orc.loss(lg, onehot, z, z, alpha=1.0, beta=1.0, decay=1.0)
+    assert np.allclose(ce, lse - lg[np.arange(N), y], rtol=1e-12) and abs(tot - ce.sum()) < 1e-10
+    q = torch.softmax(torch.tensor(lg), dim=1).numpy()
+    tot, ce, fl = orc.loss(lg, q, z, z)
+    assert np.allclose(ce, -(q * np.log(q)).sum(1), rtol=1e-12)
+    # the weights follow the depth: only the last layer carries weight 1
+    tot, ce, fl = orc.loss(lg, onehot, z, z, alpha=1.0, beta=0.0, decay=0.5)
+    assert abs(tot - sum(0.5 ** (N - 1 - i) * ce[i] for i in range(N))) < 1e-12
+
+
 def pin_zero_blocks(orc):
     """W_o = W_down = 0: every layer passes x0 through, so all N distributions coincide."""
     cfg = mini_cfg(n_layers=3, B=1)
@@ -419,6 +460,6 @@ def pin_zero_blocks(orc):
         assert list(tok[1 + i * k: 1 + (i + 1) * k]) == list(tok[1:1 + k])
 
 
-ALL_PINS = [pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
+ALL_PINS = [pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
             pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]
