@@ -55,8 +55,8 @@ TRAFFIC = {
     #     -k regex:linear_kernel -s 18 -c 6 on `bench.py --set n_layers=1` (one draft's six
     # linear launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down); the five-layer draft
     # repeats the four per-layer launches five times with the same shapes.
-    "vic13b": {"bytes_per_draft": 160491008 + 105316864 + 5 * (157492480 + 52532480 + 283694080 + 141830656),
-               "src": "42b9bf7bf13086c0"},
+    "vic13b": {"bytes_per_draft": 160379136 + 105180416 + 5 * (157504512 + 52528128 + 283563520 + 141821440),
+               "src": "3288142b22327a17"},
 }
 KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
 
