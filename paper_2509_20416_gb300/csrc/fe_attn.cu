@@ -21,6 +21,8 @@
 // the usual max-shifted weights and writes o. The item holding key P_b also rotates the
 // new key and writes the row's key and value into cache slot P_b (keys are cached after
 // RoPE); the own row is used from shared memory, unrounded.
+#include <cstdlib>
+
 #include "fe_kernels.h"
 #include "fe_common.cuh"
 #include "fe_stream.cuh"
@@ -449,13 +451,506 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
-// Keys per work item: aim at ~4 CTAs per SM over all (sequence, KV head) pairs, in whole
-// multiples of one chunk per warp (128 keys), so that every warp of a CTA has work and the
-// last split's combine has few partials to read.
+// ---- tensor-core attention (bf16 caches, hd = 128, G >= 2 query heads per KV head) -----------
+// The same work items, chunk ownership, own-row append and split combine as attn_kernel;
+// the per-chunk arithmetic runs on mma.sync (m16n8k16, bf16 operands, float32 accumulate)
+// with the keys and the head dimensions as the long matrix sides:
+//   S^T (32 keys x 8 heads) = K (32 x 128) . Q^T            2 key tiles x 8 k-steps
+//   O^T (128 dims x 8 heads) += V^T (128 x 32) . P^T          8 dim tiles x 2 k-steps
+// so a KV head's G <= 8 query heads fill the 8-wide side. Q and P enter as bf16 hi + lo
+// pairs (two products each), which keeps scores and outputs at float32-level accuracy; K
+// and V are bf16 in the cache already.
+//   - Rows arrive by cp.async (16 bytes per lane, two rows per warp instruction, each lane
+//     with its own address), so every row can go to its own place: 16-byte chunk c of row
+//     r lands at chunk c ^ (r % 8), which puts the eight rows an ldmatrix phase reads into
+//     eight different bank groups. Rows without a key are zero-filled by the copy itself.
+//   - K and V of a chunk are separate copy groups: the next chunk's K rows are requested as
+//     soon as S is formed and its V rows as soon as P.V is done, so each copy overlaps the
+//     other half of the chunk's arithmetic.
+//   - P^T changes fragment layout by shuffles within the warp.
+//   - Softmax runs in base 2 (log2 e is folded into the query scale).
+//   - The row's own key and value (position P, float32) enter as the first key of warp
+//     0's online softmax.
+constexpr uint32_t kTcHalfBytes = kChunkKeys * 256;  // the K (or V) rows of one chunk
+
+// x0 -> bits 0..15, x1 -> bits 16..31, rounded to nearest even
+__device__ __forceinline__ uint32_t bf16x2_rn(float x0, float x1) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(x1), "f"(x0));
+    return r;
+}
+
+// (x0, x1) as bf16x2 hi + lo words: x = hi + lo to about 16 significant bits
+__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    hi = bf16x2_rn(x0, x1);
+    lo = bf16x2_rn(x0 - __uint_as_float(hi << 16), x1 - __uint_as_float(hi & 0xFFFF0000u));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+
+// d += A B for one m16n8k16 tile (A row-major 16 x 16, B column-major 16 x 8)
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// 16 bytes global -> shared, bypassing L1; src_bytes = 0 writes 16 zero bytes instead
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <int G>
+__global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnArgs a) {
+    using CT = bf16_t;
+    constexpr int HD = 128;
+    constexpr int HALF = HD / 2;
+    constexpr uint32_t CB = kTcHalfBytes;
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ __align__(16) float qs[G][HD];
+    __shared__ __align__(16) float kn[HD];
+    __shared__ __align__(16) float vn[HD];
+    __shared__ float wm[kAttnWarps][G], wl[kAttnWarps][G];
+    __shared__ float s_own[G];  // the own key's score per head (base 2)
+    __shared__ int s_last;
+
+    const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int P = a.prefix_len[b];
+    const int ldq = (a.H + 2 * a.Hkv) * HD;
+
+    float* out = a.out + (size_t)b * a.H * HD + (size_t)g * G * HD;
+    const bool valid = P >= 0 && P + 1 <= a.max_seq;
+    if (!valid) {
+        griddep_launch_dependents();
+        griddep_wait();
+        if (s == 0) {
+            if (g == 0 && t == 0) atomicOr(a.status, ST_CAPACITY);
+            for (int i = t; i < G * HD; i += blockDim.x) out[i] = 0.f;
+        }
+        return;
+    }
+    const int t0 = s * a.split;
+    if (t0 > P) {  // beyond this sequence's keys: not an active split
+        griddep_launch_dependents();
+        return;
+    }
+    const int t1 = min(t0 + a.split, P + 1);
+    const int n_act = min(a.n_split, P / a.split + 1);
+    const int tc = min(t1, P);  // cached keys [t0, tc); key P, when t1 > P, is the row's own
+    const int nchunks = tc > t0 ? (tc - t0 + kChunkKeys - 1) / kChunkKeys : 0;
+
+    unsigned char* kc = dsm + (size_t)warp * 2 * CB;  // this warp's 32 K rows, then its 32 V rows
+    unsigned char* vc = kc + CB;
+    // Paged caches: this item's page ids, read once into shared memory after the K/V rows
+    // (-1 marks an invalid id)
+    int* spg = reinterpret_cast<int*>(dsm + (size_t)kAttnWarps * 2 * CB);
+    const int pg0 = a.page_table ? t0 / a.page_size : 0;
+    if (a.page_table) {
+        const int npg = tc > t0 ? (tc - 1) / a.page_size - pg0 + 1 : 0;
+        for (int i = t; i < npg; i += blockDim.x) {
+            const int pg = a.page_table[(size_t)b * a.max_pages + pg0 + i];
+            spg[i] = (pg < 0 || pg >= a.n_pages) ? -1 : pg;
+        }
+    }
+    __syncthreads();  // page ids staged
+
+    // Chunk j of this warp covers keys [c0, c0 + 32), c0 = t0 + (warp + 4 j) * 32; lane r
+    // looks up row c0 + r. Returns 1 and the row's index in the cache (in rows of hd
+    // elements) when it holds a cached key, 0 past the item's keys, -1 on an invalid page id.
+    auto plan = [&](int j, uint32_t& ri) -> int {
+        const int pos = t0 + (warp + kAttnWarps * j) * kChunkKeys + lane;
+        if (pos >= tc) return 0;
+        if (a.page_table) {
+            const int pg = spg[pos / a.page_size - pg0];
+            if (pg < 0) return -1;
+            ri = (uint32_t)(((size_t)pg * a.Hkv + g) * a.page_size + pos % a.page_size);
+        } else {
+            ri = (uint32_t)(((size_t)b * a.Hkv + g) * a.max_seq + pos);
+        }
+        return 1;
+    };
+    // One half (K or V) of a chunk as one copy group: warp instruction i moves rows 2 i and
+    // 2 i + 1, lane l chunk l % 16 of row 2 i + l / 16 (row indices come from their lanes).
+    auto copy_half = [&](unsigned char* dst, const void* cache, uint32_t ri, uint32_t live) {
+        const int h = lane >> 4, c = lane & 15;
+        const uint32_t d0 = smem_u32(dst);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int r = 2 * i + h;
+            const uint32_t rr = __shfl_sync(0xffffffffu, ri, r);
+            const bool ok = (live >> r) & 1u;
+            const CT* src = (const CT*)cache + (ok ? (size_t)rr * HD + c * 8 : 0);
+            cp_async16(d0 + r * 256 + ((c ^ (r & 7)) << 4), src, ok ? 16u : 0u);
+        }
+        cp_async_commit();
+    };
+    const int my_chunks = warp < nchunks ? (nchunks - warp + kAttnWarps - 1) / kAttnWarps : 0;
+    uint32_t ri = 0, live = 0, bad = 0;  // lane's row index; the chunk's rows holding a key / on invalid pages
+    // cached prefix rows are not written by the earlier kernels of this draft: copy the
+    // first chunk before waiting for the QKV projection
+    if (my_chunks > 0) {
+        const int code = plan(0, ri);
+        live = __ballot_sync(0xffffffffu, code > 0);
+        bad = __ballot_sync(0xffffffffu, code < 0);
+        copy_half(kc, a.kc, ri, live);
+        copy_half(vc, a.vc, ri, live);
+    }
+    griddep_launch_dependents();
+    griddep_wait();
+
+    // queries of the group, rotated at position P and pre-scaled by log2(e) / sqrt(hd)
+    const float* cs = a.rope_cs + (size_t)P * HALF * 2;
+    const float scale = 1.4426950408889634f / sqrtf((float)HD);
+    for (int idx = t; idx < G * HALF; idx += blockDim.x) {
+        const int j = idx / HALF, i = idx % HALF;
+        const float* q = a.qkv + (size_t)b * ldq + (size_t)(g * G + j) * HD;
+        const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+        qs[j][i] = (x1 * c - x2 * sn) * scale;
+        qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+    }
+    const bool own = t1 == P + 1;  // this item holds the row's own key
+    if (own) {  // rotate the new key and append k, v at slot P
+        const float* kq = a.qkv + (size_t)b * ldq + (size_t)a.H * HD + (size_t)g * HD;
+        const float* vq = kq + (size_t)a.Hkv * HD;
+        CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
+        CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
+        if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
+        for (int i = t; i < HALF; i += blockDim.x) {
+            const float x1 = kq[i], x2 = kq[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            const float r1 = x1 * c - x2 * sn, r2 = x2 * c + x1 * sn;
+            kn[i] = r1;
+            kn[i + HALF] = r2;
+            if (krow) {
+                Storage<CT>::store(krow, i, r1);
+                Storage<CT>::store(krow, i + HALF, r2);
+            }
+        }
+        for (int i = t; i < HD; i += blockDim.x) {
+            vn[i] = vq[i];
+            if (vrow) Storage<CT>::store(vrow, i, vq[i]);
+        }
+    }
+    __syncthreads();
+    if (own)  // the own key's score per head: warp w takes heads w, w + 4
+        for (int h = warp; h < G; h += kAttnWarps) {
+            float v = 0.f;
+#pragma unroll
+            for (int i = lane; i < HD; i += 32) v = fmaf(qs[h][i], kn[i], v);
+            v = warp_sum(v);
+            if (lane == 0) s_own[h] = v;
+        }
+    __syncthreads();
+
+    // Fragment ownership: gid = lane / 4, tig = lane % 4. Thread (gid, tig) holds Q^T's
+    // B fragments for head gid (zero for gid >= G) and accumulates heads 2 tig and 2 tig + 1.
+    const int gid = lane >> 2, tig = lane & 3;
+    uint32_t qh[8][2], ql[8][2];  // k-step ks: dims 16 ks + 2 tig (+1) and 16 ks + 8 + 2 tig (+1)
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+            const int c = ks * 16 + hf * 8 + tig * 2;
+            split_pack(gid < G ? qs[gid][c] : 0.f, gid < G ? qs[gid][c + 1] : 0.f, qh[ks][hf], ql[ks][hf]);
+        }
+    // Running state of heads 2 tig + e (base 2). Warp 0 of the item holding key P starts
+    // from the row's own key and value (float32, unrounded) as its first key.
+    const bool first = own && warp == 0;
+    float m[2], l[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+        m[e] = first ? s_own[min(2 * tig + e, G - 1)] : -INFINITY;
+        l[e] = first ? 1.f : 0.f;
+    }
+    float o[8][4];  // dim tile mt: (16 mt + gid, heads 2 tig, 2 tig + 1), (16 mt + gid + 8, same heads)
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+        const float v0 = first ? vn[16 * mt + gid] : 0.f, v1 = first ? vn[16 * mt + gid + 8] : 0.f;
+        o[mt][0] = o[mt][1] = v0;
+        o[mt][2] = o[mt][3] = v1;
+    }
+
+    // ldmatrix addresses (chunk c of row r sits at chunk c ^ (r % 8), and r % 8 = lane % 8
+    // for every row a lane addresses): K as the A operand, 16 keys x 16 dims per x4, lane l
+    // naming row (l % 8) + 8 ((l / 8) % 2) at dims 8 (l / 16) ..; V^T through .trans, lane l
+    // naming key 8 (l / 16) + l % 8 at dims 8 ((l / 8) % 2) ..
+    const int sw = lane & 7;
+    const uint32_t rowa = smem_u32(kc) + (uint32_t)(sw + 8 * ((lane >> 3) & 1)) * 256;
+    const uint32_t rowv = smem_u32(vc) + (uint32_t)(8 * (lane >> 4) + sw) * 256;
+    const int ca = lane >> 4, cv = (lane >> 3) & 1;
+    // P^T's B fragments gather keys 2 tig and 2 tig + 1 of every 8 from lanes 4 (2 tig) +
+    // gid / 2 and 4 (2 tig + 1) + gid / 2, value e = gid % 2 of theirs
+    const int src0 = 4 * (2 * tig) + (gid >> 1), src1 = src0 + 4;
+    const bool odd = gid & 1;
+    for (int j = 0; j < my_chunks; ++j) {
+        if (bad && lane == 0) atomicOr(a.status, ST_DEVICE);
+        const bool more = j + 1 < my_chunks;
+        uint32_t nri = 0, nlive = 0, nbad = 0;
+        if (more) {
+            const int code = plan(j + 1, nri);
+            nlive = __ballot_sync(0xffffffffu, code > 0);
+            nbad = __ballot_sync(0xffffffffu, code < 0);
+        }
+        // this chunk's K rows (groups in flight: K(j), V(j))
+        cp_async_wait<1>();
+        __syncwarp();
+        // S^T = K Q^T; four independent accumulators (key tile x hi/lo)
+        float sc[2][4];
+        {
+            float acc[4][4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+                const uint32_t col = (uint32_t)((2 * ks + ca) ^ sw) << 4;
+                uint32_t a0[4], a1[4];
+                ldsm_x4(rowa + col, a0);
+                ldsm_x4(rowa + 16 * 256 + col, a1);
+                mma_16816(acc[0], a0, qh[ks][0], qh[ks][1]);
+                mma_16816(acc[1], a1, qh[ks][0], qh[ks][1]);
+                mma_16816(acc[2], a0, ql[ks][0], ql[ks][1]);
+                mma_16816(acc[3], a1, ql[ks][0], ql[ks][1]);
+            }
+#pragma unroll
+            for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) sc[mt][i] = acc[mt][i] + acc[2 + mt][i];
+        }
+        __syncwarp();  // every lane's K reads are done: the K rows may be refilled
+        if (more) copy_half(kc, a.kc, nri, nlive);
+        // online softmax: head 2 tig + e sees keys 16 mt + 8 hi + gid here and in the 7
+        // other lanes of its column (lanes tig, tig + 4, ...)
+        float p[2][4];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            float mx = -INFINITY;
+#pragma unroll
+            for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                for (int hi = 0; hi < 2; ++hi)
+                    if ((live >> (16 * mt + 8 * hi + gid)) & 1u) mx = fmaxf(mx, sc[mt][2 * hi + e]);
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+            const float mn = fmaxf(m[e], mx);
+            const float corr = m[e] == -INFINITY ? 0.f : exp2f(m[e] - mn);
+            float rs = 0.f;
+#pragma unroll
+            for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                for (int hi = 0; hi < 2; ++hi) {
+                    const float pv =
+                        ((live >> (16 * mt + 8 * hi + gid)) & 1u) ? exp2f(sc[mt][2 * hi + e] - mn) : 0.f;
+                    p[mt][2 * hi + e] = pv;
+                    rs += pv;
+                }
+            rs += __shfl_xor_sync(0xffffffffu, rs, 4);
+            rs += __shfl_xor_sync(0xffffffffu, rs, 8);
+            rs += __shfl_xor_sync(0xffffffffu, rs, 16);
+            l[e] = l[e] * corr + rs;
+            m[e] = mn;
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                o[mt][e] *= corr;
+                o[mt][2 + e] *= corr;
+            }
+        }
+        // P^T's B fragments: word w[q][e] = key 8 q + gid of head 2 tig + e as bf16 (hi, lo);
+        // k-step kk, half hf takes keys 16 kk + 8 hf + 2 tig (+1) of head gid
+        uint32_t w[4][2];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t hi, lo;
+            split_pack(p[q >> 1][2 * (q & 1)], p[q >> 1][2 * (q & 1) + 1], hi, lo);
+            w[q][0] = __byte_perm(hi, lo, 0x5410);
+            w[q][1] = __byte_perm(hi, lo, 0x7632);
+        }
+        uint32_t pb[4][2];  // [q = 2 kk + hf][hi / lo]
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t x0 = __shfl_sync(0xffffffffu, w[q][0], src0), y0 = __shfl_sync(0xffffffffu, w[q][1], src0);
+            const uint32_t x1 = __shfl_sync(0xffffffffu, w[q][0], src1), y1 = __shfl_sync(0xffffffffu, w[q][1], src1);
+            const uint32_t v0 = odd ? y0 : x0, v1 = odd ? y1 : x1;
+            pb[q][0] = __byte_perm(v0, v1, 0x5410);
+            pb[q][1] = __byte_perm(v0, v1, 0x7632);
+        }
+        // this chunk's V rows (groups in flight: V(j), and K(j + 1) unless this is the last)
+        if (more) cp_async_wait<1>();
+        else cp_async_wait<0>();
+        __syncwarp();
+        // O^T += V^T P^T, four dim tiles at a time: each accumulator's two products are four
+        // MMAs apart
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk)
+#pragma unroll
+            for (int mg = 0; mg < 2; ++mg) {
+                uint32_t af[4][4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    ldsm_x4_trans(rowv + kk * 16 * 256 + ((uint32_t)((2 * (4 * mg + i) + cv) ^ sw) << 4), af[i]);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) mma_16816(o[4 * mg + i], af[i], pb[2 * kk][0], pb[2 * kk + 1][0]);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) mma_16816(o[4 * mg + i], af[i], pb[2 * kk][1], pb[2 * kk + 1][1]);
+            }
+        __syncwarp();  // every lane's V reads are done
+        if (more) copy_half(vc, a.vc, nri, nlive);
+        live = nlive;
+        bad = nbad;
+    }
+
+    // ---- merge the warps into this split's partial per head (every copy group has been
+    // waited for: the K/V rows are free and hold the warps' accumulators)
+    float (*wacc)[G][HD] = reinterpret_cast<float (*)[G][HD]>(dsm);
+    __syncthreads();
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+        const int h = 2 * tig + e;
+        if (h < G) {
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                wacc[warp][h][16 * mt + gid] = o[mt][e];
+                wacc[warp][h][16 * mt + gid + 8] = o[mt][2 + e];
+            }
+            if (gid == 0) {
+                wm[warp][h] = m[e];
+                wl[warp][h] = l[e];
+            }
+        }
+    }
+    __syncthreads();
+    for (int idx = t; idx < G * HD; idx += blockDim.x) {
+        const int hh = idx / HD, dd = idx % HD;
+        float M = wm[0][hh];
+        for (int w = 1; w < kAttnWarps; ++w) M = fmaxf(M, wm[w][hh]);
+        float v = 0.f, L = 0.f;
+        for (int w = 0; w < kAttnWarps; ++w) {
+            if (wm[w][hh] == -INFINITY) continue;
+            const float f = exp2f(wm[w][hh] - M);
+            v = fmaf(f, wacc[w][hh][dd], v);
+            L = fmaf(f, wl[w][hh], L);
+        }
+        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * (HD + 2);
+        pp[dd] = v;
+        if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
+    }
+    // ---- the last active split of (b, g) combines all splits
+    __threadfence();
+    __syncthreads();
+    if (t == 0) s_last = atomicAdd(&a.counters[b * a.Hkv + g], 1) == n_act - 1;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // Each split's (max, sum) per head goes to shared memory (the K/V slots are free now) in
+    // one round trip; each head's weights exp(M_q - M) are formed there; each output then
+    // sums its splits with eight loads in flight (a load-then-accumulate loop would wait a
+    // full L2 round trip per split).
+    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * (HD + 2);
+    float* wq = reinterpret_cast<float*>(dsm);  // [n_act][G] weights, then [n_act][G] sums
+    float* lq = wq + n_act * G;
+    __shared__ float hl[G];
+    if ((size_t)2 * n_act * G * sizeof(float) <= (size_t)kAttnWarps * 2 * CB) {
+        for (int idx = t; idx < n_act * G; idx += blockDim.x) {
+            const int q = idx / G, hh = idx % G;
+            const float* p = pb0 + ((size_t)hh * a.n_split + q) * (HD + 2) + HD;
+            wq[idx] = __ldcg(p);
+            lq[idx] = __ldcg(p + 1);
+        }
+        __syncthreads();
+        for (int hh = warp; hh < G; hh += kAttnWarps) {
+            float M = -INFINITY;
+            for (int q = lane; q < n_act; q += 32) M = fmaxf(M, wq[q * G + hh]);
+            M = warp_max(M);
+            float L = 0.f;
+            for (int q = lane; q < n_act; q += 32) {
+                const float mq = wq[q * G + hh];
+                const float f = mq == -INFINITY ? 0.f : exp2f(mq - M);
+                wq[q * G + hh] = f;
+                L = fmaf(f, lq[q * G + hh], L);
+            }
+            L = warp_sum(L);
+            if (lane == 0) hl[hh] = L;
+        }
+        __syncthreads();
+        // thread t owns outputs t, t + 128, ... (NO of them) and loads QB splits of each at once
+        constexpr int NO = (G * HD + kAttnWarps * 32 - 1) / (kAttnWarps * 32);
+        constexpr int QB = NO >= 32 ? 1 : 32 / NO;
+        float v[NO];
+#pragma unroll
+        for (int o = 0; o < NO; ++o) v[o] = 0.f;
+        for (int q0 = 0; q0 < n_act; q0 += QB) {
+            float x[NO][QB];
+#pragma unroll
+            for (int o = 0; o < NO; ++o) {
+                const int idx = t + o * kAttnWarps * 32, hh = idx / HD, dd = idx % HD;
+                const float* p = pb0 + (size_t)hh * a.n_split * (HD + 2) + dd;
+#pragma unroll
+                for (int u = 0; u < QB; ++u)
+                    x[o][u] = idx < G * HD && q0 + u < n_act ? __ldcg(p + (size_t)(q0 + u) * (HD + 2)) : 0.f;
+            }
+#pragma unroll
+            for (int o = 0; o < NO; ++o) {
+                const int idx = t + o * kAttnWarps * 32, hh = (idx / HD) % G;
+#pragma unroll
+                for (int u = 0; u < QB; ++u)
+                    if (q0 + u < n_act) v[o] = fmaf(wq[(q0 + u) * G + hh], x[o][u], v[o]);
+            }
+        }
+#pragma unroll
+        for (int o = 0; o < NO; ++o) {
+            const int idx = t + o * kAttnWarps * 32;
+            if (idx < G * HD) {
+                const int hh = idx / HD, dd = idx % HD;
+                out[(size_t)hh * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
+            }
+        }
+    } else {  // more splits than the slots hold: the same sums, one split at a time
+        for (int idx = t; idx < G * HD; idx += blockDim.x) {
+            const int hh = idx / HD, dd = idx % HD;
+            const float* pb = pb0 + (size_t)hh * a.n_split * (HD + 2);
+            float M = -INFINITY;
+            for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
+            float v = 0.f, L = 0.f;
+            for (int q = 0; q < n_act; ++q) {
+                const float* p = pb + (size_t)q * (HD + 2);
+                const float mq = __ldcg(p + HD);
+                if (mq == -INFINITY) continue;
+                const float f = exp2f(mq - M);
+                v = fmaf(f, __ldcg(p + dd), v);
+                L = fmaf(f, __ldcg(p + HD + 1), L);
+            }
+            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
+        }
+    }
+    if (t == 0) a.counters[b * a.Hkv + g] = 0;
+}
+
+// Keys per work item: aim at ~8 CTAs per SM over all (sequence, KV head) pairs, in whole
+// multiples of one chunk per warp (128 keys), so that every warp of a CTA has work. About
+// three CTAs are resident per SM, so ragged prefixes leave several waves of items that the
+// block scheduler balances; the last split's combine still has few partials to read.
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev) {
     constexpr int unit = kAttnWarps * kChunkKeys;
     const int items = B * Hkv;
-    int per = (4 * dev.num_sms + items - 1) / items;  // splits per (sequence, KV head)
+    int per = (8 * dev.num_sms + items - 1) / items;  // splits per (sequence, KV head)
     if (per < 1) per = 1;
     int split = (max_seq + per - 1) / per;
     split = ((split + unit - 1) / unit) * unit;
@@ -482,9 +977,24 @@ static cudaError_t prepare_g() {
                                 (int)attn_smem(HD, sizeof(CT), max_slots(HD, sizeof(CT))) + kAttnPageSmem);
 }
 
+// bf16, hd 128, G >= 2 runs on the tensor-core kernel unless FE_DRAFT_ATTN_TC=0 selects
+// the CUDA-core kernel (kept for comparison)
+static bool attn_tc_enabled() {
+    const char* e = getenv("FE_DRAFT_ATTN_TC");
+    return !(e && e[0] == '0');
+}
+
 template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
     const int S = attn_slots(a.split, HD, sizeof(CT));
+    if constexpr (sizeof(CT) == 2 && HD == 128 && G >= 2) {
+        if (attn_tc_enabled()) {
+            const size_t pg = attn_page_ints(a) * sizeof(int);
+            if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
+            return launch_k(attn_tc_kernel<G>, dim3(a.n_split, a.Hkv, a.B), dim3(kAttnWarps * 32),
+                            (size_t)kAttnWarps * 2 * kTcHalfBytes + pg, st, a.pdl, a);
+        }
+    }
     const size_t pg = attn_page_ints(a) * sizeof(int);
     if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
     dim3 grid(a.n_split, a.Hkv, a.B);
@@ -514,6 +1024,10 @@ static cudaError_t prepare_hd() {
 
 cudaError_t attention_prepare() {
     cudaError_t e;
+    for (auto k : {attn_tc_kernel<2>, attn_tc_kernel<4>, attn_tc_kernel<8>})
+        if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)(kAttnWarps * 2 * kTcHalfBytes) + kAttnPageSmem)) != cudaSuccess)
+            return e;
     if ((e = prepare_hd<float, 64>()) != cudaSuccess) return e;
     if ((e = prepare_hd<float, 128>()) != cudaSuccess) return e;
     if ((e = prepare_hd<bf16_t, 64>()) != cudaSuccess) return e;

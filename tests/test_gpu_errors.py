@@ -74,11 +74,14 @@ def test_capacity_and_token_range_reported(small):
     assert g["status"] == fe.FE_OK
 
 
-def test_bad_page_id_reported():
+@pytest.mark.parametrize("d,n_heads,n_kv_heads,head_dim", [(256, 4, 2, 64), (512, 4, 1, 128)])
+def test_bad_page_id_reported(d, n_heads, n_kv_heads, head_dim):
+    """An out-of-pool page id is reported, not dereferenced (hd 128 with G = 4 runs on the
+    tensor-core attention kernel, hd 64 on the CUDA-core one)."""
     import paper_2509_20416_gb300 as fe
-    cfg = wl.make_config(dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=512, vocab=1000, n_layers=1,
-                              dtype="bf16", B=2, prefix=0, top_k=4, rope_theta=1e4, seed=10, page_size=16),
-                         prefix_list=[40, 3])
+    cfg = wl.make_config(dict(d=d, n_heads=n_heads, n_kv_heads=n_kv_heads, head_dim=head_dim, ffn=512, vocab=1000,
+                              n_layers=1, dtype="bf16", B=2, prefix=0, top_k=4, rope_theta=1e4, seed=10,
+                              page_size=16), prefix_list=[40, 3])
     W = wl.make_weights(cfg)
     I = wl.make_inputs(cfg)
     ks, vs = wl.make_caches(cfg)

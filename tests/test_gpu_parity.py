@@ -96,6 +96,18 @@ SMALL = {
                                       n_layers=3, dtype="bf16", B=12, prefix=0, top_k=8, rope_theta=1e4,
                                       seed=14, page_size=0, parallel_layers=1),
                             prefix_list=[37, 0, 150, 1, 64, 5, 300, 2, 128, 129, 7, 90]),
+    # bf16, hd 128, G >= 2: the tensor-core attention kernel. Prefixes on both sides of
+    # the 32-key chunk and 128-key split boundaries, an empty prefix, several splits per
+    # sequence (combined by the last split), page sizes 16 and 8, and contiguous caches.
+    "tc_attn_g4_paged16": dict(name=dict(d=512, n_heads=4, n_kv_heads=1, head_dim=128, ffn=1376, vocab=3001,
+                                         n_layers=2, dtype="bf16", B=6, prefix=0, top_k=8, rope_theta=5e5,
+                                         seed=15, page_size=16), prefix_list=[0, 1, 31, 32, 129, 700]),
+    "tc_attn_g8_contig": dict(name=dict(d=1024, n_heads=8, n_kv_heads=1, head_dim=128, ffn=1024, vocab=3001,
+                                        n_layers=2, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
+                                        seed=16, page_size=0), prefix_list=[33, 0, 517]),
+    "tc_attn_g2_paged8": dict(name=dict(d=512, n_heads=4, n_kv_heads=2, head_dim=128, ffn=1376, vocab=3001,
+                                        n_layers=2, dtype="bf16", B=4, prefix=0, top_k=4, rope_theta=5e5,
+                                        seed=17, page_size=8), prefix_list=[7, 8, 9, 260]),
     # N * B = 160 rows: the wide tensor-core LM head with three 64-row transpose groups
     "wide_lmhead_r160": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=3001,
                                        n_layers=5, dtype="bf16", B=32, prefix=0, top_k=8, rope_theta=1e4,
@@ -131,6 +143,22 @@ def test_parity_tensor_core_linear_forced(orc, monkeypatch, B):
     g = H.run_gpu(cfg, W, I, ks, vs)
     assert g["status"] == 0, g["status"]
     for b in sorted({0, B - 1, B // 2}):
+        o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
+        H.compare(orc, cfg, g, o, b)
+        _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
+
+
+@pytest.mark.parametrize("case", ["tc_attn_g4_paged16", "tc_attn_g8_contig"])
+def test_parity_cuda_core_attention_forced(orc, monkeypatch, case):
+    """bf16 GQA attention at hd 128 on the CUDA-core kernel (FE_DRAFT_ATTN_TC=0), which the
+    tensor-core kernel replaces by default for these shapes."""
+    monkeypatch.setenv("FE_DRAFT_ATTN_TC", "0")
+    spec = dict(SMALL[case])
+    cfg = wl.make_config(spec.pop("name"), **spec)
+    W, I, ks, vs = _problem(cfg)
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert g["status"] == 0, g["status"]
+    for b in range(cfg["B"]):
         o = H.run_oracle(orc, cfg, W, I, ks, vs, b)
         H.compare(orc, cfg, g, o, b)
         _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
