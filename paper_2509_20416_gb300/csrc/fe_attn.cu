@@ -508,6 +508,13 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4],
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// 2^x by the hardware approximation (relative error about 2^-22; 2^-inf = 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // 16 bytes global -> shared, bypassing L1; src_bytes = 0 writes 16 zero bytes instead
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
@@ -576,13 +583,18 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     // Chunk j of this warp covers keys [c0, c0 + 32), c0 = t0 + (warp + 4 j) * 32; lane r
     // looks up row c0 + r. Returns 1 and the row's index in the cache (in rows of hd
     // elements) when it holds a cached key, 0 past the item's keys, -1 on an invalid page id.
+    // (power-of-two page sizes take shifts instead of divisions)
+    const int ps_shift = a.page_table && !(a.page_size & (a.page_size - 1)) ? __ffs(a.page_size) - 1 : -1;
     auto plan = [&](int j, uint32_t& ri) -> int {
         const int pos = t0 + (warp + kAttnWarps * j) * kChunkKeys + lane;
+        ri = 0;  // rows without a key copy from row 0 with zero source bytes
         if (pos >= tc) return 0;
         if (a.page_table) {
-            const int pg = spg[pos / a.page_size - pg0];
+            const int lp = ps_shift >= 0 ? pos >> ps_shift : pos / a.page_size;
+            const int in = ps_shift >= 0 ? pos & (a.page_size - 1) : pos % a.page_size;
+            const int pg = spg[lp - pg0];
             if (pg < 0) return -1;
-            ri = (uint32_t)(((size_t)pg * a.Hkv + g) * a.page_size + pos % a.page_size);
+            ri = (uint32_t)(((size_t)pg * a.Hkv + g) * a.page_size + in);
         } else {
             ri = (uint32_t)(((size_t)b * a.Hkv + g) * a.max_seq + pos);
         }
@@ -590,16 +602,19 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     };
     // One half (K or V) of a chunk as one copy group: warp instruction i moves rows 2 i and
     // 2 i + 1, lane l chunk l % 16 of row 2 i + l / 16 (row indices come from their lanes).
+    // The swizzle c ^ (r % 8) repeats every four instructions.
+    const int hrow = lane >> 4, cchunk = lane & 15;
+    uint32_t xo[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) xo[k] = (uint32_t)(hrow * 256 + ((cchunk ^ ((2 * k + hrow) & 7)) << 4));
     auto copy_half = [&](unsigned char* dst, const void* cache, uint32_t ri, uint32_t live) {
-        const int h = lane >> 4, c = lane & 15;
         const uint32_t d0 = smem_u32(dst);
+        const unsigned char* src0 = (const unsigned char*)cache + cchunk * 16;
+        const uint32_t lh = live >> hrow;
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-            const int r = 2 * i + h;
-            const uint32_t rr = __shfl_sync(0xffffffffu, ri, r);
-            const bool ok = (live >> r) & 1u;
-            const CT* src = (const CT*)cache + (ok ? (size_t)rr * HD + c * 8 : 0);
-            cp_async16(d0 + r * 256 + ((c ^ (r & 7)) << 4), src, ok ? 16u : 0u);
+            const uint32_t rr = __shfl_sync(0xffffffffu, ri, 2 * i + hrow);
+            cp_async16(d0 + 2 * i * 256 + xo[i & 3], src0 + (size_t)rr * 256, (lh >> (2 * i)) & 1u ? 16u : 0u);
         }
         cp_async_commit();
     };
@@ -678,7 +693,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
         m[e] = first ? s_own[min(2 * tig + e, G - 1)] : -INFINITY;
-        l[e] = first ? 1.f : 0.f;
+        l[e] = first && gid == 0 ? 1.f : 0.f;  // (one lane of the column holds the own key's share)
     }
     float o[8][4];  // dim tile mt: (16 mt + gid, heads 2 tig, 2 tig + 1), (16 mt + gid + 8, same heads)
 #pragma unroll
@@ -736,41 +751,43 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
         }
         __syncwarp();  // every lane's K reads are done: the K rows may be refilled
         if (more) copy_half(kc, a.kc, nri, nlive);
-        // online softmax: head 2 tig + e sees keys 16 mt + 8 hi + gid here and in the 7
-        // other lanes of its column (lanes tig, tig + 4, ...)
-        float p[2][4];
+        // online softmax: head 2 tig + e sees keys 8 q + gid (q = 2 mt + hi) here and in the
+        // 7 other lanes of its column (lanes tig, tig + 4, ...)
+        bool kl[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) kl[q] = (live >> (8 * q + gid)) & 1u;
+        float p[2][4], corr[2];
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             float mx = -INFINITY;
 #pragma unroll
-            for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-                for (int hi = 0; hi < 2; ++hi)
-                    if ((live >> (16 * mt + 8 * hi + gid)) & 1u) mx = fmaxf(mx, sc[mt][2 * hi + e]);
+            for (int q = 0; q < 4; ++q)
+                if (kl[q]) mx = fmaxf(mx, sc[q >> 1][2 * (q & 1) + e]);
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
             const float mn = fmaxf(m[e], mx);
-            const float corr = m[e] == -INFINITY ? 0.f : exp2f(m[e] - mn);
+            corr[e] = m[e] == mn ? 1.f : ex2_approx(m[e] - mn);  // (0 when m was -inf)
+            // l[e] holds this lane's share of the sum (its keys); the column's lanes add
+            // their shares once, after the last chunk
             float rs = 0.f;
 #pragma unroll
-            for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-                for (int hi = 0; hi < 2; ++hi) {
-                    const float pv =
-                        ((live >> (16 * mt + 8 * hi + gid)) & 1u) ? exp2f(sc[mt][2 * hi + e] - mn) : 0.f;
-                    p[mt][2 * hi + e] = pv;
-                    rs += pv;
-                }
-            rs += __shfl_xor_sync(0xffffffffu, rs, 4);
-            rs += __shfl_xor_sync(0xffffffffu, rs, 8);
-            rs += __shfl_xor_sync(0xffffffffu, rs, 16);
-            l[e] = l[e] * corr + rs;
+            for (int q = 0; q < 4; ++q) {
+                const float pv = kl[q] ? ex2_approx(sc[q >> 1][2 * (q & 1) + e] - mn) : 0.f;
+                p[q >> 1][2 * (q & 1) + e] = pv;
+                rs += pv;
+            }
+            l[e] = l[e] * corr[e] + rs;
             m[e] = mn;
+        }
+        // rescale the accumulators only when some head's maximum moved
+        if (__any_sync(0xffffffffu, corr[0] != 1.f || corr[1] != 1.f)) {
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) {
-                o[mt][e] *= corr;
-                o[mt][2 + e] *= corr;
+                o[mt][0] *= corr[0];
+                o[mt][1] *= corr[1];
+                o[mt][2] *= corr[0];
+                o[mt][3] *= corr[1];
             }
         }
         // P^T's B fragments: word w[q][e] = key 8 q + gid of head 2 tig + e as bf16 (hi, lo);
@@ -817,6 +834,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
         bad = nbad;
     }
 
+    // the sums of exp over each head's keys: add the shares of the column's 8 lanes
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+        l[e] += __shfl_xor_sync(0xffffffffu, l[e], 4);
+        l[e] += __shfl_xor_sync(0xffffffffu, l[e], 8);
+        l[e] += __shfl_xor_sync(0xffffffffu, l[e], 16);
+    }
     // ---- merge the warps into this split's partial per head (every copy group has been
     // waited for: the K/V rows are free and hold the warps' accumulators)
     float (*wacc)[G][HD] = reinterpret_cast<float (*)[G][HD]>(dsm);
