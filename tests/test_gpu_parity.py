@@ -108,6 +108,14 @@ SMALL = {
     "tc_attn_g2_paged8": dict(name=dict(d=512, n_heads=4, n_kv_heads=2, head_dim=128, ffn=1376, vocab=3001,
                                         n_layers=2, dtype="bf16", B=4, prefix=0, top_k=4, rope_theta=5e5,
                                         seed=17, page_size=8), prefix_list=[7, 8, 9, 260]),
+    # page sizes 64 (a chunk inside one page) and 24 (chunks straddling pages, division
+    # rather than shifts for the page lookup)
+    "tc_attn_g8_paged64": dict(name=dict(d=1024, n_heads=8, n_kv_heads=1, head_dim=128, ffn=1024, vocab=3001,
+                                         n_layers=2, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
+                                         seed=18, page_size=64), prefix_list=[63, 64, 300]),
+    "tc_attn_g4_paged24": dict(name=dict(d=512, n_heads=4, n_kv_heads=1, head_dim=128, ffn=1376, vocab=3001,
+                                         n_layers=2, dtype="bf16", B=4, prefix=0, top_k=8, rope_theta=5e5,
+                                         seed=19, page_size=24), prefix_list=[23, 24, 47, 400]),
     # N * B = 160 rows: the wide tensor-core LM head with three 64-row transpose groups
     "wide_lmhead_r160": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=3001,
                                        n_layers=5, dtype="bf16", B=32, prefix=0, top_k=8, rope_theta=1e4,
