@@ -147,27 +147,38 @@ __device__ __forceinline__ int unit_owner(int64_t u, int64_t U, int G) {
 template <int BP>
 __device__ __forceinline__ void lin_epilogue(const LinearArgs& a, int m, const float (&v)[BP]) {
     const int lane = threadIdx.x & 31;
+    // Every operand is read before any result is written: a load after a store to the same
+    // buffer would wait for it, making the 32 rows one chain of L2 round trips.
     if (a.epi == EPI_SWIGLU) {
+        float o[BP];
 #pragma unroll
-        for (int b = 0; b < BP; ++b) {
-            const float up = __shfl_xor_sync(0xffffffffu, v[b], 1);
-            if (b < a.B && !(lane & 1) && m + 1 < a.M) a.y[(size_t)b * a.ldy + (m >> 1)] = silu(v[b]) * up;
-        }
+        for (int b = 0; b < BP; ++b) o[b] = silu(v[b]) * __shfl_xor_sync(0xffffffffu, v[b], 1);
+        if ((lane & 1) || m + 1 >= a.M) return;
+        float* y = a.y + (m >> 1);
+#pragma unroll
+        for (int b = 0; b < BP; ++b)
+            if (b < a.B) y[(size_t)b * a.ldy] = o[b];
         return;
     }
     if (m >= a.M) return;
+    float* y = a.y + m;
+    if (a.epi == EPI_RESID) {
+        const float* base = a.ybase ? a.ybase + m : y;
+        float r[BP];
 #pragma unroll
-    for (int b = 0; b < BP; ++b) {
-        if (b >= a.B) break;
-        float* yp = a.y + (size_t)b * a.ldy + m;
-        if (a.epi == EPI_RESID) {
-            const float nv = __ldcg(a.ybase ? a.ybase + (size_t)b * a.ldy + m : yp) + v[b];
-            *yp = nv;
+        for (int b = 0; b < BP; ++b) r[b] = b < a.B ? __ldcg(base + (size_t)b * a.ldy) : 0.f;
+#pragma unroll
+        for (int b = 0; b < BP; ++b) {
+            if (b >= a.B) break;
+            const float nv = r[b] + v[b];
+            y[(size_t)b * a.ldy] = nv;
             if (a.y2) a.y2[(size_t)b * a.ldy2 + m] = nv;
-        } else {
-            *yp = v[b];
         }
+        return;
     }
+#pragma unroll
+    for (int b = 0; b < BP; ++b)
+        if (b < a.B) y[(size_t)b * a.ldy] = v[b];
 }
 
 template <int BP>  // B_pad: 8, 16, 24 or 32
@@ -291,13 +302,13 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             float* pp = part + ((size_t)(cta * 2 + slot) * BP) * 128 + r;
 #pragma unroll
             for (int b = 0; b < BP; ++b) pp[(size_t)b * 128] = v[b];
-            __threadfence();
+            // lane 0's acquire-release add publishes the warp's shares (ordered before it by
+            // the warp barrier) and, in the last warp to arrive, orders the reads below
             __syncwarp();
             int last = 0;
-            if (lane == 0) last = atomicAdd(&counters[tile * 4 + warp], 1) == c_last - c_first;
+            if (lane == 0) last = atom_add_acq_rel_gpu(&counters[tile * 4 + warp], 1) == c_last - c_first;
             last = __shfl_sync(0xffffffffu, last, 0);
             if (!last) continue;
-            __threadfence();
             float s[BP];
 #pragma unroll
             for (int b = 0; b < BP; ++b) s[b] = 0.f;
