@@ -57,9 +57,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearA
     // weights do not depend on the previous kernel: start streaming them first
     const int issued = stream_begin<WT>((const unsigned char*)a.W, a.K, g0, g1, s, D);
     griddep_launch_dependents();
-    griddep_wait();
+    // gains and embedding rows do not depend on the previous kernel either
     ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
-    stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red);
+    const bool pre = stage_pre<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status);
+    griddep_wait();
+    stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red, pre);
     __syncthreads();
     LinearEpi<BT> e{&a, b0, nb};
     stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e, issued);

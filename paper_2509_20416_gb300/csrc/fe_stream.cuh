@@ -384,14 +384,85 @@ __device__ __forceinline__ void scale_span(const T* __restrict__ gamma, float* d
     }
 }
 
+// The part of the prologue that reads nothing an earlier kernel writes, for a caller to run
+// before griddep_wait(): the RMSNorm gains, widened into X (the rows' activations then need
+// one read of x and one pass over shared memory), or the token-embedding half of a
+// concatenation. Returns true when it ran; stage_activations must then get pre = true.
+// (For RMSNorm only when a row fits the single-round register path: K <= 8192, aligned.)
+template <typename WT>
+__device__ bool stage_pre(const ProParams& p, int K, float* X, int Kpad, int b0, int nb, int* status) {
+    const int t = threadIdx.x;
+    if (p.pro == PRO_RMSNORM) {
+        if (K % 4 != 0 || K / 4 > kStreamThreads * 8 || p.ldx % 4 != 0 ||
+            (reinterpret_cast<uintptr_t>(p.x) & 15) != 0)
+            return false;
+        for (int b = 0; b < nb; ++b) stage_span<WT, false>((const WT*)p.gamma, X + (size_t)b * Kpad, K);
+        return true;
+    }
+    if (p.pro == PRO_CONCAT_EMB) {
+        const int de = K - p.d_split;
+        for (int b = 0; b < nb; ++b) {
+            float* Xb = X + (size_t)b * Kpad;
+            int tok = p.tok[b0 + b];
+            if (tok < 0 || tok >= p.vocab) {
+                if (t == 0) atomicOr(status, ST_DEVICE);
+                for (int k = t; k < de; k += kStreamThreads) Xb[p.d_split + k] = 0.f;
+            } else {
+                stage_span<WT, false>((const WT*)p.embed + (size_t)tok * de, Xb + p.d_split, de);
+            }
+        }
+        return true;
+    }
+    return false;
+}
+
 template <typename WT>
 __device__ void stage_activations(const ProParams& p, int K, float* X, int Kpad, int b0, int nb, int* status,
-                                  float* scratch /* >= kWarps floats */) {
+                                  float* scratch /* >= kWarps floats */, bool pre = false) {
     const int t = threadIdx.x;
     for (int b = 0; b < nb; ++b) {
         const int row = b0 + b;
         float* Xb = X + (size_t)b * Kpad;
-        if (p.pro == PRO_F32) {
+        if (pre && p.pro == PRO_CONCAT_EMB) {  // the embedding half is in place
+            stage_span<float, false>((const float*)p.x + (size_t)row * p.ldx, Xb, p.d_split);
+        } else if (pre && p.pro == PRO_RMSNORM) {
+            // Xb holds gamma: one round of up to 8 float4 loads of x per thread, the sum of
+            // squares in the same order as stage_span, then Xb = (x * rs) * gamma in place
+            const float4* x4 = reinterpret_cast<const float4*>((const float*)p.x + (size_t)row * p.ldx);
+            const int nv = K / 4;
+            float4 r[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = t + u * kStreamThreads;
+                r[u] = i < nv ? __ldcg(x4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            float ss = 0.f;
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                if (t + u * kStreamThreads < nv) {
+                    ss = fmaf(r[u].x, r[u].x, ss);
+                    ss = fmaf(r[u].y, r[u].y, ss);
+                    ss = fmaf(r[u].z, r[u].z, ss);
+                    ss = fmaf(r[u].w, r[u].w, ss);
+                }
+            ss = warp_sum(ss);
+            if ((t & 31) == 0) scratch[t >> 5] = ss;
+            __syncthreads();
+            float tot = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) tot += scratch[w];
+            const float rs = 1.0f / sqrtf(tot / (float)K + p.eps);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = t + u * kStreamThreads;
+                if (i < nv) {
+                    float4* d = reinterpret_cast<float4*>(Xb) + i;
+                    const float4 gm = *d;
+                    *d = make_float4(r[u].x * rs * gm.x, r[u].y * rs * gm.y, r[u].z * rs * gm.z, r[u].w * rs * gm.w);
+                }
+            }
+            __syncthreads();  // scratch reuse by the next row
+        } else if (p.pro == PRO_F32) {
             stage_span<float, false>((const float*)p.x + (size_t)row * p.ldx, Xb, K);
         } else if (p.pro == PRO_STORAGE) {
             stage_span<WT, false>((const WT*)p.x + (size_t)row * p.ldx, Xb, K);
