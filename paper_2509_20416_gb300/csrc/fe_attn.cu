@@ -451,13 +451,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
-// ---- tensor-core attention (bf16 caches, hd = 128, G >= 2 query heads per KV head) -----------
+// ---- tensor-core attention (bf16 caches, hd = 128, G = 1..8 query heads per KV head) ---------
 // The same work items, chunk ownership, own-row append and split combine as attn_kernel;
 // the per-chunk arithmetic runs on mma.sync (m16n8k16, bf16 operands, float32 accumulate)
 // with the keys and the head dimensions as the long matrix sides:
 //   S^T (32 keys x 8 heads) = K (32 x 128) . Q^T            2 key tiles x 8 k-steps
 //   O^T (128 dims x 8 heads) += V^T (128 x 32) . P^T          8 dim tiles x 2 k-steps
-// so a KV head's G <= 8 query heads fill the 8-wide side. Q and P enter as bf16 hi + lo
+// so a KV head's G <= 8 query heads fill the 8-wide side (with G = 1 seven columns idle: the
+// products are still far cheaper than the CUDA-core kernel's shuffle reductions). Q and P enter as bf16 hi + lo
 // pairs (two products each), which keeps scores and outputs at float32-level accuracy; K
 // and V are bf16 in the cache already.
 //   - Rows arrive by cp.async (16 bytes per lane, two rows per warp instruction, each lane
@@ -1001,7 +1002,7 @@ static cudaError_t prepare_g() {
                                 (int)attn_smem(HD, sizeof(CT), max_slots(HD, sizeof(CT))) + kAttnPageSmem);
 }
 
-// bf16, hd 128, G >= 2 runs on the tensor-core kernel unless FE_DRAFT_ATTN_TC=0 selects
+// bf16 at hd 128 runs on the tensor-core kernel unless FE_DRAFT_ATTN_TC=0 selects
 // the CUDA-core kernel (kept for comparison)
 static bool attn_tc_enabled() {
     const char* e = getenv("FE_DRAFT_ATTN_TC");
@@ -1011,7 +1012,7 @@ static bool attn_tc_enabled() {
 template <typename CT, int HD, int G>
 static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
     const int S = attn_slots(a.split, HD, sizeof(CT));
-    if constexpr (sizeof(CT) == 2 && HD == 128 && G >= 2) {
+    if constexpr (sizeof(CT) == 2 && HD == 128) {
         if (attn_tc_enabled()) {
             const size_t pg = attn_page_ints(a) * sizeof(int);
             if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
@@ -1048,7 +1049,7 @@ static cudaError_t prepare_hd() {
 
 cudaError_t attention_prepare() {
     cudaError_t e;
-    for (auto k : {attn_tc_kernel<2>, attn_tc_kernel<4>, attn_tc_kernel<8>})
+    for (auto k : {attn_tc_kernel<1>, attn_tc_kernel<2>, attn_tc_kernel<4>, attn_tc_kernel<8>})
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)(kAttnWarps * 2 * kTcHalfBytes) + kAttnPageSmem)) != cudaSuccess)
             return e;

@@ -96,7 +96,7 @@ SMALL = {
                                       n_layers=3, dtype="bf16", B=12, prefix=0, top_k=8, rope_theta=1e4,
                                       seed=14, page_size=0, parallel_layers=1),
                             prefix_list=[37, 0, 150, 1, 64, 5, 300, 2, 128, 129, 7, 90]),
-    # bf16, hd 128, G >= 2: the tensor-core attention kernel. Prefixes on both sides of
+    # bf16, hd 128, G = 2, 4, 8 (G = 1 below and at full size): the tensor-core attention kernel. Prefixes on both sides of
     # the 32-key chunk and 128-key split boundaries, an empty prefix, several splits per
     # sequence (combined by the last split), page sizes 16 and 8, and contiguous caches.
     "tc_attn_g4_paged16": dict(name=dict(d=512, n_heads=4, n_kv_heads=1, head_dim=128, ffn=1376, vocab=3001,
