@@ -27,7 +27,7 @@ _lock = threading.Lock()
 _cache: dict = {}
 
 # Number of planted-mistake variants compiled by build(mutant=n) (n = 1..N_MUTANTS).
-N_MUTANTS = 33
+N_MUTANTS = 36
 _UNUSED_MUTANTS = {25}  # ids with no planted mistake
 
 
@@ -95,7 +95,7 @@ class Oracle:
                                    ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, _D, _D, _D]
         L.or_silu_mul.argtypes = [_D, _D, ctypes.c_int64, _D]
         L.or_layer.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(_P), ctypes.c_double, _P, _P,
-                               ctypes.c_int64, ctypes.c_int32, _D]
+                               ctypes.c_int64, ctypes.c_int32, _D, _D, _D]
         L.or_lm_head.argtypes = [ctypes.POINTER(Config), _P, _P, _D, _D]
         L.or_softmax.argtypes = [_D, ctypes.c_int64, ctypes.c_double, _D, _D]
         L.or_topk.argtypes = [_D, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]
@@ -117,6 +117,9 @@ class Oracle:
                                    ctypes.POINTER(ctypes.c_int32), _D, _D]
         L.or_draft_seq.restype = ctypes.c_int32
         L.or_max_threads.restype = ctypes.c_int32
+        L.or_commit_seq.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(_P), _P, _I, ctypes.c_int32,
+                                    ctypes.c_int32, ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.c_int64]
+        L.or_commit_seq.restype = ctypes.c_int32
         self.L = L
         self.path = path
 
@@ -262,8 +265,30 @@ class Oracle:
                 lw["w_up"], lw["w_down"]]
         warr = (_P * 7)(*[_ptr(t) for t in ptrs])
         x = np.array(x, dtype=np.float64)
-        self.L.or_layer(ctypes.byref(c), warr, float(pos), _ptr(kc), _ptr(vc), cap, P, _dp(x))
+        self.L.or_layer(ctypes.byref(c), warr, float(pos), _ptr(kc), _ptr(vc), cap, P, _dp(x), None, None)
         return x
+
+    def commit_seq(self, cfg: dict, weights: dict, feats, toks, P: int, kcs, vcs, cap: int,
+                   rope_layer_offset: int = 0):
+        """Commit len(toks) accepted rows of one sequence at positions P, P + 1, .. (Sec. 2.4,
+        "Update and Iterate"): feats [n, 3d] in the storage type, toks [n]; ``kcs``/``vcs``
+        are N host buffers of this sequence's [Hkv, cap, hd] cache, written in place."""
+        c = config_struct(cfg, rope_layer_offset, 1)
+        N = cfg["n_layers"]
+        ptrs = [weights["w_fuse"], weights["w_in"], weights["embed"], weights["lm_head"],
+                weights["final_norm"]]
+        for lw in weights["layers"]:
+            ptrs += [lw["attn_norm"], lw["w_qkv"], lw["w_o"], lw["mlp_norm"], lw["w_gate"],
+                     lw["w_up"], lw["w_down"]]
+        warr = (_P * len(ptrs))(*[_ptr(t) for t in ptrs])
+        karr = (_P * N)(*[_ptr(t) for t in kcs])
+        varr = (_P * N)(*[_ptr(t) for t in vcs])
+        toks = np.ascontiguousarray(np.asarray(toks), dtype=np.int32)
+        rc = self.L.or_commit_seq(ctypes.byref(c), warr, _ptr(feats) if len(toks) else None,
+                                  toks.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), len(toks), int(P),
+                                  karr, varr, int(cap))
+        if rc != 0:
+            raise ValueError("oracle rejected the arguments")
 
 
 def config_struct(cfg: dict, rope_layer_offset: int = 0, final_norm: int = 1) -> Config:

@@ -64,6 +64,38 @@ static double ld(const void *p, int32_t dtype, int64_t i)
     return (double)f;
 }
 
+/* Store v in the cache's storage type: float32 by C's double -> float conversion (round to
+ * nearest), bfloat16 by rounding the double to the nearest bfloat16 (ties to even). The
+ * cache holds stored values: a later row reads the rounded one. */
+static void st(void *p, int32_t dtype, int64_t i, double v)
+{
+    if (dtype == 0) {
+        ((float *)p)[i] = (float)v;
+        return;
+    }
+    if (isnan(v)) {
+        ((uint16_t *)p)[i] = 0x7FC0;
+        return;
+    }
+    /* the two bfloat16 neighbours of v (bfloat16 values are exact floats, so compare in
+       double): truncate the float nearest below |v|, then pick the closer, ties to even */
+    const double a = fabs(v);
+    float f = (float)a;
+    if ((double)f > a)
+        f = nextafterf(f, 0.0f);
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    uint32_t lo = u & 0xFFFF0000u, hi = lo + 0x10000u;
+    float flo, fhi;
+    memcpy(&flo, &lo, 4);
+    memcpy(&fhi, &hi, 4);
+    const double dlo = a - (double)flo, dhi = (double)fhi - a;
+    uint32_t r = (dlo < dhi || (dlo == dhi && !((lo >> 16) & 1u))) ? lo : hi;
+    if (v < 0)
+        r |= 0x80000000u;
+    ((uint16_t *)p)[i] = (uint16_t)(r >> 16);
+}
+
 void or_widen(const void *src, int32_t dtype, int64_t n, double *dst)
 {
     for (int64_t i = 0; i < n; ++i)
@@ -194,9 +226,10 @@ void or_silu_mul(const double *gate, const double *up, int64_t n, double *y)
 /* One cascade layer L_i (Eq. 2) for one sequence, x updated in place.
  * lw: attn_norm, w_qkv [(H+2Hkv)hd, d], w_o [d, H hd], mlp_norm, w_gate [F,d],
  * w_up [F,d], w_down [d,F]. The drafted row sits at sequence position `pos`; it
- * attends to its P prefix rows in (kc, vc) plus its own key/value. */
+ * attends to its P prefix rows in (kc, vc) plus its own key/value. When k_out / v_out
+ * are given they receive the row's own key (rotated) and value, [Hkv][hd]. */
 void or_layer(const or_config *c, const void *const *lw, double pos, const void *kc,
-              const void *vc, int64_t cap, int32_t P, double *x)
+              const void *vc, int64_t cap, int32_t P, double *x, double *k_out, double *v_out)
 {
     const int32_t d = c->d, H = c->n_heads, Hkv = c->n_kv_heads, hd = c->head_dim, F = c->ffn;
     const int64_t nq = (int64_t)H * hd, nkv = (int64_t)Hkv * hd;
@@ -221,6 +254,10 @@ void or_layer(const or_config *c, const void *const *lw, double pos, const void 
             or_rope(v + (int64_t)g * hd, hd, pos, c->rope_theta);
     }
     or_attention(q, H, Hkv, hd, kc, vc, c->dtype, cap, P, k, v, o);
+    if (k_out)
+        memcpy(k_out, k, sizeof(double) * (size_t)nkv);
+    if (v_out)
+        memcpy(v_out, v, sizeof(double) * (size_t)nkv);
     or_matvec(lw[2], c->dtype, d, nq, o, t);
     for (int32_t j = 0; j < d; ++j)
         x[j] = MUT(7) ? t[j] : x[j] + t[j];
@@ -408,21 +445,13 @@ int32_t or_accept_greedy(int32_t T, const int32_t *tok, const int32_t *parent, c
  *   kc, vc: N pointers, each this sequence's [Hkv][cap][hd] cache of layer i
  * Outputs: hidden [N][d]; logits [N][V] (may be NULL); lse [N]; topk_id [N][k];
  * topk_logit [N][k]; topk_prob [N][k]. */
-int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat, int32_t tok,
-                     int32_t P, const void *const *kc, const void *const *vc, int64_t cap,
-                     int32_t top_k, double temperature, double *hidden, double *logits,
-                     double *lse, int32_t *topk_id, double *topk_logit, double *topk_prob)
+/* Eq. 1 for one row: g = FC(concat(l, m, h)) of feat [3d], e = Embed[tok],
+ * x0 = FC(concat(g, e)); w as for or_draft_seq. */
+static void input_row(const or_config *c, const void *const *w, const void *feat, int32_t tok, double *x0)
 {
-    const int32_t d = c->d, V = c->vocab, N = c->n_layers;
-    if (tok < 0 || tok >= V || P < 0 || P + 1 > cap || top_k < 1 || top_k > V)
-        return -1;
+    const int32_t d = c->d, V = c->vocab;
     double *f = (double *)malloc(sizeof(double) * (size_t)(3 * d));
     double *ge = (double *)malloc(sizeof(double) * (size_t)(2 * d));
-    double *x0 = (double *)malloc(sizeof(double) * (size_t)d);
-    double *x = (double *)malloc(sizeof(double) * (size_t)d);
-    double *lg = (double *)malloc(sizeof(double) * (size_t)V);
-    double *pr = (double *)malloc(sizeof(double) * (size_t)V);
-
     /* g = FC(concat(l, m, h)) */
     or_widen(feat, c->dtype, 3 * d, f);
     if (MUT(18))
@@ -437,6 +466,23 @@ int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat,
         e[j] = ld(w[2], c->dtype, row * d + j);
     /* x0 = FC(concat(g, e))   (Eq. 1) */
     or_matvec(w[1], c->dtype, d, 2 * d, ge, x0);
+    free(f); free(ge);
+}
+
+int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat, int32_t tok,
+                     int32_t P, const void *const *kc, const void *const *vc, int64_t cap,
+                     int32_t top_k, double temperature, double *hidden, double *logits,
+                     double *lse, int32_t *topk_id, double *topk_logit, double *topk_prob)
+{
+    const int32_t d = c->d, V = c->vocab, N = c->n_layers;
+    if (tok < 0 || tok >= V || P < 0 || P + 1 > cap || top_k < 1 || top_k > V)
+        return -1;
+    double *x0 = (double *)malloc(sizeof(double) * (size_t)d);
+    double *x = (double *)malloc(sizeof(double) * (size_t)d);
+    double *lg = (double *)malloc(sizeof(double) * (size_t)V);
+    double *pr = (double *)malloc(sizeof(double) * (size_t)V);
+
+    input_row(c, w, feat, tok, x0);
     memcpy(x, x0, sizeof(double) * (size_t)d);
 
     /* h_i = L_i(h_{i-1})      (Eq. 2), or h_i = L_i(x0) for the parallel ablation */
@@ -444,7 +490,7 @@ int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat,
         if (c->parallel_layers || MUT(10))
             memcpy(x, x0, sizeof(double) * (size_t)d);
         double pos = (double)P + (c->rope_layer_offset ? (double)i : 0.0) + (MUT(19) ? 1.0 : 0.0);
-        or_layer(c, w + 5 + 7 * i, pos, kc[i], vc[i], cap, P, x);
+        or_layer(c, w + 5 + 7 * i, pos, kc[i], vc[i], cap, P, x, NULL, NULL);
         memcpy(hidden + (int64_t)i * d, x, sizeof(double) * (size_t)d);
     }
 
@@ -461,7 +507,52 @@ int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat,
         if (logits)
             memcpy(logits + (int64_t)i * V, lg, sizeof(double) * (size_t)V);
     }
-    free(f); free(ge); free(x0); free(x); free(lg); free(pr);
+    free(x0); free(x); free(lg); free(pr);
+    return 0;
+}
+
+/* Sec. 2.4, "Update and Iterate" (the commit step of reading C15): once the target has
+ * accepted a path, the drafter's per-layer caches get rows for the accepted positions.
+ * Row i (0 <= i < n) sits at sequence position P + i; its inputs are feat[i] ([3d], the
+ * target's fused features of the position before it) and tok[i] (the token at P + i). It
+ * goes through Eq. 1 and the cascade exactly like a drafted row (no LM head): layer l
+ * attends to cache rows 0 .. P + i - 1 -- which include the rows of this commit before it
+ * -- plus its own key and value, and then stores its key (rotated) and value in slot
+ * P + i of layer l's cache, in the cache's storage type (see st()). kc / vc: N pointers to
+ * this sequence's [Hkv][cap][hd] caches, written in place. Returns 0, or -1 on an invalid
+ * argument (nothing written). */
+int32_t or_commit_seq(const or_config *c, const void *const *w, const void *feat, const int32_t *tok,
+                      int32_t n, int32_t P, void *const *kc, void *const *vc, int64_t cap)
+{
+    const int32_t d = c->d, V = c->vocab, N = c->n_layers, Hkv = c->n_kv_heads, hd = c->head_dim;
+    if (n < 0 || P < 0 || (int64_t)P + n > cap)
+        return -1;
+    for (int32_t i = 0; i < n; ++i)
+        if (tok[i] < 0 || tok[i] >= V)
+            return -1;
+    const int64_t nkv = (int64_t)Hkv * hd;
+    double *x0 = (double *)malloc(sizeof(double) * (size_t)d);
+    double *x = (double *)malloc(sizeof(double) * (size_t)d);
+    double *kn = (double *)malloc(sizeof(double) * (size_t)nkv);
+    double *vn = (double *)malloc(sizeof(double) * (size_t)nkv);
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t p = P + i;
+        input_row(c, w, (const unsigned char *)feat + (size_t)i * 3 * d * (c->dtype == 0 ? 4 : 2), tok[i], x0);
+        memcpy(x, x0, sizeof(double) * (size_t)d);
+        for (int32_t l = 0; l < N; ++l) {
+            if (c->parallel_layers)
+                memcpy(x, x0, sizeof(double) * (size_t)d);
+            const double pos = (double)p + (c->rope_layer_offset ? (double)l : 0.0) + (MUT(36) ? 1.0 : 0.0);
+            or_layer(c, w + 5 + 7 * l, pos, kc[l], vc[l], cap, MUT(34) ? P : p, x, kn, vn);
+            const int32_t slot = MUT(35) ? p + 1 < cap ? p + 1 : p : p;
+            for (int32_t g = 0; g < Hkv; ++g)
+                for (int32_t j = 0; j < hd; ++j) {
+                    st(kc[l], c->dtype, ((int64_t)g * cap + slot) * hd + j, kn[(int64_t)g * hd + j]);
+                    st(vc[l], c->dtype, ((int64_t)g * cap + slot) * hd + j, vn[(int64_t)g * hd + j]);
+                }
+        }
+    }
+    free(x0); free(x); free(kn); free(vn);
     return 0;
 }
 

@@ -460,6 +460,65 @@ def pin_zero_blocks(orc):
         assert list(tok[1 + i * k: 1 + (i + 1) * k]) == list(tok[1:1 + k])
 
 
-ALL_PINS = [pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
+def pin_commit(orc):
+    """The commit of accepted rows (Sec. 2.4, "Update and Iterate"): against the torch
+    reference (each row through Eq. 1 and the cascade, its keys and values stored before
+    the next row runs); one commit of n rows equals n commits of one row; rows other than
+    P .. P + n - 1 stay untouched; a row does not depend on the rows after it; n = 0 is a
+    no-op; bfloat16 storage rounds to the nearest value."""
+    cfg = mini_cfg(n_layers=3, B=1, max_seq=12)
+    W, I, ks, vs = _mini_problem(cfg)
+    N, d, cap, P, n = cfg["n_layers"], cfg["d"], cfg["max_seq"], 3, 4
+    feats = torch.empty(n, 3 * d, dtype=torch.float32)
+    fe_synth.fill_normal(feats, 31, 1, 1.0)
+    toks = [5, 0, cfg["vocab"] - 1, 17]
+    base_k = [k[0].clone() for k in ks]
+    base_v = [v[0].clone() for v in vs]
+
+    def run(feat_rows, tok_rows, P0, kc, vc):
+        orc.commit_seq(cfg, W, feat_rows.contiguous(), tok_rows, P0, kc, vc, cap)
+
+    ko, vo = [t.clone() for t in base_k], [t.clone() for t in base_v]
+    run(feats, toks, P, ko, vo)
+    kr, vr = [t.clone() for t in base_k], [t.clone() for t in base_v]
+    torch_ref.commit(cfg, W, feats, toks, P, kr, vr)
+    for l in range(N):
+        for a, b, base in ((ko[l], kr[l], base_k[l]), (vo[l], vr[l], base_v[l])):
+            rows = slice(P, P + n)
+            assert torch.allclose(a[:, rows], b[:, rows], rtol=1e-6, atol=1e-6), l
+            assert torch.equal(a[:, :P], base[:, :P]) and torch.equal(a[:, P + n:], base[:, P + n:]), l
+            assert not torch.equal(a[:, rows], base[:, rows])
+    # n commits of one row each
+    k1, v1 = [t.clone() for t in base_k], [t.clone() for t in base_v]
+    for i in range(n):
+        run(feats[i:i + 1], toks[i:i + 1], P + i, k1, v1)
+    assert all(torch.equal(a, b) for a, b in zip(k1 + v1, ko + vo))
+    # causality: changing the last row leaves the earlier rows as they were
+    k2, v2 = [t.clone() for t in base_k], [t.clone() for t in base_v]
+    run(feats, toks[:-1] + [toks[-1] + 1], P, k2, v2)
+    for l in range(N):
+        assert torch.equal(k2[l][:, :P + n - 1], ko[l][:, :P + n - 1])
+        assert not torch.equal(k2[l][:, P + n - 1], ko[l][:, P + n - 1])
+    # nothing to commit
+    k3, v3 = [t.clone() for t in base_k], [t.clone() for t in base_v]
+    run(feats[:0], [], P, k3, v3)
+    assert all(torch.equal(a, b) for a, b in zip(k3 + v3, base_k + base_v))
+    # bfloat16 caches: the stored value is the nearest bfloat16 of the exact one
+    cb = mini_cfg(n_layers=2, B=1, max_seq=12, dtype="bf16")
+    Wb, Ib, ksb, vsb = _mini_problem(cb)
+    kb, vb = [k[0].clone() for k in ksb], [v[0].clone() for v in vsb]
+    fb = feats[:2].to(torch.bfloat16)
+    orc.commit_seq(cb, Wb, fb.contiguous(), toks[:2], P, kb, vb, cap)
+    kx, vx = [k[0].clone().double() for k in ksb], [v[0].clone().double() for v in vsb]
+    torch_ref.commit(cb, Wb, fb, toks[:1], P, kx, vx)  # the first row, exact (float64)
+    for l in range(2):
+        for a, x in ((kb[l], kx[l]), (vb[l], vx[l])):
+            got = a[:, P].double()
+            ex = x[:, P]
+            ulp = torch.exp2(torch.floor(torch.log2(ex.abs().clamp_min(1e-30))) - 7)
+            assert ((got - ex).abs() <= 0.5 * ulp * (1 + 1e-12) + 1e-300).all(), l
+
+
+ALL_PINS = [pin_commit, pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
             pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]

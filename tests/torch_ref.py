@@ -31,6 +31,12 @@ def rope_complex(x: torch.Tensor, pos: float, theta: float) -> torch.Tensor:
 def layer(cfg: dict, L: dict, x: torch.Tensor, pos: float, kc: torch.Tensor, vc: torch.Tensor,
           P: int) -> torch.Tensor:
     """One pre-norm decoder layer for one sequence; kc, vc [Hkv, cap, hd]."""
+    return layer_kv(cfg, L, x, pos, kc, vc, P)[0]
+
+
+def layer_kv(cfg: dict, L: dict, x: torch.Tensor, pos: float, kc: torch.Tensor, vc: torch.Tensor,
+             P: int):
+    """layer() returning also the row's own key (rotated) and value, [Hkv, hd] each."""
     d, H, Hkv, hd = cfg["d"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
     eps = cfg["rms_eps"]
     u = F.rms_norm(x, (d,), weight=_d(L["attn_norm"]), eps=eps)
@@ -49,7 +55,7 @@ def layer(cfg: dict, L: dict, x: torch.Tensor, pos: float, kc: torch.Tensor, vc:
     x = x + _d(L["w_o"]) @ o.reshape(H * hd)
     u = F.rms_norm(x, (d,), weight=_d(L["mlp_norm"]), eps=eps)
     a = F.silu(_d(L["w_gate"]) @ u) * (_d(L["w_up"]) @ u)
-    return x + _d(L["w_down"]) @ a
+    return x + _d(L["w_down"]) @ a, k, v
 
 
 def draft(cfg: dict, W: dict, feat: torch.Tensor, tok: int, P: int, kcs, vcs, top_k: int,
@@ -71,3 +77,17 @@ def draft(cfg: dict, W: dict, feat: torch.Tensor, tok: int, P: int, kcs, vcs, to
     lse = torch.logsumexp(logits / T, dim=-1)
     order = torch.sort(-logits, dim=-1, stable=True).indices[:, :top_k]
     return dict(hidden=h, logits=logits, lse=lse, prob=logp.exp(), topk_id=order)
+
+
+def commit(cfg: dict, W: dict, feats: torch.Tensor, toks, P: int, kcs, vcs) -> None:
+    """Commit rows at positions P, P + 1, ..: each row runs Eq. 1 and the cascade, then its
+    per-layer key and value are stored (in the caches' dtype) in slot P + i before the next
+    row runs; kcs[i], vcs[i] [Hkv, cap, hd] are written in place."""
+    for i, tok in enumerate(toks):
+        g = _d(W["w_fuse"]) @ _d(feats[i])
+        e = _d(W["embed"])[int(tok)]
+        x = _d(W["w_in"]) @ torch.cat([g, e])
+        for l, L in enumerate(W["layers"]):
+            x, k, v = layer_kv(cfg, L, x, P + i, kcs[l], vcs[l], P + i)
+            kcs[l][:, P + i, :] = k.to(kcs[l].dtype)
+            vcs[l][:, P + i, :] = v.to(vcs[l].dtype)
