@@ -350,6 +350,24 @@ def main():
     if st != fe.FE_OK:
         raise SystemExit(f"device status after the loss forward: {fe.fe_status_str(st)}")
 
+    # ---- update step (not part of the draft step): fe_commit of N accepted rows per sequence;
+    # written over rows the caches already hold (P_b - N ..), so paged pools need no new pages
+    cfeat = torch.randn((B, N, 3 * d), generator=g).to(wl.torch_dtype(cfg)).cuda()
+    ctok = torch.randint(0, cfg["vocab"], (B, N), generator=g, dtype=torch.int32).cuda()
+    cn = torch.full((B,), N, dtype=torch.int32).cuda()
+    cplen = torch.clamp(I["prefix_len"] - N, min=0).to(torch.int32).cuda()
+    for _ in range(3):
+        fe.fe_commit(h, cfeat, ctok, cn, cplen, kd, vd, page_table=table, n_pages=n_pages, stream=stream)
+    v0.record(stream)
+    for _ in range(10):
+        fe.fe_commit(h, cfeat, ctok, cn, cplen, kd, vd, page_table=table, n_pages=n_pages, stream=stream)
+    v1.record(stream)
+    v1.synchronize()
+    commit_us = 1000.0 * v0.elapsed_time(v1) / 10
+    st = fe.fe_last_device_status(h)
+    if st != fe.FE_OK:
+        raise SystemExit(f"device status after the commits: {fe.fe_status_str(st)}")
+
     # ---- roofline of the dominant kernel (and of the whole step, for context) ----------------
     peak, peak_kind = peaks()
     plist = I["prefix_len"].tolist()
@@ -384,6 +402,10 @@ def main():
             "kernels": kernels,
             "verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
                               "note": "fe_verify_greedy after the step (positions + greedy acceptance walk)"},
+            "commit": {"us_per_call": commit_us, "rows_per_sequence": N,
+                       "note": "fe_commit of N accepted rows per sequence (Sec. 2.4 Update and Iterate): "
+                               "Eq. 1 and the cascade over the rows, one weight stream per 32 rows; "
+                               "outside the timed step"},
             "draft_loss": {"us_per_call": loss_us,
                            "note": "fe_draft_loss: the draft with logits [B,N,V] and hidden states written out, "
                                    "then CE + Smooth L1 (Sec. 2.3); outside the timed step"},

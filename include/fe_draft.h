@@ -217,6 +217,39 @@ FE_API fe_status fe_verify_greedy(fe_handle *h, int32_t B, int32_t top_k, const 
                                   const fe_tree *tree, const int32_t *target_next, int32_t *pos_ids,
                                   int32_t *path, int32_t *n_accept, int32_t *bonus, void *stream);
 
+/* The update step of a cycle (Sec. 2.4, "Update and Iterate"): before the next draft can
+ * attend to the positions the target accepted, each layer's cache needs their rows. For
+ * each sequence b, rows i = 0 .. n_rows[b]-1 sit at positions prefix_len[b] + i; row i has
+ * inputs feat[b][i] (the target's concat(l, m, h) of the position before it) and tok[b][i]
+ * (the token at its position). Each row runs through Eq. 1 and the cascade exactly like a
+ * drafted row (no LM head): layer l attends to cache rows 0 .. prefix_len[b] + i - 1
+ * (which include the rows committed before it in this call) plus its own key and value,
+ * and stores its key (after RoPE) and value, rounded to the cache type, in slot
+ * prefix_len[b] + i. The call does not advance prefix_len.
+ *
+ *  B, L        sequences (1..max_batch) and rows per sequence in feat / tok (1..n_layers)
+ *  feat        device [B, L, 3d] dtype, 16-byte aligned
+ *  tok         device [B, L] int32; entries at i >= n_rows[b] are ignored
+ *  n_rows      device [B] int32 in 0..L
+ *  prefix_len  device [B] int32; capacity: prefix_len[b] + n_rows[b] <= max_seq
+ *  k_cache, v_cache, page_table, n_pages: as for fe_draft_forward
+ * Asynchronous on `stream`; FE_ERR_INVALID_ARG for bad host-side arguments, device-side
+ * range errors through fe_last_device_status (as fe_draft_forward). The rows of one call
+ * share one stream of the weights when B * L <= 32 (in blocks of 32 rows otherwise). */
+typedef struct {
+    int32_t B, L;
+    const void *feat;
+    const int32_t *tok;
+    const int32_t *n_rows;
+    const int32_t *prefix_len;
+    void *const *k_cache;
+    void *const *v_cache;
+    const int32_t *page_table;
+    int32_t n_pages;
+} fe_commit_args;
+
+FE_API fe_status fe_commit(fe_handle *h, const fe_commit_args *args, void *stream);
+
 /* Kernel families of one draft, as fe_profile_forward reports them. */
 typedef enum {
     FE_KERNEL_LINEAR = 0,    /* weight-streaming linear phase (W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down) */

@@ -61,6 +61,12 @@ class fe_tree(ctypes.Structure):
     _fields_ = [("tok", _vp), ("parent", _vp), ("depth", _vp), ("mask", _vp)]
 
 
+class fe_commit_args(ctypes.Structure):
+    _fields_ = [("B", _i32), ("L", _i32), ("feat", _vp), ("tok", _vp), ("n_rows", _vp), ("prefix_len", _vp),
+                ("k_cache", ctypes.POINTER(_vp)), ("v_cache", ctypes.POINTER(_vp)),
+                ("page_table", _vp), ("n_pages", _i32)]
+
+
 _lib.fe_draft_init.argtypes = [ctypes.POINTER(fe_config), ctypes.POINTER(fe_weights), _vp, ctypes.POINTER(_vp)]
 _lib.fe_draft_init.restype = ctypes.c_int
 _lib.fe_draft_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp]
@@ -86,6 +92,8 @@ _lib.fe_draft_loss.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, c
 _lib.fe_draft_loss.restype = ctypes.c_int
 _lib.fe_verify_greedy.argtypes = [_vp, _i32, _i32, _vp, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp]
 _lib.fe_verify_greedy.restype = ctypes.c_int
+_lib.fe_commit.argtypes = [_vp, ctypes.POINTER(fe_commit_args), _vp]
+_lib.fe_commit.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
 _lib.fe_last_error_detail.restype = ctypes.c_char_p
 
@@ -278,6 +286,18 @@ def fe_verify_greedy(h: Handle, prefix_len, tree: dict, target_next, top_k: int,
                                  _p(out["pos_ids"]), _p(out["path"]), _p(out["n_accept"]), _p(out["bonus"]),
                                  _stream(stream)), "fe_verify_greedy")
     return out
+
+
+def fe_commit(h: Handle, feat, tok, n_rows, prefix_len, k_cache, v_cache, page_table=None, n_pages: int = 0,
+              stream=None) -> None:
+    """Commit accepted rows into the caches (include/fe_draft.h): feat [B, L, 3d], tok [B, L]
+    int32, n_rows [B] int32, prefix_len [B] int32 (device tensors)."""
+    B, L = int(tok.shape[0]), int(tok.shape[1])
+    N = h.cfg["n_layers"]
+    kc = (_vp * N)(*[_p(t) for t in k_cache])
+    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    a = fe_commit_args(B, L, _p(feat), _p(tok), _p(n_rows), _p(prefix_len), kc, vc, _p(page_table), int(n_pages))
+    _check(_lib.fe_commit(h.ptr, ctypes.byref(a), _stream(stream)), "fe_commit")
 
 
 def fe_last_device_status(h: Handle, stream=None) -> int:

@@ -91,10 +91,17 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
 
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int P = a.prefix_len[b];
+    // (a commit launch handles row index pos_add of every sequence: its position is
+    // prefix_len + pos_add, and sequences with fewer rows to commit have no work here)
+    if (a.n_rows && a.pos_add >= a.n_rows[b]) {
+        griddep_launch_dependents();
+        return;
+    }
+    const int P = a.prefix_len[b] + a.pos_add;
+    const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
     const int ldq = (a.H + 2 * a.Hkv) * HD;
 
-    float* out = a.out + (size_t)b * a.H * HD + (size_t)g * G * HD;
+    float* out = a.out + qrow * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
         griddep_launch_dependents();
@@ -192,13 +199,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     const float scale = 1.0f / sqrtf((float)HD);
     for (int idx = t; idx < G * HALF; idx += blockDim.x) {
         const int j = idx / HALF, i = idx % HALF;
-        const float* q = a.qkv + (size_t)b * ldq + (size_t)(g * G + j) * HD;
+        const float* q = a.qkv + qrow * ldq + (size_t)(g * G + j) * HD;
         const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
         qs[j][i] = (x1 * c - x2 * sn) * scale;
         qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
     }
     if (t1 == P + 1) {  // this item holds the row's own key: rotate it and append k, v at slot P
-        const float* kq = a.qkv + (size_t)b * ldq + (size_t)a.H * HD + (size_t)g * HD;
+        const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
         const float* vq = kq + (size_t)a.Hkv * HD;
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
@@ -542,10 +549,17 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
 
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-    const int P = a.prefix_len[b];
+    // (a commit launch handles row index pos_add of every sequence: its position is
+    // prefix_len + pos_add, and sequences with fewer rows to commit have no work here)
+    if (a.n_rows && a.pos_add >= a.n_rows[b]) {
+        griddep_launch_dependents();
+        return;
+    }
+    const int P = a.prefix_len[b] + a.pos_add;
+    const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
     const int ldq = (a.H + 2 * a.Hkv) * HD;
 
-    float* out = a.out + (size_t)b * a.H * HD + (size_t)g * G * HD;
+    float* out = a.out + qrow * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
         griddep_launch_dependents();
@@ -638,14 +652,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     const float scale = 1.4426950408889634f / sqrtf((float)HD);
     for (int idx = t; idx < G * HALF; idx += blockDim.x) {
         const int j = idx / HALF, i = idx % HALF;
-        const float* q = a.qkv + (size_t)b * ldq + (size_t)(g * G + j) * HD;
+        const float* q = a.qkv + qrow * ldq + (size_t)(g * G + j) * HD;
         const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
         qs[j][i] = (x1 * c - x2 * sn) * scale;
         qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
     }
     const bool own = t1 == P + 1;  // this item holds the row's own key
     if (own) {  // rotate the new key and append k, v at slot P
-        const float* kq = a.qkv + (size_t)b * ldq + (size_t)a.H * HD + (size_t)g * HD;
+        const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
         const float* vq = kq + (size_t)a.Hkv * HD;
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);

@@ -199,6 +199,11 @@ struct AttnArgs {
     float* out;             // [B, H * hd]
     int* status;
     bool pdl;
+    // rows of qkv / out: sequence b's is row b * row_stride + row_off (a draft: 1, 0); the
+    // row sits at position prefix_len[b] + pos_add; with n_rows, sequences with
+    // n_rows[b] <= pos_add are skipped (a commit of accepted rows)
+    int row_stride = 1, row_off = 0, pos_add = 0;
+    const int* n_rows = nullptr;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();
@@ -209,6 +214,9 @@ inline int attention_launches() { return 1; }
 cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,
                         int* depth, uint8_t* mask, int* status, cudaStream_t st);
 cudaError_t launch_timeout_probe(int64_t timeout_ns, int* status, cudaStream_t st);
+// commit (fe_commit.cu): gather rows i0 .. i0 + nb - 1 of every sequence into a dense block
+cudaError_t launch_commit_gather(const void* feat, const int* tok, const int* n_rows, int B, int L, int i0, int nb,
+                                 int row_bytes, void* cfeat, int* ctok, cudaStream_t st);
 // training-objective forward (fe_loss.cu): ce, fl [B, N]; total [B]
 cudaError_t launch_loss(int N, int B, int V, int d, const float* logits, const float* teacher, const float* hidden,
                         const float* feat, float alpha, float beta, float decay, float* ce, float* fl, float* total,

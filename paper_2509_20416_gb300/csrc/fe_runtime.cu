@@ -58,6 +58,8 @@ struct fe_handle {
     const void *w_fuse = nullptr, *w_in = nullptr, *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
     std::vector<LayerPacked> layers;
     float* rope_cs = nullptr;
+    void* cfeat = nullptr;  // commit: one block's gathered feature rows [<= 32, 3d]
+    int* ctok = nullptr;    // commit: their tokens
     void* sbuf = nullptr;
     float *g = nullptr, *x = nullptr, *qkv = nullptr, *o = nullptr, *act = nullptr, *hid = nullptr;
     float* x0 = nullptr;  // the cascade input x0 (Eq. 1), kept for layer 1 and the parallel ablation
@@ -326,6 +328,86 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
 #undef FE_LINEAR
 }
 
+// The commit of accepted rows (include/fe_draft.h): blocks of up to 32 rows (whole row
+// indices of every sequence); per block the rows are gathered, then Eq. 1 and the cascade
+// run over them like a draft's rows, with one attention launch per row index (row i of a
+// sequence reads the rows before it from the cache, so they must be stored first).
+fe_status enqueue_commit(fe_handle* h, const fe_commit_args* a, cudaStream_t st) {
+    const fe_config& c = h->cfg;
+    const int B = a->B, d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
+    const int N = c.n_layers, nqkv = (H + 2 * Hkv) * hd;
+    const fe_dtype dt = c.dtype;
+    const bool pdl = h->use_pdl;
+    const int nb_max = std::max(1, std::min(a->L, 32 / B));
+    auto linear = [&](const LinearArgs& L) -> fe_status {
+        const cudaError_t e = h->lin_mma ? launch_linear_mma(L, h->lin_xb, h->lin_part, h->lin_counters, h->dev, st, nullptr)
+                                         : launch_linear(dt, L, h->dev, st);
+        return e == cudaSuccess ? FE_OK : fail(e, "commit linear phase launch", __LINE__);
+    };
+    fe_status rc;
+    for (int i0 = 0; i0 < a->L; i0 += nb_max) {
+        const int nb = std::min(nb_max, a->L - i0), R = B * nb;
+        FE_TRY(launch_commit_gather(a->feat, a->tok, a->n_rows, B, a->L, i0, nb, 3 * d * (int)h->es, h->cfeat, h->ctok,
+                                    st));
+        LinearArgs la{};
+        la.status = h->status;
+        la.eps = c.rms_eps;
+        la.B = R;
+        la.pdl = false;  // the gather kernel does not trigger programmatic launch
+        la.W = h->w_fuse; la.M = d; la.K = 3 * d;
+        la.pro = PRO_STORAGE; la.x = h->cfeat; la.ldx = 3 * d;
+        la.epi = EPI_STORE; la.y = h->g; la.ldy = d;
+        if ((rc = linear(la)) != FE_OK) return rc;
+        la.pdl = pdl;
+        la.W = h->w_in; la.M = d; la.K = 2 * d;
+        la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = h->ctok;
+        la.d_split = d; la.vocab = V;
+        la.epi = EPI_STORE; la.y = h->x0; la.ldy = d;
+        if ((rc = linear(la)) != FE_OK) return rc;
+
+        AttnArgs aa{};
+        aa.qkv = h->qkv; aa.prefix_len = a->prefix_len; aa.page_table = a->page_table;
+        aa.page_size = c.page_size; aa.max_seq = c.max_seq; aa.n_pages = a->n_pages;
+        aa.max_pages = c.page_size > 0 ? (c.max_seq + c.page_size - 1) / c.page_size : 0;
+        aa.rope_cs = h->rope_cs; aa.B = B; aa.H = H; aa.Hkv = Hkv; aa.hd = hd;
+        aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
+        aa.part = h->attn_part; aa.counters = h->attn_counters; aa.out = h->o; aa.status = h->status;
+        aa.pdl = pdl;
+        aa.row_stride = nb; aa.n_rows = a->n_rows;
+        for (int l = 0; l < N; ++l) {
+            const LayerPacked& Lw = h->layers[l];
+            const bool from_x0 = l == 0 || c.parallel_layers;
+            la.W = Lw.w_qkv; la.M = nqkv; la.K = d;
+            la.pro = PRO_RMSNORM; la.x = from_x0 ? h->x0 : h->x; la.ldx = d; la.gamma = Lw.attn_norm;
+            la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr; la.ybase = nullptr;
+            if ((rc = linear(la)) != FE_OK) return rc;
+            aa.kc = a->k_cache[l]; aa.vc = a->v_cache[l];
+            for (int j = 0; j < nb; ++j) {
+                aa.row_off = j;
+                aa.pos_add = i0 + j;
+                // row j reads the rows the launches before it appended: it must not start
+                // (and copy cache rows) before they finish
+                aa.pdl = j == 0 && pdl;
+                FE_TRY(launch_attention(dt, aa, st));
+            }
+            aa.pdl = pdl;
+            la.W = Lw.w_o; la.M = d; la.K = H * hd;
+            la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
+            la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.ybase = from_x0 ? h->x0 : nullptr;
+            if ((rc = linear(la)) != FE_OK) return rc;
+            la.W = Lw.w_gu; la.M = 2 * F; la.K = d;
+            la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = Lw.mlp_norm; la.ybase = nullptr;
+            la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
+            if ((rc = linear(la)) != FE_OK) return rc;
+            la.W = Lw.w_down; la.M = d; la.K = F;
+            la.pro = PRO_F32; la.x = h->act; la.ldx = F;
+            la.epi = EPI_RESID; la.y = h->x; la.ldy = d;
+            if ((rc = linear(la)) != FE_OK) return rc;
+        }
+    }
+    return FE_OK;
+}
+
 bool forward_args_ok(const fe_handle* h, const fe_forward_args* a) {
     if (!h || !a) return false;
     const fe_config& c = h->cfg;
@@ -550,6 +632,9 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
 
         // ---- scratch ----
         const size_t B = c.max_batch, d = c.d, F = c.ffn, H = c.n_heads, hd = c.head_dim;
+        // rows of the per-row work buffers: a draft's B, or a commit block's up to 32
+        const size_t Rw = std::max<size_t>(B, std::min<size_t>(32, B * (size_t)std::max(1, c.n_layers)));
+        const int Rmma = (int)std::min<size_t>(32, Rw);
         const size_t nqkv = (size_t)(c.n_heads + 2 * c.n_kv_heads) * hd;
         h->attn_split_rows = attn_split(c.max_batch, c.n_kv_heads, c.max_seq, h->dev);
         h->attn_nsplit = (c.max_seq + h->attn_split_rows - 1) / h->attn_split_rows;
@@ -558,11 +643,11 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         const size_t k = c.top_k_max;
         const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
         const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
-        size_t off[20], n = 0, tot = 0;
-        const size_t bytes[20] = {
+        size_t off[22], n = 0, tot = 0;
+        const size_t bytes[22] = {
             cs.size() * sizeof(float),                             // rope
-            B * d * 4, B * d * 4, B * nqkv * 4, B * H * hd * 4,   // g, x, qkv, o
-            B * F * 4, R * d * 4,                                  // act, hid
+            Rw * d * 4, Rw * d * 4, Rw * nqkv * 4, Rw * H * hd * 4,   // g, x, qkv, o
+            Rw * F * 4, R * d * 4,                                  // act, hid
             B * H * h->attn_nsplit * (hd + 2) * 4,                 // attention partials
             R * h->lm_slabs * k * 4, R * h->lm_slabs * k * 4,      // LM-head partial ids, values
             R * h->lm_slabs * 2 * 4,                               // LM-head partial (max, sum)
@@ -571,12 +656,14 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             R * 4,                                                 // LM-head slab counters
             h->lm_mma ? std::max(lmhead_mma_zb_bytes((int)std::min<size_t>(R, 16), c.d),
                                  lmhead_wide_zb_bytes((int)R, c.d)) : 0,  // tensor-core LM-head operand
-            h->lin_mma ? linear_mma_xb_bytes((int)kmax, c.max_batch) : 0,  // tensor-core linear operand
-            h->lin_mma ? linear_mma_part_bytes(c.max_batch, h->dev) : 0,   // its split-tile partials
+            h->lin_mma ? linear_mma_xb_bytes((int)kmax, std::max(c.max_batch, Rmma)) : 0,  // tensor-core linear operand
+            h->lin_mma ? linear_mma_part_bytes(std::max(c.max_batch, Rmma), h->dev) : 0,   // its split-tile partials
             h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0,      // its completion counters
             h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0,  // stack barrier counters
-            B * d * 4};                                                       // x0
-        for (n = 0; n < 20; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            Rw * d * 4,                                                       // x0
+            Rw * 3 * d * h->es,                                               // commit: gathered features
+            Rw * sizeof(int)};                                                // commit: gathered tokens
+        for (n = 0; n < 22; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -599,6 +686,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->lin_counters = h->lin_mma ? (int*)(s + off[17]) : nullptr;
         h->stack_bar = h->use_stack ? (uint32_t*)(s + off[18]) : nullptr;
         h->x0 = (float*)(s + off[19]);
+        h->cfeat = s + off[20];
+        h->ctok = (int*)(s + off[21]);
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
@@ -717,6 +806,22 @@ fe_status fe_verify_greedy(fe_handle* h, int32_t B, int32_t top_k, const int32_t
     FE_TRY(launch_verify(B, T, N, prefix_len, tree->tok, tree->parent, tree->depth, target_next, pos_ids, path,
                          n_accept, bonus, (cudaStream_t)stream));
     return FE_OK;
+}
+
+fe_status fe_commit(fe_handle* h, const fe_commit_args* a, void* stream) {
+    if (!h || !a) return FE_ERR_INVALID_ARG;
+    const fe_config& c = h->cfg;
+    if (a->B < 1 || a->B > c.max_batch || a->L < 1 || a->L > c.n_layers) return FE_ERR_INVALID_ARG;
+    if (!a->feat || !a->tok || !a->n_rows || !a->prefix_len || !a->k_cache || !a->v_cache) return FE_ERR_INVALID_ARG;
+    for (int i = 0; i < c.n_layers; ++i)
+        if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
+    if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(a->feat) & 15) return FE_ERR_INVALID_ARG;  // copied as 16-byte vectors
+    try {
+        return enqueue_commit(h, a, (cudaStream_t)stream);
+    } catch (...) {
+        return FE_ERR_OOM;
+    }
 }
 
 fe_status fe_last_device_status(fe_handle* h, void* stream) {
