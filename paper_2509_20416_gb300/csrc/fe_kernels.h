@@ -153,9 +153,10 @@ size_t lmhead_mma_zb_bytes(int R, int d);
 size_t mma_packed_bytes(int M, int K);
 cudaError_t launch_pack_mma(const void* src, void* dst, int M, int K, cudaStream_t st);
 cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);
-// after_prep (optional): an event recorded on st between the two kernels it launches
+// Three kernels: operand prep, the product with per-slab statistics and top-k, the per-row
+// merge; after_prep / after_main (optional): events recorded on st after the first two
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
-                              cudaEvent_t after_prep = nullptr);
+                              cudaEvent_t after_prep = nullptr, cudaEvent_t after_main = nullptr);
 
 // wide tensor-core LM head (bf16, 16 < R <= 256 rows, top_k <= 16, d % 64 == 0): the same
 // packed W, z rounded to bf16 (zb of lmhead_wide_zb_bytes()), n_slabs = lmhead_wide_slabs()

@@ -649,16 +649,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             }
         }
     }
-    // ---- the last CTA merges every row
-    griddep_wait();  // (already satisfied: the producer waited; makes the order explicit for all threads)
-    __threadfence();
-    __syncthreads();
-    if (t == 0) st.last = atomicAdd(&a.counters[0], 1) == (int)gridDim.x - 1;
-    __syncthreads();
-    if (!st.last) return;
-    __threadfence();
-    merge_rows(a, 0, R, ring, (size_t)S * stage_bytes);
-    if (t == 0) a.counters[0] = 0;
+    // (lmhead_merge_kernel, one CTA per row, merges the slabs)
 }
 
 // ---- host side ----------------------------------------------------------------------------
@@ -741,13 +732,17 @@ size_t lmhead_mma_zb_bytes(int R, int d) {
     return (size_t)2 * R_pad * d * 2;
 }
 
+__global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, size_t smem_bytes);
+
 cudaError_t lmhead_mma_prepare(const DeviceInfo& dev) {
-    return cudaFuncSetAttribute(lmhead_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                dev.max_smem_optin - (int)sizeof(MmaState) - 256);
+    const cudaError_t e = cudaFuncSetAttribute(lmhead_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               dev.max_smem_optin - (int)sizeof(MmaState) - 256);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
 }
 
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
-                              cudaEvent_t after_prep) {
+                              cudaEvent_t after_prep, cudaEvent_t after_main) {
     if (!lmhead_mma_ok(a) || (reinterpret_cast<uintptr_t>(a.hid) & 15)) return cudaErrorInvalidValue;
     const int R_pad = (a.R + 7) / 8 * 8;
     const int N = 2 * R_pad;
@@ -764,12 +759,17 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     int S = (int)((budget - 1024 - slab_bytes) / stage_bytes);
     S = S > kMmaMaxStages ? kMmaMaxStages : S;
     if (S < 2) return cudaErrorInvalidValue;
-    if ((size_t)S * stage_bytes < merge_smem_bytes(kMmaThreads / 32, a.n_slabs, a.top_k)) return cudaErrorInvalidValue;
+    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k);
+    if (msmem > 64 * 1024) return cudaErrorInvalidValue;
     const size_t smem = 1024 + (size_t)S * stage_bytes + slab_bytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
-    return launch_k(lmhead_mma_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb,
-                    R_pad, S, stage_bytes, cols, slab_cap);
+    e = launch_k(lmhead_mma_kernel, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb,
+                 R_pad, S, stage_bytes, cols, slab_cap);
+    if (e != cudaSuccess) return e;
+    if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;
+    // one CTA per row merges the slabs (a last-CTA merge would hold every row on one SM)
+    return launch_k(lmhead_merge_kernel, dim3(a.R), dim3(128), msmem, st, a.pdl, a, msmem);
 }
 
 

@@ -298,11 +298,13 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     if (h->lm_mma && N * B <= 16) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         if (pf) {
-            if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
+            if (pf->n + 3 > pf->cap) return FE_ERR_INVALID_ARG;
             pf->kinds[pf->n] = FE_KERNEL_LM_PREP;
-            ++pf->n;
+            pf->kinds[pf->n + 1] = FE_KERNEL_LM_HEAD;
+            pf->n += 2;
         }
-        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n] : nullptr));
+        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n - 1] : nullptr,
+                                 pf ? pf->ev[pf->n] : nullptr));
         FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     } else if (h->lm_mma) {
         lm.n_slabs = lmhead_wide_slabs(V, h->dev);
@@ -852,7 +854,7 @@ int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     // stacked: N + 1 stack launches hold all linear phases
     const int lin_total = (h->use_stack && B == 1) ? N + 1 : 2 * lin + N * 4 * lin;
     int n = lin_total + N * attention_launches() +
-            (h->lm_mma ? (N * B <= 16 ? 2 : 3) : lmhead_launches(N * B, h->cfg.d, h->dev));
+            (h->lm_mma ? 3 : lmhead_launches(N * B, h->cfg.d, h->dev));
     return n + (with_tree ? 1 : 0);
 }
 
