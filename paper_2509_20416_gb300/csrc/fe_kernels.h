@@ -76,6 +76,7 @@ struct LinearArgs {
     float* y2;
     int ldy2;
     const float* ybase;  // EPI_RESID: y = ybase + acc (same layout as y) when set, else y += acc
+    int slots;           // streaming kernel: pipeline slots per warp (0: the default)
     int* status;
     bool pdl;  // launch overlapping the previous kernel (programmatic dependent launch)
 };

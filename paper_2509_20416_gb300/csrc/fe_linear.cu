@@ -117,7 +117,9 @@ __global__ void __launch_bounds__(kStreamThreads, 1) stack_kernel(const StackArg
 namespace {
 
 constexpr size_t kXBudget = 128 * 1024;  // activations held in shared memory per CTA
-constexpr int kPreferredSlots = 2;       // per-warp pipeline depth (2 x 8 KB measured best)
+// Per-warp pipeline depth: three 8 KB slots where shared memory allows (more bytes in flight
+// per SM), two next to attention (its CTAs start early on the same SMs and need the room).
+constexpr int kPreferredSlots = 3;
 
 template <typename WT, int BT>
 cudaError_t set_attr(const DeviceInfo& dev) {
@@ -137,7 +139,8 @@ cudaError_t launch_bt(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t s
     const int Kpad = (a.K + 3) & ~3;
     const int xrows = BT < a.B ? BT : a.B;
     int D = stream_slots((size_t)dev.max_smem_optin, stream_smem_bytes(0, xrows, Kpad, BT));
-    D = D > kPreferredSlots ? kPreferredSlots : D;
+    const int pref = a.slots > 0 ? a.slots : kPreferredSlots;
+    D = D > pref ? pref : D;
     if (D < 1) return cudaErrorInvalidValue;
     const size_t smem = stream_smem_bytes(D, xrows, Kpad, BT);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;

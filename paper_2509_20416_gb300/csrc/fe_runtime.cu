@@ -168,6 +168,12 @@ Sizes weight_sizes(const fe_config& c, size_t es, bool mma) {
     return s;
 }
 
+// Pipeline slots of a streaming linear phase next to attention: 3 (the default) for a matrix
+// of 64 MB or more, whose stream outlasts attention's early start; 2 for a smaller one, so
+// that attention's CTAs fit beside it on the SMs (measured on the LLaMA-3.1-8B and
+// Vicuna-13B shapes).
+int near_attention_slots(int M, int K, int es) { return (size_t)M * K * es >= ((size_t)64 << 20) ? 0 : 2; }
+
 fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t st, Prof* pf = nullptr) {
     const fe_config& c = h->cfg;
     const int B = a->B, d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
@@ -259,6 +265,8 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         const LayerPacked& L = h->layers[i];
         // qkv = W_qkv RMSNorm(x)
         la.W = L.w_qkv; la.M = nqkv; la.K = d;
+        // the phases next to attention leave room for its CTAs unless they are large
+        la.slots = near_attention_slots(nqkv, d, (int)h->es);
         // L_1 (and every L_i of the parallel ablation) reads x0; the cascade's L_i reads h_{i-1}
         const bool from_x0 = i == 0 || c.parallel_layers;
         la.pro = PRO_RMSNORM; la.x = from_x0 ? h->x0 : h->x; la.ldx = d; la.gamma = L.attn_norm;
@@ -270,11 +278,13 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         FE_TRY(launch_attention(dt, aa, st));
         FE_TRY(mark(pf, FE_KERNEL_ATTENTION, st));
         // x += W_o o
+        la.slots = near_attention_slots(d, H * hd, (int)h->es);
         la.W = L.w_o; la.M = d; la.K = H * hd;
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr; la.ybase = from_x0 ? h->x0 : nullptr;
         FE_LINEAR(la);
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
+        la.slots = 0;
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm; la.ybase = nullptr;
         la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
