@@ -55,8 +55,8 @@ TRAFFIC = {
     #     -k regex:linear_kernel -s 18 -c 6 on `bench.py --set n_layers=1` (one draft's six
     # linear launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down); the five-layer draft
     # repeats the four per-layer launches five times with the same shapes.
-    "vic13b": {"bytes_per_draft": 160970496 + 105212928 + 5 * (157469184 + 52540416 + 283366656 + 141993728),
-               "src": "e09fe4eab8f4c523"},
+    "vic13b": {"bytes_per_draft": 160356608 + 105004032 + 5 * (157437696 + 52540928 + 283344384 + 141732352),
+               "src": "66b1fbb81a51953f"},
 }
 KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
 

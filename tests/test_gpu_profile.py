@@ -12,7 +12,11 @@ pytestmark = pytest.mark.gpu
 @pytest.mark.parametrize("spec", [dict(name="tiny"),
                                   dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376,
                                                  vocab=5003, n_layers=3, dtype="bf16", B=2, prefix=40, top_k=8,
-                                                 rope_theta=1e4, seed=41, page_size=0))])
+                                                 rope_theta=1e4, seed=41, page_size=0)),
+                                  # batched: tensor-core linear phases (operand prep + product)
+                                  dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1408,
+                                                 vocab=5003, n_layers=3, dtype="bf16", B=12, prefix=40, top_k=8,
+                                                 rope_theta=1e4, seed=42, page_size=0))])
 def test_profile_forward_matches_forward(spec):
     import paper_2509_20416_gb300 as fe
     cfg = wl.make_config(spec["name"])
@@ -38,6 +42,9 @@ def test_profile_forward_matches_forward(spec):
     n_lin = kinds.count("linear")
     assert n_lin in (2 + 4 * N, N + 1)
     assert all(kinds[j - 1] == "linear" for j in att)
-    assert kinds[0] == "linear" and kinds[-1] == "lm_head"
+    if cfg["B"] > 8:  # every tensor-core phase: its operand prep right before it
+        assert kinds.count("linear_prep") == n_lin
+        assert all(kinds[j + 1] == "linear" for j, kd in enumerate(kinds) if kd == "linear_prep")
+    assert kinds[0] in ("linear", "linear_prep") and kinds[-1] == "lm_head"
     assert all(us > 0 for _, us in prof)
     h.close()
