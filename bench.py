@@ -268,23 +268,18 @@ def main():
         raise SystemExit(f"device status after the timed region: {fe.fe_status_str(st)}")
 
     # ---- end to end through the public API with host buffers ------------------------------
-    pin = {n: t.pin_memory() for n, t in (("feat", I["feat"]), ("tok", I["next_tok"]),
-                                          ("plen", I["prefix_len"]))}
-    host_out = {n: torch.empty_like(t, device="cpu").pin_memory() for n, t in out.items()}
-    host_tree = {n: torch.empty_like(t, device="cpu").pin_memory() for n, t in tree.items()}
-    h2d = sum(t.numel() * t.element_size() for t in pin.values())
-    d2h = sum(t.numel() * t.element_size() for t in list(out.values()) + list(tree.values()))
+    # fe_draft_step_host: host inputs -> (pinned staging -> device copy, draft, tree, device
+    # -> pinned copy, as one CUDA graph) -> host outputs; the call returns with the outputs
+    # in host memory
+    host_in = {n: t.contiguous().pin_memory() for n, t in (("feat", I["feat"]), ("tok", I["next_tok"]),
+                                                           ("plen", I["prefix_len"]))}
+    host_out = fe.alloc_host_step_outputs(h, B, k)
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
 
     def e2e_step():
-        feat.copy_(pin["feat"], non_blocking=True)
-        tok.copy_(pin["tok"], non_blocking=True)
-        plen.copy_(pin["plen"], non_blocking=True)
-        step()
-        for n, t in out.items():
-            host_out[n].copy_(t, non_blocking=True)
-        for n, t in tree.items():
-            host_tree[n].copy_(t, non_blocking=True)
-        stream.synchronize()
+        fe.fe_draft_step_host(h, host_in["feat"], host_in["tok"], host_in["plen"], kd, vd, k, cfg["temperature"],
+                              page_table=table, n_pages=n_pages, out=host_out, stream=stream)
 
     for _ in range(3):
         e2e_step()
@@ -410,7 +405,9 @@ def main():
                            "note": "fe_draft_loss: the draft with logits [B,N,V] and hidden states written out, "
                                    "then CE + Smooth L1 (Sec. 2.3); outside the timed step"},
             "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
+                    "d2h_bytes_per_step": d2h,
+                    "call": "fe_draft_step_host (host inputs and outputs; copies, draft and tree in one graph; "
+                            "returns with the outputs in host memory)"},
             "gpu_launches": launches * args.steps, "launches_per_step": launches,
             "clocks": clocks}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:

@@ -164,6 +164,42 @@ FE_API fe_status fe_draft_forward(fe_handle *h, const fe_forward_args *args, voi
 FE_API fe_status fe_build_tree(fe_handle *h, int32_t B, int32_t top_k, const int32_t *next_tok,
                         const int32_t *topk_id, fe_tree *out, void *stream);
 
+/* One draft step from and to HOST memory (Sec. 2.4, the drafting step of the cycle): the
+ * step's inputs go to the device, fe_draft_forward and fe_build_tree run, and the outputs
+ * come back, all as one CUDA graph per argument set (the copies are graph nodes between the
+ * handle's pinned staging buffers and its device buffers), so a step costs one launch.
+ *
+ *  feat [B, 3d] dtype, next_tok [B] int32, prefix_len [B] int32: HOST inputs, as in
+ *    fe_forward_args (any host memory; copied into the handle's pinned staging before the
+ *    launch, except page-locked features at a 16-byte boundary, which the graph copies
+ *    from directly: keep such a buffer's address across calls to replay the graph)
+ *  k_cache, v_cache, page_table, n_pages, top_k, temperature: as in fe_forward_args
+ *    (the caches and the page table stay in device memory)
+ *  topk_id [B, N, top_k] int32, topk_logit, topk_prob [B, N, top_k] float32, lse [B, N]
+ *    float32, tree_tok, tree_parent, tree_depth [B, T] int32, tree_mask [B, T, T] uint8
+ *    (T = 1 + N top_k): HOST outputs, as fe_draft_forward and fe_build_tree define them
+ *
+ * The call synchronises `stream` and returns once the outputs are in host memory. Errors:
+ * FE_ERR_INVALID_ARG (null pointer, B or top_k out of range), FE_ERR_CUDA / FE_ERR_OOM;
+ * device-side conditions are reported by fe_last_device_status as for fe_draft_forward. */
+typedef struct {
+    int32_t B, top_k;
+    float temperature;
+    const void *feat;
+    const int32_t *next_tok;
+    const int32_t *prefix_len;
+    void *const *k_cache;
+    void *const *v_cache;
+    const int32_t *page_table;
+    int32_t n_pages;
+    int32_t *topk_id;
+    float *topk_logit, *topk_prob, *lse;
+    int32_t *tree_tok, *tree_parent, *tree_depth;
+    uint8_t *tree_mask;
+} fe_host_step_args;
+
+FE_API fe_status fe_draft_step_host(fe_handle *h, const fe_host_step_args *args, void *stream);
+
 /* Synchronise `stream`, return and clear the handle's device status word
  * (FE_OK, FE_ERR_CAPACITY, FE_ERR_DEVICE or FE_ERR_TIMEOUT). */
 FE_API fe_status fe_last_device_status(fe_handle *h, void *stream);

@@ -67,6 +67,13 @@ class fe_commit_args(ctypes.Structure):
                 ("page_table", _vp), ("n_pages", _i32)]
 
 
+class fe_host_step_args(ctypes.Structure):
+    _fields_ = [("B", _i32), ("top_k", _i32), ("temperature", ctypes.c_float), ("feat", _vp), ("next_tok", _vp),
+                ("prefix_len", _vp), ("k_cache", ctypes.POINTER(_vp)), ("v_cache", ctypes.POINTER(_vp)),
+                ("page_table", _vp), ("n_pages", _i32), ("topk_id", _vp), ("topk_logit", _vp), ("topk_prob", _vp),
+                ("lse", _vp), ("tree_tok", _vp), ("tree_parent", _vp), ("tree_depth", _vp), ("tree_mask", _vp)]
+
+
 _lib.fe_draft_init.argtypes = [ctypes.POINTER(fe_config), ctypes.POINTER(fe_weights), _vp, ctypes.POINTER(_vp)]
 _lib.fe_draft_init.restype = ctypes.c_int
 _lib.fe_draft_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp]
@@ -92,6 +99,8 @@ _lib.fe_draft_loss.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, c
 _lib.fe_draft_loss.restype = ctypes.c_int
 _lib.fe_verify_greedy.argtypes = [_vp, _i32, _i32, _vp, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp]
 _lib.fe_verify_greedy.restype = ctypes.c_int
+_lib.fe_draft_step_host.argtypes = [_vp, ctypes.POINTER(fe_host_step_args), _vp]
+_lib.fe_draft_step_host.restype = ctypes.c_int
 _lib.fe_commit.argtypes = [_vp, ctypes.POINTER(fe_commit_args), _vp]
 _lib.fe_commit.restype = ctypes.c_int
 _lib.fe_last_error_detail.argtypes = []
@@ -265,6 +274,40 @@ def fe_build_tree(h: Handle, next_tok, topk_id, top_k: int, out: dict | None = N
     t = fe_tree(_p(out["tok"]), _p(out["parent"]), _p(out["depth"]), _p(out["mask"]))
     _check(_lib.fe_build_tree(h.ptr, B, top_k, _p(next_tok), _p(topk_id), ctypes.byref(t), _stream(stream)),
            "fe_build_tree")
+    return out
+
+
+def alloc_host_step_outputs(h: Handle, B: int, top_k: int) -> dict:
+    """Host (pinned) tensors for fe_draft_step_host's outputs."""
+    N = h.cfg["n_layers"]
+    T = 1 + N * top_k
+    e = lambda shape, dt: torch.empty(shape, dtype=dt).pin_memory()
+    return dict(topk_id=e((B, N, top_k), torch.int32), topk_logit=e((B, N, top_k), torch.float32),
+                topk_prob=e((B, N, top_k), torch.float32), lse=e((B, N), torch.float32),
+                tree_tok=e((B, T), torch.int32), tree_parent=e((B, T), torch.int32), tree_depth=e((B, T), torch.int32),
+                tree_mask=e((B, T, T), torch.uint8))
+
+
+def fe_draft_step_host(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int, temperature: float = 0.0,
+                       page_table=None, n_pages: int = 0, out: dict | None = None, stream=None) -> dict:
+    """One draft step from and to host memory (include/fe_draft.h): feat [B, 3d], next_tok
+    [B], prefix_len [B] are CPU tensors; the caches (and page table) are device tensors.
+    Returns CPU tensors topk_id, topk_logit, topk_prob, lse, tree_tok, tree_parent,
+    tree_depth, tree_mask."""
+    for t in (feat, next_tok, prefix_len):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError("fe_draft_step_host takes contiguous host tensors")
+    B = int(next_tok.shape[0])
+    if out is None:
+        out = alloc_host_step_outputs(h, B, top_k)
+    N = h.cfg["n_layers"]
+    kc = (_vp * N)(*[_p(t) for t in k_cache])
+    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    a = fe_host_step_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
+                          _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
+                          _p(out["topk_prob"]), _p(out["lse"]), _p(out["tree_tok"]), _p(out["tree_parent"]),
+                          _p(out["tree_depth"]), _p(out["tree_mask"]))
+    _check(_lib.fe_draft_step_host(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_step_host")
     return out
 
 

@@ -47,6 +47,50 @@ struct GraphKey {
     }
 };
 
+// what a fe_draft_step_host graph was captured for
+struct HostKey {
+    int B = 0, top_k = 0;
+    float temperature = 0.f;
+    const void* feat_direct = nullptr;  // the caller's pinned features, copied from directly
+    const int32_t* page_table = nullptr;
+    int n_pages = 0;
+    std::vector<void*> kc, vc;
+    bool operator==(const HostKey& o) const {
+        return B == o.B && top_k == o.top_k && temperature == o.temperature && feat_direct == o.feat_direct &&
+               page_table == o.page_table &&
+               n_pages == o.n_pages && kc == o.kc && vc == o.vc;
+    }
+};
+
+// fe_draft_step_host's packing of one step's inputs and outputs (16-byte aligned pieces),
+// the same in the pinned staging buffers and in their device copies
+struct StepLayout {
+    size_t feat, tok, plen, in_bytes;
+    size_t id, logit, prob, lse, ttok, tpar, tdep, tmask, out_bytes;
+};
+
+StepLayout step_layout(const fe_config& c, size_t es, int B, int k) {
+    auto al = [](size_t x) { return (x + 15) & ~(size_t)15; };
+    const size_t b = (size_t)B, N = (size_t)c.n_layers, T = 1 + N * (size_t)k;
+    StepLayout L{};
+    size_t o = 0;
+    L.feat = o; o = al(o + b * 3 * (size_t)c.d * es);
+    L.tok = o; o = al(o + b * 4);
+    L.plen = o; o = al(o + b * 4);
+    L.in_bytes = o;
+    o = 0;
+    L.id = o; o = al(o + b * N * k * 4);
+    L.logit = o; o = al(o + b * N * k * 4);
+    L.prob = o; o = al(o + b * N * k * 4);
+    L.lse = o; o = al(o + b * N * 4);
+    L.ttok = o; o = al(o + b * T * 4);
+    L.tpar = o; o = al(o + b * T * 4);
+    L.tdep = o; o = al(o + b * T * 4);
+    L.tmask = o; o = al(o + b * T * T);
+    L.out_bytes = o;
+    return L;
+}
+
 }  // namespace
 
 struct fe_handle {
@@ -84,6 +128,11 @@ struct fe_handle {
     bool use_graph = true;
     bool use_pdl = true;
     std::vector<cudaEvent_t> prof_ev;  // fe_profile_forward's events (created on first use)
+    // fe_draft_step_host: pinned staging of a step's inputs and outputs, their device
+    // copies (sized for max_batch and top_k_max) and the step's graph
+    unsigned char *hs_in = nullptr, *hs_out = nullptr, *ds_in = nullptr, *ds_out = nullptr;
+    cudaGraphExec_t hexec = nullptr;
+    HostKey hkey;
 };
 
 namespace {
@@ -439,6 +488,11 @@ void release(fe_handle* h) {
     if (!h) return;
     for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    if (h->hexec) cudaGraphExecDestroy(h->hexec);
+    if (h->hs_in) cudaFreeHost(h->hs_in);
+    if (h->hs_out) cudaFreeHost(h->hs_out);
+    if (h->ds_in) cudaFree(h->ds_in);
+    if (h->ds_out) cudaFree(h->ds_out);
     if (h->cap) cudaStreamDestroy(h->cap);
     if (h->wbuf) cudaFree(h->wbuf);
     if (h->sbuf) cudaFree(h->sbuf);
@@ -706,6 +760,13 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, off[13] + bytes[13] - off[11], st))) != FE_OK) break;
         if (h->lin_mma && (rc = from_cuda(cudaMemsetAsync(h->lin_counters, 0, bytes[17], st))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking))) != FE_OK) break;
+        {  // fe_draft_step_host's staging (pinned) and device buffers
+            const StepLayout L = step_layout(c, h->es, c.max_batch, c.top_k_max);
+            if ((rc = from_cuda(cudaMallocHost((void**)&h->hs_in, L.in_bytes))) != FE_OK) break;
+            if ((rc = from_cuda(cudaMallocHost((void**)&h->hs_out, L.out_bytes))) != FE_OK) break;
+            if ((rc = from_cuda(cudaMalloc((void**)&h->ds_in, L.in_bytes))) != FE_OK) break;
+            if ((rc = from_cuda(cudaMalloc((void**)&h->ds_out, L.out_bytes))) != FE_OK) break;
+        }
         if ((rc = from_cuda(cudaStreamSynchronize(st))) != FE_OK) break;
     } while (0);
     if (rc != FE_OK) {
@@ -782,6 +843,111 @@ fe_status fe_profile_forward(fe_handle* h, const fe_forward_args* a, void* strea
     } catch (...) {
         return FE_ERR_OOM;
     }
+}
+
+namespace {
+
+// the device work of one fe_draft_step_host call: inputs in, draft, tree, outputs out
+// (feat_direct: the caller's features are page-locked and copied from where they are; the
+// staging then holds only the tokens and prefix lengths)
+fe_status enqueue_host_step(fe_handle* h, const fe_host_step_args* a, const StepLayout& L, bool feat_direct,
+                            cudaStream_t st) {
+    const fe_config& c = h->cfg;
+    if (feat_direct) {
+        FE_TRY(cudaMemcpyAsync(h->ds_in + L.feat, a->feat, (size_t)a->B * 3 * c.d * h->es, cudaMemcpyHostToDevice, st));
+        FE_TRY(cudaMemcpyAsync(h->ds_in + L.tok, h->hs_in + L.tok, L.in_bytes - L.tok, cudaMemcpyHostToDevice, st));
+    } else {
+        FE_TRY(cudaMemcpyAsync(h->ds_in, h->hs_in, L.in_bytes, cudaMemcpyHostToDevice, st));
+    }
+    fe_forward_args fa{};
+    fa.B = a->B; fa.top_k = a->top_k; fa.temperature = a->temperature;
+    fa.feat = h->ds_in + L.feat;
+    fa.next_tok = reinterpret_cast<const int32_t*>(h->ds_in + L.tok);
+    fa.prefix_len = reinterpret_cast<const int32_t*>(h->ds_in + L.plen);
+    fa.k_cache = a->k_cache; fa.v_cache = a->v_cache; fa.page_table = a->page_table; fa.n_pages = a->n_pages;
+    fa.topk_id = reinterpret_cast<int32_t*>(h->ds_out + L.id);
+    fa.topk_logit = reinterpret_cast<float*>(h->ds_out + L.logit);
+    fa.topk_prob = reinterpret_cast<float*>(h->ds_out + L.prob);
+    fa.lse = reinterpret_cast<float*>(h->ds_out + L.lse);
+    if (!forward_args_ok(h, &fa)) return FE_ERR_INVALID_ARG;
+    const fe_status rc = enqueue_forward(h, &fa, st);
+    if (rc != FE_OK) return rc;
+    FE_TRY(launch_tree(a->B, c.n_layers, a->top_k, c.vocab, fa.next_tok, fa.topk_id,
+                       reinterpret_cast<int32_t*>(h->ds_out + L.ttok), reinterpret_cast<int32_t*>(h->ds_out + L.tpar),
+                       reinterpret_cast<int32_t*>(h->ds_out + L.tdep), h->ds_out + L.tmask, h->status, st));
+    FE_TRY(cudaMemcpyAsync(h->hs_out, h->ds_out, L.out_bytes, cudaMemcpyDeviceToHost, st));
+    return FE_OK;
+}
+
+}  // namespace
+
+fe_status fe_draft_step_host(fe_handle* h, const fe_host_step_args* a, void* stream) {
+    if (!h || !a) return FE_ERR_INVALID_ARG;
+    const fe_config& c = h->cfg;
+    if (a->B < 1 || a->B > c.max_batch || a->top_k < 1 || a->top_k > c.top_k_max) return FE_ERR_INVALID_ARG;
+    if (!a->feat || !a->next_tok || !a->prefix_len || !a->k_cache || !a->v_cache || !a->topk_id || !a->topk_logit ||
+        !a->topk_prob || !a->lse || !a->tree_tok || !a->tree_parent || !a->tree_depth || !a->tree_mask)
+        return FE_ERR_INVALID_ARG;
+    for (int i = 0; i < c.n_layers; ++i)
+        if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
+    if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
+    if (!(a->temperature == a->temperature)) return FE_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    const StepLayout L = step_layout(c, h->es, a->B, a->top_k);
+    const size_t B = (size_t)a->B, N = (size_t)c.n_layers, k = (size_t)a->top_k, T = 1 + N * k;
+    // page-locked features (e.g. the caller's own pinned buffer) need no staging copy
+    cudaPointerAttributes pa{};
+    const bool feat_direct = cudaPointerGetAttributes(&pa, a->feat) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+                             (reinterpret_cast<uintptr_t>(a->feat) & 15) == 0;
+    cudaGetLastError();  // (an unregistered pointer may leave an error behind on older runtimes)
+    // (the previous call synchronised its stream: the staging buffers are free)
+    if (!feat_direct) memcpy(h->hs_in + L.feat, a->feat, B * 3 * (size_t)c.d * h->es);
+    memcpy(h->hs_in + L.tok, a->next_tok, B * 4);
+    memcpy(h->hs_in + L.plen, a->prefix_len, B * 4);
+    try {
+        if (!h->use_graph) {
+            const fe_status rc = enqueue_host_step(h, a, L, feat_direct, st);
+            if (rc != FE_OK) return rc;
+        } else {
+            HostKey key;
+            key.B = a->B; key.top_k = a->top_k; key.temperature = a->temperature;
+            key.feat_direct = feat_direct ? a->feat : nullptr;
+            key.page_table = a->page_table; key.n_pages = a->n_pages;
+            key.kc.assign(a->k_cache, a->k_cache + c.n_layers);
+            key.vc.assign(a->v_cache, a->v_cache + c.n_layers);
+            if (!h->hexec || !(key == h->hkey)) {
+                cudaGraph_t graph = nullptr;
+                FE_TRY(cudaStreamBeginCapture(h->cap, cudaStreamCaptureModeThreadLocal));
+                const fe_status rc = enqueue_host_step(h, a, L, feat_direct, h->cap);
+                cudaError_t e = cudaStreamEndCapture(h->cap, &graph);
+                if (rc != FE_OK) {
+                    if (graph) cudaGraphDestroy(graph);
+                    return rc;
+                }
+                FE_TRY(e);
+                cudaGraphExec_t ex = nullptr;
+                e = cudaGraphInstantiate(&ex, graph, 0);
+                cudaGraphDestroy(graph);
+                FE_TRY(e);
+                if (h->hexec) cudaGraphExecDestroy(h->hexec);
+                h->hexec = ex;
+                h->hkey = key;
+            }
+            FE_TRY(cudaGraphLaunch(h->hexec, st));
+        }
+        FE_TRY(cudaStreamSynchronize(st));
+    } catch (...) {
+        return FE_ERR_OOM;
+    }
+    memcpy(a->topk_id, h->hs_out + L.id, B * N * k * 4);
+    memcpy(a->topk_logit, h->hs_out + L.logit, B * N * k * 4);
+    memcpy(a->topk_prob, h->hs_out + L.prob, B * N * k * 4);
+    memcpy(a->lse, h->hs_out + L.lse, B * N * 4);
+    memcpy(a->tree_tok, h->hs_out + L.ttok, B * T * 4);
+    memcpy(a->tree_parent, h->hs_out + L.tpar, B * T * 4);
+    memcpy(a->tree_depth, h->hs_out + L.tdep, B * T * 4);
+    memcpy(a->tree_mask, h->hs_out + L.tmask, B * T * T);
+    return FE_OK;
 }
 
 fe_status fe_build_tree(fe_handle* h, int32_t B, int32_t top_k, const int32_t* next_tok, const int32_t* topk_id,

@@ -59,6 +59,7 @@ def test_host_side_validation_needs_no_gpu(lib):
     assert so.fe_build_tree(None, 1, 1, None, None, None, None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_last_device_status(None, None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_commit(None, None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_draft_step_host(None, None, None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_launch_count(None, 1, 1) == -1
     so.fe_free(None)  # no-op
 
