@@ -134,6 +134,12 @@ struct LmHeadArgs {
     float* part_val;   // [R, n_slabs, top_k]
     float* part_ms;    // [R, n_slabs, 2] (max, sum of exp) of logit * inv_temp
     int* counters;     // [ceil(R / 8)] slab-completion counters, zero between calls
+    // tensor-core LM head (N * B <= 16): with these, (vocabulary tile, 64-column block) units
+    // are split evenly over the CTAs; a tile split between CTAs c and c + 1 is finished by c
+    // from c + 1's partial. split_part [n_slabs][128][R_pad] floats; split_flag [n_slabs]
+    // ints, zero between calls. Without them each CTA takes whole tiles.
+    float* split_part;
+    int* split_flag;
     float* dbg_logits; // [B, N, V] or null
     int* topk_id;       // [B, N, k]
     float* topk_logit;  // [B, N, k]
@@ -151,6 +157,7 @@ cudaError_t launch_lmhead(fe_dtype dt, const LmHeadArgs& a, const DeviceInfo& de
 // layout (launch_pack_mma), zb scratch of lmhead_mma_zb_bytes(); n_slabs = CTAs
 bool lmhead_mma_ok(const LmHeadArgs& a);
 size_t lmhead_mma_zb_bytes(int R, int d);
+size_t lmhead_mma_split_bytes(int R, const DeviceInfo& dev);  // split_part
 size_t mma_packed_bytes(int M, int K);
 cudaError_t launch_pack_mma(const void* src, void* dst, int M, int K, cudaStream_t st);
 cudaError_t lmhead_mma_prepare(const DeviceInfo& dev);

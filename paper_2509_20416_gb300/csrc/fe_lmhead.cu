@@ -506,7 +506,7 @@ __global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* 
 }
 
 struct MmaState {
-    uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2];
+    uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2], ebar;
     uint32_t tmem_base;
     int last, abort;
 };
@@ -524,8 +524,22 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     const int N = 2 * R_pad, R = a.R, k = a.top_k;
     const int nkb = a.d / 64;
     const int ntiles = (a.V + 127) / 128;
-    const int t0 = (int)(((int64_t)blockIdx.x * ntiles) / gridDim.x);
-    const int t1 = (int)(((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x);
+    // (tile, 64-column block) units in tile-major order, split evenly over the CTAs (whole
+    // tiles without the split buffers). gridDim.x <= ntiles, so a CTA covers at least nkb
+    // units and a tile is shared by two CTAs at most: a CTA whose range starts inside a
+    // tile computes that tile's second part first and leaves it in split_part (the tile
+    // belongs to the previous CTA, which streams the first part last); a CTA whose range
+    // ends inside a tile owns it and adds the next CTA's part before the epilogue.
+    const int64_t U = (int64_t)ntiles * nkb;
+    const bool stream_k = a.split_part != nullptr;
+    auto ubegin = [&](int c) -> int64_t {
+        return stream_k ? (int64_t)c * U / gridDim.x : ((int64_t)c * ntiles / gridDim.x) * nkb;
+    };
+    const int64_t u0 = ubegin(blockIdx.x), u1 = ubegin(blockIdx.x + 1);
+    const int tf = (int)(u0 / nkb), tl = (int)((u1 - 1) / nkb);  // first and last tile touched
+    const bool head_part = u0 % nkb != 0;  // the first piece is another CTA's tile
+    const bool tail_part = u1 % nkb != 0;  // the last tile's second part comes from CTA + 1
+    const int t0 = head_part ? tf + 1 : tf, t1 = tl + 1;  // the tiles of this slab
 
     if (t == 0) {
         for (int i = 0; i < S; ++i) {
@@ -536,6 +550,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             mbar_init(&st.tfull[i], 1);
             mbar_init(&st.tempty[i], 4);
         }
+        mbar_init(&st.ebar, 4);  // the four epilogue warps (split-tile hand-offs)
         st.abort = 0;
         mbar_fence_init();
     }
@@ -548,27 +563,27 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
     griddep_launch_dependents();
     if (warp == 4) {  // ---- TMA producer
         if (lane == 0) {
-            // the first stages' weight blocks do not depend on the previous kernel (zprep)
-            const int total = (t1 - t0) * nkb;
+            // the first stages' weight blocks do not depend on the previous kernel (zprep);
+            // unit u's weight block sits at u * 16 KB (tile-major packing)
+            const int total = (int)(u1 - u0);
             const int pre = min(S, total);
             for (int it = 0; it < pre; ++it) {
                 mbar_arrive_expect_tx(&st.full[it], 16384u + (uint32_t)N * 128u);
-                const int tile = t0 + it / nkb, kb = it % nkb;
-                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384,
-                         16384, &st.full[it]);
+                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384,
+                         &st.full[it]);
             }
             griddep_wait();
             for (int it = 0; it < pre; ++it)
-                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * N * 128,
-                         (uint32_t)N * 128, &st.full[it]);
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384,
+                         (const unsigned char*)zb + (size_t)((u0 + it) % nkb) * N * 128, (uint32_t)N * 128, &st.full[it]);
             for (int it = pre; it < total; ++it) {
                 const int slot = it % S;
                 const uint32_t u = (uint32_t)(it / S);
                 if (!mbar_wait_abortable(&st.empty[slot], (u & 1u) ^ 1u, a.status, &st.abort)) break;
-                const int tile = t0 + it / nkb, kb = it % nkb;
+                const int kb = (int)((u0 + it) % nkb);
                 unsigned char* dst = ring + (size_t)slot * stage_bytes;
                 mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
-                bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)tile * nkb + kb) * 16384, 16384, &st.full[slot]);
+                bulk_g2s(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot]);
                 bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
                          &st.full[slot]);
             }
@@ -577,13 +592,15 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, N);
             int it = 0;
-            for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
+            int64_t u = u0;
+            for (int tile = tf, j = 0; tile <= tl; ++tile, ++j) {  // one piece (accumulator) per tile
                 const int buf = j & 1;
                 if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * N);
+                const int64_t ue = min(u1, (int64_t)(tile + 1) * nkb);
                 bool ok = true;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                for (bool first = true; u < ue; ++u, ++it, first = false) {
                     const int slot = it % S;
                     if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
                         ok = false;
@@ -594,7 +611,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                     const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + 16384);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)  // K = 16 per MMA: +32 bytes inside the swizzled rows
-                        tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
+                        tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (!first || kk) ? 1u : 0u);
                     tc_commit(&st.empty[slot]);
                 }
                 if (!ok) break;
@@ -602,7 +619,14 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             }
         }
     } else {  // ---- epilogue warps 0..3: TMEM lanes 32 w .. 32 w + 31 = vocabulary rows of the tile
-        for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
+        const int tr = warp * 32 + lane;  // row of the tile
+        uint32_t eb = 0;                  // phases of st.ebar passed
+        auto epi_sync = [&]() -> bool {   // the four epilogue warps; bounded like every wait
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&st.ebar);
+            return mbar_wait_abortable(&st.ebar, (eb++) & 1u, a.status, &st.abort);
+        };
+        for (int tile = tf, j = 0; tile <= tl; ++tile, ++j) {
             const int buf = j & 1;
             if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort, 20000)) break;
             tc_fence_after();
@@ -612,10 +636,49 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&st.tempty[buf]);
-            const int row = j * 128 + warp * 32 + lane;  // row of the slab
-            const int v = tile * 128 + warp * 32 + lane;
+            if (tile == tf && head_part) {  // the previous CTA's tile: leave this part for it
+                float* p = a.split_part + ((size_t)blockIdx.x * 128 + tr) * R_pad;
+#pragma unroll
+                for (int r = 0; r < kMmaMaxRows; r += 4)
+                    if (r < R_pad)
+                        *reinterpret_cast<float4*>(p + r) =
+                            make_float4(acc[r] + acc[R_pad + r], acc[r + 1] + acc[R_pad + r + 1],
+                                        acc[r + 2] + acc[R_pad + r + 2], acc[r + 3] + acc[R_pad + r + 3]);
+                if (!epi_sync()) break;  // the four warps' parts are written
+                if (t == 0) {
+                    __threadfence();
+                    st_release_gpu(a.split_flag + blockIdx.x, 1);
+                }
+                continue;
+            }
+            float add[kMmaMaxRows];  // the next CTA's part of this tile, when it has one
+#pragma unroll
+            for (int r = 0; r < kMmaMaxRows; ++r) add[r] = 0.f;
+            if (tile == tl && tail_part) {
+                if (t == 0) {  // bounded wait for CTA + 1 (resident: it launched before this one could end)
+                    const uint64_t t_0 = globaltimer_ns();
+                    while (ld_acquire_gpu(a.split_flag + blockIdx.x + 1) == 0) {
+                        if ((int64_t)(globaltimer_ns() - t_0) > kWaitBudgetNs) {
+                            atomicOr(a.status, ST_TIMEOUT);
+                            break;
+                        }
+                        __nanosleep(64);
+                    }
+                    a.split_flag[blockIdx.x + 1] = 0;  // (read again only by the next launch)
+                }
+                if (!epi_sync()) break;
+                const float* p = a.split_part + ((size_t)(blockIdx.x + 1) * 128 + tr) * R_pad;
+#pragma unroll
+                for (int r = 0; r < kMmaMaxRows; r += 4)
+                    if (r < R_pad) {
+                        const float4 q = __ldcg(reinterpret_cast<const float4*>(p + r));
+                        add[r] = q.x; add[r + 1] = q.y; add[r + 2] = q.z; add[r + 3] = q.w;
+                    }
+            }
+            const int row = (tile - t0) * 128 + tr;  // row of the slab
+            const int v = tile * 128 + tr;
             for (int r = 0; r < R; ++r) {
-                const float lg = acc[r] + acc[R_pad + r];
+                const float lg = (acc[r] + acc[R_pad + r]) + add[r];
                 slab[(size_t)r * slab_cap + row] = v < a.V ? lg : -INFINITY;
                 if (v < a.V && a.dbg_logits) {
                     const int i = r / a.B, sb = r % a.B;
@@ -753,7 +816,13 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(MmaState) - 256;
     const int ntiles = (a.V + 127) / 128;
-    const int slab_cap = (ntiles + a.n_slabs - 1) / a.n_slabs * 128;  // rows of the largest slab
+    if (a.n_slabs < 1 || a.n_slabs > ntiles || (a.split_part && !a.split_flag)) return cudaErrorInvalidValue;
+    // rows of the largest slab: whole tiles, or (split units) the tiles a range of
+    // ceil(U / n_slabs) units ends in, plus one
+    const int nkb = a.d / 64;
+    const int64_t U = (int64_t)ntiles * nkb;
+    const int slab_cap = (a.split_part ? (int)(((U + a.n_slabs - 1) / a.n_slabs + nkb - 1) / nkb) + 1
+                                       : (ntiles + a.n_slabs - 1) / a.n_slabs) * 128;
     const size_t slab_bytes = (size_t)a.R * slab_cap * sizeof(float);
     if (budget < 1024 + slab_bytes + 2 * (size_t)stage_bytes) return cudaErrorInvalidValue;
     int S = (int)((budget - 1024 - slab_bytes) / stage_bytes);
@@ -1059,6 +1128,10 @@ __global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, s
 bool lmhead_wide_ok(const LmHeadArgs& a) {
     return a.R > 0 && a.R <= kWideRowsMax && a.d % 64 == 0 && a.d <= kZprepMaxChunks * 8 * 256 &&
            a.top_k >= 1 && a.top_k <= kWideKMax;
+}
+
+size_t lmhead_mma_split_bytes(int R, const DeviceInfo& dev) {
+    return (size_t)dev.num_sms * 128 * ((R + 7) / 8 * 8) * sizeof(float);
 }
 
 size_t lmhead_wide_zb_bytes(int R, int d) { return (size_t)((R + 15) / 16 * 16) * d * 2; }

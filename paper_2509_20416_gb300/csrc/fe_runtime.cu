@@ -121,6 +121,8 @@ struct fe_handle {
     bool use_stack = false;      // B = 1 drafts run their linear phases as persistent stacks
     uint32_t* stack_bar = nullptr;  // grid-barrier counters, one per stack of a draft
     uint16_t* lm_zb = nullptr;  // tensor-core LM head: bf16 hi/lo operand of the hidden rows
+    float* lm_split_part = nullptr;  // tensor-core LM head: parts of tiles split between CTAs
+    int* lm_split_flag = nullptr;    // ... and their hand-off flags (zero between calls)
     int attn_split_rows = 0, attn_nsplit = 0, lm_slabs = 0;
     cudaStream_t cap = nullptr;
     cudaGraphExec_t gexec = nullptr;
@@ -356,6 +358,8 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.pdl = pdl;
     if (h->lm_mma && N * B <= 16) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
+        lm.split_part = h->lm_split_part;  // (tile, column block) units split evenly over the CTAs
+        lm.split_flag = h->lm_split_flag;
         if (pf) {
             if (pf->n + 3 > pf->cap) return FE_ERR_INVALID_ARG;
             pf->kinds[pf->n] = FE_KERNEL_LM_PREP;
@@ -709,8 +713,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         const size_t k = c.top_k_max;
         const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
         const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
-        size_t off[22], n = 0, tot = 0;
-        const size_t bytes[22] = {
+        size_t off[24], n = 0, tot = 0;
+        const size_t bytes[24] = {
             cs.size() * sizeof(float),                             // rope
             Rw * d * 4, Rw * d * 4, Rw * nqkv * 4, Rw * H * hd * 4,   // g, x, qkv, o
             Rw * F * 4, R * d * 4,                                  // act, hid
@@ -728,8 +732,10 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0,  // stack barrier counters
             Rw * d * 4,                                                       // x0
             Rw * 3 * d * h->es,                                               // commit: gathered features
-            Rw * sizeof(int)};                                                // commit: gathered tokens
-        for (n = 0; n < 22; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            Rw * sizeof(int),                                                 // commit: gathered tokens
+            h->lm_mma ? lmhead_mma_split_bytes(16, h->dev) : 0,                // LM head: split-tile parts
+            h->lm_mma ? (size_t)h->dev.num_sms * sizeof(int) : 0};            // ... and their flags
+        for (n = 0; n < 24; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -754,11 +760,14 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->x0 = (float*)(s + off[19]);
         h->cfeat = s + off[20];
         h->ctok = (int*)(s + off[21]);
+        h->lm_split_part = h->lm_mma ? (float*)(s + off[22]) : nullptr;
+        h->lm_split_flag = h->lm_mma ? (int*)(s + off[23]) : nullptr;
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
         if ((rc = from_cuda(cudaMemsetAsync(h->status, 0, off[13] + bytes[13] - off[11], st))) != FE_OK) break;
         if (h->lin_mma && (rc = from_cuda(cudaMemsetAsync(h->lin_counters, 0, bytes[17], st))) != FE_OK) break;
+        if (h->lm_mma && (rc = from_cuda(cudaMemsetAsync(h->lm_split_flag, 0, bytes[23], st))) != FE_OK) break;
         if ((rc = from_cuda(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking))) != FE_OK) break;
         {  // fe_draft_step_host's staging (pinned) and device buffers
             const StepLayout L = step_layout(c, h->es, c.max_batch, c.top_k_max);
