@@ -505,6 +505,16 @@ __global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* 
     }
 }
 
+__device__ __forceinline__ void st_release_gpu(int* p, int v) {
+    asm volatile("st.release.gpu.global.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
 struct MmaState {
     uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2], ebar;
     uint32_t tmem_base;
