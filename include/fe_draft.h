@@ -45,7 +45,7 @@ extern "C" {
 typedef enum {
     FE_OK = 0,
     FE_ERR_INVALID_ARG = -1, /* a null pointer, a bad shape or an out-of-range scalar */
-    FE_ERR_UNSUPPORTED = -2, /* a legal shape this build does not implement */
+    FE_ERR_UNSUPPORTED = -2, /* a legal shape the library does not implement */
     FE_ERR_CUDA = -3,        /* a CUDA runtime call failed */
     FE_ERR_OOM = -4,         /* device allocation failed */
     FE_ERR_CAPACITY = -5,    /* a prefix does not fit its cache (P_b + 1 > max_seq) */

@@ -171,7 +171,7 @@ bool valid_config(const fe_config* c) {
     return true;
 }
 
-// legal shapes this build's kernels cover
+// legal shapes the library's kernels cover
 bool supported_config(const fe_config* c) {
     const int G = c->n_heads / c->n_kv_heads;
     if (c->head_dim != 64 && c->head_dim != 128) return false;
