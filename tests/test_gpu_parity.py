@@ -116,6 +116,11 @@ SMALL = {
     "tc_attn_g4_paged24": dict(name=dict(d=512, n_heads=4, n_kv_heads=1, head_dim=128, ffn=1376, vocab=3001,
                                          n_layers=2, dtype="bf16", B=4, prefix=0, top_k=8, rope_theta=5e5,
                                          seed=19, page_size=24), prefix_list=[23, 24, 47, 400]),
+    # 313 vocabulary tiles (the last one ragged) over at most 152 CTAs with d = 256: the
+    # 16-row LM head splits tiles between neighbouring CTAs; 12 rows, temperature 0.7
+    "lmhead_split_v40k": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=40003,
+                                        n_layers=4, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
+                                        seed=21, page_size=0), prefix_list=[5, 0, 70], temperature=0.7),
     # N * B = 160 rows: the wide tensor-core LM head with three 64-row transpose groups
     "wide_lmhead_r160": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=3001,
                                        n_layers=5, dtype="bf16", B=32, prefix=0, top_k=8, rope_theta=1e4,
