@@ -131,6 +131,24 @@ def dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(x: float, ws: int, device) -> float:
+    """The largest of the ranks' values (the slowest rank's time); the value itself at
+    one process."""
+    if ws <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(ws: int, B: int, seconds_per_step: float) -> float:
+    """Whole-job drafts/s: every replica drafts its own B sequences per step, and the job's
+    step takes as long as its slowest rank."""
+    return ws * B / seconds_per_step
+
+
 def make_problem(name: str, overrides=()):
     from fe_synth import workloads as wl
     kw = {}
@@ -255,14 +273,9 @@ def main():
     torch.cuda.synchronize()
     barrier()
     clocks = sampler.stop()
-    ms = e0.elapsed_time(e1)
-    if ws > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1), ws, "cuda")
     ms_step = ms / args.steps
-    value = ws * B / (ms_step / 1e3)
+    value = job_rate(ws, B, ms_step / 1e3)
     st = fe.fe_last_device_status(h)
     if st != fe.FE_OK:
         raise SystemExit(f"device status after the timed region: {fe.fe_status_str(st)}")
@@ -287,12 +300,7 @@ def main():
     t0 = time.perf_counter()
     for _ in range(args.e2e_steps):
         e2e_step()
-    e2e_s = (time.perf_counter() - t0) / args.e2e_steps
-    if ws > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, ws, "cuda")
 
     # ---- per-kernel device times: every launch bracketed by CUDA events on its stream -----
     per = {}
@@ -404,7 +412,7 @@ def main():
             "draft_loss": {"us_per_call": loss_us,
                            "note": "fe_draft_loss: the draft with logits [B,N,V] and hidden states written out, "
                                    "then CE + Smooth L1 (Sec. 2.3); outside the timed step"},
-            "e2e": {"value": ws * B / e2e_s, "unit": "drafts/s", "h2d_bytes_per_step": h2d,
+            "e2e": {"value": job_rate(ws, B, e2e_s), "unit": "drafts/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,
                     "call": "fe_draft_step_host (host inputs and outputs; copies, draft and tree in one graph; "
                             "returns with the outputs in host memory)"},

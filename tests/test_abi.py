@@ -68,3 +68,17 @@ def test_profile_entry_point_validates_on_host(lib):
     so = lib._lib
     n = ctypes.c_int32(0)
     assert so.fe_profile_forward(None, None, None, 8, None, None, ctypes.byref(n)) == lib.FE_ERR_INVALID_ARG
+
+
+def test_next_row_entry_points_validate_on_host(lib):
+    """The verification, loss, allocation-free LM head and timeout self-test calls reject a
+    missing handle or arguments before they touch CUDA, so a bad call never launches."""
+    so = lib._lib
+    tree = lib.fe_tree()
+    assert so.fe_verify_greedy(None, 1, 1, None, ctypes.byref(tree), None, None, None, None, None,
+                               None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_draft_loss(None, None, None, None, 0.1, 1.0, 0.9, None, None, None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_lm_head_topk_noalloc(None, None, 1, 1, 0.0, None, None, None, None, None) == lib.FE_ERR_INVALID_ARG
+    for ns in (0, 999, 10**9 + 1):  # outside 1e3..1e9 ns, and a null handle
+        assert so.fe_selftest_timeout(None, ns, None) == lib.FE_ERR_INVALID_ARG
+    assert isinstance(lib.fe_last_error_detail(), str)

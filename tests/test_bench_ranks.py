@@ -1,0 +1,74 @@
+"""bench.py's multi-process bookkeeping on CPU, as two gloo ranks: the job's time is the
+slowest rank's, the job's rate counts every replica's sequences, and the reference arm
+runs on rank 0 only. (The drafter runs as independent replicas, one per GPU, with no
+exchange on the data path; these are the only cross-rank steps.)"""
+import os
+import socket
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, ws, port, q):
+    sys.path.insert(0, ROOT)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(ws))
+    import torch.distributed as dist
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=ws)
+    try:
+        times = [3.0, 5.0, 4.0, 1.0]
+        slowest = bench.max_over_ranks(times[rank], ws, "cpu")
+        q.put((rank, "max", slowest))
+        q.put((rank, "dist_env", bench.dist_env()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_slowest_rank_time_and_job_rate():
+    import torch.multiprocessing as mp
+    ws = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, ws, port, q)) for r in range(ws)]
+    for p in procs:
+        p.start()
+    got = {}
+    try:
+        for _ in range(2 * ws):  # two results per rank
+            r, what, v = q.get(timeout=120)
+            got[(r, what)] = v
+    finally:
+        for p in procs:
+            p.join(timeout=60)
+            if p.exitcode is None:
+                p.kill()
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    assert got[(0, "max")] == got[(1, "max")] == 5.0
+    assert got[(0, "dist_env")] == (2, 0, 0) and got[(1, "dist_env")] == (2, 1, 0)
+
+
+def test_single_process_needs_no_process_group():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.max_over_ranks(2.5, 1, "cpu") == 2.5
+    # two replicas of B = 32 sequences, 1.346 ms per step: 47548 drafts/s for the job
+    assert bench.job_rate(2, 32, 1.346e-3) == pytest.approx(2 * 32 / 1.346e-3)
+    assert bench.job_rate(1, 1, 1e-3) == pytest.approx(1000.0)
+
+
+def test_reference_arm_runs_on_rank_zero_only(capsys):
+    sys.path.insert(0, ROOT)
+    import bench
+    # a non-zero rank returns at once, before reading its arguments, building any input or
+    # touching the oracle
+    assert bench.run_reference(None, 2, 1) is None
+    assert capsys.readouterr().out == ""
