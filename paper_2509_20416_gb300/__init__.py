@@ -134,12 +134,23 @@ def _stream(stream) -> int:
 
 
 def _p(t) -> int | None:
+    """The address of a contiguous tensor (host or device memory), or the int / None given."""
     if t is None:
         return None
     if isinstance(t, int):
         return t
-    assert t.is_contiguous(), "buffers passed to the drafter must be contiguous"
+    if not t.is_contiguous():
+        raise ValueError("buffers passed to the drafter must be contiguous")
     return t.data_ptr()
+
+
+def _dp(t) -> int | None:
+    """As _p, for a buffer the kernels read or write: a tensor must be on a CUDA device. A
+    host address given to a kernel faults, or, on a GPU that can reach host memory, reads
+    and writes host memory the caller did not mean to share."""
+    if t is not None and not isinstance(t, int) and not t.is_cuda:
+        raise ValueError("buffers the kernels access must be CUDA tensors")
+    return _p(t)
 
 
 def make_config(cfg: dict) -> fe_config:
@@ -200,11 +211,11 @@ def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, to
     if out is None:
         out = alloc_outputs(h, B, top_k, feat.device)
     N = h.cfg["n_layers"]
-    kc = (_vp * N)(*[_p(t) for t in k_cache])
-    vc = (_vp * N)(*[_p(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
-                        _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
-                        _p(out["topk_prob"]), _p(out["lse"]), _p(dbg_logits), _p(dbg_hidden))
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
+                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
+                        _dp(out["topk_prob"]), _dp(out["lse"]), _dp(dbg_logits), _dp(dbg_hidden))
     _check(_lib.fe_draft_forward(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_forward")
     return out
 
@@ -221,11 +232,11 @@ def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
     if out is None:
         out = alloc_outputs(h, B, top_k, feat.device)
     N = h.cfg["n_layers"]
-    kc = (_vp * N)(*[_p(t) for t in k_cache])
-    vc = (_vp * N)(*[_p(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
-                        _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
-                        _p(out["topk_prob"]), _p(out["lse"]), None, _p(dbg_hidden))
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
+                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
+                        _dp(out["topk_prob"]), _dp(out["lse"]), None, _dp(dbg_hidden))
     cap = fe_launch_count(h, B, False) + 1
     kinds = (_i32 * cap)()
     usec = (ctypes.c_float * cap)()
@@ -248,13 +259,13 @@ def fe_draft_loss(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, teach
     out.update(logits=torch.empty((B, N, V), device=dev), hidden=torch.empty((N, B, d), device=dev),
                ce=torch.empty((B, N), device=dev), feat_loss=torch.empty((B, N), device=dev),
                total=torch.empty(B, device=dev))
-    kc = (_vp * N)(*[_p(t) for t in k_cache])
-    vc = (_vp * N)(*[_p(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, 1.0, _p(feat), _p(next_tok), _p(prefix_len), kc, vc, _p(page_table),
-                        int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]), _p(out["topk_prob"]),
-                        _p(out["lse"]), _p(out["logits"]), _p(out["hidden"]))
-    _check(_lib.fe_draft_loss(h.ptr, ctypes.byref(a), _p(teacher_p), _p(target_feat), float(alpha), float(beta),
-                              float(decay), _p(out["ce"]), _p(out["feat_loss"]), _p(out["total"]), _stream(stream)),
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, 1.0, _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc, _dp(page_table),
+                        int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]), _dp(out["topk_prob"]),
+                        _dp(out["lse"]), _dp(out["logits"]), _dp(out["hidden"]))
+    _check(_lib.fe_draft_loss(h.ptr, ctypes.byref(a), _dp(teacher_p), _dp(target_feat), float(alpha), float(beta),
+                              float(decay), _dp(out["ce"]), _dp(out["feat_loss"]), _dp(out["total"]), _stream(stream)),
            "fe_draft_loss")
     return out
 
@@ -271,8 +282,8 @@ def fe_build_tree(h: Handle, next_tok, topk_id, top_k: int, out: dict | None = N
     B = int(next_tok.shape[0])
     if out is None:
         out = alloc_tree(h, B, top_k, next_tok.device)
-    t = fe_tree(_p(out["tok"]), _p(out["parent"]), _p(out["depth"]), _p(out["mask"]))
-    _check(_lib.fe_build_tree(h.ptr, B, top_k, _p(next_tok), _p(topk_id), ctypes.byref(t), _stream(stream)),
+    t = fe_tree(_dp(out["tok"]), _dp(out["parent"]), _dp(out["depth"]), _dp(out["mask"]))
+    _check(_lib.fe_build_tree(h.ptr, B, top_k, _dp(next_tok), _dp(topk_id), ctypes.byref(t), _stream(stream)),
            "fe_build_tree")
     return out
 
@@ -301,10 +312,10 @@ def fe_draft_step_host(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
     if out is None:
         out = alloc_host_step_outputs(h, B, top_k)
     N = h.cfg["n_layers"]
-    kc = (_vp * N)(*[_p(t) for t in k_cache])
-    vc = (_vp * N)(*[_p(t) for t in v_cache])
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
     a = fe_host_step_args(B, top_k, float(temperature), _p(feat), _p(next_tok), _p(prefix_len), kc, vc,
-                          _p(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
+                          _dp(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
                           _p(out["topk_prob"]), _p(out["lse"]), _p(out["tree_tok"]), _p(out["tree_parent"]),
                           _p(out["tree_depth"]), _p(out["tree_mask"]))
     _check(_lib.fe_draft_step_host(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_step_host")
@@ -324,9 +335,9 @@ def fe_verify_greedy(h: Handle, prefix_len, tree: dict, target_next, top_k: int,
                    path=torch.empty((B, N), dtype=torch.int32, device=dev),
                    n_accept=torch.empty(B, dtype=torch.int32, device=dev),
                    bonus=torch.empty(B, dtype=torch.int32, device=dev))
-    t = fe_tree(_p(tree["tok"]), _p(tree["parent"]), _p(tree["depth"]), _p(tree["mask"]))
-    _check(_lib.fe_verify_greedy(h.ptr, B, int(top_k), _p(prefix_len), ctypes.byref(t), _p(target_next),
-                                 _p(out["pos_ids"]), _p(out["path"]), _p(out["n_accept"]), _p(out["bonus"]),
+    t = fe_tree(_dp(tree["tok"]), _dp(tree["parent"]), _dp(tree["depth"]), _dp(tree["mask"]))
+    _check(_lib.fe_verify_greedy(h.ptr, B, int(top_k), _dp(prefix_len), ctypes.byref(t), _dp(target_next),
+                                 _dp(out["pos_ids"]), _dp(out["path"]), _dp(out["n_accept"]), _dp(out["bonus"]),
                                  _stream(stream)), "fe_verify_greedy")
     return out
 
@@ -337,9 +348,9 @@ def fe_commit(h: Handle, feat, tok, n_rows, prefix_len, k_cache, v_cache, page_t
     int32, n_rows [B] int32, prefix_len [B] int32 (device tensors)."""
     B, L = int(tok.shape[0]), int(tok.shape[1])
     N = h.cfg["n_layers"]
-    kc = (_vp * N)(*[_p(t) for t in k_cache])
-    vc = (_vp * N)(*[_p(t) for t in v_cache])
-    a = fe_commit_args(B, L, _p(feat), _p(tok), _p(n_rows), _p(prefix_len), kc, vc, _p(page_table), int(n_pages))
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
+    a = fe_commit_args(B, L, _dp(feat), _dp(tok), _dp(n_rows), _dp(prefix_len), kc, vc, _dp(page_table), int(n_pages))
     _check(_lib.fe_commit(h.ptr, ctypes.byref(a), _stream(stream)), "fe_commit")
 
 
@@ -366,7 +377,7 @@ def fe_lm_head_topk_noalloc(h: Handle, hidden, B: int, top_k: int, temperature: 
     are allocated here by PyTorch unless given in ``out``."""
     if out is None:
         out = alloc_outputs(h, B, top_k, hidden.device)
-    _check(_lib.fe_lm_head_topk_noalloc(h.ptr, _p(hidden), int(B), int(top_k), float(temperature),
-                                        _p(out["topk_id"]), _p(out["topk_logit"]), _p(out["topk_prob"]),
-                                        _p(out["lse"]), _stream(stream)), "fe_lm_head_topk_noalloc")
+    _check(_lib.fe_lm_head_topk_noalloc(h.ptr, _dp(hidden), int(B), int(top_k), float(temperature),
+                                        _dp(out["topk_id"]), _dp(out["topk_logit"]), _dp(out["topk_prob"]),
+                                        _dp(out["lse"]), _stream(stream)), "fe_lm_head_topk_noalloc")
     return out

@@ -82,3 +82,35 @@ def test_next_row_entry_points_validate_on_host(lib):
     for ns in (0, 999, 10**9 + 1):  # outside 1e3..1e9 ns, and a null handle
         assert so.fe_selftest_timeout(None, ns, None) == lib.FE_ERR_INVALID_ARG
     assert isinstance(lib.fe_last_error_detail(), str)
+
+
+def test_binding_rejects_host_and_strided_buffers_before_the_library(lib):
+    """The binding hands raw addresses to kernels, so it refuses a host tensor where the
+    kernels read or write (fe_draft_forward, the tree, the loss, the commit, ...) and any
+    non-contiguous buffer, with a ValueError and before any library call (the handle here
+    is a null stand-in that the library would reject)."""
+    import torch
+    cfg = dict(d=8, n_layers=2, vocab=16)
+    h = lib.Handle(0, cfg)
+    B, k = 2, 2
+    feat, tok, plen = torch.zeros(B, 24), torch.zeros(B, dtype=torch.int32), torch.zeros(B, dtype=torch.int32)
+    caches = [torch.zeros(B, 1, 4, 8) for _ in range(2)]
+    with pytest.raises(ValueError, match="CUDA"):
+        lib.fe_draft_forward(h, feat, tok, plen, caches, caches, k)
+    with pytest.raises(ValueError, match="CUDA"):
+        lib.fe_build_tree(h, tok, torch.zeros(B, 2, k, dtype=torch.int32), k)
+    with pytest.raises(ValueError, match="CUDA"):
+        lib.fe_commit(h, torch.zeros(B, 1, 24), torch.zeros(B, 1, dtype=torch.int32), plen, plen, caches, caches)
+    with pytest.raises(ValueError, match="CUDA"):
+        lib.fe_lm_head_topk_noalloc(h, torch.zeros(2, B, 8), B, k)
+    # fe_draft_step_host takes host inputs and outputs, but its caches are device buffers
+    out = dict(topk_id=torch.zeros(B, 2, k, dtype=torch.int32), topk_logit=torch.zeros(B, 2, k),
+               topk_prob=torch.zeros(B, 2, k), lse=torch.zeros(B, 2), tree_tok=torch.zeros(B, 5, dtype=torch.int32),
+               tree_parent=torch.zeros(B, 5, dtype=torch.int32), tree_depth=torch.zeros(B, 5, dtype=torch.int32),
+               tree_mask=torch.zeros(B, 5, 5, dtype=torch.uint8))
+    with pytest.raises(ValueError, match="CUDA"):
+        lib.fe_draft_step_host(h, feat, tok, plen, caches, caches, k, out=out)
+    # a strided view is refused even where host memory is allowed (the weights of fe_draft_init)
+    with pytest.raises(ValueError, match="contiguous"):
+        lib._p(torch.zeros(4, 4).t())
+    assert lib._dp(None) is None and lib._dp(0) == 0  # null and raw addresses pass through
