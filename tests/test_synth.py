@@ -2,6 +2,8 @@
 and the moments of its normal deviates (CPU only)."""
 import struct
 
+import pytest
+
 import numpy as np
 import torch
 
@@ -69,3 +71,38 @@ def test_page_plan_covers_every_row():
     for b in range(cfg["B"]):
         need = (int(plen[b]) + 1 + 15) // 16
         assert (table[b, :need] >= 0).all() and (table[b, need:] < 0).all()
+
+
+def _weight_numel(W):
+    """Elements of every weight tensor make_weights builds, by name (embedding separately)."""
+    mats = [W["w_fuse"], W["w_in"], W["lm_head"], W["final_norm"]]
+    for L in W["layers"]:
+        mats += [L[n] for n in ("attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate", "w_up", "w_down")]
+    return sum(t.numel() for t in mats), W["embed"].shape, W["w_fuse"].element_size()
+
+
+@pytest.mark.parametrize("name", ["tiny", "vic13b", "l31_8b", "l33_70b", "b32_l31"])
+def test_roofline_bytes_and_flops_count_the_generated_tensors(monkeypatch, name):
+    """The bytes and flops the roofline divides by equal a count over the tensors the
+    generator actually builds (shapes only: meta tensors, so full-size workloads cost
+    nothing): every weight once, the gathered embedding rows, the features, and each
+    layer's K/V prefix read plus the new row; flops = 2 per weight element per row (the
+    LM head for all N rows) + 4·H·hd per key."""
+    monkeypatch.setattr(wl, "_normal", lambda shape, seed, tid, std, dt: torch.empty(shape, dtype=dt, device="meta"))
+    cfg = wl.make_config(name)
+    W = wl.make_weights(cfg)
+    n_w, emb_shape, es = _weight_numel(W)
+    V, d = emb_shape
+    B, N, Hkv, hd, H = cfg["B"], cfg["n_layers"], cfg["n_kv_heads"], cfg["head_dim"], cfg["n_heads"]
+    plen = wl.make_inputs(cfg)["prefix_len"].tolist() if name == "b32_l31" else [cfg["prefix"]] * B
+    kv_elems = N * sum(p + 1 for p in plen) * 2 * Hkv * hd
+    want = (n_w + B * d + B * 3 * d + kv_elems) * es
+    assert wl.algorithmic_bytes(cfg, plen) == want
+    parts = wl.kernel_bytes(cfg, plen)
+    assert sum(parts.values()) == want
+    assert parts["attention"] == kv_elems * es and parts["lm_head"] == (V * d + d) * es
+    # matrices only (norm gains are not multiplied), per row; the LM head over all N rows
+    mats = [W["w_fuse"], W["w_in"]] + [L[n] for L in W["layers"] for n in ("w_qkv", "w_o", "w_gate", "w_up", "w_down")]
+    flops = 2 * sum(t.numel() for t in mats) * B + 2 * W["lm_head"].numel() * N * B
+    flops += N * sum(4 * H * hd * (p + 1) for p in plen)
+    assert wl.algorithmic_flops(cfg, plen) == flops
