@@ -114,3 +114,47 @@ def test_binding_rejects_host_and_strided_buffers_before_the_library(lib):
     with pytest.raises(ValueError, match="contiguous"):
         lib._p(torch.zeros(4, 4).t())
     assert lib._dp(None) is None and lib._dp(0) == 0  # null and raw addresses pass through
+
+
+BASE_CFG = dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=688, vocab=4096, n_layers=2, top_k_max=8,
+                max_seq=80, rope_theta=1e4, rms_eps=1e-5, dtype="f32")
+
+
+@pytest.mark.parametrize("change,code", [
+    (dict(n_layers=0), "INVALID_ARG"), (dict(n_layers=17), "INVALID_ARG"),
+    (dict(top_k_max=0), "INVALID_ARG"), (dict(top_k_max=33), "INVALID_ARG"),
+    (dict(top_k_max=8, vocab=7), "INVALID_ARG"), (dict(n_kv_heads=3), "INVALID_ARG"),
+    (dict(head_dim=63), "INVALID_ARG"), (dict(rope_theta=0.0), "INVALID_ARG"),
+    (dict(rope_theta=float("nan")), "INVALID_ARG"), (dict(rms_eps=-1e-6), "INVALID_ARG"),
+    (dict(max_batch=0), "INVALID_ARG"), (dict(max_seq=0), "INVALID_ARG"), (dict(page_size=-1), "INVALID_ARG"),
+    (dict(parallel_layers=2), "INVALID_ARG"), (dict(d=0), "INVALID_ARG"),
+    # legal, but outside what the kernels cover
+    (dict(head_dim=96), "UNSUPPORTED"), (dict(head_dim=32), "UNSUPPORTED"),
+    (dict(n_heads=6, n_kv_heads=2), "UNSUPPORTED"), (dict(n_heads=16, n_kv_heads=1), "UNSUPPORTED"),
+    (dict(d=260), "UNSUPPORTED"), (dict(ffn=690), "UNSUPPORTED"),
+])
+def test_init_rejects_configs_before_any_cuda_call(lib, change, code):
+    """fe_draft_init checks the configuration (and that every weight pointer is set) before
+    it touches CUDA, so these run without a GPU: the weight pointers are non-null stand-ins
+    that are never read."""
+    so = lib._lib
+    cfg = dict(BASE_CFG, **change)
+    c = lib.make_config(cfg)
+    n = max(1, min(cfg["n_layers"], 16))
+    layers = (lib.fe_layer_weights * n)(*[lib.fe_layer_weights(*([8] * 7)) for _ in range(n)])
+    w = lib.fe_weights(8, 8, 8, 8, 8, layers)
+    out = ctypes.c_void_p()
+    assert so.fe_draft_init(ctypes.byref(c), ctypes.byref(w), None, ctypes.byref(out)) == getattr(lib, "FE_ERR_" + code)
+    assert out.value is None
+
+
+def test_init_rejects_a_missing_layer_weight(lib):
+    so = lib._lib
+    c = lib.make_config(BASE_CFG)
+    layers = (lib.fe_layer_weights * 2)(lib.fe_layer_weights(*([8] * 7)), lib.fe_layer_weights(*([8] * 6 + [0])))
+    w = lib.fe_weights(8, 8, 8, 8, 8, layers)
+    out = ctypes.c_void_p()
+    assert so.fe_draft_init(ctypes.byref(c), ctypes.byref(w), None, ctypes.byref(out)) == lib.FE_ERR_INVALID_ARG
+    layers[1] = lib.fe_layer_weights(*([8] * 7))
+    c.dtype = 7  # neither FE_F32 nor FE_BF16
+    assert so.fe_draft_init(ctypes.byref(c), ctypes.byref(w), None, ctypes.byref(out)) == lib.FE_ERR_INVALID_ARG
