@@ -27,7 +27,7 @@ _lock = threading.Lock()
 _cache: dict = {}
 
 # Number of planted-mistake variants compiled by build(mutant=n) (n = 1..N_MUTANTS).
-N_MUTANTS = 36
+N_MUTANTS = 40
 _UNUSED_MUTANTS = {25}  # ids with no planted mistake
 
 
@@ -117,6 +117,12 @@ class Oracle:
                                    ctypes.POINTER(ctypes.c_int32), _D, _D]
         L.or_draft_seq.restype = ctypes.c_int32
         L.or_max_threads.restype = ctypes.c_int32
+        L.or_splitmix64.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
+        L.or_splitmix64.restype = ctypes.c_uint64
+        L.or_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
+        L.or_uniform.restype = ctypes.c_double
+        L.or_topk_sample_rows.argtypes = [_D, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_double,
+                                          ctypes.c_uint64, ctypes.c_int64, _I, _I]
         L.or_commit_seq.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(_P), _P, _I, ctypes.c_int32,
                                     ctypes.c_int32, ctypes.POINTER(_P), ctypes.POINTER(_P), ctypes.c_int64]
         L.or_commit_seq.restype = ctypes.c_int32
@@ -177,6 +183,27 @@ class Oracle:
         ids = np.zeros(k, dtype=np.int32)
         self.L.or_topk(_dp(lg), lg.size, k, ids.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
         return ids
+
+    def splitmix64(self, seed: int, n: int) -> int:
+        return int(self.L.or_splitmix64(seed, n))
+
+    def uniform(self, seed: int, n: int) -> float:
+        return float(self.L.or_uniform(seed, n))
+
+    def topk_sample(self, logits, k: int, T: float, seed: int, row0: int = 0):
+        """k candidates drawn without replacement from softmax(logits / T) per row (reading
+        C16, Gumbel-top-k). logits [R, V] (or [V]); row r uses counter row0 + r. Returns
+        (ids by descending logit, ids in draw order), each [R, k] (or [k])."""
+        lg = np.ascontiguousarray(logits, dtype=np.float64)
+        one = lg.ndim == 1
+        lg = lg.reshape(-1, lg.shape[-1])
+        R, V = lg.shape
+        ids = np.zeros((R, k), np.int32)
+        drawn = np.zeros((R, k), np.int32)
+        i32 = ctypes.POINTER(ctypes.c_int32)
+        self.L.or_topk_sample_rows(_dp(lg), R, V, k, float(T), seed, row0, ids.ctypes.data_as(i32),
+                                   drawn.ctypes.data_as(i32))
+        return (ids[0], drawn[0]) if one else (ids, drawn)
 
     def tree(self, N, k, root, topk):
         topk = np.ascontiguousarray(topk, dtype=np.int32).reshape(N, k)

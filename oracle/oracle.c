@@ -19,7 +19,8 @@
  *   - Sec. 2.1: every h_i goes through the target's frozen LM head (after the
  *     target's final RMSNorm) to give the distribution q_{t+i}.
  *   - Sec. 2.2: top-k per depth and the Backbone Expansion tree with its
- *     tree-attention (ancestor-or-self) mask.
+ *     tree-attention (ancestor-or-self) mask; for stochastic drafting, k candidates
+ *     drawn without replacement from q_{t+i} (Gumbel-top-k over counter-based deviates).
  * Every stored bf16/fp32 input is widened exactly to double; nothing is rounded in
  * between. Loops are the definitions written out: no blocking, no fusion, no
  * reordering of a sum. OpenMP only splits independent output rows across threads,
@@ -327,6 +328,89 @@ void or_topk(const double *logits, int64_t V, int32_t k, int32_t *ids)
         taken[best] = 1;
     }
     free(taken);
+}
+
+/* ---- stochastic drafting (Sec. 2.2 "sample k candidates", reading C16) ---------- */
+
+/* SplitMix64 (Steele, Lea and Flood, "Fast splittable pseudorandom number generators",
+ * OOPSLA 2014): the generator seeded with s returns, as its n-th output (n >= 1), the
+ * finaliser below applied to s + n * 0x9E3779B97F4A7C15 (arithmetic mod 2^64). */
+uint64_t or_splitmix64(uint64_t seed, uint64_t n)
+{
+    uint64_t z = seed + n * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+/* A uniform deviate in (0, 1) from the top 23 bits of output n: (floor(x / 2^41) + 1/2)
+ * / 2^23. Every value is an odd multiple of 2^-24 (24 significant bits), so it is exact in
+ * float32 as in double, and never 0 or 1. */
+double or_uniform(uint64_t seed, uint64_t n)
+{
+    const uint64_t x = or_splitmix64(seed, n);
+    return ((double)(x >> 41) + 0.5) / 8388608.0;
+}
+
+/* k distinct candidates drawn without replacement from q = softmax(logits / T), T > 0, by
+ * the Gumbel-top-k trick (Vieira 2014; Kool, van Hoof and Welling, ICML 2019): with
+ * U_v uniform on (0, 1) and G_v = -log(-log U_v) a standard Gumbel deviate, the tokens
+ * with the k largest keys logits_v / T + G_v, taken by descending key, have the law of k
+ * successive draws without replacement from q. Token v of row `row` uses output
+ * n = row * V + v + 1 of SplitMix64 seeded with `seed`, so every (row, token) has its own
+ * deviate. Ties of keys go to the smaller id.
+ *   drawn[k]: the candidates in draw order (descending key), or NULL;
+ *   ids[k]:   the same k tokens by descending logit (ties: ascending id), so that ids[0],
+ *             the most probable candidate, is the one the Backbone Expansion tree extends
+ *             (Sec. 2.2). */
+void or_topk_sample(const double *logits, int64_t V, int32_t k, double T, uint64_t seed, int64_t row,
+                    int32_t *ids, int32_t *drawn)
+{
+    double *key = (double *)malloc((size_t)V * sizeof(double));
+    int32_t *d = (int32_t *)malloc((size_t)k * sizeof(int32_t));
+    unsigned char *taken = (unsigned char *)calloc((size_t)V, 1);
+    for (int64_t v = 0; v < V; ++v) {
+        const uint64_t n = MUT(38) ? (uint64_t)v + 1 : (uint64_t)row * (uint64_t)V + (uint64_t)v + 1;
+        const double u = or_uniform(seed, n);
+        const double g = MUT(37) ? log(-log(u)) : -log(-log(u));
+        key[v] = (MUT(39) ? logits[v] : logits[v] / T) + g;
+    }
+    for (int32_t r = 0; r < k; ++r) {
+        int64_t best = -1;
+        for (int64_t v = 0; v < V; ++v)
+            if (!taken[v] && (best < 0 || key[v] > key[best]))
+                best = v;
+        d[r] = (int32_t)best;
+        taken[best] = 1;
+    }
+    if (drawn)
+        memcpy(drawn, d, (size_t)k * sizeof(int32_t));
+    /* order the drawn set by (descending logit, ascending id): insertion sort */
+    for (int32_t r = 0; r < k; ++r)
+        ids[r] = d[r];
+    if (!MUT(40))
+        for (int32_t r = 1; r < k; ++r) {
+            const int32_t t = ids[r];
+            int32_t j = r - 1;
+            while (j >= 0 && (logits[ids[j]] < logits[t] || (logits[ids[j]] == logits[t] && ids[j] > t))) {
+                ids[j + 1] = ids[j];
+                --j;
+            }
+            ids[j + 1] = t;
+        }
+    free(taken);
+    free(d);
+    free(key);
+}
+
+/* or_topk_sample over R rows of logits [R, V]: row r uses counter row r0 + r. Rows are
+ * independent, so OpenMP splits them. */
+void or_topk_sample_rows(const double *logits, int64_t R, int64_t V, int32_t k, double T, uint64_t seed,
+                         int64_t r0, int32_t *ids, int32_t *drawn)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < R; ++r)
+        or_topk_sample(logits + r * V, V, k, T, seed, r0 + r, ids + r * k, drawn ? drawn + r * k : NULL);
 }
 
 /* Sec. 2.2, Backbone Expansion, in level-major order with T = 1 + N k nodes.

@@ -195,6 +195,67 @@ def pin_topk(orc):
         assert np.array_equal(orc.topk(lg, k), want), k
 
 
+def pin_topk_sample(orc):
+    """Stochastic drafting (Sec. 2.2 "sample k candidates", reading C16): the counter-based
+    deviates, the law of the draws without replacement, and the order the tree uses."""
+    # SplitMix64 seeded with 0: its first outputs as published (Steele et al. 2014)
+    for n, want in enumerate([0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F], start=1):
+        assert orc.splitmix64(0, n) == want
+        u = orc.uniform(0, n)
+        assert u == ((want >> 41) + 0.5) / 2 ** 23 and float(np.float32(u)) == u  # exact in float32
+    us = [orc.uniform(12345, n) for n in range(1, 20001)]
+    assert 0.0 < min(us) and max(us) < 1.0 and abs(np.mean(us) - 0.5) < 0.01
+
+    # the law of two draws without replacement from q = softmax(l / T), brute force over all
+    # 20 ordered pairs of a 5-token vocabulary: P(a, then b) = q_a q_b / (1 - q_a)
+    lg = np.array([0.3, -1.2, 1.0, 0.0, 0.7])
+    R = 200_000
+    for T in (1.0, 0.5):
+        q = np.exp(lg / T - np.max(lg / T))
+        q /= q.sum()
+        ids, drawn = orc.topk_sample(np.tile(lg, (R, 1)), 2, T, seed=99)
+        counts = np.zeros((5, 5))
+        np.add.at(counts, (drawn[:, 0], drawn[:, 1]), 1)
+        for a in range(5):
+            for b in range(5):
+                p = 0.0 if a == b else q[a] * q[b] / (1 - q[a])
+                tol = 5 * math.sqrt(p * (1 - p) / R) + 1e-4
+                assert abs(counts[a, b] / R - p) <= tol, (T, a, b, counts[a, b] / R, p)
+    # the first draw of a larger vocabulary follows q itself
+    rng = np.random.default_rng(3)
+    lg = rng.standard_normal(40)
+    q = np.exp(lg - lg.max())
+    q /= q.sum()
+    _, drawn = orc.topk_sample(np.tile(lg, (R, 1)), 3, 1.0, seed=5)
+    freq = np.bincount(drawn[:, 0], minlength=40) / R
+    assert np.all(np.abs(freq - q) <= 5 * np.sqrt(q * (1 - q) / R) + 1e-4)
+    assert all(len(set(r)) == 3 for r in drawn[:1000])  # without replacement
+
+    # row r of a batch draws with counter row0 + r, as a single-row call with that counter
+    lg = rng.standard_normal((6, 50))
+    ids_b, drawn_b = orc.topk_sample(lg, 4, 0.8, seed=7, row0=11)
+    for r in range(6):
+        ids_1, drawn_1 = orc.topk_sample(lg[r], 4, 0.8, seed=7, row0=11 + r)
+        assert np.array_equal(ids_b[r], ids_1) and np.array_equal(drawn_b[r], drawn_1)
+
+    # the tree's order: the drawn set by descending logit, ties to the smaller id, so rank 0
+    # is the most probable candidate (the backbone)
+    lg = np.array([1.0, 1.0, 1.0, 1.0, 0.0, 0.0, 2.0])
+    ids, drawn = orc.topk_sample(np.tile(lg, (500, 1)), 4, 1.0, seed=3)
+    for i, d in zip(ids, drawn):
+        assert sorted(i) == sorted(d)
+        assert list(i) == sorted(d, key=lambda v: (-lg[v], v))
+    # k = V: every token, in the stable descending-logit order
+    ids, _ = orc.topk_sample(lg, 7, 1.0, seed=4)
+    assert np.array_equal(ids, np.argsort(-lg, kind="stable"))
+    # T -> 0: the draws become the greedy top-k (the Gumbel deviates are bounded by the
+    # uniforms on the 2^-24 grid: |G| < 17, far below the logit gaps / T)
+    lg = rng.permutation(np.arange(30) * 1e-3)
+    for seed in range(5):
+        ids, drawn = orc.topk_sample(lg, 5, 1e-9, seed=seed)
+        assert np.array_equal(ids, orc.topk(lg, 5)) and np.array_equal(drawn, orc.topk(lg, 5))
+
+
 def _check_tree_invariants(N, k, root, topk, tok, par, dep, mask):
     T = 1 + N * k
     assert tok.shape == (T,) and mask.shape == (T, T)
@@ -520,5 +581,5 @@ def pin_commit(orc):
 
 
 ALL_PINS = [pin_commit, pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
-            pin_softmax, pin_topk, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
+            pin_softmax, pin_topk, pin_topk_sample, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]
