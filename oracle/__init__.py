@@ -27,7 +27,7 @@ _lock = threading.Lock()
 _cache: dict = {}
 
 # Number of planted-mistake variants compiled by build(mutant=n) (n = 1..N_MUTANTS).
-N_MUTANTS = 40
+N_MUTANTS = 44
 _UNUSED_MUTANTS = {25}  # ids with no planted mistake
 
 
@@ -121,6 +121,8 @@ class Oracle:
         L.or_splitmix64.restype = ctypes.c_uint64
         L.or_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
         L.or_uniform.restype = ctypes.c_double
+        L.or_accept_sampled.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _I, _I, _I,
+                                        _I, _D, _D, _D, _D, _I, _I, _I]
         L.or_topk_sample_rows.argtypes = [_D, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_double,
                                           ctypes.c_uint64, ctypes.c_int64, _I, _I]
         L.or_commit_seq.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(_P), _P, _I, ctypes.c_int32,
@@ -204,6 +206,24 @@ class Oracle:
         self.L.or_topk_sample_rows(_dp(lg), R, V, k, float(T), seed, row0, ids.ctypes.data_as(i32),
                                    drawn.ctypes.data_as(i32))
         return (ids[0], drawn[0]) if one else (ids, drawn)
+
+    def accept_sampled(self, tok, parent, depth, rank, q, p, u_acc, u_bonus):
+        """Lossless verification of B sampled trees (Sec. 2.4, reading C17): tok, parent,
+        depth, rank [B, T] int; q [B, N, V], p [B, T, V], u_acc, u_bonus [B, T] float.
+        Returns (path [B, N] with -1 after the accepted nodes, n_accept [B], bonus [B])."""
+        i32 = ctypes.POINTER(ctypes.c_int32)
+        tok, parent, depth, rank = (np.ascontiguousarray(a, dtype=np.int32) for a in (tok, parent, depth, rank))
+        q, p, u_acc, u_bonus = (np.ascontiguousarray(a, dtype=np.float64) for a in (q, p, u_acc, u_bonus))
+        B, T = tok.shape
+        N, V = q.shape[1], q.shape[2]
+        assert p.shape == (B, T, V) and q.shape == (B, N, V) and u_acc.shape == u_bonus.shape == (B, T)
+        path = np.zeros((B, N), np.int32)
+        n = np.zeros(B, np.int32)
+        bonus = np.zeros(B, np.int32)
+        self.L.or_accept_sampled(B, T, N, V, *(a.ctypes.data_as(i32) for a in (tok, parent, depth, rank)),
+                                 _dp(q), _dp(p), _dp(u_acc), _dp(u_bonus), path.ctypes.data_as(i32),
+                                 n.ctypes.data_as(i32), bonus.ctypes.data_as(i32))
+        return path, n, bonus
 
     def tree(self, N, k, root, topk):
         topk = np.ascontiguousarray(topk, dtype=np.int32).reshape(N, k)

@@ -519,6 +519,111 @@ int32_t or_accept_greedy(int32_t T, const int32_t *tok, const int32_t *parent, c
     return n;
 }
 
+/* Lossless verification of a sampled draft tree (Sec. 2.4, "the speculative sampling
+ * algorithm identifies the longest accepted token path"; reading C17), for B sequences:
+ *   tok, parent, depth [B][T]  the trees (or_tree's layout), T = 1 + N k;
+ *   rank [B][T]    a node's position in its level's draw order (0 = drawn first; the root's
+ *                  entry is not read);
+ *   q [B][N][V]    the drafter's proposal at each depth, softmax(l_i / T) (the law the
+ *                  level's candidates were drawn from, without replacement);
+ *   p [B][T][V]    the target's next-token distribution after each node (given the node's
+ *                  root path), at the same temperature;
+ *   u_acc, u_bonus [B][T]  uniform deviates on (0, 1), one test and one bonus draw per node.
+ * Recursive rejection sampling over draws without replacement (the multi-candidate form of
+ * speculative sampling, Leviathan et al. and Chen et al. 2023; Jeon et al. 2024): at the
+ * current node, with r = its p and s = the next depth's q, the children are tested in draw
+ * order; child c with token x is accepted iff u_acc[c] * s(x) <= r(x), that is with
+ * probability min(1, r(x) / s(x)); on rejection r becomes max(r - s, 0) renormalised and x
+ * is removed from s (renormalised), the law of the next draw. An accepted child becomes the
+ * current node. When every child is rejected, or the node has none, the bonus token is drawn
+ * from r by inverse CDF: the smallest x with u_bonus[current] < r(0) + ... + r(x).
+ * path[b][0..n) are the accepted node ids (-1 after), n_accept[b] = n, bonus[b] the drawn
+ * token. Every emitted token then has the target's law. */
+void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t *tok, const int32_t *parent,
+                       const int32_t *depth, const int32_t *rank, const double *q, const double *p,
+                       const double *u_acc, const double *u_bonus, int32_t *path, int32_t *n_accept,
+                       int32_t *bonus)
+{
+#pragma omp parallel for schedule(static)
+    for (int32_t b = 0; b < B; ++b) {
+        const int32_t *tk = tok + (int64_t)b * T, *par = parent + (int64_t)b * T, *dep = depth + (int64_t)b * T;
+        const int32_t *rk = rank + (int64_t)b * T;
+        double *r = (double *)malloc((size_t)V * sizeof(double));
+        double *s = (double *)malloc((size_t)V * sizeof(double));
+        int32_t *kids = (int32_t *)malloc((size_t)T * sizeof(int32_t));
+        int32_t cur = 0, n = 0;
+        memcpy(r, p + ((int64_t)b * T + cur) * V, (size_t)V * sizeof(double));
+        for (;;) {
+            /* the children of cur, in draw order */
+            int32_t m = 0;
+            for (int32_t c = 1; c < T; ++c)
+                if (par[c] == cur)
+                    kids[m++] = c;
+            for (int32_t i = 1; i < m; ++i) {
+                const int32_t t = kids[i];
+                int32_t j = i - 1;
+                while (j >= 0 && (MUT(44) ? kids[j] > t : rk[kids[j]] > rk[t])) {
+                    kids[j + 1] = kids[j];
+                    --j;
+                }
+                kids[j + 1] = t;
+            }
+            if (m == 0 || n >= N)
+                break;
+            memcpy(s, q + ((int64_t)b * N + dep[cur]) * V, (size_t)V * sizeof(double));
+            int32_t next = -1;
+            for (int32_t i = 0; i < m && next < 0; ++i) {
+                const int32_t c = kids[i], x = tk[c];
+                const int accept = MUT(41) ? u_acc[(int64_t)b * T + c] * r[x] <= s[x]
+                                           : u_acc[(int64_t)b * T + c] * s[x] <= r[x];
+                if (accept) {
+                    next = c;
+                    break;
+                }
+                double sr = 0.0;
+                for (int64_t v = 0; v < V; ++v) {
+                    const double dlt = r[v] - s[v];
+                    r[v] = (MUT(42) || dlt > 0.0) ? dlt : 0.0;
+                    sr += r[v];
+                }
+                if (sr > 0.0)
+                    for (int64_t v = 0; v < V; ++v)
+                        r[v] /= sr;
+                if (!MUT(43)) {
+                    const double sx = s[x];
+                    s[x] = 0.0;
+                    if (sx < 1.0)
+                        for (int64_t v = 0; v < V; ++v)
+                            s[v] /= 1.0 - sx;
+                }
+            }
+            if (next < 0)
+                break;
+            path[(int64_t)b * N + n++] = next;
+            cur = next;
+            memcpy(r, p + ((int64_t)b * T + cur) * V, (size_t)V * sizeof(double));
+        }
+        for (int32_t i = n; i < N; ++i)
+            path[(int64_t)b * N + i] = -1;
+        n_accept[b] = n;
+        /* the bonus token: inverse CDF of r */
+        const double u = u_bonus[(int64_t)b * T + cur];
+        double cum = 0.0;
+        int32_t pick = -1, last = 0;
+        for (int64_t v = 0; v < V && pick < 0; ++v) {
+            if (r[v] > 0.0)
+                last = (int32_t)v;
+            cum += r[v];
+            if (u < cum)
+                pick = (int32_t)v;
+        }
+        bonus[b] = pick >= 0 ? pick : last; /* u above a sum rounded below 1 */
+        free(kids);
+        free(s);
+        free(r);
+    }
+}
+
 /* The whole draft of one sequence (Eq. 1, Eq. 2, Sec. 2.1 LM head, Sec. 2.2 top-k).
  *   w     : 5 + 7N pointers: w_fuse [d,3d], w_in [d,2d], embed [V,d], lm_head [V,d],
  *           final_norm [d], then per layer attn_norm, w_qkv, w_o, mlp_norm, w_gate,

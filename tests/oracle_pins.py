@@ -457,6 +457,100 @@ def pin_accept_greedy(orc):
         assert path[:n].tolist() == chain[::-1] and (path[n:] == -1).all()
 
 
+def _sampled_trees(orc, N, k, V, drafter_logits, R, seed):
+    """R Backbone Expansion trees whose levels are drawn by orc.topk_sample (T = 1):
+    returns tok, parent, depth, rank [R, T] and the tree order ids [R, N, k]."""
+    lg = np.tile(np.asarray(drafter_logits), (R, 1))  # row r * N + i: depth i + 1 of trial r
+    ids, drawn = orc.topk_sample(lg, k, 1.0, seed=seed)
+    ids, drawn = ids.reshape(R, N, k), drawn.reshape(R, N, k)
+    T = 1 + N * k
+    tok = np.zeros((R, T), np.int32)
+    tok[:, 1:] = ids.reshape(R, N * k)
+    par = np.array([-1] + [0 if i == 0 else 1 + (i - 1) * k for i in range(N) for _ in range(k)], np.int32)
+    dep = np.array([0] + [i + 1 for i in range(N) for _ in range(k)], np.int32)
+    rank = np.zeros((R, T), np.int32)
+    rank[:, 1:] = np.argmax(ids[:, :, :, None] == drawn[:, :, None, :], axis=3).reshape(R, N * k)
+    return tok, np.tile(par, (R, 1)), np.tile(dep, (R, 1)), rank, ids
+
+
+def pin_accept_sampled(orc):
+    """Lossless verification of a sampled tree (Sec. 2.4, reading C17): with a one-hot
+    target it is the greedy walk; with the target equal to the drafter it accepts the first
+    draw; and every emitted token has the target's law (Monte Carlo on a 4-token vocabulary,
+    5 sigma), which a wrong test ratio, residual, proposal update or test order breaks."""
+    rng = np.random.default_rng(21)
+    sm = lambda x: np.exp(x - x.max(-1, keepdims=True)) / np.exp(x - x.max(-1, keepdims=True)).sum(-1, keepdims=True)
+    # (a) one-hot targets reduce the walk to or_accept_greedy, for any proposal and test order
+    for N, k in ((1, 1), (2, 3), (3, 2), (4, 4), (5, 1)):
+        B, V, T = 40, 12, 1 + N * k
+        topk = np.stack([np.stack([rng.permutation(V)[:k] for _ in range(N)]) for _ in range(B)]).astype(np.int32)
+        trees = [orc.tree(N, k, int(rng.integers(0, V)), topk[b]) for b in range(B)]
+        tok, par, dep = (np.stack([t[j] for t in trees]) for j in range(3))
+        rank = np.zeros((B, T), np.int32)
+        for b in range(B):
+            for i in range(N):
+                rank[b, 1 + i * k:1 + (i + 1) * k] = rng.permutation(k)
+        tn = rng.integers(0, V, (B, T)).astype(np.int32)
+        for b in range(B):
+            for a in range(1, T):
+                if rng.random() < 0.6:
+                    tn[b, par[b, a]] = tok[b, a]
+        p = np.zeros((B, T, V))
+        np.put_along_axis(p, tn[:, :, None], 1.0, axis=2)
+        q = sm(rng.standard_normal((B, N, V)) * 2)
+        path, n, bonus = orc.accept_sampled(tok, par, dep, rank, q, p, rng.random((B, T)), rng.random((B, T)))
+        for b in range(B):
+            _, gpath, gn, gbonus = orc.accept_greedy(tok[b], par[b], dep[b], tn[b], 0, N)
+            assert (n[b], path[b].tolist(), bonus[b]) == (gn, gpath.tolist(), gbonus), (N, k, b)
+    # (b) target = drafter at every node with children: the first-drawn child is accepted
+    N, k, V, R = 3, 3, 9, 300
+    lg = rng.standard_normal((N, V))
+    tok, par, dep, rank, ids = _sampled_trees(orc, N, k, V, lg, R, seed=8)
+    q = np.tile(sm(lg), (R, 1, 1))
+    p = np.zeros((R, 1 + N * k, V))
+    p[:, 0] = q[:, 0]
+    p[:, 1:1 + (N - 1) * k] = np.repeat(q[:, 1:], k, axis=1)
+    p[:, 1 + (N - 1) * k:] = 1.0 / V
+    path, n, _ = orc.accept_sampled(tok, par, dep, rank, q, p, rng.random((R, 1 + N * k)),
+                                    rng.random((R, 1 + N * k)))
+    for r in range(R):
+        for j in range(n[r]):
+            assert rank[r, path[r, j]] == 0
+        assert n[r] >= 1
+    # (c) the law of the emitted tokens equals the target's, token by token
+    N, k, V, R = 2, 2, 4, 400_000
+    lg = np.array([[2.0, 0.5, 0.0, -1.0], [-0.5, 1.5, 0.0, 1.0]])  # the drafter's depth-1 and depth-2 logits
+    q = sm(lg)
+    p_root = np.array([0.1, 0.2, 0.6, 0.1])
+    p_a = sm(rng.standard_normal((V, V)) * 1.5)        # after token a
+    p_ab = sm(rng.standard_normal((V, V, V)) * 1.5)    # after tokens a, b
+    tok, par, dep, rank, ids = _sampled_trees(orc, N, k, V, lg, R, seed=77)
+    P = np.zeros((R, 1 + N * k, V))
+    P[:, 0] = p_root
+    P[:, 1:1 + k] = p_a[tok[:, 1:1 + k]]
+    P[:, 1 + k:] = p_ab[tok[:, 1][:, None], tok[:, 1 + k:]]  # level 2 hangs under the level-1 backbone
+    path, n, bonus = orc.accept_sampled(tok, par, dep, rank, np.tile(q, (R, 1, 1)), P, rng.random((R, 1 + N * k)),
+                                        rng.random((R, 1 + N * k)))
+    rows = np.arange(R)
+    emitted = np.full((R, N + 1), -1)
+    for j in range(N):
+        emitted[:, j] = np.where(n > j, tok[rows, np.maximum(path[:, j], 0)], -1)
+    emitted[rows, n] = bonus
+
+    def law(sel, want, what):
+        cnt = int(sel.sum())
+        if cnt < 2000:
+            return
+        freq = np.bincount(emitted[sel, len(what)], minlength=V) / cnt
+        tol = 5 * np.sqrt(want * (1 - want) / cnt) + 1e-4
+        assert np.all(np.abs(freq - want) <= tol), (what, freq, want)
+    law(np.ones(R, bool), p_root, ())
+    for a in range(V):
+        law((n >= 1) & (emitted[:, 0] == a), p_a[a], (a,))
+        for b in range(V):
+            law((n >= 2) & (emitted[:, 0] == a) & (emitted[:, 1] == b), p_ab[a, b], (a, b))
+
+
 def pin_loss(orc):
     """The training objective of Sec. 2.3 (Eq. 3-6): Smooth L1 closed forms, a two-layer,
     three-token example worked by hand, and the reductions of the cross-entropy to a library
@@ -581,5 +675,5 @@ def pin_commit(orc):
 
 
 ALL_PINS = [pin_commit, pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
-            pin_softmax, pin_topk, pin_topk_sample, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
+            pin_softmax, pin_topk, pin_topk_sample, pin_accept_sampled, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]
