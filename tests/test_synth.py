@@ -73,6 +73,22 @@ def test_page_plan_covers_every_row():
         assert (table[b, :need] >= 0).all() and (table[b, need:] < 0).all()
 
 
+@pytest.mark.parametrize("ps", [8, 16, 24])
+def test_paginate_places_every_row_at_its_page_and_slot(ps):
+    """Row p of sequence b lands at pool[table[b, p // ps], :, p % ps]: the addressing the
+    paged attention uses, for page sizes that do and do not divide the chunk length."""
+    cfg = wl.make_config("tiny", B=3, prefix=0, page_size=ps, max_seq=70)
+    plen = torch.tensor([0, 23, 69], dtype=torch.int32)
+    table, n_pages = wl.page_plan(cfg, plen)
+    g = torch.Generator().manual_seed(1)
+    logical = torch.randn((3, 2, 70, 8), generator=g)
+    pool = wl.paginate(cfg, logical, table, n_pages)
+    assert pool.shape == (n_pages, 2, ps, 8)
+    for b in range(3):
+        for p in range(int(plen[b]) + 1):
+            assert torch.equal(pool[int(table[b, p // ps]), :, p % ps], logical[b, :, p])
+
+
 def _weight_numel(W):
     """Elements of every weight tensor make_weights builds, by name (embedding separately)."""
     mats = [W["w_fuse"], W["w_in"], W["lm_head"], W["final_norm"]]
