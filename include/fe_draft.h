@@ -23,8 +23,10 @@
  *    a prefix longer than the cache, a bad page id, a timed-out device wait) are
  *    recorded in a device status word and reported by fe_last_device_status();
  *    the offending work item is skipped, and no kernel traps.
- *  - No global state: several handles may coexist. One handle must not be used
- *    from two streams concurrently (its scratch buffers are shared by its calls).
+ *  - No global state beyond two exceptions: the per-thread detail string of
+ *    fe_last_error_detail() and the fixed scratch array of fe_lm_head_topk_noalloc().
+ *    Several handles may coexist. One handle must not be used from two streams
+ *    concurrently (its scratch buffers are shared by its calls).
  *  - No exceptions cross the ABI.
  */
 #ifndef FE_DRAFT_H
