@@ -360,6 +360,61 @@ def _agree(o, r, tol=1e-10):
         assert np.allclose(o["topk_logit"][i], o["logits"][i][o["topk_id"][i]], rtol=0, atol=0)
 
 
+def _handworked_layer2(x0_or_h1):
+    """Layer 2 of the hand-worked draft, in the closed form derived in the fixture. Its
+    input normalises to u = (0.2, 1.4) under both readings, so the attention output is
+    the same; the residual base is h1 (the cascade) or x0 (the parallel ablation)."""
+    c, s = math.cos(1.0), math.sin(1.0)
+    s_c = (0.2 * c - 1.4 * s) / math.sqrt(2.0)
+    w_c = 1.0 / (1.0 + math.exp(math.sqrt(2.0) - s_c))
+    o = (w_c * -1.0 + (1 - w_c) * 7.0, w_c * 3.0 + (1 - w_c) * 1.0)
+    x = (x0_or_h1[0] + o[0], x0_or_h1[1] + o[1])
+    r = math.sqrt((x[0] ** 2 + x[1] ** 2) / 2)
+    u2 = (x[0] / r, x[1] / r)
+    silu = u2[0] / (1.0 + math.exp(-u2[0]))
+    h2 = (x[0], x[1] + silu * u2[1])
+    rz = math.sqrt((h2[0] ** 2 + h2[1] ** 2) / 2)
+    z2 = (2 * h2[0] / rz, h2[1] / rz)
+    return np.array(h2), np.array([5 * z2[0], 5 * z2[1], 5 * (z2[0] + z2[1])])
+
+
+def pin_draft_handworked(orc):
+    """The whole draft on a 2-wide, two-layer model worked by hand
+    (tests/golden/draft_handworked_n2_k2.json): Eq. 1's fusion and concat order, the
+    attention over the cached row and the row's own key (scale, RoPE at position P), the
+    residuals, SwiGLU's gate/up order, the final norm's gain, the LM head, top-k, the tree,
+    and the parallel ablation's residual base."""
+    g = json.load(open(os.path.join(GOLDEN, "draft_handworked_n2_k2.json")))
+    cfg = dict(g["cfg"], parallel_layers=0)
+    f32 = lambda a: torch.tensor(a, dtype=torch.float32)
+    W = dict(w_fuse=f32(g["w_fuse"]), w_in=f32(g["w_in"]), embed=f32(g["embed"]), lm_head=f32(g["lm_head"]),
+             final_norm=f32(g["final_norm"]),
+             layers=[{k: f32(v) for k, v in L.items() if not k.endswith("row0")} for L in g["layers"]])
+    kcs, vcs = [], []
+    for L in g["layers"]:
+        kc, vc = torch.zeros((1, 2, 2)), torch.zeros((1, 2, 2))
+        kc[0, 0], vc[0, 0] = f32(L["k_cache_row0"]), f32(L["v_cache_row0"])
+        kcs.append(kc)
+        vcs.append(vc)
+    feat = f32(g["feat"])
+    h2, lg2 = _handworked_layer2(g["h1"])
+    for par in (0, 1):
+        cfg["parallel_layers"] = par
+        o = orc.draft_seq(cfg, W, feat, g["tok"], g["P"], kcs, vcs, 2, 2)
+        assert np.allclose(o["hidden"][0], g["h1"], rtol=1e-13, atol=1e-13), par
+        assert np.allclose(o["logits"][0], g["logits1"], rtol=1e-13, atol=1e-13), par
+        assert o["topk_id"][0].tolist() == g["topk1"]
+        assert abs(o["lse"][0] - math.log(math.exp(2) + math.exp(7) + math.exp(9))) < 1e-12
+        want_h2, want_lg2 = (h2, lg2) if par == 0 else _handworked_layer2((1.0, 7.0))
+        assert np.allclose(o["hidden"][1], want_h2, rtol=1e-12, atol=1e-12), (par, o["hidden"][1], want_h2)
+        assert np.allclose(o["logits"][1], want_lg2, rtol=1e-12, atol=1e-12), (par, o["logits"][1], want_lg2)
+        if par == 0:
+            assert o["topk_id"][1].tolist() == g["topk2"]
+            tok, parent, depth, _ = orc.tree(2, 2, g["tok"], o["topk_id"])
+            assert (tok.tolist(), parent.tolist(), depth.tolist()) == (g["tree_tok"], g["tree_parent"],
+                                                                       g["tree_depth"])
+
+
 def pin_draft_n1(orc):
     """N = 1: the drafter is a single EAGLE-style decoder layer plus the LM head."""
     for dtype in ("f32", "bf16"):
@@ -675,5 +730,5 @@ def pin_commit(orc):
 
 
 ALL_PINS = [pin_commit, pin_loss, pin_accept_greedy, pin_parallel_layers, pin_matvec_bruteforce, pin_rmsnorm, pin_rope, pin_attention, pin_silu_mul,
-            pin_softmax, pin_topk, pin_topk_sample, pin_accept_sampled, pin_tree, pin_draft_n1, pin_cascade, pin_truncation,
+            pin_softmax, pin_topk, pin_topk_sample, pin_accept_sampled, pin_tree, pin_draft_handworked, pin_draft_n1, pin_cascade, pin_truncation,
             pin_zero_blocks]
