@@ -1,6 +1,6 @@
 """bench.py's multi-process bookkeeping on CPU, as two gloo ranks: the job's time is the
 slowest rank's, the job's rate counts every replica's sequences, and the reference arm
-runs on rank 0 only. (The drafter runs as independent replicas, one per GPU, with no
+runs on rank 0 only and prints one line of the benchmark's JSON contract. (The drafter runs as independent replicas, one per GPU, with no
 exchange on the data path; these are the only cross-rank steps.)"""
 import os
 import socket
