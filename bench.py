@@ -3,12 +3,20 @@
 
 One step = fe_draft_forward + fe_build_tree over one batch of the workload (the whole
 hot path: fused-feature input FCs, N cascade layers, LM head with fused softmax/top-k,
-Backbone Expansion tree). Default workload: the Vicuna-13B-shaped drafter (d=5120,
-40 heads x 128, F=13824, V=32000, N=5, B=1, P=512, k=8, bf16 weights/caches), with
-seeded synthetic inputs. The 3.8 GB of weights read per step exceed the 129 MB L2, so
-no flush is needed between steps.
+Backbone Expansion tree). Default workload: the largest single-GPU drafter, shaped like
+LLaMA-3.3-70B (d=8192, 64 query / 8 KV heads x 128, F=28672, V=128256, N=8, B=1, P=2048,
+k=10, bf16 weights and caches; 16.5 GB streamed per draft). The same JSON line carries a
+record of the batched-serving workload (LLaMA-3.1-8B shape, B=32, ragged prefixes in
+[256, 4096] over a 16-token page pool) with its own rate, roofline, e2e and CPU baseline.
+Inputs are seeded synthetic tensors; every step streams all weights (GBs, far above the
+129 MB L2), so no flush is needed between steps.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--also NAME ...]
+                  [--impl ours|reference]
+
+Per-kernel times come from the GPU's own stamps inside the graph the step runs as
+(fe_profile_graph): each launch's first-CTA start and last-warp exit, so per family the
+time a launch adds to the step (its end minus the previous launch's end) sums to the step.
 
 Multi-GPU (torchrun): replicas only. Every rank drafts its own batch with its own copy
 of the drafter; there is no collective on the data path (a barrier brackets the timed
@@ -19,6 +27,7 @@ from __future__ import annotations
 import argparse
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -27,36 +36,42 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-HBM_FALLBACK_GBS = 6800.0  # used only when MEASURED_PEAKS.json is absent
+HBM_FALLBACK_GBS = 6800.0      # used only when MEASURED_PEAKS.json is absent
+BF16_FALLBACK_TFLOPS = 1900.0  # burst
+BF16_FALLBACK_SUSTAINED = 1700.0
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--workload", default="vic13b")
+    ap.add_argument("--workload", default="l33_70b")
+    ap.add_argument("--also", nargs="*", default=["b32_l31"],
+                    help="further workloads measured in the same run, as sub-records of the JSON line")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=200)
-    ap.add_argument("--profile-steps", type=int, default=50,
-                    help="drafts timed launch by launch (CUDA events) for the per-kernel roofline")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget")
+    ap.add_argument("--profile-steps", type=int, default=30,
+                    help="graph replays with per-kernel GPU stamps for the per-kernel roofline")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle sample budget per workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true", help="skip the verification / loss / commit timings")
     ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
                     help="override a workload field (e.g. n_layers=1) for profiling runs")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 # DRAM traffic of the dominant kernel family from an ncu capture (dram__bytes_read.sum +
-# dram__bytes_write.sum over the linear launches of one draft of this workload), with the
-# SHA-256 of the kernel sources it was taken on: a changed kernel reports traffic null.
+# dram__bytes_write.sum over the linear launches of a one-layer draft of the workload,
+# scaled to the full draft by the launches' shapes), with the SHA-256 of the kernel
+# sources it was taken on: a changed kernel reports traffic null.
 TRAFFIC = {
-    # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum
-    #     -k regex:linear_kernel -s 18 -c 6 on `bench.py --set n_layers=1` (one draft's six
-    # linear launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down); the five-layer draft
-    # repeats the four per-layer launches five times with the same shapes.
-    "vic13b": {"bytes_per_draft": 160356608 + 105004032 + 5 * (157437696 + 52540928 + 283344384 + 141732352),
-               "src": "66b1fbb81a51953f"},
+    # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum -k regex:linear_kernel
+    #     -s 18 -c 6 on `bench.py --workload l33_70b --set n_layers=1 --also ...` (one draft's six linear
+    # launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down; the eight-layer draft repeats the last four)
+    "l33_70b": {"bytes_per_draft": (402788096 + 3366912) + (268564480 + 122624)
+                + 8 * ((167900672 + 48896) + (134358272 + 344064) + (939682048 + 208128) + (469999616 + 81408)),
+                "src": "cac667a35be22899"},
 }
 KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
 
@@ -71,12 +86,33 @@ def kernel_source_hash() -> str:
 
 
 def peaks():
+    """(HBM GB/s, bf16 TFLOP/s burst, bf16 TFLOP/s sustained, 'measured' | 'fallback')."""
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         with open(p) as f:
             j = json.load(f)
-        return float(j["hbm_gbs"]), "measured"
-    return HBM_FALLBACK_GBS, "fallback"
+        return (float(j["hbm_gbs"]), float(j["bf16_tflops"]),
+                float(j.get("bf16_tflops_sustained", j["bf16_tflops"])), "measured")
+    return HBM_FALLBACK_GBS, BF16_FALLBACK_TFLOPS, BF16_FALLBACK_SUSTAINED, "fallback"
+
+
+def cpu_model() -> str:
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                k = line.split(":", 1)[0].strip().lower()
+                if k in ("model name", "cpu model"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.processor() or platform.machine()
 
 
 class ClockSampler:
@@ -149,6 +185,58 @@ def job_rate(ws: int, B: int, seconds_per_step: float) -> float:
     return ws * B / seconds_per_step
 
 
+def family_times(launches, n_replays: int) -> dict:
+    """Per kernel family, from in_step_times() summed over n_replays graph replays: launches
+    per draft, the time the family adds to the step and its summed spans (us per draft).
+    A tensor-core phase's operand prep counts with its phase ('linear_prep' -> 'linear',
+    'lm_prep' -> 'lm_head'); the main launches alone are counted."""
+    fam = {}
+    for kind, span, add in launches:
+        key = {"linear_prep": "linear", "lm_prep": "lm_head"}.get(kind, kind)
+        c = fam.setdefault(key, {"launches": 0, "added_us": 0.0, "span_us": 0.0})
+        if kind == key:
+            c["launches"] += 1
+        c["added_us"] += add
+        c["span_us"] += span
+    out = {}
+    for key, c in fam.items():
+        out[key] = {"launches_per_draft": c["launches"] / n_replays, "us_per_draft": c["added_us"] / n_replays,
+                    "span_us_per_draft": c["span_us"] / n_replays}
+    return out
+
+
+def roofline_block(kernels: dict, kbytes: dict, kflops: dict, ms_step: float, alg_bytes: int, alg_flops: int,
+                   traffic, n_replays: int) -> dict:
+    """The dominant kernel family's HBM roofline (algorithmic bytes per launch over the time a
+    launch adds inside the graph-replayed step), the whole step's, and the tensor-pipe
+    fractions (algorithmic flops over time, against the measured bf16 peaks)."""
+    hbm, tf_burst, tf_sus, kind = peaks()
+    top = max((k for k in kernels if k in kbytes), key=lambda x: kernels[x]["us_per_draft"])
+    kt = kernels[top]
+    launches = max(kt["launches_per_draft"], 1e-9)
+    us_per_launch = kt["us_per_draft"] / launches
+    bpl = kbytes[top] / launches
+    achieved = bpl / (us_per_launch * 1e-6) / 1e9
+    step_gbs = alg_bytes / (ms_step * 1e-3) / 1e9
+    step_tflops = alg_flops / (ms_step * 1e-3) / 1e12
+    per_gemm = {}
+    for k, fl in kflops.items():
+        if k in kernels and kernels[k]["us_per_draft"] > 0:
+            t = fl / (kernels[k]["us_per_draft"] * 1e-6) / 1e12
+            per_gemm[k] = {"tflops": t, "frac_burst": t / tf_burst, "frac_sustained": t / tf_sus}
+    return {"bound": "hbm", "kernel": top, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+            "frac": achieved / hbm, "peak_kind": kind, "traffic": traffic,
+            "algorithmic_bytes_per_launch": bpl, "us_per_launch": us_per_launch,
+            "span_us_per_launch": kt["span_us_per_draft"] / launches, "launches_per_draft": launches,
+            "timing": (f"GPU %globaltimer stamps of every launch inside the graph-replayed step "
+                       f"(fe_profile_graph, {n_replays} replays); per launch the time it adds to the step "
+                       f"(its end minus the previous launch's end)"),
+            "step": {"achieved": step_gbs, "frac": step_gbs / hbm, "algorithmic_bytes": alg_bytes},
+            "tensor": {"algorithmic_flops": alg_flops, "tflops": step_tflops, "peak_burst": tf_burst,
+                       "peak_sustained": tf_sus, "frac_burst": step_tflops / tf_burst,
+                       "frac_sustained": step_tflops / tf_sus, "peak_kind": kind, "per_gemm_family": per_gemm}}
+
+
 def make_problem(name: str, overrides=()):
     from fe_synth import workloads as wl
     kw = {}
@@ -182,7 +270,8 @@ def time_oracle(cfg, W, I, ks, vs, budget_s: float, max_runs: int | None = None)
 
 
 def workload_config(cfg, wl) -> dict:
-    return {"workload": cfg.get("name", "") + "".join(f" {o}" for o in cfg.get("overrides", [])), "shape": wl.describe(cfg), "B": cfg["B"], "N": cfg["n_layers"],
+    return {"workload": cfg.get("name", "") + "".join(f" {o}" for o in cfg.get("overrides", [])),
+            "shape": wl.describe(cfg), "B": cfg["B"], "N": cfg["n_layers"],
             "top_k": cfg["top_k"], "d": cfg["d"], "vocab": cfg["vocab"], "accum": "f32",
             "l2": "inputs larger than L2 (every step streams all weights, >129 MB)" if cfg["dtype"] == "bf16"
             else "L2-resident (no flush)"}
@@ -207,28 +296,22 @@ def run_reference(args, ws, rank):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
             "config": workload_config(cfg, wl), "impl": "reference",
             "cpu_baseline": {"value": value, "unit": "drafts/s", "cores": thr, "kind": "oracle",
+                             "cpu_model": cpu_model(),
                              "sample": f"{runs} single-sequence drafts of the workload"},
             "e2e": {"value": value, "unit": "drafts/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
-def main():
-    args = parse()
-    ws, rank, local = dist_env()
-    if args.impl == "reference":
-        run_reference(args, ws, rank)
-        return
+def measure(args, name: str, overrides, ws: int, rank: int, local: int, extras: bool) -> dict:
+    """One workload: the timed steps, e2e, in-graph per-kernel times, roofline and (rank 0,
+    one process) the oracle's rate. Returns the record (on every rank)."""
     import torch
-    torch.cuda.set_device(local)
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     import paper_2509_20416_gb300 as fe
     from fe_synth import workloads as wl
 
-    cfg, W, I, ks, vs = make_problem(args.workload, args.set)
-    cfg["name"] = args.workload
-    cfg["overrides"] = list(args.set)
+    cfg, W, I, ks, vs = make_problem(name, overrides)
+    cfg["name"] = name
+    cfg["overrides"] = list(overrides)
     B, N, k = cfg["B"], cfg["n_layers"], cfg["top_k"]
     h = fe.fe_draft_init(dict(cfg, max_batch=B), W)
     if cfg["page_size"]:
@@ -253,12 +336,15 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
+    def check(where):
+        st = fe.fe_last_device_status(h)
+        if st != fe.FE_OK:
+            raise SystemExit(f"{name}: device status {where}: {fe.fe_status_str(st)}")
+
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize()
-    st = fe.fe_last_device_status(h)
-    if st != fe.FE_OK:
-        raise SystemExit(f"device status after warm-up: {fe.fe_status_str(st)}")
+    check("after warm-up")
 
     sampler = ClockSampler(local)
     time.sleep(0.3)
@@ -276,9 +362,7 @@ def main():
     ms = max_over_ranks(e0.elapsed_time(e1), ws, "cuda")
     ms_step = ms / args.steps
     value = job_rate(ws, B, ms_step / 1e3)
-    st = fe.fe_last_device_status(h)
-    if st != fe.FE_OK:
-        raise SystemExit(f"device status after the timed region: {fe.fe_status_str(st)}")
+    check("after the timed region")
 
     # ---- end to end through the public API with host buffers ------------------------------
     # fe_draft_step_host: host inputs -> (pinned staging -> device copy, draft, tree, device
@@ -302,24 +386,75 @@ def main():
         e2e_step()
     e2e_s = max_over_ranks((time.perf_counter() - t0) / args.e2e_steps, ws, "cuda")
 
-    # ---- per-kernel device times: every launch bracketed by CUDA events on its stream -----
-    per = {}
-    n_prof = 0
-    for _ in range(max(1, args.profile_steps)):
-        for kind, us in fe.fe_profile_forward(h, feat, tok, plen, kd, vd, k, cfg["temperature"], page_table=table,
-                                              n_pages=n_pages, out=out, stream=stream):
-            c = per.setdefault(kind, [0, 0.0])
-            c[0] += 1
-            c[1] += us
-        n_prof += 1
-    st = fe.fe_last_device_status(h)
-    if st != fe.FE_OK:
-        raise SystemExit(f"device status after the profiled drafts: {fe.fe_status_str(st)}")
-    prof_total = sum(v[1] for v in per.values())
-    kernels = {kind: {"launches_per_draft": v[0] / n_prof, "us_per_draft": v[1] / n_prof,
-                      "us_per_launch": v[1] / v[0], "share": v[1] / prof_total} for kind, v in per.items()}
+    # ---- per-kernel times inside the graph-replayed step (GPU stamps) ---------------------
+    launches, n_rep, steps_us = [], max(1, args.profile_steps), []
+    for _ in range(n_rep):
+        stamps = fe.fe_profile_graph(h, feat, tok, plen, kd, vd, k, cfg["temperature"], page_table=table,
+                                     n_pages=n_pages, out=out, tree=tree, stream=stream)
+        its = fe.in_step_times(stamps)
+        launches.extend(its)
+        steps_us.append(sum(a for _, _, a in its))
+    check("after the stamped replays")
+    kernels = family_times(launches, n_rep)
+    stamped_us = statistics.median(steps_us)
 
-    # ---- verification side (not part of the draft step): positions + greedy acceptance walk --
+    # ---- verification / training / update calls (not part of the draft step) --------------
+    extra = {}
+    if extras:
+        extra = time_extras(fe, h, cfg, wl, feat, tok, plen, kd, vd, table, n_pages, tree, stream, I, check)
+
+    # ---- roofline of the dominant kernel family (and of the whole step) --------------------
+    plist = I["prefix_len"].tolist()
+    alg_bytes = wl.algorithmic_bytes(cfg, plist)
+    alg_flops = wl.algorithmic_flops(cfg, plist)
+    kbytes = wl.kernel_bytes(cfg, plist)
+    kflops = wl.kernel_flops(cfg, plist)
+    for kind, v in kernels.items():
+        if kind in kbytes and v["us_per_draft"] > 0:
+            v["algorithmic_bytes_per_draft"] = kbytes[kind]
+            v["achieved_gbs"] = kbytes[kind] / (v["us_per_draft"] * 1e-6) / 1e9
+        v["share_of_step"] = v["us_per_draft"] / (ms_step * 1e3)
+    traffic = None
+    tr = TRAFFIC.get(f"{name}{''.join(' ' + o for o in overrides)}")
+    if tr and tr["src"] == kernel_source_hash() and "linear" in kernels:
+        traffic = tr["bytes_per_draft"] / kernels["linear"]["launches_per_draft"]
+    roof = roofline_block(kernels, kbytes, kflops, ms_step, alg_bytes, alg_flops, traffic, n_rep)
+    if roof["kernel"] != "linear":
+        roof["traffic"] = None
+    launches_per_step = fe.fe_launch_count(h, B, True)
+
+    rec = {"metric": "drafts/s", "value": value, "unit": "drafts/s", "n_gpus": ws, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms_step, "us_per_draft": ms_step * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
+           "data": "synthetic (seeded generator)", "config": workload_config(cfg, wl),
+           "roofline": roof, "kernels": kernels,
+           "in_step": {"stamped_step_us": stamped_us, "families_sum_us": sum(v["us_per_draft"] for v in kernels.values()),
+                       "event_step_us": ms_step * 1e3,
+                       "note": "the per-family added times partition the stamped span of one graph replay "
+                               "(first kernel start to tree kernel end), which lies inside the event-timed step"},
+           "e2e": {"value": job_rate(ws, B, e2e_s), "unit": "drafts/s", "h2d_bytes_per_step": h2d,
+                   "d2h_bytes_per_step": d2h,
+                   "call": "fe_draft_step_host (host inputs and outputs; copies, draft and tree in one graph; "
+                           "returns with the outputs in host memory)"},
+           "gpu_launches": launches_per_step * args.steps, "launches_per_step": launches_per_step,
+           "clocks": clocks}
+    rec.update(extra)
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        rate, runs, thr, el = time_oracle(cfg, W, I, ks, vs, args.cpu_seconds)
+        rec["cpu_baseline"] = {"value": rate, "unit": "drafts/s", "cores": thr, "kind": "oracle",
+                               "cpu_model": cpu_model(),
+                               "sample": f"{runs} single-sequence drafts of the workload ({el:.1f} s)"}
+    h.close()
+    del W, ks, vs, kd, vd
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return rec
+
+
+def time_extras(fe, h, cfg, wl, feat, tok, plen, kd, vd, table, n_pages, tree, stream, I, check) -> dict:
+    """fe_verify_greedy, fe_draft_loss and fe_commit on the same workload (outside the step)."""
+    import torch
+    B, N, k = cfg["B"], cfg["n_layers"], cfg["top_k"]
     T = 1 + N * k
     g = torch.Generator().manual_seed(1)
     target_next = torch.randint(0, cfg["vocab"], (B, T), generator=g, dtype=torch.int32).cuda()
@@ -334,8 +469,6 @@ def main():
     v1.synchronize()
     verify_us = 1000.0 * v0.elapsed_time(v1) / 100
 
-    # ---- training-objective forward (not part of the draft step): fe_draft_loss = the draft with
-    # its full-vocabulary logits and hidden states written out, then the loss kernels ----------
     V, d = cfg["vocab"], cfg["d"]
     teacher = torch.softmax(torch.randn((B, N, V), generator=g), dim=-1).cuda()
     target_feat = torch.randn((N, B, d), generator=g).cuda()
@@ -343,18 +476,16 @@ def main():
         fe.fe_draft_loss(h, feat, tok, plen, kd, vd, teacher, target_feat, k, page_table=table, n_pages=n_pages,
                          stream=stream)
     v0.record(stream)
-    for _ in range(20):
+    for _ in range(10):
         fe.fe_draft_loss(h, feat, tok, plen, kd, vd, teacher, target_feat, k, page_table=table, n_pages=n_pages,
                          stream=stream)
     v1.record(stream)
     v1.synchronize()
-    loss_us = 1000.0 * v0.elapsed_time(v1) / 20
-    st = fe.fe_last_device_status(h)
-    if st != fe.FE_OK:
-        raise SystemExit(f"device status after the loss forward: {fe.fe_status_str(st)}")
+    loss_us = 1000.0 * v0.elapsed_time(v1) / 10
+    check("after the loss forward")
 
-    # ---- update step (not part of the draft step): fe_commit of N accepted rows per sequence;
-    # written over rows the caches already hold (P_b - N ..), so paged pools need no new pages
+    # fe_commit of N accepted rows per sequence, written over rows the caches already hold
+    # (P_b - N ..), so paged pools need no new pages
     cfeat = torch.randn((B, N, 3 * d), generator=g).to(wl.torch_dtype(cfg)).cuda()
     ctok = torch.randint(0, cfg["vocab"], (B, N), generator=g, dtype=torch.int32).cuda()
     cn = torch.full((B,), N, dtype=torch.int32).cuda()
@@ -362,48 +493,13 @@ def main():
     for _ in range(3):
         fe.fe_commit(h, cfeat, ctok, cn, cplen, kd, vd, page_table=table, n_pages=n_pages, stream=stream)
     v0.record(stream)
-    for _ in range(10):
+    for _ in range(5):
         fe.fe_commit(h, cfeat, ctok, cn, cplen, kd, vd, page_table=table, n_pages=n_pages, stream=stream)
     v1.record(stream)
     v1.synchronize()
-    commit_us = 1000.0 * v0.elapsed_time(v1) / 10
-    st = fe.fe_last_device_status(h)
-    if st != fe.FE_OK:
-        raise SystemExit(f"device status after the commits: {fe.fe_status_str(st)}")
-
-    # ---- roofline of the dominant kernel (and of the whole step, for context) ----------------
-    peak, peak_kind = peaks()
-    plist = I["prefix_len"].tolist()
-    alg_bytes = wl.algorithmic_bytes(cfg, plist)
-    kbytes = wl.kernel_bytes(cfg, plist)
-    for kind, v in kernels.items():
-        if kind in kbytes:
-            v["algorithmic_bytes_per_draft"] = kbytes[kind]
-            v["achieved_gbs"] = kbytes[kind] / (v["us_per_draft"] * 1e-6) / 1e9
-    top = max(kernels, key=lambda x: kernels[x]["us_per_draft"])
-    kt = kernels[top]
-    bytes_per_launch = kbytes.get(top, 0) / kt["launches_per_draft"]
-    achieved = bytes_per_launch / (kt["us_per_launch"] * 1e-6) / 1e9
-    traffic = None
-    tr = TRAFFIC.get(f"{args.workload}{''.join(' ' + o for o in args.set)}")
-    if tr and top == "linear" and tr["src"] == kernel_source_hash():
-        traffic = tr["bytes_per_draft"] / kt["launches_per_draft"]
-    step_achieved = alg_bytes / (ms_step / 1e3) / 1e9
-    launches = fe.fe_launch_count(h, B, True)
-
-    line = {"metric": "drafts/s", "value": value, "unit": "drafts/s", "n_gpus": ws, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_step, "us_per_draft": ms_step * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
-            "data": "synthetic (seeded generator)", "config": workload_config(cfg, wl),
-            "roofline": {"bound": "hbm", "kernel": top, "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "peak_kind": peak_kind, "traffic": traffic,
-                         "algorithmic_bytes_per_launch": bytes_per_launch,
-                         "us_per_launch": kt["us_per_launch"], "launches_per_draft": kt["launches_per_draft"],
-                         "timing": f"CUDA events around every launch, {n_prof} drafts launched eagerly",
-                         "step": {"achieved": step_achieved, "frac": step_achieved / peak,
-                                  "algorithmic_bytes": alg_bytes}},
-            "kernels": kernels,
-            "verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
+    commit_us = 1000.0 * v0.elapsed_time(v1) / 5
+    check("after the commits")
+    return {"verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
                               "note": "fe_verify_greedy after the step (positions + greedy acceptance walk)"},
             "commit": {"us_per_call": commit_us, "rows_per_sequence": N,
                        "note": "fe_commit of N accepted rows per sequence (Sec. 2.4 Update and Iterate): "
@@ -411,18 +507,29 @@ def main():
                                "outside the timed step"},
             "draft_loss": {"us_per_call": loss_us,
                            "note": "fe_draft_loss: the draft with logits [B,N,V] and hidden states written out, "
-                                   "then CE + Smooth L1 (Sec. 2.3); outside the timed step"},
-            "e2e": {"value": job_rate(ws, B, e2e_s), "unit": "drafts/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h,
-                    "call": "fe_draft_step_host (host inputs and outputs; copies, draft and tree in one graph; "
-                            "returns with the outputs in host memory)"},
-            "gpu_launches": launches * args.steps, "launches_per_step": launches,
-            "clocks": clocks}
-    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        rate, runs, thr, el = time_oracle(cfg, W, I, ks, vs, args.cpu_seconds)
-        line["cpu_baseline"] = {"value": rate, "unit": "drafts/s", "cores": thr, "kind": "oracle",
-                                "sample": f"{runs} single-sequence drafts of the workload ({el:.1f} s)"}
-    h.close()
+                                   "then CE + Smooth L1 (Sec. 2.3); outside the timed step"}}
+
+
+def main():
+    args = parse()
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    import torch
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    line = measure(args, args.workload, args.set, ws, rank, local, extras=not args.no_extras)
+    subs = {}
+    for name in args.also or []:
+        if name == args.workload:
+            continue
+        subs[name] = measure(args, name, (), ws, rank, local, extras=False)
+    if subs:
+        line["workloads"] = subs
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:

@@ -220,6 +220,18 @@ def algorithmic_flops(cfg: dict, prefix_len) -> int:
     return int(f)
 
 
+def kernel_flops(cfg: dict, prefix_len) -> dict:
+    """algorithmic_flops split by kernel family (the parts sum to it): 'linear' = the
+    products with every weight matrix but the LM head, 'attention' = q.K and p.V over each
+    layer's P_b + 1 keys, 'lm_head' = the LM head over all N * B hidden rows."""
+    d, H, Hkv, hd, F, V, N = (cfg[k] for k in ("d", "n_heads", "n_kv_heads", "head_dim", "ffn",
+                                               "vocab", "n_layers"))
+    B = len(prefix_len)
+    per_row = d * 3 * d + d * 2 * d + N * ((H + 2 * Hkv) * hd * d + d * H * hd + 3 * F * d)
+    att = sum(4 * H * hd * (int(p) + 1) for p in prefix_len) * N
+    return {"linear": int(2 * per_row * B), "attention": int(att), "lm_head": int(2 * V * d * N * B)}
+
+
 def n_tree(cfg: dict, top_k=None) -> int:
     return 1 + cfg["n_layers"] * (top_k or cfg["top_k"])
 

@@ -17,6 +17,10 @@
  *  - "device" pointers are CUDA device (or managed) memory on the handle's device;
  *    "host" pointers are ordinary host memory. Memory passed to a call stays owned
  *    by the caller.
+ *  - A handle belongs to the CUDA device that was current when fe_draft_init created it.
+ *    Every later call on the handle (except fe_free) must be made with that device
+ *    current; otherwise it returns FE_ERR_INVALID_ARG (fe_last_error_detail() names
+ *    both devices) and enqueues nothing. fe_free switches to the handle's device itself.
  *  - Calls that take a stream enqueue work on it and return before it runs.
  *    Argument errors are detected on the host and returned synchronously, with
  *    nothing enqueued. Errors found while the kernels run (an out-of-range token,
@@ -144,7 +148,10 @@ typedef struct {
 
 typedef struct fe_handle fe_handle;
 
-/* Create a drafter on the current CUDA device. Copies (and repacks) every weight into
+/* Create a drafter on the current CUDA device: the N cascade layers L_1..L_N of Eq. 2,
+ * the two input FCs of Sec. 2.1 / Eq. 1 (feature fusion, then concat with the token
+ * embedding) and the target's frozen LM head with its final norm (Sec. 2.1, shared by
+ * every depth). Copies (and repacks) every weight into
  * memory the handle owns, so the caller may free its weights once the call returns.
  * Weight pointers may be host or device memory (any memory cudaMemcpyDefault reads).
  * Precomputes the RoPE table in double precision. `stream` orders the copies; the
@@ -295,7 +302,8 @@ typedef enum {
     FE_KERNEL_LM_PREP = 2,   /* tensor-core LM head: RMSNorm of the hidden rows into its bf16 operand */
     FE_KERNEL_LM_HEAD = 3,   /* LM head + softmax statistics + top-k (and its merge) */
     FE_KERNEL_COPY = 4,      /* the dbg_hidden copy */
-    FE_KERNEL_LINEAR_PREP = 5 /* tensor-core linear phase: prologue into its bf16 operand */
+    FE_KERNEL_LINEAR_PREP = 5, /* tensor-core linear phase: prologue into its bf16 operand */
+    FE_KERNEL_TREE = 6       /* the Backbone Expansion tree (fe_profile_graph with a tree) */
 } fe_kernel_kind;
 
 /* Measurement aid: runs one draft exactly as fe_draft_forward computes it, but launched
@@ -309,6 +317,25 @@ typedef enum {
 FE_API fe_status fe_profile_forward(fe_handle *h, const fe_forward_args *args, void *stream, int32_t cap,
                                     int32_t *kinds, float *usec, int32_t *n_launches);
 
+/* Measurement aid: the draft timed inside the CUDA graph it really runs as. Captures (once
+ * per argument set, cached like fe_draft_forward's graph) the same launch sequence as
+ * fe_draft_forward, with programmatic dependent launch, plus fe_build_tree's kernel when
+ * `tree` is given (tree buffers as fe_build_tree's, built from args->topk_id), and runs it
+ * once on `stream`. Each kernel records, with the GPU's global nanosecond timer, when its
+ * first CTA started and when its last warp exited. The call then waits for the stream and
+ * writes, for launch j < *n_launches in stream order, its family kinds[j] (fe_kernel_kind),
+ * start_us[j] and end_us[j]: microseconds from the earliest start of the run (-1 for a
+ * launch that records nothing, the dbg_hidden copy). Because a programmatic launch starts
+ * while its predecessor finishes, consecutive spans overlap; end_us[j] - end_us[j - 1] is
+ * the time launch j adds to the step, and these sum to end_us of the last launch. kinds,
+ * start_us, end_us: HOST arrays of `cap` entries; cap >= fe_launch_count(h, B, tree != 0)
+ * + 1 is enough. Errors as fe_draft_forward, and FE_ERR_INVALID_ARG for too small a cap.
+ * The stamps cost two atomic operations per CTA and warp; fe_draft_forward's own graph has
+ * none. Not for use inside stream capture. */
+FE_API fe_status fe_profile_graph(fe_handle *h, const fe_forward_args *args, const fe_tree *tree, void *stream,
+                                  int32_t cap, int32_t *kinds, double *start_us, double *end_us,
+                                  int32_t *n_launches);
+
 /* The LM head with its fused softmax statistics and top-k (the tail of fe_draft_forward)
  * over caller-provided hidden states, for callers that cannot allocate device memory at
  * the point they need it (a frozen memory pool or arena, a path that must not call
@@ -319,13 +346,15 @@ FE_API fe_status fe_profile_forward(fe_handle *h, const fe_forward_args *args, v
  *   outputs    device topk_id [B, N, top_k] int32, topk_logit / topk_prob [B, N, top_k],
  *              lse [B, N] float32, as fe_draft_forward; temperature as there
  * It allocates nothing: it reads the LM head and final norm the handle already holds and
- * keeps its working memory in one fixed ~2.1 MB device array that the library reserves on
- * every device it is loaded on, for the life of the process. Limits: n_layers * B <= 16,
- * d <= 16384, top_k <= 32; larger requests return FE_ERR_INVALID_ARG (reason in
- * fe_last_error_detail()). All calls share that array and leave their data in it: calls
- * that can overlap on the GPU (several streams or host threads) race and must be
- * serialised by the caller. The first call on a device looks the array up with
- * cudaGetSymbolAddress; make that first call before any stream capture. */
+ * keeps its working memory in one fixed ~2.1 MB device array, for the life of the process.
+ * fe_draft_init looks that array up on its device (cudaGetSymbolAddress), which, under
+ * CUDA's default lazy module loading, is when the array is reserved; so no call of this
+ * entry point allocates or looks anything up. Limits: n_layers * B <= 16, d <= 16384,
+ * top_k <= 32, at most 256 vocabulary slabs; larger requests return FE_ERR_INVALID_ARG
+ * (reason in fe_last_error_detail()), as does a call made with another device current than
+ * the handle's. All calls share that array and leave their data in it: calls that can
+ * overlap on the GPU (several streams or host threads) race and must be serialised by the
+ * caller. */
 FE_API fe_status fe_lm_head_topk_noalloc(fe_handle *h, const float *hidden, int32_t B, int32_t top_k,
                                          float temperature, int32_t *topk_id, float *topk_logit,
                                          float *topk_prob, float *lse, void *stream);

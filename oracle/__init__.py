@@ -193,8 +193,8 @@ class Oracle:
         return float(self.L.or_uniform(seed, n))
 
     def topk_sample(self, logits, k: int, T: float, seed: int, row0: int = 0):
-        """k candidates drawn without replacement from softmax(logits / T) per row (reading
-        C16, Gumbel-top-k). logits [R, V] (or [V]); row r uses counter row0 + r. Returns
+        """k candidates drawn without replacement from softmax(logits / T) per row (the
+        Gumbel-top-k trick: the k largest logit / T + G). logits [R, V] (or [V]); row r uses counter row0 + r. Returns
         (ids by descending logit, ids in draw order), each [R, k] (or [k])."""
         lg = np.ascontiguousarray(logits, dtype=np.float64)
         one = lg.ndim == 1
@@ -208,7 +208,8 @@ class Oracle:
         return (ids[0], drawn[0]) if one else (ids, drawn)
 
     def accept_sampled(self, tok, parent, depth, rank, q, p, u_acc, u_bonus):
-        """Lossless verification of B sampled trees (Sec. 2.4, reading C17): tok, parent,
+        """Lossless verification of B sampled trees (Sec. 2.4; recursive rejection
+        sampling over each node's children in draw order): tok, parent,
         depth, rank [B, T] int; q [B, N, V], p [B, T, V], u_acc, u_bonus [B, T] float.
         Returns (path [B, N] with -1 after the accepted nodes, n_accept [B], bonus [B])."""
         i32 = ctypes.POINTER(ctypes.c_int32)
@@ -305,6 +306,17 @@ class Oracle:
             raise ValueError("oracle rejected the arguments")
         return dict(hidden=hidden, logits=logits, lse=lse, topk_id=tid, topk_logit=tlg,
                     topk_prob=tpr)
+
+    def lm_head(self, cfg: dict, weights: dict, hidden) -> np.ndarray:
+        """Logits [R, V] of R given hidden states [R, d] (Sec. 2.1: the final RMSNorm, then
+        the frozen LM head), row by row through or_lm_head."""
+        c = config_struct(cfg, 0, 1)
+        h = np.ascontiguousarray(np.asarray(hidden, dtype=np.float64).reshape(-1, cfg["d"]))
+        out = np.zeros((h.shape[0], cfg["vocab"]))
+        for r in range(h.shape[0]):
+            self.L.or_lm_head(ctypes.byref(c), _ptr(weights["lm_head"]), _ptr(weights["final_norm"]),
+                              _dp(h[r]), _dp(out[r]))
+        return out
 
     def layer(self, cfg: dict, lw: dict, pos: float, kc, vc, cap: int, P: int, x):
         c = config_struct(cfg, 0, 1)

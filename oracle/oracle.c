@@ -330,7 +330,9 @@ void or_topk(const double *logits, int64_t V, int32_t k, int32_t *ids)
     free(taken);
 }
 
-/* ---- stochastic drafting (Sec. 2.2 "sample k candidates", reading C16) ---------- */
+/* ---- stochastic drafting (Sec. 2.2 "sample k candidates"): read as k draws without
+ * replacement from softmax(l / T), taken by the Gumbel-top-k trick over counter-based
+ * deviates, so that both sides can draw the same numbers ------------------------------ */
 
 /* SplitMix64 (Steele, Lea and Flood, "Fast splittable pseudorandom number generators",
  * OOPSLA 2014): the generator seeded with s returns, as its n-th output (n >= 1), the
@@ -520,7 +522,9 @@ int32_t or_accept_greedy(int32_t T, const int32_t *tok, const int32_t *parent, c
 }
 
 /* Lossless verification of a sampled draft tree (Sec. 2.4, "the speculative sampling
- * algorithm identifies the longest accepted token path"; reading C17), for B sequences:
+ * algorithm identifies the longest accepted token path"; the paper names no variant, and it
+ * is read as recursive rejection sampling over each node's children in draw order), for B
+ * sequences:
  *   tok, parent, depth [B][T]  the trees (or_tree's layout), T = 1 + N k;
  *   rank [B][T]    a node's position in its level's draw order (0 = drawn first; the root's
  *                  entry is not read);
@@ -700,8 +704,10 @@ int32_t or_draft_seq(const or_config *c, const void *const *w, const void *feat,
     return 0;
 }
 
-/* Sec. 2.4, "Update and Iterate" (the commit step of reading C15): once the target has
- * accepted a path, the drafter's per-layer caches get rows for the accepted positions.
+/* Sec. 2.4, "Update and Iterate": the paper appends the accepted tokens and updates the
+ * target's cache; the drafter's per-layer caches are read as needing rows for the accepted
+ * positions too, before the next draft attends to them. Once the target has accepted a
+ * path, this commit step gives them those rows.
  * Row i (0 <= i < n) sits at sequence position P + i; its inputs are feat[i] ([3d], the
  * target's fused features of the position before it) and tok[i] (the token at P + i). It
  * goes through Eq. 1 and the cascade exactly like a drafted row (no LM head): layer l

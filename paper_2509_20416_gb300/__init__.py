@@ -94,6 +94,9 @@ _lib.fe_lm_head_topk_noalloc.argtypes = [_vp, _vp, _i32, _i32, ctypes.c_float, _
 _lib.fe_lm_head_topk_noalloc.restype = ctypes.c_int
 _lib.fe_profile_forward.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _i32, _vp, _vp, ctypes.POINTER(_i32)]
 _lib.fe_profile_forward.restype = ctypes.c_int
+_lib.fe_profile_graph.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, _i32, _vp, _vp, _vp,
+                                  ctypes.POINTER(_i32)]
+_lib.fe_profile_graph.restype = ctypes.c_int
 _lib.fe_draft_loss.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, ctypes.c_float, ctypes.c_float,
                                ctypes.c_float, _vp, _vp, _vp, _vp]
 _lib.fe_draft_loss.restype = ctypes.c_int
@@ -220,7 +223,8 @@ def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, to
     return out
 
 
-FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "copy", 5: "linear_prep"}
+FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "copy", 5: "linear_prep",
+                   6: "tree"}
 
 
 def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
@@ -244,6 +248,50 @@ def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
     _check(_lib.fe_profile_forward(h.ptr, ctypes.byref(a), _stream(stream), cap, ctypes.cast(kinds, _vp),
                                    ctypes.cast(usec, _vp), ctypes.byref(n)), "fe_profile_forward")
     return [(FE_KERNEL_NAMES.get(kinds[j], str(kinds[j])), float(usec[j])) for j in range(n.value)]
+
+
+def fe_profile_graph(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
+                     temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
+                     tree: dict | None = None, stream=None) -> list[tuple[str, float, float]]:
+    """One draft (plus the tree kernel when ``tree`` is given) run as the CUDA graph
+    fe_draft_forward uses, with every kernel's first start and last exit stamped on the GPU
+    (include/fe_draft.h). Returns [(kernel family, start us, end us)] in launch order, times
+    from the run's earliest start."""
+    B = int(next_tok.shape[0])
+    if out is None:
+        out = alloc_outputs(h, B, top_k, feat.device)
+    N = h.cfg["n_layers"]
+    kc = (_vp * N)(*[_dp(t) for t in k_cache])
+    vc = (_vp * N)(*[_dp(t) for t in v_cache])
+    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
+                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
+                        _dp(out["topk_prob"]), _dp(out["lse"]), None, None)
+    t = None
+    if tree is not None:
+        t = fe_tree(_dp(tree["tok"]), _dp(tree["parent"]), _dp(tree["depth"]), _dp(tree["mask"]))
+    cap = fe_launch_count(h, B, tree is not None) + 1
+    kinds = (_i32 * cap)()
+    t0 = (ctypes.c_double * cap)()
+    t1 = (ctypes.c_double * cap)()
+    n = _i32(0)
+    _check(_lib.fe_profile_graph(h.ptr, ctypes.byref(a), ctypes.byref(t) if t is not None else None, _stream(stream),
+                                 cap, ctypes.cast(kinds, _vp), ctypes.cast(t0, _vp), ctypes.cast(t1, _vp),
+                                 ctypes.byref(n)), "fe_profile_graph")
+    return [(FE_KERNEL_NAMES.get(kinds[j], str(kinds[j])), float(t0[j]), float(t1[j])) for j in range(n.value)]
+
+
+def in_step_times(launches: list[tuple[str, float, float]]) -> list[tuple[str, float, float]]:
+    """[(family, span us, added us)] from fe_profile_graph's stamps: the span is a launch's
+    first start to last exit; the added time is how far its end lies past the previous
+    launch's end (the first launch: its span), so the added times partition the step."""
+    res, prev_end = [], None
+    for kind, s, e in launches:
+        if s < 0 or e < 0:
+            continue
+        add = (e - s) if prev_end is None else max(0.0, e - prev_end)
+        res.append((kind, e - s, add))
+        prev_end = e if prev_end is None else max(prev_end, e)
+    return res
 
 
 def fe_draft_loss(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, teacher_p, target_feat, top_k: int,

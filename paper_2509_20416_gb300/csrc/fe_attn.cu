@@ -74,6 +74,7 @@ __device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int
 
 template <typename CT, int HD, int G>
 __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a, int S) {
+    const LaunchStamp stamp(a.stamp);
     constexpr int HALF = HD / 2;
     constexpr int DPL = HD / 32;                  // dims per lane
     constexpr int KB = 32 / G;                    // keys per score batch (KB * G = 32 scores)
@@ -535,6 +536,7 @@ __device__ __forceinline__ void cp_async_wait() {
 
 template <int G>
 __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnArgs a) {
+    const LaunchStamp stamp(a.stamp);
     using CT = bf16_t;
     constexpr int HD = 128;
     constexpr int HALF = HD / 2;

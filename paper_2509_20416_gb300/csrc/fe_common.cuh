@@ -66,6 +66,25 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
     return t;
 }
 
+// ---- in-graph launch timing ------------------------------------------------------------
+// When a launch is given a stamp pair p (both words zero before the graph runs), the CTA's
+// thread 0 records its start and each warp's first active lane its exit, as %globaltimer
+// nanoseconds: p[0] = max over CTAs of ~start (so ~p[0] is the earliest start and zero
+// means "never stamped"), p[1] = max over warps of the exit time. Declared first in a
+// kernel, the object's destructor runs on every return path.
+struct LaunchStamp {
+    unsigned long long* p;
+    __device__ __forceinline__ explicit LaunchStamp(unsigned long long* s) : p(s) {
+        if (p && threadIdx.x == 0) atomicMax(p, ~(unsigned long long)globaltimer_ns());
+    }
+    __device__ __forceinline__ ~LaunchStamp() {
+        if (p) {
+            const unsigned m = __activemask();
+            if ((int)(threadIdx.x & 31) == __ffs(m) - 1) atomicMax(p + 1, (unsigned long long)globaltimer_ns());
+        }
+    }
+};
+
 // ---- mbarrier -------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);

@@ -79,6 +79,9 @@ struct LinearArgs {
     int slots;           // streaming kernel: pipeline slots per warp (0: the default)
     int* status;
     bool pdl;  // launch overlapping the previous kernel (programmatic dependent launch)
+    // in-graph timing (fe_profile_graph): the (start, end) stamp pair of this phase's
+    // first kernel, the next kernel of the phase at stamp + 2; null when not profiling
+    unsigned long long* stamp = nullptr;
 };
 
 struct DeviceInfo {
@@ -147,6 +150,9 @@ struct LmHeadArgs {
     float* lse;         // [B, N]
     int* status;
     bool pdl;
+    // in-graph timing: stamp pairs of the head's kernels (operand prep, product, merge in
+    // that order; the CUDA-core head uses the first); null when not profiling
+    unsigned long long* stamp = nullptr;
 };
 cudaError_t lmhead_prepare(const DeviceInfo& dev);
 int lmhead_slabs(int V, const DeviceInfo& dev);
@@ -187,10 +193,14 @@ struct LmHeadView {
     float eps;
     int* status;
     DeviceInfo dev;
+    int device;  // the CUDA device the handle's memory lives on
 };
 bool handle_lmhead_view(const fe_handle* h, LmHeadView* v);
 // record a message for fe_last_error_detail() (calling thread)
 void set_error_detail(const char* msg);
+// fe_noalloc.cu: look up the allocation-free LM head's scratch array on the current device
+// (once per device; called by fe_draft_init with the handle's device current)
+cudaError_t noalloc_resolve_scratch(int device);
 
 // ---- decode attention ----------------------------------------------------------------
 struct AttnArgs {
@@ -213,6 +223,7 @@ struct AttnArgs {
     // n_rows[b] <= pos_add are skipped (a commit of accepted rows)
     int row_stride = 1, row_off = 0, pos_add = 0;
     const int* n_rows = nullptr;
+    unsigned long long* stamp = nullptr;  // in-graph timing stamp pair, or null
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();
@@ -221,7 +232,7 @@ inline int attention_launches() { return 1; }
 
 // ---- draft tree + failure-detection probe ------------------------------------------------
 cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,
-                        int* depth, uint8_t* mask, int* status, cudaStream_t st);
+                        int* depth, uint8_t* mask, int* status, cudaStream_t st, unsigned long long* stamp = nullptr);
 cudaError_t launch_timeout_probe(int64_t timeout_ns, int* status, cudaStream_t st);
 // commit (fe_commit.cu): gather rows i0 .. i0 + nb - 1 of every sequence into a dense block
 cudaError_t launch_commit_gather(const void* feat, const int* tok, const int* n_rows, int B, int L, int i0, int nb,

@@ -46,6 +46,7 @@ struct LinearEpi {
 
 template <typename WT, int BT>
 __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int D) {
+    const LaunchStamp stamp(a.stamp);
     extern __shared__ __align__(128) unsigned char smem[];
     const int Kpad = (a.K + 3) & ~3;
     const int b0 = blockIdx.y * BT;
@@ -77,6 +78,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearA
 // partition, same order of operations).
 template <typename WT, int BT>
 __global__ void __launch_bounds__(kStreamThreads, 1) stack_kernel(const StackArgs sa, int D, int Kpad_max) {
+    const LaunchStamp stamp(sa.ph[0].stamp);
     extern __shared__ __align__(128) unsigned char smem[];
     StreamSmem s = carve_stream_smem(smem, D, 1, Kpad_max, BT);
     int issued = 0;

@@ -56,6 +56,7 @@ __device__ __forceinline__ void split_bf16(float z, uint16_t& hi, uint16_t& lo) 
 constexpr int kXprepChunks = 256;  // 16-byte chunks per CTA (one per thread)
 
 __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
+    const LaunchStamp stamp(a.stamp);
     const int b = blockIdx.x, t = threadIdx.x;
     const int N = 2 * B_pad, K = a.K, nc = K / 8;
     __shared__ float red[8];
@@ -185,6 +186,7 @@ template <int BP>  // B_pad: 8, 16, 24 or 32
 __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearArgs a, const uint16_t* xb, int S,
                                                                    int stage_bytes, uint32_t tmem_cols, float* part,
                                                                    int* counters) {
+    const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     constexpr int N = 2 * BP;
     extern __shared__ unsigned char dsm_raw[];
     __shared__ LinMmaState st;

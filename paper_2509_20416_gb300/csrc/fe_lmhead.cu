@@ -357,6 +357,7 @@ __host__ __device__ inline size_t merge_smem_bytes(int nwarps, int n_slabs, int 
 
 template <typename WT, int BT>
 __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadArgs a, int D, size_t smem_bytes) {
+    const LaunchStamp stamp(a.stamp);
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ TopkState st;
     const int K = a.d;
@@ -444,7 +445,9 @@ template <typename WT>
 // and is deliberately not a __restrict__ pointer, whose loads the compiler may treat as
 // invariant and move above the wait.
 __global__ void __launch_bounds__(256) zprep_kernel(const float* hid, const WT* __restrict__ gamma, int R,
-                                                    int R_pad, int d, float eps, uint16_t* zb, int with_lo) {
+                                                    int R_pad, int d, float eps, uint16_t* zb, int with_lo,
+                                                    unsigned long long* stamp_pair) {
+    const LaunchStamp stamp(stamp_pair);
     static_assert(sizeof(WT) == 2, "the tensor-core LM head takes bf16 weights");
     const int r = blockIdx.x, t = threadIdx.x;
     const int N = with_lo ? 2 * R_pad : R_pad;
@@ -524,6 +527,7 @@ struct MmaState {
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
                                                                     int S, int stage_bytes, uint32_t tmem_cols,
                                                                     int slab_cap) {
+    const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     extern __shared__ unsigned char dsm_raw[];
     __shared__ MmaState st;
     // 1024-byte aligned ring (the 128B swizzle pattern is a function of address bits 4..9),
@@ -674,7 +678,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                         }
                         __nanosleep(64);
                     }
-                    a.split_flag[blockIdx.x + 1] = 0;  // (read again only by the next launch)
+                    // (lmhead_merge_kernel clears the flags once every CTA has exited)
                 }
                 if (!epi_sync()) break;
                 const float* p = a.split_part + ((size_t)(blockIdx.x + 1) * 128 + tr) * R_pad;
@@ -820,7 +824,7 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     const int R_pad = (a.R + 7) / 8 * 8;
     const int N = 2 * R_pad;
     cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
-                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 1);
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 1, a.stamp);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int stage_bytes = (16384 + N * 128 + 1023) / 1024 * 1024;
@@ -995,6 +999,7 @@ struct WideRow {
 template <int KM>
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
                                                                      int S, int stage_bytes, uint32_t tmem_cols) {
+    const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     extern __shared__ unsigned char dsm_raw[];
     __shared__ WideState st;
     unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
@@ -1129,9 +1134,15 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
 
 // One CTA per row: merges every slab's partial of that row (merge_rows).
 __global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, size_t smem_bytes) {
+    const LaunchStamp stamp(a.stamp ? a.stamp + 4 : nullptr);
     extern __shared__ __align__(16) unsigned char msm[];
     griddep_launch_dependents();
     griddep_wait();
+    // Every CTA of the product kernel has exited, so no split-tile flag can be set after
+    // this: clear them for the next launch here (a CTA that gave up waiting on a flag
+    // cannot leave it set for the next launch to take as ready).
+    if (a.split_flag && blockIdx.x == 0)
+        for (int j = threadIdx.x; j < a.n_slabs; j += blockDim.x) a.split_flag[j] = 0;
     merge_rows(a, blockIdx.x, blockIdx.x + 1, msm, smem_bytes);
 }
 
@@ -1166,7 +1177,7 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
     if (!lmhead_wide_ok(a) || (reinterpret_cast<uintptr_t>(a.hid) & 15)) return cudaErrorInvalidValue;
     const int R_pad = (a.R + 15) / 16 * 16;
     cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
-                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 0);
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 0, a.stamp);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int stage_bytes = 16384 + R_pad * 128;

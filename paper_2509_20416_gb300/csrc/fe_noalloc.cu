@@ -8,17 +8,23 @@
 // (and final RMSNorm gain) that fe_draft_init already packed into the handle, takes the
 // hidden rows and the outputs from the caller, and keeps its working memory (per-slab
 // partial results, completion counters and the tensor-core operand) in one file-scope
-// __device__ array of a fixed size, reserved when the library is loaded on a device and
-// held until the process exits.
+// __device__ array of a fixed size, held until the process exits.
+//
+// When the array is reserved: fe_draft_init looks up its device address with
+// cudaGetSymbolAddress, once per device, with that device current. Under CUDA's lazy
+// module loading (the default since CUDA 12.2, CUDA_MODULE_LOADING=LAZY) that lookup is
+// what loads this file's module and reserves the array, so the memory is taken inside
+// fe_draft_init, which allocates anyway; with CUDA_MODULE_LOADING=EAGER it is reserved
+// when the library's modules load on the device. Either way no call of
+// fe_lm_head_topk_noalloc allocates or looks anything up.
 //
 // Limits: at most kMaxRows hidden rows (n_layers * B), d <= kMaxD, top_k <= 32.
 // Sharing: every call uses the same array and leaves its contents behind. Calls that may
 // overlap on the GPU (different streams, or different host threads) race with each other
 // and must be serialised by the caller. The completion counters, which must start at
 // zero, are cleared by every call.
-// First call per device: it looks up the array's device address with
-// cudaGetSymbolAddress (once per device, with that device current); make that first call
-// before any stream capture.
+// Device: the call must be made with the handle's device current (the array, the LM head
+// and the status word it uses all live there); otherwise it returns FE_ERR_INVALID_ARG.
 #include <cstdio>
 #include <mutex>
 
@@ -50,6 +56,18 @@ unsigned char* g_scratch_dev[kMaxDevices] = {};  // device address of g_scratch,
 
 using namespace fe;
 
+cudaError_t fe::noalloc_resolve_scratch(int device) {
+    if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (g_scratch_dev[device]) return cudaSuccess;
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+    if (e != cudaSuccess) return e;
+    if (!p) return cudaErrorInvalidSymbol;
+    g_scratch_dev[device] = (unsigned char*)p;
+    return cudaSuccess;
+}
+
 extern "C" FE_API fe_status fe_lm_head_topk_noalloc(fe_handle* h, const float* hidden, int32_t B, int32_t top_k,
                                                     float temperature, int32_t* topk_id, float* topk_logit,
                                                     float* topk_prob, float* lse, void* stream) {
@@ -61,25 +79,37 @@ extern "C" FE_API fe_status fe_lm_head_topk_noalloc(fe_handle* h, const float* h
         return FE_ERR_INVALID_ARG;
     if (!(temperature == temperature)) return FE_ERR_INVALID_ARG;
     const int R = v.N * B;
-    if (R > kMaxRows || v.d > kMaxD || v.n_slabs > kMaxSlabs) {
-        char msg[200];
+    char msg[200];
+    if (R > kMaxRows || v.d > kMaxD) {
         snprintf(msg, sizeof(msg),
                  "fe_lm_head_topk_noalloc: n_layers*B = %d (max %d) or d = %d (max %d) exceeds its fixed scratch", R,
                  kMaxRows, v.d, kMaxD);
         set_error_detail(msg);
         return FE_ERR_INVALID_ARG;
     }
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FE_ERR_CUDA;
+    if (v.n_slabs > kMaxSlabs) {
+        snprintf(msg, sizeof(msg),
+                 "fe_lm_head_topk_noalloc: the LM head's %d vocabulary slabs exceed its fixed scratch (max %d)",
+                 v.n_slabs, kMaxSlabs);
+        set_error_detail(msg);
+        return FE_ERR_INVALID_ARG;
+    }
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return FE_ERR_CUDA;
+    if (dev != v.device) {
+        snprintf(msg, sizeof(msg), "fe_lm_head_topk_noalloc: the current CUDA device (%d) is not the handle's (%d)",
+                 dev, v.device);
+        set_error_detail(msg);
+        return FE_ERR_INVALID_ARG;
+    }
     unsigned char* base = nullptr;
     {
         std::lock_guard<std::mutex> lock(g_mu);
-        if (!g_scratch_dev[dev]) {
-            void* p = nullptr;
-            if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return FE_ERR_CUDA;
-            g_scratch_dev[dev] = (unsigned char*)p;
-        }
-        base = g_scratch_dev[dev];
+        base = dev >= 0 && dev < kMaxDevices ? g_scratch_dev[dev] : nullptr;
+    }
+    if (!base) {  // fe_draft_init resolved it for the handle's device; this does not happen
+        set_error_detail("fe_lm_head_topk_noalloc: the scratch array was not resolved for this device");
+        return FE_ERR_CUDA;
     }
     cudaStream_t st = (cudaStream_t)stream;
     LmHeadArgs lm{};

@@ -130,6 +130,14 @@ struct fe_handle {
     bool use_graph = true;
     bool use_pdl = true;
     std::vector<cudaEvent_t> prof_ev;  // fe_profile_forward's events (created on first use)
+    // fe_profile_graph: the stamp pairs (device, allocated on first use), the stamped
+    // graph and what it was captured for
+    unsigned long long* prof_stamps = nullptr;
+    int prof_stamp_cap = 0;
+    cudaGraphExec_t pexec = nullptr;
+    GraphKey pkey;
+    fe_tree ptree{};
+    std::vector<int32_t> pkinds;
     // fe_draft_step_host: pinned staging of a step's inputs and outputs, their device
     // copies (sized for max_batch and top_k_max) and the step's graph
     unsigned char *hs_in = nullptr, *hs_out = nullptr, *ds_in = nullptr, *ds_out = nullptr;
@@ -156,6 +164,21 @@ fe_status fail(cudaError_t e, const char* what, int line) {
         cudaError_t _e = (call);                           \
         if (_e != cudaSuccess) return fail(_e, #call, __LINE__); \
     } while (0)
+
+// Every call that enqueues work requires the handle's device to be the calling thread's
+// current device: the handle's weights, scratch and status word live there, and a launch
+// on another device would reach them across devices (or fault).
+fe_status check_device(const fe_handle* h) {
+    int dev = -1;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(e, "cudaGetDevice", __LINE__);
+    if (dev != h->device) {
+        snprintf(g_detail, sizeof(g_detail), "the current CUDA device (%d) is not the handle's device (%d)", dev,
+                 h->device);
+        return FE_ERR_INVALID_ARG;
+    }
+    return FE_OK;
+}
 
 bool valid_config(const fe_config* c) {
     if (!c) return false;
@@ -185,10 +208,13 @@ struct Sizes {
     size_t w_fuse, w_in, embed, lm_head, norm, qkv, wo, gu, down;
 };
 
-// fe_profile_forward's recorder: ev[0] is recorded before the first launch and ev[j + 1]
-// after launch j, whose family is kinds[j]
+// The profilers' recorder. Event mode (fe_profile_forward, ev set): ev[0] is recorded
+// before the first launch and ev[j + 1] after launch j. Stamp mode (fe_profile_graph,
+// stamps set): launch j gets the stamp pair stamps + 2 j. Either way launch j's family is
+// kinds[j].
 struct Prof {
     cudaEvent_t* ev;
+    unsigned long long* stamps;
     int32_t* kinds;
     int cap, n;
 };
@@ -197,7 +223,13 @@ inline cudaError_t mark(Prof* pf, int kind, cudaStream_t st) {
     if (!pf) return cudaSuccess;
     if (pf->n >= pf->cap) return cudaErrorInvalidValue;
     pf->kinds[pf->n] = kind;
-    return cudaEventRecord(pf->ev[++pf->n], st);
+    ++pf->n;
+    return pf->ev ? cudaEventRecord(pf->ev[pf->n], st) : cudaSuccess;
+}
+
+// the stamp pair of the next launch (stamp mode), else null
+inline unsigned long long* next_stamp(const Prof* pf) {
+    return pf && pf->stamps && pf->n < pf->cap ? pf->stamps + 2 * (size_t)pf->n : nullptr;
 }
 
 // bytes of each matrix in the tile-packed layout (rows padded to a multiple of 4); the
@@ -230,13 +262,13 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     const int B = a->B, d = c.d, H = c.n_heads, Hkv = c.n_kv_heads, hd = c.head_dim, F = c.ffn, V = c.vocab;
     const int N = c.n_layers, nqkv = (H + 2 * Hkv) * hd;
     const fe_dtype dt = c.dtype;
-    const bool pdl = h->use_pdl && !pf;  // profiled launches do not overlap
+    const bool pdl = h->use_pdl && !(pf && pf->ev);  // event-profiled launches do not overlap
     const bool stacked = h->use_stack && B == 1;
     if (stacked) {
         // the stacks' barrier counters start at zero in every draft
         FE_TRY(cudaMemsetAsync(h->stack_bar, 0, (size_t)(N + 1) * sizeof(uint32_t), st));
     }
-    if (pf) FE_TRY(cudaEventRecord(pf->ev[0], st));
+    if (pf && pf->ev) FE_TRY(cudaEventRecord(pf->ev[0], st));
     // one linear phase: the CUDA-core streaming kernel, or operand prep + tensor-core product
     // persistent stacks: linear phases are queued and launched together at the next
     // attention (or at the LM head)
@@ -246,6 +278,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     auto flush_stack = [&]() -> fe_status {
         if (sq.nph == 0) return FE_OK;
         sq.barrier = h->stack_bar + nstack;
+        sq.ph[0].stamp = next_stamp(pf);
         cudaError_t e = launch_stack(dt, sq, h->dev, st);
         if (e != cudaSuccess) return fail(e, "linear stack launch", __LINE__);
         if ((e = mark(pf, FE_KERNEL_LINEAR, st)) != cudaSuccess) return fail(e, "profiling event", __LINE__);
@@ -253,8 +286,10 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         ++nstack;
         return FE_OK;
     };
-    auto linear = [&](const LinearArgs& L) -> fe_status {
+    auto linear = [&](const LinearArgs& L0) -> fe_status {
         cudaError_t e;
+        LinearArgs L = L0;
+        L.stamp = stacked ? nullptr : next_stamp(pf);
         if (stacked) {
             if (sq.nph == kMaxStackPhases) {
                 const fe_status r = flush_stack();
@@ -268,7 +303,8 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
                 if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
                 pf->kinds[pf->n++] = FE_KERNEL_LINEAR_PREP;
             }
-            e = launch_linear_mma(L, h->lin_xb, h->lin_part, h->lin_counters, h->dev, st, pf ? pf->ev[pf->n] : nullptr);
+            e = launch_linear_mma(L, h->lin_xb, h->lin_part, h->lin_counters, h->dev, st,
+                                  pf && pf->ev ? pf->ev[pf->n] : nullptr);
         } else {
             e = launch_linear(dt, L, h->dev, st);
         }
@@ -326,6 +362,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
         if ((lrc = flush_stack()) != FE_OK) return lrc;
+        aa.stamp = next_stamp(pf);
         FE_TRY(launch_attention(dt, aa, st));
         FE_TRY(mark(pf, FE_KERNEL_ATTENTION, st));
         // x += W_o o
@@ -356,6 +393,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
     lm.pdl = pdl;
+    lm.stamp = next_stamp(pf);
     if (h->lm_mma && N * B <= 16) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         lm.split_part = h->lm_split_part;  // (tile, column block) units split evenly over the CTAs
@@ -366,8 +404,8 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
             pf->kinds[pf->n + 1] = FE_KERNEL_LM_HEAD;
             pf->n += 2;
         }
-        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n - 1] : nullptr,
-                                 pf ? pf->ev[pf->n] : nullptr));
+        FE_TRY(launch_lmhead_mma(lm, h->lm_zb, h->dev, st, pf && pf->ev ? pf->ev[pf->n - 1] : nullptr,
+                                 pf && pf->ev ? pf->ev[pf->n] : nullptr));
         FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     } else if (h->lm_mma) {
         lm.n_slabs = lmhead_wide_slabs(V, h->dev);
@@ -377,8 +415,8 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
             pf->kinds[pf->n + 1] = FE_KERNEL_LM_HEAD;
             pf->n += 2;
         }
-        FE_TRY(launch_lmhead_wide(lm, h->lm_zb, h->dev, st, pf ? pf->ev[pf->n - 1] : nullptr,
-                                  pf ? pf->ev[pf->n] : nullptr));
+        FE_TRY(launch_lmhead_wide(lm, h->lm_zb, h->dev, st, pf && pf->ev ? pf->ev[pf->n - 1] : nullptr,
+                                  pf && pf->ev ? pf->ev[pf->n] : nullptr));
         FE_TRY(mark(pf, FE_KERNEL_LM_HEAD, st));
     } else {
         FE_TRY(launch_lmhead(dt, lm, h->dev, st));
@@ -492,6 +530,8 @@ void release(fe_handle* h) {
     if (!h) return;
     for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
     if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    if (h->pexec) cudaGraphExecDestroy(h->pexec);
+    if (h->prof_stamps) cudaFree(h->prof_stamps);
     if (h->hexec) cudaGraphExecDestroy(h->hexec);
     if (h->hs_in) cudaFreeHost(h->hs_in);
     if (h->hs_out) cudaFreeHost(h->hs_out);
@@ -522,6 +562,7 @@ bool fe::handle_lmhead_view(const fe_handle* h, LmHeadView* v) {
     v->eps = h->cfg.rms_eps;
     v->status = h->status;
     v->dev = h->dev;
+    v->device = h->device;
     return true;
 }
 
@@ -578,6 +619,9 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         if ((rc = from_cuda(lmhead_mma_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(linear_mma_prepare(h->dev))) != FE_OK) break;
         if ((rc = from_cuda(lmhead_wide_prepare(h->dev))) != FE_OK) break;
+        // the allocation-free LM head's fixed scratch array: its address on this device is
+        // looked up here, so that entry point itself never loads a module or allocates
+        if ((rc = from_cuda(noalloc_resolve_scratch(h->device))) != FE_OK) break;
         // the linear phases run on the tensor cores for batched handles (bf16, every K a
         // multiple of 64, at most kLinMmaMaxBatch sequences); FE_DRAFT_LINEAR_MMA=1 / 0
         // forces the choice where the shapes allow it
@@ -789,6 +833,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
 
 fe_status fe_draft_forward(fe_handle* h, const fe_forward_args* a, void* stream) {
     if (!forward_args_ok(h, a)) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     const fe_config& c = h->cfg;
     cudaStream_t st = (cudaStream_t)stream;
     try {
@@ -828,6 +874,8 @@ fe_status fe_profile_forward(fe_handle* h, const fe_forward_args* a, void* strea
                              float* usec, int32_t* n_launches) {
     if (!forward_args_ok(h, a) || !kinds || !usec || !n_launches || cap < 1 || cap > 4096) return FE_ERR_INVALID_ARG;
     if (cap < fe_launch_count(h, a->B, 0) + (a->dbg_hidden ? 1 : 0)) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     cudaStream_t st = (cudaStream_t)stream;
     try {
         while ((int)h->prof_ev.size() < cap + 1) {
@@ -835,7 +883,7 @@ fe_status fe_profile_forward(fe_handle* h, const fe_forward_args* a, void* strea
             FE_TRY(cudaEventCreate(&e));
             h->prof_ev.push_back(e);
         }
-        Prof pf{h->prof_ev.data(), kinds, cap, 0};
+        Prof pf{h->prof_ev.data(), nullptr, kinds, cap, 0};
         const fe_status rc = enqueue_forward(h, a, st, &pf);
         if (rc != FE_OK) {
             cudaStreamSynchronize(st);
@@ -848,6 +896,94 @@ fe_status fe_profile_forward(fe_handle* h, const fe_forward_args* a, void* strea
             usec[j] = 1000.f * ms;
         }
         *n_launches = pf.n;
+        return FE_OK;
+    } catch (...) {
+        return FE_ERR_OOM;
+    }
+}
+
+fe_status fe_profile_graph(fe_handle* h, const fe_forward_args* a, const fe_tree* tree, void* stream, int32_t cap,
+                           int32_t* kinds, double* start_us, double* end_us, int32_t* n_launches) {
+    if (!forward_args_ok(h, a) || !kinds || !start_us || !end_us || !n_launches || cap < 1 || cap > 4096)
+        return FE_ERR_INVALID_ARG;
+    if (tree && (!tree->tok || !tree->parent || !tree->depth || !tree->mask)) return FE_ERR_INVALID_ARG;
+    const int need = fe_launch_count(h, a->B, tree ? 1 : 0) + (a->dbg_hidden ? 1 : 0);
+    if (cap < need) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
+    const fe_config& c = h->cfg;
+    cudaStream_t st = (cudaStream_t)stream;
+    try {
+        if (h->prof_stamp_cap < need) {
+            if (h->pexec) {
+                cudaGraphExecDestroy(h->pexec);
+                h->pexec = nullptr;
+            }
+            if (h->prof_stamps) cudaFree(h->prof_stamps);
+            h->prof_stamps = nullptr;
+            h->prof_stamp_cap = 0;
+            FE_TRY(cudaMalloc(&h->prof_stamps, (size_t)2 * need * sizeof(unsigned long long)));
+            h->prof_stamp_cap = need;
+        }
+        GraphKey key;
+        key.args = *a;
+        key.args.k_cache = nullptr;
+        key.args.v_cache = nullptr;
+        key.kc.assign(a->k_cache, a->k_cache + c.n_layers);
+        key.vc.assign(a->v_cache, a->v_cache + c.n_layers);
+        const fe_tree tk = tree ? *tree : fe_tree{};
+        const bool same_tree = tk.tok == h->ptree.tok && tk.parent == h->ptree.parent && tk.depth == h->ptree.depth &&
+                               tk.mask == h->ptree.mask;
+        if (!h->pexec || !(key == h->pkey) || !same_tree) {
+            // the same launch sequence as fe_draft_forward's graph (programmatic launches
+            // included), each kernel given its stamp pair; the pairs are cleared first
+            h->pkinds.assign(need, -1);
+            Prof pf{nullptr, h->prof_stamps, h->pkinds.data(), need, 0};
+            cudaGraph_t graph = nullptr;
+            FE_TRY(cudaStreamBeginCapture(h->cap, cudaStreamCaptureModeThreadLocal));
+            fe_status rc = FE_OK;
+            cudaError_t e = cudaMemsetAsync(h->prof_stamps, 0, (size_t)2 * need * sizeof(unsigned long long), h->cap);
+            if (e != cudaSuccess) rc = fail(e, "stamp clear", __LINE__);
+            if (rc == FE_OK) rc = enqueue_forward(h, a, h->cap, &pf);
+            if (rc == FE_OK && tree) {
+                unsigned long long* sp = next_stamp(&pf);
+                e = launch_tree(a->B, c.n_layers, a->top_k, c.vocab, a->next_tok, a->topk_id, tk.tok, tk.parent,
+                                tk.depth, tk.mask, h->status, h->cap, sp);
+                if (e == cudaSuccess) e = mark(&pf, FE_KERNEL_TREE, h->cap);
+                if (e != cudaSuccess) rc = fail(e, "tree launch", __LINE__);
+            }
+            e = cudaStreamEndCapture(h->cap, &graph);
+            if (rc != FE_OK) {
+                if (graph) cudaGraphDestroy(graph);
+                return rc;
+            }
+            FE_TRY(e);
+            cudaGraphExec_t ex = nullptr;
+            e = cudaGraphInstantiate(&ex, graph, 0);
+            cudaGraphDestroy(graph);
+            FE_TRY(e);
+            if (h->pexec) cudaGraphExecDestroy(h->pexec);
+            h->pexec = ex;
+            h->pkey = key;
+            h->ptree = tk;
+            h->pkinds.resize(pf.n);
+        }
+        FE_TRY(cudaGraphLaunch(h->pexec, st));
+        const int n = (int)h->pkinds.size();
+        std::vector<unsigned long long> raw((size_t)2 * n);
+        FE_TRY(cudaMemcpyAsync(raw.data(), h->prof_stamps, raw.size() * sizeof(unsigned long long),
+                               cudaMemcpyDeviceToHost, st));
+        FE_TRY(cudaStreamSynchronize(st));
+        unsigned long long t0 = ~0ull;
+        for (int j = 0; j < n; ++j)
+            if (raw[2 * j]) t0 = std::min(t0, ~raw[2 * j]);
+        for (int j = 0; j < n; ++j) {
+            kinds[j] = h->pkinds[j];
+            const bool ok = raw[2 * j] != 0 && raw[2 * j + 1] != 0;
+            start_us[j] = ok ? (double)(~raw[2 * j] - t0) * 1e-3 : -1.0;
+            end_us[j] = ok ? (double)(raw[2 * j + 1] - t0) * 1e-3 : -1.0;
+        }
+        *n_launches = n;
         return FE_OK;
     } catch (...) {
         return FE_ERR_OOM;
@@ -901,6 +1037,8 @@ fe_status fe_draft_step_host(fe_handle* h, const fe_host_step_args* a, void* str
         if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
     if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
     if (!(a->temperature == a->temperature)) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     cudaStream_t st = (cudaStream_t)stream;
     const StepLayout L = step_layout(c, h->es, a->B, a->top_k);
     const size_t B = (size_t)a->B, N = (size_t)c.n_layers, k = (size_t)a->top_k, T = 1 + N * k;
@@ -964,6 +1102,8 @@ fe_status fe_build_tree(fe_handle* h, int32_t B, int32_t top_k, const int32_t* n
     if (!h || !out || !next_tok || !topk_id) return FE_ERR_INVALID_ARG;
     if (!out->tok || !out->parent || !out->depth || !out->mask) return FE_ERR_INVALID_ARG;
     if (B < 1 || B > h->cfg.max_batch || top_k < 1 || top_k > h->cfg.top_k_max) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     FE_TRY(launch_tree(B, h->cfg.n_layers, top_k, h->cfg.vocab, next_tok, topk_id, out->tok, out->parent, out->depth,
                        out->mask, h->status, (cudaStream_t)stream));
     return FE_OK;
@@ -975,7 +1115,7 @@ fe_status fe_draft_loss(fe_handle* h, const fe_forward_args* a, const float* tea
         !feat_loss || !total)
         return FE_ERR_INVALID_ARG;
     if (!(alpha == alpha) || !(beta == beta) || !(decay == decay)) return FE_ERR_INVALID_ARG;
-    const fe_status rc = fe_draft_forward(h, a, stream);
+    const fe_status rc = fe_draft_forward(h, a, stream);  // (checks the device)
     if (rc != FE_OK) return rc;
     const fe_config& c = h->cfg;
     FE_TRY(launch_loss(c.n_layers, a->B, c.vocab, c.d, a->dbg_logits, teacher_p, a->dbg_hidden, target_feat, alpha,
@@ -989,6 +1129,8 @@ fe_status fe_verify_greedy(fe_handle* h, int32_t B, int32_t top_k, const int32_t
     if (!h || !tree || !prefix_len || !target_next || !pos_ids || !path || !n_accept || !bonus) return FE_ERR_INVALID_ARG;
     if (!tree->tok || !tree->parent || !tree->depth) return FE_ERR_INVALID_ARG;
     if (B < 1 || B > h->cfg.max_batch || top_k < 1 || top_k > h->cfg.top_k_max) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     const int N = h->cfg.n_layers, T = 1 + N * top_k;
     FE_TRY(launch_verify(B, T, N, prefix_len, tree->tok, tree->parent, tree->depth, target_next, pos_ids, path,
                          n_accept, bonus, (cudaStream_t)stream));
@@ -1004,6 +1146,8 @@ fe_status fe_commit(fe_handle* h, const fe_commit_args* a, void* stream) {
         if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
     if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(a->feat) & 15) return FE_ERR_INVALID_ARG;  // copied as 16-byte vectors
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     try {
         return enqueue_commit(h, a, (cudaStream_t)stream);
     } catch (...) {
@@ -1013,6 +1157,8 @@ fe_status fe_commit(fe_handle* h, const fe_commit_args* a, void* stream) {
 
 fe_status fe_last_device_status(fe_handle* h, void* stream) {
     if (!h) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     cudaStream_t st = (cudaStream_t)stream;
     int v = 0;
     FE_TRY(cudaStreamSynchronize(st));
@@ -1026,8 +1172,14 @@ fe_status fe_last_device_status(fe_handle* h, void* stream) {
 
 void fe_free(fe_handle* h) {
     if (!h) return;
+    // release on the handle's device, whichever device the caller has current
+    int cur = -1;
+    const bool have_cur = cudaGetDevice(&cur) == cudaSuccess;
+    if (have_cur && cur != h->device) cudaSetDevice(h->device);
     cudaDeviceSynchronize();
+    const int dev = h->device;
     release(h);
+    if (have_cur && cur != dev) cudaSetDevice(cur);
 }
 
 const char* fe_last_error_detail(void) { return g_detail; }
@@ -1045,6 +1197,8 @@ int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
 
 fe_status fe_selftest_timeout(fe_handle* h, int64_t timeout_ns, void* stream) {
     if (!h || timeout_ns < 1000 || timeout_ns > 1000000000LL) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
     FE_TRY(launch_timeout_probe(timeout_ns, h->status, (cudaStream_t)stream));
     return FE_OK;
 }

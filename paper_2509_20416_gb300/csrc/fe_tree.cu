@@ -14,7 +14,9 @@
 namespace fe {
 
 __global__ void tree_kernel(int N, int k, int V, const int* __restrict__ next_tok, const int* __restrict__ topk_id,
-                            int* tok, int* parent, int* depth, uint8_t* mask, int* status) {
+                            int* tok, int* parent, int* depth, uint8_t* mask, int* status,
+                            unsigned long long* stamp_pair) {
+    const LaunchStamp stamp(stamp_pair);
     const int b = blockIdx.x;
     const int T = 1 + N * k;
     bool bad = false;
@@ -47,8 +49,8 @@ __global__ void tree_kernel(int N, int k, int V, const int* __restrict__ next_to
 }
 
 cudaError_t launch_tree(int B, int N, int k, int V, const int* next_tok, const int* topk_id, int* tok, int* parent,
-                        int* depth, uint8_t* mask, int* status, cudaStream_t st) {
-    tree_kernel<<<B, 256, 0, st>>>(N, k, V, next_tok, topk_id, tok, parent, depth, mask, status);
+                        int* depth, uint8_t* mask, int* status, cudaStream_t st, unsigned long long* stamp) {
+    tree_kernel<<<B, 256, 0, st>>>(N, k, V, next_tok, topk_id, tok, parent, depth, mask, status, stamp);
     return cudaGetLastError();
 }
 

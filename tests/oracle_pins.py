@@ -196,7 +196,8 @@ def pin_topk(orc):
 
 
 def pin_topk_sample(orc):
-    """Stochastic drafting (Sec. 2.2 "sample k candidates", reading C16): the counter-based
+    """Stochastic drafting (Sec. 2.2 "sample k candidates", read as k draws without
+    replacement by the Gumbel-top-k trick): the counter-based
     deviates, the law of the draws without replacement, and the order the tree uses."""
     # SplitMix64 seeded with 0: its first outputs as published (Steele et al. 2014)
     for n, want in enumerate([0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F], start=1):
@@ -529,7 +530,8 @@ def _sampled_trees(orc, N, k, V, drafter_logits, R, seed):
 
 
 def pin_accept_sampled(orc):
-    """Lossless verification of a sampled tree (Sec. 2.4, reading C17): with a one-hot
+    """Lossless verification of a sampled tree (Sec. 2.4, read as recursive rejection
+    sampling over the children in draw order): with a one-hot
     target it is the greedy walk; with the target equal to the drafter it accepts the first
     draw; and every emitted token has the target's law (Monte Carlo on a 4-token vocabulary,
     5 sigma), which a wrong test ratio, residual, proposal update or test order breaks."""

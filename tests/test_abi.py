@@ -68,6 +68,7 @@ def test_profile_entry_point_validates_on_host(lib):
     so = lib._lib
     n = ctypes.c_int32(0)
     assert so.fe_profile_forward(None, None, None, 8, None, None, ctypes.byref(n)) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_profile_graph(None, None, None, None, 8, None, None, None, ctypes.byref(n)) == lib.FE_ERR_INVALID_ARG
 
 
 def test_next_row_entry_points_validate_on_host(lib):

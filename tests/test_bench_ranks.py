@@ -94,3 +94,25 @@ def test_reference_arm_prints_one_contract_line():
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"] == {"value": line["value"], "unit": "drafts/s", "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
+
+
+def test_in_step_times_partition_the_stamped_span():
+    """fe_profile_graph's stamps -> per-launch added time: with programmatic launches the
+    spans overlap, and each launch is charged only the time its end lies past the previous
+    end, so the charges sum to the run's span; bench.py folds operand preps into their
+    phase's family."""
+    sys.path.insert(0, ROOT)
+    import importlib
+    fe_binding = importlib.import_module("paper_2509_20416_gb300")
+    import bench
+    stamps = [("linear", 0.0, 10.0), ("attention", 8.0, 13.0), ("linear", 9.0, 20.0), ("lm_prep", 19.5, 21.0),
+              ("lm_head", 20.0, 30.0), ("lm_head", 29.0, 31.0), ("copy", -1.0, -1.0), ("tree", 31.0, 31.5)]
+    its = fe_binding.in_step_times(stamps)
+    assert [k for k, _, _ in its] == ["linear", "attention", "linear", "lm_prep", "lm_head", "lm_head", "tree"]
+    assert [a for _, _, a in its] == pytest.approx([10.0, 3.0, 7.0, 1.0, 9.0, 1.0, 0.5])
+    assert sum(a for _, _, a in its) == pytest.approx(31.5)
+    fam = bench.family_times(its + its, 2)
+    assert fam["linear"]["launches_per_draft"] == 2 and fam["linear"]["us_per_draft"] == pytest.approx(17.0)
+    assert fam["lm_head"]["launches_per_draft"] == 2 and fam["lm_head"]["us_per_draft"] == pytest.approx(11.0)
+    assert sum(v["us_per_draft"] for v in fam.values()) == pytest.approx(31.5)
+    assert fam["linear"]["span_us_per_draft"] == pytest.approx(21.0)

@@ -7,3 +7,23 @@ import oracle_pins as pins
 @pytest.mark.parametrize("pin", pins.ALL_PINS, ids=lambda f: f.__name__)
 def test_pin(orc, pin):
     pin(orc)
+
+
+def test_lm_head_binding_reproduces_the_draft(orc):
+    """Oracle.lm_head (the LM head over given hidden rows, used to check the allocation-free
+    LM head) hands or_lm_head the right buffers: on a draft's own hidden states it returns
+    that draft's logits exactly, and the final norm's gain enters (a gain of 2 doubles the
+    logits)."""
+    import numpy as np
+    import torch
+    from fe_synth import workloads as wl
+    cfg = wl.make_config(dict(d=64, n_heads=2, n_kv_heads=1, head_dim=32, ffn=96, vocab=300, n_layers=3,
+                              dtype="bf16", B=1, prefix=5, top_k=4, rope_theta=1e4, seed=9, page_size=0))
+    W, I = wl.make_weights(cfg), wl.make_inputs(cfg)
+    ks, vs = wl.make_caches(cfg)
+    o = orc.draft_seq(cfg, W, I["feat"][0].contiguous(), int(I["next_tok"][0]), int(I["prefix_len"][0]),
+                      [k[0].contiguous() for k in ks], [v[0].contiguous() for v in vs], cfg["max_seq"], 4)
+    lg = orc.lm_head(cfg, W, o["hidden"])
+    assert np.array_equal(lg, o["logits"])
+    W2 = dict(W, final_norm=torch.full_like(W["final_norm"], 2.0))
+    assert np.allclose(orc.lm_head(cfg, W2, o["hidden"]), 2.0 * o["logits"], rtol=1e-12, atol=1e-12)

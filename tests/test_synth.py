@@ -122,3 +122,7 @@ def test_roofline_bytes_and_flops_count_the_generated_tensors(monkeypatch, name)
     flops = 2 * sum(t.numel() for t in mats) * B + 2 * W["lm_head"].numel() * N * B
     flops += N * sum(4 * H * hd * (p + 1) for p in plen)
     assert wl.algorithmic_flops(cfg, plen) == flops
+    fparts = wl.kernel_flops(cfg, plen)
+    assert sum(fparts.values()) == flops
+    assert fparts["lm_head"] == 2 * W["lm_head"].numel() * N * B
+    assert fparts["attention"] == N * sum(4 * H * hd * (p + 1) for p in plen)

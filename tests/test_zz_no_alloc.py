@@ -38,7 +38,7 @@ def _setup(case):
 
 
 @pytest.mark.parametrize("case", list(CASES))
-def test_noalloc_lm_head_matches_forward_twice(case):
+def test_noalloc_lm_head_matches_forward_twice(case, orc):
     fe, cfg, h, I, ks, vs = _setup(case)
     B, N, d, k, T = cfg["B"], cfg["n_layers"], cfg["d"], cfg["top_k"], cfg["temperature"]
     hidden = torch.empty((N, B, d), device="cuda")
@@ -55,7 +55,34 @@ def test_noalloc_lm_head_matches_forward_twice(case):
             assert torch.allclose(out[key], ref[key], rtol=1e-6, atol=1e-6), (call, key)
         ids = out["topk_id"].cpu().numpy()
         assert ((ids >= 0) & (ids < cfg["vocab"])).all()
+    # and against the fp64 oracle's LM head over the same hidden rows (the final norm, the
+    # logits, their softmax at T and the top-k), under the parity contract
+    _check_against_oracle(orc, cfg, h, hidden, out)
     h.close()
+
+
+def _check_against_oracle(orc, cfg, h, hidden, out):
+    import numpy as np
+    import harness as H
+    W = wl.make_weights(cfg)
+    B, N, k, T = cfg["B"], cfg["n_layers"], cfg["top_k"], cfg["temperature"]
+    hid = hidden.cpu().numpy().astype(np.float64)  # [N, B, d]
+    lg = orc.lm_head(cfg, W, hid.reshape(N * B, -1)).reshape(N, B, -1)
+    ids, tl, tp, lse = (out[key].cpu().numpy() for key in ("topk_id", "topk_logit", "topk_prob", "lse"))
+    for b in range(B):
+        for i in range(N):
+            ref = lg[i, b]
+            p_ref, lse_ref = orc.softmax(ref, T if T > 0 else 1.0)
+            H.check_topk(ids[b, i], ref, k)
+            if cfg["dtype"] == "f32":
+                scale = np.abs(ref).max()
+                assert abs(lse[b, i] - lse_ref) <= H.TOL_F32_REL * abs(lse_ref), (b, i)
+                assert np.abs(tl[b, i] - ref[ids[b, i]]).max() <= H.TOL_F32_REL * scale, (b, i)
+                assert np.abs(tp[b, i] - p_ref[ids[b, i]]).max() <= H.TOL_F32_REL * max(1e-3, p_ref.max()), (b, i)
+            else:
+                assert abs(lse[b, i] - lse_ref) <= H.TOL_BF16_LOGIT, (b, i)
+                assert np.abs(tl[b, i] - ref[ids[b, i]]).max() <= H.TOL_BF16_LOGIT, (b, i)
+                assert np.abs(tp[b, i] - p_ref[ids[b, i]]).max() <= H.TOL_BF16_PROB, (b, i)
 
 
 def test_noalloc_rejects_more_rows_than_its_scratch_holds():
