@@ -364,6 +364,37 @@ def measure(args, name: str, overrides, ws: int, rank: int, local: int, extras: 
     value = job_rate(ws, B, ms_step / 1e3)
     check("after the timed region")
 
+    # ---- the same step with stochastic drafting at T = 1 (Sec. 2.2, "sample k candidates") --
+    # (outside the headline: its cost next to the greedy step)
+    def step_sampled():
+        fe.fe_draft_forward(h, feat, tok, plen, kd, vd, k, 1.0, page_table=table, n_pages=n_pages, out=out,
+                            stream=stream, sample=True, seed=0x5EED)
+        fe.fe_build_tree(h, tok, out["topk_id"], k, out=tree, stream=stream)
+
+    for _ in range(3):
+        step_sampled()
+    n_smp = max(3, args.steps // 4)
+    barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(n_smp):
+        step_sampled()
+    e1.record(stream)
+    e1.synchronize()
+    ms_smp = max_over_ranks(e0.elapsed_time(e1), ws, "cuda") / n_smp
+    smp_launches = []
+    for _ in range(5):
+        smp_launches.extend(fe.in_step_times(fe.fe_profile_graph(
+            h, feat, tok, plen, kd, vd, k, 1.0, page_table=table, n_pages=n_pages, out=out, tree=tree,
+            stream=stream, sample=True, seed=0x5EED)))
+    smp_fam = family_times(smp_launches, 5)
+    check("after the sampled steps")
+    sampled = {"temperature": 1.0, "seed": 0x5EED, "steps": n_smp, "ms_per_step": ms_smp,
+               "value": job_rate(ws, B, ms_smp / 1e3), "unit": "drafts/s",
+               "lm_head_us_per_draft": smp_fam.get("lm_head", {}).get("us_per_draft"),
+               "note": "the same step with sample=1 (Gumbel-top-k draws without replacement at T = 1); "
+                       "lm_head_us_per_draft from GPU stamps inside the replayed graph"}
+
     # ---- end to end through the public API with host buffers ------------------------------
     # fe_draft_step_host: host inputs -> (pinned staging -> device copy, draft, tree, device
     # -> pinned copy, as one CUDA graph) -> host outputs; the call returns with the outputs
@@ -437,7 +468,7 @@ def measure(args, name: str, overrides, ws: int, rank: int, local: int, extras: 
                    "call": "fe_draft_step_host (host inputs and outputs; copies, draft and tree in one graph; "
                            "returns with the outputs in host memory)"},
            "gpu_launches": launches_per_step * args.steps, "launches_per_step": launches_per_step,
-           "clocks": clocks}
+           "clocks": clocks, "sampled": sampled}
     rec.update(extra)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         rate, runs, thr, el = time_oracle(cfg, W, I, ks, vs, args.cpu_seconds)
@@ -470,6 +501,32 @@ def time_extras(fe, h, cfg, wl, feat, tok, plen, kd, vd, table, n_pages, tree, s
     verify_us = 1000.0 * v0.elapsed_time(v1) / 100
 
     V, d = cfg["vocab"], cfg["d"]
+    # lossless verification of a sampled tree (fe_verify_sampled): a T = 1 sampled draft's tree,
+    # draw ranks and q = softmax(logits), synthetic target distributions per node
+    smp = fe.alloc_outputs(h, B, k)
+    logits = torch.empty((B, N, V), device="cuda")
+    fe.fe_draft_forward(h, feat, tok, plen, kd, vd, k, 1.0, page_table=table, n_pages=n_pages, out=smp,
+                        dbg_logits=logits, stream=stream, sample=True, seed=0x5EED)
+    stree = fe.fe_build_tree(h, tok, smp["topk_id"], k, stream=stream)
+    q = torch.softmax(logits, dim=-1)
+    nxt = torch.clamp(stree["depth"], max=N - 1).long()
+    p = torch.softmax(logits[torch.arange(B, device="cuda")[:, None], nxt]
+                      + 0.5 * torch.randn((B, T, V), generator=g).cuda(), dim=-1)
+    u_acc = torch.rand((B, T), generator=g).clamp(1e-7, 1 - 1e-7).cuda()
+    u_bonus = torch.rand((B, T), generator=g).clamp(1e-7, 1 - 1e-7).cuda()
+    vs_out = fe.fe_verify_sampled(h, stree, smp["topk_rank"], q, p, u_acc, u_bonus, k, stream=stream)
+    for _ in range(3):
+        fe.fe_verify_sampled(h, stree, smp["topk_rank"], q, p, u_acc, u_bonus, k, out=vs_out, stream=stream)
+    v0.record(stream)
+    for _ in range(20):
+        fe.fe_verify_sampled(h, stree, smp["topk_rank"], q, p, u_acc, u_bonus, k, out=vs_out, stream=stream)
+    v1.record(stream)
+    v1.synchronize()
+    verify_sampled_us = 1000.0 * v0.elapsed_time(v1) / 20
+    accepted = int(vs_out["n_accept"].sum())
+    del p, q, logits
+    check("after the sampled verification")
+
     teacher = torch.softmax(torch.randn((B, N, V), generator=g), dim=-1).cuda()
     target_feat = torch.randn((N, B, d), generator=g).cuda()
     for _ in range(3):
@@ -501,6 +558,10 @@ def time_extras(fe, h, cfg, wl, feat, tok, plen, kd, vd, table, n_pages, tree, s
     check("after the commits")
     return {"verify_greedy": {"us_per_call": verify_us, "sequences": B, "tree_nodes": T,
                               "note": "fe_verify_greedy after the step (positions + greedy acceptance walk)"},
+            "verify_sampled": {"us_per_call": verify_sampled_us, "sequences": B, "tree_nodes": T,
+                               "accepted_tokens": accepted,
+                               "note": "fe_verify_sampled on a T = 1 sampled draft's tree (recursive rejection "
+                                       "sampling in draw order, Sec. 2.4); synthetic target distributions"},
             "commit": {"us_per_call": commit_us, "rows_per_sequence": N,
                        "note": "fe_commit of N accepted rows per sequence (Sec. 2.4 Update and Iterate): "
                                "Eq. 1 and the cascade over the rows, one weight stream per 32 rows; "

@@ -116,10 +116,20 @@ typedef struct {
  *             are ignored), n_pages the pool size (paged only)
  *  top_k      candidates per depth, 1..top_k_max
  *  temperature  T > 0 scales the reported probabilities and lse as softmax(logit / T);
- *             T <= 0 (greedy) reports the T = 1 distribution. Candidates are always the
- *             k largest logits, ties broken by the smaller token id.
+ *             T <= 0 (greedy) reports the T = 1 distribution. Unless sample is set, the
+ *             candidates are the k largest logits, ties broken by the smaller token id.
+ *  sample, seed  stochastic drafting (Sec. 2.2, "sample k candidates"). sample != 0 needs
+ *             T > 0: depth i's candidates of sequence b are then k draws without replacement
+ *             from softmax(logit / T), taken as the k largest keys logit_v / T + G_v
+ *             (Gumbel-top-k), G_v = -log(-log U_v) and U_v = (floor(x / 2^41) + 1/2) / 2^23,
+ *             where x is output n = (b N + i - 1) V + v + 1 of SplitMix64 seeded with `seed`
+ *             (Steele, Lea and Flood 2014). The drawn set is reported ordered by logit like
+ *             the greedy candidates (descending, ties to the smaller id), so the tree rule is
+ *             unchanged: the most probable drawn token is the backbone.
  * Outputs (device, float32 unless stated):
  *  topk_id [B, N, top_k] int32, topk_logit [B, N, top_k], topk_prob [B, N, top_k], lse [B, N]
+ *  topk_rank [B, N, top_k] int32 or NULL: each candidate's position in draw order (0 =
+ *             drawn first, i.e. the largest key); r for the r-th greedy candidate
  *  dbg_logits [B, N, V] or NULL: full logits, for parity checks only (costs V floats a row)
  *  dbg_hidden [N, B, d] or NULL: the cascade's hidden states h_i
  */
@@ -136,6 +146,9 @@ typedef struct {
     int32_t *topk_id;
     float *topk_logit, *topk_prob, *lse;
     float *dbg_logits, *dbg_hidden;
+    int32_t sample;
+    uint64_t seed;
+    int32_t *topk_rank;
 } fe_forward_args;
 
 /* The draft tree of B sequences, device buffers with T = 1 + N * top_k nodes each:
@@ -187,6 +200,8 @@ FE_API fe_status fe_build_tree(fe_handle *h, int32_t B, int32_t top_k, const int
  *  topk_id [B, N, top_k] int32, topk_logit, topk_prob [B, N, top_k] float32, lse [B, N]
  *    float32, tree_tok, tree_parent, tree_depth [B, T] int32, tree_mask [B, T, T] uint8
  *    (T = 1 + N top_k): HOST outputs, as fe_draft_forward and fe_build_tree define them
+ *  sample, seed: stochastic drafting, as in fe_forward_args; topk_rank [B, N, top_k] int32:
+ *    HOST output of the draw positions, or NULL
  *
  * The call synchronises `stream` and returns once the outputs are in host memory. Errors:
  * FE_ERR_INVALID_ARG (null pointer, B or top_k out of range), FE_ERR_CUDA / FE_ERR_OOM;
@@ -205,6 +220,9 @@ typedef struct {
     float *topk_logit, *topk_prob, *lse;
     int32_t *tree_tok, *tree_parent, *tree_depth;
     uint8_t *tree_mask;
+    int32_t sample;
+    uint64_t seed;
+    int32_t *topk_rank;
 } fe_host_step_args;
 
 FE_API fe_status fe_draft_step_host(fe_handle *h, const fe_host_step_args *args, void *stream);
@@ -257,10 +275,40 @@ FE_API fe_status fe_draft_loss(fe_handle *h, const fe_forward_args *args, const 
  *   next token, which a cycle emits in addition.
  * All pointers are device pointers (tree: tok, parent and depth are read; mask is not);
  * target_next [B, T] int32. Asynchronous on `stream`; FE_ERR_INVALID_ARG for bad arguments.
- * Stochastic (T > 0) speculative sampling over the tree is not covered. */
+ * Stochastic (T > 0) verification of a sampled tree is fe_verify_sampled. */
 FE_API fe_status fe_verify_greedy(fe_handle *h, int32_t B, int32_t top_k, const int32_t *prefix_len,
                                   const fe_tree *tree, const int32_t *target_next, int32_t *pos_ids,
                                   int32_t *path, int32_t *n_accept, int32_t *bonus, void *stream);
+
+/* Lossless verification of a SAMPLED draft tree (Sec. 2.4: the target verifies the tree and
+ * speculative sampling finds the longest accepted path; the paper names no variant), the
+ * counterpart of fe_verify_greedy for stochastic drafting. Read as recursive rejection
+ * sampling over each node's children in draw order (the multi-candidate form of
+ * speculative sampling, matching candidates drawn without replacement). For each sequence
+ * b, from the root: with r = the target's distribution after the current node and s = the
+ * drafter's proposal of the next depth, the children are tested in draw order; child c
+ * with token x is accepted iff u_acc[b, c] * s(x) <= r(x); on rejection r becomes
+ * max(r - s, 0) renormalised and x leaves s (renormalised). An accepted child becomes the
+ * current node (r its distribution); the walk ends when every child is rejected, the node
+ * has none, or N tokens are accepted, and the bonus token is the smallest x with
+ * u_bonus[b, current] < r(0) + ... + r(x) (the last token with r > 0 if rounding leaves the
+ * sum below u). Every emitted token then has the target's law.
+ *  tree      fe_build_tree's tree (tok, parent, depth read), T = 1 + N top_k nodes
+ *  topk_rank device [B, N, top_k] int32, fe_draft_forward's draw positions: node c >= 1 of
+ *            the tree has draw position topk_rank[b][c - 1] (nodes in level-major order)
+ *  q         device [B, N, V] float32: the drafter's proposal at each depth, softmax(l_i / T)
+ *  p         device [B, T, V] float32: the target's next-token distribution after each node
+ *            (given its root path), at the same temperature
+ *  u_acc, u_bonus  device [B, T] float32 uniform deviates in (0, 1)
+ *  path      device [B, N] int32: accepted node ids, -1 after n_accept[b]
+ *  n_accept  device [B] int32; bonus device [B] int32
+ * Asynchronous on `stream`; FE_ERR_INVALID_ARG for bad host-side arguments; a token or depth
+ * out of range in the tree ends that sequence's walk and sets FE_ERR_DEVICE in the status
+ * word. The handle holds one V-float residual buffer per sequence for it. */
+FE_API fe_status fe_verify_sampled(fe_handle *h, int32_t B, int32_t top_k, const fe_tree *tree,
+                                   const int32_t *topk_rank, const float *q, const float *p, const float *u_acc,
+                                   const float *u_bonus, int32_t *path, int32_t *n_accept, int32_t *bonus,
+                                   void *stream);
 
 /* The update step of a cycle (Sec. 2.4, "Update and Iterate"): before the next draft can
  * attend to the positions the target accepted, each layer's cache needs their rows. For

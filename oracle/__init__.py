@@ -122,7 +122,8 @@ class Oracle:
         L.or_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
         L.or_uniform.restype = ctypes.c_double
         L.or_accept_sampled.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _I, _I, _I,
-                                        _I, _D, _D, _D, _D, _I, _I, _I]
+                                        _I, _D, _D, _D, _D, _I, _I, _I, _D]
+        L.or_sample_keys.argtypes = [_D, ctypes.c_int64, ctypes.c_double, ctypes.c_uint64, ctypes.c_int64, _D]
         L.or_topk_sample_rows.argtypes = [_D, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_double,
                                           ctypes.c_uint64, ctypes.c_int64, _I, _I]
         L.or_commit_seq.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(_P), _P, _I, ctypes.c_int32,
@@ -207,11 +208,20 @@ class Oracle:
                                    drawn.ctypes.data_as(i32))
         return (ids[0], drawn[0]) if one else (ids, drawn)
 
-    def accept_sampled(self, tok, parent, depth, rank, q, p, u_acc, u_bonus):
+    def sample_keys(self, logits, T: float, seed: int, row: int) -> np.ndarray:
+        """The keys logits / T + G of topk_sample's draw for one row (the value the draw
+        ranks by), [V] float64."""
+        lg = np.ascontiguousarray(logits, dtype=np.float64).reshape(-1)
+        key = np.zeros_like(lg)
+        self.L.or_sample_keys(_dp(lg), lg.size, float(T), seed, row, _dp(key))
+        return key
+
+    def accept_sampled(self, tok, parent, depth, rank, q, p, u_acc, u_bonus, want_margin: bool = False):
         """Lossless verification of B sampled trees (Sec. 2.4; recursive rejection
         sampling over each node's children in draw order): tok, parent,
         depth, rank [B, T] int; q [B, N, V], p [B, T, V], u_acc, u_bonus [B, T] float.
-        Returns (path [B, N] with -1 after the accepted nodes, n_accept [B], bonus [B])."""
+        Returns (path [B, N] with -1 after the accepted nodes, n_accept [B], bonus [B]), and
+        with want_margin each sequence's closest decision margin [B] (probability units)."""
         i32 = ctypes.POINTER(ctypes.c_int32)
         tok, parent, depth, rank = (np.ascontiguousarray(a, dtype=np.int32) for a in (tok, parent, depth, rank))
         q, p, u_acc, u_bonus = (np.ascontiguousarray(a, dtype=np.float64) for a in (q, p, u_acc, u_bonus))
@@ -221,10 +231,11 @@ class Oracle:
         path = np.zeros((B, N), np.int32)
         n = np.zeros(B, np.int32)
         bonus = np.zeros(B, np.int32)
+        margin = np.zeros(B)
         self.L.or_accept_sampled(B, T, N, V, *(a.ctypes.data_as(i32) for a in (tok, parent, depth, rank)),
                                  _dp(q), _dp(p), _dp(u_acc), _dp(u_bonus), path.ctypes.data_as(i32),
-                                 n.ctypes.data_as(i32), bonus.ctypes.data_as(i32))
-        return path, n, bonus
+                                 n.ctypes.data_as(i32), bonus.ctypes.data_as(i32), _dp(margin))
+        return (path, n, bonus, margin) if want_margin else (path, n, bonus)
 
     def tree(self, N, k, root, topk):
         topk = np.ascontiguousarray(topk, dtype=np.int32).reshape(N, k)

@@ -365,18 +365,24 @@ double or_uniform(uint64_t seed, uint64_t n)
  *   ids[k]:   the same k tokens by descending logit (ties: ascending id), so that ids[0],
  *             the most probable candidate, is the one the Backbone Expansion tree extends
  *             (Sec. 2.2). */
-void or_topk_sample(const double *logits, int64_t V, int32_t k, double T, uint64_t seed, int64_t row,
-                    int32_t *ids, int32_t *drawn)
+/* The keys of the draw above: key[v] = logits[v] / T + G_v for row `row`. */
+void or_sample_keys(const double *logits, int64_t V, double T, uint64_t seed, int64_t row, double *key)
 {
-    double *key = (double *)malloc((size_t)V * sizeof(double));
-    int32_t *d = (int32_t *)malloc((size_t)k * sizeof(int32_t));
-    unsigned char *taken = (unsigned char *)calloc((size_t)V, 1);
     for (int64_t v = 0; v < V; ++v) {
         const uint64_t n = MUT(38) ? (uint64_t)v + 1 : (uint64_t)row * (uint64_t)V + (uint64_t)v + 1;
         const double u = or_uniform(seed, n);
         const double g = MUT(37) ? log(-log(u)) : -log(-log(u));
         key[v] = (MUT(39) ? logits[v] : logits[v] / T) + g;
     }
+}
+
+void or_topk_sample(const double *logits, int64_t V, int32_t k, double T, uint64_t seed, int64_t row,
+                    int32_t *ids, int32_t *drawn)
+{
+    double *key = (double *)malloc((size_t)V * sizeof(double));
+    int32_t *d = (int32_t *)malloc((size_t)k * sizeof(int32_t));
+    unsigned char *taken = (unsigned char *)calloc((size_t)V, 1);
+    or_sample_keys(logits, V, T, seed, row, key);
     for (int32_t r = 0; r < k; ++r) {
         int64_t best = -1;
         for (int64_t v = 0; v < V; ++v)
@@ -542,11 +548,20 @@ int32_t or_accept_greedy(int32_t T, const int32_t *tok, const int32_t *parent, c
  * current node. When every child is rejected, or the node has none, the bonus token is drawn
  * from r by inverse CDF: the smallest x with u_bonus[current] < r(0) + ... + r(x).
  * path[b][0..n) are the accepted node ids (-1 after), n_accept[b] = n, bonus[b] the drawn
- * token. Every emitted token then has the target's law. */
+ * token. Every emitted token then has the target's law.
+ * margin[b] (or NULL): how far the sequence's closest decision was from going the other way,
+ * in units of the error bound of a float32 walk: |u_acc * s(x) - r(x)| for a test, and the
+ * distance of u_bonus to the nearer edge of the picked token's CDF interval, each divided by
+ * E = 2^-24 (2 S / Z + 5). Z is the current residual's normaliser (1 for a target
+ * distribution itself) and S bounds the error mass a float32 residual carries: 0 for a
+ * target distribution; each rejection adds at most 5 roundings of mass one (r, s and their
+ * difference, each summing to at most 1) after dividing what it carried by the normaliser it
+ * consumed, S <- S / Z + 5 2^-24. A float32 walk with exact sums can only decide differently
+ * where the margin is below 1. The margin does not enter the walk. */
 void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t *tok, const int32_t *parent,
                        const int32_t *depth, const int32_t *rank, const double *q, const double *p,
                        const double *u_acc, const double *u_bonus, int32_t *path, int32_t *n_accept,
-                       int32_t *bonus)
+                       int32_t *bonus, double *margin)
 {
 #pragma omp parallel for schedule(static)
     for (int32_t b = 0; b < B; ++b) {
@@ -556,6 +571,9 @@ void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t
         double *s = (double *)malloc((size_t)V * sizeof(double));
         int32_t *kids = (int32_t *)malloc((size_t)T * sizeof(int32_t));
         int32_t cur = 0, n = 0;
+        double closest = INFINITY;
+        const double ulp = 1.0 / 16777216.0;  /* 2^-24 */
+        double zcur = 1.0, serr = 0.0;        /* the error model of the margin (see above) */
         memcpy(r, p + ((int64_t)b * T + cur) * V, (size_t)V * sizeof(double));
         for (;;) {
             /* the children of cur, in draw order */
@@ -580,6 +598,8 @@ void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t
                 const int32_t c = kids[i], x = tk[c];
                 const int accept = MUT(41) ? u_acc[(int64_t)b * T + c] * r[x] <= s[x]
                                            : u_acc[(int64_t)b * T + c] * s[x] <= r[x];
+                closest = fmin(closest, fabs(u_acc[(int64_t)b * T + c] * s[x] - r[x]) /
+                                            (ulp * (2.0 * serr / zcur + 5.0)));
                 if (accept) {
                     next = c;
                     break;
@@ -590,6 +610,8 @@ void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t
                     r[v] = (MUT(42) || dlt > 0.0) ? dlt : 0.0;
                     sr += r[v];
                 }
+                serr = serr / zcur + 5.0;  /* in units of 2^-24 */
+                zcur = sr > 0.0 ? sr : 1.0;
                 if (sr > 0.0)
                     for (int64_t v = 0; v < V; ++v)
                         r[v] /= sr;
@@ -605,6 +627,8 @@ void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t
                 break;
             path[(int64_t)b * N + n++] = next;
             cur = next;
+            zcur = 1.0;
+            serr = 0.0;
             memcpy(r, p + ((int64_t)b * T + cur) * V, (size_t)V * sizeof(double));
         }
         for (int32_t i = n; i < N; ++i)
@@ -618,10 +642,16 @@ void or_accept_sampled(int32_t B, int32_t T, int32_t N, int64_t V, const int32_t
             if (r[v] > 0.0)
                 last = (int32_t)v;
             cum += r[v];
-            if (u < cum)
+            if (u < cum) {
                 pick = (int32_t)v;
+                closest = fmin(closest, fmin(u - (cum - r[v]), cum - u) / (ulp * (2.0 * serr / zcur + 5.0)));
+            }
         }
+        if (pick < 0)
+            closest = fmin(closest, (u - cum) / (ulp * (2.0 * serr / zcur + 5.0)));
         bonus[b] = pick >= 0 ? pick : last; /* u above a sum rounded below 1 */
+        if (margin)
+            margin[b] = closest;
         free(kids);
         free(s);
         free(r);

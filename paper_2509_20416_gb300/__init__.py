@@ -54,7 +54,8 @@ class fe_forward_args(ctypes.Structure):
                 ("k_cache", ctypes.POINTER(_vp)), ("v_cache", ctypes.POINTER(_vp)),
                 ("page_table", _vp), ("n_pages", _i32),
                 ("topk_id", _vp), ("topk_logit", _vp), ("topk_prob", _vp), ("lse", _vp),
-                ("dbg_logits", _vp), ("dbg_hidden", _vp)]
+                ("dbg_logits", _vp), ("dbg_hidden", _vp), ("sample", _i32), ("seed", ctypes.c_uint64),
+                ("topk_rank", _vp)]
 
 
 class fe_tree(ctypes.Structure):
@@ -71,7 +72,8 @@ class fe_host_step_args(ctypes.Structure):
     _fields_ = [("B", _i32), ("top_k", _i32), ("temperature", ctypes.c_float), ("feat", _vp), ("next_tok", _vp),
                 ("prefix_len", _vp), ("k_cache", ctypes.POINTER(_vp)), ("v_cache", ctypes.POINTER(_vp)),
                 ("page_table", _vp), ("n_pages", _i32), ("topk_id", _vp), ("topk_logit", _vp), ("topk_prob", _vp),
-                ("lse", _vp), ("tree_tok", _vp), ("tree_parent", _vp), ("tree_depth", _vp), ("tree_mask", _vp)]
+                ("lse", _vp), ("tree_tok", _vp), ("tree_parent", _vp), ("tree_depth", _vp), ("tree_mask", _vp),
+                ("sample", _i32), ("seed", ctypes.c_uint64), ("topk_rank", _vp)]
 
 
 _lib.fe_draft_init.argtypes = [ctypes.POINTER(fe_config), ctypes.POINTER(fe_weights), _vp, ctypes.POINTER(_vp)]
@@ -102,6 +104,9 @@ _lib.fe_draft_loss.argtypes = [_vp, ctypes.POINTER(fe_forward_args), _vp, _vp, c
 _lib.fe_draft_loss.restype = ctypes.c_int
 _lib.fe_verify_greedy.argtypes = [_vp, _i32, _i32, _vp, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp]
 _lib.fe_verify_greedy.restype = ctypes.c_int
+_lib.fe_verify_sampled.argtypes = [_vp, _i32, _i32, ctypes.POINTER(fe_tree), _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                   _vp]
+_lib.fe_verify_sampled.restype = ctypes.c_int
 _lib.fe_draft_step_host.argtypes = [_vp, ctypes.POINTER(fe_host_step_args), _vp]
 _lib.fe_draft_step_host.restype = ctypes.c_int
 _lib.fe_commit.argtypes = [_vp, ctypes.POINTER(fe_commit_args), _vp]
@@ -202,23 +207,37 @@ def alloc_outputs(h: Handle, B: int, top_k: int, device="cuda") -> dict:
     return dict(topk_id=torch.empty((B, N, top_k), dtype=torch.int32, device=device),
                 topk_logit=torch.empty((B, N, top_k), dtype=torch.float32, device=device),
                 topk_prob=torch.empty((B, N, top_k), dtype=torch.float32, device=device),
-                lse=torch.empty((B, N), dtype=torch.float32, device=device))
+                lse=torch.empty((B, N), dtype=torch.float32, device=device),
+                topk_rank=torch.empty((B, N, top_k), dtype=torch.int32, device=device))
+
+
+def _forward_args(h: Handle, feat, next_tok, prefix_len, kc, vc, top_k, temperature, page_table, n_pages, out,
+                  dbg_logits, dbg_hidden, sample, seed) -> fe_forward_args:
+    a = fe_forward_args(int(next_tok.shape[0]), top_k, float(temperature), _dp(feat), _dp(next_tok),
+                        _dp(prefix_len), kc, vc, _dp(page_table), int(n_pages), _dp(out["topk_id"]),
+                        _dp(out["topk_logit"]), _dp(out["topk_prob"]), _dp(out["lse"]), _dp(dbg_logits),
+                        _dp(dbg_hidden))
+    a.sample = 1 if sample else 0
+    a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF
+    a.topk_rank = _dp(out.get("topk_rank"))
+    return a
 
 
 def fe_draft_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
                      temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
-                     dbg_logits=None, dbg_hidden=None, stream=None) -> dict:
+                     dbg_logits=None, dbg_hidden=None, stream=None, sample: bool = False, seed: int = 0) -> dict:
     """One draft. feat [B, 3d], next_tok [B] i32, prefix_len [B] i32 (device tensors);
-    k_cache / v_cache: lists of per-layer device tensors (see include/fe_draft.h)."""
+    k_cache / v_cache: lists of per-layer device tensors (see include/fe_draft.h). With
+    sample (and temperature > 0) the candidates are drawn (stochastic drafting, seeded by
+    ``seed``); out["topk_rank"] then gives each one's position in draw order."""
     B = int(next_tok.shape[0])
     if out is None:
         out = alloc_outputs(h, B, top_k, feat.device)
     N = h.cfg["n_layers"]
     kc = (_vp * N)(*[_dp(t) for t in k_cache])
     vc = (_vp * N)(*[_dp(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
-                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
-                        _dp(out["topk_prob"]), _dp(out["lse"]), _dp(dbg_logits), _dp(dbg_hidden))
+    a = _forward_args(h, feat, next_tok, prefix_len, kc, vc, top_k, temperature, page_table, n_pages, out,
+                      dbg_logits, dbg_hidden, sample, seed)
     _check(_lib.fe_draft_forward(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_forward")
     return out
 
@@ -229,7 +248,7 @@ FE_KERNEL_NAMES = {0: "linear", 1: "attention", 2: "lm_prep", 3: "lm_head", 4: "
 
 def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
                        temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
-                       dbg_hidden=None, stream=None) -> list[tuple[str, float]]:
+                       dbg_hidden=None, stream=None, sample: bool = False, seed: int = 0) -> list[tuple[str, float]]:
     """One draft launched eagerly with a CUDA event after every launch (include/fe_draft.h).
     Returns [(kernel family, device microseconds)] in launch order."""
     B = int(next_tok.shape[0])
@@ -238,9 +257,8 @@ def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
     N = h.cfg["n_layers"]
     kc = (_vp * N)(*[_dp(t) for t in k_cache])
     vc = (_vp * N)(*[_dp(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
-                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
-                        _dp(out["topk_prob"]), _dp(out["lse"]), None, _dp(dbg_hidden))
+    a = _forward_args(h, feat, next_tok, prefix_len, kc, vc, top_k, temperature, page_table, n_pages, out, None,
+                      dbg_hidden, sample, seed)
     cap = fe_launch_count(h, B, False) + 1
     kinds = (_i32 * cap)()
     usec = (ctypes.c_float * cap)()
@@ -252,7 +270,8 @@ def fe_profile_forward(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
 
 def fe_profile_graph(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int,
                      temperature: float = 0.0, page_table=None, n_pages: int = 0, out: dict | None = None,
-                     tree: dict | None = None, stream=None) -> list[tuple[str, float, float]]:
+                     tree: dict | None = None, stream=None, sample: bool = False,
+                     seed: int = 0) -> list[tuple[str, float, float]]:
     """One draft (plus the tree kernel when ``tree`` is given) run as the CUDA graph
     fe_draft_forward uses, with every kernel's first start and last exit stamped on the GPU
     (include/fe_draft.h). Returns [(kernel family, start us, end us)] in launch order, times
@@ -263,9 +282,8 @@ def fe_profile_graph(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, to
     N = h.cfg["n_layers"]
     kc = (_vp * N)(*[_dp(t) for t in k_cache])
     vc = (_vp * N)(*[_dp(t) for t in v_cache])
-    a = fe_forward_args(B, top_k, float(temperature), _dp(feat), _dp(next_tok), _dp(prefix_len), kc, vc,
-                        _dp(page_table), int(n_pages), _dp(out["topk_id"]), _dp(out["topk_logit"]),
-                        _dp(out["topk_prob"]), _dp(out["lse"]), None, None)
+    a = _forward_args(h, feat, next_tok, prefix_len, kc, vc, top_k, temperature, page_table, n_pages, out, None,
+                      None, sample, seed)
     t = None
     if tree is not None:
         t = fe_tree(_dp(tree["tok"]), _dp(tree["parent"]), _dp(tree["depth"]), _dp(tree["mask"]))
@@ -343,12 +361,14 @@ def alloc_host_step_outputs(h: Handle, B: int, top_k: int) -> dict:
     e = lambda shape, dt: torch.empty(shape, dtype=dt).pin_memory()
     return dict(topk_id=e((B, N, top_k), torch.int32), topk_logit=e((B, N, top_k), torch.float32),
                 topk_prob=e((B, N, top_k), torch.float32), lse=e((B, N), torch.float32),
+                topk_rank=e((B, N, top_k), torch.int32),
                 tree_tok=e((B, T), torch.int32), tree_parent=e((B, T), torch.int32), tree_depth=e((B, T), torch.int32),
                 tree_mask=e((B, T, T), torch.uint8))
 
 
 def fe_draft_step_host(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, top_k: int, temperature: float = 0.0,
-                       page_table=None, n_pages: int = 0, out: dict | None = None, stream=None) -> dict:
+                       page_table=None, n_pages: int = 0, out: dict | None = None, stream=None, sample: bool = False,
+                       seed: int = 0) -> dict:
     """One draft step from and to host memory (include/fe_draft.h): feat [B, 3d], next_tok
     [B], prefix_len [B] are CPU tensors; the caches (and page table) are device tensors.
     Returns CPU tensors topk_id, topk_logit, topk_prob, lse, tree_tok, tree_parent,
@@ -366,6 +386,9 @@ def fe_draft_step_host(h: Handle, feat, next_tok, prefix_len, k_cache, v_cache, 
                           _dp(page_table), int(n_pages), _p(out["topk_id"]), _p(out["topk_logit"]),
                           _p(out["topk_prob"]), _p(out["lse"]), _p(out["tree_tok"]), _p(out["tree_parent"]),
                           _p(out["tree_depth"]), _p(out["tree_mask"]))
+    a.sample = 1 if sample else 0
+    a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF
+    a.topk_rank = _p(out.get("topk_rank"))
     _check(_lib.fe_draft_step_host(h.ptr, ctypes.byref(a), _stream(stream)), "fe_draft_step_host")
     return out
 
@@ -387,6 +410,26 @@ def fe_verify_greedy(h: Handle, prefix_len, tree: dict, target_next, top_k: int,
     _check(_lib.fe_verify_greedy(h.ptr, B, int(top_k), _dp(prefix_len), ctypes.byref(t), _dp(target_next),
                                  _dp(out["pos_ids"]), _dp(out["path"]), _dp(out["n_accept"]), _dp(out["bonus"]),
                                  _stream(stream)), "fe_verify_greedy")
+    return out
+
+
+def fe_verify_sampled(h: Handle, tree: dict, topk_rank, q, p, u_acc, u_bonus, top_k: int, out: dict | None = None,
+                      stream=None) -> dict:
+    """Lossless verification of a sampled tree (include/fe_draft.h): tree from fe_build_tree,
+    topk_rank [B, N, k] int32 (fe_draft_forward's draw positions), q [B, N, V] and p [B, T, V]
+    float32 distributions, u_acc / u_bonus [B, T] float32 uniforms (device tensors). Returns
+    path [B, N], n_accept [B] and bonus [B]."""
+    B = int(topk_rank.shape[0])
+    N = h.cfg["n_layers"]
+    dev = topk_rank.device
+    if out is None:
+        out = dict(path=torch.empty((B, N), dtype=torch.int32, device=dev),
+                   n_accept=torch.empty(B, dtype=torch.int32, device=dev),
+                   bonus=torch.empty(B, dtype=torch.int32, device=dev))
+    t = fe_tree(_dp(tree["tok"]), _dp(tree["parent"]), _dp(tree["depth"]), _dp(tree["mask"]))
+    _check(_lib.fe_verify_sampled(h.ptr, B, int(top_k), ctypes.byref(t), _dp(topk_rank), _dp(q), _dp(p), _dp(u_acc),
+                                  _dp(u_bonus), _dp(out["path"]), _dp(out["n_accept"]), _dp(out["bonus"]),
+                                  _stream(stream)), "fe_verify_sampled")
     return out
 
 

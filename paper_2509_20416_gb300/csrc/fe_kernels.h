@@ -150,6 +150,14 @@ struct LmHeadArgs {
     float* lse;         // [B, N]
     int* status;
     bool pdl;
+    // stochastic drafting (Sec. 2.2): with sample, each row's candidates are the top_k keys
+    // logit * inv_temp + G (fe_sample.cuh) instead of the top_k logits; the partials then
+    // hold keys in part_val and the candidates' logits in part_lg [R, n_slabs, top_k]; the
+    // merge orders the drawn set by logit and writes each one's draw position to topk_rank
+    int sample = 0;
+    unsigned long long seed = 0;
+    float* part_lg = nullptr;
+    int* topk_rank = nullptr;  // [B, N, k] or null
     // in-graph timing: stamp pairs of the head's kernels (operand prep, product, merge in
     // that order; the CUDA-core head uses the first); null when not profiling
     unsigned long long* stamp = nullptr;
@@ -244,5 +252,18 @@ cudaError_t launch_loss(int N, int B, int V, int d, const float* logits, const f
 cudaError_t launch_verify(int B, int T, int max_path, const int* prefix_len, const int* tok, const int* parent,
                           const int* depth, const int* target_next, int* pos, int* path, int* n_accept, int* bonus,
                           cudaStream_t st);
+// lossless verification of a sampled tree (fe_verify.cu): one CTA per sequence
+struct VerifySampledArgs {
+    int T, N, V;
+    const int *tok, *parent, *depth;  // [B, T] trees in fe_build_tree's layout
+    const int* rank;                  // [B, T - 1]: node c >= 1's draw position at rank[c - 1]
+    const float* q;                   // [B, N, V] the drafter's proposal per depth
+    const float* p;                   // [B, T, V] the target's distribution after each node
+    const float *u_acc, *u_bonus;     // [B, T]
+    float* rbuf;                      // [B, V] scratch: each sequence's residual
+    int *path, *n_accept, *bonus;     // [B, N], [B], [B]
+    int* status;
+};
+cudaError_t launch_verify_sampled(const VerifySampledArgs& a, int B, cudaStream_t st);
 
 }  // namespace fe

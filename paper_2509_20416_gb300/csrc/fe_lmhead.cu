@@ -20,6 +20,7 @@
 #include <float.h>
 
 #include "fe_kernels.h"
+#include "fe_sample.cuh"
 #include "fe_stream.cuh"
 #include "fe_tc.cuh"
 
@@ -66,14 +67,33 @@ __device__ __forceinline__ float warp_kth_largest(float x, int k) {
     return __shfl_sync(0xffffffffu, x, k - 1);
 }
 
-// Top-k of n candidates vals[j] with ids ids[j] (or id_base + j when ids is null), in
-// shared memory; sv / si: this warp's scratch of kMergeCap entries. Calls out(q, value, id)
-// on lane 0 for q < k; past the finite candidates the value is -inf and the id INT_MAX.
-// With STATS, also returns (max, sum of exp(x - max)) of x = value * inv_temp over the
-// finite candidates (all lanes). vals may be overwritten.
-template <bool STATS, typename Out>
+// The value a candidate is ranked by: its logit (greedy top-k) ...
+struct KeyLogit {
+    __device__ __forceinline__ float operator()(float v, int) const { return v; }
+    __device__ __forceinline__ bool may_reach(float, float) const { return true; }
+};
+// ... or its sampling key logit / T + G (stochastic drafting; fe_sample.cuh). may_reach is
+// a cheap necessary condition for key >= th (G never exceeds kGumbelMax), so most
+// candidates are ruled out without drawing their deviate.
+struct KeySample {
+    float inv_temp;
+    unsigned long long seed;
+    int row, V;
+    __device__ __forceinline__ float operator()(float v, int id) const {
+        return v == -INFINITY ? -INFINITY : sample_key(v, inv_temp, seed, row, V, id);
+    }
+    __device__ __forceinline__ bool may_reach(float v, float th) const { return fmaf(v, inv_temp, kGumbelMax) >= th; }
+};
+
+// Top-k of n candidates vals[j] with ids ids[j] (or id_base + j when ids is null), ranked
+// by key(vals[j], id) (larger first, then smaller id), in shared memory; sv / si: this
+// warp's scratch of kMergeCap entries. Calls out(q, key, id) on lane 0 for q < k; past the
+// finite candidates the key is -inf and the id INT_MAX. With STATS, also returns (max, sum
+// of exp(x - max)) of x = vals[j] * inv_temp over the finite candidates (all lanes). vals
+// may be overwritten (a taken candidate becomes -inf), but only after out() reports it.
+template <bool STATS, typename Key, typename Out>
 __device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_base, int n, int k, float inv_temp,
-                                            float* sv, int* si, Out&& out) {
+                                            float* sv, int* si, const Key& key, Out&& out) {
     const int lane = threadIdx.x & 31;
     constexpr int U = 4;
     float lv = -INFINITY, m = -INFINITY, sum = 0.f;
@@ -89,7 +109,8 @@ __device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            if (better(v[u], id[u], lv, li)) { lv = v[u]; li = id[u]; }
+            const float kv = key(v[u], id[u]);
+            if (better(kv, id[u], lv, li)) { lv = kv; li = id[u]; }
             if (STATS && v[u] != -INFINITY) {
                 const float x = v[u] * inv_temp;
                 if (x > m) { sum = sum * expf(m - x) + 1.f; m = x; }
@@ -118,10 +139,13 @@ __device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int j = j0 + 32 * u + lane;
-            const bool p = j < n && v[u] >= T;
+            const int idj = j < n ? (ids ? ids[j] : id_base + j) : INT_MAX;
+            float kv = -INFINITY;
+            if (j < n && key.may_reach(v[u], T)) kv = key(v[u], idj);
+            const bool p = j < n && kv >= T;
             const unsigned bal = __ballot_sync(0xffffffffu, p);
             const int pos = cnt + __popc(bal & ((1u << lane) - 1u));
-            if (p && pos < kMergeCap) { sv[pos] = v[u]; si[pos] = ids ? ids[j] : id_base + j; }
+            if (p && pos < kMergeCap) { sv[pos] = kv; si[pos] = idj; }
             cnt += __popc(bal);
         }
     }
@@ -161,8 +185,8 @@ __device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_
             bi = INT_MAX;
             bp = -1;
             for (int j = lane; j < n; j += 32) {
-                const float v = vals[j];
                 const int id = ids ? ids[j] : id_base + j;
+                const float v = key(vals[j], id);
                 if (bp < 0 || better(v, id, bv, bi)) { bv = v; bi = id; bp = j; }
             }
         };
@@ -182,31 +206,36 @@ __device__ __forceinline__ float2 warp_topk(float* vals, const int* ids, int id_
     return make_float2(m, sum);
 }
 
+// A row's running top-k, sorted (larger value first, then smaller id). val is the value
+// the row is ranked by (the logit, or the sampling key); lg the candidate's logit.
 struct TopkState {
     int id[kLmTile][kMaxTopK];
     float val[kLmTile][kMaxTopK];
+    float lg[kLmTile][kMaxTopK];
     int cnt[kLmTile];
     int last;
 };
 
-__device__ __forceinline__ void topk_insert(TopkState* st, int b, int k, float lg, int v) {
+__device__ __forceinline__ void topk_insert(TopkState* st, int b, int k, float key, int v, float lg) {
     const int c = st->cnt[b];
     int pos;
     if (c < k) {
         pos = c;
         st->cnt[b] = c + 1;
-    } else if (better(lg, v, st->val[b][k - 1], st->id[b][k - 1])) {
+    } else if (better(key, v, st->val[b][k - 1], st->id[b][k - 1])) {
         pos = k - 1;
     } else {
         return;
     }
-    while (pos > 0 && better(lg, v, st->val[b][pos - 1], st->id[b][pos - 1])) {
+    while (pos > 0 && better(key, v, st->val[b][pos - 1], st->id[b][pos - 1])) {
         st->val[b][pos] = st->val[b][pos - 1];
         st->id[b][pos] = st->id[b][pos - 1];
+        st->lg[b][pos] = st->lg[b][pos - 1];
         --pos;
     }
-    st->val[b][pos] = lg;
+    st->val[b][pos] = key;
     st->id[b][pos] = v;
+    st->lg[b][pos] = lg;
 }
 
 template <int BT>
@@ -240,6 +269,7 @@ struct LmEpi {
             const int k = a->top_k;
             const int n = min(ng * kGroupRows, a->V - cg0 * kGroupRows);
             const float* sb = cbuf + warp * CW;
+            const int srow = sample_row(b0 + warp, a->B, a->N);
             for (int base = 0; base < n; base += 32) {
                 const int idx = base + lane;
                 const bool valid = idx < n;
@@ -254,13 +284,19 @@ struct LmEpi {
                     }
                 }
                 const int v = cg0 * kGroupRows + idx;
-                const bool pass =
-                    valid && (st->cnt[warp] < k || better(lg, v, st->val[warp][k - 1], st->id[warp][k - 1]));
+                // the value the row is ranked by: the logit, or (sampling) its key
+                const bool full = st->cnt[warp] >= k;
+                const float th = full ? st->val[warp][k - 1] : -INFINITY;
+                float key = lg;
+                if (a->sample && valid)
+                    key = (!full || fmaf(lg, a->inv_temp, kGumbelMax) >= th)
+                              ? sample_key(lg, a->inv_temp, a->seed, srow, a->V, v) : -INFINITY;
+                const bool pass = valid && (!full || better(key, v, th, st->id[warp][k - 1]));
                 unsigned mask = __ballot_sync(0xffffffffu, pass);
                 while (mask) {
                     const int j = __ffs(mask) - 1;
                     mask &= mask - 1;
-                    if (lane == j) topk_insert(st, warp, k, lg, v);
+                    if (lane == j) topk_insert(st, warp, k, key, v, lg);
                     __syncwarp();
                 }
             }
@@ -277,11 +313,19 @@ struct LmEpi {
 //   nothing below tau can be among the k best); the candidates >= tau (all of them if
 //   there are more than kMergeCap) go through k rounds of a warp arg-max (descending
 //   value, ascending id); probabilities are exp(logit / T - lse).
+// Stochastic drafting: the partials' values are sampling keys, and the k largest keys
+// (in that order: the draw order) are the drawn candidates; their logits come from the
+// partials' part_lg, and they are written ordered by logit (ties: smaller id) with each
+// one's draw position in topk_rank.
+constexpr size_t kMergeWarpBytes = (size_t)kMergeCap * 8 + 16 + 32 * 8;  // selection scratch + winners
+constexpr int kMergeMaxSmem = 100 * 1024;  // dynamic shared memory of lmhead_merge_kernel, at most
+
 __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* buf, size_t buf_bytes) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5, nw = blockDim.x >> 5;
     const int ns = a.n_slabs, k = a.top_k;
-    const size_t per_row = (size_t)ns * (2 * k + 2) * 4;
-    const size_t per_warp = (size_t)kMergeCap * 8 + 16;
+    const bool smp = a.sample != 0;
+    const size_t per_row = (size_t)ns * ((smp ? 3 : 2) * k + 2) * 4;
+    const size_t per_warp = kMergeWarpBytes;
     if (buf_bytes <= nw * per_warp + per_row) return;  // never happens: the host sizes the buffer
     const int batch = (int)((buf_bytes - nw * per_warp) / per_row);
     float* cand_v = (float*)(buf + nw * per_warp);  // [batch][ns * k]
@@ -290,6 +334,7 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
         float* bv_ = cand_v;
         int* bi_ = (int*)(cand_v + (size_t)nr * ns * k);
         float* bm_ = (float*)(bi_ + (size_t)nr * ns * k);
+        float* bl_ = bm_ + (size_t)nr * ns * 2;  // sampling: the candidates' logits
         // 8 independent loads in flight per thread (a load-then-store loop would wait a full
         // L2 round trip per element)
         const size_t nc = (size_t)nr * ns * k, nm = (size_t)nr * ns * 2;
@@ -306,6 +351,21 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
             for (int u = 0; u < 8; ++u) {
                 const size_t q = q0 + u * (size_t)blockDim.x;
                 if (q < nc) { bv_[q] = v[u]; bi_[q] = id[u]; }
+            }
+        }
+        if (smp) {
+            for (size_t q0 = t; q0 < nc; q0 += 8 * (size_t)blockDim.x) {
+                float v[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const size_t q = q0 + u * (size_t)blockDim.x;
+                    v[u] = q < nc ? __ldcg(a.part_lg + (size_t)rb * ns * k + q) : 0.f;
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const size_t q = q0 + u * (size_t)blockDim.x;
+                    if (q < nc) bl_[q] = v[u];
+                }
             }
         }
         for (size_t q0 = t; q0 < nm; q0 += 8 * (size_t)blockDim.x) {
@@ -339,11 +399,46 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
             const float lse = M + logf(S);
             const int i = zr / a.B, b = zr % a.B;
             const size_t ob = ((size_t)b * a.N + i) * k;
-            warp_topk<false>(pv, pi, 0, ns * k, k, a.inv_temp, sv, si, [&](int q, float v, int id) {
-                a.topk_id[ob + q] = id;
-                a.topk_logit[ob + q] = v;
-                a.topk_prob[ob + q] = v == -INFINITY ? 0.f : expf(v * a.inv_temp - lse);
-            });
+            if (!smp) {
+                warp_topk<false>(pv, pi, 0, ns * k, k, a.inv_temp, sv, si, KeyLogit{}, [&](int q, float v, int id) {
+                    a.topk_id[ob + q] = id;
+                    a.topk_logit[ob + q] = v;
+                    a.topk_prob[ob + q] = v == -INFINITY ? 0.f : expf(v * a.inv_temp - lse);
+                    if (a.topk_rank) a.topk_rank[ob + q] = q;
+                });
+            } else {
+                // the k largest keys, in draw order, into this warp's winner slots
+                float* wl = (float*)(buf + warp * per_warp + (size_t)kMergeCap * 8 + 16);
+                int* wi = (int*)(wl + 32);
+                if (lane < 32) { wl[lane] = -INFINITY; wi[lane] = INT_MAX; }
+                __syncwarp();
+                warp_topk<false>(pv, pi, 0, ns * k, k, a.inv_temp, sv, si, KeyLogit{},
+                                 [&](int q, float, int id) { wi[q] = id; });
+                __syncwarp();
+                // the winners' logits: every candidate id occurs once (the slabs are disjoint)
+                const float* pl = bl_ + (size_t)rr * ns * k;
+                for (int j = lane; j < ns * k; j += 32) {
+                    const int idj = pi[j];
+                    for (int q = 0; q < k; ++q)
+                        if (wi[q] == idj && idj != INT_MAX) wl[q] = pl[j];
+                }
+                __syncwarp();
+                const float lg = lane < k ? wl[lane] : -INFINITY;
+                const int id = lane < k ? wi[lane] : INT_MAX;
+                int pos = 0;  // this winner's place by (logit desc, id asc)
+                for (int j = 0; j < k; ++j) {
+                    const float oj = __shfl_sync(0xffffffffu, lg, j);
+                    const int ij = __shfl_sync(0xffffffffu, id, j);
+                    if (j != lane && better(oj, ij, lg, id)) ++pos;
+                }
+                if (lane < k) {
+                    a.topk_id[ob + pos] = id;
+                    a.topk_logit[ob + pos] = lg;
+                    a.topk_prob[ob + pos] = lg == -INFINITY ? 0.f : expf(lg * a.inv_temp - lse);
+                    if (a.topk_rank) a.topk_rank[ob + pos] = lane;
+                }
+                __syncwarp();
+            }
             if (lane == 0) a.lse[(size_t)b * a.N + i] = lse;
         }
         __syncthreads();
@@ -351,8 +446,8 @@ __device__ void merge_rows(const LmHeadArgs& a, int r0, int r1, unsigned char* b
 }
 
 // shared memory merge_rows needs for at least one row at a time
-__host__ __device__ inline size_t merge_smem_bytes(int nwarps, int n_slabs, int top_k) {
-    return (size_t)nwarps * (kMergeCap * 8 + 16) + (size_t)n_slabs * (2 * top_k + 2) * 4 + 64;
+__host__ __device__ inline size_t merge_smem_bytes(int nwarps, int n_slabs, int top_k, bool sample) {
+    return (size_t)nwarps * kMergeWarpBytes + (size_t)n_slabs * ((sample ? 3 : 2) * top_k + 2) * 4 + 64;
 }
 
 template <typename WT, int BT>
@@ -398,6 +493,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) lmhead_kernel(const LmHeadA
             const bool ok = j < st.cnt[warp];
             a.part_id[base * a.top_k + j] = ok ? st.id[warp][j] : INT_MAX;
             a.part_val[base * a.top_k + j] = ok ? st.val[warp][j] : -INFINITY;
+            if (a.sample) a.part_lg[base * a.top_k + j] = ok ? st.lg[warp][j] : -INFINITY;
         }
         if (lane == 0) {
             a.part_ms[base * 2 + 0] = m;
@@ -715,11 +811,16 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
         int* si = (int*)(sv + kMergeCap);
         for (int r = warp; r < R; r += kMmaThreads / 32) {
             const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
-            const float2 ms = warp_topk<true>(slab + (size_t)r * slab_cap, nullptr, first, n, k, a.inv_temp, sv, si,
-                                              [&](int q, float v, int id) {
-                                                  a.part_id[base * k + q] = id;
-                                                  a.part_val[base * k + q] = v;
-                                              });
+            float* row = slab + (size_t)r * slab_cap;
+            auto out = [&](int q, float v, int id) {
+                a.part_id[base * k + q] = id;
+                a.part_val[base * k + q] = v;
+                if (a.sample) a.part_lg[base * k + q] = id == INT_MAX ? -INFINITY : row[id - first];
+            };
+            const float2 ms =
+                a.sample ? warp_topk<true>(row, nullptr, first, n, k, a.inv_temp, sv, si,
+                                           KeySample{a.inv_temp, a.seed, sample_row(r, a.B, a.N), a.V}, out)
+                         : warp_topk<true>(row, nullptr, first, n, k, a.inv_temp, sv, si, KeyLogit{}, out);
             if (lane == 0) {
                 a.part_ms[base * 2 + 0] = ms.x;
                 a.part_ms[base * 2 + 1] = ms.y;
@@ -753,7 +854,7 @@ cudaError_t launch_bt(const LmHeadArgs& a, const DeviceInfo& dev, cudaStream_t s
     const int Kpad = (a.d + 3) & ~3;
     const int xrows = BT < a.R ? BT : a.R;
     const size_t budget = (size_t)dev.max_smem_optin - kStaticReserve;
-    const size_t merge = merge_smem_bytes(kStreamThreads / 32, a.n_slabs, a.top_k);
+    const size_t merge = merge_smem_bytes(kStreamThreads / 32, a.n_slabs, a.top_k, a.sample != 0);
     int D = stream_slots(budget, stream_smem_bytes(0, xrows, Kpad, BT));
     D = D > kPreferredSlots ? kPreferredSlots : D;
     if (D < 1) return cudaErrorInvalidValue;
@@ -815,7 +916,7 @@ cudaError_t lmhead_mma_prepare(const DeviceInfo& dev) {
     const cudaError_t e = cudaFuncSetAttribute(lmhead_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                dev.max_smem_optin - (int)sizeof(MmaState) - 256);
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeMaxSmem);
 }
 
 cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
@@ -842,8 +943,8 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
     int S = (int)((budget - 1024 - slab_bytes) / stage_bytes);
     S = S > kMmaMaxStages ? kMmaMaxStages : S;
     if (S < 2) return cudaErrorInvalidValue;
-    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k);
-    if (msmem > 64 * 1024) return cudaErrorInvalidValue;
+    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k, a.sample != 0);
+    if (msmem > kMergeMaxSmem) return cudaErrorInvalidValue;
     const size_t smem = 1024 + (size_t)S * stage_bytes + slab_bytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
@@ -899,17 +1000,51 @@ __device__ __forceinline__ void wide_insert(float (&tv)[KM], int (&ti)[KM], int 
     }
 }
 
+// the same, carrying each entry's logit beside its key (stochastic drafting)
+template <int KM>
+__device__ __forceinline__ void wide_insert(float (&tv)[KM], int (&ti)[KM], float (&tl)[KM], int k, float x, int id,
+                                            float lx) {
+#pragma unroll
+    for (int q = 0; q < KM; ++q) {
+        const bool sw = q < k && better(x, id, tv[q], ti[q]);
+        const float ov = tv[q], ol = tl[q];
+        const int oi = ti[q];
+        tv[q] = sw ? x : ov;
+        ti[q] = sw ? id : oi;
+        tl[q] = sw ? lx : ol;
+        x = sw ? ov : x;
+        id = sw ? oi : id;
+        lx = sw ? ol : lx;
+    }
+}
+
+// Stochastic drafting: the smallest 23-bit deviate code m (U = (m + 1/2) / 2^23) with which
+// a logit at most M can still give a key logit / T + G >= th, minus a safety margin. With
+// c = th - M / T, G >= c needs U >= exp(-exp(-c)); the bound is taken from 1 - U <=
+// -expm1(-exp(-(c - 1e-3))), which errs towards admitting more (1e-3 in c moves the bound
+// by a relative 1e-3, far above the functions' rounding). A tile's entries with a smaller
+// code cannot enter the list and skip their logarithms.
+__device__ __forceinline__ uint32_t sample_code_floor(float th, float M_scaled) {
+    if (th == -INFINITY) return 0u;
+    const float c = th - M_scaled - 1e-3f;
+    if (c <= -30.f) return 0u;
+    const float tail = -expm1f(-expf(-c));                    // an upper bound on 1 - U
+    const float f = floorf(8388607.5f - tail * 8388608.0f) - 1.0f;
+    return f <= 0.f ? 0u : (uint32_t)f;
+}
+
 // A running (softmax statistics, top-k) state of one hidden row: the first k of the KM
 // entries form the sorted list (larger value first, ties to the smaller id; the rest stay
 // -inf); (m, s) are the max and sum of exp of logit / T so far.
 template <int KM>
 struct WideRow {
-    float v[KM];
+    float v[KM];  // the values the list is ranked by: logits, or sampling keys
     int i[KM];
+    float l[KM];  // sampling only: the entries' logits
     float m, s;
     __device__ __forceinline__ void init() {
 #pragma unroll
-        for (int q = 0; q < KM; ++q) { v[q] = -INFINITY; i[q] = INT_MAX; }
+        for (int q = 0; q < KM; ++q) { v[q] = -INFINITY; i[q] = INT_MAX; l[q] = -INFINITY; }
         m = -INFINITY;
         s = 0.f;
     }
@@ -960,7 +1095,7 @@ struct WideRow {
                     }                                                                              \
                     _Pragma("unroll") for (int u = 0; u < 8; ++u) {                                \
                         M = fmaxf(M, x[u]);                                                        \
-                        bits |= (x[u] >= th ? 1u : 0u) << (b0 + u);                                \
+                        if (!SMP) bits |= (x[u] >= th ? 1u : 0u) << (b0 + u);                      \
                     }                                                                              \
                 }                                                                                  \
                 if (wd == 0) cm0 = bits;                                                           \
@@ -968,12 +1103,38 @@ struct WideRow {
                 else if (wd == 2) cm2 = bits;                                                      \
                 else cm3 = bits;                                                                   \
             }                                                                                      \
+            if (SMP) { /* keys: a deviate code per entry, logarithms only past the code floor */   \
+                const int srow = sample_row(r, a.B, a.N);                                          \
+                const uint32_t mlo = sample_code_floor(th, M * a.inv_temp);                        \
+                _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                 \
+                    uint32_t bits = 0u;                                                            \
+                    for (int e0 = 0; e0 < 32; ++e0) {                                              \
+                        const int e = wd * 32 + e0;                                                \
+                        if (e >= nv) break;                                                        \
+                        const uint32_t m23 = (uint32_t)(splitmix64_at(a.seed,                      \
+                            sample_counter(srow, a.V, id0 + e)) >> 41);                            \
+                        if (m23 < mlo) continue;                                                   \
+                        const float key = fmaf(col[(size_t)e * kWideTileStride], a.inv_temp,       \
+                            gumbel_of(((float)m23 + 0.5f) * (1.0f / 8388608.0f)));                 \
+                        bits |= (key >= th ? 1u : 0u) << e0;                                       \
+                    }                                                                              \
+                    if (wd == 0) cm0 = bits;                                                       \
+                    else if (wd == 1) cm1 = bits;                                                  \
+                    else if (wd == 2) cm2 = bits;                                                  \
+                    else cm3 = bits;                                                               \
+                }                                                                                  \
+            }                                                                                      \
             _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                     \
                 uint32_t bits = wd == 0 ? cm0 : wd == 1 ? cm1 : wd == 2 ? cm2 : cm3;               \
                 while (bits) {                                                                     \
                     const int e = wd * 32 + __ffs(bits) - 1;                                       \
                     bits &= bits - 1u;                                                             \
-                    wide_insert(w.v, w.i, k, col[(size_t)e * kWideTileStride], id0 + e);           \
+                    const float xe = col[(size_t)e * kWideTileStride];                             \
+                    if (SMP)                                                                       \
+                        wide_insert(w.v, w.i, w.l, k, sample_key(xe, a.inv_temp, a.seed,           \
+                                    sample_row(r, a.B, a.N), a.V, id0 + e), id0 + e, xe);          \
+                    else                                                                           \
+                        wide_insert(w.v, w.i, k, xe, id0 + e);                                     \
                 }                                                                                  \
             }                                                                                      \
             if (nv > 0) {                                                                          \
@@ -996,7 +1157,7 @@ struct WideRow {
         ok = epi_sync();                                                                           \
     } while (0)
 
-template <int KM>
+template <int KM, bool SMP>
 __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
                                                                      int S, int stage_bytes, uint32_t tmem_cols) {
     const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
@@ -1115,6 +1276,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
             if (q < k) {                                                                               \
                 a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];                      \
                 a.part_val[base * k + q] = w.v[q];                                                     \
+                if (SMP) a.part_lg[base * k + q] = w.l[q];                                             \
             }                                                                                          \
         }                                                                                              \
         a.part_ms[base * 2 + 0] = w.m;                                                                 \
@@ -1163,13 +1325,18 @@ int lmhead_wide_slabs(int V, const DeviceInfo& dev) {
 }
 
 cudaError_t lmhead_wide_prepare(const DeviceInfo& dev) {
-    cudaError_t e = cudaFuncSetAttribute(lmhead_wide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         dev.max_smem_optin - (int)sizeof(WideState) - 256);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(lmhead_wide_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             dev.max_smem_optin - (int)sizeof(WideState) - 256);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+    const int wsm = dev.max_smem_optin - (int)sizeof(WideState) - 256;
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(lmhead_wide_kernel<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
+            cudaSuccess ||
+        (e = cudaFuncSetAttribute(lmhead_wide_kernel<16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
+            cudaSuccess ||
+        (e = cudaFuncSetAttribute(lmhead_wide_kernel<8, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
+            cudaSuccess ||
+        (e = cudaFuncSetAttribute(lmhead_wide_kernel<16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
+            cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeMaxSmem);
 }
 
 cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceInfo& dev, cudaStream_t st,
@@ -1189,14 +1356,14 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
     const size_t smem = 1024 + (size_t)S * stage_bytes + tbytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * R_pad)) cols <<= 1;
-    e = a.top_k <= 8 ? launch_k(lmhead_wide_kernel<8>, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a,
-                                (const uint16_t*)zb, R_pad, S, stage_bytes, cols)
-                     : launch_k(lmhead_wide_kernel<16>, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a,
-                                (const uint16_t*)zb, R_pad, S, stage_bytes, cols);
+    auto kern = a.sample ? (a.top_k <= 8 ? lmhead_wide_kernel<8, true> : lmhead_wide_kernel<16, true>)
+                         : (a.top_k <= 8 ? lmhead_wide_kernel<8, false> : lmhead_wide_kernel<16, false>);
+    e = launch_k(kern, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad, S,
+                 stage_bytes, cols);
     if (e != cudaSuccess) return e;
     if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;
-    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k);
-    if (msmem > 64 * 1024) return cudaErrorInvalidValue;
+    const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k, a.sample != 0);
+    if (msmem > kMergeMaxSmem) return cudaErrorInvalidValue;
     return launch_k(lmhead_merge_kernel, dim3(a.R), dim3(128), msmem, st, a.pdl, a, msmem);
 }
 

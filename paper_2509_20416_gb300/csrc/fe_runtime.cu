@@ -43,7 +43,8 @@ struct GraphKey {
                x.next_tok == y.next_tok && x.prefix_len == y.prefix_len && x.page_table == y.page_table &&
                x.n_pages == y.n_pages && x.topk_id == y.topk_id && x.topk_logit == y.topk_logit &&
                x.topk_prob == y.topk_prob && x.lse == y.lse && x.dbg_logits == y.dbg_logits &&
-               x.dbg_hidden == y.dbg_hidden && kc == o.kc && vc == o.vc;
+               x.dbg_hidden == y.dbg_hidden && x.sample == y.sample && x.seed == y.seed &&
+               x.topk_rank == y.topk_rank && kc == o.kc && vc == o.vc;
     }
 };
 
@@ -51,12 +52,15 @@ struct GraphKey {
 struct HostKey {
     int B = 0, top_k = 0;
     float temperature = 0.f;
+    int sample = 0;
+    uint64_t seed = 0;
     const void* feat_direct = nullptr;  // the caller's pinned features, copied from directly
     const int32_t* page_table = nullptr;
     int n_pages = 0;
     std::vector<void*> kc, vc;
     bool operator==(const HostKey& o) const {
-        return B == o.B && top_k == o.top_k && temperature == o.temperature && feat_direct == o.feat_direct &&
+        return B == o.B && top_k == o.top_k && temperature == o.temperature && sample == o.sample &&
+               seed == o.seed && feat_direct == o.feat_direct &&
                page_table == o.page_table &&
                n_pages == o.n_pages && kc == o.kc && vc == o.vc;
     }
@@ -66,7 +70,7 @@ struct HostKey {
 // the same in the pinned staging buffers and in their device copies
 struct StepLayout {
     size_t feat, tok, plen, in_bytes;
-    size_t id, logit, prob, lse, ttok, tpar, tdep, tmask, out_bytes;
+    size_t id, logit, prob, lse, rank, ttok, tpar, tdep, tmask, out_bytes;
 };
 
 StepLayout step_layout(const fe_config& c, size_t es, int B, int k) {
@@ -83,6 +87,7 @@ StepLayout step_layout(const fe_config& c, size_t es, int B, int k) {
     L.logit = o; o = al(o + b * N * k * 4);
     L.prob = o; o = al(o + b * N * k * 4);
     L.lse = o; o = al(o + b * N * 4);
+    L.rank = o; o = al(o + b * N * k * 4);
     L.ttok = o; o = al(o + b * T * 4);
     L.tpar = o; o = al(o + b * T * 4);
     L.tdep = o; o = al(o + b * T * 4);
@@ -110,6 +115,8 @@ struct fe_handle {
     float* attn_part = nullptr;
     int* lm_part_id = nullptr;
     float *lm_part_val = nullptr, *lm_part_ms = nullptr;
+    float* lm_part_lg = nullptr;  // sampling: the logits of the partials' candidates
+    float* vs_rbuf = nullptr;     // fe_verify_sampled: each sequence's residual distribution [max_batch, V]
     int* status = nullptr;
     int* attn_counters = nullptr;
     int* lm_counters = nullptr;
@@ -392,6 +399,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.part_id = h->lm_part_id; lm.part_val = h->lm_part_val; lm.part_ms = h->lm_part_ms;
     lm.counters = h->lm_counters; lm.dbg_logits = a->dbg_logits; lm.status = h->status;
     lm.topk_id = a->topk_id; lm.topk_logit = a->topk_logit; lm.topk_prob = a->topk_prob; lm.lse = a->lse;
+    lm.sample = a->sample ? 1 : 0; lm.seed = a->seed; lm.part_lg = h->lm_part_lg; lm.topk_rank = a->topk_rank;
     lm.pdl = pdl;
     lm.stamp = next_stamp(pf);
     if (h->lm_mma && N * B <= 16) {
@@ -522,6 +530,7 @@ bool forward_args_ok(const fe_handle* h, const fe_forward_args* a) {
         if (!a->k_cache[i] || !a->v_cache[i]) return false;
     if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return false;
     if (!(a->temperature == a->temperature)) return false;  // NaN
+    if (a->sample && !(a->temperature > 0.f)) return false;  // draws need a temperature
     if (h->lin_mma && (reinterpret_cast<uintptr_t>(a->feat) & 15)) return false;  // read as 16-byte vectors
     return true;
 }
@@ -757,8 +766,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         const size_t k = c.top_k_max;
         const size_t kmax = std::max({(size_t)3 * c.d, (size_t)c.ffn, (size_t)c.n_heads * hd});
         const size_t mmax = std::max({(size_t)c.d, nqkv, (size_t)2 * c.ffn});
-        size_t off[24], n = 0, tot = 0;
-        const size_t bytes[24] = {
+        size_t off[26], n = 0, tot = 0;
+        const size_t bytes[26] = {
             cs.size() * sizeof(float),                             // rope
             Rw * d * 4, Rw * d * 4, Rw * nqkv * 4, Rw * H * hd * 4,   // g, x, qkv, o
             Rw * F * 4, R * d * 4,                                  // act, hid
@@ -778,8 +787,10 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             Rw * 3 * d * h->es,                                               // commit: gathered features
             Rw * sizeof(int),                                                 // commit: gathered tokens
             h->lm_mma ? lmhead_mma_split_bytes(16, h->dev) : 0,                // LM head: split-tile parts
-            h->lm_mma ? (size_t)h->dev.num_sms * sizeof(int) : 0};            // ... and their flags
-        for (n = 0; n < 24; ++n) { off[n] = tot; tot += align256(bytes[n]); }
+            h->lm_mma ? (size_t)h->dev.num_sms * sizeof(int) : 0,             // ... and their flags
+            R * h->lm_slabs * k * 4,                                          // LM-head partial logits (sampling)
+            B * (size_t)c.vocab * 4};                                         // sampled verification's residuals
+        for (n = 0; n < 26; ++n) { off[n] = tot; tot += align256(bytes[n]); }
         if ((rc = from_cuda(cudaMalloc(&h->sbuf, tot))) != FE_OK) break;
         char* s = (char*)h->sbuf;
         h->rope_cs = (float*)(s + off[0]);
@@ -806,6 +817,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
         h->ctok = (int*)(s + off[21]);
         h->lm_split_part = h->lm_mma ? (float*)(s + off[22]) : nullptr;
         h->lm_split_flag = h->lm_mma ? (int*)(s + off[23]) : nullptr;
+        h->lm_part_lg = (float*)(s + off[24]);
+        h->vs_rbuf = (float*)(s + off[25]);
         if ((rc = from_cuda(cudaMemcpyAsync(h->rope_cs, cs.data(), bytes[0], cudaMemcpyHostToDevice, st))) != FE_OK)
             break;
         // status word and completion counters start (and stay, between calls) at zero
@@ -1014,6 +1027,9 @@ fe_status enqueue_host_step(fe_handle* h, const fe_host_step_args* a, const Step
     fa.topk_logit = reinterpret_cast<float*>(h->ds_out + L.logit);
     fa.topk_prob = reinterpret_cast<float*>(h->ds_out + L.prob);
     fa.lse = reinterpret_cast<float*>(h->ds_out + L.lse);
+    fa.sample = a->sample;
+    fa.seed = a->seed;
+    fa.topk_rank = reinterpret_cast<int32_t*>(h->ds_out + L.rank);
     if (!forward_args_ok(h, &fa)) return FE_ERR_INVALID_ARG;
     const fe_status rc = enqueue_forward(h, &fa, st);
     if (rc != FE_OK) return rc;
@@ -1037,6 +1053,7 @@ fe_status fe_draft_step_host(fe_handle* h, const fe_host_step_args* a, void* str
         if (!a->k_cache[i] || !a->v_cache[i]) return FE_ERR_INVALID_ARG;
     if (c.page_size > 0 && (!a->page_table || a->n_pages < 1)) return FE_ERR_INVALID_ARG;
     if (!(a->temperature == a->temperature)) return FE_ERR_INVALID_ARG;
+    if (a->sample && !(a->temperature > 0.f)) return FE_ERR_INVALID_ARG;
     const fe_status dv = check_device(h);
     if (dv != FE_OK) return dv;
     cudaStream_t st = (cudaStream_t)stream;
@@ -1058,6 +1075,7 @@ fe_status fe_draft_step_host(fe_handle* h, const fe_host_step_args* a, void* str
         } else {
             HostKey key;
             key.B = a->B; key.top_k = a->top_k; key.temperature = a->temperature;
+            key.sample = a->sample ? 1 : 0; key.seed = a->seed;
             key.feat_direct = feat_direct ? a->feat : nullptr;
             key.page_table = a->page_table; key.n_pages = a->n_pages;
             key.kc.assign(a->k_cache, a->k_cache + c.n_layers);
@@ -1090,6 +1108,7 @@ fe_status fe_draft_step_host(fe_handle* h, const fe_host_step_args* a, void* str
     memcpy(a->topk_logit, h->hs_out + L.logit, B * N * k * 4);
     memcpy(a->topk_prob, h->hs_out + L.prob, B * N * k * 4);
     memcpy(a->lse, h->hs_out + L.lse, B * N * 4);
+    if (a->topk_rank) memcpy(a->topk_rank, h->hs_out + L.rank, B * N * k * 4);
     memcpy(a->tree_tok, h->hs_out + L.ttok, B * T * 4);
     memcpy(a->tree_parent, h->hs_out + L.tpar, B * T * 4);
     memcpy(a->tree_depth, h->hs_out + L.tdep, B * T * 4);
@@ -1134,6 +1153,27 @@ fe_status fe_verify_greedy(fe_handle* h, int32_t B, int32_t top_k, const int32_t
     const int N = h->cfg.n_layers, T = 1 + N * top_k;
     FE_TRY(launch_verify(B, T, N, prefix_len, tree->tok, tree->parent, tree->depth, target_next, pos_ids, path,
                          n_accept, bonus, (cudaStream_t)stream));
+    return FE_OK;
+}
+
+fe_status fe_verify_sampled(fe_handle* h, int32_t B, int32_t top_k, const fe_tree* tree, const int32_t* topk_rank,
+                            const float* q, const float* p, const float* u_acc, const float* u_bonus, int32_t* path,
+                            int32_t* n_accept, int32_t* bonus, void* stream) {
+    if (!h || !tree || !topk_rank || !q || !p || !u_acc || !u_bonus || !path || !n_accept || !bonus)
+        return FE_ERR_INVALID_ARG;
+    if (!tree->tok || !tree->parent || !tree->depth) return FE_ERR_INVALID_ARG;
+    if (B < 1 || B > h->cfg.max_batch || top_k < 1 || top_k > h->cfg.top_k_max) return FE_ERR_INVALID_ARG;
+    const fe_status dv = check_device(h);
+    if (dv != FE_OK) return dv;
+    VerifySampledArgs va{};
+    va.N = h->cfg.n_layers;
+    va.T = 1 + va.N * top_k;
+    va.V = h->cfg.vocab;
+    va.tok = tree->tok; va.parent = tree->parent; va.depth = tree->depth; va.rank = topk_rank;
+    va.q = q; va.p = p; va.u_acc = u_acc; va.u_bonus = u_bonus;
+    va.rbuf = h->vs_rbuf;
+    va.path = path; va.n_accept = n_accept; va.bonus = bonus; va.status = h->status;
+    FE_TRY(launch_verify_sampled(va, B, (cudaStream_t)stream));
     return FE_OK;
 }
 

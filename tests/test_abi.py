@@ -79,6 +79,8 @@ def test_next_row_entry_points_validate_on_host(lib):
     assert so.fe_verify_greedy(None, 1, 1, None, ctypes.byref(tree), None, None, None, None, None,
                                None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_draft_loss(None, None, None, None, 0.1, 1.0, 0.9, None, None, None, None) == lib.FE_ERR_INVALID_ARG
+    assert so.fe_verify_sampled(None, 1, 1, ctypes.byref(tree), None, None, None, None, None, None, None, None,
+                                None) == lib.FE_ERR_INVALID_ARG
     assert so.fe_lm_head_topk_noalloc(None, None, 1, 1, 0.0, None, None, None, None, None) == lib.FE_ERR_INVALID_ARG
     for ns in (0, 999, 10**9 + 1):  # outside 1e3..1e9 ns, and a null handle
         assert so.fe_selftest_timeout(None, ns, None) == lib.FE_ERR_INVALID_ARG

@@ -21,6 +21,10 @@ CASES = {
     # fp32 storage
     "f32_b3": (dict(d=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=688, vocab=4096, n_layers=3, dtype="f32",
                     B=3, prefix=0, top_k=4, rope_theta=1e4, seed=63, page_size=0), [5, 0, 63], 0.0),
+    # stochastic drafting (Sec. 2.2) through the host step: the drawn set and its ranks
+    "bf16_b12_paged_sampled": (dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1408, vocab=3001, n_layers=2,
+                                    dtype="bf16", B=12, prefix=0, top_k=4, rope_theta=1e4, seed=64, page_size=16),
+                               [3, 0, 17, 40, 8, 1, 30, 12, 5, 60, 22, 9], 1.0, 77),
 }
 
 
@@ -40,10 +44,11 @@ def _setup(spec, plist):
     return fe, cfg, h, I, kd, vd, table, n_pages
 
 
-def _device_step(fe, cfg, h, I, kd, vd, table, n_pages, temp, B=None):
+def _device_step(fe, cfg, h, I, kd, vd, table, n_pages, temp, B=None, seed=None):
     B = B or cfg["B"]
     feat, tok, plen = I["feat"][:B].cuda(), I["next_tok"][:B].cuda(), I["prefix_len"][:B].cuda()
-    out = fe.fe_draft_forward(h, feat, tok, plen, kd, vd, cfg["top_k"], temp, page_table=table, n_pages=n_pages)
+    out = fe.fe_draft_forward(h, feat, tok, plen, kd, vd, cfg["top_k"], temp, page_table=table, n_pages=n_pages,
+                              sample=seed is not None, seed=seed or 0)
     tree = fe.fe_build_tree(h, tok, out["topk_id"], cfg["top_k"])
     torch.cuda.synchronize()
     return {**{k: v.cpu() for k, v in out.items()}, **{"tree_" + k: v.cpu() for k, v in tree.items()}}
@@ -51,15 +56,16 @@ def _device_step(fe, cfg, h, I, kd, vd, table, n_pages, temp, B=None):
 
 @pytest.mark.parametrize("case", list(CASES))
 def test_host_step_matches_device_step(case):
-    spec, plist, temp = CASES[case]
+    spec, plist, temp = CASES[case][:3]
+    seed = CASES[case][3] if len(CASES[case]) > 3 else None
     fe, cfg, h, I, kd, vd, table, n_pages = _setup(spec, plist)
-    ref = _device_step(fe, cfg, h, I, kd, vd, table, n_pages, temp)
+    ref = _device_step(fe, cfg, h, I, kd, vd, table, n_pages, temp, seed=seed)
     # pageable features go through the handle's pinned staging, page-locked ones are
     # copied from directly (a graph of its own)
     for feat in (I["feat"], I["feat"].pin_memory(), I["feat"]):
         for _ in range(2):  # the first call captures the step's graph, the second replays it
             got = fe.fe_draft_step_host(h, feat, I["next_tok"], I["prefix_len"], kd, vd, cfg["top_k"], temp,
-                                        page_table=table, n_pages=n_pages)
+                                        page_table=table, n_pages=n_pages, sample=seed is not None, seed=seed or 0)
             for key, want in ref.items():
                 assert torch.equal(got[key], want), (case, feat.is_pinned(), key)
     assert fe.fe_last_device_status(h) == fe.FE_OK

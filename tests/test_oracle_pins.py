@@ -27,3 +27,18 @@ def test_lm_head_binding_reproduces_the_draft(orc):
     assert np.array_equal(lg, o["logits"])
     W2 = dict(W, final_norm=torch.full_like(W["final_norm"], 2.0))
     assert np.allclose(orc.lm_head(cfg, W2, o["hidden"]), 2.0 * o["logits"], rtol=1e-12, atol=1e-12)
+
+
+def test_sample_keys_binding_gives_the_draw_order(orc):
+    """Oracle.sample_keys (the keys the parity test's near-tie exemption reads) are the keys
+    topk_sample draws by: its draw order is their descending order (ties: smaller id), for
+    several rows, temperatures and seeds."""
+    import numpy as np
+    rng = np.random.default_rng(5)
+    for T, seed, row in ((1.0, 7, 0), (0.7, 123, 5), (2.5, 2**63 + 11, 41)):
+        lg = rng.normal(0, 2, 777)
+        keys = orc.sample_keys(lg, T, seed, row)
+        ids, drawn = orc.topk_sample(lg[None, :], 12, T, seed, row0=row)
+        order = sorted(range(lg.size), key=lambda v: (-keys[v], v))[:12]
+        assert list(drawn[0]) == order
+        assert set(ids[0]) == set(order)
