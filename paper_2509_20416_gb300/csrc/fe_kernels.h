@@ -82,6 +82,26 @@ struct LinearArgs {
     // in-graph timing (fe_profile_graph): the (start, end) stamp pair of this phase's
     // first kernel, the next kernel of the phase at stamp + 2; null when not profiling
     unsigned long long* stamp = nullptr;
+    // tensor-core path: whether another tensor-core phase follows (next_W non-null) and
+    // reads this phase's output, which lets this phase defer its split tiles to it
+    const void* next_W = nullptr;
+    // tensor-core path, deferred split-tile reduction. With defer, a tile whose units are
+    // split between CTAs leaves each CTA's share in the partial buffer and nothing else; the
+    // next tensor-core phase's operand prep, given this phase as `prev`, sums the shares in
+    // CTA order, applies this phase's epilogue and stores the result before using it (the
+    // same operations, in the same order, as the in-kernel reduction).
+    int defer = 0;
+    struct Prev {
+        int active = 0;
+        const float* part = nullptr;  // the partial buffer the phase wrote
+        int M = 0, K = 0, G = 0;      // its shape and grid
+        int epi = 0;
+        float* y = nullptr;
+        int ldy = 0;
+        float* y2 = nullptr;
+        int ldy2 = 0;
+        const float* ybase = nullptr;
+    } prev;
 };
 
 struct DeviceInfo {

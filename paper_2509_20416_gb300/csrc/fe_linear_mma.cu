@@ -33,7 +33,9 @@ namespace fe {
 namespace {
 
 constexpr int kLmThreads = 192;  // 4 epilogue warps, 1 producer warp, 1 MMA warp
+constexpr size_t kXprepRowSmem = 16384 * sizeof(float);  // a finished row of up to 16384 columns
 constexpr int kLinMaxStages = 8;
+
 
 struct LinMmaState {
     uint64_t full[kLinMaxStages], empty[kLinMaxStages], tfull[2], tempty[2];
@@ -48,12 +50,127 @@ __device__ __forceinline__ void split_bf16(float z, uint16_t& hi, uint16_t& lo) 
 
 }  // namespace
 
+// ---- stream-K partition ---------------------------------------------------------------------
+// first unit of CTA c when U units are split over G CTAs
+__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
+
+// the CTA whose range holds unit u
+__device__ __forceinline__ int unit_owner(int64_t u, int64_t U, int G) {
+    int c = (int)((u * G) / U);
+    while (c + 1 < G && unit_begin(c + 1, U, G) <= u) ++c;
+    while (c > 0 && unit_begin(c, U, G) > u) --c;
+    return c;
+}
+
 // ---- activation operand ------------------------------------------------------------------
 // Grid (B_pad, ceil(K / 2048)): CTA (b, y) writes row b's 16-byte chunks [256 y, 256 y + 256)
 // (rows b >= B are zero); with RMSNorm every CTA of the row reads the whole row for its sum
 // of squares (an L2 read of 4 d bytes). Reads what the previous kernel wrote only after
 // griddep_wait(), through L2, and never through a __restrict__ pointer.
+// When the previous tensor-core phase deferred its split tiles (a.prev.active), the input
+// columns of those tiles are finished here first (prev_finish); with RMSNorm, one CTA per
+// row (grid (B_pad, 1)) finishes the whole row into shared memory before normalising it.
 constexpr int kXprepChunks = 256;  // 16-byte chunks per CTA (one per thread)
+
+// sum of squares of 8 values, in one fixed order
+__device__ __forceinline__ float sumsq8(const float (&v)[8]) {
+    float s = v[0] * v[0];
+#pragma unroll
+    for (int e = 1; e < 8; ++e) s = fmaf(v[e], v[e], s);
+    return s;
+}
+
+// The previous phase's finished output at columns k0 .. k0 + 7 of row b (this phase's
+// input). Columns of a tile the previous phase finished itself are read from where its
+// epilogue stored them; a split tile's shares are summed in CTA order, its epilogue applied
+// (residual add with the copy into y2, SwiGLU over the interleaved gate/up rows, or a plain
+// store) and the result stored, exactly as the phase's own fix-up would have.
+// GLU: the previous phase is the SwiGLU one (16 rows per 8 columns); otherwise 8 rows.
+template <bool GLU>
+__device__ __forceinline__ void prev_finish_t(const LinearArgs::Prev& p, int BP, int b, int k0, float (&v)[8]) {
+    constexpr int NR = GLU ? 16 : 8;  // the previous phase's rows behind these 8 columns
+    constexpr bool glu = GLU;
+    const int nkb = p.K / 64;
+    const int64_t U = (int64_t)((p.M + 127) / 128) * nkb;
+    const int row0 = glu ? 2 * k0 : k0;  // the previous phase's first output row of these columns
+    const int tile = row0 / 128, r0 = row0 % 128;
+    const int c_first = unit_owner((int64_t)tile * nkb, U, p.G);
+    const int c_last = unit_owner((int64_t)(tile + 1) * nkb - 1, U, p.G);
+    float* y = p.y + (size_t)b * p.ldy + k0;
+    if (c_first == c_last) {  // a whole tile: the phase stored it
+        const float4 q0 = __ldcg(reinterpret_cast<const float4*>(y)), q1 = __ldcg(reinterpret_cast<const float4*>(y) + 1);
+        v[0] = q0.x; v[1] = q0.y; v[2] = q0.z; v[3] = q0.w; v[4] = q1.x; v[5] = q1.y; v[6] = q1.z; v[7] = q1.w;
+        return;
+    }
+    float sm[NR];
+#pragma unroll
+    for (int i = 0; i < NR; ++i) sm[i] = 0.f;
+    // the shares in batches of kPrevBatch CTAs: every load of a batch is issued before any
+    // is summed (one L2 round trip per batch), the sums still in CTA order
+    constexpr int kPrevBatch = GLU ? 4 : 8;  // (register budget: NR floats per share)
+    for (int c0 = c_first; c0 <= c_last; c0 += kPrevBatch) {
+        float x[kPrevBatch][NR];
+#pragma unroll
+        for (int j = 0; j < kPrevBatch; ++j) {
+            const int c = c0 + j;
+            if (c > c_last) break;
+            const int cs = (int)(unit_begin(c, U, p.G) / nkb) == tile ? 0 : 1;
+            const float4* q = reinterpret_cast<const float4*>(p.part + ((size_t)(c * 2 + cs) * BP + b) * 128 + r0);
+#pragma unroll
+            for (int i = 0; i < NR / 4; ++i) {
+                const float4 w = __ldcg(q + i);
+                x[j][4 * i] = w.x; x[j][4 * i + 1] = w.y; x[j][4 * i + 2] = w.z; x[j][4 * i + 3] = w.w;
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < kPrevBatch; ++j) {
+            if (c0 + j > c_last) break;
+#pragma unroll
+            for (int i = 0; i < NR; ++i) sm[i] += x[j][i];
+        }
+    }
+    if constexpr (GLU) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = silu(sm[2 * e]) * sm[2 * e + 1];
+    } else if (p.epi == EPI_RESID) {
+        const float* base = p.ybase ? p.ybase + (size_t)b * p.ldy + k0 : y;
+        const float4 b0 = __ldcg(reinterpret_cast<const float4*>(base)), b1 = __ldcg(reinterpret_cast<const float4*>(base) + 1);
+        const float r[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = r[e] + sm[e];
+        if (p.y2) {
+            float* y2 = p.y2 + (size_t)b * p.ldy2 + k0;
+            reinterpret_cast<float4*>(y2)[0] = make_float4(v[0], v[1], v[2], v[3]);
+            reinterpret_cast<float4*>(y2)[1] = make_float4(v[4], v[5], v[6], v[7]);
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = sm[e];
+    }
+    reinterpret_cast<float4*>(y)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4*>(y)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+__device__ __forceinline__ void prev_finish(const LinearArgs::Prev& p, int BP, int b, int k0, float (&v)[8]) {
+    if (p.epi == EPI_SWIGLU) prev_finish_t<true>(p, BP, b, k0, v);
+    else prev_finish_t<false>(p, BP, b, k0, v);
+}
+
+// the bf16 hi / lo operand chunk c of row b from 8 values
+__device__ __forceinline__ void put_operand(uint16_t* xb, int N, int B_pad, int b, int c, const float (&v)[8]) {
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) {
+        uint16_t h0, l0, h1, l1;
+        split_bf16(v[e], h0, l0);
+        split_bf16(v[e + 1], h1, l1);
+        hi[e / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+        lo[e / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+    }
+    unsigned char* blk = (unsigned char*)xb + (size_t)(c / 8) * N * 128;
+    *reinterpret_cast<uint4*>(blk + sw128_offset(b, c % 8)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *reinterpret_cast<uint4*>(blk + sw128_offset(B_pad + b, c % 8)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+}
 
 __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
     const LaunchStamp stamp(a.stamp);
@@ -63,6 +180,7 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
     griddep_launch_dependents();
     griddep_wait();
     const bool live = b < a.B;
+    const bool fin = live && a.prev.active;  // (RMSNorm inputs take xprep_row_kernel instead)
     int tok = 0;
     if (live && a.pro == PRO_CONCAT_EMB) {
         tok = a.tok[b];
@@ -72,6 +190,16 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
         }
     }
     const float* xf = (const float*)a.x + (size_t)b * a.ldx;
+    // 1 / sqrt(mean of squares + eps) from each thread's partial sum (CTA-wide)
+    auto rs_of = [&](float ss) {
+        ss = warp_sum(ss);
+        if ((t & 31) == 0) red[t >> 5] = ss;
+        __syncthreads();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        return 1.0f / sqrtf(tot / (float)K + a.eps);
+    };
     float rs = 1.f;
     if (live && a.pro == PRO_RMSNORM) {
         float ss = 0.f;
@@ -79,15 +207,10 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
         for (int c = t; c < nc; c += 256) {
             const float4 p = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c);
             const float4 q = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c + 1);
-            ss += p.x * p.x + p.y * p.y + p.z * p.z + p.w * p.w + q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+            const float v[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
+            ss += sumsq8(v);
         }
-        ss = warp_sum(ss);
-        if ((t & 31) == 0) red[t >> 5] = ss;
-        __syncthreads();
-        float tot = 0.f;
-#pragma unroll
-        for (int w = 0; w < 8; ++w) tot += red[w];
-        rs = 1.0f / sqrtf(tot / (float)K + a.eps);
+        rs = rs_of(ss);
     }
     {
         const int c = blockIdx.y * kXprepChunks + t;
@@ -104,6 +227,8 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
                     Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.embed +
                                                                          (size_t)tok * (K - a.d_split) + (k0 - a.d_split)),
                                          v);
+            } else if (fin) {  // the previous phase's output, its split tiles finished here
+                prev_finish(a.prev, B_pad, b, k0, v);
             } else {  // float32 input (PRO_F32, PRO_RMSNORM, or the float part of PRO_CONCAT_EMB)
                 const float4 p = __ldcg(reinterpret_cast<const float4*>(xf + k0));
                 const float4 q = __ldcg(reinterpret_cast<const float4*>(xf + k0) + 1);
@@ -116,33 +241,57 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
                 }
             }
         }
-        uint32_t hi[4], lo[4];
+        put_operand(xb, N, B_pad, b, c, v);
+    }
+}
+
+// The deferred-input prep of an RMSNorm phase: one CTA of kRowThreads per row b finishes the
+// previous phase's output over the whole row into shared memory (its split tiles, as
+// prev_finish), sums its squares and writes the normalised row's operand. Thread t owns
+// chunks t, t + kRowThreads, ... (the same per-thread order of the sum as xprep_kernel).
+constexpr int kRowThreads = 512;
+
+__global__ void __launch_bounds__(kRowThreads) xprep_row_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
+    const LaunchStamp stamp(a.stamp);
+    extern __shared__ __align__(16) float xrow[];  // the finished row [K]
+    const int b = blockIdx.x, t = threadIdx.x;
+    const int N = 2 * B_pad, K = a.K, nc = K / 8;
+    __shared__ float red[kRowThreads / 32];
+    griddep_launch_dependents();
+    griddep_wait();
+    if (b >= a.B) {  // a padding row of the operand is zero
+        const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int c = t; c < nc; c += kRowThreads) put_operand(xb, N, B_pad, b, c, z);
+        return;
+    }
+    float ss = 0.f;
+    for (int c = t; c < nc; c += kRowThreads) {
+        float v[8];
+        prev_finish_t<false>(a.prev, B_pad, b, 8 * c, v);  // (an RMSNorm input is never SwiGLU's output)
+        ss += sumsq8(v);
+        reinterpret_cast<float4*>(xrow)[2 * c] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4*>(xrow)[2 * c + 1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+    ss = warp_sum(ss);
+    if ((t & 31) == 0) red[t >> 5] = ss;
+    __syncthreads();  // (also publishes xrow)
+    float tot = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; e += 2) {
-            uint16_t h0, l0, h1, l1;
-            split_bf16(v[e], h0, l0);
-            split_bf16(v[e + 1], h1, l1);
-            hi[e / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-            lo[e / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
-        }
-        unsigned char* blk = (unsigned char*)xb + (size_t)(c / 8) * N * 128;
-        *reinterpret_cast<uint4*>(blk + sw128_offset(b, c % 8)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(blk + sw128_offset(B_pad + b, c % 8)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
+    const float rs = 1.0f / sqrtf(tot / (float)K + a.eps);
+    for (int c = t; c < nc; c += kRowThreads) {
+        float v[8], g[8];
+        const float4 p = reinterpret_cast<const float4*>(xrow)[2 * c];
+        const float4 q = reinterpret_cast<const float4*>(xrow)[2 * c + 1];
+        v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
+        Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + 8 * c), g);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = v[e] * rs * g[e];
+        put_operand(xb, N, B_pad, b, c, v);
     }
 }
 
 // ---- the product ---------------------------------------------------------------------------
-// first unit of CTA c when U units are split over G CTAs
-__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
-
-// the CTA whose range holds unit u
-__device__ __forceinline__ int unit_owner(int64_t u, int64_t U, int G) {
-    int c = (int)((u * G) / U);
-    while (c + 1 < G && unit_begin(c + 1, U, G) <= u) ++c;
-    while (c > 0 && unit_begin(c, U, G) > u) --c;
-    return c;
-}
-
 // Epilogue for output row m of all B sequences; v[b] is the finished dot product.
 // SwiGLU pairs rows (2j, 2j + 1) held by neighbouring lanes of one warp.
 template <int BP>
@@ -304,6 +453,7 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             float* pp = part + ((size_t)(cta * 2 + slot) * BP) * 128 + r;
 #pragma unroll
             for (int b = 0; b < BP; ++b) pp[(size_t)b * 128] = v[b];
+            if (a.defer) continue;  // the next phase's operand prep finishes this tile
             // lane 0's acquire-release add publishes the warp's shares (ordered before it by
             // the warp barrier) and, in the last warp to arrive, orders the reads below
             __syncwarp();
@@ -376,7 +526,9 @@ size_t linear_mma_part_bytes(int B, const DeviceInfo& dev) {
 }
 
 cudaError_t linear_mma_prepare(const DeviceInfo& dev) {
-    cudaError_t e;
+    cudaError_t e = cudaFuncSetAttribute(xprep_row_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kXprepRowSmem);
+    if (e != cudaSuccess) return e;
     if ((e = set_attr<8>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<16>(dev)) != cudaSuccess) return e;
     if ((e = set_attr<24>(dev)) != cudaSuccess) return e;
@@ -387,8 +539,12 @@ cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, in
                               cudaStream_t st, cudaEvent_t after_prep) {
     if (!linear_mma_ok(a.M, a.K, a.B)) return cudaErrorInvalidValue;
     const int BP = linear_mma_bpad(a.B);
+    const bool row_cta = a.prev.active && a.pro == PRO_RMSNORM;  // finish + normalise a row per CTA
+    if (row_cta && ((size_t)a.K * sizeof(float) > kXprepRowSmem || a.prev.epi == EPI_SWIGLU)) return cudaErrorInvalidValue;
     const int ny = (a.K / 8 + kXprepChunks - 1) / kXprepChunks;
-    cudaError_t e = launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb);
+    cudaError_t e = row_cta ? launch_k(xprep_row_kernel, dim3(BP), dim3(kRowThreads), (size_t)a.K * sizeof(float), st,
+                                       a.pdl, a, BP, xb)
+                            : launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     const int grid = linear_mma_grid(a.M, a.K, dev);

@@ -122,6 +122,7 @@ struct fe_handle {
     int* lm_counters = nullptr;
     bool lm_mma = false;      // LM head packed for (and run on) the tensor cores
     bool lin_mma = false;     // linear phases packed for (and run on) the tensor cores
+    bool lin_defer = true;    // tensor-core phases leave split tiles to the next phase's prep
     uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
     float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
     int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
@@ -293,10 +294,36 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         ++nstack;
         return FE_OK;
     };
+    // a tensor-core phase followed by another defers its split tiles to that phase's operand
+    // prep (LinearArgs::defer / prev): `pending` carries the deferring phase to the next one
+    LinearArgs::Prev pending{};
+    const void* next_in = nullptr;  // the buffer the next tensor-core phase reads (set by next_is below)
     auto linear = [&](const LinearArgs& L0) -> fe_status {
         cudaError_t e;
         LinearArgs L = L0;
         L.stamp = stacked ? nullptr : next_stamp(pf);
+        if (h->lin_mma) {
+            if (pending.active && pending.y != L.x) {  // a deferred phase must be finished by its reader
+                set_error_detail("internal: a deferred linear phase is not followed by its reader");
+                return FE_ERR_CUDA;
+            }
+            L.prev = pending;
+            pending = LinearArgs::Prev{};
+            L.defer = h->lin_defer && L.next_W && next_in == L.y ? 1 : 0;
+            if (L.defer) {
+                pending.active = 1;
+                pending.part = h->lin_part;
+                pending.M = L.M;
+                pending.K = L.K;
+                pending.G = linear_mma_grid(L.M, L.K, h->dev);
+                pending.epi = L.epi;
+                pending.y = L.y;
+                pending.ldy = L.ldy;
+                pending.y2 = L.y2;
+                pending.ldy2 = L.ldy2;
+                pending.ybase = L.ybase;
+            }
+        }
         if (stacked) {
             if (sq.nph == kMaxStackPhases) {
                 const fe_status r = flush_stack();
@@ -330,6 +357,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.status = h->status;
     la.eps = c.rms_eps;
     la.B = B;
+    // tensor-core phases: the phase that follows and the buffer it reads (a phase defers its
+    // split tiles only to a tensor-core successor that reads its output)
+    auto next_is = [&](const void* W, int, int, const void* in) {
+        la.next_W = h->lin_mma ? W : nullptr;
+        next_in = W ? in : nullptr;
+    };
     // g = W_fuse concat(l, m, h). The first kernel of a draft waits for everything before it
     // on the stream (it is launched without programmatic dependence); later kernels may
     // overlap their predecessor's tail (see griddep_wait()).
@@ -337,6 +370,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.W = h->w_fuse; la.M = d; la.K = 3 * d;
     la.pro = PRO_STORAGE; la.x = a->feat; la.ldx = 3 * d;
     la.epi = EPI_STORE; la.y = h->g; la.ldy = d; la.y2 = nullptr;
+    next_is(h->w_in, d, 2 * d, h->g);
     FE_LINEAR(la);
     la.pdl = pdl;
     // x0 = W_in concat(g, e)
@@ -344,6 +378,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     la.pro = PRO_CONCAT_EMB; la.x = h->g; la.ldx = d; la.embed = h->embed; la.tok = a->next_tok;
     la.d_split = d; la.vocab = V;
     la.epi = EPI_STORE; la.y = h->x0; la.ldy = d;
+    next_is(h->layers[0].w_qkv, nqkv, d, h->x0);
     FE_LINEAR(la);
 
     AttnArgs aa{};
@@ -365,6 +400,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         const bool from_x0 = i == 0 || c.parallel_layers;
         la.pro = PRO_RMSNORM; la.x = from_x0 ? h->x0 : h->x; la.ldx = d; la.gamma = L.attn_norm;
         la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
+        next_is(nullptr, 0, 0, nullptr);  // attention follows
         FE_LINEAR(la);
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
@@ -377,17 +413,21 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         la.W = L.w_o; la.M = d; la.K = H * hd;
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr; la.ybase = from_x0 ? h->x0 : nullptr;
+        next_is(L.w_gu, 2 * F, d, h->x);
         FE_LINEAR(la);
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
         la.slots = 0;
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
         la.pro = PRO_RMSNORM; la.x = h->x; la.ldx = d; la.gamma = L.mlp_norm; la.ybase = nullptr;
         la.epi = EPI_SWIGLU; la.y = h->act; la.ldy = F;
+        next_is(L.w_down, d, F, h->act);
         FE_LINEAR(la);
         // x += W_down a; h_i = x
         la.W = L.w_down; la.M = d; la.K = F;
         la.pro = PRO_F32; la.x = h->act; la.ldx = F;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = h->hid + (size_t)i * B * d; la.ldy2 = d;
+        if (i + 1 < N) next_is(h->layers[i + 1].w_qkv, nqkv, d, c.parallel_layers ? h->x0 : h->x);
+        else next_is(nullptr, 0, 0, nullptr);  // the LM head follows
         FE_LINEAR(la);
     }
 
@@ -646,6 +686,8 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             // programmatic dependent launch inside the CUDA graph are faster (720 vs 762 us
             // per Vicuna-13B-shaped draft); the stacks win only without programmatic launch.
             const int kmax = std::max({3 * c.d, c.ffn, c.n_heads * c.head_dim});
+            const char* df = getenv("FE_DRAFT_LIN_DEFER");
+            h->lin_defer = !(df && df[0] == '0');
             const char* sk = getenv("FE_DRAFT_STACK");
             h->use_stack = !h->lin_mma && sk && sk[0] == '1' && stack_slots(kmax, h->dev) >= 1;
         }

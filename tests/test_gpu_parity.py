@@ -212,3 +212,22 @@ def test_parity_full_size(orc, name):
         stats.append(H.compare(orc, cfg, g, o, b))
         _check_cache_rows(cfg, W, I, ks, vs, g, o, b)
     print(name, stats)
+
+
+@pytest.mark.parametrize("case", ["tc_linear_b12_ragged", "tc_linear_b9_paged", "parallel_tc_b12"])
+def test_deferred_split_tiles_bit_identical(monkeypatch, case):
+    """A tensor-core phase followed by another leaves the tiles it shares with other CTAs to
+    that phase's operand prep, which sums the shares in CTA order and applies the epilogue
+    there. The draft must equal the one with the reduction inside each phase
+    (FE_DRAFT_LIN_DEFER=0) bit for bit: logits, hidden states, candidates, caches."""
+    spec = dict(SMALL[case])
+    cfg = wl.make_config(spec.pop("name"), **spec)
+    W, I, ks, vs = _problem(cfg)
+    a = H.run_gpu(cfg, W, I, ks, vs)
+    monkeypatch.setenv("FE_DRAFT_LIN_DEFER", "0")
+    b = H.run_gpu(cfg, W, I, ks, vs)
+    assert a["status"] == 0 and b["status"] == 0
+    for key in ("logits", "hidden", "topk_id", "topk_logit", "topk_prob", "lse", "tree_tok"):
+        assert np.array_equal(a[key], b[key]), key
+    for i in range(cfg["n_layers"]):
+        assert torch.equal(a["k_cache"][i], b["k_cache"][i]) and torch.equal(a["v_cache"][i], b["v_cache"][i]), i
