@@ -250,4 +250,13 @@ __device__ __forceinline__ float warp_max(float v) {
 // SiLU(a) = a / (1 + e^-a)
 __device__ __forceinline__ float silu(float a) { return a / (1.0f + expf(-a)); }
 
+// 2^x by the hardware approximation (relative error about 2^-22; 2^-inf = 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+
 }  // namespace fe

@@ -367,36 +367,47 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
     const uint32_t tmem = st.tmem_base;
     griddep_launch_dependents();
 
+    // Ring positions advance by counters (slot, phase bit), not by division: the producer and
+    // the MMA issuer are single threads whose every instruction is on the stream's critical
+    // path.
     if (warp == 4) {  // ---- TMA producer
         if (lane == 0) {
             const int total = (int)(u1 - u0);
             const int pre = min(S, total);
             const uint32_t xbytes = (uint32_t)N * 128u;
+            const unsigned char* Wsrc = (const unsigned char*)a.W + (size_t)u0 * 16384;
             // the weights do not depend on earlier kernels: the first stages go out at once
             for (int it = 0; it < pre; ++it) {
                 mbar_arrive_expect_tx(&st.full[it], 16384u + xbytes);
-                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384,
-                         &st.full[it]);
+                bulk_g2s(ring + (size_t)it * stage_bytes, Wsrc + (size_t)it * 16384, 16384, &st.full[it]);
             }
             griddep_wait();
-            for (int it = 0; it < pre; ++it)
-                bulk_g2s(ring + (size_t)it * stage_bytes + 16384,
-                         (const unsigned char*)xb + (size_t)((u0 + it) % nkb) * xbytes, xbytes, &st.full[it]);
+            int kx = (int)(u0 % nkb);  // activation block of the next copy: (u0 + it) % nkb
+            for (int it = 0; it < pre; ++it) {
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)xb + (size_t)kx * xbytes, xbytes,
+                         &st.full[it]);
+                if (++kx == nkb) kx = 0;
+            }
+            // iteration it >= S reuses slot it % S after the MMAs of iteration it - S: completion
+            // (it - S) / S of empty[slot]
+            int slot = 0;
+            uint32_t pe = 0;
             for (int it = pre; it < total; ++it) {
-                const int slot = it % S;
-                if (!mbar_wait_abortable(&st.empty[slot], ((uint32_t)(it / S) & 1u) ^ 1u, a.status, &st.abort)) break;
+                if (!mbar_wait_abortable(&st.empty[slot], pe, a.status, &st.abort)) break;
                 unsigned char* dst = ring + (size_t)slot * stage_bytes;
                 mbar_arrive_expect_tx(&st.full[slot], 16384u + xbytes);
-                bulk_g2s(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot]);
-                bulk_g2s(dst + 16384, (const unsigned char*)xb + (size_t)((u0 + it) % nkb) * xbytes, xbytes,
-                         &st.full[slot]);
+                bulk_g2s(dst, Wsrc + (size_t)it * 16384, 16384, &st.full[slot]);
+                bulk_g2s(dst + 16384, (const unsigned char*)xb + (size_t)kx * xbytes, xbytes, &st.full[slot]);
+                if (++kx == nkb) kx = 0;
+                if (++slot == S) { slot = 0; pe ^= 1u; }
             }
         }
     } else if (warp == 5) {  // ---- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, N);
             int64_t u = u0;
-            int it = 0;
+            int slot = 0;
+            uint32_t pf = 0;  // phase bit of full[slot]
             for (int tile = tile0, j = 0; tile <= tile1; ++tile, ++j) {
                 const int buf = j & 1;
                 const int64_t ue = min(u1, (int64_t)(tile + 1) * nkb);
@@ -404,9 +415,8 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * N);
                 bool ok = true;
-                for (bool first = true; u < ue; ++u, ++it, first = false) {
-                    const int slot = it % S;
-                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                for (bool first = true; u < ue; ++u, first = false) {
+                    if (!mbar_wait_abortable(&st.full[slot], pf, a.status, &st.abort)) {
                         ok = false;
                         break;
                     }
@@ -417,6 +427,7 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
                     for (int kk = 0; kk < 4; ++kk)
                         tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (!first || kk) ? 1u : 0u);
                     tc_commit(&st.empty[slot]);
+                    if (++slot == S) { slot = 0; pf ^= 1u; }
                 }
                 if (!ok) break;
                 tc_commit(&st.tfull[buf]);

@@ -683,25 +683,34 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                          &st.full[it]);
             }
             griddep_wait();
-            for (int it = 0; it < pre; ++it)
-                bulk_g2s(ring + (size_t)it * stage_bytes + 16384,
-                         (const unsigned char*)zb + (size_t)((u0 + it) % nkb) * N * 128, (uint32_t)N * 128, &st.full[it]);
+            // ring positions advance by counters, not by division (a single thread on the
+            // stream's critical path)
+            int kb = (int)(u0 % nkb);  // z block of the next copy: (u0 + it) % nkb
+            for (int it = 0; it < pre; ++it) {
+                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)zb + (size_t)kb * N * 128,
+                         (uint32_t)N * 128, &st.full[it]);
+                if (++kb == nkb) kb = 0;
+            }
+            // iteration it >= S reuses slot it % S after the MMAs of iteration it - S: completion
+            // (it - S) / S of empty[slot]
+            int slot = 0;
+            uint32_t pe = 0;
             for (int it = pre; it < total; ++it) {
-                const int slot = it % S;
-                const uint32_t u = (uint32_t)(it / S);
-                if (!mbar_wait_abortable(&st.empty[slot], (u & 1u) ^ 1u, a.status, &st.abort)) break;
-                const int kb = (int)((u0 + it) % nkb);
+                if (!mbar_wait_abortable(&st.empty[slot], pe, a.status, &st.abort)) break;
                 unsigned char* dst = ring + (size_t)slot * stage_bytes;
                 mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
                 bulk_g2s(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot]);
                 bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
                          &st.full[slot]);
+                if (++kb == nkb) kb = 0;
+                if (++slot == S) { slot = 0; pe ^= 1u; }
             }
         }
     } else if (warp == 5) {  // ---- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, N);
-            int it = 0;
+            int slot = 0;
+            uint32_t pf = 0;  // phase bit of full[slot]
             int64_t u = u0;
             for (int tile = tf, j = 0; tile <= tl; ++tile, ++j) {  // one piece (accumulator) per tile
                 const int buf = j & 1;
@@ -710,9 +719,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * N);
                 const int64_t ue = min(u1, (int64_t)(tile + 1) * nkb);
                 bool ok = true;
-                for (bool first = true; u < ue; ++u, ++it, first = false) {
-                    const int slot = it % S;
-                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                for (bool first = true; u < ue; ++u, first = false) {
+                    if (!mbar_wait_abortable(&st.full[slot], pf, a.status, &st.abort)) {
                         ok = false;
                         break;
                     }
@@ -723,6 +731,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                     for (int kk = 0; kk < 4; ++kk)  // K = 16 per MMA: +32 bytes inside the swizzled rows
                         tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (!first || kk) ? 1u : 0u);
                     tc_commit(&st.empty[slot]);
+                    if (++slot == S) { slot = 0; pf ^= 1u; }
                 }
                 if (!ok) break;
                 tc_commit(&st.tfull[buf]);
@@ -964,23 +973,35 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
 //   - z is rounded once to bf16 (N = R_pad MMA columns, R_pad <= 256); every product is
 //     accumulated in float32. The logit error this leaves is of the order of
 //     |W_v| |z| 2^-9 / sqrt(3), a few 1e-3 at d = 4096 with weights ~ N(0, 0.02^2).
+//   - The weight blocks and the z blocks travel in two rings of their own: a weight block
+//     comes from HBM and a z block from L2 (every CTA reads all of z once per tile), so the
+//     weight ring runs as many stages ahead as shared memory allows (the bytes in flight
+//     that keep HBM busy) while a few stages cover the z block's L2 latency.
 //   - TMEM holds two R_pad-column accumulators, so the epilogue of tile j overlaps the
 //     MMAs of tile j + 1.
-//   - The epilogue transposes each tile through shared memory, 128 rows at a time, so that
-//     a thread owns one hidden row r (two for R > 128) and reads the tile's 128 logits of
-//     that row: its softmax statistics are exact (the tile's max, then its sum of exp, then
-//     one rescale of the running pair) and its running top-k is a sorted list in registers
-//     (an entry enters only if it beats the current k-th best, ties to the smaller id),
-//     with no cross-thread reduction per tile. At the end of the slab it writes the row's
-//     partial.
+//   - Eight epilogue warps, one hidden row per thread: warps 4 g .. 4 g + 3 own rows
+//     128 g .. 128 g + 127. A tile's accumulator has the vocabulary entries as TMEM lanes
+//     and the rows as columns, so each row group transposes it through shared memory in two
+//     rounds of 64 entries x 128 rows (the two warps whose lanes hold those entries copy
+//     them). A thread then reads its row's logits in batches of 32 held in registers: the
+//     batch max, a mask of the entries that reach the running top-k list's k-th value (only
+//     those run through the list's insertion network), the sum of exp against the batch
+//     max (base 2, on the hardware's 2^x) and one rescale of the running (max, sum). The
+//     list is sorted in registers (larger value first, ties to the smaller id); there is no
+//     cross-thread reduction. At the end of the slab each thread writes its row's partial.
 //   - lmhead_merge_kernel (one CTA per row) then merges the slabs as merge_rows does.
 constexpr int kWideKMax = 16;     // top_k limit of this kernel (a sorted list in registers)
 constexpr int kWideRowsMax = 256;
-constexpr int kWideGroup = 128;   // rows staged per transpose round (one per epilogue thread)
+constexpr int kWideGroup = 128;   // rows of a row group (one per thread of its four warps)
+constexpr int kWideHalf = 64;     // vocabulary entries staged per transpose round (half a tile)
 constexpr int kWideTileStride = kWideGroup + 1;  // floats per staged vocabulary entry (no bank conflicts)
+constexpr int kWideMaxW = 12;     // weight-ring stages (16 KB each)
+constexpr int kWideMaxZ = 4;      // z-ring stages at most (R_pad x 128 B each)
+constexpr int kWideThreads = 10 * 32;  // 8 epilogue warps, 1 producer warp, 1 MMA warp
 
 struct WideState {
-    uint64_t full[kMmaMaxStages], empty[kMmaMaxStages], tfull[2], tempty[2], ebar[2];
+    uint64_t wfull[kWideMaxW], zfull[kWideMaxW], done[kWideMaxW], tfull[2], tempty[2],
+        ebar[2][2];
     uint32_t tmem_base;
     int abort;
 };
@@ -1050,121 +1071,74 @@ struct WideRow {
     }
 };
 
-// One 128-row group g of a tile for row state w (inside lmhead_wide_kernel's epilogue).
-// Expanded textually for each group: written as a lambda or function taking the state by
-// reference, the compiler keeps a state in local memory, and each step of the loop below
-// then waits on a round trip to L2.
-//   stage:   warp w copies TMEM lanes 32 w .. 32 w + 31 (vocabulary entries) x the group's
-//            128 columns (hidden rows) into tbuf[entry][row];
-//   consume: thread t reads row r = 128 g + t across the tile's entries: the max (eight
-//            independent loads at a time) and a 128-bit mask of the entries that reach the
-//            list's last value; only those (a few per tile) run through the branch-free
-//            insertion network, whose serial compare-exchange chain is too slow to run on
-//            every entry; then the sum of exp against that max and one rescale of the
-//            running (max, sum).
-#define FE_WIDE_GROUP(w, g)                                                                        \
+// One batch of up to 32 of a round's entries (round entries e0 .. e0 + 31, vocabulary ids
+// id0 + e) for the thread's row state w (inside lmhead_wide_kernel's epilogue).
+// col[e * kWideTileStride] is the row's logit of round entry e; nv entries of the round are
+// valid. Expanded textually: written as a function taking the state by reference, the
+// compiler keeps the state in local memory.
+#define FE_WIDE_BATCH(e0)                                                                          \
     do {                                                                                           \
-        if ((g) >= ngroups || !ok) break;                                                          \
-        float* trow = tbuf + (size_t)(warp * 32 + lane) * kWideTileStride;                         \
-        for (int c0 = 0; c0 < kWideGroup && (g) * kWideGroup + c0 < R_pad; c0 += 16) {             \
-            float v16[16];                                                                         \
-            tc_ld16(taddr + (uint32_t)((g) * kWideGroup + c0), v16);                               \
-            _Pragma("unroll") for (int i = 0; i < 16; ++i) trow[c0 + i] = v16[i];                  \
-        }                                                                                          \
-        if ((g) == ngroups - 1) { /* the accumulator is read: hand it back to the MMA warp */      \
-            tc_fence_before();                                                                     \
-            __syncwarp();                                                                          \
-            if (lane == 0) mbar_arrive(&st.tempty[buf]);                                           \
-        }                                                                                          \
-        if (!(ok = epi_sync())) break;                                                             \
-        const int r = (g) * kWideGroup + t;                                                        \
-        if (r < R) {                                                                               \
-            const int id0 = tile * 128;                                                            \
-            const int nv = min(128, a.V - id0);                                                    \
-            const float* col = tbuf + t;                                                           \
-            const float th = w.v[KM - 1];                                                          \
-            float M = -INFINITY;                                                                   \
-            uint32_t cm0 = 0u, cm1 = 0u, cm2 = 0u, cm3 = 0u; /* entries >= th, one bit each */     \
-            _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                     \
-                uint32_t bits = 0u;                                                                \
-                for (int b0 = 0; b0 < 32; b0 += 8) {                                               \
-                    float x[8];                                                                    \
-                    _Pragma("unroll") for (int u = 0; u < 8; ++u) {                                \
-                        const int e = wd * 32 + b0 + u;                                            \
-                        x[u] = e < nv ? col[(size_t)e * kWideTileStride] : -INFINITY;              \
-                    }                                                                              \
-                    _Pragma("unroll") for (int u = 0; u < 8; ++u) {                                \
-                        M = fmaxf(M, x[u]);                                                        \
-                        if (!SMP) bits |= (x[u] >= th ? 1u : 0u) << (b0 + u);                      \
-                    }                                                                              \
-                }                                                                                  \
-                if (wd == 0) cm0 = bits;                                                           \
-                else if (wd == 1) cm1 = bits;                                                      \
-                else if (wd == 2) cm2 = bits;                                                      \
-                else cm3 = bits;                                                                   \
-            }                                                                                      \
-            if (SMP) { /* keys: a deviate code per entry, logarithms only past the code floor */   \
-                const int srow = sample_row(r, a.B, a.N);                                          \
-                const uint32_t mlo = sample_code_floor(th, M * a.inv_temp);                        \
-                _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                 \
-                    uint32_t bits = 0u;                                                            \
-                    for (int e0 = 0; e0 < 32; ++e0) {                                              \
-                        const int e = wd * 32 + e0;                                                \
-                        if (e >= nv) break;                                                        \
-                        const uint32_t m23 = (uint32_t)(splitmix64_at(a.seed,                      \
-                            sample_counter(srow, a.V, id0 + e)) >> 41);                            \
-                        if (m23 < mlo) continue;                                                   \
-                        const float key = fmaf(col[(size_t)e * kWideTileStride], a.inv_temp,       \
+        if ((e0) >= nv) break;                                                                     \
+        float x[32];                                                                               \
+        _Pragma("unroll") for (int u = 0; u < 32; ++u)                                             \
+            x[u] = (e0) + u < nv ? col[(size_t)((e0) + u) * kWideTileStride] : -INFINITY;          \
+        float m4[4] = {x[0], x[1], x[2], x[3]};                                                    \
+        _Pragma("unroll") for (int u = 4; u < 32; ++u) m4[u & 3] = fmaxf(m4[u & 3], x[u]);         \
+        const float M = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));                           \
+        /* the list's k-th value (-inf until k entries are in): its smallest of the first k */    \
+        float th = w.v[0];                                                                         \
+        _Pragma("unroll") for (int q = 1; q < KM; ++q) th = q < k ? fminf(th, w.v[q]) : th;        \
+        uint32_t bits = 0u; /* entries that can enter the list */                                  \
+        if (!SMP) {                                                                                \
+            _Pragma("unroll") for (int u = 0; u < 32; ++u)                                         \
+                bits |= ((e0) + u < nv && x[u] >= th ? 1u : 0u) << u;                              \
+        } else { /* keys: a deviate code per entry, logarithms only past the code floor */         \
+            const int srow = sample_row(r, a.B, a.N);                                              \
+            const uint32_t mlo = sample_code_floor(th, M * a.inv_temp);                            \
+            _Pragma("unroll") for (int u = 0; u < 32; ++u) {                                       \
+                if ((e0) + u < nv) {                                                               \
+                    const uint32_t m23 = (uint32_t)(splitmix64_at(a.seed,                          \
+                        sample_counter(srow, a.V, id0 + (e0) + u)) >> 41);                         \
+                    if (m23 >= mlo) {                                                              \
+                        const float key = fmaf(x[u], a.inv_temp,                                   \
                             gumbel_of(((float)m23 + 0.5f) * (1.0f / 8388608.0f)));                 \
-                        bits |= (key >= th ? 1u : 0u) << e0;                                       \
+                        bits |= (key >= th ? 1u : 0u) << u;                                        \
                     }                                                                              \
-                    if (wd == 0) cm0 = bits;                                                       \
-                    else if (wd == 1) cm1 = bits;                                                  \
-                    else if (wd == 2) cm2 = bits;                                                  \
-                    else cm3 = bits;                                                               \
                 }                                                                                  \
-            }                                                                                      \
-            _Pragma("unroll") for (int wd = 0; wd < 4; ++wd) {                                     \
-                uint32_t bits = wd == 0 ? cm0 : wd == 1 ? cm1 : wd == 2 ? cm2 : cm3;               \
-                while (bits) {                                                                     \
-                    const int e = wd * 32 + __ffs(bits) - 1;                                       \
-                    bits &= bits - 1u;                                                             \
-                    const float xe = col[(size_t)e * kWideTileStride];                             \
-                    if (SMP)                                                                       \
-                        wide_insert(w.v, w.i, w.l, k, sample_key(xe, a.inv_temp, a.seed,           \
-                                    sample_row(r, a.B, a.N), a.V, id0 + e), id0 + e, xe);          \
-                    else                                                                           \
-                        wide_insert(w.v, w.i, k, xe, id0 + e);                                     \
-                }                                                                                  \
-            }                                                                                      \
-            if (nv > 0) {                                                                          \
-                const float Mt = M * a.inv_temp;                                                   \
-                float S = 0.f;                                                                     \
-                for (int u0 = 0; u0 < nv; u0 += 8) {                                               \
-                    _Pragma("unroll") for (int u = 0; u < 8; ++u)                                  \
-                        if (u0 + u < nv) S += expf(col[(size_t)(u0 + u) * kWideTileStride] * a.inv_temp - Mt); \
-                }                                                                                  \
-                const float nm = fmaxf(w.m, Mt);                                                   \
-                w.s = (w.m == -INFINITY ? 0.f : w.s * expf(w.m - nm)) + S * expf(Mt - nm);         \
-                w.m = nm;                                                                          \
-            }                                                                                      \
-            if (a.dbg_logits) {                                                                    \
-                const int rb = r % a.B, ri = r / a.B;                                              \
-                for (int u = 0; u < nv; ++u)                                                       \
-                    a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id0 + u] = col[(size_t)u * kWideTileStride]; \
             }                                                                                      \
         }                                                                                          \
-        ok = epi_sync();                                                                           \
+        while (bits) {                                                                             \
+            const int e = (e0) + __ffs(bits) - 1;                                                  \
+            bits &= bits - 1u;                                                                     \
+            const float xe = col[(size_t)e * kWideTileStride];                                     \
+            if (SMP)                                                                               \
+                wide_insert(w.v, w.i, w.l, k, sample_key(xe, a.inv_temp, a.seed,                   \
+                            sample_row(r, a.B, a.N), a.V, id0 + e), id0 + e, xe);                  \
+            else                                                                                   \
+                wide_insert(w.v, w.i, k, xe, id0 + e);                                             \
+        }                                                                                          \
+        /* sum of exp(x / T - M / T) in base 2: 2^(x c - M c), c = log2(e) / T */                 \
+        const float c2 = a.inv_temp * kLog2e, mc = M * c2;                                         \
+        float s4[4] = {0.f, 0.f, 0.f, 0.f};                                                        \
+        _Pragma("unroll") for (int u = 0; u < 32; ++u) s4[u & 3] += ex2_approx(fmaf(x[u], c2, -mc)); \
+        const float S = (s4[0] + s4[1]) + (s4[2] + s4[3]);                                         \
+        const float Mt = M * a.inv_temp;                                                           \
+        const float nm = fmaxf(w.m, Mt);                                                           \
+        w.s = (w.m == -INFINITY ? 0.f : w.s * ex2_approx((w.m - nm) * kLog2e)) + S * ex2_approx((Mt - nm) * kLog2e); \
+        w.m = nm;                                                                                  \
     } while (0)
 
 template <int KM, bool SMP>
-__global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
-                                                                     int S, int stage_bytes, uint32_t tmem_cols) {
+__global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
+                                                                      int SW, int SZ, uint32_t tmem_cols) {
     const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     extern __shared__ unsigned char dsm_raw[];
     __shared__ WideState st;
-    unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
-    float* tbuf = (float*)(ring + (size_t)S * stage_bytes);  // [128 vocab][kWideTileStride]
+    const uint32_t zbytes = (uint32_t)R_pad * 128u;
+    // [weight ring: SW x 16 KB][z ring: SZ x zbytes][transpose buffers: one per row group]
+    unsigned char* wring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char* zring = wring + (size_t)SW * 16384;
+    float* tbuf = (float*)(zring + (size_t)SZ * zbytes);  // [group][64 vocab][kWideTileStride]
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int R = a.R, k = a.top_k;
     const int nkb = a.d / 64;
@@ -1172,17 +1146,18 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
     const int t0 = (int)(((int64_t)blockIdx.x * ntiles) / gridDim.x);
     const int t1 = (int)(((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x);
     const int ngroups = (R_pad + kWideGroup - 1) / kWideGroup;
-    const uint32_t zbytes = (uint32_t)R_pad * 128u;
 
     if (t == 0) {
-        for (int i = 0; i < S; ++i) {
-            mbar_init(&st.full[i], 1);
-            mbar_init(&st.empty[i], 1);
+        for (int i = 0; i < SW; ++i) {
+            mbar_init(&st.wfull[i], 1);
+            mbar_init(&st.zfull[i], 1);
+            mbar_init(&st.done[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&st.tfull[i], 1);
-            mbar_init(&st.tempty[i], 4);
-            mbar_init(&st.ebar[i], 4);
+            mbar_init(&st.tempty[i], 4 * ngroups);  // every warp of a present row group
+            mbar_init(&st.ebar[i][0], 4);
+            mbar_init(&st.ebar[i][1], 4);
         }
         st.abort = 0;
         mbar_fence_init();
@@ -1194,97 +1169,144 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
     const uint32_t tmem = st.tmem_base;
     griddep_launch_dependents();
 
-    if (warp == 4) {  // ---- TMA producer
+    // Ring positions advance by counters (slot, phase bit), not by division: the producer and
+    // the MMA issuer are single threads whose every instruction is on the stream's critical
+    // path.
+    if (warp == 8) {  // ---- TMA producer
         if (lane == 0) {
-            const int total = (t1 - t0) * nkb;
-            const int pre = min(S, total);
-            for (int it = 0; it < pre; ++it) {
-                mbar_arrive_expect_tx(&st.full[it], 16384u + zbytes);
-                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + ((size_t)t0 * nkb + it) * 16384,
-                         16384, &st.full[it]);
+            const int total = (t1 - t0) * nkb;  // iteration it: weight block t0 * nkb + it, z block it % nkb
+            const unsigned char* Wsrc = (const unsigned char*)a.W + (size_t)t0 * nkb * 16384;
+            const unsigned char* Zsrc = (const unsigned char*)zb;
+            const int prew = min(SW, total), prez = min(SZ, total);
+            // the weights do not depend on earlier kernels: the first stages go out at once
+            for (int it = 0; it < prew; ++it) {
+                mbar_arrive_expect_tx(&st.wfull[it], 16384u);
+                bulk_g2s(wring + (size_t)it * 16384, Wsrc + (size_t)it * 16384, 16384, &st.wfull[it]);
             }
             griddep_wait();
-            for (int it = 0; it < pre; ++it)
-                bulk_g2s(ring + (size_t)it * stage_bytes + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * zbytes,
-                         zbytes, &st.full[it]);
-            for (int it = pre; it < total; ++it) {
-                const int slot = it % S;
-                if (!mbar_wait_abortable(&st.empty[slot], ((uint32_t)(it / S) & 1u) ^ 1u, a.status, &st.abort)) break;
-                unsigned char* dst = ring + (size_t)slot * stage_bytes;
-                mbar_arrive_expect_tx(&st.full[slot], 16384u + zbytes);
-                bulk_g2s(dst, (const unsigned char*)a.W + ((size_t)t0 * nkb + it) * 16384, 16384, &st.full[slot]);
-                bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)(it % nkb) * zbytes, zbytes, &st.full[slot]);
+            int kz = 0;  // z block of the next z copy
+            for (int it = 0; it < prez; ++it) {
+                mbar_arrive_expect_tx(&st.zfull[it], zbytes);
+                bulk_g2s(zring + (size_t)it * zbytes, Zsrc + (size_t)kz * zbytes, zbytes, &st.zfull[it]);
+                if (++kz == nkb) kz = 0;
+            }
+            // once the MMAs of iteration c are done (done[c % SW]), its z slot takes iteration
+            // c + SZ and its weight slot iteration c + SW
+            int cw = 0, cz = 0;  // c % SW, c % SZ
+            uint32_t pd = 0;     // phase bit of done[cw]
+            for (int c = 0; c + SZ < total; ++c) {
+                if (!mbar_wait_abortable(&st.done[cw], pd, a.status, &st.abort)) break;
+                mbar_arrive_expect_tx(&st.zfull[cz], zbytes);
+                bulk_g2s(zring + (size_t)cz * zbytes, Zsrc + (size_t)kz * zbytes, zbytes, &st.zfull[cz]);
+                if (++kz == nkb) kz = 0;
+                if (c + SW < total) {
+                    mbar_arrive_expect_tx(&st.wfull[cw], 16384u);
+                    bulk_g2s(wring + (size_t)cw * 16384, Wsrc + (size_t)(c + SW) * 16384, 16384, &st.wfull[cw]);
+                }
+                if (++cz == SZ) cz = 0;
+                if (++cw == SW) { cw = 0; pd ^= 1u; }
             }
         }
-    } else if (warp == 5) {  // ---- MMA issuer
+    } else if (warp == 9) {  // ---- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, R_pad);
-            int it = 0;
+            int sw = 0, sz = 0;          // it % SW, it % SZ
+            uint32_t pw = 0, pz = 0;     // phase bits of wfull[sw], zfull[sz]
             for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
                 const int buf = j & 1;
                 if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)(buf * R_pad);
                 bool ok = true;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
-                    const int slot = it % S;
-                    if (!mbar_wait_abortable(&st.full[slot], (uint32_t)(it / S) & 1u, a.status, &st.abort)) {
+                for (int kb = 0; kb < nkb; ++kb) {
+                    if (!mbar_wait_abortable(&st.wfull[sw], pw, a.status, &st.abort) ||
+                        !mbar_wait_abortable(&st.zfull[sz], pz, a.status, &st.abort)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = smem_u32(ring + (size_t)slot * stage_bytes);
-                    const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + 16384);
+                    const uint64_t adesc = sw128_desc(smem_u32(wring + (size_t)sw * 16384));
+                    const uint64_t bdesc = sw128_desc(smem_u32(zring + (size_t)sz * zbytes));
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) tc_mma(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, idesc, (kb | kk) != 0);
-                    tc_commit(&st.empty[slot]);
+                    tc_commit(&st.done[sw]);
+                    if (++sw == SW) { sw = 0; pw ^= 1u; }
+                    if (++sz == SZ) { sz = 0; pz ^= 1u; }
                 }
                 if (!ok) break;
                 tc_commit(&st.tfull[buf]);
             }
         }
-    } else {  // ---- epilogue warps 0..3: thread t owns rows t and 128 + t
+    } else if ((warp >> 2) < ngroups) {  // ---- epilogue warps of row group g = warp / 4
+        const int g = warp >> 2, qd = warp & 3;  // row group; TMEM lane quadrant 32 qd .. 32 qd + 31
+        const int r = g * kWideGroup + qd * 32 + lane;  // this thread's hidden row
+        float* tb = tbuf + (size_t)g * kWideHalf * kWideTileStride;
+        const float* col = tb + qd * 32 + lane;  // the row's column of the staged entries
         griddep_wait();
-        WideRow<KM> w0, w1;
-        w0.init();
-        w1.init();
-        uint32_t eb = 0;  // epilogue barriers passed (two mbarriers used alternately)
+        WideRow<KM> w;
+        w.init();
+        uint32_t eb = 0;  // group barriers passed (two mbarriers used alternately)
         auto epi_sync = [&]() -> bool {
             __syncwarp();
-            uint64_t* bar = &st.ebar[eb & 1];
+            uint64_t* bar = &st.ebar[g][eb & 1];
             if (lane == 0) mbar_arrive(bar);
-            const bool r = mbar_wait_abortable(bar, (eb >> 1) & 1u, a.status, &st.abort);
+            const bool ok = mbar_wait_abortable(bar, (eb >> 1) & 1u, a.status, &st.abort);
             ++eb;
-            return r;
+            return ok;
         };
         bool ok = true;
         for (int tile = t0, j = 0; tile < t1 && ok; ++tile, ++j) {
             const int buf = j & 1;
             if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
             tc_fence_after();
-            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * R_pad);
-            FE_WIDE_GROUP(w0, 0);
-            FE_WIDE_GROUP(w1, 1);
+            // the group's 128 columns of this warp's 32 lanes (vocabulary entries)
+            const uint32_t taddr = tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(buf * R_pad + g * kWideGroup);
+            const int ncols = min(kWideGroup, R_pad - g * kWideGroup);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (!ok) break;
+                if ((qd >> 1) == h) {  // stage: entries 64 h + 32 (qd & 1) + lane x the group's rows
+                    float* trow = tb + (size_t)((qd & 1) * 32 + lane) * kWideTileStride;
+                    for (int c0 = 0; c0 < ncols; c0 += 32) {
+                        float v32[32];
+                        tc_ld32(taddr + (uint32_t)c0, v32);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) trow[c0 + i] = v32[i];
+                    }
+                    // this warp's last read of the accumulator: hand it back to the MMA warp
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&st.tempty[buf]);
+                }
+                if (!(ok = epi_sync())) break;
+                if (r < R) {
+                    const int id0 = tile * 128 + h * kWideHalf;
+                    const int nv = min(kWideHalf, a.V - id0);
+                    FE_WIDE_BATCH(0);
+                    FE_WIDE_BATCH(32);
+                    if (a.dbg_logits) {
+                        const int rb = r % a.B, ri = r / a.B;
+                        for (int u = 0; u < nv; ++u)
+                            a.dbg_logits[((size_t)rb * a.N + ri) * a.V + id0 + u] = col[(size_t)u * kWideTileStride];
+                    }
+                }
+                ok = epi_sync();
+            }
         }
-        // ---- the slab's partial of each owned row
-#define FE_WIDE_FINISH(w, g)                                                                           \
-    do {                                                                                               \
-        const int r = (g) * kWideGroup + t;                                                            \
-        if ((g) >= ngroups || !ok || r >= R) break;                                                    \
-        const size_t base = (size_t)r * a.n_slabs + blockIdx.x;                                        \
-        _Pragma("unroll") for (int q = 0; q < KM; ++q) {                                               \
-            if (q < k) {                                                                               \
-                a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];                      \
-                a.part_val[base * k + q] = w.v[q];                                                     \
-                if (SMP) a.part_lg[base * k + q] = w.l[q];                                             \
-            }                                                                                          \
-        }                                                                                              \
-        a.part_ms[base * 2 + 0] = w.m;                                                                 \
-        a.part_ms[base * 2 + 1] = w.s;                                                                 \
-    } while (0)
-        FE_WIDE_FINISH(w0, 0);
-        FE_WIDE_FINISH(w1, 1);
-#undef FE_WIDE_FINISH
+        // ---- the slab's partial of this thread's row
+        if (ok && r < R) {
+            const size_t base = (size_t)r * a.n_slabs + blockIdx.x;
+#pragma unroll
+            for (int q = 0; q < KM; ++q) {
+                if (q < k) {
+                    a.part_id[base * k + q] = w.v[q] == -INFINITY ? INT_MAX : w.i[q];
+                    a.part_val[base * k + q] = w.v[q];
+                    if (SMP) a.part_lg[base * k + q] = w.l[q];
+                }
+            }
+            a.part_ms[base * 2 + 0] = w.m;
+            a.part_ms[base * 2 + 1] = w.s;
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -1292,7 +1314,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_wide_kernel(const LmHea
     if (warp == 0) tc_dealloc(tmem, tmem_cols);
 }
 
-#undef FE_WIDE_GROUP
+#undef FE_WIDE_BATCH
 
 // One CTA per row: merges every slab's partial of that row (merge_rows).
 __global__ void __launch_bounds__(128) lmhead_merge_kernel(const LmHeadArgs a, size_t smem_bytes) {
@@ -1347,19 +1369,24 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
                              (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 0, a.stamp);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
-    const int stage_bytes = 16384 + R_pad * 128;
-    const size_t tbytes = (size_t)128 * kWideTileStride * sizeof(float);
+    // shared memory: the transpose buffers (one per row group), then up to kWideMaxZ z stages
+    // (R_pad x 128 B) and the rest to the weight ring (at least as many stages)
+    const size_t zst = (size_t)R_pad * 128;
+    const size_t tbytes = (size_t)((R_pad + kWideGroup - 1) / kWideGroup) * kWideHalf * kWideTileStride * sizeof(float);
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(WideState) - 256;
-    if (budget < 1024 + tbytes + 2 * (size_t)stage_bytes) return cudaErrorInvalidValue;
-    int S = (int)((budget - 1024 - tbytes) / stage_bytes);
-    S = S > kMmaMaxStages ? kMmaMaxStages : S;
-    const size_t smem = 1024 + (size_t)S * stage_bytes + tbytes;
+    if (budget < 1024 + tbytes + 2 * (16384 + zst)) return cudaErrorInvalidValue;
+    const size_t avail = budget - 1024 - tbytes;
+    int SZ = (int)(avail / (16384 + zst));
+    SZ = SZ > kWideMaxZ ? kWideMaxZ : SZ;
+    int SW = (int)((avail - SZ * zst) / 16384);
+    SW = SW > kWideMaxW ? kWideMaxW : SW;
+    const size_t zring = SZ * zst;
+    const size_t smem = 1024 + (size_t)SW * 16384 + zring + tbytes;
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * R_pad)) cols <<= 1;
     auto kern = a.sample ? (a.top_k <= 8 ? lmhead_wide_kernel<8, true> : lmhead_wide_kernel<16, true>)
                          : (a.top_k <= 8 ? lmhead_wide_kernel<8, false> : lmhead_wide_kernel<16, false>);
-    e = launch_k(kern, dim3(a.n_slabs), dim3(kMmaThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad, S,
-                 stage_bytes, cols);
+    e = launch_k(kern, dim3(a.n_slabs), dim3(kWideThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad, SW, SZ, cols);
     if (e != cudaSuccess) return e;
     if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;
     const size_t msmem = merge_smem_bytes(4, a.n_slabs, a.top_k, a.sample != 0);
