@@ -101,7 +101,14 @@ struct LinearArgs {
         float* y2 = nullptr;
         int ldy2 = 0;
         const float* ybase = nullptr;
+        // the phase normalised its input after the product (norm_post): its per-row RMSNorm
+        // scales, which multiply the summed shares before its epilogue
+        const float* rs = nullptr;
     } prev;
+    // tensor-core path, RMSNorm input: the operand is gamma * x (the prep runs column-parallel
+    // and leaves per-CTA sums of squares) and the per-row scale 1 / sqrt(mean(x^2) + eps)
+    // multiplies the products; otherwise the prep scales the operand itself (a whole-row pass)
+    int norm_post = 0;
 };
 
 struct DeviceInfo {
@@ -137,6 +144,11 @@ size_t linear_mma_xb_bytes(int K, int B);
 size_t linear_mma_part_bytes(int B, const DeviceInfo& dev);
 int linear_mma_grid(int M, int K, const DeviceInfo& dev);
 cudaError_t linear_mma_prepare(const DeviceInfo& dev);
+// the completion-counter buffer: the last norm_post phase's per-row scales and its prep's
+// sums of squares, then 4 * ceil(M_max / 128) ints of split-tile counters; zero at init
+size_t linear_mma_counter_bytes(int M_max, const DeviceInfo& dev);
+// where a norm_post phase leaves its per-row scales (inside the counter buffer)
+float* linear_mma_rs(int* counters);
 // after_prep (optional): an event recorded on st between the two kernels it launches
 cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, int* counters, const DeviceInfo& dev,
                               cudaStream_t st, cudaEvent_t after_prep = nullptr);

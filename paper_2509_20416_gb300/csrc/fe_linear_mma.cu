@@ -51,15 +51,18 @@ __device__ __forceinline__ void split_bf16(float z, uint16_t& hi, uint16_t& lo) 
 }  // namespace
 
 // ---- stream-K partition ---------------------------------------------------------------------
-// first unit of CTA c when U units are split over G CTAs
-__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) { return (int64_t)c * U / G; }
+// first unit of CTA c when U units are split over G CTAs (32-bit division whenever U * G
+// fits, as it does for every drafter shape: a 64-bit division is a long software sequence)
+__device__ __forceinline__ int64_t unit_begin(int c, int64_t U, int G) {
+    if (U * G <= 0xFFFFFFFFll) return (int64_t)((uint32_t)c * (uint32_t)U / (uint32_t)G);
+    return (int64_t)c * U / G;
+}
 
-// the CTA whose range holds unit u
+// the CTA whose range holds unit u: the largest c with floor(c U / G) <= u, i.e. with
+// c U / G < u + 1, which is floor(((u + 1) G - 1) / U)
 __device__ __forceinline__ int unit_owner(int64_t u, int64_t U, int G) {
-    int c = (int)((u * G) / U);
-    while (c + 1 < G && unit_begin(c + 1, U, G) <= u) ++c;
-    while (c > 0 && unit_begin(c, U, G) > u) --c;
-    return c;
+    if (U * G <= 0xFFFFFFFFll) return (int)(((uint32_t)u * (uint32_t)G + (uint32_t)G - 1u) / (uint32_t)U);
+    return (int)(((u + 1) * G - 1) / U);
 }
 
 // ---- activation operand ------------------------------------------------------------------
@@ -102,19 +105,31 @@ __device__ __forceinline__ void prev_finish_t(const LinearArgs::Prev& p, int BP,
         v[0] = q0.x; v[1] = q0.y; v[2] = q0.z; v[3] = q0.w; v[4] = q1.x; v[5] = q1.y; v[6] = q1.z; v[7] = q1.w;
         return;
     }
+    // the residual (EPI_RESID) and the previous phase's RMSNorm scale are loaded before the
+    // shares, so the round trips overlap
+    const float prs = p.rs ? __ldcg(p.rs + b) : 1.f;
+    float4 rb0 = make_float4(0.f, 0.f, 0.f, 0.f), rb1 = rb0;
+    if (!GLU && p.epi == EPI_RESID) {
+        const float* base = p.ybase ? p.ybase + (size_t)b * p.ldy + k0 : y;
+        rb0 = __ldcg(reinterpret_cast<const float4*>(base));
+        rb1 = __ldcg(reinterpret_cast<const float4*>(base) + 1);
+    }
     float sm[NR];
 #pragma unroll
     for (int i = 0; i < NR; ++i) sm[i] = 0.f;
     // the shares in batches of kPrevBatch CTAs: every load of a batch is issued before any
     // is summed (one L2 round trip per batch), the sums still in CTA order
     constexpr int kPrevBatch = GLU ? 4 : 8;  // (register budget: NR floats per share)
+    // a tile is the first of every CTA after c_first that shares it (their shares sit in slot
+    // 0); it is c_first's first tile only if c_first's range starts at the tile's first unit
+    const int cs_first = unit_begin(c_first, U, p.G) < (int64_t)tile * nkb ? 1 : 0;
     for (int c0 = c_first; c0 <= c_last; c0 += kPrevBatch) {
         float x[kPrevBatch][NR];
 #pragma unroll
         for (int j = 0; j < kPrevBatch; ++j) {
             const int c = c0 + j;
             if (c > c_last) break;
-            const int cs = (int)(unit_begin(c, U, p.G) / nkb) == tile ? 0 : 1;
+            const int cs = c == c_first ? cs_first : 0;
             const float4* q = reinterpret_cast<const float4*>(p.part + ((size_t)(c * 2 + cs) * BP + b) * 128 + r0);
 #pragma unroll
             for (int i = 0; i < NR / 4; ++i) {
@@ -129,13 +144,15 @@ __device__ __forceinline__ void prev_finish_t(const LinearArgs::Prev& p, int BP,
             for (int i = 0; i < NR; ++i) sm[i] += x[j][i];
         }
     }
+    if (p.rs) {
+#pragma unroll
+        for (int i = 0; i < NR; ++i) sm[i] *= prs;
+    }
     if constexpr (GLU) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = silu(sm[2 * e]) * sm[2 * e + 1];
     } else if (p.epi == EPI_RESID) {
-        const float* base = p.ybase ? p.ybase + (size_t)b * p.ldy + k0 : y;
-        const float4 b0 = __ldcg(reinterpret_cast<const float4*>(base)), b1 = __ldcg(reinterpret_cast<const float4*>(base) + 1);
-        const float r[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+        const float r[8] = {rb0.x, rb0.y, rb0.z, rb0.w, rb1.x, rb1.y, rb1.z, rb1.w};
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = r[e] + sm[e];
         if (p.y2) {
@@ -172,15 +189,31 @@ __device__ __forceinline__ void put_operand(uint16_t* xb, int N, int B_pad, int 
     *reinterpret_cast<uint4*>(blk + sw128_offset(B_pad + b, c % 8)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
 }
 
-__global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb) {
+__global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pad, uint16_t* xb, float* sq) {
     const LaunchStamp stamp(a.stamp);
     const int b = blockIdx.x, t = threadIdx.x;
     const int N = 2 * B_pad, K = a.K, nc = K / 8;
+    const int c = blockIdx.y * kXprepChunks + t;  // this thread's 16-byte chunk of row b
+    const int k0 = 8 * c;
     __shared__ float red[8];
     griddep_launch_dependents();
+    // weights do not depend on the previous kernel: the RMSNorm gains are loaded, and the
+    // embedding row's line is prefetched into L2 (from a token id read early: a stale id
+    // only warms a wrong line), before the wait
+    uint4 gq = make_uint4(0, 0, 0, 0);
+    if (b < a.B && c < nc) {
+        if (a.pro == PRO_RMSNORM) gq = *reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + k0);
+        if (a.pro == PRO_CONCAT_EMB && k0 >= a.d_split) {
+            const int tk = a.tok[b];
+            if (tk >= 0 && tk < a.vocab)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"((const bf16_t*)a.embed + (size_t)tk * (K - a.d_split) +
+                                                               (k0 - a.d_split)));
+        }
+    }
     griddep_wait();
     const bool live = b < a.B;
-    const bool fin = live && a.prev.active;  // (RMSNorm inputs take xprep_row_kernel instead)
+    const bool fin = live && a.prev.active;  // (without norm_post, RMSNorm inputs take xprep_row_kernel)
+    const bool post = a.norm_post && a.pro == PRO_RMSNORM;  // the scale goes on the products
     int tok = 0;
     if (live && a.pro == PRO_CONCAT_EMB) {
         tok = a.tok[b];
@@ -190,59 +223,61 @@ __global__ void __launch_bounds__(256) xprep_kernel(const LinearArgs a, int B_pa
         }
     }
     const float* xf = (const float*)a.x + (size_t)b * a.ldx;
-    // 1 / sqrt(mean of squares + eps) from each thread's partial sum (CTA-wide)
-    auto rs_of = [&](float ss) {
+    // the CTA's sum of per-thread partials in a fixed order
+    auto cta_sum = [&](float ss) {
         ss = warp_sum(ss);
         if ((t & 31) == 0) red[t >> 5] = ss;
         __syncthreads();
         float tot = 0.f;
 #pragma unroll
         for (int w = 0; w < 8; ++w) tot += red[w];
-        return 1.0f / sqrtf(tot / (float)K + a.eps);
+        return tot;
     };
     float rs = 1.f;
-    if (live && a.pro == PRO_RMSNORM) {
+    if (live && a.pro == PRO_RMSNORM && !post) {  // 1 / sqrt(mean of squares + eps) over the whole row
         float ss = 0.f;
 #pragma unroll 4
-        for (int c = t; c < nc; c += 256) {
-            const float4 p = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c);
-            const float4 q = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * c + 1);
+        for (int cc = t; cc < nc; cc += 256) {
+            const float4 p = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * cc);
+            const float4 q = __ldcg(reinterpret_cast<const float4*>(xf) + 2 * cc + 1);
             const float v[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
             ss += sumsq8(v);
         }
-        rs = rs_of(ss);
+        rs = 1.0f / sqrtf(cta_sum(ss) / (float)K + a.eps);
     }
-    {
-        const int c = blockIdx.y * kXprepChunks + t;
-        if (c >= nc) return;
-        float v[8];
+    float v[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = 0.f;
-        if (live) {
-            const int k0 = 8 * c;
-            if (a.pro == PRO_STORAGE) {
-                Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.x + (size_t)b * a.ldx + k0), v);
-            } else if (a.pro == PRO_CONCAT_EMB && k0 >= a.d_split) {
-                if (tok >= 0)
-                    Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.embed +
-                                                                         (size_t)tok * (K - a.d_split) + (k0 - a.d_split)),
-                                         v);
-            } else if (fin) {  // the previous phase's output, its split tiles finished here
-                prev_finish(a.prev, B_pad, b, k0, v);
-            } else {  // float32 input (PRO_F32, PRO_RMSNORM, or the float part of PRO_CONCAT_EMB)
-                const float4 p = __ldcg(reinterpret_cast<const float4*>(xf + k0));
-                const float4 q = __ldcg(reinterpret_cast<const float4*>(xf + k0) + 1);
-                v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
-                if (a.pro == PRO_RMSNORM) {
-                    float g[8];
-                    Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + k0), g);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) v[e] = v[e] * rs * g[e];
-                }
-            }
+    for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    if (live && c < nc) {
+        if (a.pro == PRO_STORAGE) {
+            Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.x + (size_t)b * a.ldx + k0), v);
+        } else if (a.pro == PRO_CONCAT_EMB && k0 >= a.d_split) {
+            if (tok >= 0)
+                Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.embed +
+                                                                     (size_t)tok * (K - a.d_split) + (k0 - a.d_split)),
+                                     v);
+        } else if (fin) {  // the previous phase's output, its split tiles finished here
+            prev_finish(a.prev, B_pad, b, k0, v);
+        } else {  // float32 input (PRO_F32, PRO_RMSNORM, or the float part of PRO_CONCAT_EMB)
+            const float4 p = __ldcg(reinterpret_cast<const float4*>(xf + k0));
+            const float4 q = __ldcg(reinterpret_cast<const float4*>(xf + k0) + 1);
+            v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
         }
-        put_operand(xb, N, B_pad, b, c, v);
     }
+    if (a.pro == PRO_RMSNORM) {
+        float g[8];
+        Vec16<bf16_t>::widen(gq, g);
+        if (post) {  // gamma * x here; this CTA's sum of squares of x for the product kernel
+            const float tot = cta_sum(sumsq8(v));
+            if (t == 0) sq[blockIdx.y * B_pad + b] = tot;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] *= g[e];
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = v[e] * rs * g[e];
+        }
+    }
+    if (c < nc) put_operand(xb, N, B_pad, b, c, v);
 }
 
 // The deferred-input prep of an RMSNorm phase: one CTA of kRowThreads per row b finishes the
@@ -258,6 +293,16 @@ __global__ void __launch_bounds__(kRowThreads) xprep_row_kernel(const LinearArgs
     const int N = 2 * B_pad, K = a.K, nc = K / 8;
     __shared__ float red[kRowThreads / 32];
     griddep_launch_dependents();
+    // the RMSNorm gains of this thread's first kPreChunks chunks (weights: loaded before the
+    // wait; d <= 8192 needs no more)
+    constexpr int kRowChunks = kXprepRowSmem / sizeof(float) / 8 / kRowThreads;
+    constexpr int kPreChunks = 2;
+    uint4 gq[kPreChunks];
+#pragma unroll
+    for (int j = 0; j < kPreChunks; ++j) {
+        const int c = t + j * kRowThreads;
+        gq[j] = b < a.B && c < nc ? *reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + 8 * c) : make_uint4(0, 0, 0, 0);
+    }
     griddep_wait();
     if (b >= a.B) {  // a padding row of the operand is zero
         const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -279,17 +324,31 @@ __global__ void __launch_bounds__(kRowThreads) xprep_row_kernel(const LinearArgs
 #pragma unroll
     for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
     const float rs = 1.0f / sqrtf(tot / (float)K + a.eps);
-    for (int c = t; c < nc; c += kRowThreads) {
+#pragma unroll
+    for (int j = 0; j < kRowChunks; ++j) {
+        const int c = t + j * kRowThreads;
+        if (c >= nc) break;
         float v[8], g[8];
         const float4 p = reinterpret_cast<const float4*>(xrow)[2 * c];
         const float4 q = reinterpret_cast<const float4*>(xrow)[2 * c + 1];
         v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
-        Vec16<bf16_t>::widen(*reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + 8 * c), g);
+        Vec16<bf16_t>::widen(j < kPreChunks ? gq[j < kPreChunks ? j : 0]
+                                            : *reinterpret_cast<const uint4*>((const bf16_t*)a.gamma + 8 * c),
+                             g);
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[e] = v[e] * rs * g[e];
         put_operand(xb, N, B_pad, b, c, v);
     }
 }
+
+// ---- the RMSNorm scale after the product (LinearArgs::norm_post) ---------------------------
+// The operand prep of an RMSNorm phase writes gamma * x and, per CTA (row b, column range
+// y), the sum of squares of x over its columns in sq[y * B_pad + b]; the product kernel sums
+// them (fixed order) to 1 / sqrt(mean(x^2) + eps) and multiplies its products by it. So
+// the prep needs no whole-row pass and runs column-parallel like any other.
+constexpr int kAuxRs = 0;      // bytes into the counter buffer: the last normalised phase's scales
+constexpr int kAuxSq = 256;    // the prep's sums of squares [ny][kLinMmaMaxBatch]
+constexpr int kAuxEnd = 1280;  // (ny <= 8: K <= 16384)
 
 // ---- the product ---------------------------------------------------------------------------
 // Epilogue for output row m of all B sequences; v[b] is the finished dot product.
@@ -332,13 +391,14 @@ __device__ __forceinline__ void lin_epilogue(const LinearArgs& a, int m, const f
 }
 
 template <int BP>  // B_pad: 8, 16, 24 or 32
-__global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearArgs a, const uint16_t* xb, int S,
+__global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearArgs a, uint16_t* xb, int S,
                                                                    int stage_bytes, uint32_t tmem_cols, float* part,
-                                                                   int* counters) {
+                                                                   int* counters, unsigned char* aux) {
     const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     constexpr int N = 2 * BP;
     extern __shared__ unsigned char dsm_raw[];
     __shared__ LinMmaState st;
+    __shared__ float rs_s[BP];  // norm_post: the rows' RMSNorm scales
     unsigned char* ring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int G = gridDim.x, cta = blockIdx.x;
@@ -434,7 +494,33 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             }
         }
     } else {  // ---- epilogue warps 0..3: TMEM lane 32 w + l = output row of the tile
+        float rsv[BP];  // per-row factor of the products (norm_post: the RMSNorm scales, else 1)
+#pragma unroll
+        for (int b = 0; b < BP; ++b) rsv[b] = 1.f;
         griddep_wait();  // the epilogue reads and writes activations of earlier kernels
+        if (a.norm_post && a.pro == PRO_RMSNORM) {  // the rows' scales from the prep's sums of squares
+            const float* sq = (const float*)(aux + kAuxSq);
+            const int ny = (a.K / 8 + kXprepChunks - 1) / kXprepChunks;
+            // row b = t / 4 sums column ranges y = t % 4, t % 4 + 4 (loads first, then in
+            // order), then the four lanes combine in a fixed pattern
+            const int b = t >> 2, p0 = t & 3;
+            float q0 = 0.f, q1 = 0.f;
+            if (b < BP) {
+                if (p0 < ny) q0 = __ldcg(sq + (size_t)p0 * BP + b);
+                if (p0 + 4 < ny) q1 = __ldcg(sq + (size_t)(p0 + 4) * BP + b);
+            }
+            float acc4 = q0 + q1;
+            acc4 += __shfl_xor_sync(0xffffffffu, acc4, 1);
+            acc4 += __shfl_xor_sync(0xffffffffu, acc4, 2);
+            if (b < BP && p0 == 0) rs_s[b] = 1.0f / sqrtf(acc4 / (float)a.K + a.eps);
+            named_sync(1, 128);  // (the four epilogue warps)
+#pragma unroll
+            for (int bb = 0; bb < BP; ++bb) rsv[bb] = rs_s[bb];
+            // a deferred split tile of this phase is finished by the next phase's prep, which
+            // reads these (the previous phase's scales were read by this phase's prep,
+            // complete before this kernel's griddep_wait returned)
+            if (cta == 0 && t < BP) ((float*)(aux + kAuxRs))[t] = rs_s[t];
+        }
         const int r = warp * 32 + lane;
         for (int tile = tile0, j = 0; tile <= tile1; ++tile, ++j) {
             const int buf = j & 1;
@@ -447,13 +533,15 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&st.tempty[buf]);
-            float v[BP];
+            float v[BP];  // this CTA's products (a split tile's share stays unscaled)
 #pragma unroll
             for (int b = 0; b < BP; ++b) v[b] = acc[b] + acc[BP + b];
             const int m = tile * 128 + r;
             const int c_first = unit_owner((int64_t)tile * nkb, U, G);
             const int c_last = unit_owner((int64_t)(tile + 1) * nkb - 1, U, G);
             if (c_first == c_last) {  // the whole tile was ours
+#pragma unroll
+                for (int b = 0; b < BP; ++b) v[b] *= rsv[b];
                 lin_epilogue<BP>(a, m, v);
                 continue;
             }
@@ -475,8 +563,10 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             float s[BP];
 #pragma unroll
             for (int b = 0; b < BP; ++b) s[b] = 0.f;
+            // (slot 1 only for c_first, when the tile is not its first: see prev_finish_t)
+            const int cs_first = unit_begin(c_first, U, G) < (int64_t)tile * nkb ? 1 : 0;
             for (int c = c_first; c <= c_last; ++c) {
-                const int cs = (int)(unit_begin(c, U, G) / nkb) == tile ? 0 : 1;
+                const int cs = c == c_first ? cs_first : 0;
                 const float* q = part + ((size_t)(c * 2 + cs) * BP) * 128 + r;
                 float x[BP];
 #pragma unroll
@@ -484,6 +574,8 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
 #pragma unroll
                 for (int b = 0; b < BP; ++b) s[b] += x[b];
             }
+#pragma unroll
+            for (int b = 0; b < BP; ++b) s[b] *= rsv[b];
             lin_epilogue<BP>(a, m, s);
             if (lane == 0) counters[tile * 4 + warp] = 0;
         }
@@ -504,8 +596,8 @@ cudaError_t set_attr(const DeviceInfo& dev) {
 }
 
 template <int BP>
-cudaError_t launch_bp(const LinearArgs& a, const uint16_t* xb, float* part, int* counters, const DeviceInfo& dev,
-                      cudaStream_t st, int grid) {
+cudaError_t launch_bp(const LinearArgs& a, uint16_t* xb, float* part, int* counters, unsigned char* aux,
+                      const DeviceInfo& dev, cudaStream_t st, int grid) {
     constexpr int N = 2 * BP;
     const int stage_bytes = 16384 + N * 128;
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(LinMmaState) - 256 - 1024;
@@ -516,7 +608,7 @@ cudaError_t launch_bp(const LinearArgs& a, const uint16_t* xb, float* part, int*
     uint32_t cols = 32;
     while (cols < (uint32_t)(2 * N)) cols <<= 1;
     return launch_k(linear_mma_kernel<BP>, dim3(grid), dim3(kLmThreads), smem, st, a.pdl, a, xb, S, stage_bytes, cols,
-                    part, counters);
+                    part, counters, aux);
 }
 
 }  // namespace
@@ -536,6 +628,17 @@ size_t linear_mma_part_bytes(int B, const DeviceInfo& dev) {
     return (size_t)dev.num_sms * 2 * linear_mma_bpad(B) * 128 * sizeof(float);
 }
 
+namespace {
+// the split-tile counters' offset in the counter buffer (after the RMSNorm scales and sums)
+size_t tile_counter_offset(const DeviceInfo&) { return kAuxEnd; }
+}  // namespace
+
+size_t linear_mma_counter_bytes(int M_max, const DeviceInfo& dev) {
+    return tile_counter_offset(dev) + 4 * (size_t)((M_max + 127) / 128) * sizeof(int);
+}
+
+float* linear_mma_rs(int* counters) { return (float*)((unsigned char*)counters + kAuxRs); }
+
 cudaError_t linear_mma_prepare(const DeviceInfo& dev) {
     cudaError_t e = cudaFuncSetAttribute(xprep_row_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kXprepRowSmem);
@@ -550,20 +653,26 @@ cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, in
                               cudaStream_t st, cudaEvent_t after_prep) {
     if (!linear_mma_ok(a.M, a.K, a.B)) return cudaErrorInvalidValue;
     const int BP = linear_mma_bpad(a.B);
-    const bool row_cta = a.prev.active && a.pro == PRO_RMSNORM;  // finish + normalise a row per CTA
+    unsigned char* aux = (unsigned char*)counters;
+    int* tctr = (int*)(aux + tile_counter_offset(dev));
+    const int grid = linear_mma_grid(a.M, a.K, dev);
+    // finish + normalise a row per CTA (only when the scale goes on the operand)
+    const bool row_cta = !a.norm_post && a.prev.active && a.pro == PRO_RMSNORM;
     if (row_cta && ((size_t)a.K * sizeof(float) > kXprepRowSmem || a.prev.epi == EPI_SWIGLU)) return cudaErrorInvalidValue;
     const int ny = (a.K / 8 + kXprepChunks - 1) / kXprepChunks;
+    if (a.norm_post && a.pro == PRO_RMSNORM && (size_t)ny * kLinMmaMaxBatch * sizeof(float) > kAuxEnd - kAuxSq)
+        return cudaErrorInvalidValue;
     cudaError_t e = row_cta ? launch_k(xprep_row_kernel, dim3(BP), dim3(kRowThreads), (size_t)a.K * sizeof(float), st,
                                        a.pdl, a, BP, xb)
-                            : launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb);
+                            : launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb,
+                                       (float*)(aux + kAuxSq));
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
-    const int grid = linear_mma_grid(a.M, a.K, dev);
     switch (BP) {
-        case 8: return launch_bp<8>(a, xb, part, counters, dev, st, grid);
-        case 16: return launch_bp<16>(a, xb, part, counters, dev, st, grid);
-        case 24: return launch_bp<24>(a, xb, part, counters, dev, st, grid);
-        default: return launch_bp<32>(a, xb, part, counters, dev, st, grid);
+        case 8: return launch_bp<8>(a, xb, part, tctr, aux, dev, st, grid);
+        case 16: return launch_bp<16>(a, xb, part, tctr, aux, dev, st, grid);
+        case 24: return launch_bp<24>(a, xb, part, tctr, aux, dev, st, grid);
+        default: return launch_bp<32>(a, xb, part, tctr, aux, dev, st, grid);
     }
 }
 

@@ -123,6 +123,7 @@ struct fe_handle {
     bool lm_mma = false;      // LM head packed for (and run on) the tensor cores
     bool lin_mma = false;     // linear phases packed for (and run on) the tensor cores
     bool lin_defer = true;    // tensor-core phases leave split tiles to the next phase's prep
+    bool lin_normpost = true; // tensor-core RMSNorm phases: the scale on the products (column-parallel prep)
     uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
     float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
     int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
@@ -309,6 +310,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
             }
             L.prev = pending;
             pending = LinearArgs::Prev{};
+            L.norm_post = h->lin_normpost ? 1 : 0;
             L.defer = h->lin_defer && L.next_W && next_in == L.y ? 1 : 0;
             if (L.defer) {
                 pending.active = 1;
@@ -322,6 +324,7 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
                 pending.y2 = L.y2;
                 pending.ldy2 = L.ldy2;
                 pending.ybase = L.ybase;
+                pending.rs = L.norm_post && L.pro == PRO_RMSNORM ? linear_mma_rs(h->lin_counters) : nullptr;
             }
         }
         if (stacked) {
@@ -688,6 +691,11 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             const int kmax = std::max({3 * c.d, c.ffn, c.n_heads * c.head_dim});
             const char* df = getenv("FE_DRAFT_LIN_DEFER");
             h->lin_defer = !(df && df[0] == '0');
+            // FE_DRAFT_LIN_NORMPOST=0: an RMSNorm phase's prep scales the operand itself (one
+            // CTA per row when it also finishes the previous phase's split tiles; kept for
+            // comparison)
+            const char* np = getenv("FE_DRAFT_LIN_NORMPOST");
+            h->lin_normpost = !(np && np[0] == '0');
             const char* sk = getenv("FE_DRAFT_STACK");
             h->use_stack = !h->lin_mma && sk && sk[0] == '1' && stack_slots(kmax, h->dev) >= 1;
         }
@@ -823,7 +831,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
                                  lmhead_wide_zb_bytes((int)R, c.d)) : 0,  // tensor-core LM-head operand
             h->lin_mma ? linear_mma_xb_bytes((int)kmax, std::max(c.max_batch, Rmma)) : 0,  // tensor-core linear operand
             h->lin_mma ? linear_mma_part_bytes(std::max(c.max_batch, Rmma), h->dev) : 0,   // its split-tile partials
-            h->lin_mma ? 4 * ((mmax + 127) / 128) * sizeof(int) : 0,      // its completion counters
+            h->lin_mma ? linear_mma_counter_bytes((int)mmax, h->dev) : 0,   // its counters and fused-prep sums
             h->use_stack ? (size_t)(c.n_layers + 1) * sizeof(uint32_t) : 0,  // stack barrier counters
             Rw * d * 4,                                                       // x0
             Rw * 3 * d * h->es,                                               // commit: gathered features

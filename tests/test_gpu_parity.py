@@ -231,3 +231,21 @@ def test_deferred_split_tiles_bit_identical(monkeypatch, case):
         assert np.array_equal(a[key], b[key]), key
     for i in range(cfg["n_layers"]):
         assert torch.equal(a["k_cache"][i], b["k_cache"][i]) and torch.equal(a["v_cache"][i], b["v_cache"][i]), i
+
+
+@pytest.mark.parametrize("case", ["tc_linear_b12_ragged", "parallel_tc_b12"])
+def test_norm_on_operand_matches_oracle(orc, monkeypatch, case):
+    """The tensor-core RMSNorm phases with the scale applied to the operand by their prep
+    (FE_DRAFT_LIN_NORMPOST=0) instead of to the products, against the oracle, and against
+    the default draft within float32 rounding of the two orders of that scale."""
+    spec = dict(SMALL[case])
+    cfg = wl.make_config(spec.pop("name"), **spec)
+    W, I, ks, vs = _problem(cfg)
+    a = H.run_gpu(cfg, W, I, ks, vs)
+    monkeypatch.setenv("FE_DRAFT_LIN_NORMPOST", "0")
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert a["status"] == 0 and g["status"] == 0
+    for b in range(cfg["B"]):
+        H.compare(orc, cfg, g, H.run_oracle(orc, cfg, W, I, ks, vs, b), b)
+    scale = np.abs(g["hidden"]).max()
+    assert np.abs(a["hidden"] - g["hidden"]).max() <= 1e-5 * scale
