@@ -173,14 +173,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
                 const CT* kr = prow((CT*)a.kc, p);
                 const CT* vr = prow((CT*)a.vc, p);
                 if (kr && vr) {
-                    bulk_g2s(kd + (size_t)(p - c0) * ROWB, kr, n * ROWB, &bar[slot]);
-                    bulk_g2s(vd + (size_t)(p - c0) * ROWB, vr, n * ROWB, &bar[slot]);
+                    bulk_g2s_hint(kd + (size_t)(p - c0) * ROWB, kr, n * ROWB, &bar[slot], l2_evict_first());
+                    bulk_g2s_hint(vd + (size_t)(p - c0) * ROWB, vr, n * ROWB, &bar[slot], l2_evict_first());
                 }
                 p += n;
             }
         } else if (rows > 0) {
-            bulk_g2s(kd, cache_row<CT>((CT*)a.kc, a, b, g, c0, HD), rows * ROWB, &bar[slot]);
-            bulk_g2s(vd, cache_row<CT>((CT*)a.vc, a, b, g, c0, HD), rows * ROWB, &bar[slot]);
+            bulk_g2s_hint(kd, cache_row<CT>((CT*)a.kc, a, b, g, c0, HD), rows * ROWB, &bar[slot], l2_evict_first());
+            bulk_g2s_hint(vd, cache_row<CT>((CT*)a.vc, a, b, g, c0, HD), rows * ROWB, &bar[slot], l2_evict_first());
         }
         return bad;
     };
@@ -518,8 +518,11 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4],
 }
 
 // 16 bytes global -> shared, bypassing L1; src_bytes = 0 writes 16 zero bytes instead
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+// with an L2 cache policy (the cached prefix is read once per draft: l2_evict_first())
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes, uint64_t pol) {
+    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(dst), "l"(src), "r"(src_bytes),
+                 "l"(pol)
+                 : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
@@ -617,6 +620,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     uint32_t xo[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) xo[k] = (uint32_t)(hrow * 256 + ((cchunk ^ ((2 * k + hrow) & 7)) << 4));
+    const uint64_t kvpol = l2_evict_first();
     auto copy_half = [&](unsigned char* dst, const void* cache, uint32_t ri, uint32_t live) {
         const uint32_t d0 = smem_u32(dst);
         const unsigned char* src0 = (const unsigned char*)cache + cchunk * 16;
@@ -624,7 +628,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const uint32_t rr = __shfl_sync(0xffffffffu, ri, 2 * i + hrow);
-            cp_async16(d0 + 2 * i * 256 + xo[i & 3], src0 + (size_t)rr * 256, (lh >> (2 * i)) & 1u ? 16u : 0u);
+            cp_async16(d0 + 2 * i * 256 + xo[i & 3], src0 + (size_t)rr * 256, (lh >> (2 * i)) & 1u ? 16u : 0u, kvpol);
         }
         cp_async_commit();
     };

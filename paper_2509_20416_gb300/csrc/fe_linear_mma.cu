@@ -436,10 +436,11 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
             const int pre = min(S, total);
             const uint32_t xbytes = (uint32_t)N * 128u;
             const unsigned char* Wsrc = (const unsigned char*)a.W + (size_t)u0 * 16384;
+            const uint64_t wpol = l2_evict_first();  // weights are read once per draft
             // the weights do not depend on earlier kernels: the first stages go out at once
             for (int it = 0; it < pre; ++it) {
                 mbar_arrive_expect_tx(&st.full[it], 16384u + xbytes);
-                bulk_g2s(ring + (size_t)it * stage_bytes, Wsrc + (size_t)it * 16384, 16384, &st.full[it]);
+                bulk_g2s_hint(ring + (size_t)it * stage_bytes, Wsrc + (size_t)it * 16384, 16384, &st.full[it], wpol);
             }
             griddep_wait();
             int kx = (int)(u0 % nkb);  // activation block of the next copy: (u0 + it) % nkb
@@ -456,7 +457,7 @@ __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearA
                 if (!mbar_wait_abortable(&st.empty[slot], pe, a.status, &st.abort)) break;
                 unsigned char* dst = ring + (size_t)slot * stage_bytes;
                 mbar_arrive_expect_tx(&st.full[slot], 16384u + xbytes);
-                bulk_g2s(dst, Wsrc + (size_t)it * 16384, 16384, &st.full[slot]);
+                bulk_g2s_hint(dst, Wsrc + (size_t)it * 16384, 16384, &st.full[slot], wpol);
                 bulk_g2s(dst + 16384, (const unsigned char*)xb + (size_t)kx * xbytes, xbytes, &st.full[slot]);
                 if (++kx == nkb) kx = 0;
                 if (++slot == S) { slot = 0; pe ^= 1u; }

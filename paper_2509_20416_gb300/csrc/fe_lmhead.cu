@@ -677,10 +677,11 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
             // unit u's weight block sits at u * 16 KB (tile-major packing)
             const int total = (int)(u1 - u0);
             const int pre = min(S, total);
+            const uint64_t wpol = l2_evict_first();  // the LM head is read once per draft
             for (int it = 0; it < pre; ++it) {
                 mbar_arrive_expect_tx(&st.full[it], 16384u + (uint32_t)N * 128u);
-                bulk_g2s(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384,
-                         &st.full[it]);
+                bulk_g2s_hint(ring + (size_t)it * stage_bytes, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384,
+                              16384, &st.full[it], wpol);
             }
             griddep_wait();
             // ring positions advance by counters, not by division (a single thread on the
@@ -699,7 +700,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) lmhead_mma_kernel(const LmHead
                 if (!mbar_wait_abortable(&st.empty[slot], pe, a.status, &st.abort)) break;
                 unsigned char* dst = ring + (size_t)slot * stage_bytes;
                 mbar_arrive_expect_tx(&st.full[slot], 16384u + (uint32_t)N * 128u);
-                bulk_g2s(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot]);
+                bulk_g2s_hint(dst, (const unsigned char*)a.W + (size_t)(u0 + it) * 16384, 16384, &st.full[slot], wpol);
                 bulk_g2s(dst + 16384, (const unsigned char*)zb + (size_t)kb * N * 128, (uint32_t)N * 128,
                          &st.full[slot]);
                 if (++kb == nkb) kb = 0;
@@ -1178,10 +1179,11 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
             const unsigned char* Wsrc = (const unsigned char*)a.W + (size_t)t0 * nkb * 16384;
             const unsigned char* Zsrc = (const unsigned char*)zb;
             const int prew = min(SW, total), prez = min(SZ, total);
+            const uint64_t wpol = l2_evict_first();  // the LM head is read once per draft
             // the weights do not depend on earlier kernels: the first stages go out at once
             for (int it = 0; it < prew; ++it) {
                 mbar_arrive_expect_tx(&st.wfull[it], 16384u);
-                bulk_g2s(wring + (size_t)it * 16384, Wsrc + (size_t)it * 16384, 16384, &st.wfull[it]);
+                bulk_g2s_hint(wring + (size_t)it * 16384, Wsrc + (size_t)it * 16384, 16384, &st.wfull[it], wpol);
             }
             griddep_wait();
             int kz = 0;  // z block of the next z copy
@@ -1201,7 +1203,7 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
                 if (++kz == nkb) kz = 0;
                 if (c + SW < total) {
                     mbar_arrive_expect_tx(&st.wfull[cw], 16384u);
-                    bulk_g2s(wring + (size_t)cw * 16384, Wsrc + (size_t)(c + SW) * 16384, 16384, &st.wfull[cw]);
+                    bulk_g2s_hint(wring + (size_t)cw * 16384, Wsrc + (size_t)(c + SW) * 16384, 16384, &st.wfull[cw], wpol);
                 }
                 if (++cz == SZ) cz = 0;
                 if (++cw == SW) { cw = 0; pd ^= 1u; }

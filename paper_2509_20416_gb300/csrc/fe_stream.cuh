@@ -191,7 +191,9 @@ __device__ __forceinline__ void stream_issue(const unsigned char* Wt, int K, int
     const int g = g0 + i / nks, ks = i % nks;
     const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
     mbar_arrive_expect_tx(&full[slot], bytes);
-    bulk_g2s(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot]);
+    // weights are read once per draft: evict first, keeping L2 for the activations
+    bulk_g2s_hint(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot],
+                  l2_evict_first());
 }
 
 // First half of a stream: initialise the per-warp barriers and issue every warp's first D
