@@ -997,7 +997,7 @@ constexpr int kWideGroup = 128;   // rows of a row group (one per thread of its 
 constexpr int kWideHalf = 64;     // vocabulary entries staged per transpose round (half a tile)
 constexpr int kWideTileStride = kWideGroup + 1;  // floats per staged vocabulary entry (no bank conflicts)
 constexpr int kWideMaxW = 12;     // weight-ring stages (16 KB each)
-constexpr int kWideMaxZ = 4;      // z-ring stages at most (R_pad x 128 B each)
+constexpr int kWideMaxZ = 3;      // z-ring stages at most (R_pad x 128 B each)
 constexpr int kWideThreads = 10 * 32;  // 8 epilogue warps, 1 producer warp, 1 MMA warp
 
 struct WideState {
