@@ -982,9 +982,10 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
 //     MMAs of tile j + 1.
 //   - Eight epilogue warps, one hidden row per thread: warps 4 g .. 4 g + 3 own rows
 //     128 g .. 128 g + 127. A tile's accumulator has the vocabulary entries as TMEM lanes
-//     and the rows as columns, so each row group transposes it through shared memory in two
-//     rounds of 64 entries x 128 rows (the two warps whose lanes hold those entries copy
-//     them). A thread then reads its row's logits in batches of 32 held in registers: the
+//     and the rows as columns, so each row group transposes it through shared memory in
+//     rounds of kWideRound entries x 128 rows (the warps whose lanes hold those entries copy
+//     them; a small round leaves shared memory to the weight ring). A thread then reads its
+//     row's logits in batches of 32 held in registers: the
 //     batch max, a mask of the entries that reach the running top-k list's k-th value (only
 //     those run through the list's insertion network), the sum of exp against the batch
 //     max (base 2, on the hardware's 2^x) and one rescale of the running (max, sum). The
@@ -994,7 +995,8 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
 constexpr int kWideKMax = 16;     // top_k limit of this kernel (a sorted list in registers)
 constexpr int kWideRowsMax = 256;
 constexpr int kWideGroup = 128;   // rows of a row group (one per thread of its four warps)
-constexpr int kWideHalf = 64;     // vocabulary entries staged per transpose round (half a tile)
+constexpr int kWideRound = 32;    // vocabulary entries staged per transpose round (a quarter of a tile)
+constexpr int kWideRoundWarps = kWideRound / 32;  // the warps that stage one round
 constexpr int kWideTileStride = kWideGroup + 1;  // floats per staged vocabulary entry (no bank conflicts)
 constexpr int kWideMaxW = 12;     // weight-ring stages (16 KB each)
 constexpr int kWideMaxZ = 3;      // z-ring stages at most (R_pad x 128 B each)
@@ -1242,7 +1244,7 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
     } else if ((warp >> 2) < ngroups) {  // ---- epilogue warps of row group g = warp / 4
         const int g = warp >> 2, qd = warp & 3;  // row group; TMEM lane quadrant 32 qd .. 32 qd + 31
         const int r = g * kWideGroup + qd * 32 + lane;  // this thread's hidden row
-        float* tb = tbuf + (size_t)g * kWideHalf * kWideTileStride;
+        float* tb = tbuf + (size_t)g * kWideRound * kWideTileStride;
         const float* col = tb + qd * 32 + lane;  // the row's column of the staged entries
         griddep_wait();
         WideRow<KM> w;
@@ -1265,10 +1267,10 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
             const uint32_t taddr = tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(buf * R_pad + g * kWideGroup);
             const int ncols = min(kWideGroup, R_pad - g * kWideGroup);
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < 128 / kWideRound; ++h) {
                 if (!ok) break;
-                if ((qd >> 1) == h) {  // stage: entries 64 h + 32 (qd & 1) + lane x the group's rows
-                    float* trow = tb + (size_t)((qd & 1) * 32 + lane) * kWideTileStride;
+                if (qd / kWideRoundWarps == h) {  // stage: this warp's 32 entries x the group's rows
+                    float* trow = tb + (size_t)((qd % kWideRoundWarps) * 32 + lane) * kWideTileStride;
                     for (int c0 = 0; c0 < ncols; c0 += 32) {
                         float v32[32];
                         tc_ld32(taddr + (uint32_t)c0, v32);
@@ -1282,10 +1284,10 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
                 }
                 if (!(ok = epi_sync())) break;
                 if (r < R) {
-                    const int id0 = tile * 128 + h * kWideHalf;
-                    const int nv = min(kWideHalf, a.V - id0);
+                    const int id0 = tile * 128 + h * kWideRound;
+                    const int nv = min(kWideRound, a.V - id0);
                     FE_WIDE_BATCH(0);
-                    FE_WIDE_BATCH(32);
+                    if (kWideRound > 32) FE_WIDE_BATCH(32);
                     if (a.dbg_logits) {
                         const int rb = r % a.B, ri = r / a.B;
                         for (int u = 0; u < nv; ++u)
@@ -1374,7 +1376,7 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
     // shared memory: the transpose buffers (one per row group), then up to kWideMaxZ z stages
     // (R_pad x 128 B) and the rest to the weight ring (at least as many stages)
     const size_t zst = (size_t)R_pad * 128;
-    const size_t tbytes = (size_t)((R_pad + kWideGroup - 1) / kWideGroup) * kWideHalf * kWideTileStride * sizeof(float);
+    const size_t tbytes = (size_t)((R_pad + kWideGroup - 1) / kWideGroup) * kWideRound * kWideTileStride * sizeof(float);
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(WideState) - 256;
     if (budget < 1024 + tbytes + 2 * (16384 + zst)) return cudaErrorInvalidValue;
     const size_t avail = budget - 1024 - tbytes;
