@@ -72,6 +72,111 @@ __device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int
     return base + (((size_t)b * a.Hkv + g) * a.max_seq + pos) * hd;
 }
 
+// A split's partial per head: the weighted value sum [HD], then its max and its sum of
+// weights, padded to a multiple of four floats so that rows start on 16-byte boundaries.
+template <int HD>
+constexpr int part_row() { return HD + 4; }
+
+// The last split of (sequence, KV head) combines every active split's partials into the
+// G heads' outputs: out = sum_q w_q acc_q / sum_q w_q l_q with w_q = exp(m_q - max m). The
+// partial rows of as many heads as `smem` holds are staged into shared memory by bulk
+// copies (one per head: its splits' rows are contiguous), then each head's weights are
+// formed once and every output sums its splits from shared memory. BASE2: the maxima are
+// in base 2 (scores pre-scaled by log2 e).
+template <int HD, int G, bool BASE2>
+__device__ __forceinline__ void combine_splits(const AttnArgs& a, const float* pb0, int n_act, float* out,
+                                               unsigned char* smem, size_t smem_bytes) {
+    constexpr int RS = part_row<HD>();
+    constexpr int NW = kAttnWarps;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    __shared__ float hl[G];
+    const size_t per_head = (size_t)n_act * (RS + 1) * sizeof(float);  // its rows and weights
+    const int Hp = (int)min((size_t)G, smem_bytes / per_head);
+    if (Hp < 1) {  // more splits than shared memory holds: one split at a time from L2
+        for (int idx = t; idx < G * HD; idx += NW * 32) {
+            const int hh = idx / HD, dd = idx % HD;
+            const float* pb = pb0 + (size_t)hh * a.n_split * RS;
+            float M = -INFINITY;
+            for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * RS + HD));
+            float v = 0.f, L = 0.f;
+            for (int q = 0; q < n_act; ++q) {
+                const float* p = pb + (size_t)q * RS;
+                const float mq = __ldcg(p + HD);
+                if (mq == -INFINITY) continue;
+                const float f = BASE2 ? exp2f(mq - M) : expf(mq - M);
+                v = fmaf(f, __ldcg(p + dd), v);
+                L = fmaf(f, __ldcg(p + HD + 1), L);
+            }
+            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
+        }
+        return;
+    }
+    float* rows = reinterpret_cast<float*>(smem);  // [hn][n_act][RS]
+    __shared__ uint64_t cbar;                      // completion of a pass's bulk copies
+    if (t == 0) {
+        mbar_init(&cbar, 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    for (int h0 = 0, pass = 0; h0 < G; h0 += Hp, ++pass) {
+        const int hn = min(Hp, G - h0);
+        float* wq = rows + (size_t)hn * n_act * RS;  // [hn][n_act] weights
+        // a head's rows of every split are contiguous: one bulk copy per head
+        if (t == 0) {
+            const uint32_t hb = (uint32_t)(n_act * RS * sizeof(float));
+            // the partials were written by other CTAs (generic proxy) and this shared memory
+            // was last written by this CTA's threads: both before the async-proxy copies
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive_expect_tx(&cbar, hb * hn);
+            for (int hh = 0; hh < hn; ++hh)
+                bulk_g2s(rows + (size_t)hh * n_act * RS, pb0 + (size_t)(h0 + hh) * a.n_split * RS, hb, &cbar);
+        }
+        if (!mbar_wait(&cbar, (uint32_t)pass & 1u, a.status)) return;  // (bounded; ST_TIMEOUT recorded)
+        for (int hh = warp; hh < hn; hh += NW) {
+            const float* hr = rows + (size_t)hh * n_act * RS;
+            float M = -INFINITY;
+            for (int q = lane; q < n_act; q += 32) M = fmaxf(M, hr[(size_t)q * RS + HD]);
+            M = warp_max(M);
+            float L = 0.f;
+            for (int q = lane; q < n_act; q += 32) {
+                const float mq = hr[(size_t)q * RS + HD];
+                const float f = mq == -INFINITY ? 0.f : (BASE2 ? exp2f(mq - M) : expf(mq - M));
+                wq[hh * n_act + q] = f;
+                L = fmaf(f, hr[(size_t)q * RS + HD + 1], L);
+            }
+            L = warp_sum(L);
+            if (lane == 0) hl[hh] = L;
+        }
+        __syncthreads();
+        // thread t owns outputs t, t + 128, ...: the splits in the outer loop, so that its
+        // outputs' sums advance together
+        constexpr int NO = (G * HD + NW * 32 - 1) / (NW * 32);
+        float v[NO];
+#pragma unroll
+        for (int o = 0; o < NO; ++o) v[o] = 0.f;
+        for (int q = 0; q < n_act; ++q) {
+#pragma unroll
+            for (int o = 0; o < NO; ++o) {
+                const int idx = t + o * NW * 32;
+                if (idx < hn * HD) {
+                    const int hh = idx / HD, dd = idx - hh * HD;
+                    v[o] = fmaf(wq[hh * n_act + q], rows[((size_t)hh * n_act + q) * RS + dd], v[o]);
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 0; o < NO; ++o) {
+            const int idx = t + o * NW * 32;
+            if (idx < hn * HD) {
+                const int hh = idx / HD, dd = idx - hh * HD;
+                out[(size_t)(h0 + hh) * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
+            }
+        }
+        __syncthreads();  // the next pass overwrites the rows
+    }
+}
+
 template <typename CT, int HD, int G>
 __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a, int S) {
     const LaunchStamp stamp(a.stamp);
@@ -131,7 +236,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     if (t == 0) s_abort = 0;
     // Paged caches: this item's page ids, read once into shared memory (after the K/V slots;
     // -1 marks an invalid id), so that issuing a chunk needs no round trip to the table.
-    int* spg = reinterpret_cast<int*>(dsm + (size_t)kAttnWarps * S * 2 * CHB);
+    int* spg = reinterpret_cast<int*>(dsm + (size_t)a.combine_smem);  // (after the slots / combine area)
     const int pg0 = a.page_table ? t0 / a.page_size : 0;
     if (a.page_table) {
         const int last_row = min(t1, P) - 1;  // cached rows are < P
@@ -364,7 +469,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
             v = fmaf(f, wacc[w][hh][dd], v);
             L = fmaf(f, wl[w][hh], L);
         }
-        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * (HD + 2);
+        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * part_row<HD>();
         pp[dd] = v;
         if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
     }
@@ -375,87 +480,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    // Each split's (max, sum) per head goes to shared memory (the K/V slots are free now) in
-    // one round trip; each head's weights exp(M_q - M) are formed there; each output then
-    // sums its splits with eight loads in flight (a load-then-accumulate loop would wait a
-    // full L2 round trip per split).
-    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * (HD + 2);
-    float* wq = reinterpret_cast<float*>(dsm);  // [n_act][G] weights, then [n_act][G] sums
-    float* lq = wq + n_act * G;
-    __shared__ float hl[G];
-    if ((size_t)2 * n_act * G * sizeof(float) <= (size_t)kAttnWarps * S * 2 * CHB) {
-        for (int idx = t; idx < n_act * G; idx += blockDim.x) {
-            const int q = idx / G, hh = idx % G;
-            const float* p = pb0 + ((size_t)hh * a.n_split + q) * (HD + 2) + HD;
-            wq[idx] = __ldcg(p);
-            lq[idx] = __ldcg(p + 1);
-        }
-        __syncthreads();
-        for (int hh = warp; hh < G; hh += kAttnWarps) {
-            float M = -INFINITY;
-            for (int q = lane; q < n_act; q += 32) M = fmaxf(M, wq[q * G + hh]);
-            M = warp_max(M);
-            float L = 0.f;
-            for (int q = lane; q < n_act; q += 32) {
-                const float mq = wq[q * G + hh];
-                const float f = mq == -INFINITY ? 0.f : expf(mq - M);
-                wq[q * G + hh] = f;
-                L = fmaf(f, lq[q * G + hh], L);
-            }
-            L = warp_sum(L);
-            if (lane == 0) hl[hh] = L;
-        }
-        __syncthreads();
-        // thread t owns outputs t, t + 128, ... (NO of them) and loads QB splits of each at once
-        constexpr int NO = (G * HD + kAttnWarps * 32 - 1) / (kAttnWarps * 32);
-        constexpr int QB = NO >= 32 ? 1 : 32 / NO;
-        float v[NO];
-#pragma unroll
-        for (int o = 0; o < NO; ++o) v[o] = 0.f;
-        for (int q0 = 0; q0 < n_act; q0 += QB) {
-            float x[NO][QB];
-#pragma unroll
-            for (int o = 0; o < NO; ++o) {
-                const int idx = t + o * kAttnWarps * 32, hh = idx / HD, dd = idx % HD;
-                const float* p = pb0 + (size_t)hh * a.n_split * (HD + 2) + dd;
-#pragma unroll
-                for (int u = 0; u < QB; ++u)
-                    x[o][u] = idx < G * HD && q0 + u < n_act ? __ldcg(p + (size_t)(q0 + u) * (HD + 2)) : 0.f;
-            }
-#pragma unroll
-            for (int o = 0; o < NO; ++o) {
-                const int idx = t + o * kAttnWarps * 32, hh = (idx / HD) % G;
-#pragma unroll
-                for (int u = 0; u < QB; ++u)
-                    if (q0 + u < n_act) v[o] = fmaf(wq[(q0 + u) * G + hh], x[o][u], v[o]);
-            }
-        }
-#pragma unroll
-        for (int o = 0; o < NO; ++o) {
-            const int idx = t + o * kAttnWarps * 32;
-            if (idx < G * HD) {
-                const int hh = idx / HD, dd = idx % HD;
-                out[(size_t)hh * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
-            }
-        }
-    } else {  // more splits than the slots hold: the same sums, one split at a time
-        for (int idx = t; idx < G * HD; idx += blockDim.x) {
-            const int hh = idx / HD, dd = idx % HD;
-            const float* pb = pb0 + (size_t)hh * a.n_split * (HD + 2);
-            float M = -INFINITY;
-            for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
-            float v = 0.f, L = 0.f;
-            for (int q = 0; q < n_act; ++q) {
-                const float* p = pb + (size_t)q * (HD + 2);
-                const float mq = __ldcg(p + HD);
-                if (mq == -INFINITY) continue;
-                const float f = expf(mq - M);
-                v = fmaf(f, __ldcg(p + dd), v);
-                L = fmaf(f, __ldcg(p + HD + 1), L);
-            }
-            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
-        }
-    }
+    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
+    combine_splits<HD, G, false>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
@@ -582,7 +608,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     unsigned char* vc = kc + CB;
     // Paged caches: this item's page ids, read once into shared memory after the K/V rows
     // (-1 marks an invalid id)
-    int* spg = reinterpret_cast<int*>(dsm + (size_t)kAttnWarps * 2 * CB);
+    int* spg = reinterpret_cast<int*>(dsm + (size_t)a.combine_smem);  // (after the slots / combine area)
     const int pg0 = a.page_table ? t0 / a.page_size : 0;
     if (a.page_table) {
         const int npg = tc > t0 ? (tc - 1) / a.page_size - pg0 + 1 : 0;
@@ -886,7 +912,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
             v = fmaf(f, wacc[w][hh][dd], v);
             L = fmaf(f, wl[w][hh], L);
         }
-        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * (HD + 2);
+        float* pp = a.part + (((size_t)b * a.H + g * G + hh) * a.n_split + s) * part_row<HD>();
         pp[dd] = v;
         if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
     }
@@ -897,87 +923,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    // Each split's (max, sum) per head goes to shared memory (the K/V slots are free now) in
-    // one round trip; each head's weights exp(M_q - M) are formed there; each output then
-    // sums its splits with eight loads in flight (a load-then-accumulate loop would wait a
-    // full L2 round trip per split).
-    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * (HD + 2);
-    float* wq = reinterpret_cast<float*>(dsm);  // [n_act][G] weights, then [n_act][G] sums
-    float* lq = wq + n_act * G;
-    __shared__ float hl[G];
-    if ((size_t)2 * n_act * G * sizeof(float) <= (size_t)kAttnWarps * 2 * CB) {
-        for (int idx = t; idx < n_act * G; idx += blockDim.x) {
-            const int q = idx / G, hh = idx % G;
-            const float* p = pb0 + ((size_t)hh * a.n_split + q) * (HD + 2) + HD;
-            wq[idx] = __ldcg(p);
-            lq[idx] = __ldcg(p + 1);
-        }
-        __syncthreads();
-        for (int hh = warp; hh < G; hh += kAttnWarps) {
-            float M = -INFINITY;
-            for (int q = lane; q < n_act; q += 32) M = fmaxf(M, wq[q * G + hh]);
-            M = warp_max(M);
-            float L = 0.f;
-            for (int q = lane; q < n_act; q += 32) {
-                const float mq = wq[q * G + hh];
-                const float f = mq == -INFINITY ? 0.f : exp2f(mq - M);
-                wq[q * G + hh] = f;
-                L = fmaf(f, lq[q * G + hh], L);
-            }
-            L = warp_sum(L);
-            if (lane == 0) hl[hh] = L;
-        }
-        __syncthreads();
-        // thread t owns outputs t, t + 128, ... (NO of them) and loads QB splits of each at once
-        constexpr int NO = (G * HD + kAttnWarps * 32 - 1) / (kAttnWarps * 32);
-        constexpr int QB = NO >= 32 ? 1 : 32 / NO;
-        float v[NO];
-#pragma unroll
-        for (int o = 0; o < NO; ++o) v[o] = 0.f;
-        for (int q0 = 0; q0 < n_act; q0 += QB) {
-            float x[NO][QB];
-#pragma unroll
-            for (int o = 0; o < NO; ++o) {
-                const int idx = t + o * kAttnWarps * 32, hh = idx / HD, dd = idx % HD;
-                const float* p = pb0 + (size_t)hh * a.n_split * (HD + 2) + dd;
-#pragma unroll
-                for (int u = 0; u < QB; ++u)
-                    x[o][u] = idx < G * HD && q0 + u < n_act ? __ldcg(p + (size_t)(q0 + u) * (HD + 2)) : 0.f;
-            }
-#pragma unroll
-            for (int o = 0; o < NO; ++o) {
-                const int idx = t + o * kAttnWarps * 32, hh = (idx / HD) % G;
-#pragma unroll
-                for (int u = 0; u < QB; ++u)
-                    if (q0 + u < n_act) v[o] = fmaf(wq[(q0 + u) * G + hh], x[o][u], v[o]);
-            }
-        }
-#pragma unroll
-        for (int o = 0; o < NO; ++o) {
-            const int idx = t + o * kAttnWarps * 32;
-            if (idx < G * HD) {
-                const int hh = idx / HD, dd = idx % HD;
-                out[(size_t)hh * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
-            }
-        }
-    } else {  // more splits than the slots hold: the same sums, one split at a time
-        for (int idx = t; idx < G * HD; idx += blockDim.x) {
-            const int hh = idx / HD, dd = idx % HD;
-            const float* pb = pb0 + (size_t)hh * a.n_split * (HD + 2);
-            float M = -INFINITY;
-            for (int q = 0; q < n_act; ++q) M = fmaxf(M, __ldcg(pb + (size_t)q * (HD + 2) + HD));
-            float v = 0.f, L = 0.f;
-            for (int q = 0; q < n_act; ++q) {
-                const float* p = pb + (size_t)q * (HD + 2);
-                const float mq = __ldcg(p + HD);
-                if (mq == -INFINITY) continue;
-                const float f = exp2f(mq - M);
-                v = fmaf(f, __ldcg(p + dd), v);
-                L = fmaf(f, __ldcg(p + HD + 1), L);
-            }
-            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
-        }
-    }
+    const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
+    combine_splits<HD, G, true>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
@@ -1022,22 +969,34 @@ static bool attn_tc_enabled() {
     return !(e && e[0] == '0');
 }
 
+// The combine's shared memory: the K/V slots (`slots` bytes), grown to hold every split's
+// partial rows at once (one staging pass) when that fits beside the page ids within the
+// kernel's limit (slots + kAttnPageSmem); the page ids then follow it.
+template <int HD, int G>
+static size_t combine_bytes(const AttnArgs& a, size_t slots, size_t pg) {
+    const size_t all = (size_t)G * a.n_split * (part_row<HD>() + 1) * sizeof(float);
+    const size_t cap = slots + (size_t)kAttnPageSmem - pg;
+    return all <= slots ? slots : (all <= cap ? (all + 15) & ~(size_t)15 : slots);
+}
+
 template <typename CT, int HD, int G>
-static cudaError_t launch_g(const AttnArgs& a, cudaStream_t st) {
+static cudaError_t launch_g(const AttnArgs& a0, cudaStream_t st) {
+    AttnArgs a = a0;
     const int S = attn_slots(a.split, HD, sizeof(CT));
-    if constexpr (sizeof(CT) == 2 && HD == 128) {
-        if (attn_tc_enabled()) {
-            const size_t pg = attn_page_ints(a) * sizeof(int);
-            if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
-            return launch_k(attn_tc_kernel<G>, dim3(a.n_split, a.Hkv, a.B), dim3(kAttnWarps * 32),
-                            (size_t)kAttnWarps * 2 * kTcHalfBytes + pg, st, a.pdl, a);
-        }
-    }
     const size_t pg = attn_page_ints(a) * sizeof(int);
     if (pg > (size_t)kAttnPageSmem) return cudaErrorInvalidValue;
+    if constexpr (sizeof(CT) == 2 && HD == 128) {
+        if (attn_tc_enabled()) {
+            const size_t slots = (size_t)kAttnWarps * 2 * kTcHalfBytes;
+            a.combine_smem = (int)combine_bytes<HD, G>(a, slots, pg);
+            return launch_k(attn_tc_kernel<G>, dim3(a.n_split, a.Hkv, a.B), dim3(kAttnWarps * 32),
+                            (size_t)a.combine_smem + pg, st, a.pdl, a);
+        }
+    }
+    const size_t slots = attn_smem(HD, sizeof(CT), S);
+    a.combine_smem = (int)combine_bytes<HD, G>(a, slots, pg);
     dim3 grid(a.n_split, a.Hkv, a.B);
-    return launch_k(attn_kernel<CT, HD, G>, grid, dim3(kAttnWarps * 32), attn_smem(HD, sizeof(CT), S) + pg, st, a.pdl,
-                    a, S);
+    return launch_k(attn_kernel<CT, HD, G>, grid, dim3(kAttnWarps * 32), (size_t)a.combine_smem + pg, st, a.pdl, a, S);
 }
 
 template <typename CT, int HD>

@@ -253,7 +253,7 @@ struct AttnArgs {
     const float* rope_cs;   // [max_seq, hd/2, 2] (cos, sin)
     int B, H, Hkv, hd;
     int split, n_split;     // keys per work item, work items per (sequence, KV head)
-    float* part;            // [B, H, n_split, hd + 2]
+    float* part;            // [B, H, n_split, hd + 4]: value sum [hd], max, sum of weights, padding
     int* counters;          // [B, Hkv] split-completion counters, zero between calls
     float* out;             // [B, H * hd]
     int* status;
@@ -264,6 +264,9 @@ struct AttnArgs {
     int row_stride = 1, row_off = 0, pos_add = 0;
     const int* n_rows = nullptr;
     unsigned long long* stamp = nullptr;  // in-graph timing stamp pair, or null
+    // bytes at the start of dynamic shared memory the last split's combine may use (set by
+    // launch_attention: the K/V slots, or more when every split's partials then fit at once)
+    int combine_smem = 0;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();

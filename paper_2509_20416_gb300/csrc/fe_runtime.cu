@@ -821,7 +821,7 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             cs.size() * sizeof(float),                             // rope
             Rw * d * 4, Rw * d * 4, Rw * nqkv * 4, Rw * H * hd * 4,   // g, x, qkv, o
             Rw * F * 4, R * d * 4,                                  // act, hid
-            B * H * h->attn_nsplit * (hd + 2) * 4,                 // attention partials
+            B * H * h->attn_nsplit * (hd + 4) * 4,                 // attention partials (rows of hd + 4)
             R * h->lm_slabs * k * 4, R * h->lm_slabs * k * 4,      // LM-head partial ids, values
             R * h->lm_slabs * 2 * 4,                               // LM-head partial (max, sum)
             256,                                                   // status
