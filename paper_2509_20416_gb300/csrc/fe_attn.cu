@@ -473,13 +473,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
         pp[dd] = v;
         if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
     }
-    // ---- the last active split of (b, g) combines all splits
-    __threadfence();
+    // ---- the last active split of (b, g) combines all splits. Thread 0's acquire-release
+    // add publishes the CTA's partial (ordered before it by the barrier) and, in the last
+    // split, orders the combine's reads after every other split's.
     __syncthreads();
-    if (t == 0) s_last = atomicAdd(&a.counters[b * a.Hkv + g], 1) == n_act - 1;
+    if (t == 0) s_last = atom_add_acq_rel_gpu(&a.counters[b * a.Hkv + g], 1) == n_act - 1;
     __syncthreads();
     if (!s_last) return;
-    __threadfence();
     const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
     combine_splits<HD, G, false>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
@@ -562,6 +562,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     using CT = bf16_t;
     constexpr int HD = 128;
     constexpr int HALF = HD / 2;
+    static_assert(kAttnWarps * 32 == HD, "one thread per head dimension (the own key and value)");
     constexpr uint32_t CB = kTcHalfBytes;
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(16) float qs[G][HD];
@@ -672,9 +673,23 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     griddep_launch_dependents();
     griddep_wait();
 
-    // queries of the group, rotated at position P and pre-scaled by log2(e) / sqrt(hd)
+    // queries of the group, rotated at position P and pre-scaled by log2(e) / sqrt(hd); the
+    // item holding key P loads the row's own key and value with them (one round trip)
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
     const float scale = 1.4426950408889634f / sqrtf((float)HD);
+    const bool own = t1 == P + 1;  // this item holds the row's own key
+    const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
+    const float* vq = kq + (size_t)a.Hkv * HD;
+    float ok1 = 0.f, ok2 = 0.f, okc = 0.f, oks = 0.f, ov = 0.f;  // (blockDim.x == HD: one element each)
+    if (own) {
+        if (t < HALF) {
+            ok1 = kq[t];
+            ok2 = kq[t + HALF];
+            okc = cs[2 * t];
+            oks = cs[2 * t + 1];
+        }
+        ov = vq[t];
+    }
     for (int idx = t; idx < G * HALF; idx += blockDim.x) {
         const int j = idx / HALF, i = idx % HALF;
         const float* q = a.qkv + qrow * ldq + (size_t)(g * G + j) * HD;
@@ -682,27 +697,21 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
         qs[j][i] = (x1 * c - x2 * sn) * scale;
         qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
     }
-    const bool own = t1 == P + 1;  // this item holds the row's own key
     if (own) {  // rotate the new key and append k, v at slot P
-        const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
-        const float* vq = kq + (size_t)a.Hkv * HD;
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
         if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
-        for (int i = t; i < HALF; i += blockDim.x) {
-            const float x1 = kq[i], x2 = kq[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
-            const float r1 = x1 * c - x2 * sn, r2 = x2 * c + x1 * sn;
-            kn[i] = r1;
-            kn[i + HALF] = r2;
+        if (t < HALF) {
+            const float r1 = ok1 * okc - ok2 * oks, r2 = ok2 * okc + ok1 * oks;
+            kn[t] = r1;
+            kn[t + HALF] = r2;
             if (krow) {
-                Storage<CT>::store(krow, i, r1);
-                Storage<CT>::store(krow, i + HALF, r2);
+                Storage<CT>::store(krow, t, r1);
+                Storage<CT>::store(krow, t + HALF, r2);
             }
         }
-        for (int i = t; i < HD; i += blockDim.x) {
-            vn[i] = vq[i];
-            if (vrow) Storage<CT>::store(vrow, i, vq[i]);
-        }
+        vn[t] = ov;
+        if (vrow) Storage<CT>::store(vrow, t, ov);
     }
     __syncthreads();
     if (own)  // the own key's score per head: warp w takes heads w, w + 4
@@ -916,13 +925,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
         pp[dd] = v;
         if (dd == 0) { pp[HD] = M; pp[HD + 1] = L; }
     }
-    // ---- the last active split of (b, g) combines all splits
-    __threadfence();
+    // ---- the last active split of (b, g) combines all splits. Thread 0's acquire-release
+    // add publishes the CTA's partial (ordered before it by the barrier) and, in the last
+    // split, orders the combine's reads after every other split's.
     __syncthreads();
-    if (t == 0) s_last = atomicAdd(&a.counters[b * a.Hkv + g], 1) == n_act - 1;
+    if (t == 0) s_last = atom_add_acq_rel_gpu(&a.counters[b * a.Hkv + g], 1) == n_act - 1;
     __syncthreads();
     if (!s_last) return;
-    __threadfence();
     const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
     combine_splits<HD, G, true>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
