@@ -69,17 +69,22 @@ TRAFFIC = {
     # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum -k regex:linear_kernel
     #     -s 18 -c 6 on `bench.py --workload l33_70b --set n_layers=1 --also ...` (one draft's six linear
     # launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down; the eight-layer draft repeats the last four)
-    "l33_70b": {"bytes_per_draft": (402788096 + 3366912) + (268564480 + 122624)
-                + 8 * ((167900672 + 48896) + (134358272 + 344064) + (939682048 + 208128) + (469999616 + 81408)),
-                "src": "cac667a35be22899"},
+    "l33_70b": {"bytes_per_draft": (402779648 + 3221504) + (268562176 + 86272)
+                + 8 * ((167900160 + 56320) + (134357760 + 63744) + (939677696 + 256512) + (469996032 + 85248)),
+                "sources": ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh"), "src": "d49661301765124c"},
+    # the same metrics with -k regex:linear_mma_kernel -s 18 -c 6 on `bench.py --workload b32_l31 --set
+    # n_layers=1 --also ...` (the tensor-core products of the six phases; the six-layer draft repeats
+    # the last four)
+    "b32_l31": {"bytes_per_draft": (102311680 + 2799104) + (68231936 + 512)
+                + 6 * ((50935808 + 0) + (34152704 + 0) + (235485184 + 2010880) + (119887872 + 135680)),
+                "sources": ("fe_linear_mma.cu", "fe_tc.cuh", "fe_common.cuh"), "src": "519855c393da0488"},
 }
-KERNEL_SOURCES = ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh")
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(sources) -> str:
     import hashlib
     hsh = hashlib.sha256()
-    for n in KERNEL_SOURCES:
+    for n in sources:
         with open(os.path.join(ROOT, "paper_2509_20416_gb300", "csrc", n), "rb") as f:
             hsh.update(f.read())
     return hsh.hexdigest()[:16]
@@ -447,7 +452,7 @@ def measure(args, name: str, overrides, ws: int, rank: int, local: int, extras: 
         v["share_of_step"] = v["us_per_draft"] / (ms_step * 1e3)
     traffic = None
     tr = TRAFFIC.get(f"{name}{''.join(' ' + o for o in overrides)}")
-    if tr and tr["src"] == kernel_source_hash() and "linear" in kernels:
+    if tr and tr["src"] == kernel_source_hash(tr["sources"]) and "linear" in kernels:
         traffic = tr["bytes_per_draft"] / kernels["linear"]["launches_per_draft"]
     roof = roofline_block(kernels, kbytes, kflops, ms_step, alg_bytes, alg_flops, traffic, n_rep)
     if roof["kernel"] != "linear":
