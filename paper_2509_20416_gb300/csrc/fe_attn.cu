@@ -26,6 +26,7 @@
 #include "fe_kernels.h"
 #include "fe_common.cuh"
 #include "fe_stream.cuh"
+#include "fe_tc.cuh"
 
 namespace fe {
 
@@ -72,6 +73,23 @@ __device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int
     return base + (((size_t)b * a.Hkv + g) * a.max_seq + pos) * hd;
 }
 
+// Output `head`, dimension dd of row qrow: into `out`, or (a.xb) as the bf16 hi + lo pair of
+// the O projection's operand (x = hi + lo to ~16 significant bits, as the operand prep
+// splits it), column head * HD + dd, in the 128-byte-swizzled K-major layout.
+template <int HD>
+__device__ __forceinline__ void put_out(const AttnArgs& a, size_t qrow, int head, int dd, float v) {
+    if (a.xb) {
+        const int k = head * HD + dd;
+        const uint16_t hi = f32_to_bf16(v), lo = f32_to_bf16(v - bf16_to_f32(hi));
+        unsigned char* blk = (unsigned char*)a.xb + (size_t)(k >> 6) * (2 * a.xb_bpad) * 128;
+        const uint32_t ch = (uint32_t)(k & 63) >> 3, el = (uint32_t)(k & 7);
+        *reinterpret_cast<uint16_t*>(blk + sw128_offset((uint32_t)qrow, ch) + 2 * el) = hi;
+        *reinterpret_cast<uint16_t*>(blk + sw128_offset((uint32_t)(a.xb_bpad + qrow), ch) + 2 * el) = lo;
+    } else {
+        a.out[qrow * a.H * HD + (size_t)head * HD + dd] = v;
+    }
+}
+
 // A split's partial per head: the weighted value sum [HD], then its max and its sum of
 // weights, padded to a multiple of four floats so that rows start on 16-byte boundaries.
 template <int HD>
@@ -84,7 +102,7 @@ constexpr int part_row() { return HD + 4; }
 // formed once and every output sums its splits from shared memory. BASE2: the maxima are
 // in base 2 (scores pre-scaled by log2 e).
 template <int HD, int G, bool BASE2>
-__device__ __forceinline__ void combine_splits(const AttnArgs& a, const float* pb0, int n_act, float* out,
+__device__ __forceinline__ void combine_splits(const AttnArgs& a, const float* pb0, int n_act, size_t qrow, int head0,
                                                unsigned char* smem, size_t smem_bytes) {
     constexpr int RS = part_row<HD>();
     constexpr int NW = kAttnWarps;
@@ -107,7 +125,7 @@ __device__ __forceinline__ void combine_splits(const AttnArgs& a, const float* p
                 v = fmaf(f, __ldcg(p + dd), v);
                 L = fmaf(f, __ldcg(p + HD + 1), L);
             }
-            out[(size_t)hh * HD + dd] = L > 0.f ? v / L : 0.f;
+            put_out<HD>(a, qrow, head0 + hh, dd, L > 0.f ? v / L : 0.f);
         }
         return;
     }
@@ -170,7 +188,7 @@ __device__ __forceinline__ void combine_splits(const AttnArgs& a, const float* p
             const int idx = t + o * NW * 32;
             if (idx < hn * HD) {
                 const int hh = idx / HD, dd = idx - hh * HD;
-                out[(size_t)(h0 + hh) * HD + dd] = hl[hh] > 0.f ? v[o] / hl[hh] : 0.f;
+                put_out<HD>(a, qrow, head0 + h0 + hh, dd, hl[hh] > 0.f ? v[o] / hl[hh] : 0.f);
             }
         }
         __syncthreads();  // the next pass overwrites the rows
@@ -207,14 +225,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
     const int ldq = (a.H + 2 * a.Hkv) * HD;
 
-    float* out = a.out + qrow * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
         griddep_launch_dependents();
         griddep_wait();
         if (s == 0) {
             if (g == 0 && t == 0) atomicOr(a.status, ST_CAPACITY);
-            for (int i = t; i < G * HD; i += blockDim.x) out[i] = 0.f;
+            for (int i = t; i < G * HD; i += blockDim.x) put_out<HD>(a, qrow, g * G + i / HD, i % HD, 0.f);
         }
         return;
     }
@@ -481,7 +498,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     __syncthreads();
     if (!s_last) return;
     const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
-    combine_splits<HD, G, false>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
+    combine_splits<HD, G, false>(a, pb0, n_act, qrow, g * G, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 
@@ -584,14 +601,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
     const int ldq = (a.H + 2 * a.Hkv) * HD;
 
-    float* out = a.out + qrow * a.H * HD + (size_t)g * G * HD;
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
         griddep_launch_dependents();
         griddep_wait();
         if (s == 0) {
             if (g == 0 && t == 0) atomicOr(a.status, ST_CAPACITY);
-            for (int i = t; i < G * HD; i += blockDim.x) out[i] = 0.f;
+            for (int i = t; i < G * HD; i += blockDim.x) put_out<HD>(a, qrow, g * G + i / HD, i % HD, 0.f);
         }
         return;
     }
@@ -933,7 +949,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     __syncthreads();
     if (!s_last) return;
     const float* pb0 = a.part + ((size_t)b * a.H + g * G) * a.n_split * part_row<HD>();
-    combine_splits<HD, G, true>(a, pb0, n_act, out, dsm, (size_t)a.combine_smem);
+    combine_splits<HD, G, true>(a, pb0, n_act, qrow, g * G, dsm, (size_t)a.combine_smem);
     if (t == 0) a.counters[b * a.Hkv + g] = 0;
 }
 

@@ -91,6 +91,8 @@ struct LinearArgs {
     // CTA order, applies this phase's epilogue and stores the result before using it (the
     // same operations, in the same order, as the in-kernel reduction).
     int defer = 0;
+    // tensor-core path: the operand is already in place (written by the attention kernel)
+    int prepped = 0;
     struct Prev {
         int active = 0;
         const float* part = nullptr;  // the partial buffer the phase wrote
@@ -267,6 +269,11 @@ struct AttnArgs {
     // bytes at the start of dynamic shared memory the last split's combine may use (set by
     // launch_attention: the K/V slots, or more when every split's partials then fit at once)
     int combine_smem = 0;
+    // batched drafts: the outputs go straight into the O projection's tensor-core operand (bf16
+    // hi/lo, the 128-byte-swizzled layout of fe_tc.cuh, rows [0, xb_bpad) hi and [xb_bpad,
+    // 2 xb_bpad) lo per 64-column block) instead of `out`, so that phase needs no prep kernel
+    uint16_t* xb = nullptr;
+    int xb_bpad = 0;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();

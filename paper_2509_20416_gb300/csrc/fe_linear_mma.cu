@@ -394,7 +394,7 @@ template <int BP>  // B_pad: 8, 16, 24 or 32
 __global__ void __launch_bounds__(kLmThreads, 1) linear_mma_kernel(const LinearArgs a, uint16_t* xb, int S,
                                                                    int stage_bytes, uint32_t tmem_cols, float* part,
                                                                    int* counters, unsigned char* aux) {
-    const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
+    const LaunchStamp stamp(a.stamp ? a.stamp + (a.prepped ? 0 : 2) : nullptr);
     constexpr int N = 2 * BP;
     extern __shared__ unsigned char dsm_raw[];
     __shared__ LinMmaState st;
@@ -663,6 +663,15 @@ cudaError_t launch_linear_mma(const LinearArgs& a, uint16_t* xb, float* part, in
     const int ny = (a.K / 8 + kXprepChunks - 1) / kXprepChunks;
     if (a.norm_post && a.pro == PRO_RMSNORM && (size_t)ny * kLinMmaMaxBatch * sizeof(float) > kAuxEnd - kAuxSq)
         return cudaErrorInvalidValue;
+    if (a.prepped) {  // the operand is in place (the attention kernel wrote it)
+        if (a.prev.active) return cudaErrorInvalidValue;
+        switch (BP) {
+            case 8: return launch_bp<8>(a, xb, part, tctr, aux, dev, st, grid);
+            case 16: return launch_bp<16>(a, xb, part, tctr, aux, dev, st, grid);
+            case 24: return launch_bp<24>(a, xb, part, tctr, aux, dev, st, grid);
+            default: return launch_bp<32>(a, xb, part, tctr, aux, dev, st, grid);
+        }
+    }
     cudaError_t e = row_cta ? launch_k(xprep_row_kernel, dim3(BP), dim3(kRowThreads), (size_t)a.K * sizeof(float), st,
                                        a.pdl, a, BP, xb)
                             : launch_k(xprep_kernel, dim3(BP, ny), dim3(256), 0, st, a.pdl, a, BP, xb,

@@ -124,6 +124,7 @@ struct fe_handle {
     bool lin_mma = false;     // linear phases packed for (and run on) the tensor cores
     bool lin_defer = true;    // tensor-core phases leave split tiles to the next phase's prep
     bool lin_normpost = true; // tensor-core RMSNorm phases: the scale on the products (column-parallel prep)
+    bool attn_operand = true; // tensor-core O projection: its operand written by the attention kernel
     uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
     float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
     int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
@@ -336,12 +337,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
             return FE_OK;
         }
         if (h->lin_mma) {
-            if (pf) {
+            if (pf && !L.prepped) {
                 if (pf->n + 2 > pf->cap) return FE_ERR_INVALID_ARG;
                 pf->kinds[pf->n++] = FE_KERNEL_LINEAR_PREP;
             }
             e = launch_linear_mma(L, h->lin_xb, h->lin_part, h->lin_counters, h->dev, st,
-                                  pf && pf->ev ? pf->ev[pf->n] : nullptr);
+                                  pf && pf->ev && !L.prepped ? pf->ev[pf->n] : nullptr);
         } else {
             e = launch_linear(dt, L, h->dev, st);
         }
@@ -392,6 +393,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     aa.split = h->attn_split_rows; aa.n_split = h->attn_nsplit;
     aa.part = h->attn_part; aa.counters = h->attn_counters; aa.out = h->o; aa.status = h->status;
     aa.pdl = pdl;
+    // batched handles: attention writes the O projection's tensor-core operand itself
+    const bool o_direct = h->lin_mma && h->attn_operand && !stacked;
+    if (o_direct) {
+        aa.xb = h->lin_xb;
+        aa.xb_bpad = linear_mma_bpad(B);
+    }
 
     for (int i = 0; i < N; ++i) {
         const LayerPacked& L = h->layers[i];
@@ -417,7 +424,9 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         la.pro = PRO_F32; la.x = h->o; la.ldx = H * hd;
         la.epi = EPI_RESID; la.y = h->x; la.ldy = d; la.y2 = nullptr; la.ybase = from_x0 ? h->x0 : nullptr;
         next_is(L.w_gu, 2 * F, d, h->x);
+        la.prepped = o_direct ? 1 : 0;
         FE_LINEAR(la);
+        la.prepped = 0;
         // a = silu(W_gate u) * (W_up u), u = RMSNorm(x)
         la.slots = 0;
         la.W = L.w_gu; la.M = 2 * F; la.K = d;
@@ -696,6 +705,10 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             // comparison)
             const char* np = getenv("FE_DRAFT_LIN_NORMPOST");
             h->lin_normpost = !(np && np[0] == '0');
+            // FE_DRAFT_ATTN_OPERAND=0: the attention output goes through float32 and the O
+            // projection's own prep (kept for comparison)
+            const char* ao = getenv("FE_DRAFT_ATTN_OPERAND");
+            h->attn_operand = !(ao && ao[0] == '0');
             const char* sk = getenv("FE_DRAFT_STACK");
             h->use_stack = !h->lin_mma && sk && sk[0] == '1' && stack_slots(kmax, h->dev) >= 1;
         }
@@ -1279,7 +1292,8 @@ int32_t fe_launch_count(const fe_handle* h, int32_t B, int32_t with_tree) {
     const int N = h->cfg.n_layers;
     const int lin = h->lin_mma ? 2 : linear_launches();
     // stacked: N + 1 stack launches hold all linear phases
-    const int lin_total = (h->use_stack && B == 1) ? N + 1 : 2 * lin + N * 4 * lin;
+    // (on batched handles the O projection's operand comes from the attention kernel: no prep)
+    const int lin_total = (h->use_stack && B == 1) ? N + 1 : 2 * lin + N * 4 * lin - (h->lin_mma && h->attn_operand ? N : 0);
     int n = lin_total + N * attention_launches() +
             (h->lm_mma ? 3 : lmhead_launches(N * B, h->cfg.d, h->dev));
     return n + (with_tree ? 1 : 0);

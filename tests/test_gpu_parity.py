@@ -249,3 +249,19 @@ def test_norm_on_operand_matches_oracle(orc, monkeypatch, case):
         H.compare(orc, cfg, g, H.run_oracle(orc, cfg, W, I, ks, vs, b), b)
     scale = np.abs(g["hidden"]).max()
     assert np.abs(a["hidden"] - g["hidden"]).max() <= 1e-5 * scale
+
+
+@pytest.mark.parametrize("case", ["tc_linear_b12_ragged", "parallel_tc_b12"])
+def test_attention_operand_path_is_exact(monkeypatch, case):
+    """Batched tensor-core drafts: the attention kernel writes the O projection's bf16 hi / lo
+    operand itself. The same draft with the attention output stored in float32 and split by
+    the projection's own prep (FE_DRAFT_ATTN_OPERAND=0) gives identical results."""
+    spec = dict(SMALL[case])
+    cfg = wl.make_config(spec.pop("name"), **spec)
+    W, I, ks, vs = _problem(cfg)
+    a = H.run_gpu(cfg, W, I, ks, vs)
+    monkeypatch.setenv("FE_DRAFT_ATTN_OPERAND", "0")
+    b = H.run_gpu(cfg, W, I, ks, vs)
+    assert a["status"] == 0 and b["status"] == 0
+    for key in ("logits", "hidden", "topk_id", "topk_logit", "topk_prob", "lse", "tree_tok"):
+        assert np.array_equal(a[key], b[key]), key

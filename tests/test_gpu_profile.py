@@ -42,9 +42,11 @@ def test_profile_forward_matches_forward(spec):
     n_lin = kinds.count("linear")
     assert n_lin in (2 + 4 * N, N + 1)
     assert all(kinds[j - 1] == "linear" for j in att)
-    if cfg["B"] > 8:  # every tensor-core phase: its operand prep right before it
-        assert kinds.count("linear_prep") == n_lin
+    if cfg["B"] > 8:  # every tensor-core phase: its operand prep right before it, except the
+        # O projection, whose operand the attention kernel writes
+        assert kinds.count("linear_prep") == n_lin - N
         assert all(kinds[j + 1] == "linear" for j, kd in enumerate(kinds) if kd == "linear_prep")
+        assert all(kinds[j + 1] == "linear" for j in att)
     assert kinds[0] in ("linear", "linear_prep") and kinds[-1] == "lm_head"
     assert all(us > 0 for _, us in prof)
     h.close()
