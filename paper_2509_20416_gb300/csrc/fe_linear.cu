@@ -44,28 +44,30 @@ struct LinearEpi {
     }
 };
 
+// n0 > 0: the activations are staged in two passes of n0 and the remaining slices' columns
+// (X holds Kx columns per row), so that a long row leaves room for more pipeline slots
 template <typename WT, int BT>
-__global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int D) {
+__global__ void __launch_bounds__(kStreamThreads, 1) linear_kernel(const LinearArgs a, int D, int n0) {
     const LaunchStamp stamp(a.stamp);
     extern __shared__ __align__(128) unsigned char smem[];
-    const int Kpad = (a.K + 3) & ~3;
+    const int Kx = n0 > 0 ? n0 * StreamGeom<WT>::kKS : (a.K + 3) & ~3;
     const int b0 = blockIdx.y * BT;
     const int nb = min(BT, a.B - b0);
-    StreamSmem s = carve_stream_smem(smem, D, min(BT, a.B), Kpad, BT);
+    StreamSmem s = carve_stream_smem(smem, D, min(BT, a.B), Kx, BT);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     const int g0 = (int)(((int64_t)blockIdx.x * GM) / gridDim.x);
     const int g1 = (int)(((int64_t)(blockIdx.x + 1) * GM) / gridDim.x);
     // weights do not depend on the previous kernel: start streaming them first
-    const int issued = stream_begin<WT>((const unsigned char*)a.W, a.K, g0, g1, s, D);
+    const int issued = stream_begin<WT>((const unsigned char*)a.W, a.K, g0, g1, s, D, false, n0);
     griddep_launch_dependents();
     // gains and embedding rows do not depend on the previous kernel either
     ProParams pp{a.pro, a.x, a.ldx, a.gamma, a.eps, a.embed, a.tok, a.d_split, a.vocab};
-    const bool pre = stage_pre<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status);
+    const bool pre = n0 > 0 ? false : stage_pre<WT>(pp, a.K, s.X, Kx, b0, nb, a.status);
     griddep_wait();
-    stage_activations<WT>(pp, a.K, s.X, Kpad, b0, nb, a.status, s.red, pre);
+    stage_activations<WT>(pp, n0 > 0 ? Kx : a.K, s.X, Kx, b0, nb, a.status, s.red, pre);
     __syncthreads();
     LinearEpi<BT> e{&a, b0, nb};
-    stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kpad, nb, a.status, e, issued);
+    stream_run<WT, BT>((const unsigned char*)a.W, a.K, g0, g1, s, D, Kx, nb, a.status, e, issued, n0, &pp, b0);
 }
 
 // ---- persistent stack of linear phases --------------------------------------------------------
@@ -140,14 +142,34 @@ template <typename WT, int BT>
 cudaError_t launch_bt(const LinearArgs& a, const DeviceInfo& dev, cudaStream_t st) {
     const int Kpad = (a.K + 3) & ~3;
     const int xrows = BT < a.B ? BT : a.B;
-    int D = stream_slots((size_t)dev.max_smem_optin, stream_smem_bytes(0, xrows, Kpad, BT));
     const int pref = a.slots > 0 ? a.slots : kPreferredSlots;
-    D = D > pref ? pref : D;
-    if (D < 1) return cudaErrorInvalidValue;
-    const size_t smem = stream_smem_bytes(D, xrows, Kpad, BT);
+    auto slots_for = [&](int kx) {
+        const int d = stream_slots((size_t)dev.max_smem_optin, stream_smem_bytes(0, xrows, kx, BT));
+        return d > pref ? pref : d;
+    };
+    int D = slots_for(Kpad);
     const int GM = (a.M + kGroupRows - 1) / kGroupRows;
     dim3 grid(GM < dev.num_sms ? GM : dev.num_sms, (a.B + BT - 1) / BT);
-    return launch_k(linear_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D);
+    // A row too long for two slots per warp next to it (the FC over the concatenated target
+    // features, the down projection of a wide MLP) is staged in two passes when that buys a
+    // deeper pipeline and the CTA's row groups fit one epilogue chunk. Plain float32 or
+    // storage-type inputs only (no row-wide RMSNorm, no concatenation).
+    int n0 = 0, Kx = Kpad;
+    constexpr int KS = StreamGeom<WT>::kKS;
+    const int nks = (a.K + KS - 1) / KS;
+    if (D < 2 && nks >= 2 && (a.pro == PRO_F32 || a.pro == PRO_STORAGE) &&
+        (GM + (int)grid.x - 1) / (int)grid.x <= chunk_groups(BT)) {
+        const int h = (nks + 1) / 2;
+        const int d2 = slots_for(h * KS);
+        if (d2 > D) {
+            D = d2;
+            n0 = h;
+            Kx = h * KS;
+        }
+    }
+    if (D < 1) return cudaErrorInvalidValue;
+    const size_t smem = stream_smem_bytes(D, xrows, Kx, BT);
+    return launch_k(linear_kernel<WT, BT>, grid, dim3(kStreamThreads), smem, st, a.pdl, a, D, n0);
 }
 
 template <typename WT>

@@ -179,117 +179,6 @@ __device__ __forceinline__ void tile_compute(const unsigned char* st, const floa
     }
 }
 
-// Stream the row groups [g0, g1) of the tile-packed W through the per-warp pipelines.
-// Must be called by all 256 threads after X is staged. Calls epi.chunk(cg0, cg1, red)
-// on all threads once per chunk of up to kChunk groups; the epilogue reads values with
-// chunk_value<BT>(red, g - cg0, r, b).
-// Issue copy i (the warp's item i of the CTA's tile range) into the warp's slot.
-template <typename WT>
-__device__ __forceinline__ void stream_issue(const unsigned char* Wt, int K, int g0, int nks, int i, int slot,
-                                             uint64_t* full, unsigned char* ring) {
-    using G = StreamGeom<WT>;
-    const int g = g0 + i / nks, ks = i % nks;
-    const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
-    mbar_arrive_expect_tx(&full[slot], bytes);
-    // weights are read once per draft: evict first, keeping L2 for the activations
-    bulk_g2s_hint(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot],
-                  l2_evict_first());
-}
-
-// First half of a stream: initialise the per-warp barriers and issue every warp's first D
-// copies. Touches only the (read-only) weights, so it may run before griddep_wait().
-// Must be called by all 256 threads; returns the number of copies this warp issued.
-// `again`: a later stream of the same CTA (persistent kernel): the barriers are retired
-// first (the previous stream consumed every copy) and the abort flag is kept.
-template <typename WT>
-__device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D,
-                            bool again = false) {
-    using G = StreamGeom<WT>;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nks = (K + G::kKS - 1) / G::kKS;
-    const int total = (g1 - g0) * nks;
-    uint64_t* full = s.full + warp * D;
-    unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
-    int issued = 0;
-    if (lane == 0) {
-        for (int d = 0; d < D; ++d) {
-            if (again) mbar_inval(&full[d]);
-            mbar_init(&full[d], 1);
-        }
-        if (warp == 0 && !again) *s.abort = 0;
-        mbar_fence_init();
-        for (int j = 0; j < D && warp + kWarps * j < total; ++j, ++issued)
-            stream_issue<WT>(Wt, K, g0, nks, warp + kWarps * j, j, full, ring);
-    }
-    return issued;
-}
-
-// Second half: the main loop. `issued` is stream_begin's return value.
-template <typename WT, int BT, typename Epi>
-__device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D, int Kpad, int nb,
-                           int* status, Epi& epi, int issued) {
-    using G = StreamGeom<WT>;
-    using R = WarpMultiSum<kGroupRows * BT>;
-    constexpr int RV = kGroupRows * BT;
-    constexpr int CH = chunk_groups(BT);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nks = (K + G::kKS - 1) / G::kKS;
-    const int total = (g1 - g0) * nks;
-    uint64_t* full = s.full + warp * D;
-    unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
-
-    for (int i = threadIdx.x; i < CH * kWarps * RV; i += kStreamThreads) s.red[i] = 0.f;
-    __syncthreads();
-    auto issue = [&](int i, int slot) { stream_issue<WT>(Wt, K, g0, nks, i, slot, full, ring); };
-
-    float acc[kGroupRows][BT];
-#pragma unroll
-    for (int r = 0; r < kGroupRows; ++r)
-#pragma unroll
-        for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
-    int cur_g = -1;
-    int chunk_end = g0 + CH;
-    for (int j = 0;; ++j) {
-        const int i = warp + kWarps * j;
-        const int g = i < total ? g0 + i / nks : g1;
-        if (g != cur_g && cur_g >= 0) {  // leaving a group: fold this warp's partials into the chunk buffer
-            R::run(&acc[0][0], lane);
-            if (R::owner(lane)) s.red[((size_t)(cur_g - chunk_end + CH) * kWarps + warp) * RV + R::index(lane)] += acc[0][0];
-#pragma unroll
-            for (int r = 0; r < kGroupRows; ++r)
-#pragma unroll
-                for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
-        }
-        // every warp passes every chunk boundary once: when its next group lies beyond the
-        // chunk, or (for the last, possibly partial, chunks) when its items are exhausted
-        while ((g >= chunk_end || i >= total) && chunk_end - CH < g1) {
-            __syncthreads();
-            epi.chunk(chunk_end - CH, min(chunk_end, g1), s.red);
-            __syncthreads();
-            for (int q = threadIdx.x; q < CH * kWarps * RV; q += kStreamThreads) s.red[q] = 0.f;
-            __syncthreads();
-            chunk_end += CH;
-        }
-        if (i >= total) break;
-        cur_g = g;
-        const int slot = j % D;
-        if (mbar_wait_abortable(&full[slot], (uint32_t)(j / D) & 1u, status, s.abort)) {
-            const int kc = (i % nks) * G::kKS;
-            tile_compute<WT, BT>(ring + (size_t)slot * kTileBytes, s.X, Kpad, kc, min(G::kKS, K - kc), nb, lane, acc);
-        }
-        __syncwarp();
-        if (lane == 0 && i + kWarps * D < total && !*(volatile int*)s.abort) {
-            issue(i + kWarps * D, slot);
-            ++issued;
-        }
-        __syncwarp();
-    }
-    // Never leave with copies in flight (only possible after an abort): wait for them.
-    if (lane == 0 && *(volatile int*)s.abort) {
-        for (int jj = 0; jj < issued; ++jj) mbar_wait(&full[jj % D], (uint32_t)(jj / D) & 1u, status, 100000000LL);
-    }
-}
-
 // Stage activations X[b][k] (b < nb, k < K) into shared memory (see Prologue).
 struct ProParams {
     int pro;
@@ -497,6 +386,160 @@ __device__ void stage_activations(const ProParams& p, int K, float* X, int Kpad,
     for (int b = 0; b < nb; ++b)
         for (int k = K + t; k < Kpad; k += kStreamThreads) X[(size_t)b * Kpad + k] = 0.f;
 }
+
+// Item i of a CTA's range is tile (g, ks). With the activations staged in one pass the
+// items run group-major (the n0 = nks slices of group g0, then of g0 + 1, ...). When X holds
+// only the first n0 < nks slices' columns at a time, they run pass-major: slices [0, n0) of
+// every group, then slices [n0, nks) of every group (items0 = groups x n0 items first).
+__device__ __forceinline__ void stream_item(int i, int g0, int nks, int n0, int items0, int& g, int& ks) {
+    if (i < items0) {
+        g = g0 + i / n0;
+        ks = i % n0;
+    } else {
+        const int n1 = nks - n0, i1 = i - items0;
+        g = g0 + i1 / n1;
+        ks = n0 + i1 % n1;
+    }
+}
+
+// Issue copy i (the warp's item i of the CTA's tile range) into the warp's slot.
+template <typename WT>
+__device__ __forceinline__ void stream_issue(const unsigned char* Wt, int K, int g0, int nks, int n0, int items0,
+                                             int i, int slot, uint64_t* full, unsigned char* ring) {
+    using G = StreamGeom<WT>;
+    int g, ks;
+    stream_item(i, g0, nks, n0, items0, g, ks);
+    const uint32_t bytes = (uint32_t)kGroupRows * (uint32_t)min(G::kKS, K - ks * G::kKS) * G::kES;
+    mbar_arrive_expect_tx(&full[slot], bytes);
+    // weights are read once per draft: evict first, keeping L2 for the activations
+    bulk_g2s_hint(ring + (size_t)slot * kTileBytes, Wt + tile_offset<WT>(g, ks, K) * G::kES, bytes, &full[slot],
+                  l2_evict_first());
+}
+
+// First half of a stream: initialise the per-warp barriers and issue every warp's first D
+// copies. Touches only the (read-only) weights, so it may run before griddep_wait().
+// Must be called by all 256 threads; returns the number of copies this warp issued.
+// `again`: a later stream of the same CTA (persistent kernel): the barriers are retired
+// first (the previous stream consumed every copy) and the abort flag is kept. `n0`: slices
+// per activation pass (0: one pass over all of K; see stream_item).
+template <typename WT>
+__device__ int stream_begin(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D,
+                            bool again = false, int n0 = 0) {
+    using G = StreamGeom<WT>;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nks = (K + G::kKS - 1) / G::kKS;
+    const int total = (g1 - g0) * nks;
+    if (n0 <= 0 || n0 > nks) n0 = nks;
+    const int items0 = (g1 - g0) * n0;
+    uint64_t* full = s.full + warp * D;
+    unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
+    int issued = 0;
+    if (lane == 0) {
+        for (int d = 0; d < D; ++d) {
+            if (again) mbar_inval(&full[d]);
+            mbar_init(&full[d], 1);
+        }
+        if (warp == 0 && !again) *s.abort = 0;
+        mbar_fence_init();
+        for (int j = 0; j < D && warp + kWarps * j < total; ++j, ++issued)
+            stream_issue<WT>(Wt, K, g0, nks, n0, items0, warp + kWarps * j, j, full, ring);
+    }
+    return issued;
+}
+
+// Second half, the main loop: stream the row groups [g0, g1) of the tile-packed W through
+// the per-warp pipelines. Must be called by all 256 threads after X is staged. Calls
+// epi.chunk(cg0, cg1, red) on all threads once per chunk of up to kChunk groups; the
+// epilogue reads values with chunk_value<BT>(red, g - cg0, r, b). `issued` is
+// stream_begin's return value. Two activation
+// passes (n0 > 0, pass1 set): X holds columns [0, n0 kKS) at first; once every warp is
+// past its pass-0 items the CTA stages columns [n0 kKS, K) in their place (pass1 gives
+// that prologue; plain float32 or storage-type rows only) and the pass-1 items read them.
+// The caller guarantees that the CTA's groups fit one chunk (g1 - g0 <= chunk_groups(BT)),
+// so the epilogue runs once, after both passes, and every partial sum of a group, from
+// either pass, lands in its warp's slot of the chunk buffer.
+template <typename WT, int BT, typename Epi>
+__device__ void stream_run(const unsigned char* Wt, int K, int g0, int g1, StreamSmem& s, int D, int Kpad, int nb,
+                           int* status, Epi& epi, int issued, int n0 = 0, const ProParams* pass1 = nullptr,
+                           int b0 = 0) {
+    using G = StreamGeom<WT>;
+    using R = WarpMultiSum<kGroupRows * BT>;
+    constexpr int RV = kGroupRows * BT;
+    constexpr int CH = chunk_groups(BT);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nks = (K + G::kKS - 1) / G::kKS;
+    const int total = (g1 - g0) * nks;
+    if (n0 <= 0 || n0 > nks || !pass1) n0 = nks;
+    const int items0 = (g1 - g0) * n0;
+    const int kx0 = n0 * G::kKS;  // the first column of pass 1
+    bool crossed = n0 == nks;
+    uint64_t* full = s.full + warp * D;
+    unsigned char* ring = s.ring + (size_t)warp * D * kTileBytes;
+
+    for (int i = threadIdx.x; i < CH * kWarps * RV; i += kStreamThreads) s.red[i] = 0.f;
+    __syncthreads();
+    auto issue = [&](int i, int slot) { stream_issue<WT>(Wt, K, g0, nks, n0, items0, i, slot, full, ring); };
+
+    float acc[kGroupRows][BT];
+#pragma unroll
+    for (int r = 0; r < kGroupRows; ++r)
+#pragma unroll
+        for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
+    int cur_g = -1;
+    int chunk_end = g0 + CH;
+    for (int j = 0;; ++j) {
+        const int i = warp + kWarps * j;
+        int g = g1, ks = 0;
+        if (i < total) stream_item(i, g0, nks, n0, items0, g, ks);
+        if (g != cur_g && cur_g >= 0) {  // leaving a group: fold this warp's partials into the chunk buffer
+            R::run(&acc[0][0], lane);
+            if (R::owner(lane)) s.red[((size_t)(cur_g - chunk_end + CH) * kWarps + warp) * RV + R::index(lane)] += acc[0][0];
+#pragma unroll
+            for (int r = 0; r < kGroupRows; ++r)
+#pragma unroll
+                for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
+        }
+        // every warp crosses into pass 1 once (before any chunk boundary: all groups are
+        // in one chunk then)
+        if (!crossed && i >= items0) {
+            crossed = true;
+            __syncthreads();  // no warp reads pass-0 columns any more
+            ProParams p1 = *pass1;
+            p1.x = (const unsigned char*)p1.x + (size_t)kx0 * (p1.pro == PRO_F32 ? sizeof(float) : (size_t)G::kES);
+            stage_activations<WT>(p1, K - kx0, s.X, Kpad, b0, nb, status, nullptr);
+            __syncthreads();
+        }
+        // every warp passes every chunk boundary once: when its next group lies beyond the
+        // chunk, or (for the last, possibly partial, chunks) when its items are exhausted
+        while ((g >= chunk_end || i >= total) && chunk_end - CH < g1) {
+            __syncthreads();
+            epi.chunk(chunk_end - CH, min(chunk_end, g1), s.red);
+            __syncthreads();
+            for (int q = threadIdx.x; q < CH * kWarps * RV; q += kStreamThreads) s.red[q] = 0.f;
+            __syncthreads();
+            chunk_end += CH;
+        }
+        if (i >= total) break;
+        cur_g = g;
+        const int slot = j % D;
+        if (mbar_wait_abortable(&full[slot], (uint32_t)(j / D) & 1u, status, s.abort)) {
+            const int kc = ks * G::kKS;
+            tile_compute<WT, BT>(ring + (size_t)slot * kTileBytes, s.X, Kpad, ks < n0 ? kc : kc - kx0,
+                                 min(G::kKS, K - kc), nb, lane, acc);
+        }
+        __syncwarp();
+        if (lane == 0 && i + kWarps * D < total && !*(volatile int*)s.abort) {
+            issue(i + kWarps * D, slot);
+            ++issued;
+        }
+        __syncwarp();
+    }
+    // Never leave with copies in flight (only possible after an abort): wait for them.
+    if (lane == 0 && *(volatile int*)s.abort) {
+        for (int jj = 0; jj < issued; ++jj) mbar_wait(&full[jj % D], (uint32_t)(jj / D) & 1u, status, 100000000LL);
+    }
+}
+
 
 // Slots per warp that fit next to `fixed` bytes of other shared memory (0 if none fits).
 inline int stream_slots(size_t smem_budget, size_t fixed) {

@@ -96,6 +96,16 @@ SMALL = {
                                       n_layers=3, dtype="bf16", B=12, prefix=0, top_k=8, rope_theta=1e4,
                                       seed=14, page_size=0, parallel_layers=1),
                             prefix_list=[37, 0, 150, 1, 64, 5, 300, 2, 128, 129, 7, 90]),
+    # rows too long for two weight slots per warp beside them: the activations are staged in
+    # two column passes. B = 1 with a 27000-wide MLP (down projection over 27 slices, the last
+    # one ragged); float32 weights, B = 3 (two activation rows per CTA, then one) through the
+    # 12288-column feature FC
+    "twopass_down_b1": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=27000, vocab=3001,
+                                      n_layers=2, dtype="bf16", B=1, prefix=0, top_k=8, rope_theta=1e4,
+                                      seed=20, page_size=0), prefix_list=[77]),
+    "twopass_fuse_f32_b3": dict(name=dict(d=4096, n_heads=32, n_kv_heads=8, head_dim=128, ffn=1024, vocab=3001,
+                                          n_layers=1, dtype="f32", B=3, prefix=0, top_k=4, rope_theta=5e5,
+                                          seed=21, page_size=0), prefix_list=[5, 0, 70]),
     # bf16, hd 128, G = 2, 4, 8 (G = 1 below and at full size): the tensor-core attention kernel. Prefixes on both sides of
     # the 32-key chunk and 128-key split boundaries, an empty prefix, several splits per
     # sequence (combined by the last split), page sizes 16 and 8, and contiguous caches.
