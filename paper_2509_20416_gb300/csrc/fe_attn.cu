@@ -27,6 +27,7 @@
 #include "fe_common.cuh"
 #include "fe_stream.cuh"
 #include "fe_tc.cuh"
+#include "fe_splitk.cuh"
 
 namespace fe {
 
@@ -76,6 +77,43 @@ __device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int
 // Output `head`, dimension dd of row qrow: into `out`, or (a.xb) as the bf16 hi + lo pair of
 // the O projection's operand (x = hi + lo to ~16 significant bits, as the operand prep
 // splits it), column head * HD + dd, in the 128-byte-swizzled K-major layout.
+// The finished (pre-RoPE) query columns of heads [g G, g G + G) of row qrow into q (G x HD,
+// heads consecutive) and, when `own`, the row's key and value into kn / vn: read from qkv as
+// the QKV phase stored it or, when that phase deferred its split tiles (a.qprev.active),
+// summed here from their shares in CTA order (the phase's own fix-up). One 8-column chunk per
+// thread and step, every load of a step issued before the first is used.
+template <int HD, int G>
+__device__ __forceinline__ void load_qkv(const AttnArgs& a, size_t qrow, int g, bool own, float* q, float* kn,
+                                         float* vn) {
+    constexpr int NQ = G * HD / 8, NO = HD / 8;
+    const int ldq = (a.H + 2 * a.Hkv) * HD;
+    const int n = NQ + (own ? 2 * NO : 0);
+    for (int c = threadIdx.x; c < n; c += blockDim.x) {
+        int k0;
+        float* dst;
+        if (c < NQ) {
+            k0 = g * G * HD + 8 * c;
+            dst = q + 8 * c;
+        } else if (c < NQ + NO) {
+            k0 = (a.H + g) * HD + 8 * (c - NQ);
+            dst = kn + 8 * (c - NQ);
+        } else {
+            k0 = (a.H + a.Hkv + g) * HD + 8 * (c - NQ - NO);
+            dst = vn + 8 * (c - NQ - NO);
+        }
+        float v[8];
+        if (a.qprev.active) {
+            prev_finish_t<false, false>(a.qprev, a.qprev_bpad, (int)qrow, k0, v);
+        } else {
+            const float4* p = reinterpret_cast<const float4*>(a.qkv + qrow * ldq + k0);
+            const float4 x0 = p[0], x1 = p[1];
+            v[0] = x0.x; v[1] = x0.y; v[2] = x0.z; v[3] = x0.w; v[4] = x1.x; v[5] = x1.y; v[6] = x1.z; v[7] = x1.w;
+        }
+        reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
 template <int HD>
 __device__ __forceinline__ void put_out(const AttnArgs& a, size_t qrow, int head, int dd, float v) {
     if (a.xb) {
@@ -223,7 +261,6 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     }
     const int P = a.prefix_len[b] + a.pos_add;
     const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
-    const int ldq = (a.H + 2 * a.Hkv) * HD;
 
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
@@ -320,21 +357,21 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     // queries of the group, rotated at position P and pre-scaled by 1/sqrt(hd)
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
     const float scale = 1.0f / sqrtf((float)HD);
+    const bool own = t1 == P + 1;  // this item holds the row's own key
+    load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
+    __syncthreads();
     for (int idx = t; idx < G * HALF; idx += blockDim.x) {
         const int j = idx / HALF, i = idx % HALF;
-        const float* q = a.qkv + qrow * ldq + (size_t)(g * G + j) * HD;
-        const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+        const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
         qs[j][i] = (x1 * c - x2 * sn) * scale;
         qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
     }
-    if (t1 == P + 1) {  // this item holds the row's own key: rotate it and append k, v at slot P
-        const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
-        const float* vq = kq + (size_t)a.Hkv * HD;
+    if (own) {  // rotate the row's own key and append k, v at slot P
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
         if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
         for (int i = t; i < HALF; i += blockDim.x) {
-            const float x1 = kq[i], x2 = kq[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            const float x1 = kn[i], x2 = kn[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
             const float r1 = x1 * c - x2 * sn, r2 = x2 * c + x1 * sn;
             kn[i] = r1;
             kn[i + HALF] = r2;
@@ -343,10 +380,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
                 Storage<CT>::store(krow, i + HALF, r2);
             }
         }
-        for (int i = t; i < HD; i += blockDim.x) {
-            vn[i] = vq[i];
-            if (vrow) Storage<CT>::store(vrow, i, vq[i]);
-        }
+        if (vrow)
+            for (int i = t; i < HD; i += blockDim.x) Storage<CT>::store(vrow, i, vn[i]);
     }
     __syncthreads();
 
@@ -599,7 +634,6 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     }
     const int P = a.prefix_len[b] + a.pos_add;
     const size_t qrow = (size_t)b * a.row_stride + a.row_off;  // this row in qkv and out
-    const int ldq = (a.H + 2 * a.Hkv) * HD;
 
     const bool valid = P >= 0 && P + 1 <= a.max_seq;
     if (!valid) {
@@ -694,30 +728,20 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
     const float scale = 1.4426950408889634f / sqrtf((float)HD);
     const bool own = t1 == P + 1;  // this item holds the row's own key
-    const float* kq = a.qkv + qrow * ldq + (size_t)a.H * HD + (size_t)g * HD;
-    const float* vq = kq + (size_t)a.Hkv * HD;
-    float ok1 = 0.f, ok2 = 0.f, okc = 0.f, oks = 0.f, ov = 0.f;  // (blockDim.x == HD: one element each)
-    if (own) {
-        if (t < HALF) {
-            ok1 = kq[t];
-            ok2 = kq[t + HALF];
-            okc = cs[2 * t];
-            oks = cs[2 * t + 1];
-        }
-        ov = vq[t];
-    }
+    load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
+    __syncthreads();
     for (int idx = t; idx < G * HALF; idx += blockDim.x) {
         const int j = idx / HALF, i = idx % HALF;
-        const float* q = a.qkv + qrow * ldq + (size_t)(g * G + j) * HD;
-        const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+        const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
         qs[j][i] = (x1 * c - x2 * sn) * scale;
         qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
     }
-    if (own) {  // rotate the new key and append k, v at slot P
+    if (own) {  // rotate the new key and append k, v at slot P (blockDim.x == HD: one element each)
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
         if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
         if (t < HALF) {
+            const float ok1 = kn[t], ok2 = kn[t + HALF], okc = cs[2 * t], oks = cs[2 * t + 1];
             const float r1 = ok1 * okc - ok2 * oks, r2 = ok2 * okc + ok1 * oks;
             kn[t] = r1;
             kn[t + HALF] = r2;
@@ -726,8 +750,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
                 Storage<CT>::store(krow, t + HALF, r2);
             }
         }
-        vn[t] = ov;
-        if (vrow) Storage<CT>::store(vrow, t, ov);
+        if (vrow) Storage<CT>::store(vrow, t, vn[t]);
     }
     __syncthreads();
     if (own)  // the own key's score per head: warp w takes heads w, w + 4

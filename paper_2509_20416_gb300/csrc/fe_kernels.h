@@ -274,6 +274,11 @@ struct AttnArgs {
     // 2 xb_bpad) lo per 64-column block) instead of `out`, so that phase needs no prep kernel
     uint16_t* xb = nullptr;
     int xb_bpad = 0;
+    // batched drafts: the QKV phase left the tiles it split between CTAs to this kernel, which
+    // sums their shares for the columns it reads (fe_splitk.cuh); qprev_bpad is that phase's
+    // operand row padding (its shares' row stride)
+    LinearArgs::Prev qprev{};
+    int qprev_bpad = 0;
 };
 int attn_split(int B, int Hkv, int max_seq, const DeviceInfo& dev);
 cudaError_t attention_prepare();

@@ -410,8 +410,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
         const bool from_x0 = i == 0 || c.parallel_layers;
         la.pro = PRO_RMSNORM; la.x = from_x0 ? h->x0 : h->x; la.ldx = d; la.gamma = L.attn_norm;
         la.epi = EPI_STORE; la.y = h->qkv; la.ldy = nqkv; la.y2 = nullptr;
-        next_is(nullptr, 0, 0, nullptr);  // attention follows
+        // attention follows; on batched handles it finishes this phase's split tiles itself
+        next_is(h->lin_mma ? L.w_qkv : nullptr, 0, 0, h->qkv);
         FE_LINEAR(la);
+        aa.qprev = pending;
+        aa.qprev_bpad = pending.active ? linear_mma_bpad(B) : 0;
+        pending = LinearArgs::Prev{};
         // attention over the layer's cache (+ own row), appends slot P_b
         aa.kc = a->k_cache[i]; aa.vc = a->v_cache[i];
         if ((lrc = flush_stack()) != FE_OK) return lrc;

@@ -228,8 +228,10 @@ def test_parity_full_size(orc, name):
 def test_deferred_split_tiles_bit_identical(monkeypatch, case):
     """A tensor-core phase followed by another leaves the tiles it shares with other CTAs to
     that phase's operand prep, which sums the shares in CTA order and applies the epilogue
-    there. The draft must equal the one with the reduction inside each phase
-    (FE_DRAFT_LIN_DEFER=0) bit for bit: logits, hidden states, candidates, caches."""
+    there; the QKV phase leaves them to the attention kernel, which sums the shares of the
+    query, key and value columns it reads. The draft must equal the one with the reduction
+    inside each phase (FE_DRAFT_LIN_DEFER=0) bit for bit: logits, hidden states, candidates,
+    caches."""
     spec = dict(SMALL[case])
     cfg = wl.make_config(spec.pop("name"), **spec)
     W, I, ks, vs = _problem(cfg)
