@@ -77,40 +77,34 @@ __device__ __forceinline__ CT* cache_row(CT* base, const AttnArgs& a, int b, int
 // Output `head`, dimension dd of row qrow: into `out`, or (a.xb) as the bf16 hi + lo pair of
 // the O projection's operand (x = hi + lo to ~16 significant bits, as the operand prep
 // splits it), column head * HD + dd, in the 128-byte-swizzled K-major layout.
-// The finished (pre-RoPE) query columns of heads [g G, g G + G) of row qrow into q (G x HD,
-// heads consecutive) and, when `own`, the row's key and value into kn / vn: read from qkv as
-// the QKV phase stored it or, when that phase deferred its split tiles (a.qprev.active),
-// summed here from their shares in CTA order (the phase's own fix-up). One 8-column chunk per
-// thread and step, every load of a step issued before the first is used.
+// A QKV phase that deferred its split tiles (a.qprev): the finished (pre-RoPE) query
+// columns of heads [g G, g G + G) of row qrow into q (G x HD, heads consecutive) and, when
+// `own`, the row's key and value into kn / vn, each 8-column chunk summed from the phase's
+// shares in CTA order (its own fix-up). Thread t takes chunks t, t + blockDim.x, ...
 template <int HD, int G>
 __device__ __forceinline__ void load_qkv(const AttnArgs& a, size_t qrow, int g, bool own, float* q, float* kn,
                                          float* vn) {
     constexpr int NQ = G * HD / 8, NO = HD / 8;
-    const int ldq = (a.H + 2 * a.Hkv) * HD;
+    constexpr int NC = (NQ + 2 * NO + kAttnWarps * 32 - 1) / (kAttnWarps * 32);
     const int n = NQ + (own ? 2 * NO : 0);
-    for (int c = threadIdx.x; c < n; c += blockDim.x) {
-        int k0;
-        float* dst;
-        if (c < NQ) {
-            k0 = g * G * HD + 8 * c;
-            dst = q + 8 * c;
-        } else if (c < NQ + NO) {
-            k0 = (a.H + g) * HD + 8 * (c - NQ);
-            dst = kn + 8 * (c - NQ);
-        } else {
-            k0 = (a.H + a.Hkv + g) * HD + 8 * (c - NQ - NO);
-            dst = vn + 8 * (c - NQ - NO);
-        }
-        float v[8];
-        if (a.qprev.active) {
-            prev_finish_t<false, false>(a.qprev, a.qprev_bpad, (int)qrow, k0, v);
-        } else {
-            const float4* p = reinterpret_cast<const float4*>(a.qkv + qrow * ldq + k0);
-            const float4 x0 = p[0], x1 = p[1];
-            v[0] = x0.x; v[1] = x0.y; v[2] = x0.z; v[3] = x0.w; v[4] = x1.x; v[5] = x1.y; v[6] = x1.z; v[7] = x1.w;
-        }
-        reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
-        reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    auto column = [&](int c) {  // first qkv column of chunk c
+        return c < NQ ? g * G * HD + 8 * c
+                      : (c < NQ + NO ? (a.H + g) * HD + 8 * (c - NQ) : (a.H + a.Hkv + g) * HD + 8 * (c - NQ - NO));
+    };
+    float v[NC][8];
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+        const int c = threadIdx.x + j * kAttnWarps * 32;
+        if (c >= n) break;
+        prev_finish_t<false, false>(a.qprev, a.qprev_bpad, (int)qrow, column(c), v[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+        const int c = threadIdx.x + j * kAttnWarps * 32;
+        if (c >= n) break;
+        float* dst = c < NQ ? q + 8 * c : (c < NQ + NO ? kn + 8 * (c - NQ) : vn + 8 * (c - NQ - NO));
+        reinterpret_cast<float4*>(dst)[0] = make_float4(v[j][0], v[j][1], v[j][2], v[j][3]);
+        reinterpret_cast<float4*>(dst)[1] = make_float4(v[j][4], v[j][5], v[j][6], v[j][7]);
     }
 }
 
@@ -354,24 +348,44 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
     griddep_launch_dependents();
     griddep_wait();
 
-    // queries of the group, rotated at position P and pre-scaled by 1/sqrt(hd)
+    // queries of the group, rotated at position P and pre-scaled by 1/sqrt(hd). A deferred
+    // QKV phase's columns are first finished into qs / kn / vn (then rotated in place);
+    // otherwise they are read from qkv here.
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
     const float scale = 1.0f / sqrtf((float)HD);
     const bool own = t1 == P + 1;  // this item holds the row's own key
-    load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
-    __syncthreads();
-    for (int idx = t; idx < G * HALF; idx += blockDim.x) {
-        const int j = idx / HALF, i = idx % HALF;
-        const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
-        qs[j][i] = (x1 * c - x2 * sn) * scale;
-        qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+    const bool dq = a.qprev.active;
+    if (dq) {
+        load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
+        __syncthreads();
+    }
+    const float* qrow_p = a.qkv + qrow * (size_t)((a.H + 2 * a.Hkv) * HD);
+    // (two loops: in the one reading qkv no load may wait for an earlier iteration's store)
+    if (dq) {
+        for (int idx = t; idx < G * HALF; idx += blockDim.x) {
+            const int j = idx / HALF, i = idx % HALF;
+            const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            qs[j][i] = (x1 * c - x2 * sn) * scale;
+            qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+        }
+    } else {
+        for (int idx = t; idx < G * HALF; idx += blockDim.x) {
+            const int j = idx / HALF, i = idx % HALF;
+            const float* q = qrow_p + (size_t)(g * G + j) * HD;
+            const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            qs[j][i] = (x1 * c - x2 * sn) * scale;
+            qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+        }
     }
     if (own) {  // rotate the row's own key and append k, v at slot P
+        const float* kq = qrow_p + (size_t)a.H * HD + (size_t)g * HD;
+        const float* vq = kq + (size_t)a.Hkv * HD;
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
         if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
         for (int i = t; i < HALF; i += blockDim.x) {
-            const float x1 = kn[i], x2 = kn[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            const float x1 = dq ? kn[i] : kq[i], x2 = dq ? kn[i + HALF] : kq[i + HALF];
+            const float c = cs[2 * i], sn = cs[2 * i + 1];
             const float r1 = x1 * c - x2 * sn, r2 = x2 * c + x1 * sn;
             kn[i] = r1;
             kn[i + HALF] = r2;
@@ -380,8 +394,11 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnArgs a,
                 Storage<CT>::store(krow, i + HALF, r2);
             }
         }
-        if (vrow)
-            for (int i = t; i < HD; i += blockDim.x) Storage<CT>::store(vrow, i, vn[i]);
+        for (int i = t; i < HD; i += blockDim.x) {
+            const float x = dq ? vn[i] : vq[i];
+            vn[i] = x;
+            if (vrow) Storage<CT>::store(vrow, i, x);
+        }
     }
     __syncthreads();
 
@@ -608,7 +625,7 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-template <int G>
+template <int G, bool DQ>
 __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnArgs a) {
     const LaunchStamp stamp(a.stamp);
     using CT = bf16_t;
@@ -724,24 +741,52 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
     griddep_wait();
 
     // queries of the group, rotated at position P and pre-scaled by log2(e) / sqrt(hd); the
-    // item holding key P loads the row's own key and value with them (one round trip)
+    // item holding key P loads the row's own key and value with them (one round trip). A
+    // deferred QKV phase's columns are first finished into qs / kn / vn (then rotated in
+    // place); otherwise they are read from qkv here.
     const float* cs = a.rope_cs + (size_t)P * HALF * 2;
     const float scale = 1.4426950408889634f / sqrtf((float)HD);
     const bool own = t1 == P + 1;  // this item holds the row's own key
-    load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
-    __syncthreads();
-    for (int idx = t; idx < G * HALF; idx += blockDim.x) {
-        const int j = idx / HALF, i = idx % HALF;
-        const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
-        qs[j][i] = (x1 * c - x2 * sn) * scale;
-        qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+    constexpr bool dq = DQ;  // (a.qprev.active: a separate instantiation)
+    if (dq) {
+        load_qkv<HD, G>(a, qrow, g, own, &qs[0][0], kn, vn);
+        __syncthreads();
     }
-    if (own) {  // rotate the new key and append k, v at slot P (blockDim.x == HD: one element each)
+    const float* qrow_p = a.qkv + qrow * (size_t)((a.H + 2 * a.Hkv) * HD);
+    const float* kq = qrow_p + (size_t)a.H * HD + (size_t)g * HD;
+    const float* vq = kq + (size_t)a.Hkv * HD;
+    float ok1 = 0.f, ok2 = 0.f, okc = 0.f, oks = 0.f, ov = 0.f;  // (blockDim.x == HD: one element each)
+    if (own) {
+        if (t < HALF) {
+            ok1 = dq ? kn[t] : kq[t];
+            ok2 = dq ? kn[t + HALF] : kq[t + HALF];
+            okc = cs[2 * t];
+            oks = cs[2 * t + 1];
+        }
+        ov = dq ? vn[t] : vq[t];
+    }
+    // (two loops: in the one reading qkv no load may wait for an earlier iteration's store)
+    if (dq) {
+        for (int idx = t; idx < G * HALF; idx += blockDim.x) {
+            const int j = idx / HALF, i = idx % HALF;
+            const float x1 = qs[j][i], x2 = qs[j][i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            qs[j][i] = (x1 * c - x2 * sn) * scale;
+            qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+        }
+    } else {
+        for (int idx = t; idx < G * HALF; idx += blockDim.x) {
+            const int j = idx / HALF, i = idx % HALF;
+            const float* q = qrow_p + (size_t)(g * G + j) * HD;
+            const float x1 = q[i], x2 = q[i + HALF], c = cs[2 * i], sn = cs[2 * i + 1];
+            qs[j][i] = (x1 * c - x2 * sn) * scale;
+            qs[j][i + HALF] = (x2 * c + x1 * sn) * scale;
+        }
+    }
+    if (own) {  // rotate the new key and append k, v at slot P
         CT* krow = cache_row<CT>((CT*)a.kc, a, b, g, P, HD);
         CT* vrow = cache_row<CT>((CT*)a.vc, a, b, g, P, HD);
         if ((!krow || !vrow) && t == 0) atomicOr(a.status, ST_DEVICE);
         if (t < HALF) {
-            const float ok1 = kn[t], ok2 = kn[t + HALF], okc = cs[2 * t], oks = cs[2 * t + 1];
             const float r1 = ok1 * okc - ok2 * oks, r2 = ok2 * okc + ok1 * oks;
             kn[t] = r1;
             kn[t + HALF] = r2;
@@ -750,7 +795,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 3) attn_tc_kernel(const AttnA
                 Storage<CT>::store(krow, t + HALF, r2);
             }
         }
-        if (vrow) Storage<CT>::store(vrow, t, vn[t]);
+        vn[t] = ov;
+        if (vrow) Storage<CT>::store(vrow, t, ov);
     }
     __syncthreads();
     if (own)  // the own key's score per head: warp w takes heads w, w + 4
@@ -1037,7 +1083,8 @@ static cudaError_t launch_g(const AttnArgs& a0, cudaStream_t st) {
         if (attn_tc_enabled()) {
             const size_t slots = (size_t)kAttnWarps * 2 * kTcHalfBytes;
             a.combine_smem = (int)combine_bytes<HD, G>(a, slots, pg);
-            return launch_k(attn_tc_kernel<G>, dim3(a.n_split, a.Hkv, a.B), dim3(kAttnWarps * 32),
+            return launch_k(a.qprev.active ? attn_tc_kernel<G, true> : attn_tc_kernel<G, false>,
+                            dim3(a.n_split, a.Hkv, a.B), dim3(kAttnWarps * 32),
                             (size_t)a.combine_smem + pg, st, a.pdl, a);
         }
     }
@@ -1069,7 +1116,9 @@ static cudaError_t prepare_hd() {
 
 cudaError_t attention_prepare() {
     cudaError_t e;
-    for (auto k : {attn_tc_kernel<1>, attn_tc_kernel<2>, attn_tc_kernel<4>, attn_tc_kernel<8>})
+    for (auto k : {attn_tc_kernel<1, false>, attn_tc_kernel<2, false>, attn_tc_kernel<4, false>,
+                   attn_tc_kernel<8, false>, attn_tc_kernel<1, true>, attn_tc_kernel<2, true>,
+                   attn_tc_kernel<4, true>, attn_tc_kernel<8, true>})
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)(kAttnWarps * 2 * kTcHalfBytes) + kAttnPageSmem)) != cudaSuccess)
             return e;
