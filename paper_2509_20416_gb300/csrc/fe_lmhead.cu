@@ -994,6 +994,7 @@ cudaError_t launch_lmhead_mma(const LmHeadArgs& a, uint16_t* zb, const DeviceInf
 //   - lmhead_merge_kernel (one CTA per row) then merges the slabs as merge_rows does.
 constexpr int kWideKMax = 16;     // top_k limit of this kernel (a sorted list in registers)
 constexpr int kWideRowsMax = 256;
+constexpr int kWideLoRows = 16;   // up to this many (padded) rows z is split into bf16 hi + lo
 constexpr int kWideGroup = 128;   // rows of a row group (one per thread of its four warps)
 constexpr int kWideRound = 32;    // vocabulary entries staged per transpose round (a quarter of a tile)
 constexpr int kWideRoundWarps = kWideRound / 32;  // the warps that stage one round
@@ -1131,13 +1132,16 @@ struct WideRow {
         w.m = nm;                                                                                  \
     } while (0)
 
-template <int KM, bool SMP>
+template <int KM, bool SMP, bool LO>
 __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHeadArgs a, const uint16_t* zb, int R_pad,
                                                                       int SW, int SZ, uint32_t tmem_cols) {
     const LaunchStamp stamp(a.stamp ? a.stamp + 2 : nullptr);
     extern __shared__ unsigned char dsm_raw[];
     __shared__ WideState st;
-    const uint32_t zbytes = (uint32_t)R_pad * 128u;
+    // LO: z as bf16 hi (rows [0, R_pad)) + lo (rows [R_pad, 2 R_pad)) parts, NZ = 2 R_pad MMA
+    // columns, the epilogue adding the two accumulator columns of a row; else z in bf16 alone
+    const int NZ = LO ? 2 * R_pad : R_pad;
+    const uint32_t zbytes = (uint32_t)NZ * 128u;
     // [weight ring: SW x 16 KB][z ring: SZ x zbytes][transpose buffers: one per row group]
     unsigned char* wring = (unsigned char*)(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* zring = wring + (size_t)SW * 16384;
@@ -1213,14 +1217,14 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
         }
     } else if (warp == 9) {  // ---- MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, R_pad);
+            const uint32_t idesc = idesc_bf16_f32(128, NZ);
             int sw = 0, sz = 0;          // it % SW, it % SZ
             uint32_t pw = 0, pz = 0;     // phase bits of wfull[sw], zfull[sz]
             for (int tile = t0, j = 0; tile < t1; ++tile, ++j) {
                 const int buf = j & 1;
                 if (!mbar_wait_abortable(&st.tempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, a.status, &st.abort)) break;
                 tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)(buf * R_pad);
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * NZ);
                 bool ok = true;
                 for (int kb = 0; kb < nkb; ++kb) {
                     if (!mbar_wait_abortable(&st.wfull[sw], pw, a.status, &st.abort) ||
@@ -1264,7 +1268,7 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
             if (!mbar_wait_abortable(&st.tfull[buf], (uint32_t)(j >> 1) & 1u, a.status, &st.abort)) break;
             tc_fence_after();
             // the group's 128 columns of this warp's 32 lanes (vocabulary entries)
-            const uint32_t taddr = tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(buf * R_pad + g * kWideGroup);
+            const uint32_t taddr = tmem + ((uint32_t)(qd * 32) << 16) + (uint32_t)(buf * NZ + g * kWideGroup);
             const int ncols = min(kWideGroup, R_pad - g * kWideGroup);
 #pragma unroll
             for (int h = 0; h < 128 / kWideRound; ++h) {
@@ -1274,6 +1278,12 @@ __global__ void __launch_bounds__(kWideThreads, 1) lmhead_wide_kernel(const LmHe
                     for (int c0 = 0; c0 < ncols; c0 += 32) {
                         float v32[32];
                         tc_ld32(taddr + (uint32_t)c0, v32);
+                        if (LO) {  // (hi + lo, the same sum the 16-row kernel forms)
+                            float l32[32];
+                            tc_ld32(taddr + (uint32_t)(R_pad + c0), l32);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v32[i] += l32[i];
+                        }
 #pragma unroll
                         for (int i = 0; i < 32; ++i) trow[c0 + i] = v32[i];
                     }
@@ -1343,7 +1353,11 @@ size_t lmhead_mma_split_bytes(int R, const DeviceInfo& dev) {
     return (size_t)dev.num_sms * 128 * ((R + 7) / 8 * 8) * sizeof(float);
 }
 
-size_t lmhead_wide_zb_bytes(int R, int d) { return (size_t)((R + 15) / 16 * 16) * d * 2; }
+// rows of at most kWideLoRows take z as bf16 hi + lo (twice the rows of the operand)
+size_t lmhead_wide_zb_bytes(int R, int d) {
+    const int R_pad = (R + 15) / 16 * 16;
+    return (size_t)(R_pad <= kWideLoRows ? 2 * R_pad : R_pad) * d * 2;
+}
 
 int lmhead_wide_slabs(int V, const DeviceInfo& dev) {
     const int ntiles = (V + 127) / 128;
@@ -1353,15 +1367,11 @@ int lmhead_wide_slabs(int V, const DeviceInfo& dev) {
 cudaError_t lmhead_wide_prepare(const DeviceInfo& dev) {
     const int wsm = dev.max_smem_optin - (int)sizeof(WideState) - 256;
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(lmhead_wide_kernel<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
-            cudaSuccess ||
-        (e = cudaFuncSetAttribute(lmhead_wide_kernel<16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
-            cudaSuccess ||
-        (e = cudaFuncSetAttribute(lmhead_wide_kernel<8, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
-            cudaSuccess ||
-        (e = cudaFuncSetAttribute(lmhead_wide_kernel<16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) !=
-            cudaSuccess)
-        return e;
+    for (auto k : {lmhead_wide_kernel<8, false, false>, lmhead_wide_kernel<16, false, false>,
+                   lmhead_wide_kernel<8, true, false>, lmhead_wide_kernel<16, true, false>,
+                   lmhead_wide_kernel<8, false, true>, lmhead_wide_kernel<16, false, true>,
+                   lmhead_wide_kernel<8, true, true>, lmhead_wide_kernel<16, true, true>})
+        if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, wsm)) != cudaSuccess) return e;
     return cudaFuncSetAttribute(lmhead_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeMaxSmem);
 }
 
@@ -1369,13 +1379,15 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
                                cudaEvent_t after_prep, cudaEvent_t after_main) {
     if (!lmhead_wide_ok(a) || (reinterpret_cast<uintptr_t>(a.hid) & 15)) return cudaErrorInvalidValue;
     const int R_pad = (a.R + 15) / 16 * 16;
+    const bool lo = R_pad <= kWideLoRows;  // z as bf16 hi + lo
+    const int NZ = lo ? 2 * R_pad : R_pad;
     cudaError_t e = launch_k(zprep_kernel<bf16_t>, dim3(R_pad), dim3(256), 0, st, a.pdl, a.hid,
-                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, 0, a.stamp);
+                             (const bf16_t*)a.gamma, a.R, R_pad, a.d, a.eps, zb, lo ? 1 : 0, a.stamp);
     if (e != cudaSuccess) return e;
     if (after_prep && (e = cudaEventRecord(after_prep, st)) != cudaSuccess) return e;
     // shared memory: the transpose buffers (one per row group), then up to kWideMaxZ z stages
     // (R_pad x 128 B) and the rest to the weight ring (at least as many stages)
-    const size_t zst = (size_t)R_pad * 128;
+    const size_t zst = (size_t)NZ * 128;
     const size_t tbytes = (size_t)((R_pad + kWideGroup - 1) / kWideGroup) * kWideRound * kWideTileStride * sizeof(float);
     const size_t budget = (size_t)dev.max_smem_optin - sizeof(WideState) - 256;
     if (budget < 1024 + tbytes + 2 * (16384 + zst)) return cudaErrorInvalidValue;
@@ -1386,10 +1398,16 @@ cudaError_t launch_lmhead_wide(const LmHeadArgs& a, uint16_t* zb, const DeviceIn
     SW = SW > kWideMaxW ? kWideMaxW : SW;
     const size_t zring = SZ * zst;
     const size_t smem = 1024 + (size_t)SW * 16384 + zring + tbytes;
+    // TMEM: two NZ-column accumulators; the epilogue reads 32 columns at a time from a row
+    // group's first column (and, with lo, from R_pad columns further on)
+    const uint32_t need = (uint32_t)(NZ + (lo ? R_pad : 0) + ((std::min(R_pad, kWideGroup) + 31) / 32) * 32);
     uint32_t cols = 32;
-    while (cols < (uint32_t)(2 * R_pad)) cols <<= 1;
-    auto kern = a.sample ? (a.top_k <= 8 ? lmhead_wide_kernel<8, true> : lmhead_wide_kernel<16, true>)
-                         : (a.top_k <= 8 ? lmhead_wide_kernel<8, false> : lmhead_wide_kernel<16, false>);
+    while (cols < (uint32_t)(2 * NZ) || cols < need) cols <<= 1;
+    if (cols > 512) return cudaErrorInvalidValue;
+    auto kern = lo ? (a.sample ? (a.top_k <= 8 ? lmhead_wide_kernel<8, true, true> : lmhead_wide_kernel<16, true, true>)
+                               : (a.top_k <= 8 ? lmhead_wide_kernel<8, false, true> : lmhead_wide_kernel<16, false, true>))
+                   : (a.sample ? (a.top_k <= 8 ? lmhead_wide_kernel<8, true, false> : lmhead_wide_kernel<16, true, false>)
+                               : (a.top_k <= 8 ? lmhead_wide_kernel<8, false, false> : lmhead_wide_kernel<16, false, false>));
     e = launch_k(kern, dim3(a.n_slabs), dim3(kWideThreads), smem, st, a.pdl, a, (const uint16_t*)zb, R_pad, SW, SZ, cols);
     if (e != cudaSuccess) return e;
     if (after_main && (e = cudaEventRecord(after_main, st)) != cudaSuccess) return e;

@@ -125,6 +125,7 @@ struct fe_handle {
     bool lin_defer = true;    // tensor-core phases leave split tiles to the next phase's prep
     bool lin_normpost = true; // tensor-core RMSNorm phases: the scale on the products (column-parallel prep)
     bool attn_operand = true; // tensor-core O projection: its operand written by the attention kernel
+    int lm_16row = -1;        // up to 16 hidden rows: 1 the 16-row tensor-core LM head, 0 the wide one where it fits, -1 by vocabulary size
     uint16_t* lin_xb = nullptr;  // tensor-core linear: bf16 hi/lo activation operand
     float* lin_part = nullptr;   // tensor-core linear: per-CTA partials of split tiles
     int* lin_counters = nullptr; // tensor-core linear: per (tile, warp) completion counters
@@ -458,7 +459,12 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.sample = a->sample ? 1 : 0; lm.seed = a->seed; lm.part_lg = h->lm_part_lg; lm.topk_rank = a->topk_rank;
     lm.pdl = pdl;
     lm.stamp = next_stamp(pf);
-    if (h->lm_mma && N * B <= 16) {
+    // Up to 16 rows the wide kernel (z as bf16 hi + lo) takes vocabularies of at least four
+    // 128-entry tiles per CTA (it hands out whole tiles, so fewer leave CTAs idle at the end):
+    // it streams the 1-2 GB heads of 128256 entries 10-11 % faster than the 16-row kernel
+    // (stream-K units), which keeps the smaller vocabularies and top_k > 16
+    const bool wide_small = h->lm_16row == 0 || (h->lm_16row < 0 && (V + 127) / 128 >= 4 * h->dev.num_sms);
+    if (h->lm_mma && N * B <= 16 && !(wide_small && lmhead_wide_ok(lm))) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         lm.split_part = h->lm_split_part;  // (tile, column block) units split evenly over the CTAs
         lm.split_flag = h->lm_split_flag;
@@ -766,6 +772,10 @@ fe_status fe_draft_init(const fe_config* cfg, const fe_weights* w, void* stream,
             h->lm_mma = c.dtype == FE_BF16 && c.d % 64 == 0 && c.d <= 16384 &&
                         (rmax <= 16 || (rmax <= 256 && c.top_k_max <= 16)) &&
                         !(getenv("FE_DRAFT_LMHEAD_CUDA_CORES") && getenv("FE_DRAFT_LMHEAD_CUDA_CORES")[0] == '1');
+            // FE_DRAFT_LMHEAD_16ROW=1 / 0: up to 16 rows, the 16-row kernel / the wide one
+            // wherever it fits, instead of the choice by vocabulary size (for comparison)
+            const char* l16 = getenv("FE_DRAFT_LMHEAD_16ROW");
+            h->lm_16row = l16 && l16[0] == '1' ? 1 : (l16 && l16[0] == '0' ? 0 : -1);
         }
         if (h->lm_mma) {
             void* dst = p;

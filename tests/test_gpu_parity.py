@@ -127,7 +127,8 @@ SMALL = {
                                          n_layers=2, dtype="bf16", B=4, prefix=0, top_k=8, rope_theta=5e5,
                                          seed=19, page_size=24), prefix_list=[23, 24, 47, 400]),
     # 313 vocabulary tiles (the last one ragged) over at most 152 CTAs with d = 256: the
-    # 16-row LM head splits tiles between neighbouring CTAs; 12 rows, temperature 0.7
+    # 16-row LM head splits tiles between neighbouring CTAs; 12 rows, temperature 0.7 (the
+    # wide LM head with z as hi + lo on the same case below)
     "lmhead_split_v40k": dict(name=dict(d=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=704, vocab=40003,
                                         n_layers=4, dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4,
                                         seed=21, page_size=0), prefix_list=[5, 0, 70], temperature=0.7),
@@ -277,3 +278,18 @@ def test_attention_operand_path_is_exact(monkeypatch, case):
     assert a["status"] == 0 and b["status"] == 0
     for key in ("logits", "hidden", "topk_id", "topk_logit", "topk_prob", "lse", "tree_tok"):
         assert np.array_equal(a[key], b[key]), key
+
+
+@pytest.mark.parametrize("case", ["lmhead_split_v40k", "gqa4_bf16_ragged", "tc_linear_b9_paged"])
+def test_wide_lm_head_hi_lo_forced(orc, monkeypatch, case):
+    """Up to 16 hidden rows the wide LM head (whole vocabulary tiles per CTA, z as bf16 hi +
+    lo) runs on vocabularies of at least four tiles per CTA (the full-size 128256-entry heads);
+    FE_DRAFT_LMHEAD_16ROW=0 selects it on these small ones, against the oracle."""
+    monkeypatch.setenv("FE_DRAFT_LMHEAD_16ROW", "0")
+    spec = dict(SMALL[case])
+    cfg = wl.make_config(spec.pop("name"), **spec)
+    W, I, ks, vs = _problem(cfg)
+    g = H.run_gpu(cfg, W, I, ks, vs)
+    assert g["status"] == 0, g["status"]
+    for b in range(cfg["B"]):
+        H.compare(orc, cfg, g, H.run_oracle(orc, cfg, W, I, ks, vs, b), b)

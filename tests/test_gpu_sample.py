@@ -9,8 +9,9 @@ tolerance carried through the 1 / T scale), and the substitute must sit in that 
 drawn set is reported ordered by logit (ties to the smaller id), its logits and
 probabilities match the oracle's, and the tree is bit-exact on the GPU's candidates. All
 three LM-head kernels are covered: the CUDA-core one (float32, and bf16 forced), the 16-row
-tensor-core one (N B <= 16) and the wide one (N B > 16, k <= 8 and k <= 16), plus the
-batched-serving workload at full size.
+tensor-core one (N B <= 16) and the wide one (N B > 16, k <= 8 and k <= 16; N B <= 16 with z
+as bf16 hi + lo, forced on the small vocabularies), plus the batched-serving workload at full
+size.
 """
 import numpy as np
 import pytest
@@ -29,7 +30,8 @@ CASES = {
     # float32, N B = 3: the CUDA-core LM head
     "tiny_f32_T1": dict(name="tiny", T=1.0, seed=11),
     "tiny_f32_T07": dict(name="tiny", T=0.7, seed=2**63 + 12),
-    # bf16, N B = 12: the 16-row tensor-core LM head (ragged prefixes, V % 128 != 0)
+    # bf16, N B = 12: the 16-row tensor-core LM head (ragged prefixes, V % 128 != 0); the wide
+    # one with z as hi + lo on the same case below
     "gqa4_bf16_16row": dict(name=dict(d=512, n_heads=8, n_kv_heads=2, head_dim=64, ffn=1376, vocab=5003, n_layers=4,
                                       dtype="bf16", B=3, prefix=0, top_k=8, rope_theta=1e4, seed=3, page_size=0),
                             prefix_list=[37, 0, 150], T=1.0, seed=7),
@@ -112,6 +114,14 @@ def _run_case(orc, spec, seqs=None):
 
 @pytest.mark.parametrize("case", list(CASES))
 def test_sampled_draft_matches_oracle(orc, case):
+    _run_case(orc, CASES[case])
+
+
+@pytest.mark.parametrize("case", ["gqa4_bf16_16row", "split_v40k_T07"])
+def test_sampled_draft_wide_lm_head_hi_lo_forced(orc, monkeypatch, case):
+    """N B <= 16 on the wide tensor-core LM head with z as bf16 hi + lo
+    (FE_DRAFT_LMHEAD_16ROW=0; by default it takes only the large vocabularies)."""
+    monkeypatch.setenv("FE_DRAFT_LMHEAD_16ROW", "0")
     _run_case(orc, CASES[case])
 
 
