@@ -459,11 +459,14 @@ fe_status enqueue_forward(fe_handle* h, const fe_forward_args* a, cudaStream_t s
     lm.sample = a->sample ? 1 : 0; lm.seed = a->seed; lm.part_lg = h->lm_part_lg; lm.topk_rank = a->topk_rank;
     lm.pdl = pdl;
     lm.stamp = next_stamp(pf);
-    // Up to 16 rows the wide kernel (z as bf16 hi + lo) takes vocabularies of at least four
-    // 128-entry tiles per CTA (it hands out whole tiles, so fewer leave CTAs idle at the end):
-    // it streams the 1-2 GB heads of 128256 entries 10-11 % faster than the 16-row kernel
-    // (stream-K units), which keeps the smaller vocabularies and top_k > 16
-    const bool wide_small = h->lm_16row == 0 || (h->lm_16row < 0 && (V + 127) / 128 >= 4 * h->dev.num_sms);
+    // Up to 16 rows the wide kernel (z as bf16 hi + lo) takes greedy calls on vocabularies of
+    // at least four 128-entry tiles per CTA (it hands out whole tiles, so fewer leave CTAs
+    // idle at the end): it streams the 1-2 GB heads of 128256 entries 10-11 % faster than the
+    // 16-row kernel (stream-K units), which keeps the smaller vocabularies, top_k > 16 and
+    // sampled calls (the wide kernel draws a row's deviates on one thread: 532 vs 388 us per
+    // 70B-shaped draft)
+    const bool wide_small = h->lm_16row == 0 ||
+                            (h->lm_16row < 0 && !a->sample && (V + 127) / 128 >= 4 * h->dev.num_sms);
     if (h->lm_mma && N * B <= 16 && !(wide_small && lmhead_wide_ok(lm))) {
         lm.n_slabs = std::min(h->dev.num_sms, (V + 127) / 128);  // one CTA per SM, at least one 128-row tile each
         lm.split_part = h->lm_split_part;  // (tile, column block) units split evenly over the CTAs
