@@ -69,15 +69,15 @@ TRAFFIC = {
     # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum -k regex:linear_kernel
     #     -s 18 -c 6 on `bench.py --workload l33_70b --set n_layers=1 --also ...` (one draft's six linear
     # launches: W_fuse, W_in, W_qkv, W_o, W_gate/up, W_down; the eight-layer draft repeats the last four)
-    "l33_70b": {"bytes_per_draft": (402779648 + 3221504) + (268562176 + 86272)
-                + 8 * ((167900160 + 56320) + (134357760 + 63744) + (939677696 + 256512) + (469996032 + 85248)),
-                "sources": ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh"), "src": "d49661301765124c"},
+    "l33_70b": {"bytes_per_draft": (402804480 + 2994944) + (268569600 + 35072)
+                + 8 * ((167912448 + 59136) + (134362112 + 127232) + (939734272 + 508160) + (470002176 + 48896)),
+                "sources": ("fe_stream.cuh", "fe_linear.cu", "fe_common.cuh"), "src": "db0896d91ededd9f"},
     # the same metrics with -k regex:linear_mma_kernel -s 18 -c 6 on `bench.py --workload b32_l31 --set
     # n_layers=1 --also ...` (the tensor-core products of the six phases; the six-layer draft repeats
     # the last four)
-    "b32_l31": {"bytes_per_draft": (102311680 + 2799104) + (68231936 + 512)
-                + 6 * ((50935808 + 0) + (34152704 + 0) + (235485184 + 2010880) + (119887872 + 135680)),
-                "sources": ("fe_linear_mma.cu", "fe_tc.cuh", "fe_common.cuh"), "src": "519855c393da0488"},
+    "b32_l31": {"bytes_per_draft": (102318080 + 2932992) + (68232192 + 13312)
+                + 6 * ((50930432 + 0) + (34153216 + 0) + (235487488 + 1959424) + (119891456 + 462080)),
+                "sources": ("fe_linear_mma.cu", "fe_tc.cuh", "fe_common.cuh"), "src": "ee529b04c166ea62"},
 }
 
 
